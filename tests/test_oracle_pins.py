@@ -1,0 +1,386 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Nothing here compares the oracle with itself: each check uses the paper's printed examples
+(tests/golden/*.txt), closed forms, invariants, or an exact brute force in Python Fractions.
+"""
+import itertools
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle import net as onet
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rows(name):
+    out = []
+    with open(os.path.join(GOLD, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                out.append(line.split())
+    return out
+
+
+def F(x):
+    return Fraction(float(x))
+
+
+def frac_q(x, k, S, fl):
+    """Quantizer as nearest member of domQ (ties to the even code), exact."""
+    y = F(x) * Fraction(2) ** fl
+    m = oracle.frac_round_half_even(y)
+    return min(max(m, -S * 2 ** (k - S)), 2 ** (k - S) - 1)
+
+
+def frac_l2(xs, k, S, fl):
+    tot = Fraction(0)
+    for x in xs:
+        d = F(x) - Fraction(frac_q(x, k, S, fl)) * Fraction(2) ** (-fl)
+        tot += d * d
+    return tot
+
+
+# ---------------------------------------------------------------- paper examples
+def test_paper_format_examples():
+    for a, b, S, x, v in _rows("paper_format_examples.txt"):
+        a, b, S = int(a), int(b), int(S)
+        k = a + b
+        code = oracle.quantize(np.array([float(x)], np.float32), k, S, b)[0]
+        assert Fraction(int(code)) * Fraction(2) ** (-b) == F(np.float32(float(v))), (a, b, x)
+
+
+def test_paper_format_value_sets():
+    # U(3,-1): values {0,2,4,6}; S(-1,3): {-0.25,-0.125,0,0.125}
+    grid = np.linspace(-20, 20, 4001).astype(np.float32)
+    u = set((oracle.quantize(grid, 2, 0, -1) * 2.0).tolist())
+    s = set((oracle.quantize(grid / 40, 2, 1, 3) / 8.0).tolist())
+    assert u == {0.0, 2.0, 4.0, 6.0}
+    assert s == {-0.25, -0.125, 0.0, 0.125}
+
+
+def test_paper_format_levels():
+    for a, b, S, k, lo, hi in _rows("paper_formats.txt"):
+        a, b, S, k, lo, hi = map(int, (a, b, S, k, lo, hi))
+        assert a + b == k
+        assert oracle.qmin(k, S) == lo and oracle.qmax(k, S) == hi
+        x = np.array([1e6, -1e6], np.float32)
+        c = oracle.quantize(x, k, S, b)
+        assert c[0] == hi and c[1] == lo
+    # 6-bit signed range [-32*2^-beta, 31*2^-beta]
+    for beta in (5, 7, 8, 9):
+        c = oracle.quantize(np.array([1e3, -1e3], np.float32), 6, 1, beta)
+        assert c[0] * 2.0 ** -beta == 31 * 2.0 ** -beta and c[1] * 2.0 ** -beta == -32 * 2.0 ** -beta
+
+
+def test_round_half_even_ties():
+    x = np.array([0.5, 1.5, 2.5, -1.5, -0.5, 3.5, -2.5], np.float32)
+    assert oracle.quantize(x, 8, 1, 0).tolist() == [0, 2, 2, -2, 0, 4, -2]
+
+
+# ---------------------------------------------------------------- quantizer
+def _adversarial(seed, n=64):
+    rng = np.random.default_rng(seed)
+    base = synth.normal(n, seed)
+    extra = np.array([0.0, -0.0, 0.5, -0.5, 1.5, 2.5, 127.5, -128.5, 255.5, 1e-40, -3e-39,
+                      2.0 ** -30, 6.0e7, -6.0e7, 0.75, 3.75, 1 - 2 ** -24, 2 ** 20 + 0.5], np.float32)
+    scale = np.float32(2.0) ** rng.integers(-6, 6, size=n).astype(np.float32)
+    return np.concatenate([base * scale, extra]).astype(np.float32)
+
+
+def test_quantize_matches_nearest_in_domQ():
+    xs = _adversarial(11)
+    for k, S, fl in itertools.product([2, 3, 5, 8, 9, 16], [0, 1], [-8, -1, 0, 3, 7, 23]):
+        got = oracle.quantize(xs, k, S, fl)
+        want = [frac_q(x, k, S, fl) for x in xs]
+        assert got.tolist() == want, (k, S, fl)
+
+
+def test_quantize_invariants():
+    xs = np.sort(_adversarial(12, 2000))
+    for k, S, fl in [(8, 1, 5), (4, 0, 2), (16, 1, 12), (3, 1, -2)]:
+        c = oracle.quantize(xs, k, S, fl)
+        v = c.astype(np.float64) * 2.0 ** -fl
+        lo, hi = oracle.qmin(k, S), oracle.qmax(k, S)
+        inside = (xs.astype(np.float64) >= lo * 2.0 ** -fl) & (xs.astype(np.float64) <= hi * 2.0 ** -fl)
+        # |x - x~| <= 2^-(FL+1) inside the range
+        assert np.all(np.abs(xs[inside].astype(np.float64) - v[inside]) <= 2.0 ** -(fl + 1))
+        # exact saturation
+        assert np.all(c[xs.astype(np.float64) > hi * 2.0 ** -fl] == hi)
+        assert np.all(c[xs.astype(np.float64) < lo * 2.0 ** -fl] == lo)
+        # monotone
+        assert np.all(np.diff(c) >= 0)
+        # idempotent on representable values
+        assert np.array_equal(oracle.quantize(v.astype(np.float32), k, S, fl), c)
+        # sign symmetry away from Qmin
+        if S == 1:
+            cn = oracle.quantize(-xs, k, S, fl)
+            ok = (c > lo) & (cn > lo)
+            assert np.array_equal(cn[ok], -c[ok])
+
+
+# ---------------------------------------------------------------- L2 error (Eq. DSB_QE)
+def test_exact_sum_accumulator_vs_fractions():
+    rng = np.random.default_rng(3)
+    for trial in range(20):
+        n = int(rng.integers(1, 200))
+        v = rng.standard_normal(n) * 2.0 ** rng.integers(-300, 300, size=n)
+        if trial % 3 == 0:  # heavy cancellation
+            v = np.concatenate([v, -v[: n // 2], [1e-300, -1e300, 1e300]])
+        want = float(sum((Fraction(float(t)) for t in v), Fraction(0)))
+        assert oracle.exact_sum(v) == want
+
+
+def test_l2_single_element_closed_form():
+    for x in [0.3, -0.7, 5.25, 1e-3, -100.0, 0.0]:
+        for k, S, fl in [(8, 1, 4), (2, 0, 1), (16, 1, 20), (5, 0, -3)]:
+            want = float(frac_l2([np.float32(x)], k, S, fl))
+            assert oracle.l2_error(np.array([x], np.float32), k, S, fl) == want
+
+
+def test_l2_zero_on_grid():
+    codes = np.arange(-128, 128)
+    for fl in [-3, 0, 5, 20]:
+        x = (codes * 2.0 ** -fl).astype(np.float32)
+        assert oracle.l2_error(x, 8, 1, fl) == 0.0
+        assert oracle.l2_error(x, 9, 1, fl) == 0.0
+        assert oracle.l2_error(x, 7, 1, fl) > 0.0  # does not fit 7 bits
+
+
+def test_l2_bruteforce_all_candidates():
+    for seed in (21, 22):
+        xs = _adversarial(seed, 10)[:16]
+        err, best, S, st = oracle.fl_search(xs, -1, 2, 16, -8, 23)
+        assert S == 1
+        for ki, k in enumerate(range(2, 17)):
+            exact = [frac_l2(xs, k, S, fl) for fl in range(-8, 24)]
+            assert err[ki].tolist() == [float(e) for e in exact]
+            m = min(exact)
+            assert best[ki] == -8 + exact.index(m)  # first minimum: ties go to the smallest FL
+
+
+def test_fl_search_tie_goes_to_smallest_fl():
+    # single x = 0.75, k = 2 unsigned: FL=0 -> code 1 (err 1/16); FL=1 -> code 2 (value 1, err 1/16)
+    x = np.array([0.75], np.float32)
+    err, best, S, _ = oracle.fl_search(x, 0, 2, 2, 0, 1)
+    assert err[0, 0] == err[0, 1] == 0.0625 and best[0] == 0
+    err, best, S, _ = oracle.fl_search(x, 0, 2, 2, -2, 3)
+    assert best[0] == 2 and err[0, 4] == 0.0
+
+
+def test_unsigned_equals_signed_one_more_bit_on_nonnegative():
+    xs = np.abs(_adversarial(31, 300))
+    for k in (2, 5, 8, 15):
+        for fl in (-4, 0, 6, 19):
+            assert np.array_equal(oracle.quantize(xs, k, 0, fl), oracle.quantize(xs, k + 1, 1, fl))
+            assert oracle.l2_error(xs, k, 0, fl) == oracle.l2_error(xs, k + 1, 1, fl)
+
+
+def test_unsigned_negative_inputs_saturate_to_zero():
+    xs = -np.abs(_adversarial(32, 100))
+    assert np.all(oracle.quantize(xs, 6, 0, 3) == 0)
+    assert oracle.l2_error(xs, 6, 0, 3) == float(sum(F(x) ** 2 for x in xs))
+
+
+def test_stats_and_sign_strategy():
+    xs = _adversarial(41, 500)
+    _, _, S, st = oracle.fl_search(xs, -1, 8, 8, 0, 1)
+    assert S == 1 and st["min"] == float(xs.min()) and st["max"] == float(xs.max())
+    assert st["sum"] == float(sum(F(x) for x in xs))
+    assert st["sumsq"] == float(sum(F(x) ** 2 for x in xs))
+    _, _, S, _ = oracle.fl_search(np.abs(xs), -1, 8, 8, 0, 1)
+    assert S == 0
+
+
+def test_fl_init_hand_cases():
+    # unsigned: psi = max/(2^k-1) = 1/255 -> beta_hat = log2(255) = 7.994
+    assert oracle.fl_init(0.0, 1.0, 8, "conservative") == (0, 7, 1)
+    assert oracle.fl_init(0.0, 1.0, 8, "neutral") == (0, 8, 0)
+    assert oracle.fl_init(0.0, 1.0, 8, "aggressive") == (0, 8, 0)
+    # signed: psi = min(2/128, 1/127) = 1/127 -> beta_hat = log2(127) = 6.989
+    assert oracle.fl_init(-2.0, 1.0, 8, "conservative") == (1, 6, 2)
+    assert oracle.fl_init(-2.0, 1.0, 8, "neutral") == (1, 7, 1)
+    # exact power of two: psi = min(0.5/128, 0.5/127) = 2^-8 -> beta = 8 for every strategy
+    for st in ("conservative", "neutral", "aggressive"):
+        assert oracle.fl_init(-0.5, 0.5, 8, st)[1] == 8
+
+
+# ---------------------------------------------------------------- integer C-Block
+def _im2col_conv(x, w, stride, pad):
+    N, H, W, C = x.shape
+    K, R, S, _ = w.shape
+    xp = np.zeros((N, H + 2 * pad, W + 2 * pad, C), np.int64)
+    xp[:, pad:pad + H, pad:pad + W] = x
+    P = (H + 2 * pad - R) // stride + 1
+    Q = (W + 2 * pad - S) // stride + 1
+    cols = np.empty((N, P, Q, R, S, C), np.int64)
+    for r in range(R):
+        for s in range(S):
+            cols[:, :, :, r, s, :] = xp[:, r:r + stride * (P - 1) + 1:stride, s:s + stride * (Q - 1) + 1:stride, :]
+    return np.matmul(cols.reshape(N * P * Q, -1), w.reshape(K, -1).astype(np.int64).T).reshape(N, P, Q, K)
+
+
+@pytest.mark.parametrize("shape", [(2, 9, 9, 5, 7, 3, 1, 1), (1, 23, 23, 3, 4, 11, 4, 2), (2, 8, 8, 16, 6, 1, 2, 0),
+                                   (3, 6, 6, 4, 5, 6, 1, 0), (1, 7, 7, 3, 2, 7, 2, 3)])
+def test_conv_matches_im2col_matmul(shape):
+    N, H, W, C, K, R, st, pad = shape
+    rng = np.random.default_rng(sum(shape))
+    x = rng.integers(0, 256, size=(N, H, W, C))
+    w = rng.integers(-128, 128, size=(K, R, R, C))
+    assert np.array_equal(oracle.conv2d(x, w, st, pad), _im2col_conv(x, w, st, pad))
+
+
+def test_conv_one_hot_weights_select_inputs():
+    rng = np.random.default_rng(5)
+    x = rng.integers(-32768, 32768, size=(2, 5, 5, 4))
+    w = np.zeros((4, 3, 3, 4), np.int64)
+    for k in range(4):
+        w[k, 1, 1, k] = 1
+    assert np.array_equal(oracle.conv2d(x, w, 1, 1), x)
+
+
+def test_requant_matches_quantizing_the_exact_value():
+    rng = np.random.default_rng(7)
+    acc = rng.integers(-2 ** 40, 2 ** 40, size=400)
+    acc[:8] = [0, 1, -1, 2 ** 10 + 2 ** 9, -(2 ** 10 + 2 ** 9), 3 * 2 ** 9, 5 * 2 ** 9, -7 * 2 ** 9]
+    for s, fl, k, S in [(20, 10, 8, 1), (20, 8, 16, 1), (13, 3, 6, 0), (5, 9, 8, 1), (30, 30, 12, 1), (10, 0, 4, 0)]:
+        got = oracle.requant(acc, s, k, S, fl)
+        for a, g in zip(acc.tolist(), got.tolist()):
+            y = Fraction(a) * Fraction(2) ** (fl - s)
+            m = oracle.frac_round_half_even(y)
+            assert g == min(max(m, -S * 2 ** (k - S)), 2 ** (k - S) - 1)
+
+
+def test_bias_alignment_preserves_value():
+    rng = np.random.default_rng(8)
+    acc = rng.integers(-2 ** 30, 2 ** 30, size=100)
+    b = rng.integers(-2 ** 15, 2 ** 15, size=100)
+    for s, flb in [(12, 4), (12, 12), (5, 19), (0, 3)]:
+        v, s2 = oracle.add_bias(acc, s, b, flb)
+        for a, bb, vv in zip(acc.tolist(), b.tolist(), v.tolist()):
+            assert Fraction(vv, 2 ** s2) == Fraction(a, 2 ** s) + Fraction(bb, 2 ** flb)
+
+
+def test_maxpool_matches_window_max():
+    rng = np.random.default_rng(9)
+    x = rng.integers(0, 256, size=(2, 13, 11, 5))
+    for k, st, pad in [(3, 2, 0), (2, 2, 0), (3, 2, 1), (3, 1, 1)]:
+        got = oracle.maxpool(x, k, st, pad)
+        xp = np.pad(x, ((0, 0), (pad, pad), (pad, pad), (0, 0)), constant_values=-1)
+        win = np.lib.stride_tricks.sliding_window_view(xp, (k, k), axis=(1, 2))[:, ::st, ::st]
+        want = win.max(axis=(-1, -2))
+        assert np.array_equal(got, want[:, :got.shape[1], :got.shape[2]])
+        # unsigned post-ReLU codes: ignoring padded taps equals zero padding
+        xz = np.pad(x, ((0, 0), (pad, pad), (pad, pad), (0, 0)), constant_values=0)
+        winz = np.lib.stride_tricks.sliding_window_view(xz, (k, k), axis=(1, 2))[:, ::st, ::st]
+        assert np.array_equal(got, winz.max(axis=(-1, -2))[:, :got.shape[1], :got.shape[2]])
+
+
+def test_eltwise_and_avgpool_exact():
+    rng = np.random.default_rng(10)
+    a = rng.integers(-128, 128, size=(2, 3, 3, 4))
+    b = rng.integers(0, 64, size=(2, 3, 3, 4))
+    v, fl = oracle.eltwise_add(a, 3, b, 6, relu=True)
+    for x, y, z in zip(a.ravel().tolist(), b.ravel().tolist(), v.ravel().tolist()):
+        assert Fraction(z, 2 ** fl) == max(Fraction(x, 8) + Fraction(y, 64), 0)
+    x = rng.integers(0, 256, size=(2, 7, 7, 3))
+    r = oracle.quantize(np.array([1 / 49], np.float32), 16, 0, 21)[0]
+    v, s = oracle.avgpool_global(x, 4, int(r), 21)
+    for n in range(2):
+        for c in range(3):
+            assert Fraction(int(v[n, c]), 2 ** s) == Fraction(int(x[n, :, :, c].sum()), 16) * Fraction(int(r), 2 ** 21)
+
+
+def test_reciprocal_format_of_avgpool():
+    # 1/49 as a 16-bit unsigned parameter: the FL search picks FL = 21 (largest unsaturated grid)
+    _, best, S, _ = oracle.fl_search(np.array([1 / 49], np.float32), -1, 16, 16, -8, 23)
+    assert S == 0 and best[0] == 21
+
+
+# ---------------------------------------------------------------- small network, exact semantics
+def _tiny_layers():
+    return [
+        {"type": "conv", "name": "c1", "C": 3, "K": 6, "R": 3, "stride": 1, "pad": 1, "relu": True, "src": None},
+        {"type": "maxpool", "name": "p1", "k": 2, "stride": 2, "pad": 0},
+        {"type": "conv", "name": "c2", "C": 6, "K": 5, "R": 3, "stride": 1, "pad": 1, "relu": False, "src": None},
+        {"type": "eltwise", "name": "e", "a": "c2", "b": "c2b", "relu": True},
+        {"type": "conv", "name": "fc", "C": 5, "K": 4, "R": 4, "stride": 1, "pad": 0, "relu": False, "src": "e"},
+    ]
+
+
+def test_tiny_network_layers_equal_quantized_exact_reals():
+    layers = _tiny_layers()
+    # second branch feeding the eltwise: a 1x1 conv on p1
+    layers.insert(3, {"type": "conv", "name": "c2b", "C": 6, "K": 5, "R": 1, "stride": 1, "pad": 0, "relu": False, "src": "p1"})
+    layers[2]["src"] = "p1"
+    rng = np.random.default_rng(13)
+    weights = {}
+    for L in layers:
+        if L["type"] == "conv":
+            fan = L["C"] * L["R"] ** 2
+            weights[L["name"]] = ((rng.standard_normal((L["K"], L["R"], L["R"], L["C"])) * np.sqrt(2 / fan)).astype(np.float32),
+                                  (rng.standard_normal(L["K"]) * 0.01).astype(np.float32))
+    plan = {"input": 8, "c1": {"w": 6, "b": 16, "a": 5}, "c2": {"w": 7, "b": 16, "a": 6},
+            "c2b": {"w": 5, "b": 16, "a": 7}, "e": {"a": 6}, "fc": {"w": 8, "b": 16}}
+    imgs = synth.images(2, 77, hw=8)
+    fmts, qp = onet.calibrate(layers, weights, imgs, plan)
+    env = onet.forward_trace(layers, fmts, qp, imgs)
+
+    def val(codes, fl):
+        return [Fraction(int(c)) * Fraction(2) ** (-fl) for c in np.asarray(codes).ravel()]
+
+    def check_q(codes, fmt, exact_vals):
+        k, S, fl = fmt
+        want = [min(max(oracle.frac_round_half_even(v * Fraction(2) ** fl), -S * 2 ** (k - S)), 2 ** (k - S) - 1)
+                for v in exact_vals]
+        assert np.asarray(codes).ravel().tolist() == want
+
+    # each conv C-Block's output codes = Q(exact real conv + bias, ReLU) under its format
+    for nm, src in [("c1", "input"), ("c2", "p1"), ("c2b", "p1")]:
+        L = next(l for l in layers if l["name"] == nm)
+        x, fx = env[src]
+        wq, bq = qp[nm]
+        fw, fb = fmts[nm]["w"], fmts[nm]["b"]
+        acc = oracle.conv2d(x, wq, L["stride"], L["pad"])
+        exact = [Fraction(int(a), 2 ** (fx[2] + fw[2])) + Fraction(int(bq[i % L["K"]])) * Fraction(2) ** (-fb[2])
+                 for i, a in enumerate(acc.ravel().tolist())]
+        if L["relu"]:
+            exact = [max(e, 0) for e in exact]
+        check_q(env[nm][0], fmts[nm]["a"], exact)
+    # eltwise: Q(relu(a + b)) of the real values
+    ea = val(env["c2"][0], fmts["c2"]["a"][2])
+    eb = val(env["c2b"][0], fmts["c2b"]["a"][2])
+    check_q(env["e"][0], fmts["e"]["a"], [max(p + q, 0) for p, q in zip(ea, eb)])
+    # maxpool keeps the input format
+    assert env["p1"][1] == fmts["c1"]["a"]
+    # calibration picked the argmin of the L2 error of the calibration output (checked for c1)
+    L = layers[0]
+    x, fx = env["input"]
+    acc = oracle.conv2d(x, qp["c1"][0], 1, 1)
+    v, s = oracle.cblock(acc, fx[2] + fmts["c1"]["w"][2], qp["c1"][1], fmts["c1"]["b"][2], True)
+    vf = oracle.to_f32(v, s)
+    errs = [frac_l2(vf.ravel()[:64], 5, 0, fl) for fl in range(-8, 24)]  # sub-sample sanity: finite & ordered
+    assert all(e >= 0 for e in errs)
+
+
+# ---------------------------------------------------------------- architecture size pins
+def test_architecture_size_pins():
+    w = {L["name"]: L for L in synth.alexnet() if L["type"] == "conv"}
+    # AlexNet CONV-1 weights: 4.25 KB per bit -> 96*3*11*11 = 34848 weights
+    assert w["conv1"]["K"] * w["conv1"]["C"] * w["conv1"]["R"] ** 2 == 34848
+    assert round(34848 / 8 / 1024, 2) == 4.25
+    # AlexNet FC-6: 4.72 MB per bit -> 9216 x 4096
+    assert w["fc6"]["C"] * w["fc6"]["R"] ** 2 == 9216 and w["fc6"]["K"] == 4096
+    assert round(9216 * 4096 / 8 / 1e6, 2) == 4.72
+    v = {L["name"]: L for L in synth.vgg16() if L["type"] == "conv"}
+    # VGG-16 FC-6: 102.76 M multiplies per image
+    assert round(v["fc6"]["C"] * v["fc6"]["R"] ** 2 * v["fc6"]["K"] / 1e6, 2) == 102.76
+    # per-image MACs: VGG-16 15.3-15.5 G, ResNet-18 1.8 G
+    assert 15.3e9 <= synth.macs_per_image("vgg16") <= 15.5e9
+    assert abs(synth.macs_per_image("resnet18") - 1.8e9) < 0.05e9
+    assert sum(1 for L in synth.vgg16() if L["type"] == "conv") == 16
