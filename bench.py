@@ -1,0 +1,311 @@
+"""Benchmark: images/s of the fixed-point network evaluation on GB300.
+
+Workload (default): VGG-16 architecture, batch 64 synthetic 224x224x3 N(0,1) images, He-init
+weights, first and last layers 16-bit (two-limb path), the rest mixed 4-8 bits; 32 candidate
+wordlength plans (seeds 7..38) as in an iterative precision-reduction search.  One step evaluates
+one candidate plan on one batch:
+  1. FL search + quantization of every weight and bias tensor at the plan's wordlengths,
+  2. calibration of every activation FL on the 8-image calibration slice (forward-optimizer order),
+  3. the integer-only forward of the whole batch through fxpq_net_forward.
+value = batch / step time (images per second), whole job over N GPUs (weak scaling: each rank
+evaluates its own plans on its own batch; no collective on the data path).
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+WORKLOADS = {
+    "vgg16": {"arch": "vgg16", "batch": 64, "seed": 7, "plans": list(range(7, 39)), "calib": 8},
+    "alexnet": {"arch": "alexnet", "batch": 256, "seed": 5, "plans": [5], "calib": 8},
+    "resnet18": {"arch": "resnet18", "batch": 128, "seed": 6, "plans": [6], "calib": 8},
+}
+L2_BYTES = 129 * 1024 * 1024
+
+
+def dist_env():
+    r = int(os.environ.get("RANK", "0"))
+    w = int(os.environ.get("WORLD_SIZE", "1"))
+    lr = int(os.environ.get("LOCAL_RANK", "0"))
+    return r, w, lr
+
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region (SM clock, max clock, throttle reasons)."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.samples = []
+        self._stop = threading.Event()
+        self._t = None
+
+    def _run(self):
+        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        while not self._stop.is_set():
+            try:
+                out = subprocess.run(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}", "--format=csv,noheader,nounits"],
+                                     capture_output=True, text=True, timeout=5).stdout.strip()
+                if out:
+                    self.samples.append([s.strip() for s in out.split(",")])
+            except Exception:
+                pass
+            self._stop.wait(0.2)
+
+    def __enter__(self):
+        self._t = threading.Thread(target=self._run, daemon=True)
+        self._t.start()
+        return self
+
+    def __exit__(self, *a):
+        self._stop.set()
+        if self._t:
+            self._t.join(timeout=10)
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm = [float(s[0]) for s in self.samples if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in self.samples for i in range(4) if len(s) > 3 + i and s[3 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d.get("hbm_gbs", 6800.0), d.get("bf16_tflops", 1900.0), d.get("bf16_tflops_sustained", 1700.0), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def run_fxpq(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, world, lrank = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(lrank)
+    dev = torch.device("cuda", lrank)
+    import __graft_entry__ as g
+    g.build()
+    from paper_2203_12091_gb300 import fxpq as F
+    from paper_2203_12091_gb300.net import QNet
+
+    wl = WORKLOADS[args.workload]
+    arch, B = wl["arch"], wl["batch"]
+    layers = synth.ARCHS[arch]()
+    W = synth.weights(arch, wl["seed"])
+    imgs_np = synth.images(B, wl["seed"] + 1000 * rank)
+    plans = [synth.bit_plan(arch, s) for s in wl["plans"]]
+    wdev = {nm: (torch.from_numpy(w).to(dev), torch.from_numpy(b).to(dev)) for nm, (w, b) in W.items()}
+    imgs = torch.from_numpy(imgs_np).to(dev)
+    pinned = torch.from_numpy(imgs_np).pin_memory()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def step(i, images):
+        q = QNet(layers, hw=224, cin=3)
+        q._dev = dev
+        plan = plans[(i + rank) % len(plans)]
+        q.quantize_params(wdev, plan)
+        q.calibrate(images[: wl["calib"]], plan)
+        logits, s = q.forward(images)
+        return q, logits, s
+
+    for i in range(args.warmup):
+        step(i, imgs)
+    torch.cuda.synchronize()
+
+    # ---- timed region (device-resident inputs): per-step CUDA events, L2 flushed between steps
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = F.fxpq_launch_count()
+    times = []
+    with ClockSampler(lrank) as clk:
+        for i in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step(args.warmup + i, imgs)
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+    torch.cuda.synchronize()
+    launches = F.fxpq_launch_count() - launches0
+    ms = sum(times) / len(times)
+    t_max = ms
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_max = float(t.item())
+    value = world * B / (t_max / 1e3)
+
+    # ---- end to end through the public API: pinned host images in, logits out, every step
+    e2e_times = []
+    for i in range(max(2, min(args.steps, 5))):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dimgs = pinned.to(dev, non_blocking=True)
+        q, logits, s = step(i, dimgs)
+        host_logits = logits.cpu()
+        torch.cuda.synchronize()
+        e2e_times.append(time.perf_counter() - t0)
+    e2e_s = sum(e2e_times) / len(e2e_times)
+    h2d = pinned.numel() * 4
+    d2h = host_logits.numel() * 8
+
+    # ---- roofline of the dominant kernel (the conv C-Block): op-by-op forward with events per conv
+    conv_ms, conv_flops, nconv = conv_roofline(q, imgs, F, stream)
+    hbm, bf16, bf16s, src = measured_peaks()
+    achieved = conv_flops / (conv_ms / 1e3) / 1e12
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        traffic = json.load(open(tpath)).get(args.workload)
+
+    if rank == 0:
+        cpu = cpu_baseline(args.workload) if (world == 1 and not args.no_cpu) else None
+        line = {
+            "metric": "images/s for fixed-point net forward (one candidate plan evaluated per step)",
+            "value": round(value, 2), "unit": "images/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(t_max, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "int (exact integer codes; fp16-valued operands)", "data": "synthetic",
+            "config": {"workload": f"{arch} batch {B}, {len(plans)} candidate plans, calib slice {wl['calib']}",
+                       "model": arch, "global_batch": B * world, "seq_len": None, "parallelism": f"replicas x{world}",
+                       "l2": "flushed between timed steps (2x L2 buffer written)"},
+            "e2e": {"value": round(world * B / e2e_s, 2), "unit": "images/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(launches),
+            "roofline": {"bound": "tensor", "kernel": "conv C-Block", "achieved": round(achieved, 3),
+                         "peak": bf16, "unit": "TFLOP/s", "frac": round(achieved / bf16, 5), "traffic": traffic,
+                         "peak_source": f"{src} bf16 dense burst (fp16 operands run at the bf16 rate)",
+                         "conv_launches_timed": nconv},
+            "clocks": clk.summary(),
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def conv_roofline(q, imgs, F, stream, iters=3):
+    """Average conv launch time over `iters` op-by-op forwards (CUDA events on the launching stream)."""
+    import torch
+    env0 = None
+    tot_ms, flops, n = 0.0, 0, 0
+    N = imgs.shape[0]
+    for it in range(iters):
+        fin = q.fmts["input"]["a"]
+        x0 = torch.empty(N * q.hw * q.hw * q.cp_in * F.planes(fin), dtype=torch.float16, device=imgs.device)
+        F.fxpq_quantize_images(imgs, fin, q.cp_in, x0)
+        env = {"input": (x0, fin)}
+        last = len(q.layers) - 1
+        for i, L_ in enumerate(q.layers):
+            nm = L_["name"]
+            mode = F.OUT_ACC64 if i == last else F.OUT_CODES
+            if L_["type"] == "conv":
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                y, s = q.run_layer(i, env, N, mode)
+                e1.record(stream)
+                e1.synchronize()
+                if it > 0:
+                    tot_ms += e0.elapsed_time(e1)
+                    H, _, K = q.shapes[nm]
+                    flops += 2 * N * H * H * K * L_["C"] * L_["R"] * L_["R"]
+                    n += 1
+            else:
+                y, s = q.run_layer(i, env, N, mode)
+            env[nm] = (y, q.fmts[nm].get("a"))
+        del env0
+        env0 = env
+    return tot_ms, flops, n
+
+
+# ----------------------------------------------------------------------------- CPU oracle arm
+def oracle_step(workload, n_images=1):
+    """The oracle evaluating one candidate plan on a bounded sample: parameter FL search and
+    quantization, calibration on a 1-image slice, forward of `n_images` images."""
+    import oracle.net as onet
+    wl = WORKLOADS[workload]
+    arch = wl["arch"]
+    layers = synth.ARCHS[arch]()
+    W = synth.weights(arch, wl["seed"])
+    imgs = synth.images(n_images, wl["seed"])
+    plan = synth.bit_plan(arch, wl["plans"][0])
+    t0 = time.perf_counter()
+    fm, qp = onet.calibrate(layers, W, imgs[:1], plan)
+    onet.forward(layers, fm, qp, imgs)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(workload):
+    t = oracle_step(workload, 1)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {"value": round(1.0 / t, 5), "unit": "images/s", "cores": cores, "kind": "oracle",
+            "sample": f"{workload}: one candidate plan -- parameter FL search + quantize, calibration on a "
+                      f"1-image slice, forward of 1 image ({t:.1f} s)"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    ts = [oracle_step(args.workload, 1) for _ in range(args.warmup)]
+    ts = [oracle_step(args.workload, 1) for _ in range(args.steps)]
+    t = sum(ts) / len(ts)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    v = round(1.0 / t, 5)
+    print(json.dumps({
+        "impl": "reference", "metric": "images/s for fixed-point net forward (one candidate plan evaluated per step)",
+        "value": v, "unit": "images/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(t * 1e3, 1), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int64 (exact)", "data": "synthetic",
+        "config": {"workload": args.workload, "model": args.workload, "global_batch": 1, "seq_len": None,
+                   "parallelism": "cpu"},
+        "cpu_baseline": {"value": v, "unit": "images/s", "cores": cores, "kind": "oracle",
+                         "sample": "one candidate plan on 1 image (calibration slice of 1 image)"},
+        "e2e": {"value": v, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="fxpq", choices=["fxpq", "reference"])
+    ap.add_argument("--workload", default="vgg16", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline leg")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_fxpq(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,241 @@
+/*
+ * fxpq.h -- C ABI of libfxpq.so: the data-parallel hot path of evaluating a CNN under a
+ * dynamic fixed-point configuration (FxP-QNet, Shawahna et al., IEEE Access 2022,
+ * arXiv 2203.12091), on one NVIDIA GB300 (sm_103a).
+ *
+ * Conventions shared by every entry point
+ *   - Pointers named d_* are device pointers; h_* are host pointers.  The caller owns every
+ *     buffer.  The library allocates no device memory: scratch comes from the caller's
+ *     workspace, sized by the matching *_workspace() query.
+ *   - Calls are asynchronous on the caller's stream (a cudaStream_t passed as void*;
+ *     NULL = the legacy default stream), except where a function says it synchronises.
+ *   - Arguments are validated on the host before any launch; a failed check returns an error
+ *     code and launches nothing.  Errors detected on the device (non-finite input, a bounded
+ *     wait that ran out) are latched in a device status word read by fxpq_get_device_status().
+ *   - Results are deterministic: no floating-point atomics; repeated calls are bit-identical.
+ *
+ * Notation follows the paper: a data-structure is a group of k-bit integer codes sharing the
+ * scale 2^-FL ("beta" in the paper); k = alpha + beta (Sec. II-A); S is the sign strategy
+ * (0 = unsigned U(alpha, beta), 1 = two's complement S(alpha, beta)).
+ *
+ * Code storage ("fp16 code tensors").  Inside the network path every code tensor is stored as
+ * fp16 values that are exact integers.  A format with k <= 8 bits uses one plane (|code| <= 255).
+ * A format with 9..16 bits uses two planes, hi and lo, with code = 256*hi + lo, lo in [0, 255]
+ * and hi = floor(code / 256); the planes are concatenated along the innermost (channel) axis:
+ * [hi_0 .. hi_{C-1}, lo_0 .. lo_{C-1}].  Channel counts are padded to a multiple of 8 with
+ * zero codes.
+ */
+#ifndef FXPQ_H
+#define FXPQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FXPQ_API __attribute__((visibility("default")))
+#else
+#define FXPQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FXPQ_OK = 0,
+    FXPQ_ERR_INVALID_ARG = 1, /* a null/misaligned pointer, a size or a format out of range     */
+    FXPQ_ERR_UNSUPPORTED = 2, /* a valid request this build does not implement                  */
+    FXPQ_ERR_NONFINITE = 3,   /* fl_search / quantize saw a NaN or Inf (latched on the device)  */
+    FXPQ_ERR_TIMEOUT = 4,     /* a bounded device-side wait gave up (latched on the device)     */
+    FXPQ_ERR_CUDA = 5,        /* a CUDA runtime call failed                                     */
+    FXPQ_ERR_WORKSPACE = 6,   /* the workspace is null or smaller than the query returned       */
+    FXPQ_ERR_RANGE = 7        /* an integer bound the exact arithmetic relies on would not hold */
+} fxpq_status;
+
+/* Storage of integer codes in device memory. */
+typedef enum {
+    FXPQ_DT_I8 = 0,  /* int8   : signed formats, k <= 8       */
+    FXPQ_DT_U8 = 1,  /* uint8  : unsigned formats, k <= 8     */
+    FXPQ_DT_I16 = 2, /* int16  : signed formats, k <= 16      */
+    FXPQ_DT_U16 = 3, /* uint16 : unsigned formats, k <= 16    */
+    FXPQ_DT_I32 = 4, /* int32  : any format                   */
+    FXPQ_DT_F16 = 5  /* fp16 code tensor (see the file header): one or two limb planes */
+} fxpq_dtype;
+
+/* Quantization parameters of one data-structure (Sec. IV-A.3 / IV-B): wordlength k = bits,
+ * sign strategy S = is_signed, fractional length beta = fl; alpha = bits - fl. */
+typedef struct {
+    int32_t bits;      /* 2..16 (32 is accepted for biases, which are int32 codes) */
+    int32_t is_signed; /* 0: U(alpha, beta), codes in [0, 2^k - 1]; 1: S(alpha, beta), [-2^(k-1), 2^(k-1) - 1] */
+    int32_t fl;        /* beta, in [-32, 40] */
+} fxpq_fmt;
+
+/* Statistics gathered by the FL-search pass over a tensor. */
+typedef struct {
+    float min, max;     /* exact                                                          */
+    int32_t is_signed;  /* sign strategy of Sec. IV-A.3: 1 iff min < 0                     */
+    int32_t nonfinite;  /* 1 if a NaN/Inf was seen (the scores are then not meaningful)    */
+    double sum, sumsq;  /* exact sums rounded once to double                               */
+    int64_t n;
+} fxpq_stats;
+
+/* ---------------------------------------------------------------------------------------- */
+/* Quantizer Q (Sec. IV-B, Eq. fp_k_bit_quantization, Eq. clip, Eq. quantization_levels):   */
+/*   code_i = clip(round_half_even(x_i * 2^fl), Qmin, Qmax),                                */
+/*   Qmin = -S * 2^(k-S), Qmax = 2^(k-S) - 1.                                                */
+/* d_x: n fp32 values.  d_codes: n codes in storage `dtype` (I8/U8/I16/U16/I32 must be wide   */
+/* enough and of the right signedness; F16 writes the limb planes of a [n/c, c] tensor with   */
+/* c = n, i.e. plane hi at [0, n) and lo at [n, 2n) for k > 8).  n may be 0.                 */
+/* NaN/Inf inputs latch FXPQ_ERR_NONFINITE and produce code 0.                               */
+/* ---------------------------------------------------------------------------------------- */
+FXPQ_API fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int32_t dtype, void* d_codes,
+                          void* stream);
+
+/* Quantize a row-major [rows, C] fp32 tensor (e.g. KRSC weights with C innermost) into an fp16
+ * code tensor [rows, Cp * planes] (planes per f.bits, see the file header); channels C..Cp-1 are
+ * zero codes.  Cp is a multiple of 8 and >= C. */
+FXPQ_API fxpq_status fxpq_quantize_rows(const float* d_x, int64_t rows, int32_t C, fxpq_fmt f, int32_t Cp, void* d_y,
+                               void* stream);
+
+/* Quantize + transpose + pack fp32 images NCHW -> NHWC fp16 code tensor with the channel count
+ * padded to c_pad (a multiple of 8, >= C) with zero codes: the FxP-QLayer inserted at the input
+ * of the network (Sec. IV-A.2).  d_y holds N*H*W*c_pad*planes fp16 values. */
+FXPQ_API fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, int32_t C, int32_t H, int32_t W,
+                                 fxpq_fmt f, int32_t c_pad, void* d_y, void* stream);
+
+/* ---------------------------------------------------------------------------------------- */
+/* FL search (Sec. IV-C, Eq. DSB_QE; sign strategy Sec. IV-A.3).                             */
+/* One pass over d_x scores every candidate (k, fl), k in [k_lo, k_hi] and fl in              */
+/* [fl_lo, fl_hi]:  L(k, fl) = sum_i (x_i - Q(x_i; k, fl) * 2^-fl)^2  -- the exact sum,       */
+/* rounded once to nearest-even double.                                                      */
+/*   is_signed: 0 or 1 fixes S; -1 picks S = 1 iff min(x) < 0.                                */
+/*   d_err  : device double[(k_hi-k_lo+1) * (fl_hi-fl_lo+1)], row-major [k][fl].              */
+/*   d_best : device int32[k_hi-k_lo+1]: the fl with the smallest L per k, exact ties to the  */
+/*            smallest fl.                                                                   */
+/*   d_stats: device fxpq_stats (may be NULL).                                               */
+/* Limits: 2 <= k_lo <= k_hi <= 16; -32 <= fl_lo <= fl_hi <= 40; fl_hi - fl_lo <= 31;         */
+/* 0 <= n <= 2^31.  Non-finite inputs latch FXPQ_ERR_NONFINITE.                              */
+/* Workspace: fxpq_fl_search_workspace() bytes, 256-byte aligned; contents are scratch.       */
+/* ---------------------------------------------------------------------------------------- */
+FXPQ_API size_t fxpq_fl_search_workspace(int64_t n);
+FXPQ_API fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo, int32_t k_hi,
+                           int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
+                           fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream);
+
+/* Initial quantization parameters (Sec. IV-A.3, Eq. initial_quantization_parameters), a host
+ * helper on statistics already copied to the host: psi from the range, beta_hat = -log2(psi),
+ * beta = floor (strategy 0, conservative) / round half-even (1, neutral) / ceil (2, aggressive).
+ * Where one of the two signed candidates for psi is not positive it is dropped. */
+FXPQ_API fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32_t strategy, fxpq_fmt* h_out);
+
+/* ---------------------------------------------------------------------------------------- */
+/* C-Block: convolution / FC on codes with exact integer accumulation and the fused epilogue */
+/* (Sec. IV-B, the C-Block paragraph and its figure; FxP-QLayer placement Sec. IV-A.2):      */
+/*   acc[n,p,q,o] = sum_{r,s,c} X[n, p*st+r-pad, q*st+s-pad, c] * W[o, r, s, c]    (exact)    */
+/*   value scale s = fl_x + fl_w; bias aligned with delta = s - fl_b: delta >= 0 adds          */
+/*   B << delta, delta < 0 shifts acc left by -delta first (no bit is dropped);               */
+/*   ReLU = max(., 0) if relu;                                                               */
+/*   out_mode CODES : FxP-QLayer -> round_half_even(v * 2^(fl_y - s)), clip to fmt_y,         */
+/*                    written as an fp16 code tensor NHWC with Kp = K padded to 8;            */
+/*   out_mode ACC64 : no QLayer (last layer): int64 v, NHWC [N,P,Q,K]; its scale exponent is   */
+/*                    returned in *h_out_scale;                                               */
+/*   out_mode F32   : fp32 nearest-even image of v * 2^-s (for calibrating fmt_y.fl).          */
+/* X: fp16 code tensor NHWC [N,H,W,Cp] (planes per fmt_x.bits); W: fp16 code tensor KRSC       */
+/* [K,R,S,Cp] (planes per fmt_w.bits); d_bias: int32 codes [K] or NULL.                       */
+/* An FC layer is a convolution whose window covers the whole input map (R = H, S = W).      */
+/* Returns FXPQ_ERR_RANGE if |acc| could exceed 2^62 after alignment.                         */
+/* ---------------------------------------------------------------------------------------- */
+enum { FXPQ_OUT_CODES = 0, FXPQ_OUT_ACC64 = 1, FXPQ_OUT_F32 = 2 };
+
+typedef struct {
+    int32_t N, H, W, C;        /* input geometry; C = true channel count                    */
+    int32_t Cp;                /* stored channel count of X and W (multiple of 8, >= C)      */
+    int32_t K, R, S;           /* output channels, window                                   */
+    int32_t stride, pad;
+    int32_t relu;
+    int32_t out_mode;          /* FXPQ_OUT_*                                                 */
+    fxpq_fmt fmt_x, fmt_w, fmt_b, fmt_y;
+} fxpq_conv_desc;
+
+FXPQ_API size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc);
+FXPQ_API fxpq_status fxpq_conv_fwd(const fxpq_conv_desc* h_desc, const void* d_x, const void* d_w,
+                          const int32_t* d_bias, void* d_y, int32_t* h_out_scale, void* d_ws,
+                          size_t ws_bytes, void* stream);
+
+/* FC layer as a GEMM: X [M, Kdim] (fp16 codes, Kdim padded to 8), W [N, Kdim]; same epilogue. */
+FXPQ_API fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_w, fxpq_fmt fmt_w,
+                      const int32_t* d_bias, fxpq_fmt fmt_b, int32_t M, int32_t N, int32_t Kdim,
+                      int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y, int32_t* h_out_scale,
+                      void* d_ws, size_t ws_bytes, void* stream);
+
+/* MAX-POOL on codes (Sec. IV-A.2: no FxP-QLayer follows; the format is unchanged).  Window
+ * k x k, stride, pad; taps outside the map are ignored.  X, Y: fp16 code tensors NHWC with
+ * Cp channels (planes per fmt.bits, pooled as whole codes). */
+FXPQ_API fxpq_status fxpq_maxpool(const void* d_x, int32_t N, int32_t H, int32_t W, int32_t Cp, fxpq_fmt fmt,
+                         int32_t k, int32_t stride, int32_t pad, void* d_y, void* stream);
+
+/* Eltwise C-Block (Sec. IV-A.2, residual add): both inputs aligned to max(fl_a, fl_b) by an
+ * exact left shift, added, optional ReLU, then the FxP-QLayer to fmt_y (or F32 / ACC64 as in
+ * fxpq_conv_fwd).  A, B, Y: NHWC with Cp channels, count = n_pix * Cp codes. */
+FXPQ_API fxpq_status fxpq_eltwise(const void* d_a, fxpq_fmt fmt_a, const void* d_b, fxpq_fmt fmt_b, int64_t n_pix,
+                         int32_t Cp, int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y,
+                         int32_t* h_out_scale, void* stream);
+
+/* Global AVG-POOL (Sec. IV-A.2: the reciprocal of the patch size is quantized like a parameter):
+ * v[n,c] = recip_code * sum_{h,w} X[n,h,w,c], scale fl_x + fmt_recip.fl, then the FxP-QLayer to
+ * fmt_y (or F32 / ACC64).  Output NHWC with H = W = 1. */
+FXPQ_API fxpq_status fxpq_avgpool(const void* d_x, int32_t N, int32_t H, int32_t W, int32_t Cp, fxpq_fmt fmt_x,
+                         int32_t recip_code, fxpq_fmt fmt_recip, int32_t out_mode, fxpq_fmt fmt_y,
+                         void* d_y, int32_t* h_out_scale, void* stream);
+
+/* ---------------------------------------------------------------------------------------- */
+/* Network forward (Sec. IV-A.2: FxP-QLayers as vertices, C-Blocks as edges).                */
+/* A network is a list of ops over numbered tensor slots; slot 0 is the input image codes.   */
+/* Every op reads its source slot(s) and writes slot `dst`.  The last op must be a CONV with  */
+/* last = 1: its int64 accumulator (no QLayer, Sec. IV-A.2) is written to d_logits            */
+/* [batch, K] and its scale exponent to *h_logits_scale.                                      */
+/* ---------------------------------------------------------------------------------------- */
+enum { FXPQ_OP_CONV = 0, FXPQ_OP_MAXPOOL = 1, FXPQ_OP_ELTWISE = 2, FXPQ_OP_AVGPOOL = 3 };
+
+typedef struct {
+    int32_t op;              /* FXPQ_OP_*                                                    */
+    int32_t src0, src1;      /* source slots (src1: second eltwise operand, else -1)         */
+    int32_t dst;             /* destination slot                                             */
+    int32_t K, R, S;         /* conv: output channels and window; maxpool: window in R (=S)   */
+    int32_t stride, pad;
+    int32_t relu;
+    int32_t last;            /* 1 for the final conv/FC (int64 logits)                       */
+    int32_t recip_code;      /* avgpool: quantized reciprocal of the patch size             */
+    fxpq_fmt fmt_w, fmt_b;   /* conv: weight and bias formats; avgpool: fmt_w = reciprocal  */
+    fxpq_fmt fmt_y;          /* format of the output QLayer (ignored for maxpool / last)    */
+    const void* d_w;         /* conv: fp16 code tensor KRSC [K, R, S, Cp_in]                 */
+    const int32_t* d_bias;   /* conv: int32 bias codes [K] or NULL                           */
+} fxpq_op_desc;
+
+typedef struct {
+    int32_t n_ops;
+    int32_t n_slots;
+    int32_t C, H, W;          /* input image geometry (NCHW fp32)                           */
+    int32_t Cp_in;            /* padded channel count of slot 0                             */
+    fxpq_fmt fmt_in;          /* input FxP-QLayer format                                    */
+    const fxpq_op_desc* ops;  /* host array of n_ops descriptors                            */
+} fxpq_net;
+
+FXPQ_API size_t fxpq_net_workspace(const fxpq_net* h_net, int32_t batch);
+FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_images_nchw, int32_t batch,
+                             int64_t* d_logits, int32_t* h_logits_scale, void* d_ws, size_t ws_bytes,
+                             void* stream);
+
+/* Synchronises `stream`, returns and clears the latched device status (FXPQ_OK if none). */
+FXPQ_API fxpq_status fxpq_get_device_status(void* stream);
+
+/* Static English description of a status code. */
+FXPQ_API const char* fxpq_status_string(fxpq_status s);
+
+/* Number of kernel launches this library issued since load (instrumentation for benchmarks). */
+FXPQ_API int64_t fxpq_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FXPQ_H */

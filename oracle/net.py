@@ -66,6 +66,8 @@ def _layer_pass(layers, i, L, env, fmts, qparams, calibrating: bool, plan):
         v, s = eltwise_add(a, fa[2], b, fb[2], L["relu"])
     elif L["type"] == "avgpool":
         x, fx = env[L.get("src") or prev]
+        if calibrating:  # reciprocal of the patch size, searched like a parameter
+            fmts[name]["r"] = search_fmt(np.array([1.0 / (x.shape[1] * x.shape[2])], dtype=np.float32), plan[name]["r"])
         rk, rS, rfl = fmts[name]["r"]
         rcode = int(quantize(np.array([1.0 / (x.shape[1] * x.shape[2])], dtype=np.float32), rk, rS, rfl)[0])
         v, s = avgpool_global(x, fx[2], rcode, rfl)
@@ -90,9 +92,6 @@ def quantize_params(layers, weights, plan):
             fb = search_fmt(b, plan[nm]["b"])
             fmts[nm]["w"], fmts[nm]["b"] = fw, fb
             qparams[nm] = (quantize(w, *fw).reshape(w.shape), quantize(b, *fb))
-        elif L["type"] == "avgpool":
-            # reciprocal of the 7x7 patch of a 224x224 input, handled like a parameter
-            fmts[nm]["r"] = search_fmt(np.array([1.0 / 49.0], dtype=np.float32), plan[nm]["r"])
     return fmts, qparams
 
 

@@ -1,0 +1,62 @@
+// fxpq_common.cuh -- internal helpers shared by the libfxpq.so translation units.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/fxpq.h"
+
+namespace fxpq {
+
+// ---------------------------------------------------------------- host-side bookkeeping
+// Device address of the latched status word (one per device; defined in fxpq_host.cu).
+int* status_ptr();
+// Count one kernel launch (for benchmarks) and check the launch error.
+fxpq_status after_launch(const char* what);
+void note_launch();
+
+inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
+
+inline bool fmt_ok(const fxpq_fmt& f, int max_bits = 16) {
+    return f.bits >= 2 && f.bits <= max_bits && (f.is_signed == 0 || f.is_signed == 1) && f.fl >= -32 &&
+           f.fl <= 40;
+}
+inline int planes_of(const fxpq_fmt& f) { return f.bits > 8 ? 2 : 1; }
+inline int64_t qmin_of(const fxpq_fmt& f) { return f.is_signed ? -(int64_t(1) << (f.bits - 1)) : 0; }
+inline int64_t qmax_of(const fxpq_fmt& f) { return (int64_t(1) << (f.bits - f.is_signed)) - 1; }
+inline bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ---------------------------------------------------------------- device helpers
+__device__ __forceinline__ void latch_status(int* st, int code) {
+    if (st) atomicCAS(st, 0, code);
+}
+
+// Round half to even of v / 2^sh for sh >= 1 (exact, int64): the FxP-QLayer's shift.
+__device__ __forceinline__ long long rne_shift(long long v, int sh) {
+    long long q = v >> sh;  // floor (arithmetic shift)
+    unsigned long long rem = (unsigned long long)(v - (q << sh));
+    unsigned long long half = 1ull << (sh - 1);
+    q += (rem > half) || (rem == half && (q & 1));
+    return q;
+}
+
+// value * 2^(fl_out - s) rounded half-even, clipped to [lo, hi]  (sh = s - fl_out)
+__device__ __forceinline__ long long requant_value(long long v, int sh, long long lo, long long hi) {
+    long long q;
+    if (sh > 0)
+        q = rne_shift(v, sh);
+    else
+        q = v << (-sh);
+    return q < lo ? lo : (q > hi ? hi : q);
+}
+
+// Code <-> fp16 limb planes: code = 256*hi + lo with lo in [0,255].
+__device__ __forceinline__ void split_limbs(int code, __half& hi, __half& lo) {
+    int h = code >> 8;  // floor division
+    int l = code - (h << 8);
+    hi = __int2half_rn(h);
+    lo = __int2half_rn(l);
+}
+
+}  // namespace fxpq

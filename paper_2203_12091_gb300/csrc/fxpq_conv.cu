@@ -1,0 +1,220 @@
+// fxpq_conv.cu -- C-Block on integer codes (Sec. IV-B): convolution / FC with exact integer
+// accumulation and the fused epilogue (bias alignment, ReLU, FxP-QLayer shift-requantize).
+//
+// This translation unit holds the CUDA-core implicit-GEMM kernel (exact int32 / int64 MACs),
+// used for every shape, and the host entry points.
+#include <math.h>
+
+#include "fxpq_common.cuh"
+#include "fxpq_conv.cuh"
+
+namespace fxpq {
+namespace {
+
+__device__ __forceinline__ int load_code(const __half* __restrict__ t, long long row, int Cp, int planes, int c) {
+    const __half* p = t + row * (long long)Cp * planes;
+    if (planes == 1) return __half2int_rn(p[c]);
+    return (__half2int_rn(p[c]) << 8) + __half2int_rn(p[Cp + c]);
+}
+
+constexpr int TM = 64, TN = 64, TK = 16, NT = 256;
+
+template <typename ACC>
+__global__ void __launch_bounds__(NT) conv_simt_kernel(ConvArgs a) {
+    __shared__ int As[TK][TM + 1];
+    __shared__ int Bs[TK][TN + 1];
+    const int tid = threadIdx.x;
+    const int tx = tid % 16, ty = tid / 16;
+    const long long M = (long long)a.N * a.P * a.Q;
+    const long long m0 = (long long)blockIdx.x * TM;
+    const int n0 = blockIdx.y * TN;
+
+    // per-thread loader coordinates: 4 (row, channel) entries of the A and B tiles
+    long long pix_n[4];
+    int pix_p[4], pix_q[4];
+    bool pix_ok[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        int e = tid + NT * i;
+        long long m = m0 + (e >> 4);
+        pix_ok[i] = m < M;
+        long long mm = pix_ok[i] ? m : 0;
+        pix_n[i] = mm / ((long long)a.P * a.Q);
+        int pq = (int)(mm - pix_n[i] * a.P * a.Q);
+        pix_p[i] = pq / a.Q;
+        pix_q[i] = pq - pix_p[i] * a.Q;
+    }
+
+    ACC acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0;
+
+    for (int r = 0; r < a.R; ++r)
+        for (int s = 0; s < a.S; ++s)
+            for (int c0 = 0; c0 < a.Cp; c0 += TK) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    int e = tid + NT * i;
+                    int cc = e & (TK - 1);
+                    int row = e >> 4;
+                    int c = c0 + cc;
+                    int code = 0;
+                    int h = pix_p[i] * a.stride + r - a.pad;
+                    int w = pix_q[i] * a.stride + s - a.pad;
+                    if (pix_ok[i] && c < a.Cp && h >= 0 && h < a.H && w >= 0 && w < a.W)
+                        code = load_code(a.x, (pix_n[i] * a.H + h) * a.W + w, a.Cp, a.px, c);
+                    As[cc][row] = code;
+                    int k = n0 + row;
+                    int wc = 0;
+                    if (k < a.K && c < a.Cp) wc = load_code(a.w, ((long long)k * a.R + r) * a.S + s, a.Cp, a.pw, c);
+                    Bs[cc][row] = wc;
+                }
+                __syncthreads();
+#pragma unroll
+                for (int cc = 0; cc < TK; ++cc) {
+                    int av[4], bv[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) av[i] = As[cc][ty * 4 + i];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) bv[j] = Bs[cc][tx * 4 + j];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) acc[i][j] += (ACC)av[i] * (ACC)bv[j];
+                }
+                __syncthreads();
+            }
+
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        long long m = m0 + ty * 4 + i;
+        if (m >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            int k = n0 + tx * 4 + j;
+            if (k < a.K) cblock_epilogue_store(a, m, k, (long long)acc[i][j]);
+        }
+    }
+}
+
+}  // namespace
+
+// Host-side planning shared by conv and gemm: fills ConvArgs, checks the integer bounds.
+fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, const int32_t* bias, void* y,
+                      ConvArgs& a, int32_t* out_scale, bool& need64) {
+    if (d.N < 0 || d.H < 1 || d.W < 1 || d.C < 1 || d.Cp < d.C || (d.Cp % 8) || d.K < 1 || d.R < 1 || d.S < 1 ||
+        d.stride < 1 || d.pad < 0)
+        return FXPQ_ERR_INVALID_ARG;
+    if (!fmt_ok(d.fmt_x) || !fmt_ok(d.fmt_w)) return FXPQ_ERR_INVALID_ARG;
+    if (bias && !fmt_ok(d.fmt_b, 32)) return FXPQ_ERR_INVALID_ARG;
+    if (d.out_mode < FXPQ_OUT_CODES || d.out_mode > FXPQ_OUT_F32) return FXPQ_ERR_INVALID_ARG;
+    if (d.out_mode == FXPQ_OUT_CODES && (!fmt_ok(d.fmt_y) || (d.K % 8))) return FXPQ_ERR_INVALID_ARG;
+    const int P = (d.H + 2 * d.pad - d.R) / d.stride + 1, Q = (d.W + 2 * d.pad - d.S) / d.stride + 1;
+    if (P < 1 || Q < 1) return FXPQ_ERR_INVALID_ARG;
+    if (d.N > 0 && (!x || !w || !y)) return FXPQ_ERR_INVALID_ARG;
+    if (!aligned(x, 16) || !aligned(w, 16) || !aligned(y, 16)) return FXPQ_ERR_INVALID_ARG;
+    // |acc| <= max|x code| * max|w code| * R*S*C
+    const double ax = ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed), aw = ldexp(1.0, d.fmt_w.bits - d.fmt_w.is_signed);
+    const double bound = ax * aw * (double)d.R * d.S * d.C;
+    if (bound >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+    need64 = bound >= ldexp(1.0, 31) - 1.0;
+    a.x = static_cast<const __half*>(x);
+    a.w = static_cast<const __half*>(w);
+    a.bias = bias;
+    a.y = y;
+    a.N = d.N, a.H = d.H, a.W = d.W, a.Cp = d.Cp, a.K = d.K, a.R = d.R, a.S = d.S;
+    a.stride = d.stride, a.pad = d.pad, a.P = P, a.Q = Q;
+    a.px = planes_of(d.fmt_x);
+    a.pw = planes_of(d.fmt_w);
+    a.relu = d.relu;
+    a.out_mode = d.out_mode;
+    int s = d.fmt_x.fl + d.fmt_w.fl;
+    a.delta = 0;
+    double vbound = bound;
+    if (bias) {
+        a.delta = s - d.fmt_b.fl;
+        const double bb = ldexp(1.0, d.fmt_b.bits - d.fmt_b.is_signed);
+        if (a.delta >= 0) {
+            if (a.delta > 40 || bb * ldexp(1.0, a.delta) + bound >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+            vbound = bound + bb * ldexp(1.0, a.delta);
+        } else {
+            if (-a.delta > 40 || bound * ldexp(1.0, -a.delta) + bb >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+            vbound = bound * ldexp(1.0, -a.delta) + bb;
+            s = d.fmt_b.fl;
+        }
+    }
+    (void)vbound;
+    a.s_out = s;
+    a.has_bias = bias != nullptr;
+    if (d.out_mode == FXPQ_OUT_CODES) {
+        a.sh = s - d.fmt_y.fl;
+        if (a.sh > 62) return FXPQ_ERR_RANGE;
+        a.lo = qmin_of(d.fmt_y);
+        a.hi = qmax_of(d.fmt_y);
+        a.py = planes_of(d.fmt_y);
+    } else {
+        a.sh = 0;
+        a.lo = a.hi = 0;
+        a.py = 1;
+    }
+    a.f32_scale = ldexpf(1.0f, -s);
+    if (out_scale) *out_scale = s;
+    return FXPQ_OK;
+}
+
+fxpq_status launch_conv(const ConvArgs& a, bool need64, cudaStream_t st) {
+    const long long M = (long long)a.N * a.P * a.Q;
+    if (M == 0) return FXPQ_OK;
+    dim3 grid((unsigned)((M + TM - 1) / TM), (unsigned)((a.K + TN - 1) / TN));
+    if (need64)
+        conv_simt_kernel<long long><<<grid, NT, 0, st>>>(a);
+    else
+        conv_simt_kernel<int><<<grid, NT, 0, st>>>(a);
+    return after_launch("conv_simt");
+}
+
+}  // namespace fxpq
+
+using namespace fxpq;
+
+extern "C" size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc) {
+    (void)h_desc;
+    return 0;
+}
+
+extern "C" fxpq_status fxpq_conv_fwd(const fxpq_conv_desc* h_desc, const void* d_x, const void* d_w,
+                                     const int32_t* d_bias, void* d_y, int32_t* h_out_scale, void* d_ws,
+                                     size_t ws_bytes, void* stream) {
+    (void)d_ws;
+    (void)ws_bytes;
+    if (!h_desc) return FXPQ_ERR_INVALID_ARG;
+    ConvArgs a;
+    bool need64 = false;
+    fxpq_status st = plan_conv(*h_desc, d_x, d_w, d_bias, d_y, a, h_out_scale, need64);
+    if (st != FXPQ_OK) return st;
+    return launch_conv(a, need64, as_stream(stream));
+}
+
+extern "C" fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_w, fxpq_fmt fmt_w,
+                                 const int32_t* d_bias, fxpq_fmt fmt_b, int32_t M, int32_t N, int32_t Kdim,
+                                 int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y, int32_t* h_out_scale,
+                                 void* d_ws, size_t ws_bytes, void* stream) {
+    fxpq_conv_desc d;
+    d.N = M;
+    d.H = d.W = 1;
+    d.C = Kdim;
+    d.Cp = Kdim;
+    d.K = N;
+    d.R = d.S = 1;
+    d.stride = 1;
+    d.pad = 0;
+    d.relu = relu;
+    d.out_mode = out_mode;
+    d.fmt_x = fmt_x;
+    d.fmt_w = fmt_w;
+    d.fmt_b = fmt_b;
+    d.fmt_y = fmt_y;
+    return fxpq_conv_fwd(&d, d_x, d_w, d_bias, d_y, h_out_scale, d_ws, ws_bytes, stream);
+}

@@ -1,0 +1,66 @@
+// fxpq_conv.cuh -- arguments and fused epilogue of the C-Block kernels (Sec. IV-B).
+#pragma once
+
+#include "fxpq_common.cuh"
+
+namespace fxpq {
+
+struct ConvArgs {
+    const __half* x;   // NHWC fp16 code tensor [N, H, W, Cp * px]
+    const __half* w;   // KRSC fp16 code tensor [K, R, S, Cp * pw]
+    const int32_t* bias;
+    void* y;           // CODES: fp16 [M, K * py]; ACC64: int64 [M, K]; F32: float [M, K]
+    int N, H, W, Cp, K, R, S, stride, pad, P, Q;
+    int px, pw, py;
+    int relu, out_mode, has_bias;
+    int delta;         // bias alignment: s_acc - fl_b
+    int s_out;         // scale exponent after alignment
+    int sh;            // FxP-QLayer right shift s_out - fl_y
+    long long lo, hi;  // clip levels of fmt_y
+    float f32_scale;   // 2^-s_out
+};
+
+// Bias alignment, ReLU and the FxP-QLayer for one output value of row m, channel k.
+__device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long long m, int k, long long v) {
+    if (a.has_bias) {
+        const long long b = a.bias[k];
+        if (a.delta >= 0)
+            v += b << a.delta;
+        else
+            v = (v << (-a.delta)) + b;
+    }
+    if (a.relu && v < 0) v = 0;
+    if (a.out_mode == FXPQ_OUT_CODES) {
+        long long q;
+        if (a.sh > 0) {
+            q = rne_shift(v, a.sh);
+        } else {
+            const int l = -a.sh;  // left shift; saturate before it could overflow
+            const long long lim = 1LL << 20;
+            if (l >= 32 || v > lim || v < -lim)
+                q = v > 0 ? a.hi : (v < 0 ? a.lo : 0);
+            else
+                q = v << l;
+        }
+        q = q < a.lo ? a.lo : (q > a.hi ? a.hi : q);
+        __half* y = static_cast<__half*>(a.y);
+        if (a.py == 1) {
+            y[m * a.K + k] = __int2half_rn((int)q);
+        } else {
+            __half h, l;
+            split_limbs((int)q, h, l);
+            y[m * 2LL * a.K + k] = h;
+            y[m * 2LL * a.K + a.K + k] = l;
+        }
+    } else if (a.out_mode == FXPQ_OUT_ACC64) {
+        static_cast<long long*>(a.y)[m * a.K + k] = v;
+    } else {
+        static_cast<float*>(a.y)[m * a.K + k] = __ll2float_rn(v) * a.f32_scale;
+    }
+}
+
+fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, const int32_t* bias, void* y,
+                      ConvArgs& a, int32_t* out_scale, bool& need64);
+fxpq_status launch_conv(const ConvArgs& a, bool need64, cudaStream_t st);
+
+}  // namespace fxpq

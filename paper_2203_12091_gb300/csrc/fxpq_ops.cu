@@ -1,0 +1,186 @@
+// fxpq_ops.cu -- the non-contraction C-Blocks of the integer-only graph (Sec. IV-A.2):
+// MAX-POOL (no FxP-QLayer), Eltwise residual add with FL alignment, global AVG-POOL with the
+// reciprocal of the patch size quantized like a parameter.  All HBM-bound, one thread per output.
+#include "fxpq_common.cuh"
+
+namespace fxpq {
+namespace {
+
+__device__ __forceinline__ int code_at(const __half* __restrict__ t, long long pix, int Cp, int planes, int c) {
+    const __half* p = t + pix * (long long)Cp * planes;
+    if (planes == 1) return __half2int_rn(p[c]);
+    return (__half2int_rn(p[c]) << 8) + __half2int_rn(p[Cp + c]);
+}
+
+__device__ __forceinline__ void put_code(__half* __restrict__ t, long long pix, int Cp, int planes, int c, int code) {
+    __half* p = t + pix * (long long)Cp * planes;
+    if (planes == 1) {
+        p[c] = __int2half_rn(code);
+    } else {
+        __half h, l;
+        split_limbs(code, h, l);
+        p[c] = h;
+        p[Cp + c] = l;
+    }
+}
+
+struct OutArgs {
+    int mode;         // FXPQ_OUT_*
+    int sh;           // requant shift (CODES)
+    long long lo, hi;
+    int py;
+    float f32_scale;  // 2^-s
+};
+
+__device__ __forceinline__ void store_out(const OutArgs& o, void* y, long long pix, int Cp, int c, long long v) {
+    if (o.mode == FXPQ_OUT_CODES) {
+        long long q;
+        if (o.sh > 0) {
+            q = rne_shift(v, o.sh);
+        } else {
+            const int l = -o.sh;
+            const long long lim = 1LL << 20;
+            if (l >= 32 || v > lim || v < -lim)
+                q = v > 0 ? o.hi : (v < 0 ? o.lo : 0);
+            else
+                q = v << l;
+        }
+        q = q < o.lo ? o.lo : (q > o.hi ? o.hi : q);
+        put_code(static_cast<__half*>(y), pix, Cp, o.py, c, (int)q);
+    } else if (o.mode == FXPQ_OUT_ACC64) {
+        static_cast<long long*>(y)[pix * Cp + c] = v;
+    } else {
+        static_cast<float*>(y)[pix * Cp + c] = __ll2float_rn(v) * o.f32_scale;
+    }
+}
+
+__global__ void maxpool_kernel(const __half* __restrict__ x, int N, int H, int W, int Cp, int planes, int k,
+                               int stride, int pad, int P, int Q, __half* __restrict__ y) {
+    const long long total = (long long)N * P * Q * Cp;
+    const long long step = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += step) {
+        const int c = (int)(i % Cp);
+        const long long pix = i / Cp;
+        const int q = (int)(pix % Q);
+        const int p = (int)((pix / Q) % P);
+        const long long n = pix / ((long long)P * Q);
+        int best = INT_MIN;
+        for (int r = 0; r < k; ++r) {
+            const int h = p * stride + r - pad;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < k; ++s) {
+                const int w = q * stride + s - pad;
+                if (w < 0 || w >= W) continue;
+                best = max(best, code_at(x, (n * H + h) * W + w, Cp, planes, c));
+            }
+        }
+        put_code(y, pix, Cp, planes, c, best);
+    }
+}
+
+__global__ void eltwise_kernel(const __half* __restrict__ a, int pa, int sa, const __half* __restrict__ b, int pb,
+                               int sb, long long npix, int Cp, int relu, OutArgs o, void* y) {
+    const long long total = npix * Cp;
+    const long long step = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += step) {
+        const int c = (int)(i % Cp);
+        const long long pix = i / Cp;
+        long long v = ((long long)code_at(a, pix, Cp, pa, c) << sa) + ((long long)code_at(b, pix, Cp, pb, c) << sb);
+        if (relu && v < 0) v = 0;
+        store_out(o, y, pix, Cp, c, v);
+    }
+}
+
+__global__ void avgpool_kernel(const __half* __restrict__ x, int N, int HW, int Cp, int planes, long long recip,
+                               OutArgs o, void* y) {
+    const long long total = (long long)N * Cp;
+    const long long step = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += step) {
+        const int c = (int)(i % Cp);
+        const long long n = i / Cp;
+        long long s = 0;
+        for (int t = 0; t < HW; ++t) s += code_at(x, n * HW + t, Cp, planes, c);
+        store_out(o, y, n, Cp, c, s * recip);
+    }
+}
+
+int grid_for(long long work) {
+    long long b = (work + 255) / 256;
+    if (b < 1) b = 1;
+    if (b > 152LL * 32) b = 152LL * 32;
+    return (int)b;
+}
+
+fxpq_status make_out(int mode, const fxpq_fmt& fy, int s, OutArgs& o, int32_t* h_out_scale) {
+    if (mode < FXPQ_OUT_CODES || mode > FXPQ_OUT_F32) return FXPQ_ERR_INVALID_ARG;
+    o.mode = mode;
+    if (mode == FXPQ_OUT_CODES) {
+        if (!fmt_ok(fy)) return FXPQ_ERR_INVALID_ARG;
+        o.sh = s - fy.fl;
+        if (o.sh > 62) return FXPQ_ERR_RANGE;
+        o.lo = qmin_of(fy);
+        o.hi = qmax_of(fy);
+        o.py = planes_of(fy);
+    } else {
+        o.sh = 0;
+        o.lo = o.hi = 0;
+        o.py = 1;
+    }
+    o.f32_scale = ldexpf(1.0f, -s);
+    if (h_out_scale) *h_out_scale = s;
+    return FXPQ_OK;
+}
+
+}  // namespace
+}  // namespace fxpq
+
+using namespace fxpq;
+
+extern "C" fxpq_status fxpq_maxpool(const void* d_x, int32_t N, int32_t H, int32_t W, int32_t Cp, fxpq_fmt fmt,
+                                    int32_t k, int32_t stride, int32_t pad, void* d_y, void* stream) {
+    if (N < 0 || H < 1 || W < 1 || Cp < 1 || (Cp % 8) || k < 1 || stride < 1 || pad < 0 || pad >= k || !fmt_ok(fmt))
+        return FXPQ_ERR_INVALID_ARG;
+    const int P = (H + 2 * pad - k) / stride + 1, Q = (W + 2 * pad - k) / stride + 1;
+    if (P < 1 || Q < 1) return FXPQ_ERR_INVALID_ARG;
+    if (N == 0) return FXPQ_OK;
+    if (!d_x || !d_y) return FXPQ_ERR_INVALID_ARG;
+    const long long total = (long long)N * P * Q * Cp;
+    maxpool_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(static_cast<const __half*>(d_x), N, H, W, Cp,
+                                                                   planes_of(fmt), k, stride, pad, P, Q,
+                                                                   static_cast<__half*>(d_y));
+    return after_launch("maxpool");
+}
+
+extern "C" fxpq_status fxpq_eltwise(const void* d_a, fxpq_fmt fmt_a, const void* d_b, fxpq_fmt fmt_b, int64_t n_pix,
+                                    int32_t Cp, int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y,
+                                    int32_t* h_out_scale, void* stream) {
+    if (n_pix < 0 || Cp < 1 || (Cp % 8) || !fmt_ok(fmt_a) || !fmt_ok(fmt_b)) return FXPQ_ERR_INVALID_ARG;
+    const int fl = fmt_a.fl > fmt_b.fl ? fmt_a.fl : fmt_b.fl;
+    const int sa = fl - fmt_a.fl, sb = fl - fmt_b.fl;
+    if (sa > 40 || sb > 40) return FXPQ_ERR_RANGE;
+    OutArgs o;
+    fxpq_status st = make_out(out_mode, fmt_y, fl, o, h_out_scale);
+    if (st != FXPQ_OK) return st;
+    if (n_pix == 0) return FXPQ_OK;
+    if (!d_a || !d_b || !d_y) return FXPQ_ERR_INVALID_ARG;
+    eltwise_kernel<<<grid_for(n_pix * Cp), 256, 0, as_stream(stream)>>>(
+        static_cast<const __half*>(d_a), planes_of(fmt_a), sa, static_cast<const __half*>(d_b), planes_of(fmt_b), sb,
+        n_pix, Cp, relu, o, d_y);
+    return after_launch("eltwise");
+}
+
+extern "C" fxpq_status fxpq_avgpool(const void* d_x, int32_t N, int32_t H, int32_t W, int32_t Cp, fxpq_fmt fmt_x,
+                                    int32_t recip_code, fxpq_fmt fmt_recip, int32_t out_mode, fxpq_fmt fmt_y,
+                                    void* d_y, int32_t* h_out_scale, void* stream) {
+    if (N < 0 || H < 1 || W < 1 || Cp < 1 || (Cp % 8) || !fmt_ok(fmt_x) || !fmt_ok(fmt_recip))
+        return FXPQ_ERR_INVALID_ARG;
+    if (recip_code < qmin_of(fmt_recip) || recip_code > qmax_of(fmt_recip)) return FXPQ_ERR_INVALID_ARG;
+    OutArgs o;
+    fxpq_status st = make_out(out_mode, fmt_y, fmt_x.fl + fmt_recip.fl, o, h_out_scale);
+    if (st != FXPQ_OK) return st;
+    if (N == 0) return FXPQ_OK;
+    if (!d_x || !d_y) return FXPQ_ERR_INVALID_ARG;
+    avgpool_kernel<<<grid_for((long long)N * Cp), 256, 0, as_stream(stream)>>>(
+        static_cast<const __half*>(d_x), N, H * W, Cp, planes_of(fmt_x), (long long)recip_code, o, d_y);
+    return after_launch("avgpool");
+}

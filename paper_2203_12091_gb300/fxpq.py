@@ -1,0 +1,166 @@
+"""Python binding of libfxpq.so: same names as include/fxpq.h, torch tensors in, argument
+marshalling only.  PyTorch provides device memory and streams; every step runs in the library's
+CUDA kernels.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _lib as L
+from ._lib import DT_F16, DT_I8, DT_I16, DT_I32, DT_U8, DT_U16, OUT_ACC64, OUT_CODES, OUT_F32, Fmt, Stats  # noqa: F401
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _s(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def fmt(bits: int, is_signed: int, fl: int) -> Fmt:
+    return Fmt(int(bits), int(is_signed), int(fl))
+
+
+def planes(f: Fmt) -> int:
+    return 2 if f.bits > 8 else 1
+
+
+_WS = {}
+
+
+def workspace(nbytes: int, device=None) -> torch.Tensor:
+    """A cached uint8 device buffer of at least nbytes (256-byte aligned by the allocator)."""
+    dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+    t = _WS.get(dev)
+    if t is None or t.numel() < nbytes:
+        t = torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=dev)
+        _WS[dev] = t
+    return t
+
+
+# ------------------------------------------------------------------------------ quantizer
+def fxpq_quantize(x, f: Fmt, dtype: int, out, stream=None):
+    L.check("fxpq_quantize", L.lib().fxpq_quantize(_p(x), x.numel(), f, dtype, _p(out), _s(stream)))
+    return out
+
+
+def fxpq_quantize_rows(x, rows: int, C: int, f: Fmt, Cp: int, out, stream=None):
+    L.check("fxpq_quantize_rows", L.lib().fxpq_quantize_rows(_p(x), rows, C, f, Cp, _p(out), _s(stream)))
+    return out
+
+
+def fxpq_quantize_images(x_nchw, f: Fmt, c_pad: int, out, stream=None):
+    N, C, H, W = x_nchw.shape
+    L.check("fxpq_quantize_images",
+            L.lib().fxpq_quantize_images(_p(x_nchw), N, C, H, W, f, c_pad, _p(out), _s(stream)))
+    return out
+
+
+# ------------------------------------------------------------------------------ FL search
+def fxpq_fl_search_workspace(n: int) -> int:
+    return int(L.lib().fxpq_fl_search_workspace(n))
+
+
+def fxpq_fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, err, best, stats, ws, stream=None):
+    L.check("fxpq_fl_search",
+            L.lib().fxpq_fl_search(_p(x), x.numel(), is_signed, k_lo, k_hi, fl_lo, fl_hi, _p(err), _p(best),
+                                   _p(stats), _p(ws), ws.numel(), _s(stream)))
+
+
+def fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, stream=None):
+    """Allocate the outputs and run fxpq_fl_search.  Returns device (err[nk, nfl], best[nk], stats bytes)."""
+    nk, nfl = k_hi - k_lo + 1, fl_hi - fl_lo + 1
+    dev = x.device
+    err = torch.empty(nk * nfl, dtype=torch.float64, device=dev)
+    best = torch.empty(nk, dtype=torch.int32, device=dev)
+    stats = torch.empty(ctypes.sizeof(Stats), dtype=torch.uint8, device=dev)
+    ws = workspace(fxpq_fl_search_workspace(x.numel()), dev)
+    fxpq_fl_search(x, is_signed, k_lo, k_hi, fl_lo, fl_hi, err, best, stats, ws, stream)
+    return err.view(nk, nfl), best, stats
+
+
+def stats_from_device(stats_bytes) -> Stats:
+    return Stats.from_buffer_copy(bytes(stats_bytes.cpu().numpy().tobytes()))
+
+
+def fxpq_fl_init(stats: Stats, bits: int, strategy: int) -> Fmt:
+    out = Fmt()
+    L.check("fxpq_fl_init", L.lib().fxpq_fl_init(ctypes.byref(stats), bits, strategy, ctypes.byref(out)))
+    return out
+
+
+# ------------------------------------------------------------------------------ C-Blocks
+def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy) -> L.ConvDesc:
+    return L.ConvDesc(N, H, W, C, Cp, K, R, S, stride, pad, int(relu), out_mode, fx, fw,
+                      fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0))
+
+
+def fxpq_conv_fwd(desc: L.ConvDesc, x, w, bias, y, stream=None) -> int:
+    scale = L.I32(0)
+    L.check("fxpq_conv_fwd", L.lib().fxpq_conv_fwd(ctypes.byref(desc), _p(x), _p(w), _p(bias), _p(y),
+                                                   ctypes.byref(scale), None, 0, _s(stream)))
+    return scale.value
+
+
+def fxpq_gemm(x, fx, w, fw, bias, fb, M, N, Kdim, relu, out_mode, fy, y, stream=None) -> int:
+    scale = L.I32(0)
+    L.check("fxpq_gemm", L.lib().fxpq_gemm(_p(x), fx, _p(w), fw, _p(bias), fb if fb is not None else Fmt(32, 1, 0),
+                                           M, N, Kdim, int(relu), out_mode, fy if fy is not None else Fmt(8, 1, 0),
+                                           _p(y), ctypes.byref(scale), None, 0, _s(stream)))
+    return scale.value
+
+
+def fxpq_maxpool(x, N, H, W, Cp, f: Fmt, k, stride, pad, y, stream=None):
+    L.check("fxpq_maxpool", L.lib().fxpq_maxpool(_p(x), N, H, W, Cp, f, k, stride, pad, _p(y), _s(stream)))
+    return y
+
+
+def fxpq_eltwise(a, fa: Fmt, b, fb: Fmt, n_pix, Cp, relu, out_mode, fy, y, stream=None) -> int:
+    scale = L.I32(0)
+    L.check("fxpq_eltwise", L.lib().fxpq_eltwise(_p(a), fa, _p(b), fb, n_pix, Cp, int(relu), out_mode,
+                                                 fy if fy is not None else Fmt(8, 1, 0), _p(y), ctypes.byref(scale),
+                                                 _s(stream)))
+    return scale.value
+
+
+def fxpq_avgpool(x, N, H, W, Cp, fx: Fmt, recip_code: int, fr: Fmt, out_mode, fy, y, stream=None) -> int:
+    scale = L.I32(0)
+    L.check("fxpq_avgpool", L.lib().fxpq_avgpool(_p(x), N, H, W, Cp, fx, int(recip_code), fr, out_mode,
+                                                 fy if fy is not None else Fmt(8, 1, 0), _p(y), ctypes.byref(scale),
+                                                 _s(stream)))
+    return scale.value
+
+
+def fxpq_net_workspace(net: L.Net, batch: int) -> int:
+    return int(L.lib().fxpq_net_workspace(ctypes.byref(net), batch))
+
+
+def fxpq_net_forward(net: L.Net, images, batch, logits, ws, stream=None) -> int:
+    scale = L.I32(0)
+    L.check("fxpq_net_forward", L.lib().fxpq_net_forward(ctypes.byref(net), _p(images), batch, _p(logits),
+                                                         ctypes.byref(scale), _p(ws), ws.numel(), _s(stream)))
+    return scale.value
+
+
+def fxpq_get_device_status(stream=None) -> int:
+    return int(L.lib().fxpq_get_device_status(_s(stream)))
+
+
+def fxpq_launch_count() -> int:
+    return int(L.lib().fxpq_launch_count())
+
+
+# ------------------------------------------------------------------------------ code tensors
+def codes_to_int(t: torch.Tensor, f: Fmt, C: int | None = None) -> torch.Tensor:
+    """Decode an fp16 code tensor [..., Cp * planes] to int64 codes [..., Cp] (host-side view for tests)."""
+    t = t.to(torch.int64)
+    if planes(f) == 1:
+        out = t
+    else:
+        cp = t.shape[-1] // 2
+        out = t[..., :cp] * 256 + t[..., cp:]
+    return out if C is None else out[..., :C]

@@ -1,0 +1,246 @@
+"""Host-side planning of an integer-only network: parameter quantization, calibration of the
+activation formats, and the op list handed to ``fxpq_net_forward`` (Sec. IV-A.2).
+
+A layer list is a list of dicts (the format the workload generators produce):
+  {"type": "conv", "name", "C", "K", "R", "stride", "pad", "relu", "src"}   (FC = conv over the map)
+  {"type": "maxpool", "name", "k", "stride", "pad"}
+  {"type": "eltwise", "name", "a", "b", "relu"}
+  {"type": "avgpool", "name", "src"}
+``src`` (or ``a``/``b``) names the producing layer; ``None`` means the previous layer, and
+"input" is the network input.  The last layer must be a conv/FC: it has no FxP-QLayer.
+
+Calibration follows the forward optimizer's order (Sec. IV-C): layer by layer, weights' FL, then
+bias FL, then the output activation FL; each FL comes from ``fxpq_fl_search`` at the planned
+wordlength over FL in [-8, 23], sign strategy by Sec. IV-A.3; activation FLs are searched on the
+fp32 image of the exact C-Block output of the calibration slice, with every preceding layer
+already quantized.  Every arithmetic step runs in libfxpq.so; this module only sequences calls
+and reads back the chosen formats.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _lib as L
+from . import fxpq as F
+
+FL_LO, FL_HI = -8, 23
+
+
+def pad8(c: int) -> int:
+    return (c + 7) // 8 * 8
+
+
+def search_fmt(x: torch.Tensor, k: int, stream=None) -> L.Fmt:
+    """FL search at one wordlength; returns the chosen (k, S, FL).  Synchronises (reads 16 bytes)."""
+    _, best, stats = F.fl_search(x.reshape(-1), -1, k, k, FL_LO, FL_HI, stream)
+    st = F.stats_from_device(stats)
+    return F.fmt(k, st.is_signed, int(best[0].item()))
+
+
+class QNet:
+    """A quantized network on one device: code tensors, formats, and the fxpq_net op list."""
+
+    def __init__(self, layers, hw=224, cin=3):
+        self.layers = layers
+        self.hw, self.cin = hw, cin
+        self.cp_in = pad8(cin)
+        self.fmts = {}
+        self.q = {}  # name -> (weight fp16 codes, bias int32 codes)
+        self.names = ["input"] + [L_["name"] for L_ in layers]
+        self.slot = {nm: i for i, nm in enumerate(self.names)}
+        self.shapes = {}
+
+    # ------------------------------------------------------------------ parameters
+    def _src(self, i, L_, key="src"):
+        s = L_.get(key)
+        return s if s is not None else (self.names[i] if i > 0 else "input")
+
+    def quantize_params(self, weights_dev, plan, stream=None):
+        """weights_dev: name -> (fp32 KRSC weight, fp32 bias) device tensors; plan: wordlengths."""
+        shapes = {"input": (self.hw, self.hw, self.cp_in)}
+        for i, L_ in enumerate(self.layers):
+            nm = L_["name"]
+            self.fmts.setdefault(nm, {})
+            if L_["type"] == "conv":
+                H, W, Cp = shapes[self._src(i, L_)]
+                w, b = weights_dev[nm]
+                K, R, _, C = w.shape
+                assert C <= Cp
+                fw = search_fmt(w, plan[nm]["w"], stream)
+                fb = search_fmt(b, plan[nm]["b"], stream)
+                wq = torch.empty(K * R * R, Cp * F.planes(fw), dtype=torch.float16, device=w.device)
+                F.fxpq_quantize_rows(w.reshape(-1, C), K * R * R, C, fw, Cp, wq, stream)
+                bq = torch.empty(K, dtype=torch.int32, device=w.device)
+                F.fxpq_quantize(b, fb, F.DT_I32, bq, stream)
+                self.fmts[nm]["w"], self.fmts[nm]["b"] = fw, fb
+                self.q[nm] = (wq, bq)
+                P = (H + 2 * L_["pad"] - R) // L_["stride"] + 1
+                shapes[nm] = (P, P, K)
+            elif L_["type"] == "maxpool":
+                H, W, Cp = shapes[self._src(i, L_)]
+                P = (H + 2 * L_["pad"] - L_["k"]) // L_["stride"] + 1
+                shapes[nm] = (P, P, Cp)
+            elif L_["type"] == "eltwise":
+                shapes[nm] = shapes[L_["a"]]
+            elif L_["type"] == "avgpool":
+                H, W, Cp = shapes[self._src(i, L_)]
+                dev = next(iter(weights_dev.values()))[0].device
+                r = torch.tensor([1.0 / (H * W)], dtype=torch.float32, device=dev)
+                fr = search_fmt(r, plan[nm]["r"], stream)
+                rc = torch.empty(1, dtype=torch.int32, device=dev)
+                F.fxpq_quantize(r, fr, F.DT_I32, rc, stream)
+                self.fmts[nm]["r"] = fr
+                self.q[nm] = (None, int(rc.item()))
+                shapes[nm] = (1, 1, Cp)
+        self.shapes = shapes
+
+    # ------------------------------------------------------------------ one C-Block on device tensors
+    def run_layer(self, i, env, N, out_mode, stream=None):
+        """Run layer i on env[name] = (tensor, fmt); returns (output tensor, scale exponent)."""
+        L_ = self.layers[i]
+        nm = L_["name"]
+        H, W, Cp = self.shapes[nm]
+        fy = self.fmts[nm].get("a")
+        if out_mode == F.OUT_CODES:
+            y = torch.empty(N * H * W * Cp * F.planes(fy), dtype=torch.float16, device=self._dev)
+        elif out_mode == F.OUT_F32:
+            y = torch.empty(N * H * W * Cp, dtype=torch.float32, device=self._dev)
+        else:
+            y = torch.empty(N * H * W * Cp, dtype=torch.int64, device=self._dev)
+        if L_["type"] == "conv":
+            src = self._src(i, L_)
+            x, fx = env[src]
+            sH, sW, sCp = self.shapes[src]
+            wq, bq = self.q[nm]
+            d = F.conv_desc(N, sH, sW, sCp, sCp, L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], L_["relu"],
+                            out_mode, fx, self.fmts[nm]["w"], self.fmts[nm]["b"], fy)
+            s = F.fxpq_conv_fwd(d, x, wq, bq, y, stream)
+        elif L_["type"] == "maxpool":
+            src = self._src(i, L_)
+            x, fx = env[src]
+            sH, sW, sCp = self.shapes[src]
+            F.fxpq_maxpool(x, N, sH, sW, sCp, fx, L_["k"], L_["stride"], L_["pad"], y, stream)
+            s = fx.fl
+        elif L_["type"] == "eltwise":
+            (a, fa), (b, fb) = env[L_["a"]], env[L_["b"]]
+            s = F.fxpq_eltwise(a, fa, b, fb, N * H * W, Cp, L_["relu"], out_mode, fy, y, stream)
+        elif L_["type"] == "avgpool":
+            src = self._src(i, L_)
+            x, fx = env[src]
+            sH, sW, sCp = self.shapes[src]
+            s = F.fxpq_avgpool(x, N, sH, sW, sCp, fx, self.q[nm][1], self.fmts[nm]["r"], out_mode, fy, y, stream)
+        else:
+            raise ValueError(L_["type"])
+        return y, s
+
+    # ------------------------------------------------------------------ calibration (Sec. IV-C order)
+    def calibrate(self, calib_images, plan, stream=None):
+        self._dev = calib_images.device
+        N = calib_images.shape[0]
+        fin = search_fmt(calib_images, plan["input"], stream)
+        self.fmts["input"] = {"a": fin}
+        x0 = torch.empty(N * self.hw * self.hw * self.cp_in * F.planes(fin), dtype=torch.float16, device=self._dev)
+        F.fxpq_quantize_images(calib_images, fin, self.cp_in, x0, stream)
+        env = {"input": (x0, fin)}
+        last = len(self.layers) - 1
+        for i, L_ in enumerate(self.layers):
+            nm = L_["name"]
+            if i == last:
+                break
+            if L_["type"] == "maxpool":
+                src = self._src(i, L_)
+                self.fmts[nm]["a"] = env[src][1]
+                y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
+                env[nm] = (y, env[src][1])
+                continue
+            v, _ = self.run_layer(i, env, N, F.OUT_F32, stream)
+            self.fmts[nm]["a"] = search_fmt(v, plan[nm]["a"], stream)
+            y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
+            env[nm] = (y, self.fmts[nm]["a"])
+        self._build_ops()
+        return self.fmts
+
+    # ------------------------------------------------------------------ forward through the C ABI
+    def _build_ops(self):
+        ops = (L.OpDesc * len(self.layers))()
+        last = len(self.layers) - 1
+        for i, L_ in enumerate(self.layers):
+            o = ops[i]
+            nm = L_["name"]
+            o.dst = 0 if i == last else self.slot[nm]
+            o.last = 1 if i == last else 0
+            o.src1 = -1
+            if L_["type"] == "conv":
+                o.op = L.OP_CONV
+                o.src0 = self.slot[self._src(i, L_)]
+                o.K, o.R, o.S, o.stride, o.pad, o.relu = L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], int(L_["relu"])
+                o.fmt_w, o.fmt_b = self.fmts[nm]["w"], self.fmts[nm]["b"]
+                o.fmt_y = self.fmts[nm].get("a", L.Fmt(8, 1, 0))
+                o.d_w = self.q[nm][0].data_ptr()
+                o.d_bias = self.q[nm][1].data_ptr()
+            elif L_["type"] == "maxpool":
+                o.op = L.OP_MAXPOOL
+                o.src0 = self.slot[self._src(i, L_)]
+                o.R = o.S = L_["k"]
+                o.stride, o.pad = L_["stride"], L_["pad"]
+            elif L_["type"] == "eltwise":
+                o.op = L.OP_ELTWISE
+                o.src0, o.src1 = self.slot[L_["a"]], self.slot[L_["b"]]
+                o.relu = int(L_["relu"])
+                o.fmt_y = self.fmts[nm]["a"]
+            elif L_["type"] == "avgpool":
+                o.op = L.OP_AVGPOOL
+                o.src0 = self.slot[self._src(i, L_)]
+                o.recip_code = self.q[nm][1]
+                o.fmt_w = self.fmts[nm]["r"]
+                o.fmt_y = self.fmts[nm]["a"]
+        self._ops = ops
+        self.net = L.Net(len(self.layers), len(self.names), self.cin, self.hw, self.hw, self.cp_in,
+                         self.fmts["input"]["a"], ctypes.cast(ops, ctypes.POINTER(L.OpDesc)))
+        self.n_classes = self.layers[-1]["K"]
+
+    def workspace_bytes(self, batch: int) -> int:
+        return F.fxpq_net_workspace(self.net, batch)
+
+    def forward(self, images, logits=None, ws=None, stream=None):
+        """images: fp32 NCHW device tensor.  Returns (int64 logits [N, classes], scale exponent)."""
+        N = images.shape[0]
+        if logits is None:
+            logits = torch.empty(N, self.n_classes, dtype=torch.int64, device=images.device)
+        if ws is None:
+            ws = F.workspace(self.workspace_bytes(N), images.device)
+        s = F.fxpq_net_forward(self.net, images, N, logits, ws, stream)
+        return logits, s
+
+    def trace(self, images, stream=None):
+        """Per-layer outputs (codes) of a forward with frozen formats, op by op (for parity tests)."""
+        self._dev = images.device
+        N = images.shape[0]
+        fin = self.fmts["input"]["a"]
+        x0 = torch.empty(N * self.hw * self.hw * self.cp_in * F.planes(fin), dtype=torch.float16, device=self._dev)
+        F.fxpq_quantize_images(images, fin, self.cp_in, x0, stream)
+        env = {"input": (x0, fin)}
+        last = len(self.layers) - 1
+        for i, L_ in enumerate(self.layers):
+            nm = L_["name"]
+            if i == last:
+                y, s = self.run_layer(i, env, N, F.OUT_ACC64, stream)
+                env[nm] = (y, s)
+                break
+            f = self.fmts[nm]["a"]
+            y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
+            env[nm] = (y, f)
+        return env
+
+
+def build_qnet(layers, weights_np, calib_images, plan, device="cuda", stream=None):
+    """Quantize parameters and calibrate on `calib_images` (fp32 NCHW device tensor)."""
+    wdev = {nm: (torch.from_numpy(w).to(device), torch.from_numpy(b).to(device)) for nm, (w, b) in weights_np.items()}
+    q = QNet(layers, hw=calib_images.shape[-1], cin=calib_images.shape[1])
+    q._dev = torch.device(device)
+    q.quantize_params(wdev, plan, stream)
+    q.calibrate(calib_images, plan, stream)
+    q.weights_dev = wdev
+    return q

@@ -1,0 +1,110 @@
+"""C ABI checks that need no GPU: the library builds and loads, exports exactly what
+include/fxpq.h declares, and its host-side validation and host-only helpers behave."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2203_12091_gb300 import _lib as L
+from paper_2203_12091_gb300 import build as B
+
+HDR = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "fxpq.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return L.lib()
+
+
+def declared():
+    src = open(HDR).read()
+    return sorted(set(re.findall(r"FXPQ_API\s+[\w\s\*]*?\b(fxpq_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared()
+    for must in ("fxpq_fl_search", "fxpq_quantize", "fxpq_conv_fwd", "fxpq_gemm", "fxpq_net_forward"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", B.LIB], capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\sT\s(fxpq_\w+)", out))
+    assert set(declared()) <= exported
+    assert set(declared()) == set(L.declared_symbols())
+    for n in declared():
+        assert hasattr(lib, n)
+
+
+def test_host_validation_rejects_bad_arguments(lib):
+    f8 = L.Fmt(8, 1, 4)
+    assert lib.fxpq_quantize(None, -1, f8, L.DT_I8, None, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_quantize(None, 4, L.Fmt(1, 1, 0), L.DT_I8, None, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_quantize(None, 4, L.Fmt(8, 1, 41), L.DT_I8, None, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_quantize(ctypes.c_void_p(256), 4, L.Fmt(9, 1, 0), L.DT_I8, ctypes.c_void_p(256), None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_quantize(ctypes.c_void_p(256), 4, L.Fmt(8, 0, 0), L.DT_I8, ctypes.c_void_p(256), None) == L.ERR_INVALID_ARG
+    p = ctypes.c_void_p(256)
+    ws = lib.fxpq_fl_search_workspace(100)
+    assert ws > 0 and ws % 256 == 0
+    # k out of range, FL span too wide, missing outputs, workspace too small / misaligned
+    assert lib.fxpq_fl_search(p, 100, -1, 1, 8, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 17, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 8, -8, 24, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, 2, 2, 8, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 8, 0, 10, None, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 8, 0, 10, p, p, None, p, ws - 1, None) == L.ERR_WORKSPACE
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 8, 0, 10, p, p, None, ctypes.c_void_p(258), ws, None) == L.ERR_WORKSPACE
+    assert lib.fxpq_fl_search(p, 100, -1, 2, 8, 0, 10, p, p, None, None, ws, None) == L.ERR_WORKSPACE
+    # conv: misaligned pointers, bad geometry, integer range
+    d = L.ConvDesc(1, 8, 8, 8, 8, 8, 3, 3, 1, 1, 1, L.OUT_CODES, f8, f8, L.Fmt(16, 1, 8), f8)
+    sc = L.I32()
+    assert lib.fxpq_conv_fwd(ctypes.byref(d), ctypes.c_void_p(258), p, None, p, ctypes.byref(sc), None, 0, None) == L.ERR_INVALID_ARG
+    d.Cp = 12
+    assert lib.fxpq_conv_fwd(ctypes.byref(d), p, p, None, p, ctypes.byref(sc), None, 0, None) == L.ERR_INVALID_ARG
+    d.Cp, d.K = 8, 12
+    assert lib.fxpq_conv_fwd(ctypes.byref(d), p, p, None, p, ctypes.byref(sc), None, 0, None) == L.ERR_INVALID_ARG
+    d.K = 8
+    d.fmt_b = L.Fmt(32, 1, -30)  # delta = 8 - (-30) = 38: B << 38 of a 32-bit bias leaves int64
+    assert lib.fxpq_conv_fwd(ctypes.byref(d), p, p, p, p, ctypes.byref(sc), None, 0, None) == L.ERR_RANGE
+    assert lib.fxpq_maxpool(p, 1, 4, 4, 8, f8, 3, 2, 3, p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_eltwise(p, f8, p, L.Fmt(8, 1, 60), 4, 8, 0, 0, f8, p, None, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_avgpool(p, 1, 7, 7, 8, f8, 70000, L.Fmt(16, 0, 21), 0, f8, p, None, None) == L.ERR_INVALID_ARG
+
+
+def test_net_planning_rejects_malformed_graphs(lib):
+    ops = (L.OpDesc * 1)()
+    ops[0].op = L.OP_MAXPOOL
+    ops[0].last = 1
+    net = L.Net(1, 2, 3, 8, 8, 8, L.Fmt(8, 1, 4), ctypes.cast(ops, ctypes.POINTER(L.OpDesc)))
+    assert lib.fxpq_net_workspace(ctypes.byref(net), 4) == 0  # last op must be a conv
+    ops[0].op = L.OP_CONV
+    ops[0].K, ops[0].R, ops[0].S, ops[0].stride = 8, 3, 3, 1
+    ops[0].d_w = 256
+    assert lib.fxpq_net_workspace(ctypes.byref(net), 4) > 0
+    ops[0].src0 = 1  # undefined source slot
+    assert lib.fxpq_net_workspace(ctypes.byref(net), 4) == 0
+
+
+@pytest.mark.parametrize("mn,mx,k", [(0.0, 1.0, 8), (-2.0, 1.0, 8), (-0.5, 0.5, 8), (0.0, 3.7, 4), (-1e-3, 2e-3, 16),
+                                     (-5.0, -1.0, 6), (0.0, 1e-4, 8)])
+def test_fl_init_matches_oracle(lib, mn, mx, k):
+    for strat, name in enumerate(("conservative", "neutral", "aggressive")):
+        st = L.Stats(mn, mx, 0, 0, 0.0, 0.0, 1)
+        out = L.Fmt()
+        code = lib.fxpq_fl_init(ctypes.byref(st), k, strat, ctypes.byref(out))
+        try:
+            S, beta, _ = oracle.fl_init(float(st.min), float(st.max), k, name)
+        except ValueError:
+            assert code == L.ERR_INVALID_ARG
+            continue
+        assert code == L.OK and (out.is_signed, out.fl, out.bits) == (S, beta, k)
+
+
+def test_status_strings(lib):
+    for c in range(8):
+        assert lib.fxpq_status_string(c)
+    assert lib.fxpq_launch_count() >= 0

@@ -1,0 +1,174 @@
+"""GPU parity of the C-Block kernels (conv / FC with the fused epilogue, max-pool, eltwise,
+avg-pool) against the CPU oracle: bit-exact codes, accumulators and fp32 calibration images."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def F():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2203_12091_gb300 import fxpq
+    return fxpq
+
+
+def rand_codes(rng, shape, k, S):
+    lo, hi = oracle.qmin(k, S), oracle.qmax(k, S)
+    c = rng.integers(lo, hi + 1, size=shape)
+    # make the extremes appear
+    flat = c.reshape(-1)
+    flat[: min(4, flat.size)] = [lo, hi, lo, hi][: min(4, flat.size)]
+    return c
+
+
+def to_f16_planes(codes, k, Cp):
+    """Storage encoding of a code tensor [..., C] as fp16 planes [..., Cp * planes] (zero padded)."""
+    c = np.zeros(codes.shape[:-1] + (Cp,), np.int64)
+    c[..., : codes.shape[-1]] = codes
+    if k <= 8:
+        return torch.from_numpy(c.astype(np.float16)).cuda()
+    hi = c >> 8
+    lo = c - (hi << 8)
+    return torch.from_numpy(np.concatenate([hi, lo], axis=-1).astype(np.float16)).cuda()
+
+
+def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp):
+    N, H, W, C = x.shape
+    K, R, S, _ = w.shape
+    P = (H + 2 * pad - R) // stride + 1
+    Q = (W + 2 * pad - S) // stride + 1
+    xd = to_f16_planes(x, fx.bits, Cp)
+    wd = to_f16_planes(w, fw.bits, Cp)
+    bd = torch.from_numpy(b.astype(np.int32)).cuda() if b is not None else None
+    if mode == F.OUT_CODES:
+        y = torch.empty(N * P * Q * K * (2 if fy.bits > 8 else 1), dtype=torch.float16, device="cuda")
+    elif mode == F.OUT_ACC64:
+        y = torch.empty(N * P * Q * K, dtype=torch.int64, device="cuda")
+    else:
+        y = torch.empty(N * P * Q * K, dtype=torch.float32, device="cuda")
+    d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy)
+    s = F.fxpq_conv_fwd(d, xd, wd, bd, y)
+    torch.cuda.synchronize()
+    assert F.fxpq_get_device_status() == 0
+    if mode == F.OUT_CODES:
+        return F.codes_to_int(y.cpu().view(N, P, Q, -1), fy).numpy(), s
+    return y.cpu().numpy().reshape(N, P, Q, K), s
+
+
+def oracle_conv(x, fx, w, fw, b, fb, stride, pad, relu, mode, fy):
+    acc = oracle.conv2d(x, w, stride, pad)
+    v, s = oracle.cblock(acc, fx.fl + fw.fl, b, fb.fl if fb is not None else 0, relu)
+    if mode == 0:
+        return oracle.requant(v, s, fy.bits, fy.is_signed, fy.fl), s
+    if mode == 1:
+        return v, s
+    return oracle.to_f32(v, s), s
+
+
+CASES = [
+    # N, H, C, K, R, stride, pad, (kx,Sx,flx), (kw,Sw,flw), (kb,flb) or None, relu, mode, (ky,Sy,fly)
+    (2, 9, 8, 16, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),
+    (3, 13, 24, 72, 5, 2, 2, (8, 0, 2), (8, 1, 9), (16, 19), True, 0, (8, 0, 5)),
+    (2, 39, 3, 96, 11, 4, 2, (8, 1, 5), (8, 1, 8), (16, 18), True, 0, (8, 0, 2)),
+    (2, 14, 64, 32, 1, 2, 0, (6, 0, 3), (7, 1, 8), (16, 17), False, 0, (7, 1, 4)),
+    (3, 6, 64, 24, 6, 1, 0, (8, 0, 4), (4, 1, 6), (16, 16), True, 0, (8, 0, 1)),
+    (2, 11, 16, 16, 3, 1, 1, (16, 1, 12), (16, 1, 14), (16, 20), True, 0, (16, 0, 9)),
+    (1, 10, 8, 8, 3, 1, 1, (16, 1, 12), (16, 1, 14), (16, 20), False, 1, None),
+    (2, 9, 16, 40, 3, 1, 1, (5, 1, 2), (4, 1, 3), (16, 9), False, 1, None),        # delta < 0: acc shifted left
+    (2, 9, 16, 40, 3, 1, 0, (8, 0, 4), (8, 1, 7), None, True, 2, None),            # no bias, fp32 calibration image
+    (2, 8, 32, 16, 3, 2, 1, (8, 0, 6), (8, 1, 8), (16, 22), False, 2, None),
+    (4, 7, 8, 8, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (4, 0, 20)),      # left-shift requant + saturate
+    (1, 5, 3, 8, 3, 1, 1, (3, 1, 1), (3, 1, 2), (16, 10), True, 0, (2, 0, 0)),
+]
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_conv_parity(F, case):
+    N, H, C, K, R, st, pad, tx, tw, tb, relu, mode, ty = case
+    rng = np.random.default_rng(H * 131 + K)
+    fx, fw = F.fmt(*tx), F.fmt(*tw)
+    fb = F.fmt(tb[0], 1, tb[1]) if tb else None
+    fy = F.fmt(*ty) if ty else None
+    x = rand_codes(rng, (N, H, H, C), tx[0], tx[1])
+    w = rand_codes(rng, (K, R, R, C), tw[0], tw[1])
+    # realistic weight magnitudes: mostly small codes
+    w = np.where(rng.random(w.shape) < 0.8, w // 4, w)
+    b = rand_codes(rng, (K,), tb[0], 1) if tb else None
+    Cp = (C + 7) // 8 * 8
+    got, s = run_conv(F, x, fx, w, fw, b, fb, st, pad, relu, mode, fy, Cp)
+    want, ws = oracle_conv(x, fx, w, fw, b, fb, st, pad, relu, mode, fy)
+    assert s == ws
+    assert np.array_equal(got[..., :K], want)
+
+
+def test_gemm_entry_point(F):
+    rng = np.random.default_rng(3)
+    M, N, Kd = 37, 48, 200
+    fx, fw, fb, fy = F.fmt(8, 0, 5), F.fmt(8, 1, 9), F.fmt(16, 1, 20), F.fmt(8, 0, 4)
+    x = rand_codes(rng, (M, Kd), 8, 0)
+    w = rand_codes(rng, (N, Kd), 8, 1) // 3
+    b = rand_codes(rng, (N,), 16, 1)
+    y = torch.empty(M * N, dtype=torch.float16, device="cuda")
+    s = F.fxpq_gemm(to_f16_planes(x, 8, Kd), fx, to_f16_planes(w, 8, Kd), fw, torch.from_numpy(b.astype(np.int32)).cuda(),
+                    fb, M, N, Kd, True, F.OUT_CODES, fy, y)
+    want, ws = oracle_conv(x.reshape(M, 1, 1, Kd), fx, w.reshape(N, 1, 1, Kd), fw, b, fb, 1, 0, True, 0, fy)
+    assert s == ws
+    assert np.array_equal(F.codes_to_int(y.cpu().view(M, N), fy).numpy(), want.reshape(M, N))
+
+
+@pytest.mark.parametrize("k,st,pad,bits", [(3, 2, 0, 8), (2, 2, 0, 6), (3, 2, 1, 8), (3, 2, 1, 12), (3, 1, 1, 4)])
+def test_maxpool_parity(F, k, st, pad, bits):
+    rng = np.random.default_rng(k + st + pad + bits)
+    N, H, C = 2, 15, 24
+    x = rand_codes(rng, (N, H, H, C), bits, 0)
+    f = F.fmt(bits, 0, 3)
+    P = (H + 2 * pad - k) // st + 1
+    y = torch.empty(N * P * P * C * (2 if bits > 8 else 1), dtype=torch.float16, device="cuda")
+    F.fxpq_maxpool(to_f16_planes(x, bits, C), N, H, H, C, f, k, st, pad, y)
+    got = F.codes_to_int(y.cpu().view(N, P, P, -1), f).numpy()
+    assert np.array_equal(got, oracle.maxpool(x, k, st, pad))
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("fa,fb,relu", [((8, 1, 5), (7, 1, 3), True), ((6, 0, 2), (8, 1, 6), False),
+                                        ((16, 1, 10), (8, 0, 4), True)])
+def test_eltwise_parity(F, mode, fa, fb, relu):
+    rng = np.random.default_rng(sum(fa) + sum(fb) + mode)
+    npix, C = 333, 16
+    a = rand_codes(rng, (npix, C), fa[0], fa[1])
+    b = rand_codes(rng, (npix, C), fb[0], fb[1])
+    FA, FB, FY = F.fmt(*fa), F.fmt(*fb), F.fmt(7, 0 if relu else 1, 4)
+    if mode == 0:
+        y = torch.empty(npix * C, dtype=torch.float16, device="cuda")
+    elif mode == 1:
+        y = torch.empty(npix * C, dtype=torch.int64, device="cuda")
+    else:
+        y = torch.empty(npix * C, dtype=torch.float32, device="cuda")
+    s = F.fxpq_eltwise(to_f16_planes(a, fa[0], C), FA, to_f16_planes(b, fb[0], C), FB, npix, C, relu, mode, FY, y)
+    v, ws = oracle.eltwise_add(a, fa[2], b, fb[2], relu)
+    assert s == ws
+    if mode == 0:
+        assert np.array_equal(F.codes_to_int(y.cpu().view(npix, C), FY).numpy(), oracle.requant(v, ws, 7, FY.is_signed, 4))
+    elif mode == 1:
+        assert np.array_equal(y.cpu().numpy().reshape(npix, C), v)
+    else:
+        assert np.array_equal(y.cpu().numpy().reshape(npix, C), oracle.to_f32(v, ws))
+
+
+@pytest.mark.parametrize("bits", [5, 8, 11])
+def test_avgpool_parity(F, bits):
+    rng = np.random.default_rng(bits)
+    N, H, C = 3, 7, 40
+    x = rand_codes(rng, (N, H, H, C), bits, 0)
+    fx, fr, fy = F.fmt(bits, 0, 4), F.fmt(16, 0, 21), F.fmt(8, 0, 5)
+    rc = int(oracle.quantize(np.array([1 / 49], np.float32), 16, 0, 21)[0])
+    y = torch.empty(N * C, dtype=torch.float16, device="cuda")
+    s = F.fxpq_avgpool(to_f16_planes(x, bits, C), N, H, H, C, fx, rc, fr, F.OUT_CODES, fy, y)
+    v, ws = oracle.avgpool_global(x, 4, rc, 21)
+    assert s == ws
+    assert np.array_equal(F.codes_to_int(y.cpu().view(N, C), fy).numpy(), oracle.requant(v, ws, 8, 0, 5))

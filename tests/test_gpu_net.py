@@ -1,0 +1,106 @@
+"""Network parity on the GPU: calibration (formats chosen by the FL search in the forward
+optimizer's order) and the integer-only forward through fxpq_net_forward, against the oracle.
+
+The forward runs on the full batch of each workload (the launch configuration the bench times);
+the oracle recomputes sampled images of that batch one by one."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import net as onet
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def NET():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2203_12091_gb300 import net
+    return net
+
+
+def fmts_equal(gpu_fmts, ora_fmts):
+    for nm, d in ora_fmts.items():
+        if nm == "input":
+            assert gpu_fmts["input"]["a"].tup() == tuple(d), nm
+            continue
+        for key, f in d.items():
+            assert gpu_fmts[nm][key].tup() == tuple(f), (nm, key)
+
+
+def _tiny():
+    L = [
+        {"type": "conv", "name": "c1", "C": 3, "K": 16, "R": 3, "stride": 2, "pad": 1, "relu": True, "src": None},
+        {"type": "maxpool", "name": "p1", "k": 3, "stride": 2, "pad": 1},
+        {"type": "conv", "name": "a", "C": 16, "K": 16, "R": 3, "stride": 1, "pad": 1, "relu": True, "src": "p1"},
+        {"type": "conv", "name": "b", "C": 16, "K": 16, "R": 3, "stride": 1, "pad": 1, "relu": False, "src": "a"},
+        {"type": "eltwise", "name": "e", "a": "b", "b": "p1", "relu": True},
+        {"type": "avgpool", "name": "gap", "src": "e"},
+        {"type": "conv", "name": "fc", "C": 16, "K": 24, "R": 1, "stride": 1, "pad": 0, "relu": False, "src": "gap"},
+    ]
+    plan = {"input": 7, "c1": {"w": 6, "b": 16, "a": 8}, "a": {"w": 5, "b": 16, "a": 6}, "b": {"w": 8, "b": 16, "a": 7},
+            "e": {"a": 5}, "gap": {"a": 8, "r": 16}, "fc": {"w": 16, "b": 16}}
+    return L, plan
+
+
+def test_tiny_residual_net(NET):
+    L, plan = _tiny()
+    rng = np.random.default_rng(1)
+    W = {}
+    for l in L:
+        if l["type"] == "conv":
+            fan = l["C"] * l["R"] ** 2
+            W[l["name"]] = ((rng.standard_normal((l["K"], l["R"], l["R"], l["C"])) * np.sqrt(2 / fan)).astype(np.float32),
+                            (rng.standard_normal(l["K"]) * 0.01).astype(np.float32))
+    imgs = synth.images(6, 2, hw=28)
+    q = NET.build_qnet(L, W, torch.from_numpy(imgs[:4]).cuda(), plan)
+    fm, qp = onet.calibrate(L, W, imgs[:4], plan)
+    fmts_equal(q.fmts, fm)
+    logits, s = q.forward(torch.from_numpy(imgs).cuda())
+    want, ws = onet.forward(L, fm, qp, imgs)
+    assert s == ws and np.array_equal(logits.cpu().numpy(), want)
+    # per-layer codes of the op-by-op path agree too
+    env = q.trace(torch.from_numpy(imgs).cuda())
+    oenv = onet.forward_trace(L, fm, qp, imgs)
+    from paper_2203_12091_gb300 import fxpq as F
+    for l in L[:-1]:
+        t, f = env[l["name"]]
+        H, _, Cp = q.shapes[l["name"]]
+        got = F.codes_to_int(t.cpu().view(6, H, H, -1), f).numpy()
+        assert np.array_equal(got[..., : oenv[l["name"]][0].shape[-1]], oenv[l["name"]][0]), l["name"]
+
+
+def _workload(NET, arch, batch, seed, plan_seed=None, calib=8, sample=(0, -1)):
+    L = synth.ARCHS[arch]()
+    W = synth.weights(arch, seed)
+    plan = synth.bit_plan(arch, seed if plan_seed is None else plan_seed)
+    imgs = synth.images(batch, seed)
+    dimgs = torch.from_numpy(imgs).cuda()
+    q = NET.build_qnet(L, W, dimgs[:calib], plan)
+    fm, qp = onet.calibrate(L, W, imgs[:calib], plan)
+    fmts_equal(q.fmts, fm)
+    logits, s = q.forward(dimgs)
+    torch.cuda.synchronize()
+    got = logits.cpu().numpy()
+    idx = [i % batch for i in sample]
+    want, ws = onet.forward(L, fm, qp, imgs[idx])
+    assert s == ws
+    assert np.array_equal(got[idx], want)
+    from paper_2203_12091_gb300 import fxpq as F
+    assert F.fxpq_get_device_status() == 0
+    return got
+
+
+def test_alexnet_batch256(NET):
+    _workload(NET, "alexnet", 256, 5)
+
+
+def test_resnet18_batch128(NET):
+    _workload(NET, "resnet18", 128, 6)
+
+
+@pytest.mark.parametrize("plan_seed", [7, 38])
+def test_vgg16_batch64_plans(NET, plan_seed):
+    _workload(NET, "vgg16", 64, 7, plan_seed=plan_seed, sample=(0,))

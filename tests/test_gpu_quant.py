@@ -1,0 +1,158 @@
+"""GPU parity of the quantizer and the FL search against the CPU oracle (bit-exact).
+
+Integer outputs (codes, chosen FL) must be identical; the L2 scores are the exact sums rounded
+once on both sides, so they are compared for equality (the stated 1e-5 relative tolerance is
+checked as well, as the contract)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+RTOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def F():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2203_12091_gb300 import fxpq
+    return fxpq
+
+
+def _adv(seed, n):
+    base = synth.normal(n, seed)
+    rng = np.random.default_rng(seed)
+    base = base * (np.float32(2.0) ** rng.integers(-12, 8, size=n).astype(np.float32))
+    extra = np.array([0.0, -0.0, 0.5, -0.5, 1.5, 2.5, 127.5, -128.5, 255.5, 1e-40, -3e-39, 2.0 ** -30, 6.0e7,
+                      -6.0e7, 0.75, 3.75, 1 - 2 ** -24, 2 ** 20 + 0.5, 1.9999999, -1.9999999, 2 ** -126,
+                      2.0 ** 30, -(2.0 ** 30), 65535.5, 0.1875, 0.0625], np.float32)
+    return np.concatenate([extra, base]).astype(np.float32)
+
+
+DT = {"I8": (0, np.int8), "U8": (1, np.uint8), "I16": (2, np.int16), "U16": (3, np.uint16), "I32": (4, np.int32)}
+
+
+@pytest.mark.parametrize("n", [0, 1, 3, 4, 1000, 4097, 1 << 20])
+@pytest.mark.parametrize("k,S,fl,dt", [(8, 1, 5, "I8"), (8, 0, 3, "U8"), (4, 1, -2, "I8"), (16, 1, 12, "I16"),
+                                       (12, 0, 20, "U16"), (16, 1, 40, "I32"), (2, 1, -32, "I8")])
+def test_quantize_parity(F, n, k, S, fl, dt):
+    x = _adv(n + k, max(n, 1))[:n]
+    code, npdt = DT[dt]
+    xd = torch.from_numpy(x).cuda()
+    out = torch.empty(max(n, 1), dtype=getattr(torch, np.dtype(npdt).name), device="cuda")
+    F.fxpq_quantize(xd, F.fmt(k, S, fl), code, out)
+    torch.cuda.synchronize()
+    want = oracle.quantize(x, k, S, fl)
+    assert np.array_equal(out.cpu().numpy()[:n].astype(np.int64), want)
+
+
+def test_quantize_unaligned_and_nonfinite(F):
+    x = _adv(5, 999)
+    xd = torch.from_numpy(x).cuda()
+    out = torch.empty(998, dtype=torch.int8, device="cuda")
+    F.fxpq_quantize(xd[1:], F.fmt(8, 1, 6), F.DT_I8, out)  # 4-byte aligned only: scalar path
+    assert np.array_equal(out.cpu().numpy().astype(np.int64), oracle.quantize(x[1:], 8, 1, 6))
+    assert F.fxpq_get_device_status() == 0
+    bad = torch.tensor([1.0, float("nan"), float("inf"), 2.0], device="cuda")
+    o2 = torch.empty(4, dtype=torch.int8, device="cuda")
+    F.fxpq_quantize(bad, F.fmt(8, 1, 0), F.DT_I8, o2)
+    assert F.fxpq_get_device_status() == 3  # FXPQ_ERR_NONFINITE latched
+    assert F.fxpq_get_device_status() == 0  # and cleared
+    assert o2.cpu().tolist() == [1, 0, 0, 2]
+
+
+@pytest.mark.parametrize("k", [4, 8, 12, 16])
+@pytest.mark.parametrize("C,Cp", [(3, 8), (27, 32), (64, 64)])
+def test_quantize_rows_and_images(F, k, C, Cp):
+    rows = 37
+    x = synth.normal(rows * C, 7 + k)
+    out = torch.empty(rows, Cp * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
+    F.fxpq_quantize_rows(torch.from_numpy(x).cuda(), rows, C, F.fmt(k, 1, k - 3), Cp, out)
+    got = F.codes_to_int(out.cpu(), F.fmt(k, 1, k - 3)).numpy()
+    want = oracle.quantize(x, k, 1, k - 3).reshape(rows, C)
+    assert np.array_equal(got[:, :C], want) and np.all(got[:, C:] == 0)
+    imgs = synth.images(2, 9, hw=13)
+    out = torch.empty(2 * 13 * 13 * 8 * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
+    F.fxpq_quantize_images(torch.from_numpy(imgs).cuda(), F.fmt(k, 1, k - 4), 8, out)
+    got = F.codes_to_int(out.cpu().view(2, 13, 13, -1), F.fmt(k, 1, k - 4)).numpy()
+    want = oracle.quantize(np.transpose(imgs, (0, 2, 3, 1)), k, 1, k - 4).reshape(2, 13, 13, 3)
+    assert np.array_equal(got[..., :3], want) and np.all(got[..., 3:] == 0)
+
+
+def _check_search(F, x, S, klo, khi, fllo, flhi):
+    err, best, st = F.fl_search(torch.from_numpy(x).cuda(), S, klo, khi, fllo, flhi)
+    torch.cuda.synchronize()
+    oerr, obest, oS, ost = oracle.fl_search(x, S, klo, khi, fllo, flhi)
+    g = err.cpu().numpy()
+    assert np.array_equal(best.cpu().numpy(), obest)
+    np.testing.assert_allclose(g, oerr, rtol=RTOL, atol=0)
+    assert np.array_equal(g, oerr)  # exact sums rounded once on both sides
+    s = F.stats_from_device(st)
+    assert s.is_signed == oS and s.n == x.size and s.nonfinite == 0
+    if x.size:
+        assert s.min == ost["min"] and s.max == ost["max"]
+        assert s.sum == ost["sum"] and s.sumsq == ost["sumsq"]
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_fl_search_adversarial_full_grid(F, seed):
+    x = _adv(seed, 3000)
+    _check_search(F, x, -1, 2, 16, -8, 23)
+    _check_search(F, np.abs(x), -1, 2, 16, -8, 23)
+    _check_search(F, x, 0, 2, 16, -8, 23)
+
+
+@pytest.mark.parametrize("dist", ["normal", "laplace", "relu_normal"])
+@pytest.mark.parametrize("n", [0, 1, 5, 1023, 70001])
+def test_fl_search_small_sizes_and_ranges(F, dist, n):
+    x = synth.sweep_tensor(dist, n, 11 + n)
+    _check_search(F, x, -1, 2, 16, -8, 23)
+    _check_search(F, x, 1, 8, 8, 0, 15)
+    _check_search(F, x, -1, 3, 9, -32, -1)
+    _check_search(F, x, -1, 13, 16, 9, 40)
+
+
+def test_fl_search_ties_pick_smallest_fl(F):
+    x = np.array([0.75], np.float32)
+    err, best, _ = F.fl_search(torch.from_numpy(x).cuda(), 0, 2, 2, 0, 1)
+    assert err.cpu().tolist() == [[0.0625, 0.0625]] and best.item() == 0
+    grid = (np.arange(-128, 128) / 32.0).astype(np.float32)  # exact on FL >= 5 at 8 bits
+    err, best, _ = F.fl_search(torch.from_numpy(grid).cuda(), 1, 8, 8, 0, 10)
+    assert best.item() == 5 and err.cpu().numpy()[0, 5] == 0.0
+
+
+def test_fl_search_nonfinite_latches_status(F):
+    x = torch.tensor([1.0, float("inf"), -2.0], device="cuda")
+    err, best, st = F.fl_search(x, -1, 8, 8, 0, 3)
+    assert F.fxpq_get_device_status() == 3
+    assert F.stats_from_device(st).nonfinite == 1
+
+
+@pytest.mark.parametrize("dist,seed", [("normal", 2), ("laplace", 3), ("relu_normal", 4)])
+def test_fl_search_config_1m_full_sweep(F, dist, seed):
+    x = synth.sweep_tensor(dist, 1 << 20, seed)
+    _check_search(F, x, -1, 2, 16, -8, 23)
+
+
+@pytest.mark.parametrize("n", [1 << 24, 1 << 26])
+def test_fl_search_config_large_sampled(F, n):
+    """Full-size sweep: sampled cells recomputed by the oracle one by one; argmin checked against
+    the GPU's own scores; stats exact."""
+    x = synth.sweep_tensor("normal", n, 2)
+    err, best, st = F.fl_search(torch.from_numpy(x).cuda(), -1, 2, 16, -8, 23)
+    g = err.cpu().numpy()
+    b = best.cpu().numpy()
+    s = F.stats_from_device(st)
+    assert s.is_signed == 1
+    for ki, k in enumerate(range(2, 17)):
+        assert b[ki] == -8 + int(np.argmin(g[ki]))
+    rng = np.random.default_rng(n)
+    cells = [(8, int(b[6])), (2, int(b[0])), (16, int(b[14])), (5, 11)] + [(int(rng.integers(2, 17)), int(rng.integers(-8, 24)))]
+    for k, fl in cells:
+        assert g[k - 2, fl + 8] == oracle.l2_error(x, k, 1, fl)
+    assert s.sumsq == oracle.exact_sum(x.astype(np.float64) ** 2)
+    assert s.min == float(x.min()) and s.max == float(x.max())
