@@ -53,7 +53,7 @@ def test_quantize_parity(F, n, k, S, fl, dt):
 def test_quantize_unaligned_and_nonfinite(F):
     x = _adv(5, 999)
     xd = torch.from_numpy(x).cuda()
-    out = torch.empty(998, dtype=torch.int8, device="cuda")
+    out = torch.empty(x.size - 1, dtype=torch.int8, device="cuda")
     F.fxpq_quantize(xd[1:], F.fmt(8, 1, 6), F.DT_I8, out)  # 4-byte aligned only: scalar path
     assert np.array_equal(out.cpu().numpy().astype(np.int64), oracle.quantize(x[1:], 8, 1, 6))
     assert F.fxpq_get_device_status() == 0
