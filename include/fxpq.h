@@ -122,6 +122,23 @@ FXPQ_API fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_sign
                            int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
                            fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream);
 
+/* fxpq_fl_search for callers that cannot allocate device memory -- for instance a plug-in whose
+ * host application owns the whole device memory pool, or a latency-critical loop that must never
+ * enter the allocator (cudaMalloc may synchronise the device).  The paper has no counterpart: this
+ * is a deployment variant of fxpq_fl_search with the same arguments, results and limits, minus
+ * the workspace.  It allocates nothing.  Its scratch is a file-scope device array of about
+ * 150 KiB inside libfxpq.so that every GPU which loads the library holds until the process exits.
+ *   - Limits: n <= 2^31 elements and at most 15 x 32 candidates (k in [2,16], fl_hi-fl_lo <= 31);
+ *     larger requests return FXPQ_ERR_INVALID_ARG before any launch.
+ *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
+ *     that device current; make that first call before any stream capture begins.
+ *   - All calls share the one array and each call clears it before use.  Calls that overlap on the
+ *     GPU (concurrent streams, or several host threads) race on it and give wrong results:
+ *     serialise them, or use fxpq_fl_search with a workspace per stream. */
+FXPQ_API fxpq_status fxpq_fl_search_noalloc(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo,
+                                            int32_t k_hi, int32_t fl_lo, int32_t fl_hi, double* d_err,
+                                            int32_t* d_best, fxpq_stats* d_stats, void* stream);
+
 /* Initial quantization parameters (Sec. IV-A.3, Eq. initial_quantization_parameters), a host
  * helper on statistics already copied to the host: psi from the range, beta_hat = -log2(psi),
  * beta = floor (strategy 0, conservative) / round half-even (1, neutral) / ceil (2, aggressive).

@@ -57,6 +57,7 @@ _SIGS = {
     "fxpq_quantize_images": (I32, [VP, I32, I32, I32, I32, Fmt, I32, VP, VP]),
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),
+    "fxpq_fl_search_noalloc": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),
     "fxpq_conv_workspace": (SZ, [ctypes.POINTER(ConvDesc)]),
     "fxpq_conv_fwd": (I32, [ctypes.POINTER(ConvDesc), VP, VP, VP, VP, ctypes.POINTER(I32), VP, SZ, VP]),

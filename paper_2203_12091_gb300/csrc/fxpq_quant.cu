@@ -17,6 +17,8 @@
 //   rounds once to nearest-even double -- the same value as the exact definition.
 #include <math.h>
 
+#include <mutex>
+
 #include "fxpq_common.cuh"
 
 namespace fxpq {
@@ -776,4 +778,50 @@ extern "C" fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int
     h_out->is_signed = S;
     h_out->fl = (int32_t)beta;
     return FXPQ_OK;
+}
+
+// ------------------------------------------------------------------------------------------
+// FL search without a caller workspace.
+//
+// Some callers cannot allocate device memory: a plug-in hosted by an application that owns the
+// whole device memory pool, or a latency-critical loop that must never enter the allocator
+// (cudaMalloc may synchronise the device).  For them the FL search's scratch (the exact integer
+// bins and per-candidate cells, a fixed size independent of n) lives in this file-scope array,
+// which every GPU that loads the library keeps until the process exits.
+// ------------------------------------------------------------------------------------------
+namespace {
+constexpr size_t kFlSearchStaticBytes = (sizeof(FsGlobal) + 255) / 256 * 256;
+static __device__ __align__(256) unsigned char g_fl_search_scratch[kFlSearchStaticBytes];
+
+std::mutex g_fl_static_mu;
+void* g_fl_static_addr[64] = {nullptr};
+
+// Device address of g_fl_search_scratch on the current device, looked up once per device.
+fxpq_status fl_search_scratch_ptr(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FXPQ_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_fl_static_mu);
+    if (!g_fl_static_addr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_fl_search_scratch) != cudaSuccess || !p) return FXPQ_ERR_CUDA;
+        g_fl_static_addr[dev] = p;
+    }
+    *out = g_fl_static_addr[dev];
+    return FXPQ_OK;
+}
+}  // namespace
+
+extern "C" fxpq_status fxpq_fl_search_noalloc(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo,
+                                              int32_t k_hi, int32_t fl_lo, int32_t fl_hi, double* d_err,
+                                              int32_t* d_best, fxpq_stats* d_stats, void* stream) {
+    if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;  // the largest tensor the bins can hold
+    if (k_lo < 2 || k_hi > 16 || k_lo > k_hi || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL)
+        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 15 x 32
+    if (fxpq_fl_search_workspace(n) > kFlSearchStaticBytes) return FXPQ_ERR_WORKSPACE;
+    void* scratch = nullptr;
+    fxpq_status st = fl_search_scratch_ptr(&scratch);
+    if (st != FXPQ_OK) return st;
+    // fxpq_fl_search clears the bins it accumulates into before its first kernel.
+    return fxpq_fl_search(d_x, n, is_signed, k_lo, k_hi, fl_lo, fl_hi, d_err, d_best, d_stats, scratch,
+                          kFlSearchStaticBytes, stream);
 }
