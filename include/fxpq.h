@@ -21,9 +21,9 @@
  * Code storage ("fp16 code tensors").  Inside the network path every code tensor is stored as
  * fp16 values that are exact integers.  A format with k <= 8 bits uses one plane (|code| <= 255).
  * A format with 9..16 bits uses two planes, hi and lo, with code = 256*hi + lo, lo in [0, 255]
- * and hi = floor(code / 256); the planes are concatenated along the innermost (channel) axis:
- * [hi_0 .. hi_{C-1}, lo_0 .. lo_{C-1}].  Channel counts are padded to a multiple of 8 with
- * zero codes.
+ * and hi = floor(code / 256).  Planes are stored plane-major: the whole hi tensor, then the whole
+ * lo tensor of the same shape (for an NHWC tensor [N,H,W,Cp] the lo plane starts N*H*W*Cp
+ * elements after the hi plane).  Channel counts are padded to a multiple of 8 with zero codes.
  */
 #ifndef FXPQ_H
 #define FXPQ_H
@@ -84,22 +84,22 @@ typedef struct {
 /*   code_i = clip(round_half_even(x_i * 2^fl), Qmin, Qmax),                                */
 /*   Qmin = -S * 2^(k-S), Qmax = 2^(k-S) - 1.                                                */
 /* d_x: n fp32 values.  d_codes: n codes in storage `dtype` (I8/U8/I16/U16/I32 must be wide   */
-/* enough and of the right signedness; F16 writes the limb planes of a [n/c, c] tensor with   */
-/* c = n, i.e. plane hi at [0, n) and lo at [n, 2n) for k > 8).  n may be 0.                 */
+/* enough and of the right signedness; F16 writes an fp16 code tensor: plane hi at [0, n) and */
+/* plane lo at [n, 2n) when k > 8).  n may be 0.                                             */
 /* NaN/Inf inputs latch FXPQ_ERR_NONFINITE and produce code 0.                               */
 /* ---------------------------------------------------------------------------------------- */
 FXPQ_API fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int32_t dtype, void* d_codes,
                           void* stream);
 
 /* Quantize a row-major [rows, C] fp32 tensor (e.g. KRSC weights with C innermost) into an fp16
- * code tensor [rows, Cp * planes] (planes per f.bits, see the file header); channels C..Cp-1 are
- * zero codes.  Cp is a multiple of 8 and >= C. */
+ * code tensor: planes (per f.bits, see the file header) of [rows, Cp]; channels C..Cp-1 are zero
+ * codes.  Cp is a multiple of 8 and >= C. */
 FXPQ_API fxpq_status fxpq_quantize_rows(const float* d_x, int64_t rows, int32_t C, fxpq_fmt f, int32_t Cp, void* d_y,
                                void* stream);
 
 /* Quantize + transpose + pack fp32 images NCHW -> NHWC fp16 code tensor with the channel count
  * padded to c_pad (a multiple of 8, >= C) with zero codes: the FxP-QLayer inserted at the input
- * of the network (Sec. IV-A.2).  d_y holds N*H*W*c_pad*planes fp16 values. */
+ * of the network (Sec. IV-A.2).  d_y holds planes x [N, H, W, c_pad] fp16 values. */
 FXPQ_API fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, int32_t C, int32_t H, int32_t W,
                                  fxpq_fmt f, int32_t c_pad, void* d_y, void* stream);
 
@@ -153,12 +153,13 @@ FXPQ_API fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32
 /*   B << delta, delta < 0 shifts acc left by -delta first (no bit is dropped);               */
 /*   ReLU = max(., 0) if relu;                                                               */
 /*   out_mode CODES : FxP-QLayer -> round_half_even(v * 2^(fl_y - s)), clip to fmt_y,         */
-/*                    written as an fp16 code tensor NHWC with Kp = K padded to 8;            */
+/*                    written as an fp16 code tensor NHWC [N,P,Q,K] (K a multiple of 8);      */
 /*   out_mode ACC64 : no QLayer (last layer): int64 v, NHWC [N,P,Q,K]; its scale exponent is   */
 /*                    returned in *h_out_scale;                                               */
 /*   out_mode F32   : fp32 nearest-even image of v * 2^-s (for calibrating fmt_y.fl).          */
 /* X: fp16 code tensor NHWC [N,H,W,Cp] (planes per fmt_x.bits); W: fp16 code tensor KRSC       */
-/* [K,R,S,Cp] (planes per fmt_w.bits); d_bias: int32 codes [K] or NULL.                       */
+/* [K,R,S,Cp] (planes per fmt_w.bits); d_bias: int32 codes [K] or NULL.  X, W, Y 16-byte      */
+/* aligned.                                                                                  */
 /* An FC layer is a convolution whose window covers the whole input map (R = H, S = W).      */
 /* Returns FXPQ_ERR_RANGE if |acc| could exceed 2^62 after alignment.                         */
 /* ---------------------------------------------------------------------------------------- */

@@ -59,4 +59,23 @@ __device__ __forceinline__ void split_limbs(int code, __half& hi, __half& lo) {
     lo = __int2half_rn(l);
 }
 
+// fp16 code tensors are plane-major: a k > 8 tensor stores its hi plane (a whole tensor) and then
+// its lo plane, plane_stride elements later.  idx indexes one plane.
+__device__ __forceinline__ int code_get(const __half* __restrict__ t, long long idx, int planes, long long plane_stride) {
+    if (planes == 1) return __half2int_rn(t[idx]);
+    return (__half2int_rn(t[idx]) << 8) + __half2int_rn(t[plane_stride + idx]);
+}
+
+__device__ __forceinline__ void code_put(__half* __restrict__ t, long long idx, int planes, long long plane_stride,
+                                         int code) {
+    if (planes == 1) {
+        t[idx] = __int2half_rn(code);
+    } else {
+        __half h, l;
+        split_limbs(code, h, l);
+        t[idx] = h;
+        t[plane_stride + idx] = l;
+    }
+}
+
 }  // namespace fxpq

@@ -4,6 +4,8 @@
 // This translation unit holds the CUDA-core implicit-GEMM kernel (exact int32 / int64 MACs),
 // used for every shape, and the host entry points.
 #include <math.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include "fxpq_common.cuh"
 #include "fxpq_conv.cuh"
@@ -11,10 +13,9 @@
 namespace fxpq {
 namespace {
 
-__device__ __forceinline__ int load_code(const __half* __restrict__ t, long long row, int Cp, int planes, int c) {
-    const __half* p = t + row * (long long)Cp * planes;
-    if (planes == 1) return __half2int_rn(p[c]);
-    return (__half2int_rn(p[c]) << 8) + __half2int_rn(p[Cp + c]);
+__device__ __forceinline__ int load_code(const __half* __restrict__ t, long long row, int Cp, int planes, int c,
+                                         long long plane_stride) {
+    return code_get(t, row * Cp + c, planes, plane_stride);
 }
 
 constexpr int TM = 64, TN = 64, TK = 16, NT = 256;
@@ -64,11 +65,12 @@ __global__ void __launch_bounds__(NT) conv_simt_kernel(ConvArgs a) {
                     int h = pix_p[i] * a.stride + r - a.pad;
                     int w = pix_q[i] * a.stride + s - a.pad;
                     if (pix_ok[i] && c < a.Cp && h >= 0 && h < a.H && w >= 0 && w < a.W)
-                        code = load_code(a.x, (pix_n[i] * a.H + h) * a.W + w, a.Cp, a.px, c);
+                        code = load_code(a.x, (pix_n[i] * a.H + h) * a.W + w, a.Cp, a.px, c, a.x_ps);
                     As[cc][row] = code;
                     int k = n0 + row;
                     int wc = 0;
-                    if (k < a.K && c < a.Cp) wc = load_code(a.w, ((long long)k * a.R + r) * a.S + s, a.Cp, a.pw, c);
+                    if (k < a.K && c < a.Cp)
+                        wc = load_code(a.w, ((long long)k * a.R + r) * a.S + s, a.Cp, a.pw, c, a.w_ps);
                     Bs[cc][row] = wc;
                 }
                 __syncthreads();
@@ -126,6 +128,9 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
     a.y = y;
     a.N = d.N, a.H = d.H, a.W = d.W, a.Cp = d.Cp, a.K = d.K, a.R = d.R, a.S = d.S;
     a.stride = d.stride, a.pad = d.pad, a.P = P, a.Q = Q;
+    a.M = (long long)d.N * P * Q;
+    a.x_ps = (long long)d.N * d.H * d.W * d.Cp;
+    a.w_ps = (long long)d.K * d.R * d.S * d.Cp;
     a.px = planes_of(d.fmt_x);
     a.pw = planes_of(d.fmt_w);
     a.relu = d.relu;
@@ -164,9 +169,20 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
     return FXPQ_OK;
 }
 
-fxpq_status launch_conv(const ConvArgs& a, bool need64, cudaStream_t st) {
+// FXPQ_CONV_PATH=simt selects the CUDA-core kernel for every shape (tests use it to cover both).
+static bool tc_path_enabled() {
+    const char* e = getenv("FXPQ_CONV_PATH");
+    return !(e && strcmp(e, "simt") == 0);
+}
+
+fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st) {
     const long long M = (long long)a.N * a.P * a.Q;
     if (M == 0) return FXPQ_OK;
+    if (tc_path_enabled()) {
+        bool launched = false;
+        fxpq_status s = launch_conv_tc(a, d, st, launched);
+        if (s != FXPQ_OK || launched) return s;
+    }
     dim3 grid((unsigned)((M + TM - 1) / TM), (unsigned)((a.K + TN - 1) / TN));
     if (need64)
         conv_simt_kernel<long long><<<grid, NT, 0, st>>>(a);
@@ -194,7 +210,7 @@ extern "C" fxpq_status fxpq_conv_fwd(const fxpq_conv_desc* h_desc, const void* d
     bool need64 = false;
     fxpq_status st = plan_conv(*h_desc, d_x, d_w, d_bias, d_y, a, h_out_scale, need64);
     if (st != FXPQ_OK) return st;
-    return launch_conv(a, need64, as_stream(stream));
+    return launch_conv(a, *h_desc, need64, as_stream(stream));
 }
 
 extern "C" fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_w, fxpq_fmt fmt_w,

@@ -6,11 +6,13 @@
 namespace fxpq {
 
 struct ConvArgs {
-    const __half* x;   // NHWC fp16 code tensor [N, H, W, Cp * px]
-    const __half* w;   // KRSC fp16 code tensor [K, R, S, Cp * pw]
+    const __half* x;   // NHWC fp16 code tensor, px planes of [N, H, W, Cp]
+    const __half* w;   // KRSC fp16 code tensor, pw planes of [K, R, S, Cp]
     const int32_t* bias;
-    void* y;           // CODES: fp16 [M, K * py]; ACC64: int64 [M, K]; F32: float [M, K]
+    void* y;           // CODES: fp16, py planes of [M, K]; ACC64: int64 [M, K]; F32: float [M, K]
     int N, H, W, Cp, K, R, S, stride, pad, P, Q;
+    long long M;       // N * P * Q output rows
+    long long x_ps, w_ps;  // plane strides (elements) of x and w
     int px, pw, py;
     int relu, out_mode, has_bias;
     int delta;         // bias alignment: s_acc - fl_b
@@ -43,15 +45,7 @@ __device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long lo
                 q = v << l;
         }
         q = q < a.lo ? a.lo : (q > a.hi ? a.hi : q);
-        __half* y = static_cast<__half*>(a.y);
-        if (a.py == 1) {
-            y[m * a.K + k] = __int2half_rn((int)q);
-        } else {
-            __half h, l;
-            split_limbs((int)q, h, l);
-            y[m * 2LL * a.K + k] = h;
-            y[m * 2LL * a.K + a.K + k] = l;
-        }
+        code_put(static_cast<__half*>(a.y), m * a.K + k, a.py, a.M * a.K, (int)q);
     } else if (a.out_mode == FXPQ_OUT_ACC64) {
         static_cast<long long*>(a.y)[m * a.K + k] = v;
     } else {
@@ -61,6 +55,8 @@ __device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long lo
 
 fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, const int32_t* bias, void* y,
                       ConvArgs& a, int32_t* out_scale, bool& need64);
-fxpq_status launch_conv(const ConvArgs& a, bool need64, cudaStream_t st);
+fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st);
+// Tensor-core path; sets launched = false when the shape needs the CUDA-core kernel instead.
+fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched);
 
 }  // namespace fxpq

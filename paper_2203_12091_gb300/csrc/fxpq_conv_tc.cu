@@ -1,0 +1,451 @@
+// fxpq_conv_tc.cu -- the C-Block contraction (Sec. IV-B) on the 5th-generation tensor cores.
+//
+// Implicit GEMM: rows = output pixels (N*P*Q), columns = output channels K, reduction over the
+// flattened (r, s, c) taps of one code plane.  Operands are fp16 values that are exact integer
+// codes (|code| <= 255 per limb), multiplied by tcgen05.mma .kind::f16 into fp32 TMEM
+// accumulators.  fp32 accumulation is exact while every partial sum stays below 2^24, so the host
+// splits the reduction into groups ("chunks") whose worst-case magnitude max|a| * max|w| * K_chunk
+// is below 2^24; after each group the epilogue warps drain the accumulator, convert it to an
+// integer (exact) and add it, shifted by the limb weight (0, 8 or 16 bits), into integer running
+// sums.  The same grouping carries the two-limb split of 9..16-bit codes
+// (v = 256 * v_hi + v_lo): one pass per (A limb, W limb) pair.
+//
+// CTA (one per SM, persistent over tiles): 9 warps.
+//   warps 0-3  producers: cp.async gather of the A tile (128 pixels x 64 taps, with zero fill for
+//              padding and ragged edges) and of the B tile (BN channels x 64 taps) into 128-byte
+//              swizzled K-major shared-memory stages.
+//   warp  4-7  epilogue: drain TMEM (tcgen05.ld), integer running sums, final bias / ReLU /
+//              FxP-QLayer (shared with the CUDA-core kernel).
+//   warp  8    TMEM allocation and the single MMA-issuing thread.
+// Every wait is bounded: on expiry the kernel latches FXPQ_ERR_TIMEOUT, stops issuing work,
+// drains its own copies and MMAs, frees TMEM and returns.
+#include <mutex>
+
+#include "fxpq_common.cuh"
+#include "fxpq_conv.cuh"
+
+namespace fxpq {
+
+namespace {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
+constexpr int TC_STAGES = 4;
+constexpr int TC_LAG = 2;  // producer arrives on a stage two k-blocks after issuing it
+constexpr int TC_THREADS = 288;
+constexpr int TC_MAX_GROUPS = 64;
+constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
+
+struct TcGroup {
+    int kb0, kb1;          // k-block range within a plane
+    int a_plane, w_plane;  // limb planes (0 = hi or the only plane, 1 = lo)
+    int shift;             // weight of this pass: 0, 8 or 16 bits
+};
+
+struct TcParams {
+    ConvArgs a;
+    int RSC;       // R * S * Cp: reduction length of one plane
+    int tiles_m, tiles_n, n_tiles;
+    int n_groups;
+    int cp64;      // Cp % 64 == 0: a k-block never straddles a tap
+    int* status;
+    TcGroup g[TC_MAX_GROUPS];
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
+// timeout status, sets the CTA abort flag) if it gave up or another role already aborted.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (clock64() - t0 > TC_WAIT_CYCLES) {
+            *abort = 1;
+            latch_status(status, FXPQ_ERR_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);          // start address
+    d |= (uint64_t)1u << 16;                          // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024u >> 4) << 32;                // stride byte offset: 8 rows x 128 B
+    d |= (uint64_t)1u << 46;                          // descriptor version
+    d |= (uint64_t)2u << 61;                          // SWIZZLE_128B
+    return d;
+}
+
+// Instruction descriptor, kind::f16: fp16 A and B (K-major), fp32 accumulator, M x N.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N) {
+    return (1u << 4)                        // D format F32
+           | (0u << 7) | (0u << 10)         // A, B format F16
+           | ((uint32_t)(N >> 3) << 17)     // N / 8
+           | ((uint32_t)(M >> 4) << 24);    // M / 16
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// ------------------------------------------------------------------ kernel
+template <int BN, typename ACC>
+__global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+    constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
+    constexpr int B_BYTES = BN * TC_BK * 2;
+    constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    unsigned char* sA = base;
+    unsigned char* sB = base + TC_STAGES * A_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + TC_STAGES * B_BYTES);
+    // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
+    volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
+    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + TC_STAGES);
+    const uint32_t accfull0 = smem_u32(bars + 2 * TC_STAGES), accempty0 = smem_u32(bars + 2 * TC_STAGES + 2);
+    const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const ConvArgs& a = P.a;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < TC_STAGES; ++s) {
+            mbar_init(full0 + 8 * s, 128);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(accfull0 + 8 * b, 1);
+            mbar_init(accempty0 + 8 * b, 128);
+        }
+        mbar_init(done_bar, 1);
+        *abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 8) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(2 * BN));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp < 4) {
+        // ============================================================ producers
+        const int row = threadIdx.x;  // 0..127: one A row and (row < BN) one B row per stage
+        const __half* xb = a.x;
+        const __half* wb = a.w;
+        uint32_t it = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            const int tm = t / P.tiles_n, tn = t % P.tiles_n;
+            const long long m = (long long)tm * TC_BM + row;
+            const bool mvalid = m < a.M;
+            const long long mm = mvalid ? m : 0;
+            const int n_img = (int)(mm / ((long long)a.P * a.Q));
+            const int pq = (int)(mm - (long long)n_img * a.P * a.Q);
+            const int p0 = (pq / a.Q) * a.stride - a.pad, q0 = (pq % a.Q) * a.stride - a.pad;
+            const int kout = tn * BN + row;
+            const bool brow = row < BN;
+            const bool kvalid = brow && kout < a.K;
+            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+                const TcGroup g = P.g[gi];
+                const __half* xp = xb + (long long)g.a_plane * a.x_ps;
+                const __half* wp = wb + (long long)g.w_plane * a.w_ps + (long long)(kvalid ? kout : 0) * P.RSC;
+                for (int kb = g.kb0; kb < g.kb1; ++kb) {
+                    const int stage = it % TC_STAGES;
+                    const uint32_t ph = (it / TC_STAGES) & 1;
+                    if (!wait_bounded(empty0 + 8 * stage, ph ^ 1, abort, P.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dA = smem_u32(sA + stage * A_BYTES) + row * 128;
+                    const uint32_t dB = smem_u32(sB + stage * B_BYTES) + row * 128;
+                    const int f0 = kb * TC_BK;
+                    int tap = 0, c0 = 0;
+                    if (P.cp64) {
+                        tap = f0 / a.Cp;
+                        c0 = f0 - tap * a.Cp;
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const int f = f0 + 8 * c;
+                        int tp = tap, cc = c0 + 8 * c;
+                        if (!P.cp64) {
+                            tp = f / a.Cp;
+                            cc = f - tp * a.Cp;
+                        }
+                        const int r = tp / a.S, s = tp - (tp / a.S) * a.S;
+                        const int h = p0 + r, w = q0 + s;
+                        const bool v = mvalid && f < P.RSC && h >= 0 && h < a.H && w >= 0 && w < a.W;
+                        const __half* src = v ? xp + (((long long)n_img * a.H + h) * a.W + w) * a.Cp + cc : xb;
+                        const uint32_t sw = (uint32_t)((c ^ (row & 7)) << 4);
+                        cp_async16(dA + sw, src, v ? 16u : 0u);
+                        if (brow) {
+                            const bool vb = kvalid && f < P.RSC;
+                            cp_async16(dB + sw, vb ? (const void*)(wp + f) : (const void*)wb, vb ? 16u : 0u);
+                        }
+                    }
+                    cp_async_commit();
+                    if (it >= TC_LAG) {
+                        cp_async_wait<TC_LAG>();
+                        fence_proxy_async();
+                        mbar_arrive(full0 + 8 * ((it - TC_LAG) % TC_STAGES));
+                    }
+                    ++it;
+                }
+            }
+        }
+        cp_async_wait<0>();
+        fence_proxy_async();
+        const uint32_t first = it >= TC_LAG ? it - TC_LAG : 0;
+        for (uint32_t j = first; j < it; ++j) mbar_arrive(full0 + 8 * (j % TC_STAGES));
+    } else if (warp < 8) {
+        // ============================================================ epilogue
+        const int quad = warp - 4;  // TMEM lane quadrant of this warp
+        const int row = quad * 32 + lane;
+        uint32_t gcount = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            const int tm = t / P.tiles_n, tn = t % P.tiles_n;
+            ACC run[BN];
+#pragma unroll
+            for (int j = 0; j < BN; ++j) run[j] = 0;
+            for (int gi = 0; gi < P.n_groups; ++gi) {
+                const int shift = P.g[gi].shift;
+                const uint32_t buf = gcount & 1;
+                if (!wait_bounded(accfull0 + 8 * buf, (gcount >> 1) & 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+#pragma unroll
+                for (int cb = 0; cb < BN / 32; ++cb) {
+                    float v[32];
+                    tmem_ld32(tmem + ((uint32_t)(quad * 32) << 16) + buf * BN + cb * 32, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) run[cb * 32 + j] += ((ACC)__float2int_rn(v[j])) << shift;
+                }
+                tc_fence_before();
+                mbar_arrive(accempty0 + 8 * buf);
+                ++gcount;
+            }
+            if (!ok) break;
+            const long long m = (long long)tm * TC_BM + row;
+            if (m < a.M) {
+#pragma unroll
+                for (int j = 0; j < BN; ++j) {
+                    const int k = tn * BN + j;
+                    if (k < a.K) cblock_epilogue_store(a, m, k, (long long)run[j]);
+                }
+            }
+        }
+    } else if (lane == 0) {
+        // ============================================================ MMA issue (one thread)
+        uint32_t it = 0, gcount = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+                const TcGroup g = P.g[gi];
+                const uint32_t buf = gcount & 1;
+                if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem + buf * BN;
+                for (int kb = g.kb0; kb < g.kb1; ++kb) {
+                    const int stage = it % TC_STAGES;
+                    if (!wait_bounded(full0 + 8 * stage, (it / TC_STAGES) & 1, abort, P.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t aS = smem_u32(sA + stage * A_BYTES), bS = smem_u32(sB + stage * B_BYTES);
+#pragma unroll
+                    for (int kk = 0; kk < TC_BK / 16; ++kk)
+                        tc_mma(d, make_sdesc(aS + kk * 32), make_sdesc(bS + kk * 32), IDESC,
+                               (kb > g.kb0 || kk > 0) ? 1u : 0u);
+                    tc_commit(empty0 + 8 * stage);
+                    ++it;
+                }
+                if (!ok) break;
+                tc_commit(accfull0 + 8 * buf);
+                ++gcount;
+            }
+        }
+        // every MMA issued by this thread has completed once `done` fires
+        tc_commit(done_bar);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 8) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
+    }
+}
+
+int g_num_sms = 0;
+std::mutex g_tc_mu;
+bool g_tc_attr_set[2] = {false, false};
+
+template <int BN>
+constexpr size_t tc_smem_bytes() {
+    return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + 256;
+}
+
+// Largest |limb| of a format's codes: the only plane (k <= 8) or the hi / lo limb (k > 8).
+long long limb_max(const fxpq_fmt& f, int plane) {
+    const long long mx = qmax_of(f), mn = -qmin_of(f);
+    if (f.bits <= 8) return mx > mn ? mx : mn;
+    if (plane == 1) return 255;
+    const long long hmx = mx >> 8, hmn = (mn + 255) >> 8;  // |floor(code / 256)|
+    return hmx > hmn ? hmx : hmn;
+}
+
+}  // namespace
+
+// Builds the group table; returns false if the tensor-core path cannot keep the sums exact.
+bool plan_tc(const ConvArgs& a, const fxpq_conv_desc& d, TcParams& P, bool& acc64) {
+    P.a = a;
+    P.RSC = a.R * a.S * a.Cp;
+    const int n_kb = (P.RSC + TC_BK - 1) / TC_BK;
+    P.cp64 = (a.Cp % TC_BK) == 0;
+    const int pa = planes_of(d.fmt_x), pw = planes_of(d.fmt_w);
+    int ng = 0;
+    bool shifted = false;
+    for (int ia = 0; ia < pa; ++ia)
+        for (int iw = 0; iw < pw; ++iw) {
+            const long long bound = limb_max(d.fmt_x, ia) * limb_max(d.fmt_w, iw);
+            if (bound == 0) continue;
+            const long long kmax = ((1LL << 24) - 1) / bound;  // taps per exact fp32 group
+            const int kb_per = (int)(kmax / TC_BK);
+            if (kb_per < 1) return false;
+            const int shift = 8 * ((pa - 1 - ia) + (pw - 1 - iw));
+            shifted |= shift > 0;
+            for (int kb0 = 0; kb0 < n_kb; kb0 += kb_per) {
+                if (ng >= TC_MAX_GROUPS) return false;
+                P.g[ng++] = TcGroup{kb0, kb0 + kb_per < n_kb ? kb0 + kb_per : n_kb, ia, iw, shift};
+            }
+        }
+    P.n_groups = ng;
+    const double total = ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed) * ldexp(1.0, d.fmt_w.bits - d.fmt_w.is_signed) *
+                         (double)a.R * a.S * a.Cp;
+    acc64 = shifted || total >= ldexp(1.0, 31) - 1.0;
+    P.status = status_ptr();
+    return ng > 0;
+}
+
+fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched) {
+    launched = false;
+    TcParams P;
+    bool acc64 = false;
+    if (!plan_tc(a, d, P, acc64)) return FXPQ_OK;
+    const int BN = acc64 ? 64 : 128;
+    P.tiles_m = (int)((a.M + TC_BM - 1) / TC_BM);
+    P.tiles_n = (a.K + BN - 1) / BN;
+    P.n_tiles = P.tiles_m * P.tiles_n;
+    if (P.n_tiles == 0) {
+        launched = true;
+        return FXPQ_OK;
+    }
+    {
+        std::lock_guard<std::mutex> lk(g_tc_mu);
+        if (g_num_sms == 0) {
+            int dev = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+            if (g_num_sms <= 0) g_num_sms = 1;
+        }
+        if (!g_tc_attr_set[acc64]) {
+            cudaError_t e = acc64 ? cudaFuncSetAttribute(conv_tc_kernel<64, long long>,
+                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<64>())
+                                  : cudaFuncSetAttribute(conv_tc_kernel<128, int>,
+                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<128>());
+            if (e != cudaSuccess) return FXPQ_ERR_CUDA;
+            g_tc_attr_set[acc64] = true;
+        }
+    }
+    const int grid = P.n_tiles < g_num_sms ? P.n_tiles : g_num_sms;
+    if (acc64)
+        conv_tc_kernel<64, long long><<<grid, TC_THREADS, tc_smem_bytes<64>(), st>>>(P);
+    else
+        conv_tc_kernel<128, int><<<grid, TC_THREADS, tc_smem_bytes<128>(), st>>>(P);
+    launched = true;
+    return after_launch("conv_tc");
+}
+
+}  // namespace fxpq

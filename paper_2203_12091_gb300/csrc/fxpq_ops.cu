@@ -6,24 +6,6 @@
 namespace fxpq {
 namespace {
 
-__device__ __forceinline__ int code_at(const __half* __restrict__ t, long long pix, int Cp, int planes, int c) {
-    const __half* p = t + pix * (long long)Cp * planes;
-    if (planes == 1) return __half2int_rn(p[c]);
-    return (__half2int_rn(p[c]) << 8) + __half2int_rn(p[Cp + c]);
-}
-
-__device__ __forceinline__ void put_code(__half* __restrict__ t, long long pix, int Cp, int planes, int c, int code) {
-    __half* p = t + pix * (long long)Cp * planes;
-    if (planes == 1) {
-        p[c] = __int2half_rn(code);
-    } else {
-        __half h, l;
-        split_limbs(code, h, l);
-        p[c] = h;
-        p[Cp + c] = l;
-    }
-}
-
 struct OutArgs {
     int mode;         // FXPQ_OUT_*
     int sh;           // requant shift (CODES)
@@ -32,7 +14,9 @@ struct OutArgs {
     float f32_scale;  // 2^-s
 };
 
-__device__ __forceinline__ void store_out(const OutArgs& o, void* y, long long pix, int Cp, int c, long long v) {
+// y plane stride for CODES output: y_ps elements
+__device__ __forceinline__ void store_out(const OutArgs& o, void* y, long long pix, int Cp, int c, long long v,
+                                          long long y_ps) {
     if (o.mode == FXPQ_OUT_CODES) {
         long long q;
         if (o.sh > 0) {
@@ -46,7 +30,7 @@ __device__ __forceinline__ void store_out(const OutArgs& o, void* y, long long p
                 q = v << l;
         }
         q = q < o.lo ? o.lo : (q > o.hi ? o.hi : q);
-        put_code(static_cast<__half*>(y), pix, Cp, o.py, c, (int)q);
+        code_put(static_cast<__half*>(y), pix * Cp + c, o.py, y_ps, (int)q);
     } else if (o.mode == FXPQ_OUT_ACC64) {
         static_cast<long long*>(y)[pix * Cp + c] = v;
     } else {
@@ -71,10 +55,10 @@ __global__ void maxpool_kernel(const __half* __restrict__ x, int N, int H, int W
             for (int s = 0; s < k; ++s) {
                 const int w = q * stride + s - pad;
                 if (w < 0 || w >= W) continue;
-                best = max(best, code_at(x, (n * H + h) * W + w, Cp, planes, c));
+                best = max(best, code_get(x, ((n * H + h) * W + w) * Cp + c, planes, (long long)N * H * W * Cp));
             }
         }
-        put_code(y, pix, Cp, planes, c, best);
+        code_put(y, pix * Cp + c, planes, total, best);
     }
 }
 
@@ -85,9 +69,9 @@ __global__ void eltwise_kernel(const __half* __restrict__ a, int pa, int sa, con
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += step) {
         const int c = (int)(i % Cp);
         const long long pix = i / Cp;
-        long long v = ((long long)code_at(a, pix, Cp, pa, c) << sa) + ((long long)code_at(b, pix, Cp, pb, c) << sb);
+        long long v = ((long long)code_get(a, i, pa, total) << sa) + ((long long)code_get(b, i, pb, total) << sb);
         if (relu && v < 0) v = 0;
-        store_out(o, y, pix, Cp, c, v);
+        store_out(o, y, pix, Cp, c, v, total);
     }
 }
 
@@ -99,8 +83,8 @@ __global__ void avgpool_kernel(const __half* __restrict__ x, int N, int HW, int 
         const int c = (int)(i % Cp);
         const long long n = i / Cp;
         long long s = 0;
-        for (int t = 0; t < HW; ++t) s += code_at(x, n * HW + t, Cp, planes, c);
-        store_out(o, y, n, Cp, c, s * recip);
+        for (int t = 0; t < HW; ++t) s += code_get(x, (n * HW + t) * Cp + c, planes, (long long)N * HW * Cp);
+        store_out(o, y, n, Cp, c, s * recip, total);
     }
 }
 

@@ -70,7 +70,7 @@ __global__ void quantize_vec4_kernel(const float4* __restrict__ x, long long n4,
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
 
-// rows x C fp32 -> fp16 code tensor rows x (Cp * planes), planes [hi | lo] when k > 8
+// rows x C fp32 -> fp16 code tensor: planes of [rows, Cp] (hi plane, then lo plane when k > 8)
 __global__ void quantize_rows_f16_kernel(const float* __restrict__ x, long long rows, int C, int Cp, int planes,
                                          QParams p, __half* __restrict__ out) {
     bool bad = false;
@@ -80,15 +80,7 @@ __global__ void quantize_rows_f16_kernel(const float* __restrict__ x, long long 
         long long r = i / Cp;
         int c = (int)(i - r * Cp);
         int code = c < C ? quant1(x[r * C + c], p, bad) : 0;
-        __half* o = out + r * (long long)Cp * planes;
-        if (planes == 1) {
-            o[c] = __int2half_rn(code);
-        } else {
-            __half h, l;
-            split_limbs(code, h, l);
-            o[c] = h;
-            o[Cp + c] = l;
-        }
+        code_put(out, i, planes, total, code);
     }
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
@@ -102,17 +94,9 @@ __global__ void quantize_images_kernel(const float* __restrict__ x, int N, int C
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < npix; i += stride) {
         long long n = i / ((long long)H * W);
         long long hw = i - n * H * W;
-        __half* o = out + i * (long long)Cp * planes;
         for (int c = 0; c < Cp; ++c) {
             int code = c < C ? quant1(x[(n * C + c) * (long long)H * W + hw], p, bad) : 0;
-            if (planes == 1) {
-                o[c] = __int2half_rn(code);
-            } else {
-                __half h, l;
-                split_limbs(code, h, l);
-                o[c] = h;
-                o[Cp + c] = l;
-            }
+            code_put(out, i * Cp + c, planes, npix * Cp, code);
         }
     }
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);

@@ -155,12 +155,10 @@ def fxpq_launch_count() -> int:
 
 
 # ------------------------------------------------------------------------------ code tensors
-def codes_to_int(t: torch.Tensor, f: Fmt, C: int | None = None) -> torch.Tensor:
-    """Decode an fp16 code tensor [..., Cp * planes] to int64 codes [..., Cp] (host-side view for tests)."""
-    t = t.to(torch.int64)
+def codes_to_int(t: torch.Tensor, f: Fmt, shape) -> torch.Tensor:
+    """Decode an fp16 code tensor (plane-major, see include/fxpq.h) to int64 codes of `shape`."""
+    t = t.reshape(-1).to(torch.int64)
     if planes(f) == 1:
-        out = t
-    else:
-        cp = t.shape[-1] // 2
-        out = t[..., :cp] * 256 + t[..., cp:]
-    return out if C is None else out[..., :C]
+        return t.view(*shape)
+    t = t.view(2, -1)
+    return (t[0] * 256 + t[1]).view(*shape)

@@ -9,12 +9,20 @@ import oracle
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(scope="module")
-def F():
+@pytest.fixture(scope="module", params=["tc", "simt"])
+def F(request):
+    """Runs every case on the tensor-core kernel (default) and on the CUDA-core kernel."""
+    import os
     import __graft_entry__ as g
     g.build()
     from paper_2203_12091_gb300 import fxpq
-    return fxpq
+    old = os.environ.get("FXPQ_CONV_PATH")
+    os.environ["FXPQ_CONV_PATH"] = request.param
+    yield fxpq
+    if old is None:
+        os.environ.pop("FXPQ_CONV_PATH", None)
+    else:
+        os.environ["FXPQ_CONV_PATH"] = old
 
 
 def rand_codes(rng, shape, k, S):
@@ -27,14 +35,14 @@ def rand_codes(rng, shape, k, S):
 
 
 def to_f16_planes(codes, k, Cp):
-    """Storage encoding of a code tensor [..., C] as fp16 planes [..., Cp * planes] (zero padded)."""
+    """Storage encoding of a code tensor [..., C] as a plane-major fp16 code tensor [..., Cp] (zero padded)."""
     c = np.zeros(codes.shape[:-1] + (Cp,), np.int64)
     c[..., : codes.shape[-1]] = codes
     if k <= 8:
         return torch.from_numpy(c.astype(np.float16)).cuda()
     hi = c >> 8
     lo = c - (hi << 8)
-    return torch.from_numpy(np.concatenate([hi, lo], axis=-1).astype(np.float16)).cuda()
+    return torch.from_numpy(np.stack([hi, lo]).astype(np.float16)).cuda()
 
 
 def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp):
@@ -56,7 +64,7 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp):
     torch.cuda.synchronize()
     assert F.fxpq_get_device_status() == 0
     if mode == F.OUT_CODES:
-        return F.codes_to_int(y.cpu().view(N, P, Q, -1), fy).numpy(), s
+        return F.codes_to_int(y.cpu(), fy, (N, P, Q, K)).numpy(), s
     return y.cpu().numpy().reshape(N, P, Q, K), s
 
 
@@ -103,7 +111,7 @@ def test_conv_parity(F, case):
     got, s = run_conv(F, x, fx, w, fw, b, fb, st, pad, relu, mode, fy, Cp)
     want, ws = oracle_conv(x, fx, w, fw, b, fb, st, pad, relu, mode, fy)
     assert s == ws
-    assert np.array_equal(got[..., :K], want)
+    assert np.array_equal(got, want)
 
 
 def test_gemm_entry_point(F):
@@ -118,7 +126,7 @@ def test_gemm_entry_point(F):
                     fb, M, N, Kd, True, F.OUT_CODES, fy, y)
     want, ws = oracle_conv(x.reshape(M, 1, 1, Kd), fx, w.reshape(N, 1, 1, Kd), fw, b, fb, 1, 0, True, 0, fy)
     assert s == ws
-    assert np.array_equal(F.codes_to_int(y.cpu().view(M, N), fy).numpy(), want.reshape(M, N))
+    assert np.array_equal(F.codes_to_int(y.cpu(), fy, (M, N)).numpy(), want.reshape(M, N))
 
 
 @pytest.mark.parametrize("k,st,pad,bits", [(3, 2, 0, 8), (2, 2, 0, 6), (3, 2, 1, 8), (3, 2, 1, 12), (3, 1, 1, 4)])
@@ -130,7 +138,7 @@ def test_maxpool_parity(F, k, st, pad, bits):
     P = (H + 2 * pad - k) // st + 1
     y = torch.empty(N * P * P * C * (2 if bits > 8 else 1), dtype=torch.float16, device="cuda")
     F.fxpq_maxpool(to_f16_planes(x, bits, C), N, H, H, C, f, k, st, pad, y)
-    got = F.codes_to_int(y.cpu().view(N, P, P, -1), f).numpy()
+    got = F.codes_to_int(y.cpu(), f, (N, P, P, C)).numpy()
     assert np.array_equal(got, oracle.maxpool(x, k, st, pad))
 
 
@@ -153,7 +161,7 @@ def test_eltwise_parity(F, mode, fa, fb, relu):
     v, ws = oracle.eltwise_add(a, fa[2], b, fb[2], relu)
     assert s == ws
     if mode == 0:
-        assert np.array_equal(F.codes_to_int(y.cpu().view(npix, C), FY).numpy(), oracle.requant(v, ws, 7, FY.is_signed, 4))
+        assert np.array_equal(F.codes_to_int(y.cpu(), FY, (npix, C)).numpy(), oracle.requant(v, ws, 7, FY.is_signed, 4))
     elif mode == 1:
         assert np.array_equal(y.cpu().numpy().reshape(npix, C), v)
     else:
@@ -171,4 +179,4 @@ def test_avgpool_parity(F, bits):
     s = F.fxpq_avgpool(to_f16_planes(x, bits, C), N, H, H, C, fx, rc, fr, F.OUT_CODES, fy, y)
     v, ws = oracle.avgpool_global(x, 4, rc, 21)
     assert s == ws
-    assert np.array_equal(F.codes_to_int(y.cpu().view(N, C), fy).numpy(), oracle.requant(v, ws, 8, 0, 5))
+    assert np.array_equal(F.codes_to_int(y.cpu(), fy, (N, C)).numpy(), oracle.requant(v, ws, 8, 0, 5))

@@ -68,7 +68,7 @@ def test_tiny_residual_net(NET):
     for l in L[:-1]:
         t, f = env[l["name"]]
         H, _, Cp = q.shapes[l["name"]]
-        got = F.codes_to_int(t.cpu().view(6, H, H, -1), f).numpy()
+        got = F.codes_to_int(t.cpu(), f, (6, H, H, Cp)).numpy()
         assert np.array_equal(got[..., : oenv[l["name"]][0].shape[-1]], oenv[l["name"]][0]), l["name"]
 
 

@@ -70,15 +70,15 @@ def test_quantize_unaligned_and_nonfinite(F):
 def test_quantize_rows_and_images(F, k, C, Cp):
     rows = 37
     x = synth.normal(rows * C, 7 + k)
-    out = torch.empty(rows, Cp * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
+    out = torch.empty(rows * Cp * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
     F.fxpq_quantize_rows(torch.from_numpy(x).cuda(), rows, C, F.fmt(k, 1, k - 3), Cp, out)
-    got = F.codes_to_int(out.cpu(), F.fmt(k, 1, k - 3)).numpy()
+    got = F.codes_to_int(out.cpu(), F.fmt(k, 1, k - 3), (rows, Cp)).numpy()
     want = oracle.quantize(x, k, 1, k - 3).reshape(rows, C)
     assert np.array_equal(got[:, :C], want) and np.all(got[:, C:] == 0)
     imgs = synth.images(2, 9, hw=13)
     out = torch.empty(2 * 13 * 13 * 8 * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
     F.fxpq_quantize_images(torch.from_numpy(imgs).cuda(), F.fmt(k, 1, k - 4), 8, out)
-    got = F.codes_to_int(out.cpu().view(2, 13, 13, -1), F.fmt(k, 1, k - 4)).numpy()
+    got = F.codes_to_int(out.cpu(), F.fmt(k, 1, k - 4), (2, 13, 13, 8)).numpy()
     want = oracle.quantize(np.transpose(imgs, (0, 2, 3, 1)), k, 1, k - 4).reshape(2, 13, 13, 3)
     assert np.array_equal(got[..., :3], want) and np.all(got[..., 3:] == 0)
 
