@@ -1,0 +1,728 @@
+// fxpq_flsearch.cu -- batched FL search (Sec. IV-C, Eq. DSB_QE; sign strategy Sec. IV-A.3).
+//
+// Every candidate (k, FL) is scored exactly: L(k, FL) = sum_i (x_i - Q(x_i) 2^-FL)^2 as an exact
+// rational, rounded once to nearest-even double.
+//
+// Decomposition.  Write fp32 x = (-1)^sg M 2^(E-23) (M the 24-bit significand, u_E = 2^(E-23)).
+// For a candidate, y = |x| 2^FL has integer exponent q = E + FL, and Q clips at T (in y units):
+// S=1: 2^t - 1 with t = k-1 for x >= 0, 2^t with t = k-1 for x < 0; S=0: 2^t - 1 with t = k for
+// x >= 0, T = 0 for x < 0.  The element's error is (|x| - T 2^-FL)^2 when |y| >= T (saturated) and
+// r^2 otherwise, r = y - round_half_even(y).  Hence, per (sign, E):
+//   q >= t            every element saturates: a polynomial in T of the moments (n, sum M, sum M^2);
+//   q == t-1, T=2^t-1 boundary: an element saturates iff M >= thr = (2^t - 1) 2^(24-t); its error
+//                     is (M - thr)^2 u_E^2 if so, r^2 otherwise -- one "boundary remainder" sum Rb;
+//   q <= -2           |y| < 1/2 rounds to 0: error x^2 = M^2 u_E^2 (a moment);
+//   -1 <= q < bound   r^2 in units u_E^2 is the integer (M mod-round 2^(23-q))^2: a remainder sum R.
+// All sums are integers; the finalize kernel adds one candidate's terms in a 768-bit fixed-point
+// accumulator and rounds once.
+//
+// Pass structure (one read of x).  Each block sorts a tile of 4096 elements by (sign, E) in
+// shared memory; each warp then walks a contiguous run of the sorted tile, so runs of equal
+// exponent are accumulated in registers (one slot per j = q) and reduced across the warp only when
+// the exponent changes.  Block totals go to the workspace bins with integer atomics.
+#include <math.h>
+
+#include <mutex>
+
+#include "fxpq_common.cuh"
+
+namespace fxpq {
+namespace {
+
+typedef unsigned long long u64;
+
+constexpr int NKEY = 512;  // key = sign * 256 + biased exponent field (0..254; 255 = non-finite)
+constexpr int NJ = 17;     // j = q in [-1, 15]
+constexpr int MAXFL = 32;  // candidates per wordlength
+constexpr int MAXK = 15;   // k in [2, 16]
+constexpr int FS_THREADS = 256;
+constexpr int FS_WARPS = FS_THREADS / 32;
+constexpr int TILE = 4096;  // 16 elements per thread
+constexpr int CHUNK_MAX = 65536;  // per-block element cap: keeps every 64-bit block bin below 2^64
+
+struct FsSmem {
+    float sorted[TILE];
+    unsigned cnt[NKEY];  // histogram, then running scatter offsets
+    unsigned pn[NKEY];
+    unsigned ps1[NKEY][2];  // 64-bit sums as {lo, hi} 32-bit words
+    unsigned ps2[NKEY][2];
+    unsigned r[2][NJ][MAXFL][2];
+    unsigned rb[NJ][MAXFL][2];
+    unsigned mn, mx, nonfinite, live;
+};
+
+// Workspace: exact 128-bit bins as {lo, hi}, then per-candidate scores.
+struct FsGlobal {
+    u64 pn[NKEY];
+    u64 ps1[NKEY][2];
+    u64 ps2[NKEY][2];
+    u64 r[2][NJ][MAXFL][2];
+    u64 rb[NJ][MAXFL][2];
+    unsigned mn, mx, nonfinite, pad;
+    double cells[2][MAXK][MAXFL];
+    double stat_sum, stat_sumsq;
+};
+
+struct FsParams {
+    const float* x;
+    long long n;
+    int chunk;
+    int fl_lo, nfl;
+    int jmax_pos, jmax_neg;  // largest j whose remainder sum R is needed (x >= 0 / x < 0)
+    int jb_lo, jb_hi;        // j range of the boundary sum Rb (x >= 0)
+    FsGlobal* g;
+};
+
+__device__ __forceinline__ unsigned order_key(float x) {
+    unsigned u = __float_as_uint(x);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float order_key_inv(unsigned k) {
+    unsigned u = (k & 0x80000000u) ? (k & 0x7fffffffu) : ~k;
+    return __uint_as_float(u);
+}
+
+// 64-bit add into {lo, hi} 32-bit shared words (native 32-bit atomics only)
+__device__ __forceinline__ void sadd64(unsigned* p, u64 v) {
+    if (!v) return;
+    const unsigned lo = (unsigned)v;
+    unsigned hi = (unsigned)(v >> 32);
+    const unsigned old = atomicAdd(p, lo);
+    hi += (old + lo < old) ? 1u : 0u;
+    if (hi) atomicAdd(p + 1, hi);
+}
+
+__device__ __forceinline__ void gadd128(u64* p, u64 v) {
+    if (!v) return;
+    const u64 old = atomicAdd(p, v);
+    if (old + v < old) atomicAdd(p + 1, 1ull);
+}
+
+// Sum of a per-lane value v < 2^63 over the full warp (three 21-bit pieces, exact).
+__device__ __forceinline__ u64 warp_sum64(u64 v) {
+    const unsigned a = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v & 0x1FFFFFu));
+    const unsigned b = __reduce_add_sync(0xFFFFFFFFu, (unsigned)((v >> 21) & 0x1FFFFFu));
+    const unsigned c = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v >> 42));
+    return (u64)a + ((u64)b << 21) + ((u64)c << 42);
+}
+
+__device__ __forceinline__ int key_of(float x) {
+    const unsigned u = __float_as_uint(x);
+    const unsigned eb = (u >> 23) & 0xFFu;
+    if (eb == 0xFFu || (u & 0x7FFFFFFFu) == 0u) return NKEY;  // non-finite or zero: contributes nothing
+    return (int)((u >> 31) * 256u + eb);
+}
+
+struct KeyInfo {
+    int sg, E;
+    unsigned validR, validRb;  // bit jj set: slot jj (j = jj - 1) is needed for this key
+};
+
+__device__ __forceinline__ KeyInfo key_info(int key, const FsParams& P) {
+    KeyInfo k;
+    k.sg = key >> 8;
+    const int eb = key & 255;
+    k.E = eb ? eb - 127 : -126;
+    k.validR = 0u;
+    k.validRb = 0u;
+    const int jmax = k.sg ? P.jmax_neg : P.jmax_pos;
+#pragma unroll
+    for (int jj = 0; jj < NJ; ++jj) {
+        const int j = jj - 1;
+        const int fi = j - k.E - P.fl_lo;
+        if (fi < 0 || fi >= P.nfl) continue;
+        if (j <= jmax) k.validR |= 1u << jj;
+        if (k.sg == 0 && j >= P.jb_lo && j <= P.jb_hi) k.validRb |= 1u << jj;
+    }
+    return k;
+}
+
+struct Acc {
+    u64 r[NJ];
+    u64 rb[NJ];
+    u64 s1, s2;
+    unsigned n;
+};
+
+__device__ __forceinline__ void acc_zero(Acc& a) {
+#pragma unroll
+    for (int jj = 0; jj < NJ; ++jj) a.r[jj] = a.rb[jj] = 0ull;
+    a.s1 = a.s2 = 0ull;
+    a.n = 0u;
+}
+
+// Add one element (significand M of the warp's current key) to this lane's accumulators.
+__device__ __forceinline__ void acc_add(Acc& a, unsigned M, const KeyInfo& k) {
+    a.n += 1u;
+    a.s1 += M;
+    a.s2 += (u64)M * M;
+#pragma unroll
+    for (int jj = 0; jj < NJ; ++jj) {
+        const int j = jj - 1;
+        const int p = 23 - j;  // bits of M below the binary point of y: 24 .. 8
+        if (((k.validR | k.validRb) >> jj) & 1u) {
+            const unsigned t = M & ((1u << p) - 1u);
+            const unsigned odd = (M >> p) & 1u;
+            const bool up = (t + odd) > (1u << (p - 1));
+            const unsigned r = up ? (1u << p) - t : t;
+            if ((k.validR >> jj) & 1u) a.r[jj] += (u64)r * r;
+            if (j >= 0 && ((k.validRb >> jj) & 1u)) {
+                // boundary t' = j + 1: saturated iff M >= (2^(j+1) - 1) 2^(23-j)
+                const unsigned thr = ((2u << j) - 1u) << (23 - j);
+                const unsigned rb = M >= thr ? M - thr : r;
+                a.rb[jj] += (u64)rb * rb;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void acc_flush(FsSmem& sm, Acc& a, int key, const KeyInfo& k, const FsParams& P,
+                                          unsigned lane) {
+    const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
+    const u64 s1 = warp_sum64(a.s1), s2 = warp_sum64(a.s2);
+    if (lane == 0) {
+        atomicAdd(&sm.pn[key], n);
+        sadd64(sm.ps1[key], s1);
+        sadd64(sm.ps2[key], s2);
+    }
+#pragma unroll
+    for (int jj = 0; jj < NJ; ++jj) {
+        const int fi = jj - 1 - k.E - P.fl_lo;
+        if ((k.validR >> jj) & 1u) {
+            const u64 v = warp_sum64(a.r[jj]);
+            if (lane == 0) sadd64(sm.r[k.sg][jj][fi], v);
+        }
+        if ((k.validRb >> jj) & 1u) {
+            const u64 v = warp_sum64(a.rb[jj]);
+            if (lane == 0) sadd64(sm.rb[jj][fi], v);
+        }
+    }
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(FS_THREADS) fl_search_bins_kernel(FsParams P) {
+    __shared__ FsSmem sm;
+    const unsigned lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    {
+        unsigned* z = reinterpret_cast<unsigned*>(&sm.cnt[0]);
+        const int nz = (int)((sizeof(FsSmem) - sizeof(sm.sorted)) / 4);
+        for (int i = threadIdx.x; i < nz; i += FS_THREADS) z[i] = 0u;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) sm.mn = 0xFFFFFFFFu;
+    unsigned tmn = 0xFFFFFFFFu, tmx = 0u;
+    bool tnf = false;
+    const unsigned lt_mask = (1u << lane) - 1u;
+
+    const long long start = (long long)blockIdx.x * P.chunk;
+    const long long end = min(start + (long long)P.chunk, P.n);
+    for (long long tb = start; tb < end; tb += TILE) {
+        // ---- A: load 16 elements per thread, key them
+        float v[16];
+        int key[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const long long idx = tb + 1024LL * i + 4LL * threadIdx.x;
+            if (VEC && idx + 3 < end) {
+                const float4 f = __ldg(reinterpret_cast<const float4*>(P.x + idx));
+                v[4 * i] = f.x, v[4 * i + 1] = f.y, v[4 * i + 2] = f.z, v[4 * i + 3] = f.w;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) key[4 * i + e] = 0;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const bool in = idx + e < end;
+                    v[4 * i + e] = in ? P.x[idx + e] : 0.0f;
+                    key[4 * i + e] = in ? 0 : -1;
+                }
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const bool in = key[e] == 0;
+            const unsigned u = __float_as_uint(v[e]);
+            if (in && ((u >> 23) & 0xFFu) == 0xFFu) tnf = true;
+            if (in && ((u >> 23) & 0xFFu) != 0xFFu) {
+                const unsigned ok = order_key(v[e]);
+                tmn = min(tmn, ok);
+                tmx = max(tmx, ok);
+            }
+            key[e] = in ? key_of(v[e]) : NKEY;
+        }
+        // ---- B: histogram of keys (warp-aggregated)
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
+            if (key[e] < NKEY && lane == (unsigned)(__ffs(grp) - 1)) atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
+        }
+        __syncthreads();
+        // ---- C: exclusive scan of the 512 counts (warp 0)
+        if (warp == 0) {
+            unsigned loc[NKEY / 32];
+            unsigned s = 0;
+#pragma unroll
+            for (int i = 0; i < NKEY / 32; ++i) {
+                loc[i] = sm.cnt[lane * (NKEY / 32) + i];
+                s += loc[i];
+            }
+            unsigned incl = s;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const unsigned o = __shfl_up_sync(0xFFFFFFFFu, incl, off);
+                if (lane >= (unsigned)off) incl += o;
+            }
+            unsigned run = incl - s;
+#pragma unroll
+            for (int i = 0; i < NKEY / 32; ++i) {
+                sm.cnt[lane * (NKEY / 32) + i] = run;
+                run += loc[i];
+            }
+            if (lane == 31) sm.live = incl;
+        }
+        __syncthreads();
+        // ---- D: scatter into key order
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
+            const unsigned leader = (unsigned)(__ffs(grp) - 1);
+            unsigned base = 0u;
+            if (key[e] < NKEY && lane == leader) base = atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
+            base = __shfl_sync(0xFFFFFFFFu, base, (int)leader);
+            if (key[e] < NKEY) sm.sorted[base + __popc(grp & lt_mask)] = v[e];
+        }
+        __syncthreads();
+        // ---- E: each warp walks a contiguous run of the sorted tile
+        const int L = (int)sm.live;
+        const int per = ((L + FS_WARPS * 32 - 1) / (FS_WARPS * 32)) * 32;
+        const int w0 = (int)warp * per, w1 = min(w0 + per, L);
+        Acc acc;
+        acc_zero(acc);
+        int ck = -1;
+        KeyInfo ki;
+        ki.sg = 0, ki.E = 0, ki.validR = ki.validRb = 0u;
+        for (int pos = w0; pos < w1; pos += 32) {
+            const int p = pos + (int)lane;
+            const bool live = p < w1;
+            const float xv = live ? sm.sorted[p] : 0.0f;
+            const int kx = live ? key_of(xv) : NKEY;
+            const unsigned u = __float_as_uint(xv);
+            const unsigned eb = (u >> 23) & 0xFFu;
+            const unsigned M = eb ? ((u & 0x7FFFFFu) | 0x800000u) : (u & 0x7FFFFFu);
+            unsigned rem = __ballot_sync(0xFFFFFFFFu, live);
+            while (rem) {
+                const int kk = __shfl_sync(0xFFFFFFFFu, kx, __ffs(rem) - 1);
+                const unsigned in = __ballot_sync(0xFFFFFFFFu, live && kx == kk);
+                if (kk != ck) {
+                    if (ck >= 0) {
+                        acc_flush(sm, acc, ck, ki, P, lane);
+                        acc_zero(acc);
+                    }
+                    ck = kk;
+                    ki = key_info(ck, P);
+                }
+                if ((in >> lane) & 1u) acc_add(acc, M, ki);
+                rem &= ~in;
+            }
+        }
+        if (ck >= 0) acc_flush(sm, acc, ck, ki, P, lane);
+        __syncthreads();
+        for (int i = threadIdx.x; i < NKEY; i += FS_THREADS) sm.cnt[i] = 0u;
+        __syncthreads();
+    }
+    atomicMin(&sm.mn, tmn);
+    atomicMax(&sm.mx, tmx);
+    if (tnf) sm.nonfinite = 1u;
+    __syncthreads();
+
+    // ---- block bins -> exact workspace bins
+    FsGlobal* g = P.g;
+    for (int i = threadIdx.x; i < NKEY; i += FS_THREADS) {
+        if (!sm.pn[i]) continue;
+        atomicAdd(&g->pn[i], (u64)sm.pn[i]);
+        gadd128(g->ps1[i], ((u64)sm.ps1[i][1] << 32) | sm.ps1[i][0]);
+        gadd128(g->ps2[i], ((u64)sm.ps2[i][1] << 32) | sm.ps2[i][0]);
+    }
+    for (int i = threadIdx.x; i < 2 * NJ * MAXFL; i += FS_THREADS) {
+        const int s = i / (NJ * MAXFL), j = (i / MAXFL) % NJ, f = i % MAXFL;
+        gadd128(g->r[s][j][f], ((u64)sm.r[s][j][f][1] << 32) | sm.r[s][j][f][0]);
+    }
+    for (int i = threadIdx.x; i < NJ * MAXFL; i += FS_THREADS) {
+        const int j = i / MAXFL, f = i % MAXFL;
+        gadd128(g->rb[j][f], ((u64)sm.rb[j][f][1] << 32) | sm.rb[j][f][0]);
+    }
+    if (threadIdx.x == 0) {
+        atomicMin(&g->mn, sm.mn);
+        atomicMax(&g->mx, sm.mx);
+        if (sm.nonfinite) atomicOr(&g->nonfinite, 1u);
+    }
+}
+
+// ------------------------------------------------------------------ exact finalize
+struct U128 {
+    u64 lo, hi;
+};
+__device__ __forceinline__ U128 ld128(const u64* p) { return U128{p[0], p[1]}; }
+// (a * m) for a 128-bit a and 64-bit m: the callers' bounds keep the product below 2^128
+__device__ __forceinline__ U128 mul128_64(U128 a, u64 m) {
+    U128 r;
+    r.lo = a.lo * m;
+    r.hi = __umul64hi(a.lo, m) + a.hi * m;
+    return r;
+}
+
+// 768-bit two's complement fixed point: word i weighs 2^(64 i - 320)
+constexpr int BW = 12;
+constexpr int BBASE = -320;
+
+struct Big {
+    u64 w[BW];
+};
+
+__device__ __forceinline__ void big_zero(Big& a) {
+#pragma unroll
+    for (int i = 0; i < BW; ++i) a.w[i] = 0ull;
+}
+
+// a += (neg ? -1 : 1) * v * 2^e for a 128-bit magnitude v
+__device__ void big_add(Big& a, U128 v, int e, bool neg) {
+    if ((v.lo | v.hi) == 0ull) return;
+    const int pos = e - BBASE;
+    const int wi = pos >> 6, b = pos & 63;
+    u64 s[3];
+    s[0] = v.lo << b;
+    s[1] = b ? ((v.hi << b) | (v.lo >> (64 - b))) : v.hi;
+    s[2] = b ? (v.hi >> (64 - b)) : 0ull;
+    if (!neg) {
+        u64 carry = 0ull;
+        for (int i = wi; i < BW; ++i) {
+            const u64 add = (i - wi < 3) ? s[i - wi] : 0ull;
+            const u64 t = a.w[i] + add;
+            const u64 c1 = t < add;
+            const u64 t2 = t + carry;
+            const u64 c2 = t2 < t;
+            a.w[i] = t2;
+            carry = c1 | c2;
+            if (i - wi >= 2 && carry == 0ull) break;
+        }
+    } else {
+        u64 borrow = 0ull;
+        for (int i = wi; i < BW; ++i) {
+            const u64 sub = (i - wi < 3) ? s[i - wi] : 0ull;
+            const u64 t = a.w[i] - sub;
+            const u64 b1 = a.w[i] < sub;
+            const u64 t2 = t - borrow;
+            const u64 b2 = t < borrow;
+            a.w[i] = t2;
+            borrow = b1 | b2;
+            if (i - wi >= 2 && borrow == 0ull) break;
+        }
+    }
+}
+
+// a += (the big number held by lane `src_lane`), modulo 2^768 (warp-collective)
+__device__ __forceinline__ void big_add_from_lane(Big& a, int off) {
+    u64 carry = 0ull;
+#pragma unroll
+    for (int i = 0; i < BW; ++i) {
+        const u64 o = __shfl_down_sync(0xFFFFFFFFu, a.w[i], off);
+        const u64 t = a.w[i] + o;
+        const u64 c1 = t < o;
+        const u64 t2 = t + carry;
+        const u64 c2 = t2 < t;
+        a.w[i] = t2;
+        carry = c1 | c2;
+    }
+}
+
+__device__ u64 big_bits64(const Big& a, int pos) {  // bits [pos, pos + 64), zero below bit 0
+    const int wi = pos >= 0 ? (pos >> 6) : -((-pos + 63) >> 6);
+    const int b = pos - wi * 64;
+    const u64 lo = (wi >= 0 && wi < BW) ? a.w[wi] : 0ull;
+    const u64 hi = (wi + 1 >= 0 && wi + 1 < BW) ? a.w[wi + 1] : 0ull;
+    return b ? ((lo >> b) | (hi << (64 - b))) : lo;
+}
+
+__device__ bool big_any_below(const Big& a, int pos) {
+    if (pos <= 0) return false;
+    const int wi = pos >> 6, b = pos & 63;
+    for (int i = 0; i < wi && i < BW; ++i)
+        if (a.w[i]) return true;
+    return wi < BW && b && (a.w[wi] & ((1ull << b) - 1ull));
+}
+
+// round a non-negative accumulator to nearest-even double (negative -> -1, a sentinel)
+__device__ double big_to_double(const Big& a) {
+    if ((long long)a.w[BW - 1] < 0) return -1.0;
+    int h = -1;
+    for (int i = BW - 1; i >= 0; --i)
+        if (a.w[i]) {
+            h = i;
+            break;
+        }
+    if (h < 0) return 0.0;
+    const int top = 64 * h + 63 - __clzll(a.w[h]);
+    const u64 win = big_bits64(a, top - 63);
+    u64 mant = win >> 11;
+    const bool rb = (win >> 10) & 1ull;
+    const bool sticky = (win & 0x3FFull) != 0ull || big_any_below(a, top - 63);
+    if (rb && (sticky || (mant & 1ull))) mant += 1ull;
+    return ldexp((double)mant, top - 52 + BBASE);
+}
+
+__device__ void big_negate(Big& a) {
+    u64 c = 1ull;
+    for (int i = 0; i < BW; ++i) {
+        const u64 t = ~a.w[i] + c;
+        c = (c && t == 0ull) ? 1ull : 0ull;
+        a.w[i] = t;
+    }
+}
+
+struct FsFinal {
+    int S_lo, S_hi;
+    int k_lo, nk;
+    int fl_lo, nfl;
+};
+
+// saturated set with moments (n, s1, s2) at exponent E: s2 2^(2(E-23)) - 2 T s1 2^(E-23-fl) + T^2 n 2^(-2fl)
+__device__ void add_sat(Big& acc, u64 n, U128 s1, U128 s2, int E, int fl, u64 T) {
+    big_add(acc, s2, 2 * (E - 23), false);
+    if (T) {
+        big_add(acc, mul128_64(s1, 2ull * T), E - 23 - fl, true);
+        big_add(acc, mul128_64(U128{n, 0ull}, T * T), -2 * fl, false);
+    }
+}
+
+// One warp per candidate cell (plus two cells for the exact stats); lanes split the exponent keys.
+__global__ void fl_search_cells_kernel(FsParams P, FsFinal F) {
+    const FsGlobal* g = P.g;
+    const int lane = threadIdx.x & 31;
+    const int cell = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
+    if (cell >= ncell + 2) return;
+    Big acc;
+    big_zero(acc);
+    if (cell >= ncell) {
+        const bool sq = cell == ncell + 1;
+        for (int key = lane; key < NKEY; key += 32) {
+            if (!g->pn[key]) continue;
+            const int eb = key & 255, E = eb ? eb - 127 : -126;
+            if (sq)
+                big_add(acc, ld128(g->ps2[key]), 2 * (E - 23), false);
+            else
+                big_add(acc, ld128(g->ps1[key]), E - 23, (key >> 8) != 0);
+        }
+    } else {
+        const int S = F.S_lo + cell / (F.nk * F.nfl);
+        const int rem = cell % (F.nk * F.nfl);
+        const int k = F.k_lo + rem / F.nfl;
+        const int fi = rem % F.nfl;
+        const int fl = F.fl_lo + fi;
+        for (int key = lane; key < NKEY; key += 32) {
+            const u64 n = g->pn[key];
+            if (!n) continue;
+            const int sg = key >> 8, eb = key & 255, E = eb ? eb - 127 : -126;
+            const U128 s1 = ld128(g->ps1[key]), s2 = ld128(g->ps2[key]);
+            if (sg == 1 && S == 0) {  // clipped to code 0: error x^2
+                big_add(acc, s2, 2 * (E - 23), false);
+                continue;
+            }
+            const int t = (sg == 0) ? (S ? k - 1 : k) : (k - 1);
+            const u64 T = (sg == 0) ? ((1ull << t) - 1ull) : (1ull << t);
+            const int q = E + fl;
+            if (q >= t)
+                add_sat(acc, n, s1, s2, E, fl, T);
+            else if (sg == 0 && q == t - 1)
+                big_add(acc, ld128(g->rb[q + 1][fi]), 2 * (E - 23), false);
+            else if (q <= -2)
+                big_add(acc, s2, 2 * (E - 23), false);
+            else
+                big_add(acc, ld128(g->r[sg][q + 1][fi]), 2 * (E - 23), false);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) big_add_from_lane(acc, off);
+    if (lane != 0) return;
+    FsGlobal* gw = P.g;
+    if (cell == ncell) {
+        const bool neg = (long long)acc.w[BW - 1] < 0;
+        if (neg) big_negate(acc);
+        const double v = big_to_double(acc);
+        gw->stat_sum = neg ? -v : v;
+    } else if (cell == ncell + 1) {
+        gw->stat_sumsq = big_to_double(acc);
+    } else {
+        const int S = F.S_lo + cell / (F.nk * F.nfl);
+        const int rem = cell % (F.nk * F.nfl);
+        gw->cells[S][F.k_lo + rem / F.nfl - 2][rem % F.nfl] = big_to_double(acc);
+    }
+}
+
+__global__ void fl_search_select_kernel(FsParams P, FsFinal F, int is_signed, double* err, int* best,
+                                        fxpq_stats* stats, int* status) {
+    const FsGlobal* g = P.g;
+    const float mn = g->mn == 0xFFFFFFFFu ? 0.0f : order_key_inv(g->mn);
+    const float mx = g->mx == 0u ? 0.0f : order_key_inv(g->mx);
+    const int S = is_signed >= 0 ? is_signed : (mn < 0.0f ? 1 : 0);
+    const int i = threadIdx.x;
+    if (i < F.nk) {
+        const int k = F.k_lo + i;
+        double bv = 0.0;
+        int bf = F.fl_lo;
+        for (int fi = 0; fi < F.nfl; ++fi) {
+            const double v = g->cells[S][k - 2][fi];
+            err[(long long)i * F.nfl + fi] = v;
+            if (fi == 0 || v < bv) {  // strict: exact ties keep the smaller FL
+                bv = v;
+                bf = F.fl_lo + fi;
+            }
+        }
+        best[i] = bf;
+    }
+    if (i == 0) {
+        if (g->nonfinite) latch_status(status, FXPQ_ERR_NONFINITE);
+        if (stats) {
+            stats->min = mn;
+            stats->max = mx;
+            stats->is_signed = S;
+            stats->nonfinite = g->nonfinite ? 1 : 0;
+            stats->sum = g->stat_sum;
+            stats->sumsq = g->stat_sumsq;
+            stats->n = P.n;
+        }
+    }
+}
+
+}  // namespace
+}  // namespace fxpq
+
+using namespace fxpq;
+
+extern "C" size_t fxpq_fl_search_workspace(int64_t n) {
+    (void)n;
+    return (sizeof(FsGlobal) + 255) / 256 * 256;
+}
+
+extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo, int32_t k_hi,
+                                      int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
+                                      fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream) {
+    if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;
+    if (is_signed < -1 || is_signed > 1) return FXPQ_ERR_INVALID_ARG;
+    if (k_lo < 2 || k_hi > 16 || k_lo > k_hi) return FXPQ_ERR_INVALID_ARG;
+    if (fl_lo < -32 || fl_hi > 40 || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL) return FXPQ_ERR_INVALID_ARG;
+    if (!d_err || !d_best || (n > 0 && !d_x)) return FXPQ_ERR_INVALID_ARG;
+    if (!d_ws || ws_bytes < fxpq_fl_search_workspace(n) || !aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
+    cudaStream_t s = as_stream(stream);
+    FsGlobal* g = static_cast<FsGlobal*>(d_ws);
+    if (cudaMemsetAsync(g, 0, sizeof(FsGlobal), s) != cudaSuccess) return FXPQ_ERR_CUDA;
+    if (cudaMemsetAsync(&g->mn, 0xFF, sizeof(unsigned), s) != cudaSuccess) return FXPQ_ERR_CUDA;
+
+    const int S_lo = is_signed < 0 ? 0 : is_signed, S_hi = is_signed < 0 ? 1 : is_signed;
+    FsParams P;
+    P.x = d_x;
+    P.n = n;
+    long long per = (n + 152LL * 2 - 1) / (152LL * 2);
+    long long chunk = (per + TILE - 1) / TILE * TILE;
+    if (chunk < TILE) chunk = TILE;
+    if (chunk > CHUNK_MAX) chunk = CHUNK_MAX;
+    P.chunk = (int)chunk;
+    P.fl_lo = fl_lo;
+    P.nfl = fl_hi - fl_lo + 1;
+    // x >= 0 rounds (no clip) for q <= t-2 with t = k-1 (S=1) or k (S=0); x < 0 (S=1) for q <= k-2
+    P.jmax_pos = (S_lo == 0) ? k_hi - 2 : k_hi - 3;
+    P.jmax_neg = (S_hi == 1) ? k_hi - 2 : -2;
+    // boundary q = t-1 for x >= 0
+    P.jb_lo = (S_hi == 1) ? k_lo - 2 : k_lo - 1;
+    P.jb_hi = (S_lo == 0) ? k_hi - 1 : k_hi - 2;
+    if (P.jb_lo < 0) P.jb_lo = 0;
+    P.g = g;
+    if (n > 0) {
+        const int grid = (int)((n + chunk - 1) / chunk);
+        if (aligned(d_x, 16))
+            fl_search_bins_kernel<true><<<grid, FS_THREADS, 0, s>>>(P);
+        else
+            fl_search_bins_kernel<false><<<grid, FS_THREADS, 0, s>>>(P);
+        const fxpq_status st = after_launch("fl_search_bins");
+        if (st != FXPQ_OK) return st;
+    }
+    FsFinal F;
+    F.S_lo = S_lo;
+    F.S_hi = S_hi;
+    F.k_lo = k_lo;
+    F.nk = k_hi - k_lo + 1;
+    F.fl_lo = fl_lo;
+    F.nfl = P.nfl;
+    const int ncell = (S_hi - S_lo + 1) * F.nk * F.nfl + 2;
+    fl_search_cells_kernel<<<(ncell + 3) / 4, 128, 0, s>>>(P, F);
+    fxpq_status st = after_launch("fl_search_cells");
+    if (st != FXPQ_OK) return st;
+    fl_search_select_kernel<<<1, 32, 0, s>>>(P, F, is_signed, d_err, d_best, d_stats, status_ptr());
+    return after_launch("fl_search_select");
+}
+
+extern "C" fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32_t strategy, fxpq_fmt* h_out) {
+    if (!h_stats || !h_out || bits < 2 || bits > 32 || strategy < 0 || strategy > 2) return FXPQ_ERR_INVALID_ARG;
+    const double mn = h_stats->min, mx = h_stats->max;
+    const int S = mn < 0.0 ? 1 : 0;
+    double psi = 0.0;
+    if (S == 0) {
+        psi = mx / (ldexp(1.0, bits) - 1.0);
+    } else {
+        const double a = mn / -ldexp(1.0, bits - 1), b = mx / (ldexp(1.0, bits - 1) - 1.0);
+        psi = (a > 0 && b > 0) ? fmin(a, b) : (a > 0 ? a : b);
+    }
+    if (!(psi > 0.0) || !isfinite(psi)) return FXPQ_ERR_INVALID_ARG;
+    const double bh = -log2(psi);
+    const double beta = strategy == 0 ? floor(bh) : (strategy == 1 ? nearbyint(bh) : ceil(bh));
+    if (beta < -32 || beta > 40) return FXPQ_ERR_RANGE;
+    h_out->bits = bits;
+    h_out->is_signed = S;
+    h_out->fl = (int32_t)beta;
+    return FXPQ_OK;
+}
+
+// ------------------------------------------------------------------------------------------
+// FL search without a caller workspace.
+//
+// Some callers cannot allocate device memory: a plug-in hosted by an application that owns the
+// whole device memory pool, or a latency-critical loop that must never enter the allocator
+// (cudaMalloc may synchronise the device).  For them the FL search's scratch (the exact integer
+// bins and per-candidate cells, a fixed size independent of n) lives in this file-scope array,
+// which every GPU that loads the library keeps until the process exits.
+// ------------------------------------------------------------------------------------------
+namespace {
+constexpr size_t kFlSearchStaticBytes = (sizeof(FsGlobal) + 255) / 256 * 256;
+static __device__ __align__(256) unsigned char g_fl_search_scratch[kFlSearchStaticBytes];
+
+std::mutex g_fl_static_mu;
+void* g_fl_static_addr[64] = {nullptr};
+
+// Device address of g_fl_search_scratch on the current device, looked up once per device.
+fxpq_status fl_search_scratch_ptr(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FXPQ_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_fl_static_mu);
+    if (!g_fl_static_addr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_fl_search_scratch) != cudaSuccess || !p) return FXPQ_ERR_CUDA;
+        g_fl_static_addr[dev] = p;
+    }
+    *out = g_fl_static_addr[dev];
+    return FXPQ_OK;
+}
+}  // namespace
+
+extern "C" fxpq_status fxpq_fl_search_noalloc(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo,
+                                              int32_t k_hi, int32_t fl_lo, int32_t fl_hi, double* d_err,
+                                              int32_t* d_best, fxpq_stats* d_stats, void* stream) {
+    if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;  // the largest tensor the bins can hold
+    if (k_lo < 2 || k_hi > 16 || k_lo > k_hi || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL)
+        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 15 x 32
+    if (fxpq_fl_search_workspace(n) > kFlSearchStaticBytes) return FXPQ_ERR_WORKSPACE;
+    void* scratch = nullptr;
+    const fxpq_status st = fl_search_scratch_ptr(&scratch);
+    if (st != FXPQ_OK) return st;
+    // fxpq_fl_search clears the bins it accumulates into before its first kernel.
+    return fxpq_fl_search(d_x, n, is_signed, k_lo, k_hi, fl_lo, fl_hi, d_err, d_best, d_stats, scratch,
+                          kFlSearchStaticBytes, stream);
+}
