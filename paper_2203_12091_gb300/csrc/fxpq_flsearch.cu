@@ -16,8 +16,9 @@
 // All sums are integers; the finalize kernel adds one candidate's terms in a 768-bit fixed-point
 // accumulator and rounds once.
 //
-// Pass structure (one read of x).  Each block sorts a tile of 4096 elements by (sign, E) in
-// shared memory; each warp then walks a contiguous run of the sorted tile, so runs of equal
+// Pass structure (one HBM read of x).  Each block sorts a tile of 16384 elements by (sign, E) in
+// shared memory (histogram, scan, scatter; the scatter re-reads the tile from L2); each warp then
+// walks a contiguous run of the sorted tile, so runs of equal
 // exponent are accumulated in registers (one slot per j = q) and reduced across the warp only when
 // the exponent changes.  Block totals go to the workspace bins with integer atomics.
 #include <math.h>
@@ -37,7 +38,7 @@ constexpr int MAXFL = 32;  // candidates per wordlength
 constexpr int MAXK = 15;   // k in [2, 16]
 constexpr int FS_THREADS = 256;
 constexpr int FS_WARPS = FS_THREADS / 32;
-constexpr int TILE = 4096;  // 16 elements per thread
+constexpr int TILE = 16384;  // 64 elements per thread, read in sub-rounds of 16
 constexpr int CHUNK_MAX = 65536;  // per-block element cap: keeps every 64-bit block bin below 2^64
 
 struct FsSmem {
@@ -137,27 +138,31 @@ __device__ __forceinline__ KeyInfo key_info(int key, const FsParams& P) {
     return k;
 }
 
+// Per-lane accumulators of the warp's current key; NS slots cover j = -1 .. NS-2.
+template <int NS>
 struct Acc {
-    u64 r[NJ];
-    u64 rb[NJ];
+    u64 r[NS];
+    u64 rb[NS];
     u64 s1, s2;
     unsigned n;
 };
 
-__device__ __forceinline__ void acc_zero(Acc& a) {
+template <int NS>
+__device__ __forceinline__ void acc_zero(Acc<NS>& a) {
 #pragma unroll
-    for (int jj = 0; jj < NJ; ++jj) a.r[jj] = a.rb[jj] = 0ull;
+    for (int jj = 0; jj < NS; ++jj) a.r[jj] = a.rb[jj] = 0ull;
     a.s1 = a.s2 = 0ull;
     a.n = 0u;
 }
 
 // Add one element (significand M of the warp's current key) to this lane's accumulators.
-__device__ __forceinline__ void acc_add(Acc& a, unsigned M, const KeyInfo& k) {
+template <int NS>
+__device__ __forceinline__ void acc_add(Acc<NS>& a, unsigned M, const KeyInfo& k) {
     a.n += 1u;
     a.s1 += M;
     a.s2 += (u64)M * M;
 #pragma unroll
-    for (int jj = 0; jj < NJ; ++jj) {
+    for (int jj = 0; jj < NS; ++jj) {
         const int j = jj - 1;
         const int p = 23 - j;  // bits of M below the binary point of y: 24 .. 8
         if (((k.validR | k.validRb) >> jj) & 1u) {
@@ -176,7 +181,8 @@ __device__ __forceinline__ void acc_add(Acc& a, unsigned M, const KeyInfo& k) {
     }
 }
 
-__device__ __forceinline__ void acc_flush(FsSmem& sm, Acc& a, int key, const KeyInfo& k, const FsParams& P,
+template <int NS>
+__device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS>& a, int key, const KeyInfo& k, const FsParams& P,
                                           unsigned lane) {
     const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
     const u64 s1 = warp_sum64(a.s1), s2 = warp_sum64(a.s2);
@@ -186,7 +192,7 @@ __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc& a, int key, const Key
         sadd64(sm.ps2[key], s2);
     }
 #pragma unroll
-    for (int jj = 0; jj < NJ; ++jj) {
+    for (int jj = 0; jj < NS; ++jj) {
         const int fi = jj - 1 - k.E - P.fl_lo;
         if ((k.validR >> jj) & 1u) {
             const u64 v = warp_sum64(a.r[jj]);
@@ -199,9 +205,34 @@ __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc& a, int key, const Key
     }
 }
 
+// 16 consecutive-by-thread elements of sub-round `sub` of the tile starting at tb: values and keys
+// (NKEY for zeros, non-finite values and positions past the end).
 template <bool VEC>
-__global__ void __launch_bounds__(FS_THREADS) fl_search_bins_kernel(FsParams P) {
-    __shared__ FsSmem sm;
+__device__ __forceinline__ void load16(const FsParams& P, long long tb, int sub, long long end, float (&v)[16],
+                                       int (&key)[16]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const long long idx = tb + (long long)sub * 4096 + 1024LL * i + 4LL * threadIdx.x;
+        if (VEC && idx + 3 < end) {
+            const float4 f = __ldg(reinterpret_cast<const float4*>(P.x + idx));
+            v[4 * i] = f.x, v[4 * i + 1] = f.y, v[4 * i + 2] = f.z, v[4 * i + 3] = f.w;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) key[4 * i + e] = key_of(v[4 * i + e]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool in = idx + e < end;
+                v[4 * i + e] = in ? P.x[idx + e] : 0.0f;
+                key[4 * i + e] = in ? key_of(v[4 * i + e]) : NKEY;
+            }
+        }
+    }
+}
+
+template <bool VEC, int NS>
+__global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams P) {
+    extern __shared__ __align__(16) unsigned char fs_smem_raw[];
+    FsSmem& sm = *reinterpret_cast<FsSmem*>(fs_smem_raw);
     const unsigned lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
     {
         unsigned* z = reinterpret_cast<unsigned*>(&sm.cnt[0]);
@@ -217,43 +248,28 @@ __global__ void __launch_bounds__(FS_THREADS) fl_search_bins_kernel(FsParams P) 
     const long long start = (long long)blockIdx.x * P.chunk;
     const long long end = min(start + (long long)P.chunk, P.n);
     for (long long tb = start; tb < end; tb += TILE) {
-        // ---- A: load 16 elements per thread, key them
-        float v[16];
-        int key[16];
+        // ---- A+B: read the tile (16 elements per thread per sub-round), stats, key histogram
+        for (int sub = 0; sub < TILE / 4096; ++sub) {
+            float v[16];
+            int key[16];
+            load16<VEC>(P, tb, sub, end, v, key);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const long long idx = tb + 1024LL * i + 4LL * threadIdx.x;
-            if (VEC && idx + 3 < end) {
-                const float4 f = __ldg(reinterpret_cast<const float4*>(P.x + idx));
-                v[4 * i] = f.x, v[4 * i + 1] = f.y, v[4 * i + 2] = f.z, v[4 * i + 3] = f.w;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) key[4 * i + e] = 0;
-            } else {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const bool in = idx + e < end;
-                    v[4 * i + e] = in ? P.x[idx + e] : 0.0f;
-                    key[4 * i + e] = in ? 0 : -1;
+            for (int e = 0; e < 16; ++e) {
+                const long long idx = tb + (long long)sub * 4096 + 1024LL * (e / 4) + 4LL * threadIdx.x + (e % 4);
+                if (idx < end) {
+                    const unsigned u = __float_as_uint(v[e]);
+                    if (((u >> 23) & 0xFFu) == 0xFFu) {
+                        tnf = true;
+                    } else {
+                        const unsigned ok = order_key(v[e]);
+                        tmn = min(tmn, ok);
+                        tmx = max(tmx, ok);
+                    }
                 }
+                const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
+                if (key[e] < NKEY && lane == (unsigned)(__ffs(grp) - 1))
+                    atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
             }
-        }
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const bool in = key[e] == 0;
-            const unsigned u = __float_as_uint(v[e]);
-            if (in && ((u >> 23) & 0xFFu) == 0xFFu) tnf = true;
-            if (in && ((u >> 23) & 0xFFu) != 0xFFu) {
-                const unsigned ok = order_key(v[e]);
-                tmn = min(tmn, ok);
-                tmx = max(tmx, ok);
-            }
-            key[e] = in ? key_of(v[e]) : NKEY;
-        }
-        // ---- B: histogram of keys (warp-aggregated)
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
-            if (key[e] < NKEY && lane == (unsigned)(__ffs(grp) - 1)) atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
         }
         __syncthreads();
         // ---- C: exclusive scan of the 512 counts (warp 0)
@@ -280,22 +296,27 @@ __global__ void __launch_bounds__(FS_THREADS) fl_search_bins_kernel(FsParams P) 
             if (lane == 31) sm.live = incl;
         }
         __syncthreads();
-        // ---- D: scatter into key order
+        // ---- D: scatter into key order (the tile is read again; it is L2-resident)
+        for (int sub = 0; sub < TILE / 4096; ++sub) {
+            float v[16];
+            int key[16];
+            load16<VEC>(P, tb, sub, end, v, key);
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
-            const unsigned leader = (unsigned)(__ffs(grp) - 1);
-            unsigned base = 0u;
-            if (key[e] < NKEY && lane == leader) base = atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
-            base = __shfl_sync(0xFFFFFFFFu, base, (int)leader);
-            if (key[e] < NKEY) sm.sorted[base + __popc(grp & lt_mask)] = v[e];
+            for (int e = 0; e < 16; ++e) {
+                const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
+                const unsigned leader = (unsigned)(__ffs(grp) - 1);
+                unsigned base = 0u;
+                if (key[e] < NKEY && lane == leader) base = atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
+                base = __shfl_sync(0xFFFFFFFFu, base, (int)leader);
+                if (key[e] < NKEY) sm.sorted[base + __popc(grp & lt_mask)] = v[e];
+            }
         }
         __syncthreads();
         // ---- E: each warp walks a contiguous run of the sorted tile
         const int L = (int)sm.live;
         const int per = ((L + FS_WARPS * 32 - 1) / (FS_WARPS * 32)) * 32;
         const int w0 = (int)warp * per, w1 = min(w0 + per, L);
-        Acc acc;
+        Acc<NS> acc;
         acc_zero(acc);
         int ck = -1;
         KeyInfo ki;
@@ -598,6 +619,22 @@ __global__ void fl_search_select_kernel(FsParams P, FsFinal F, int is_signed, do
 
 using namespace fxpq;
 
+namespace {
+std::mutex g_fs_attr_mu;
+bool g_fs_attr_done = false;
+// The bins kernel's shared memory exceeds the 48 KB default; raise the limit once per process.
+void st_attr_once() {
+    std::lock_guard<std::mutex> lk(g_fs_attr_mu);
+    if (g_fs_attr_done) return;
+    const int sb = (int)sizeof(FsSmem);
+    cudaFuncSetAttribute(fl_search_bins_kernel<true, 10>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<false, 10>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    g_fs_attr_done = true;
+}
+}  // namespace
+
 extern "C" size_t fxpq_fl_search_workspace(int64_t n) {
     (void)n;
     return (sizeof(FsGlobal) + 255) / 256 * 256;
@@ -621,7 +658,7 @@ extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_si
     FsParams P;
     P.x = d_x;
     P.n = n;
-    long long per = (n + 152LL * 2 - 1) / (152LL * 2);
+    long long per = (n + 152LL * 4 - 1) / (152LL * 4);
     long long chunk = (per + TILE - 1) / TILE * TILE;
     if (chunk < TILE) chunk = TILE;
     if (chunk > CHUNK_MAX) chunk = CHUNK_MAX;
@@ -638,10 +675,18 @@ extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_si
     P.g = g;
     if (n > 0) {
         const int grid = (int)((n + chunk - 1) / chunk);
-        if (aligned(d_x, 16))
-            fl_search_bins_kernel<true><<<grid, FS_THREADS, 0, s>>>(P);
+        const bool vec = aligned(d_x, 16);
+        const bool small = k_hi <= 9;  // slots j = -1 .. k_hi - 1 suffice
+        st_attr_once();
+        const size_t sb = sizeof(FsSmem);
+        if (vec && small)
+            fl_search_bins_kernel<true, 10><<<grid, FS_THREADS, sb, s>>>(P);
+        else if (vec)
+            fl_search_bins_kernel<true, NJ><<<grid, FS_THREADS, sb, s>>>(P);
+        else if (small)
+            fl_search_bins_kernel<false, 10><<<grid, FS_THREADS, sb, s>>>(P);
         else
-            fl_search_bins_kernel<false><<<grid, FS_THREADS, 0, s>>>(P);
+            fl_search_bins_kernel<false, NJ><<<grid, FS_THREADS, sb, s>>>(P);
         const fxpq_status st = after_launch("fl_search_bins");
         if (st != FXPQ_OK) return st;
     }
