@@ -22,30 +22,42 @@ struct ConvArgs {
     float f32_scale;   // 2^-s_out
 };
 
-// Bias alignment, ReLU and the FxP-QLayer for one output value of row m, channel k.
-__device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long long m, int k, long long v) {
+// Bias alignment (B << delta, or the accumulator shifted left when delta < 0) and ReLU: the C-Block
+// output before its FxP-QLayer, in units of 2^-s_out.
+__device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long long v, int32_t bias) {
     if (a.has_bias) {
-        const long long b = a.bias[k];
+        const long long b = bias;
         if (a.delta >= 0)
             v += b << a.delta;
         else
             v = (v << (-a.delta)) + b;
     }
     if (a.relu && v < 0) v = 0;
+    return v;
+}
+
+// FxP-QLayer: v * 2^(fl_y - s_out) rounded half to even on the dropped bits, clipped to fmt_y.
+__device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
+    long long q;
+    if (a.sh > 0) {
+        q = rne_shift(v, a.sh);
+    } else {
+        const int l = -a.sh;  // left shift; saturate before it could overflow
+        const long long lim = 1LL << 20;
+        if (l >= 32 || v > lim || v < -lim)
+            q = v > 0 ? a.hi : (v < 0 ? a.lo : 0);
+        else
+            q = v << l;
+    }
+    q = q < a.lo ? a.lo : (q > a.hi ? a.hi : q);
+    return (int)q;
+}
+
+// Bias alignment, ReLU and the FxP-QLayer for one output value of row m, channel k.
+__device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long long m, int k, long long v) {
+    v = cblock_value(a, k, v, a.has_bias ? a.bias[k] : 0);
     if (a.out_mode == FXPQ_OUT_CODES) {
-        long long q;
-        if (a.sh > 0) {
-            q = rne_shift(v, a.sh);
-        } else {
-            const int l = -a.sh;  // left shift; saturate before it could overflow
-            const long long lim = 1LL << 20;
-            if (l >= 32 || v > lim || v < -lim)
-                q = v > 0 ? a.hi : (v < 0 ? a.lo : 0);
-            else
-                q = v << l;
-        }
-        q = q < a.lo ? a.lo : (q > a.hi ? a.hi : q);
-        code_put(static_cast<__half*>(a.y), m * a.K + k, a.py, a.M * a.K, (int)q);
+        code_put(static_cast<__half*>(a.y), m * a.K + k, a.py, a.M * a.K, qlayer_code(a, v));
     } else if (a.out_mode == FXPQ_OUT_ACC64) {
         static_cast<long long*>(a.y)[m * a.K + k] = v;
     } else {

@@ -156,12 +156,84 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
+__device__ __forceinline__ void tmem_ld32u(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]),
+        "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
+        "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Final epilogue of 32 consecutive output channels k0.. of row m (16-byte stores when the block is
+// whole): bias alignment, ReLU, FxP-QLayer / int64 / fp32 image.
+template <typename ACC>
+__device__ __forceinline__ void epilogue_block32(const ConvArgs& a, long long m, int k0, const ACC (&acc)[32]) {
+    const bool whole = k0 + 32 <= a.K;
+    long long v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const int k = k0 + j;
+        const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+        v[j] = cblock_value(a, k, (long long)acc[j], b);
+    }
+    if (a.out_mode == FXPQ_OUT_CODES) {
+        __half* y = static_cast<__half*>(a.y);
+        const long long base = m * a.K + k0;
+        if (whole && a.py == 1) {
+            uint32_t w[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const __half h0 = __int2half_rn(qlayer_code(a, v[2 * j])), h1 = __int2half_rn(qlayer_code(a, v[2 * j + 1]));
+                w[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(y + base);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (k0 + j < a.K) code_put(y, base + j, a.py, a.M * a.K, qlayer_code(a, v[j]));
+        }
+    } else if (a.out_mode == FXPQ_OUT_ACC64) {
+        long long* y = static_cast<long long*>(a.y) + m * a.K + k0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (k0 + j < a.K) y[j] = v[j];
+    } else {
+        float* y = static_cast<float*>(a.y) + m * a.K + k0;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (k0 + j < a.K) y[j] = __ll2float_rn(v[j]) * a.f32_scale;
+    }
+}
+
 // ------------------------------------------------------------------ kernel
 template <int BN, typename ACC>
 __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
     constexpr int B_BYTES = BN * TC_BK * 2;
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
+    // two fp32 accumulator buffers + integer running sums, rounded up to a power of two
+    constexpr uint32_t USED_COLS = 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
+    constexpr uint32_t TMEM_COLS = USED_COLS <= 256 ? 256u : 512u;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     unsigned char* sA = base;
@@ -192,7 +264,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     }
     if (warp == 8) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(2 * BN));
+                     "r"(TMEM_COLS));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     tc_fence_before();
@@ -276,38 +348,60 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
         const int row = quad * 32 + lane;
         uint32_t gcount = 0;
         bool ok = true;
+        // Integer running sums of a tile live in TMEM columns [2 BN, 2 BN + BN * words), words = 1
+        // (int32) or 2 (int64 as lo / hi column blocks), so the drain keeps few registers.
+        const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
+        const uint32_t run_col = 2 * BN;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            ACC run[BN];
-#pragma unroll
-            for (int j = 0; j < BN; ++j) run[j] = 0;
+            const long long m = (long long)tm * TC_BM + row;
             for (int gi = 0; gi < P.n_groups; ++gi) {
                 const int shift = P.g[gi].shift;
+                const bool first = gi == 0, last = gi == P.n_groups - 1;
                 const uint32_t buf = gcount & 1;
                 if (!wait_bounded(accfull0 + 8 * buf, (gcount >> 1) & 1, abort, P.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-#pragma unroll
+#pragma unroll 1
                 for (int cb = 0; cb < BN / 32; ++cb) {
-                    float v[32];
-                    tmem_ld32(tmem + ((uint32_t)(quad * 32) << 16) + buf * BN + cb * 32, v);
+                    float f[32];
+                    tmem_ld32(lane_base + buf * BN + cb * 32, f);
+                    ACC acc[32];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) run[cb * 32 + j] += ((ACC)__float2int_rn(v[j])) << shift;
+                    for (int j = 0; j < 32; ++j) acc[j] = ((ACC)__float2int_rn(f[j])) << shift;
+                    if (!first) {
+                        uint32_t lo[32];
+                        tmem_ld32u(lane_base + run_col + cb * 32, lo);
+                        if (sizeof(ACC) == 8) {
+                            uint32_t hi[32];
+                            tmem_ld32u(lane_base + run_col + BN + cb * 32, hi);
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
+                        }
+                    }
+                    if (last) {
+                        if (m < a.M) epilogue_block32<ACC>(a, m, tn * BN + cb * 32, acc);
+                    } else {
+                        uint32_t lo[32];
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) lo[j] = (uint32_t)(unsigned long long)acc[j];
+                        tmem_st32u(lane_base + run_col + cb * 32, lo);
+                        if (sizeof(ACC) == 8) {
+                            uint32_t hi[32];
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) hi[j] = (uint32_t)((unsigned long long)acc[j] >> 32);
+                            tmem_st32u(lane_base + run_col + BN + cb * 32, hi);
+                        }
+                    }
                 }
                 tc_fence_before();
                 mbar_arrive(accempty0 + 8 * buf);
                 ++gcount;
-            }
-            if (!ok) break;
-            const long long m = (long long)tm * TC_BM + row;
-            if (m < a.M) {
-#pragma unroll
-                for (int j = 0; j < BN; ++j) {
-                    const int k = tn * BN + j;
-                    if (k < a.K) cblock_epilogue_store(a, m, k, (long long)run[j]);
-                }
             }
         }
     } else if (lane == 0) {
@@ -354,7 +448,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     __syncthreads();
     if (warp == 8) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS));
     }
 }
 
