@@ -292,8 +292,57 @@ def run_reference(args):
     }))
 
 
+def run_kernel(args):
+    """Single-kernel timing cases (also the targets of the ncu captures summarised in profiles/):
+    conv     : VGG-16 conv3_1-shaped C-Block, batch 64, 56x56x128 -> 256, 3x3 pad 1, 8-bit codes;
+    flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid."""
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    from paper_2203_12091_gb300 import fxpq as F
+    out = {}
+    if args.kernel in ("conv", "all"):
+        N, H, C, K = 64, 56, 128, 256
+        rng = np.random.default_rng(0)
+        x = torch.from_numpy(rng.integers(0, 256, size=(N, H, H, C)).astype(np.float16)).cuda()
+        w = torch.from_numpy((rng.integers(-128, 128, size=(K, 3, 3, C)) // 4).astype(np.float16)).cuda()
+        b = torch.from_numpy(rng.integers(-2 ** 15, 2 ** 15, size=K).astype(np.int32)).cuda()
+        y = torch.empty(N * H * H * K, dtype=torch.float16, device="cuda")
+        d = F.conv_desc(N, H, H, C, C, K, 3, 3, 1, 1, 1, F.OUT_CODES, F.fmt(8, 0, 4), F.fmt(8, 1, 8),
+                        F.fmt(16, 1, 18), F.fmt(8, 0, 3))
+        ts = []
+        for i in range(args.warmup + args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            F.fxpq_conv_fwd(d, x, w, b, y)
+            e1.record()
+            e1.synchronize()
+            if i >= args.warmup:
+                ts.append(e0.elapsed_time(e1))
+        ms = sum(ts) / len(ts)
+        out["conv"] = {"ms": round(ms, 4), "tflops": round(2 * N * H * H * K * C * 9 / (ms / 1e3) / 1e12, 2)}
+    if args.kernel in ("flsearch", "all"):
+        n = 1 << 26
+        x = torch.from_numpy(synth.normal(n, 2)).cuda()
+        for name, (klo, khi) in (("flsearch_k8", (8, 8)), ("flsearch_sweep", (2, 16))):
+            ts = []
+            for i in range(args.warmup + args.steps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                F.fl_search(x, -1, klo, khi, -8, 23)
+                e1.record()
+                e1.synchronize()
+                if i >= args.warmup:
+                    ts.append(e0.elapsed_time(e1))
+            ms = sum(ts) / len(ts)
+            out[name] = {"ms": round(ms, 4), "gelem_s": round(n / (ms / 1e3) / 1e9, 2),
+                         "hbm_gbs": round(4 * n / (ms / 1e3) / 1e9, 1)}
+    print(json.dumps({"kernel_timing": out}))
+
+
 def main():
     ap = argparse.ArgumentParser()
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "all"], help="time one kernel case and exit")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
@@ -301,7 +350,9 @@ def main():
     ap.add_argument("--workload", default="vgg16", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline leg")
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.kernel:
+        run_kernel(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_fxpq(args)

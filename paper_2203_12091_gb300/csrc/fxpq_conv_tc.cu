@@ -30,8 +30,8 @@ namespace {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
-constexpr int TC_STAGES = 4;
-constexpr int TC_LAG = 2;  // producer arrives on a stage two k-blocks after issuing it
+constexpr int TC_STAGES = 6;
+constexpr int TC_LAG = 3;  // producer arrives on a stage three k-blocks after issuing it
 constexpr int TC_THREADS = 288;
 constexpr int TC_MAX_GROUPS = 64;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
@@ -274,26 +274,34 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
 
     if (warp < 4) {
         // ============================================================ producers
-        const int row = threadIdx.x;  // 0..127: one A row and (row < BN) one B row per stage
+        // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
+        // threads cover one 128-byte row, so every warp instruction reads four whole rows.
+        const int c = threadIdx.x & 7;
+        const int r0 = threadIdx.x >> 3;  // 0..15
+        constexpr int AR = TC_BM / 16;    // A rows per thread
+        constexpr int BR = BN / 16;       // B rows per thread
         const __half* xb = a.x;
         const __half* wb = a.w;
         uint32_t it = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            const long long m = (long long)tm * TC_BM + row;
-            const bool mvalid = m < a.M;
-            const long long mm = mvalid ? m : 0;
-            const int n_img = (int)(mm / ((long long)a.P * a.Q));
-            const int pq = (int)(mm - (long long)n_img * a.P * a.Q);
-            const int p0 = (pq / a.Q) * a.stride - a.pad, q0 = (pq % a.Q) * a.stride - a.pad;
-            const int kout = tn * BN + row;
-            const bool brow = row < BN;
-            const bool kvalid = brow && kout < a.K;
+            int n_img[AR], p0[AR], q0[AR];
+            bool mvalid[AR];
+#pragma unroll
+            for (int i = 0; i < AR; ++i) {
+                const long long m = (long long)tm * TC_BM + r0 + 16 * i;
+                mvalid[i] = m < a.M;
+                const long long mm = mvalid[i] ? m : 0;
+                n_img[i] = (int)(mm / ((long long)a.P * a.Q));
+                const int pq = (int)(mm - (long long)n_img[i] * a.P * a.Q);
+                p0[i] = (pq / a.Q) * a.stride - a.pad;
+                q0[i] = (pq % a.Q) * a.stride - a.pad;
+            }
             for (int gi = 0; gi < P.n_groups && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const __half* xp = xb + (long long)g.a_plane * a.x_ps;
-                const __half* wp = wb + (long long)g.w_plane * a.w_ps + (long long)(kvalid ? kout : 0) * P.RSC;
+                const __half* wp = wb + (long long)g.w_plane * a.w_ps;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
                     const int stage = it % TC_STAGES;
                     const uint32_t ph = (it / TC_STAGES) & 1;
@@ -301,32 +309,28 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                         ok = false;
                         break;
                     }
-                    const uint32_t dA = smem_u32(sA + stage * A_BYTES) + row * 128;
-                    const uint32_t dB = smem_u32(sB + stage * B_BYTES) + row * 128;
-                    const int f0 = kb * TC_BK;
-                    int tap = 0, c0 = 0;
-                    if (P.cp64) {
-                        tap = f0 / a.Cp;
-                        c0 = f0 - tap * a.Cp;
+                    const uint32_t dA = smem_u32(sA + stage * A_BYTES);
+                    const uint32_t dB = smem_u32(sB + stage * B_BYTES);
+                    const int f = kb * TC_BK + 8 * c;  // this thread's chunk of the flattened (r, s, c) index
+                    const bool fvalid = f < P.RSC;
+                    const int tp = f / a.Cp;
+                    const int cc = f - tp * a.Cp;
+                    const int rr = tp / a.S, ss = tp - rr * a.S;
+#pragma unroll
+                    for (int i = 0; i < AR; ++i) {
+                        const int row = r0 + 16 * i;
+                        const int h = p0[i] + rr, w = q0[i] + ss;
+                        const bool v = mvalid[i] && fvalid && h >= 0 && h < a.H && w >= 0 && w < a.W;
+                        const __half* src = v ? xp + (((long long)n_img[i] * a.H + h) * a.W + w) * a.Cp + cc : xb;
+                        cp_async16(dA + row * 128 + (uint32_t)((c ^ (row & 7)) << 4), src, v ? 16u : 0u);
                     }
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        const int f = f0 + 8 * c;
-                        int tp = tap, cc = c0 + 8 * c;
-                        if (!P.cp64) {
-                            tp = f / a.Cp;
-                            cc = f - tp * a.Cp;
-                        }
-                        const int r = tp / a.S, s = tp - (tp / a.S) * a.S;
-                        const int h = p0 + r, w = q0 + s;
-                        const bool v = mvalid && f < P.RSC && h >= 0 && h < a.H && w >= 0 && w < a.W;
-                        const __half* src = v ? xp + (((long long)n_img * a.H + h) * a.W + w) * a.Cp + cc : xb;
-                        const uint32_t sw = (uint32_t)((c ^ (row & 7)) << 4);
-                        cp_async16(dA + sw, src, v ? 16u : 0u);
-                        if (brow) {
-                            const bool vb = kvalid && f < P.RSC;
-                            cp_async16(dB + sw, vb ? (const void*)(wp + f) : (const void*)wb, vb ? 16u : 0u);
-                        }
+                    for (int i = 0; i < BR; ++i) {
+                        const int row = r0 + 16 * i;
+                        const int kout = tn * BN + row;
+                        const bool vb = fvalid && kout < a.K;
+                        const void* src = vb ? (const void*)(wp + (long long)kout * P.RSC + f) : (const void*)wb;
+                        cp_async16(dB + row * 128 + (uint32_t)((c ^ (row & 7)) << 4), src, vb ? 16u : 0u);
                     }
                     cp_async_commit();
                     if (it >= TC_LAG) {
