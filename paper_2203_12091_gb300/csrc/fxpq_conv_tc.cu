@@ -19,6 +19,7 @@
 //   warp  8    TMEM allocation and the single MMA-issuing thread.
 // Every wait is bounded: on expiry the kernel latches FXPQ_ERR_TIMEOUT, stops issuing work,
 // drains its own copies and MMAs, frees TMEM and returns.
+#include <cuda.h>  // CUtensorMap and its enums (the encoder is fetched through the runtime)
 #include <mutex>
 
 #include "fxpq_common.cuh"
@@ -43,6 +44,7 @@ struct TcGroup {
 };
 
 struct TcParams {
+    CUtensorMap tmap_w;  // weights as [planes][K][R*S*Cp] fp16, box {64, BN, 1}, 128-byte swizzle
     ConvArgs a;
     int RSC;       // R * S * Cp: reduction length of one plane
     int tiles_m, tiles_n, n_tiles;
@@ -75,6 +77,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+// 3-D tiled TMA load (coordinates innermost first) completing on mbarrier `bar`.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
 }
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
@@ -251,7 +266,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < TC_STAGES; ++s) {
-            mbar_init(full0 + 8 * s, 128);
+            mbar_init(full0 + 8 * s, 128 + 1);  // 128 producer arrivals + the weight TMA's expect_tx
             mbar_init(empty0 + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -279,29 +294,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
         const int c = threadIdx.x & 7;
         const int r0 = threadIdx.x >> 3;  // 0..15
         constexpr int AR = TC_BM / 16;    // A rows per thread
-        constexpr int BR = BN / 16;       // B rows per thread
         const __half* xb = a.x;
-        const __half* wb = a.w;
         uint32_t it = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            int n_img[AR], p0[AR], q0[AR];
-            bool mvalid[AR];
+            long long rowoff[AR];  // element offset of the (r, s) = (0, 0) tap of each row (may be negative)
+            int p0[AR], q0[AR];
 #pragma unroll
             for (int i = 0; i < AR; ++i) {
                 const long long m = (long long)tm * TC_BM + r0 + 16 * i;
-                mvalid[i] = m < a.M;
-                const long long mm = mvalid[i] ? m : 0;
-                n_img[i] = (int)(mm / ((long long)a.P * a.Q));
-                const int pq = (int)(mm - (long long)n_img[i] * a.P * a.Q);
+                const long long mm = m < a.M ? m : 0;
+                const int n_img = (int)(mm / ((long long)a.P * a.Q));
+                const int pq = (int)(mm - (long long)n_img * a.P * a.Q);
                 p0[i] = (pq / a.Q) * a.stride - a.pad;
                 q0[i] = (pq % a.Q) * a.stride - a.pad;
+                if (m >= a.M) p0[i] = -(1 << 20);  // rows past the end read zeros
+                rowoff[i] = (((long long)n_img * a.H + p0[i]) * a.W + q0[i]) * a.Cp;
             }
             for (int gi = 0; gi < P.n_groups && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const __half* xp = xb + (long long)g.a_plane * a.x_ps;
-                const __half* wp = wb + (long long)g.w_plane * a.w_ps;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
                     const int stage = it % TC_STAGES;
                     const uint32_t ph = (it / TC_STAGES) & 1;
@@ -310,27 +323,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                         break;
                     }
                     const uint32_t dA = smem_u32(sA + stage * A_BYTES);
-                    const uint32_t dB = smem_u32(sB + stage * B_BYTES);
+                    if (threadIdx.x == 0) {  // the weight tile: one TMA, zero-filled past K and R*S*Cp
+                        mbar_arrive_expect_tx(full0 + 8 * stage, (uint32_t)B_BYTES);
+                        tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, kb * TC_BK, tn * BN, g.w_plane,
+                                    full0 + 8 * stage);
+                    }
                     const int f = kb * TC_BK + 8 * c;  // this thread's chunk of the flattened (r, s, c) index
                     const bool fvalid = f < P.RSC;
                     const int tp = f / a.Cp;
                     const int cc = f - tp * a.Cp;
                     const int rr = tp / a.S, ss = tp - rr * a.S;
+                    const long long toff = ((long long)rr * a.W + ss) * a.Cp + cc;
 #pragma unroll
                     for (int i = 0; i < AR; ++i) {
                         const int row = r0 + 16 * i;
                         const int h = p0[i] + rr, w = q0[i] + ss;
-                        const bool v = mvalid[i] && fvalid && h >= 0 && h < a.H && w >= 0 && w < a.W;
-                        const __half* src = v ? xp + (((long long)n_img[i] * a.H + h) * a.W + w) * a.Cp + cc : xb;
+                        const bool v = fvalid && (unsigned)h < (unsigned)a.H && (unsigned)w < (unsigned)a.W;
+                        const __half* src = v ? xp + rowoff[i] + toff : xb;
                         cp_async16(dA + row * 128 + (uint32_t)((c ^ (row & 7)) << 4), src, v ? 16u : 0u);
-                    }
-#pragma unroll
-                    for (int i = 0; i < BR; ++i) {
-                        const int row = r0 + 16 * i;
-                        const int kout = tn * BN + row;
-                        const bool vb = fvalid && kout < a.K;
-                        const void* src = vb ? (const void*)(wp + (long long)kout * P.RSC + f) : (const void*)wb;
-                        cp_async16(dB + row * 128 + (uint32_t)((c ^ (row & 7)) << 4), src, vb ? 16u : 0u);
                     }
                     cp_async_commit();
                     if (it >= TC_LAG) {
@@ -346,6 +356,17 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
         fence_proxy_async();
         const uint32_t first = it >= TC_LAG ? it - TC_LAG : 0;
         for (uint32_t j = first; j < it; ++j) mbar_arrive(full0 + 8 * (j % TC_STAGES));
+        if (threadIdx.x == 0) {
+            // Every weight TMA this thread issued has landed once its stage's phase completes (the MMA
+            // thread already waited for them unless the kernel aborted): bounded wait on the last ones.
+            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
+            for (uint32_t j = from; j < it; ++j) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
+                       clock64() - t0 < TC_WAIT_CYCLES) {
+                }
+            }
+        }
     } else if (warp < 8) {
         // ============================================================ epilogue
         const int quad = warp - 4;  // TMEM lane quadrant of this warp
@@ -507,12 +528,47 @@ bool plan_tc(const ConvArgs& a, const fxpq_conv_desc& d, TcParams& P, bool& acc6
     return ng > 0;
 }
 
+namespace {
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link-time driver dependency).
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    std::lock_guard<std::mutex> lk(g_tc_mu);
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+}  // namespace
+
 fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched) {
     launched = false;
     TcParams P;
     bool acc64 = false;
     if (!plan_tc(a, d, P, acc64)) return FXPQ_OK;
     const int BN = acc64 ? 64 : 128;
+    {
+        EncodeTiledFn enc = encode_tiled();
+        if (!enc) return FXPQ_OK;  // no tensor-map encoder: the CUDA-core kernel runs instead
+        const cuuint64_t dims[3] = {(cuuint64_t)P.RSC, (cuuint64_t)a.K, (cuuint64_t)a.pw};
+        const cuuint64_t strides[2] = {(cuuint64_t)P.RSC * 2, (cuuint64_t)a.K * P.RSC * 2};
+        const cuuint32_t box[3] = {(cuuint32_t)TC_BK, (cuuint32_t)BN, 1};
+        const cuuint32_t es[3] = {1, 1, 1};
+        if (enc(&P.tmap_w, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<__half*>(a.w), dims, strides, box, es,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return FXPQ_OK;
+    }
     P.tiles_m = (int)((a.M + TC_BM - 1) / TC_BM);
     P.tiles_n = (a.K + BN - 1) / BN;
     P.n_tiles = P.tiles_m * P.tiles_n;
