@@ -5,7 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/fxpq.h"
+#include "fxpq.h"
 
 namespace fxpq {
 

@@ -150,15 +150,17 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
             s = d.fmt_b.fl;
         }
     }
-    (void)vbound;
     a.s_out = s;
     a.has_bias = bias != nullptr;
+    a.v32 = 0;
     if (d.out_mode == FXPQ_OUT_CODES) {
         a.sh = s - d.fmt_y.fl;
         if (a.sh > 62) return FXPQ_ERR_RANGE;
         a.lo = qmin_of(d.fmt_y);
         a.hi = qmax_of(d.fmt_y);
         a.py = planes_of(d.fmt_y);
+        // the aligned value stays below 2^31 in magnitude and the shift is a plain right shift
+        a.v32 = (vbound < ldexp(1.0, 31) - 1.0 && a.sh >= 1 && a.sh <= 30) ? 1 : 0;
     } else {
         a.sh = 0;
         a.lo = a.hi = 0;

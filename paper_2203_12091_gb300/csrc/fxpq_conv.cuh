@@ -20,6 +20,7 @@ struct ConvArgs {
     int sh;            // FxP-QLayer right shift s_out - fl_y
     long long lo, hi;  // clip levels of fmt_y
     float f32_scale;   // 2^-s_out
+    int v32;           // 1: the aligned value and the FxP-QLayer fit 32-bit arithmetic (|v| < 2^31, 1 <= sh <= 30)
 };
 
 // Bias alignment (B << delta, or the accumulator shifted left when delta < 0) and ReLU: the C-Block
@@ -51,6 +52,19 @@ __device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
     }
     q = q < a.lo ? a.lo : (q > a.hi ? a.hi : q);
     return (int)q;
+}
+
+// The same two steps in 32-bit arithmetic, valid when a.v32 (the host checked |v| < 2^31 after the
+// alignment and 1 <= sh <= 30).  Round half to even: q = floor(v / 2^sh) rounds up iff the dropped
+// bits exceed half, or equal half with q odd -- i.e. iff rem + (q & 1) > half.
+__device__ __forceinline__ int qlayer_code32(const ConvArgs& a, int v, int32_t bias) {
+    if (a.has_bias) v = a.delta >= 0 ? v + (bias << a.delta) : (v << (-a.delta)) + bias;
+    if (a.relu) v = max(v, 0);
+    const int q = v >> a.sh;
+    const int rem = v & ((1 << a.sh) - 1);
+    int c = q + (((rem + (q & 1)) > (1 << (a.sh - 1))) ? 1 : 0);
+    c = max(c, (int)a.lo);
+    return min(c, (int)a.hi);
 }
 
 // Bias alignment, ReLU and the FxP-QLayer for one output value of row m, channel k.

@@ -45,6 +45,8 @@ struct TcGroup {
 
 struct TcParams {
     CUtensorMap tmap_w;  // weights as [planes][K][R*S*Cp] fp16, box {64, BN, 1}, 128-byte swizzle
+    CUtensorMap tmap_y;  // output codes as [M][K] fp16, box {64, 128}, 128-byte swizzle (fast_store)
+    int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
     ConvArgs a;
     int RSC;       // R * S * Cp: reduction length of one plane
     int tiles_m, tiles_n, n_tiles;
@@ -82,6 +84,18 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
+
+// 2-D tiled TMA store from shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void epi_barrier() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // 3-D tiled TMA load (coordinates innermost first) completing on mbarrier `bar`.
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
@@ -253,13 +267,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     unsigned char* sA = base;
     unsigned char* sB = base + TC_STAGES * A_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + TC_STAGES * B_BYTES);
+    unsigned char* sO = sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of [128 rows][64 codes]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2);
     // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
     volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
     const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + TC_STAGES);
     const uint32_t accfull0 = smem_u32(bars + 2 * TC_STAGES), accempty0 = smem_u32(bars + 2 * TC_STAGES + 2);
     const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
+    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by the 128 epilogue threads
+    const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const ConvArgs& a = P.a;
@@ -274,6 +291,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
             mbar_init(accempty0 + 8 * b, 128);
         }
         mbar_init(done_bar, 1);
+        mbar_init(stg_full, 128);
+        mbar_init(stg_free, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -377,6 +396,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
         // (int32) or 2 (int64 as lo / hi column blocks), so the drain keeps few registers.
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
         const uint32_t run_col = 2 * BN;
+        uint32_t u = 0;  // tiles written through the staging buffer so far
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             const long long m = (long long)tm * TC_BM + row;
@@ -389,6 +409,17 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                     break;
                 }
                 tc_fence_after();
+                if (last && P.fast_store && u > 0) {
+                    // the previous tile's TMA store must have read the staging buffer
+                    if (threadIdx.x == 128) {
+                        bulk_wait_read0();
+                        mbar_arrive(stg_free);
+                    }
+                    if (!wait_bounded(stg_free, (u - 1) & 1, abort, P.status)) {
+                        ok = false;
+                        break;
+                    }
+                }
 #pragma unroll 1
                 for (int cb = 0; cb < BN / 32; ++cb) {
                     float f[32];
@@ -409,7 +440,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                             for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
                         }
                     }
-                    if (last) {
+                    if (last && P.fast_store) {
+                        // 32 codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
+                        const int k0 = tn * BN + cb * 32;
+                        uint32_t w[16];
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int k = k0 + 2 * j;
+                            const int32_t b0 = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                            const int32_t b1 = (a.has_bias && k + 1 < a.K) ? __ldg(a.bias + k + 1) : 0;
+                            const __half h0 = __int2half_rn(qlayer_code32(a, (int)acc[2 * j], b0));
+                            const __half h1 = __int2half_rn(qlayer_code32(a, (int)acc[2 * j + 1], b1));
+                            w[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+                        }
+                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int chunk = (cb & 1) * 4 + q;
+                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                        }
+                    } else if (last) {
                         if (m < a.M) epilogue_block32<ACC>(a, m, tn * BN + cb * 32, acc);
                     } else {
                         uint32_t lo[32];
@@ -427,8 +478,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                 tc_fence_before();
                 mbar_arrive(accempty0 + 8 * buf);
                 ++gcount;
+                if (last && P.fast_store) {
+                    // make the staging writes visible to the async proxy, then one thread stores the tile
+                    fence_proxy_async();
+                    mbar_arrive(stg_full);
+                    if (threadIdx.x == 128) {
+                        if (!wait_bounded(stg_full, u & 1, abort, P.status)) {
+                            ok = false;
+                            break;
+                        }
+                        for (int hb = 0; hb < BN / 64; ++hb)
+                            tma_store_2d(&P.tmap_y, tn * BN + hb * 64, tm * TC_BM, smem_u32(sO + hb * (TC_BM * 128)));
+                        bulk_commit();
+                    }
+                    ++u;
+                }
             }
         }
+        if (threadIdx.x == 128) bulk_wait0();  // every output store has completed
     } else if (lane == 0) {
         // ============================================================ MMA issue (one thread)
         uint32_t it = 0, gcount = 0;
@@ -483,7 +550,7 @@ bool g_tc_attr_set[2] = {false, false};
 
 template <int BN>
 constexpr size_t tc_smem_bytes() {
-    return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + 256;
+    return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
 }
 
 // Largest |limb| of a format's codes: the only plane (k <= 8) or the hi / lo limb (k > 8).
@@ -568,6 +635,17 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
+        // one-plane codes with a 32-bit epilogue: stage the tile and write it with TMA stores
+        P.fast_store = 0;
+        if (a.out_mode == FXPQ_OUT_CODES && a.py == 1 && a.v32) {
+            const cuuint64_t ydims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
+            const cuuint64_t ystrides[1] = {(cuuint64_t)a.K * 2};
+            const cuuint32_t ybox[2] = {64, (cuuint32_t)TC_BM};
+            if (enc(&P.tmap_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.y, ydims, ystrides, ybox, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
+                P.fast_store = 1;
+        }
     }
     P.tiles_m = (int)((a.M + TC_BM - 1) / TC_BM);
     P.tiles_n = (a.K + BN - 1) / BN;
