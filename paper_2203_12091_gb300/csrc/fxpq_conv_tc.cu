@@ -449,8 +449,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                             const int k = k0 + 2 * j;
                             const int32_t b0 = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
                             const int32_t b1 = (a.has_bias && k + 1 < a.K) ? __ldg(a.bias + k + 1) : 0;
-                            const __half h0 = __int2half_rn(qlayer_code32(a, (int)acc[2 * j], b0));
-                            const __half h1 = __int2half_rn(qlayer_code32(a, (int)acc[2 * j + 1], b1));
+                            int c0, c1;
+                            if (a.v32) {
+                                c0 = qlayer_code32(a, (int)acc[2 * j], b0);
+                                c1 = qlayer_code32(a, (int)acc[2 * j + 1], b1);
+                            } else {
+                                c0 = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j], b0));
+                                c1 = qlayer_code(a, cblock_value(a, k + 1, (long long)acc[2 * j + 1], b1));
+                            }
+                            const __half h0 = __int2half_rn(c0);
+                            const __half h1 = __int2half_rn(c1);
                             w[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
                         }
                         unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
@@ -635,9 +643,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
-        // one-plane codes with a 32-bit epilogue: stage the tile and write it with TMA stores
+        // one-plane codes: stage the tile in shared memory and write it with TMA stores
         P.fast_store = 0;
-        if (a.out_mode == FXPQ_OUT_CODES && a.py == 1 && a.v32) {
+        if (a.out_mode == FXPQ_OUT_CODES && a.py == 1) {
             const cuuint64_t ydims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
             const cuuint64_t ystrides[1] = {(cuuint64_t)a.K * 2};
             const cuuint32_t ybox[2] = {64, (cuuint32_t)TC_BM};
