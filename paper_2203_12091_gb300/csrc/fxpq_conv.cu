@@ -159,8 +159,15 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
         a.lo = qmin_of(d.fmt_y);
         a.hi = qmax_of(d.fmt_y);
         a.py = planes_of(d.fmt_y);
-        // the aligned value stays below 2^31 in magnitude and the shift is a plain right shift
-        a.v32 = (vbound < ldexp(1.0, 31) - 1.0 && a.sh >= 1 && a.sh <= 30) ? 1 : 0;
+        // 32-bit path: N = acc + aligned integer part of the bias stays below 2^31 in magnitude and the
+        // FxP-QLayer is a right shift by 1..30 bits of N (see qlayer_code32)
+        const double two31 = ldexp(1.0, 31) - 1.0;
+        const double bb = bias ? ldexp(1.0, d.fmt_b.bits - d.fmt_b.is_signed) : 0.0;
+        const int s_acc = d.fmt_x.fl + d.fmt_w.fl;
+        a.bsh = a.delta;
+        a.sh32 = s_acc - d.fmt_y.fl;
+        const double nbound = bound + (a.delta >= 0 ? bb * ldexp(1.0, a.delta) : bb * ldexp(1.0, a.delta) + 1.0);
+        a.v32 = (nbound < two31 && a.sh32 >= 1 && a.sh32 <= 30 && a.delta >= -30 && a.delta <= 30) ? 1 : 0;
     } else {
         a.sh = 0;
         a.lo = a.hi = 0;

@@ -20,7 +20,9 @@ struct ConvArgs {
     int sh;            // FxP-QLayer right shift s_out - fl_y
     long long lo, hi;  // clip levels of fmt_y
     float f32_scale;   // 2^-s_out
-    int v32;           // 1: the aligned value and the FxP-QLayer fit 32-bit arithmetic (|v| < 2^31, 1 <= sh <= 30)
+    int v32;           // 1: qlayer_code32 applies (the host checked its 32-bit bounds)
+    int bsh;           // bias shift of the 32-bit path (= delta)
+    int sh32;          // right shift of the 32-bit path, relative to the accumulator's scale
 };
 
 // Bias alignment (B << delta, or the accumulator shifted left when delta < 0) and ReLU: the C-Block
@@ -54,16 +56,35 @@ __device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
     return (int)q;
 }
 
-// The same two steps in 32-bit arithmetic, valid when a.v32 (the host checked |v| < 2^31 after the
-// alignment and 1 <= sh <= 30).  Round half to even: q = floor(v / 2^sh) rounds up iff the dropped
-// bits exceed half, or equal half with q odd -- i.e. iff rem + (q & 1) > half.
-__device__ __forceinline__ int qlayer_code32(const ConvArgs& a, int v, int32_t bias) {
-    if (a.has_bias) v = a.delta >= 0 ? v + (bias << a.delta) : (v << (-a.delta)) + bias;
-    if (a.relu) v = max(v, 0);
-    const int q = v >> a.sh;
-    const int rem = v & ((1 << a.sh) - 1);
-    int c = q + (((rem + (q & 1)) > (1 << (a.sh - 1))) ? 1 : 0);
-    c = max(c, (int)a.lo);
+// Bias alignment, ReLU and the FxP-QLayer in 32-bit arithmetic (valid when a.v32; the host checked
+// the bounds).  The value, in units of 2^-s (s = fl_x + fl_w), is acc + B 2^-delta:
+//   delta >= 0 (bsh = delta):   N = acc + (B << delta), phi = 0;
+//   delta <  0 (bsh = delta):   N = acc + floor(B / 2^d), phi = (B mod 2^d) / 2^d in [0, 1), d = -delta;
+// and the code is round_half_even((N + phi) / 2^sh32) with sh32 = s - fl_y >= 1.  Because
+// 0 <= phi < 1, floor((N + phi) / 2^sh32) = N >> sh32, and against half = 2^(sh32-1) the remainder
+// (N mod 2^sh32) + phi is above half iff rem > half or (rem == half and phi > 0), a tie iff
+// rem == half and phi == 0.  ReLU: N + phi < 0 iff N < 0.
+__device__ __forceinline__ int qlayer_code32(const ConvArgs& a, int acc, int32_t bias) {
+    int N = acc;
+    bool phi = false;
+    if (a.has_bias) {
+        if (a.bsh >= 0) {
+            N += bias << a.bsh;
+        } else {
+            const int d = -a.bsh;
+            N += bias >> d;
+            phi = (bias & ((1 << d) - 1)) != 0;
+        }
+    }
+    if (a.relu && N < 0) {
+        N = 0;
+        phi = false;
+    }
+    const int q = N >> a.sh32;
+    const int rem = N & ((1 << a.sh32) - 1);
+    const int half = 1 << (a.sh32 - 1);
+    const bool up = rem > half || (rem == half && (phi || (q & 1)));
+    const int c = max(q + (up ? 1 : 0), (int)a.lo);
     return min(c, (int)a.hi);
 }
 

@@ -92,6 +92,11 @@ CASES = [
     (2, 8, 32, 16, 3, 2, 1, (8, 0, 6), (8, 1, 8), (16, 22), False, 2, None),
     (4, 7, 8, 8, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (4, 0, 20)),      # left-shift requant + saturate
     (1, 5, 3, 8, 3, 1, 1, (3, 1, 1), (3, 1, 2), (16, 10), True, 0, (2, 0, 0)),
+    # bias finer than the accumulator (delta < 0) on the 32-bit epilogue: fractional bias parts, ties
+    (2, 9, 16, 40, 3, 1, 1, (5, 1, 2), (4, 1, 3), (16, 9), False, 0, (6, 1, 1)),
+    (2, 9, 16, 40, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 19), True, 0, (8, 0, 6)),
+    (2, 7, 8, 16, 3, 1, 1, (3, 1, 0), (3, 1, 0), (16, 3), False, 0, (8, 1, -1)),
+    (3, 12, 64, 136, 3, 1, 1, (8, 0, 6), (8, 1, 9), (16, 24), True, 0, (8, 0, 12)),
 ]
 
 
