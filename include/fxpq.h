@@ -199,6 +199,15 @@ FXPQ_API fxpq_status fxpq_eltwise(const void* d_a, fxpq_fmt fmt_a, const void* d
                          int32_t Cp, int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y,
                          int32_t* h_out_scale, void* stream);
 
+/* FxP-QLayer (Sec. IV-A.2 and the requantization paragraph of Sec. IV-B) as a standalone op: n int64
+ * C-Block values v with scale 2^-s (e.g. the ACC64 output of fxpq_conv_fwd) become
+ *   out_mode CODES: round_half_even(v * 2^(fl_y - s)) clipped to fmt_y, as an fp16 code tensor of n
+ *                   codes (plane-major when fmt_y.bits > 8);
+ *   out_mode F32  : the fp32 nearest-even image of v * 2^-s;  ACC64: a copy of v.
+ * -64 <= s <= 80. */
+FXPQ_API fxpq_status fxpq_qlayer(const int64_t* d_v, int64_t n, int32_t s, int32_t out_mode, fxpq_fmt fmt_y,
+                                 void* d_y, void* stream);
+
 /* Global AVG-POOL (Sec. IV-A.2: the reciprocal of the patch size is quantized like a parameter):
  * v[n,c] = recip_code * sum_{h,w} X[n,h,w,c], scale fl_x + fmt_recip.fl, then the FxP-QLayer to
  * fmt_y (or F32 / ACC64).  Output NHWC with H = W = 1. */

@@ -65,6 +65,7 @@ _SIGS = {
     "fxpq_maxpool": (I32, [VP, I32, I32, I32, I32, Fmt, I32, I32, I32, VP, VP]),
     "fxpq_eltwise": (I32, [VP, Fmt, VP, Fmt, I64, I32, I32, I32, Fmt, VP, ctypes.POINTER(I32), VP]),
     "fxpq_avgpool": (I32, [VP, I32, I32, I32, I32, Fmt, I32, Fmt, I32, Fmt, VP, ctypes.POINTER(I32), VP]),
+    "fxpq_qlayer": (I32, [VP, I64, I32, I32, Fmt, VP, VP]),
     "fxpq_net_workspace": (SZ, [ctypes.POINTER(Net), I32]),
     "fxpq_net_forward": (I32, [ctypes.POINTER(Net), VP, I32, VP, ctypes.POINTER(I32), VP, SZ, VP]),
     "fxpq_get_device_status": (I32, [VP]),

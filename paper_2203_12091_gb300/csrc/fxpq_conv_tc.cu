@@ -631,7 +631,8 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     TcParams P;
     bool acc64 = false;
     if (!plan_tc(a, d, P, acc64)) return FXPQ_OK;
-    const int BN = acc64 ? 64 : 128;
+    // 64-column tiles for int64 sums and for layers with at most 64 output channels
+    const int BN = (acc64 || a.K <= 64) ? 64 : 128;
     {
         EncodeTiledFn enc = encode_tiled();
         if (!enc) return FXPQ_OK;  // no tensor-map encoder: the CUDA-core kernel runs instead
@@ -670,18 +671,22 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
             if (g_num_sms <= 0) g_num_sms = 1;
         }
-        if (!g_tc_attr_set[acc64]) {
-            cudaError_t e = acc64 ? cudaFuncSetAttribute(conv_tc_kernel<64, long long>,
-                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<64>())
-                                  : cudaFuncSetAttribute(conv_tc_kernel<128, int>,
-                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<128>());
-            if (e != cudaSuccess) return FXPQ_ERR_CUDA;
-            g_tc_attr_set[acc64] = true;
+        if (!g_tc_attr_set[0]) {
+            if (cudaFuncSetAttribute(conv_tc_kernel<64, long long>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<64>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<64, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<64>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<128, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<128>()) != cudaSuccess)
+                return FXPQ_ERR_CUDA;
+            g_tc_attr_set[0] = true;
         }
     }
     const int grid = P.n_tiles < g_num_sms ? P.n_tiles : g_num_sms;
     if (acc64)
         conv_tc_kernel<64, long long><<<grid, TC_THREADS, tc_smem_bytes<64>(), st>>>(P);
+    else if (BN == 64)
+        conv_tc_kernel<64, int><<<grid, TC_THREADS, tc_smem_bytes<64>(), st>>>(P);
     else
         conv_tc_kernel<128, int><<<grid, TC_THREADS, tc_smem_bytes<128>(), st>>>(P);
     launched = true;

@@ -62,6 +62,42 @@ __global__ void maxpool_kernel(const __half* __restrict__ x, int N, int H, int W
     }
 }
 
+// One-plane codes: 8 channels per thread with 16-byte loads and stores.  The codes are exact
+// integers in fp16, so the half-precision max is exact.
+__global__ void maxpool_vec8_kernel(const uint4* __restrict__ x, int N, int H, int W, int C8, int k, int stride,
+                                    int pad, int P, int Q, uint4* __restrict__ y) {
+    const long long total = (long long)N * P * Q * C8;
+    const long long step = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += step) {
+        const int c8 = (int)(i % C8);
+        const long long pix = i / C8;
+        const int q = (int)(pix % Q);
+        const int p = (int)((pix / Q) % P);
+        const long long n = pix / ((long long)P * Q);
+        const __half2 ninf = __halves2half2(__ushort_as_half(0xFC00u), __ushort_as_half(0xFC00u));
+        __half2 m0 = ninf, m1 = ninf, m2 = ninf, m3 = ninf;
+        for (int r = 0; r < k; ++r) {
+            const int h = p * stride + r - pad;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < k; ++s) {
+                const int w = q * stride + s - pad;
+                if (w < 0 || w >= W) continue;
+                const uint4 v = __ldg(x + ((n * H + h) * W + w) * C8 + c8);
+                m0 = __hmax2(m0, *reinterpret_cast<const __half2*>(&v.x));
+                m1 = __hmax2(m1, *reinterpret_cast<const __half2*>(&v.y));
+                m2 = __hmax2(m2, *reinterpret_cast<const __half2*>(&v.z));
+                m3 = __hmax2(m3, *reinterpret_cast<const __half2*>(&v.w));
+            }
+        }
+        uint4 o;
+        o.x = *reinterpret_cast<uint32_t*>(&m0);
+        o.y = *reinterpret_cast<uint32_t*>(&m1);
+        o.z = *reinterpret_cast<uint32_t*>(&m2);
+        o.w = *reinterpret_cast<uint32_t*>(&m3);
+        y[i] = o;
+    }
+}
+
 __global__ void eltwise_kernel(const __half* __restrict__ a, int pa, int sa, const __half* __restrict__ b, int pb,
                                int sb, long long npix, int Cp, int relu, OutArgs o, void* y) {
     const long long total = npix * Cp;
@@ -73,6 +109,13 @@ __global__ void eltwise_kernel(const __half* __restrict__ a, int pa, int sa, con
         if (relu && v < 0) v = 0;
         store_out(o, y, pix, Cp, c, v, total);
     }
+}
+
+// FxP-QLayer on int64 C-Block values (scale 2^-s): codes (fp16 code tensor), int64 copy, or fp32 image.
+__global__ void qlayer_kernel(const long long* __restrict__ v, long long n, OutArgs o, void* y) {
+    const long long step = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += step)
+        store_out(o, y, i, 1, 0, v[i], n);
 }
 
 __global__ void avgpool_kernel(const __half* __restrict__ x, int N, int HW, int Cp, int planes, long long recip,
@@ -129,6 +172,11 @@ extern "C" fxpq_status fxpq_maxpool(const void* d_x, int32_t N, int32_t H, int32
     if (N == 0) return FXPQ_OK;
     if (!d_x || !d_y) return FXPQ_ERR_INVALID_ARG;
     const long long total = (long long)N * P * Q * Cp;
+    if (planes_of(fmt) == 1 && aligned(d_x, 16) && aligned(d_y, 16)) {
+        maxpool_vec8_kernel<<<grid_for(total / 8), 256, 0, as_stream(stream)>>>(
+            static_cast<const uint4*>(d_x), N, H, W, Cp / 8, k, stride, pad, P, Q, static_cast<uint4*>(d_y));
+        return after_launch("maxpool_vec8");
+    }
     maxpool_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(static_cast<const __half*>(d_x), N, H, W, Cp,
                                                                    planes_of(fmt), k, stride, pad, P, Q,
                                                                    static_cast<__half*>(d_y));
@@ -167,4 +215,16 @@ extern "C" fxpq_status fxpq_avgpool(const void* d_x, int32_t N, int32_t H, int32
     avgpool_kernel<<<grid_for((long long)N * Cp), 256, 0, as_stream(stream)>>>(
         static_cast<const __half*>(d_x), N, H * W, Cp, planes_of(fmt_x), (long long)recip_code, o, d_y);
     return after_launch("avgpool");
+}
+
+extern "C" fxpq_status fxpq_qlayer(const int64_t* d_v, int64_t n, int32_t s, int32_t out_mode, fxpq_fmt fmt_y,
+                                   void* d_y, void* stream) {
+    if (n < 0 || s < -64 || s > 80) return FXPQ_ERR_INVALID_ARG;
+    OutArgs o;
+    const fxpq_status st = make_out(out_mode, fmt_y, s, o, nullptr);
+    if (st != FXPQ_OK) return st;
+    if (n == 0) return FXPQ_OK;
+    if (!d_v || !d_y) return FXPQ_ERR_INVALID_ARG;
+    qlayer_kernel<<<grid_for(n), 256, 0, as_stream(stream)>>>(reinterpret_cast<const long long*>(d_v), n, o, d_y);
+    return after_launch("qlayer");
 }

@@ -135,6 +135,12 @@ def fxpq_avgpool(x, N, H, W, Cp, fx: Fmt, recip_code: int, fr: Fmt, out_mode, fy
     return scale.value
 
 
+def fxpq_qlayer(v, s: int, out_mode: int, fy, y, stream=None):
+    L.check("fxpq_qlayer", L.lib().fxpq_qlayer(_p(v), v.numel(), int(s), out_mode,
+                                               fy if fy is not None else Fmt(8, 1, 0), _p(y), _s(stream)))
+    return y
+
+
 def fxpq_net_workspace(net: L.Net, batch: int) -> int:
     return int(L.lib().fxpq_net_workspace(ctypes.byref(net), batch))
 

@@ -155,9 +155,20 @@ class QNet:
                 y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
                 env[nm] = (y, env[src][1])
                 continue
-            v, _ = self.run_layer(i, env, N, F.OUT_F32, stream)
-            self.fmts[nm]["a"] = search_fmt(v, plan[nm]["a"], stream)
-            y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
+            if L_["type"] == "conv":
+                # one contraction: exact C-Block values, then the FxP-QLayer twice (fp32 image for the
+                # FL search, then the codes in the chosen format)
+                acc, s = self.run_layer(i, env, N, F.OUT_ACC64, stream)
+                v = torch.empty(acc.numel(), dtype=torch.float32, device=self._dev)
+                F.fxpq_qlayer(acc, s, F.OUT_F32, None, v, stream)
+                fa = search_fmt(v, plan[nm]["a"], stream)
+                y = torch.empty(acc.numel() * F.planes(fa), dtype=torch.float16, device=self._dev)
+                F.fxpq_qlayer(acc, s, F.OUT_CODES, fa, y, stream)
+                self.fmts[nm]["a"] = fa
+            else:
+                v, _ = self.run_layer(i, env, N, F.OUT_F32, stream)
+                self.fmts[nm]["a"] = search_fmt(v, plan[nm]["a"], stream)
+                y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
             env[nm] = (y, self.fmts[nm]["a"])
         self._build_ops()
         return self.fmts

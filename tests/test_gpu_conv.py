@@ -173,6 +173,22 @@ def test_eltwise_parity(F, mode, fa, fb, relu):
         assert np.array_equal(y.cpu().numpy().reshape(npix, C), oracle.to_f32(v, ws))
 
 
+@pytest.mark.parametrize("s,fy", [(20, (8, 0, 6)), (11, (16, 1, 3)), (5, (4, 1, 9)), (30, (8, 1, 30)), (0, (6, 1, -2))])
+def test_qlayer_parity(F, s, fy):
+    rng = np.random.default_rng(s + 100)
+    v = rng.integers(-2 ** 40, 2 ** 40, size=1001)
+    v[:6] = [0, 1, -1, 3 << 9, -(3 << 9), 5 << 9]
+    vd = torch.from_numpy(v).cuda()
+    FY = F.fmt(*fy)
+    y = torch.empty(v.size * (2 if fy[0] > 8 else 1), dtype=torch.float16, device="cuda")
+    F.fxpq_qlayer(vd, s, F.OUT_CODES, FY, y)
+    assert np.array_equal(F.codes_to_int(y.cpu(), FY, (v.size,)).numpy(), oracle.requant(v, s, *fy))
+    small = v >> 12  # the fp32 image needs |v| < 2^53 on the oracle side
+    f = torch.empty(v.size, dtype=torch.float32, device="cuda")
+    F.fxpq_qlayer(torch.from_numpy(small).cuda(), s, F.OUT_F32, None, f)
+    assert np.array_equal(f.cpu().numpy(), oracle.to_f32(small, s))
+
+
 @pytest.mark.parametrize("bits", [5, 8, 11])
 def test_avgpool_parity(F, bits):
     rng = np.random.default_rng(bits)
