@@ -32,11 +32,39 @@ def pad8(c: int) -> int:
     return (c + 7) // 8 * 8
 
 
+def search_fmts(items, stream=None):
+    """FL searches at one wordlength each, launched back to back; one device-to-host read at the end.
+
+    items: list of (tensor, k).  Returns the chosen (k, S, FL) per item (sign strategy of Sec. IV-A.3)."""
+    if not items:
+        return []
+    dev = items[0][0].device
+    nfl = FL_HI - FL_LO + 1
+    stride = 64  # bytes per result record: int32 best FL at 0, fxpq_stats at 8
+    res = torch.empty(len(items) * stride, dtype=torch.uint8, device=dev)
+    err = torch.empty(len(items) * nfl, dtype=torch.float64, device=dev)
+    ws = F.workspace(F.fxpq_fl_search_workspace(0), dev)
+    lib = L.lib()
+    s = F._s(stream)
+    base = res.data_ptr()
+    for i, (x, k) in enumerate(items):
+        x = x.reshape(-1)
+        L.check("fxpq_fl_search", lib.fxpq_fl_search(
+            ctypes.c_void_p(x.data_ptr()), x.numel(), -1, k, k, FL_LO, FL_HI,
+            ctypes.c_void_p(err.data_ptr() + 8 * nfl * i), ctypes.c_void_p(base + stride * i),
+            ctypes.c_void_p(base + stride * i + 8), ctypes.c_void_p(ws.data_ptr()), ws.numel(), s))
+    host = bytes(res.cpu().numpy().tobytes())
+    out = []
+    for i, (_, k) in enumerate(items):
+        best = int.from_bytes(host[stride * i:stride * i + 4], "little", signed=True)
+        st = L.Stats.from_buffer_copy(host[stride * i + 8:stride * i + 8 + ctypes.sizeof(L.Stats)])
+        out.append(F.fmt(k, st.is_signed, best))
+    return out
+
+
 def search_fmt(x: torch.Tensor, k: int, stream=None) -> L.Fmt:
-    """FL search at one wordlength; returns the chosen (k, S, FL).  Synchronises (reads 16 bytes)."""
-    _, best, stats = F.fl_search(x.reshape(-1), -1, k, k, FL_LO, FL_HI, stream)
-    st = F.stats_from_device(stats)
-    return F.fmt(k, st.is_signed, int(best[0].item()))
+    """FL search at one wordlength; returns the chosen (k, S, FL).  Synchronises once."""
+    return search_fmts([(x, k)], stream)[0]
 
 
 class QNet:
@@ -58,8 +86,13 @@ class QNet:
         return s if s is not None else (self.names[i] if i > 0 else "input")
 
     def quantize_params(self, weights_dev, plan, stream=None):
-        """weights_dev: name -> (fp32 KRSC weight, fp32 bias) device tensors; plan: wordlengths."""
+        """weights_dev: name -> (fp32 KRSC weight, fp32 bias) device tensors; plan: wordlengths.
+
+        Every parameter's FL search is launched first (one read-back), then every quantization."""
         shapes = {"input": (self.hw, self.hw, self.cp_in)}
+        searches, owners = [], []
+        dev = next(iter(weights_dev.values()))[0].device
+        recips = {}
         for i, L_ in enumerate(self.layers):
             nm = L_["name"]
             self.fmts.setdefault(nm, {})
@@ -68,14 +101,8 @@ class QNet:
                 w, b = weights_dev[nm]
                 K, R, _, C = w.shape
                 assert C <= Cp
-                fw = search_fmt(w, plan[nm]["w"], stream)
-                fb = search_fmt(b, plan[nm]["b"], stream)
-                wq = torch.empty(K * R * R, Cp * F.planes(fw), dtype=torch.float16, device=w.device)
-                F.fxpq_quantize_rows(w.reshape(-1, C), K * R * R, C, fw, Cp, wq, stream)
-                bq = torch.empty(K, dtype=torch.int32, device=w.device)
-                F.fxpq_quantize(b, fb, F.DT_I32, bq, stream)
-                self.fmts[nm]["w"], self.fmts[nm]["b"] = fw, fb
-                self.q[nm] = (wq, bq)
+                searches += [(w, plan[nm]["w"]), (b, plan[nm]["b"])]
+                owners += [(nm, "w"), (nm, "b")]
                 P = (H + 2 * L_["pad"] - R) // L_["stride"] + 1
                 shapes[nm] = (P, P, K)
             elif L_["type"] == "maxpool":
@@ -86,14 +113,32 @@ class QNet:
                 shapes[nm] = shapes[L_["a"]]
             elif L_["type"] == "avgpool":
                 H, W, Cp = shapes[self._src(i, L_)]
-                dev = next(iter(weights_dev.values()))[0].device
                 r = torch.tensor([1.0 / (H * W)], dtype=torch.float32, device=dev)
-                fr = search_fmt(r, plan[nm]["r"], stream)
-                rc = torch.empty(1, dtype=torch.int32, device=dev)
-                F.fxpq_quantize(r, fr, F.DT_I32, rc, stream)
-                self.fmts[nm]["r"] = fr
-                self.q[nm] = (None, int(rc.item()))
+                recips[nm] = r
+                searches.append((r, plan[nm]["r"]))
+                owners.append((nm, "r"))
                 shapes[nm] = (1, 1, Cp)
+        for (nm, key), f in zip(owners, search_fmts(searches, stream)):
+            self.fmts[nm][key] = f
+        rcodes = {}
+        for i, L_ in enumerate(self.layers):
+            nm = L_["name"]
+            if L_["type"] == "conv":
+                w, b = weights_dev[nm]
+                K, R, _, C = w.shape
+                Cp = shapes[self._src(i, L_)][2]
+                fw, fb = self.fmts[nm]["w"], self.fmts[nm]["b"]
+                wq = torch.empty(K * R * R * Cp * F.planes(fw), dtype=torch.float16, device=dev)
+                F.fxpq_quantize_rows(w.reshape(-1, C), K * R * R, C, fw, Cp, wq, stream)
+                bq = torch.empty(K, dtype=torch.int32, device=dev)
+                F.fxpq_quantize(b, fb, F.DT_I32, bq, stream)
+                self.q[nm] = (wq, bq)
+            elif L_["type"] == "avgpool":
+                rc = torch.empty(1, dtype=torch.int32, device=dev)
+                F.fxpq_quantize(recips[nm], self.fmts[nm]["r"], F.DT_I32, rc, stream)
+                rcodes[nm] = rc
+        for nm, rc in rcodes.items():
+            self.q[nm] = (None, int(rc.item()))
         self.shapes = shapes
 
     # ------------------------------------------------------------------ one C-Block on device tensors
