@@ -127,7 +127,7 @@ FXPQ_API fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_sign
  * enter the allocator (cudaMalloc may synchronise the device).  The paper has no counterpart: this
  * is a deployment variant of fxpq_fl_search with the same arguments, results and limits, minus
  * the workspace.  It allocates nothing.  Its scratch is a file-scope device array of about
- * 150 KiB inside libfxpq.so that every GPU which loads the library holds until the process exits.
+ * 53 KiB inside libfxpq.so that every GPU which loads the library holds until the process exits.
  *   - Limits: n <= 2^31 elements and at most 15 x 32 candidates (k in [2,16], fl_hi-fl_lo <= 31);
  *     larger requests return FXPQ_ERR_INVALID_ARG before any launch.
  *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
