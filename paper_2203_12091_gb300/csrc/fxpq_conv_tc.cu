@@ -11,15 +11,21 @@
 // (v = 256 * v_hi + v_lo): one pass per (A limb, W limb) pair.
 //
 // CTA (one per SM, persistent over tiles): 9 warps.
-//   warps 0-3  producers: cp.async gather of the A tile (128 pixels x 64 taps, with zero fill for
-//              padding and ragged edges) and of the B tile (BN channels x 64 taps) into 128-byte
-//              swizzled K-major shared-memory stages.
+//   warps 0-3  producers, into 128-byte swizzled K-major shared-memory stages.  The B tile
+//              (BN channels x 64 taps) always comes by TMA.  The A tile takes one of two forms:
+//              row tiles (128 consecutive output pixels): cp.async gather by 128 threads, with
+//              zero fill for padding and ragged edges;
+//              patch tiles (stride 1, Cp % 64 == 0): a TH x TW patch of output pixels of one
+//              image, whose input window for one tap and 64 channels is a single 5-D TMA box
+//              (the hardware zero-fills the padding); one thread issues both copies.
 //   warp  4-7  epilogue: drain TMEM (tcgen05.ld), integer running sums, final bias / ReLU /
 //              FxP-QLayer (shared with the CUDA-core kernel).
 //   warp  8    TMEM allocation and the single MMA-issuing thread.
 // Every wait is bounded: on expiry the kernel latches FXPQ_ERR_TIMEOUT, stops issuing work,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>  // CUtensorMap and its enums (the encoder is fetched through the runtime)
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 
 #include "fxpq_common.cuh"
@@ -33,7 +39,10 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
 constexpr int TC_STAGES = 6;
 constexpr int TC_LAG = 3;  // producer arrives on a stage three k-blocks after issuing it
-constexpr int TC_THREADS = 288;
+// Warps: 4 producers, BN / 8 epilogue warps (one 32-column chunk of one TMEM lane quadrant each),
+// one MMA / TMEM-allocation warp.
+__host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8; }
+__host__ __device__ constexpr int tc_threads(int BN) { return (5 + tc_epi_warps(BN)) * 32; }
 constexpr int TC_MAX_GROUPS = 64;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
 
@@ -45,8 +54,12 @@ struct TcGroup {
 
 struct TcParams {
     CUtensorMap tmap_w;  // weights as [planes][K][R*S*Cp] fp16, box {64, BN, 1}, 128-byte swizzle
-    CUtensorMap tmap_y;  // output codes as [M][K] fp16, box {64, 128}, 128-byte swizzle (fast_store)
+    CUtensorMap tmap_y;  // output codes: [M][K] box {64, 128} (linear tiles) or [N][P][Q][K] box {64, TW, TH, 1}
+    CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}
     int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
+    int patch;           // 1: a tile is a TH x TW patch of one image, the A tile comes by TMA
+    int TH, TW;          // patch shape (TH * TW = 128)
+    int tiles_p, tiles_q;  // patches per image along P and Q
     ConvArgs a;
     int RSC;       // R * S * Cp: reduction length of one plane
     int tiles_m, tiles_n, n_tiles;
@@ -95,7 +108,38 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int 
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void epi_barrier() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, int x, int y, int z, int w, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(z), "r"(w), "r"(src)
+                 : "memory");
+}
+
+// 5-D tiled TMA load completing on mbarrier `bar` (coordinates innermost first; out-of-range
+// positions, e.g. the convolution's padding, read as zero).
+__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
+                                            int c4, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
+        "%5, %6}], [%7];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar)
+        : "memory");
+}
+
+// Output row (linear index into N*P*Q, or -1 when outside the map) of tile row i.
+__device__ __forceinline__ long long tile_row(const TcParams& P, int tm, int i) {
+    if (!P.patch) {
+        const long long m = (long long)tm * 128 + i;
+        return m < P.a.M ? m : -1;
+    }
+    if (i >= P.TH * P.TW) return -1;
+    const int per_img = P.tiles_p * P.tiles_q;
+    const int n = tm / per_img, r = tm - n * per_img;
+    const int p = (r / P.tiles_q) * P.TH + i / P.TW, q = (r % P.tiles_q) * P.TW + i % P.TW;
+    if (p >= P.a.P || q >= P.a.Q) return -1;
+    return ((long long)n * P.a.P + p) * P.a.Q + q;
+}
 
 // 3-D tiled TMA load (coordinates innermost first) completing on mbarrier `bar`.
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
@@ -198,6 +242,26 @@ __device__ __forceinline__ void tmem_ld32u(uint32_t taddr, uint32_t (&r)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void tmem_ld16u(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t (&r)[32]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
@@ -211,52 +275,93 @@ __device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t (&r)[3
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// Final epilogue of 32 consecutive output channels k0.. of row m (16-byte stores when the block is
-// whole): bias alignment, ReLU, FxP-QLayer / int64 / fp32 image.
+// Final epilogue of 32 consecutive output channels k0.. of row m (generic outputs: two-plane codes,
+// int64 accumulators, fp32 calibration images): bias alignment, ReLU, FxP-QLayer.
 template <typename ACC>
 __device__ __forceinline__ void epilogue_block32(const ConvArgs& a, long long m, int k0, const ACC (&acc)[32]) {
-    const bool whole = k0 + 32 <= a.K;
-    long long v[32];
-#pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        const int k = k0 + j;
-        const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-        v[j] = cblock_value(a, k, (long long)acc[j], b);
-    }
     if (a.out_mode == FXPQ_OUT_CODES) {
         __half* y = static_cast<__half*>(a.y);
         const long long base = m * a.K + k0;
-        if (whole && a.py == 1) {
-            uint32_t w[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const __half h0 = __int2half_rn(qlayer_code(a, v[2 * j])), h1 = __int2half_rn(qlayer_code(a, v[2 * j + 1]));
-                w[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+        for (int j = 0; j < 32; ++j) {
+            const int k = k0 + j;
+            if (k < a.K) {
+                const int32_t b = a.has_bias ? __ldg(a.bias + k) : 0;
+                code_put(y, base + j, a.py, a.M * a.K, qlayer_code(a, cblock_value(a, k, (long long)acc[j], b)));
             }
-            uint4* dst = reinterpret_cast<uint4*>(y + base);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-        } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (k0 + j < a.K) code_put(y, base + j, a.py, a.M * a.K, qlayer_code(a, v[j]));
         }
     } else if (a.out_mode == FXPQ_OUT_ACC64) {
         long long* y = static_cast<long long*>(a.y) + m * a.K + k0;
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (k0 + j < a.K) y[j] = v[j];
+        for (int j = 0; j < 32; ++j) {
+            const int k = k0 + j;
+            if (k < a.K) y[j] = cblock_value(a, k, (long long)acc[j], a.has_bias ? __ldg(a.bias + k) : 0);
+        }
     } else {
         float* y = static_cast<float*>(a.y) + m * a.K + k0;
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (k0 + j < a.K) y[j] = __ll2float_rn(v[j]) * a.f32_scale;
+        for (int j = 0; j < 32; ++j) {
+            const int k = k0 + j;
+            if (k < a.K)
+                y[j] = __ll2float_rn(cblock_value(a, k, (long long)acc[j], a.has_bias ? __ldg(a.bias + k) : 0)) *
+                       a.f32_scale;
+        }
     }
+}
+
+// Uniform constants of the 32-bit FxP-QLayer epilogue (the same arithmetic as qlayer_code32, with
+// the bias alignment split into a left and a right shift so that it has no branches).
+struct Epi32 {
+    int bsl, bsr, fmask;  // bias term (b << bsl) >> bsr; fraction bits b & fmask (bias finer than acc)
+    int sh, rmask, half;  // requantizing right shift, its remainder mask and half
+    int lo, hi;
+    int relu, has_bias;
+};
+
+__device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
+    Epi32 e;
+    e.bsl = a.bsh > 0 ? a.bsh : 0;
+    e.bsr = a.bsh < 0 ? -a.bsh : 0;
+    e.fmask = (1 << e.bsr) - 1;
+    e.sh = a.sh32;
+    e.rmask = (1 << a.sh32) - 1;
+    e.half = 1 << (a.sh32 - 1);
+    e.lo = (int)a.lo;
+    e.hi = (int)a.hi;
+    e.relu = a.relu;
+    e.has_bias = a.has_bias;
+    return e;
+}
+
+// One code: N = acc + aligned bias; ReLU; round half to even on the dropped bits (phi: the bias had
+// nonzero bits below the accumulator's scale, so a remainder of exactly one half is above the tie).
+__device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, bool phi) {
+    int N = acc + bterm;
+    if (e.relu && N < 0) {
+        N = 0;
+        phi = false;
+    }
+    const int q = N >> e.sh;
+    const int rem = N & e.rmask;
+    const bool up = rem > e.half || (rem == e.half && (phi || (q & 1)));
+    return min(max(q + (up ? 1 : 0), e.lo), e.hi);
+}
+
+// Two codes in [-512, 511] as a packed fp16 pair: 1536 + c has the bit pattern 0x6600 + c (the
+// binade [1024, 2048) has unit spacing), and one packed subtraction of 1536 leaves c exactly.
+__device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
+    const uint32_t bits = (uint32_t)(0x6600 + c0) | ((uint32_t)(0x6600 + c1) << 16);
+    const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&bits), __halves2half2(__ushort_as_half(0x6600),
+                                                                                        __ushort_as_half(0x6600)));
+    return *reinterpret_cast<const uint32_t*>(&h);
 }
 
 // ------------------------------------------------------------------ kernel
 template <int BN, typename ACC>
-__global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+__global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+    constexpr int EPI_WARPS = tc_epi_warps(BN);
+    constexpr int EPI_THREADS = 32 * EPI_WARPS;
+    constexpr int MMA_WARP = 4 + EPI_WARPS;
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
     constexpr int B_BYTES = BN * TC_BK * 2;
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
@@ -275,7 +380,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + TC_STAGES);
     const uint32_t accfull0 = smem_u32(bars + 2 * TC_STAGES), accempty0 = smem_u32(bars + 2 * TC_STAGES + 2);
     const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
-    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by the 128 epilogue threads
+    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue thread
     const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -283,20 +388,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < TC_STAGES; ++s) {
-            mbar_init(full0 + 8 * s, 128 + 1);  // 128 producer arrivals + the weight TMA's expect_tx
+            // patch tiles: one expect_tx arrival for both TMAs; row tiles: 128 producer arrivals +
+            // the weight TMA's expect_tx
+            mbar_init(full0 + 8 * s, P.patch ? 1 : 128 + 1);
             mbar_init(empty0 + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accfull0 + 8 * b, 1);
-            mbar_init(accempty0 + 8 * b, 128);
+            mbar_init(accempty0 + 8 * b, EPI_THREADS);
         }
         mbar_init(done_bar, 1);
-        mbar_init(stg_full, 128);
+        mbar_init(stg_full, EPI_THREADS);
         mbar_init(stg_free, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 8) {
+    if (warp == MMA_WARP) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                      "r"(TMEM_COLS));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
@@ -306,8 +413,50 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp < 4) {
-        // ============================================================ producers
+    if (warp < 4 && P.patch) {
+        // ============================================================ producer, patch tiles
+        // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
+        // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
+        if (threadIdx.x == 0) {
+            const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * 128);
+            const int per_img = P.tiles_p * P.tiles_q;
+            uint32_t it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+                const int tm = t / P.tiles_n, tn = t % P.tiles_n;
+                const int n_img = tm / per_img, r = tm - n_img * per_img;
+                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
+                for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+                    const TcGroup g = P.g[gi];
+                    for (int kb = g.kb0; kb < g.kb1; ++kb) {
+                        const int stage = it % TC_STAGES;
+                        if (!wait_bounded(empty0 + 8 * stage, ((it / TC_STAGES) & 1) ^ 1, abort, P.status)) {
+                            ok = false;
+                            break;
+                        }
+                        const int f = kb * TC_BK;
+                        const int tp = f / a.Cp, cc = f - tp * a.Cp;
+                        const int rr = tp / a.S, ss = tp - rr * a.S;
+                        const uint32_t fb = full0 + 8 * stage;
+                        mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
+                        tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
+                                    g.a_plane, fb);
+                        tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, f, tn * BN, g.w_plane, fb);
+                        ++it;
+                    }
+                }
+            }
+            // bounded wait until the copies of the last stages have landed
+            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
+            for (uint32_t j = from; j < it; ++j) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
+                       clock64() - t0 < TC_WAIT_CYCLES) {
+                }
+            }
+        }
+    } else if (warp < 4) {
+        // ============================================================ producers, row tiles
         // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
         // threads cover one 128-byte row, so every warp instruction reads four whole rows.
         const int c = threadIdx.x & 7;
@@ -386,20 +535,26 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                 }
             }
         }
-    } else if (warp < 8) {
+    } else if (warp < MMA_WARP) {
         // ============================================================ epilogue
-        const int quad = warp - 4;  // TMEM lane quadrant of this warp
+        // Warp w drains TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the quadrant a warp may access) and
+        // the 32-column chunk cb = (w - 4) / 4 of every accumulator.
+        const int quad = warp & 3;
+        const int cb = (warp - 4) >> 2;
         const int row = quad * 32 + lane;
+        const bool leader = threadIdx.x == 128;  // waits for and issues the tile's TMA stores
         uint32_t gcount = 0;
         bool ok = true;
         // Integer running sums of a tile live in TMEM columns [2 BN, 2 BN + BN * words), words = 1
         // (int32) or 2 (int64 as lo / hi column blocks), so the drain keeps few registers.
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
-        const uint32_t run_col = 2 * BN;
+        const uint32_t run_col = 2 * BN + cb * 32;
+        const Epi32 e32 = make_epi32(a);
         uint32_t u = 0;  // tiles written through the staging buffer so far
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            const long long m = (long long)tm * TC_BM + row;
+            const long long m = tile_row(P, tm, row);  // -1: row outside the output
+            const int k0 = tn * BN + cb * 32;
             for (int gi = 0; gi < P.n_groups; ++gi) {
                 const int shift = P.g[gi].shift;
                 const bool first = gi == 0, last = gi == P.n_groups - 1;
@@ -411,7 +566,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                 tc_fence_after();
                 if (last && P.fast_store && u > 0) {
                     // the previous tile's TMA store must have read the staging buffer
-                    if (threadIdx.x == 128) {
+                    if (leader) {
                         bulk_wait_read0();
                         mbar_arrive(stg_free);
                     }
@@ -420,92 +575,120 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
                         break;
                     }
                 }
-#pragma unroll 1
-                for (int cb = 0; cb < BN / 32; ++cb) {
+                ACC acc[32];
+                {
                     float f[32];
                     tmem_ld32(lane_base + buf * BN + cb * 32, f);
-                    ACC acc[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) acc[j] = ((ACC)__float2int_rn(f[j])) << shift;
-                    if (!first) {
-                        uint32_t lo[32];
-                        tmem_ld32u(lane_base + run_col + cb * 32, lo);
-                        if (sizeof(ACC) == 8) {
-                            uint32_t hi[32];
-                            tmem_ld32u(lane_base + run_col + BN + cb * 32, hi);
+                }
+                if (sizeof(ACC) == 8) {
+                    // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
-                        } else {
+                    for (int hf = 0; hf < 2; ++hf) {
+                        uint32_t lo[16], hi[16];
+                        if (!first) {
+                            tmem_ld16u(lane_base + run_col + 16 * hf, lo);
+                            tmem_ld16u(lane_base + run_col + BN + 16 * hf, hi);
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
+                            for (int j = 0; j < 16; ++j)
+                                acc[16 * hf + j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
+                        }
+                        if (!last) {
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                lo[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
+                                hi[j] = (uint32_t)((unsigned long long)acc[16 * hf + j] >> 32);
+                            }
+                            tmem_st16u(lane_base + run_col + 16 * hf, lo);
+                            tmem_st16u(lane_base + run_col + BN + 16 * hf, hi);
                         }
                     }
-                    if (last && P.fast_store) {
-                        // 32 codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
-                        const int k0 = tn * BN + cb * 32;
-                        uint32_t w[16];
+                } else {
+                    if (!first) {
+                        uint32_t lo[32];
+                        tmem_ld32u(lane_base + run_col, lo);
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            const int k = k0 + 2 * j;
-                            const int32_t b0 = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                            const int32_t b1 = (a.has_bias && k + 1 < a.K) ? __ldg(a.bias + k + 1) : 0;
-                            int c0, c1;
-                            if (a.v32) {
-                                c0 = qlayer_code32(a, (int)acc[2 * j], b0);
-                                c1 = qlayer_code32(a, (int)acc[2 * j + 1], b1);
-                            } else {
-                                c0 = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j], b0));
-                                c1 = qlayer_code(a, cblock_value(a, k + 1, (long long)acc[2 * j + 1], b1));
-                            }
-                            const __half h0 = __int2half_rn(c0);
-                            const __half h1 = __int2half_rn(c1);
-                            w[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-                        }
-                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int chunk = (cb & 1) * 4 + q;
-                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
-                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-                        }
-                    } else if (last) {
-                        if (m < a.M) epilogue_block32<ACC>(a, m, tn * BN + cb * 32, acc);
-                    } else {
+                        for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
+                    }
+                    if (!last) {
                         uint32_t lo[32];
 #pragma unroll
                         for (int j = 0; j < 32; ++j) lo[j] = (uint32_t)(unsigned long long)acc[j];
-                        tmem_st32u(lane_base + run_col + cb * 32, lo);
-                        if (sizeof(ACC) == 8) {
-                            uint32_t hi[32];
-#pragma unroll
-                            for (int j = 0; j < 32; ++j) hi[j] = (uint32_t)((unsigned long long)acc[j] >> 32);
-                            tmem_st32u(lane_base + run_col + BN + cb * 32, hi);
-                        }
+                        tmem_st32u(lane_base + run_col, lo);
                     }
                 }
+                // the accumulator buffer is free for the next group's MMAs
                 tc_fence_before();
                 mbar_arrive(accempty0 + 8 * buf);
                 ++gcount;
-                if (last && P.fast_store) {
+                if (!last) continue;
+                if (P.fast_store) {
+                    // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
+                    uint32_t w[16];
+                    if (sizeof(ACC) == 4 && a.v32) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            int c2[2];
+#pragma unroll
+                            for (int h = 0; h < 2; ++h) {
+                                const int k = k0 + 2 * j + h;
+                                const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
+                                                   (b & e32.fmask) != 0);
+                            }
+                            w[j] = pack_codes_f16(c2[0], c2[1]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            int c2[2];
+#pragma unroll
+                            for (int h = 0; h < 2; ++h) {
+                                const int k = k0 + 2 * j + h;
+                                const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                c2[h] = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j + h], b));
+                            }
+                            w[j] = pack_codes_f16(c2[0], c2[1]);
+                        }
+                    }
+                    unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int chunk = (cb & 1) * 4 + q;
+                        *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                            make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                    }
                     // make the staging writes visible to the async proxy, then one thread stores the tile
                     fence_proxy_async();
                     mbar_arrive(stg_full);
-                    if (threadIdx.x == 128) {
+                    if (leader) {
                         if (!wait_bounded(stg_full, u & 1, abort, P.status)) {
                             ok = false;
                             break;
                         }
-                        for (int hb = 0; hb < BN / 64; ++hb)
-                            tma_store_2d(&P.tmap_y, tn * BN + hb * 64, tm * TC_BM, smem_u32(sO + hb * (TC_BM * 128)));
+                        if (P.patch) {
+                            const int per_img = P.tiles_p * P.tiles_q;
+                            const int n_img = tm / per_img, r = tm - n_img * per_img;
+                            for (int hb = 0; hb < BN / 64; ++hb)
+                                tma_store_4d(&P.tmap_y, tn * BN + hb * 64, (r % P.tiles_q) * P.TW,
+                                             (r / P.tiles_q) * P.TH, n_img, smem_u32(sO + hb * (TC_BM * 128)));
+                        } else {
+                            for (int hb = 0; hb < BN / 64; ++hb)
+                                tma_store_2d(&P.tmap_y, tn * BN + hb * 64, tm * TC_BM,
+                                             smem_u32(sO + hb * (TC_BM * 128)));
+                        }
                         bulk_commit();
                     }
                     ++u;
+                } else if (m >= 0) {
+                    epilogue_block32<ACC>(a, m, k0, acc);
                 }
             }
         }
-        if (threadIdx.x == 128) bulk_wait0();  // every output store has completed
+        if (leader) bulk_wait0();  // every output store has completed
     } else if (lane == 0) {
-        // ============================================================ MMA issue (one thread)
+        // ============================================================ MMA issue (one thread of MMA_WARP)
         uint32_t it = 0, gcount = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
@@ -546,7 +729,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 8) {
+    if (warp == MMA_WARP) {
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS));
     }
@@ -554,6 +737,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) conv_tc_kernel(const __grid_con
 
 int g_num_sms = 0;
 std::mutex g_tc_mu;
+
+// FXPQ_CONV_PATH=tc_rows keeps every layer on 128-row tiles (both tilings are exact; the switch
+// lets tests compare them on the same shapes).
+bool patch_enabled() {
+    const char* e = getenv("FXPQ_CONV_PATH");
+    return !(e && strcmp(e, "tc_rows") == 0);
+}
 bool g_tc_attr_set[2] = {false, false};
 
 template <int BN>
@@ -644,19 +834,61 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
+        // patch tiles for stride-1 layers whose taps are whole 64-channel blocks
+        P.patch = 0;
+        if (a.stride == 1 && P.cp64 && a.P > 0 && a.Q > 0 && a.N > 0 && patch_enabled()) {
+            int best_tw = 0, best_th = 0;
+            long long best = 0;
+            for (int tw = a.Q < TC_BM ? a.Q : TC_BM; tw >= 1; --tw) {
+                const int th = TC_BM / tw < a.P ? TC_BM / tw : a.P;
+                const long long cost = (long long)((a.P + th - 1) / th) * ((a.Q + tw - 1) / tw);
+                if (best_tw == 0 || cost < best) best = cost, best_tw = tw, best_th = th;
+            }
+            // take patches unless they compute clearly more rows than 128-row tiles of N*P*Q would
+            const long long row_tiles = (a.M + TC_BM - 1) / TC_BM;
+            if ((double)a.N * best <= 1.15 * (double)row_tiles + 1e-9) {
+                const cuuint64_t xdims[5] = {(cuuint64_t)a.Cp, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N,
+                                             (cuuint64_t)a.px};
+                const cuuint64_t xstrides[4] = {(cuuint64_t)a.Cp * 2, (cuuint64_t)a.W * a.Cp * 2,
+                                                (cuuint64_t)a.H * a.W * a.Cp * 2, (cuuint64_t)a.x_ps * 2};
+                const cuuint32_t xbox[5] = {(cuuint32_t)TC_BK, (cuuint32_t)best_tw, (cuuint32_t)best_th, 1, 1};
+                const cuuint32_t es5[5] = {1, 1, 1, 1, 1};
+                if (enc(&P.tmap_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.x), xdims, xstrides,
+                        xbox, es5, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
+                    P.patch = 1;
+                    P.TW = best_tw;
+                    P.TH = best_th;
+                    P.tiles_p = (a.P + best_th - 1) / best_th;
+                    P.tiles_q = (a.Q + best_tw - 1) / best_tw;
+                }
+            }
+        }
         // one-plane codes: stage the tile in shared memory and write it with TMA stores
         P.fast_store = 0;
         if (a.out_mode == FXPQ_OUT_CODES && a.py == 1) {
-            const cuuint64_t ydims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
-            const cuuint64_t ystrides[1] = {(cuuint64_t)a.K * 2};
-            const cuuint32_t ybox[2] = {64, (cuuint32_t)TC_BM};
-            if (enc(&P.tmap_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.y, ydims, ystrides, ybox, es,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
-                P.fast_store = 1;
+            CUresult r;
+            if (P.patch) {
+                const cuuint64_t ydims[4] = {(cuuint64_t)a.K, (cuuint64_t)a.Q, (cuuint64_t)a.P, (cuuint64_t)a.N};
+                const cuuint64_t ystrides[3] = {(cuuint64_t)a.K * 2, (cuuint64_t)a.Q * a.K * 2,
+                                                (cuuint64_t)a.P * a.Q * a.K * 2};
+                const cuuint32_t ybox[4] = {64, (cuuint32_t)P.TW, (cuuint32_t)P.TH, 1};
+                const cuuint32_t es4[4] = {1, 1, 1, 1};
+                r = enc(&P.tmap_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, a.y, ydims, ystrides, ybox, es4,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+            } else {
+                const cuuint64_t ydims[2] = {(cuuint64_t)a.K, (cuuint64_t)a.M};
+                const cuuint64_t ystrides[1] = {(cuuint64_t)a.K * 2};
+                const cuuint32_t ybox[2] = {64, (cuuint32_t)TC_BM};
+                r = enc(&P.tmap_y, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, a.y, ydims, ystrides, ybox, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+            }
+            P.fast_store = r == CUDA_SUCCESS;
         }
     }
-    P.tiles_m = (int)((a.M + TC_BM - 1) / TC_BM);
+    P.tiles_m = P.patch ? a.N * P.tiles_p * P.tiles_q : (int)((a.M + TC_BM - 1) / TC_BM);
     P.tiles_n = (a.K + BN - 1) / BN;
     P.n_tiles = P.tiles_m * P.tiles_n;
     if (P.n_tiles == 0) {
@@ -684,11 +916,11 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     }
     const int grid = P.n_tiles < g_num_sms ? P.n_tiles : g_num_sms;
     if (acc64)
-        conv_tc_kernel<64, long long><<<grid, TC_THREADS, tc_smem_bytes<64>(), st>>>(P);
+        conv_tc_kernel<64, long long><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 64)
-        conv_tc_kernel<64, int><<<grid, TC_THREADS, tc_smem_bytes<64>(), st>>>(P);
+        conv_tc_kernel<64, int><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else
-        conv_tc_kernel<128, int><<<grid, TC_THREADS, tc_smem_bytes<128>(), st>>>(P);
+        conv_tc_kernel<128, int><<<grid, tc_threads(128), tc_smem_bytes<128>(), st>>>(P);
     launched = true;
     return after_launch("conv_tc");
 }

@@ -9,9 +9,10 @@ import oracle
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(scope="module", params=["tc", "simt"])
+@pytest.fixture(scope="module", params=["tc", "tc_rows", "simt"])
 def F(request):
-    """Runs every case on the tensor-core kernel (default) and on the CUDA-core kernel."""
+    """Runs every case on the tensor-core kernel (default: patch tiles where the layer allows
+    them), on the tensor-core kernel with 128-row tiles only, and on the CUDA-core kernel."""
     import os
     import __graft_entry__ as g
     g.build()
@@ -97,6 +98,16 @@ CASES = [
     (2, 9, 16, 40, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 19), True, 0, (8, 0, 6)),
     (2, 7, 8, 16, 3, 1, 1, (3, 1, 0), (3, 1, 0), (16, 3), False, 0, (8, 1, -1)),
     (3, 12, 64, 136, 3, 1, 1, (8, 0, 6), (8, 1, 9), (16, 24), True, 0, (8, 0, 12)),
+    # stride 1, Cp % 64 == 0: patch tiles (TMA windows with zero-filled padding) on the tensor cores
+    (2, 16, 64, 128, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),       # 16 x 8 patches
+    (2, 28, 64, 72, 3, 1, 1, (8, 0, 5), (8, 1, 8), (16, 17), True, 0, (8, 0, 4)),        # 28 x 4: 112 rows, ragged K
+    (2, 18, 64, 64, 3, 1, 0, (7, 0, 3), (6, 1, 7), (16, 14), False, 0, (8, 1, 2)),       # no padding
+    (2, 16, 64, 64, 5, 1, 2, (8, 0, 4), (8, 1, 9), (16, 18), True, 0, (8, 0, 6)),        # 5 x 5 taps
+    (2, 10, 128, 64, 3, 1, 1, (8, 0, 4), (8, 1, 7), None, True, 2, None),               # 10 x 10 patch, fp32 image
+    (2, 10, 128, 64, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), False, 1, None),          # int64 accumulators
+    (1, 16, 64, 64, 3, 1, 1, (16, 1, 12), (16, 1, 14), (16, 20), True, 0, (16, 0, 9)),   # two limbs, two planes out
+    (2, 16, 64, 40, 3, 1, 1, (5, 1, 2), (4, 1, 3), (16, 9), False, 0, (6, 1, 1)),        # bias finer than acc
+    (1, 16, 256, 128, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),      # several exact groups
 ]
 
 
