@@ -308,19 +308,23 @@ def run_kernel(args):
         w = torch.from_numpy((rng.integers(-128, 128, size=(K, 3, 3, C)) // 4).astype(np.float16)).cuda()
         b = torch.from_numpy(rng.integers(-2 ** 15, 2 ** 15, size=K).astype(np.int32)).cuda()
         y = torch.empty(N * H * H * K, dtype=torch.float16, device="cuda")
-        d = F.conv_desc(N, H, H, C, C, K, 3, 3, 1, 1, 1, F.OUT_CODES, F.fmt(8, 0, 4), F.fmt(8, 1, 8),
-                        F.fmt(16, 1, 18), F.fmt(8, 0, 3))
-        ts = []
-        for i in range(args.warmup + args.steps):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            F.fxpq_conv_fwd(d, x, w, b, y)
-            e1.record()
-            e1.synchronize()
-            if i >= args.warmup:
-                ts.append(e0.elapsed_time(e1))
-        ms = sum(ts) / len(ts)
-        out["conv"] = {"ms": round(ms, 4), "tflops": round(2 * N * H * H * K * C * 9 / (ms / 1e3) / 1e12, 2)}
+        l1 = torch.zeros(1, dtype=torch.int64, device="cuda")
+        F.fxpq_code_l1max(w, K, 9 * C, l1)
+        # "conv": groups from the wordlength bound alone; "conv_l1": with the weight-code L1 bound
+        for name, w_l1 in (("conv", 0), ("conv_l1", int(l1.item()))):
+            d = F.conv_desc(N, H, H, C, C, K, 3, 3, 1, 1, 1, F.OUT_CODES, F.fmt(8, 0, 4), F.fmt(8, 1, 8),
+                            F.fmt(16, 1, 18), F.fmt(8, 0, 3), w_l1)
+            ts = []
+            for i in range(args.warmup + args.steps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                F.fxpq_conv_fwd(d, x, w, b, y)
+                e1.record()
+                e1.synchronize()
+                if i >= args.warmup:
+                    ts.append(e0.elapsed_time(e1))
+            ms = sum(ts) / len(ts)
+            out[name] = {"ms": round(ms, 4), "tflops": round(2 * N * H * H * K * C * 9 / (ms / 1e3) / 1e12, 2)}
     if args.kernel in ("flsearch", "all"):
         n = 1 << 26
         x = torch.from_numpy(synth.normal(n, 2)).cuda()

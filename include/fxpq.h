@@ -97,6 +97,13 @@ FXPQ_API fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int3
 FXPQ_API fxpq_status fxpq_quantize_rows(const float* d_x, int64_t rows, int32_t C, fxpq_fmt f, int32_t Cp, void* d_y,
                                void* stream);
 
+/* Largest L1 norm over the rows of a one-plane fp16 code tensor [rows, L] (fmt.bits <= 8):
+ * *d_out = max_r sum_j |code[r, j]| as an int64 on the device (0 when rows == 0).  For KRSC
+ * weights with L = R*S*Cp it is the w_l1 bound of fxpq_conv_desc.  Exact integer arithmetic;
+ * d_codes 16-byte aligned and L a multiple of 8.  Not part of the paper: it feeds the
+ * implementation's exact-accumulation planning. */
+FXPQ_API fxpq_status fxpq_code_l1max(const void* d_codes, int64_t rows, int64_t L, int64_t* d_out, void* stream);
+
 /* Quantize + transpose + pack fp32 images NCHW -> NHWC fp16 code tensor with the channel count
  * padded to c_pad (a multiple of 8, >= C) with zero codes: the FxP-QLayer inserted at the input
  * of the network (Sec. IV-A.2).  d_y holds planes x [N, H, W, c_pad] fp16 values. */
@@ -162,6 +169,11 @@ FXPQ_API fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32
 /* aligned.                                                                                  */
 /* An FC layer is a convolution whose window covers the whole input map (R = H, S = W).      */
 /* Returns FXPQ_ERR_RANGE if |acc| could exceed 2^62 after alignment.                         */
+/* w_l1 (optional, one-plane weights only): an upper bound on max_o sum_{r,s,c} |W[o,r,s,c]|, */
+/* e.g. from fxpq_code_l1max, 0 = none.  Every partial sum of output channel o is then at     */
+/* most max|x code| * w_l1, which lets the tensor-core path keep longer reductions in exact    */
+/* fp32 groups and the epilogue in 32-bit arithmetic.  A value below the true norm voids the  */
+/* exactness guarantee; not part of the paper (an implementation bound).                      */
 /* ---------------------------------------------------------------------------------------- */
 enum { FXPQ_OUT_CODES = 0, FXPQ_OUT_ACC64 = 1, FXPQ_OUT_F32 = 2 };
 
@@ -173,6 +185,7 @@ typedef struct {
     int32_t relu;
     int32_t out_mode;          /* FXPQ_OUT_*                                                 */
     fxpq_fmt fmt_x, fmt_w, fmt_b, fmt_y;
+    int64_t w_l1;              /* optional weight-code L1 bound (see above), 0 = none        */
 } fxpq_conv_desc;
 
 FXPQ_API size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc);
@@ -237,6 +250,7 @@ typedef struct {
     fxpq_fmt fmt_y;          /* format of the output QLayer (ignored for maxpool / last)    */
     const void* d_w;         /* conv: fp16 code tensor KRSC [K, R, S, Cp_in]                 */
     const int32_t* d_bias;   /* conv: int32 bias codes [K] or NULL                           */
+    int64_t w_l1;            /* conv: optional weight-code L1 bound (fxpq_conv_desc.w_l1)    */
 } fxpq_op_desc;
 
 typedef struct {

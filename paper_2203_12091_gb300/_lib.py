@@ -31,13 +31,13 @@ class Stats(ctypes.Structure):
 class ConvDesc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("Cp", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("out_mode", I32),
-                ("fmt_x", Fmt), ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt)]
+                ("fmt_x", Fmt), ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("w_l1", I64)]
 
 
 class OpDesc(ctypes.Structure):
     _fields_ = [("op", I32), ("src0", I32), ("src1", I32), ("dst", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("last", I32), ("recip_code", I32),
-                ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("d_w", VP), ("d_bias", VP)]
+                ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("d_w", VP), ("d_bias", VP), ("w_l1", I64)]
 
 
 class Net(ctypes.Structure):
@@ -54,6 +54,7 @@ OP_CONV, OP_MAXPOOL, OP_ELTWISE, OP_AVGPOOL = range(4)
 _SIGS = {
     "fxpq_quantize": (I32, [VP, I64, Fmt, I32, VP, VP]),
     "fxpq_quantize_rows": (I32, [VP, I64, I32, Fmt, I32, VP, VP]),
+    "fxpq_code_l1max": (I32, [VP, I64, I64, VP, VP]),
     "fxpq_quantize_images": (I32, [VP, I32, I32, I32, I32, Fmt, I32, VP, VP]),
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),

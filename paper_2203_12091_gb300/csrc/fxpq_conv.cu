@@ -119,7 +119,10 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
     if (!aligned(x, 16) || !aligned(w, 16) || !aligned(y, 16)) return FXPQ_ERR_INVALID_ARG;
     // |acc| <= max|x code| * max|w code| * R*S*C
     const double ax = ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed), aw = ldexp(1.0, d.fmt_w.bits - d.fmt_w.is_signed);
-    const double bound = ax * aw * (double)d.R * d.S * d.C;
+    double bound = ax * aw * (double)d.R * d.S * d.C;
+    // with a weight-code L1 bound: |acc| <= max|x code| * max_o sum |w code|
+    if (d.w_l1 > 0 && d.fmt_w.bits <= 8 && ax * (double)d.w_l1 < bound) bound = ax * (double)d.w_l1;
+    if (d.w_l1 < 0) return FXPQ_ERR_INVALID_ARG;
     if (bound >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
     need64 = bound >= ldexp(1.0, 31) - 1.0;
     a.x = static_cast<const __half*>(x);
@@ -159,15 +162,19 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
         a.lo = qmin_of(d.fmt_y);
         a.hi = qmax_of(d.fmt_y);
         a.py = planes_of(d.fmt_y);
-        // 32-bit path: N = acc + aligned integer part of the bias stays below 2^31 in magnitude and the
-        // FxP-QLayer is a right shift by 1..30 bits of N (see qlayer_code32)
+        // 32-bit path: N = acc + aligned integer part of the bias, plus the rounding increment
+        // 2^(sh32 - 1), stays below 2^31 in magnitude and the FxP-QLayer is a right shift by 1..30 bits
+        // of N (see qlayer_code32)
         const double two31 = ldexp(1.0, 31) - 1.0;
         const double bb = bias ? ldexp(1.0, d.fmt_b.bits - d.fmt_b.is_signed) : 0.0;
         const int s_acc = d.fmt_x.fl + d.fmt_w.fl;
         a.bsh = a.delta;
         a.sh32 = s_acc - d.fmt_y.fl;
         const double nbound = bound + (a.delta >= 0 ? bb * ldexp(1.0, a.delta) : bb * ldexp(1.0, a.delta) + 1.0);
-        a.v32 = (nbound < two31 && a.sh32 >= 1 && a.sh32 <= 30 && a.delta >= -30 && a.delta <= 30) ? 1 : 0;
+        a.v32 = (a.sh32 >= 1 && a.sh32 <= 30 && nbound + ldexp(1.0, a.sh32 - 1) < two31 && a.delta >= -30 &&
+                 a.delta <= 30)
+                    ? 1
+                    : 0;
     } else {
         a.sh = 0;
         a.lo = a.hi = 0;
@@ -241,5 +248,6 @@ extern "C" fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_
     d.fmt_w = fmt_w;
     d.fmt_b = fmt_b;
     d.fmt_y = fmt_y;
+    d.w_l1 = 0;
     return fxpq_conv_fwd(&d, d_x, d_w, d_bias, d_y, h_out_scale, d_ws, ws_bytes, stream);
 }

@@ -24,6 +24,7 @@
 // Every wait is bounded: on expiry the kernel latches FXPQ_ERR_TIMEOUT, stops issuing work,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>  // CUtensorMap and its enums (the encoder is fetched through the runtime)
+#include <climits>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -37,11 +38,16 @@ namespace {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
-constexpr int TC_STAGES = 6;
-constexpr int TC_LAG = 3;  // producer arrives on a stage three k-blocks after issuing it
-// Warps: 4 producers, BN / 8 epilogue warps (one 32-column chunk of one TMEM lane quadrant each),
-// one MMA / TMEM-allocation warp.
-__host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8; }
+// Pipeline depth: 6 stages of 32 KB (BN <= 128) or 3 of 48 KB (BN = 256, whose 64 KB output staging
+// leaves no room for a fourth).
+__host__ __device__ constexpr int tc_stages(int BN) { return BN == 256 ? 3 : 6; }
+// Row-tile producers arrive on a stage this many k-blocks after issuing its copies (cp.async groups
+// in flight).  It must stay below the stage count: a producer waiting for a stage to be consumed
+// must already have arrived on it.
+__host__ __device__ constexpr int tc_lag(int BN) { return tc_stages(BN) - 1 < 3 ? tc_stages(BN) - 1 : 3; }
+// Warps: 4 producers, epilogue warps (four per 32-column chunk group: one per TMEM lane quadrant;
+// BN / 8 of them up to 16, each then draining BN / 128 chunks), one MMA / TMEM-allocation warp.
+__host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8 < 16 ? BN / 8 : 16; }
 __host__ __device__ constexpr int tc_threads(int BN) { return (5 + tc_epi_warps(BN)) * 32; }
 constexpr int TC_MAX_GROUPS = 64;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
@@ -57,6 +63,7 @@ struct TcParams {
     CUtensorMap tmap_y;  // output codes: [M][K] box {64, 128} (linear tiles) or [N][P][Q][K] box {64, TW, TH, 1}
     CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}
     int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
+    int nbuf;            // fp32 accumulator buffers in TMEM: 2, or 1 when BN = 256 needs running sums
     int patch;           // 1: a tile is a TH x TW patch of one image, the A tile comes by TMA
     int TH, TW;          // patch shape (TH * TW = 128)
     int tiles_p, tiles_q;  // patches per image along P and Q
@@ -313,9 +320,10 @@ __device__ __forceinline__ void epilogue_block32(const ConvArgs& a, long long m,
 // the bias alignment split into a left and a right shift so that it has no branches).
 struct Epi32 {
     int bsl, bsr, fmask;  // bias term (b << bsl) >> bsr; fraction bits b & fmask (bias finer than acc)
-    int sh, rmask, half;  // requantizing right shift, its remainder mask and half
+    int sh, hm1;          // requantizing right shift and 2^(sh-1) - 1
+    int floor;            // 0 with ReLU, INT_MIN without
     int lo, hi;
-    int relu, has_bias;
+    int has_bias;
 };
 
 __device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
@@ -324,33 +332,30 @@ __device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
     e.bsr = a.bsh < 0 ? -a.bsh : 0;
     e.fmask = (1 << e.bsr) - 1;
     e.sh = a.sh32;
-    e.rmask = (1 << a.sh32) - 1;
-    e.half = 1 << (a.sh32 - 1);
+    e.hm1 = (1 << (a.sh32 - 1)) - 1;
+    e.floor = a.relu ? 0 : INT_MIN;
     e.lo = (int)a.lo;
     e.hi = (int)a.hi;
-    e.relu = a.relu;
     e.has_bias = a.has_bias;
     return e;
 }
 
-// One code: N = acc + aligned bias; ReLU; round half to even on the dropped bits (phi: the bias had
-// nonzero bits below the accumulator's scale, so a remainder of exactly one half is above the tie).
-__device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, bool phi) {
-    int N = acc + bterm;
-    if (e.relu && N < 0) {
-        N = 0;
-        phi = false;
-    }
-    const int q = N >> e.sh;
-    const int rem = N & e.rmask;
-    const bool up = rem > e.half || (rem == e.half && (phi || (q & 1)));
-    return min(max(q + (up ? 1 : 0), e.lo), e.hi);
+// One code: N = acc + aligned bias; ReLU; N / 2^sh rounded half to even, then clipped.  With
+// q = floor(N / 2^sh) and x = (q & 1) | phi, floor((N + 2^(sh-1) - 1 + x) / 2^sh) is q + 1 exactly
+// when the remainder is above one half, or equal to it with q odd or phi set (phi: the bias had
+// nonzero bits below the accumulator's scale, so the true value lies above the tie).  After a ReLU
+// clamp N = 0 and the sum stays below 2^sh whatever phi is.  The host keeps |N| + 2^(sh-1) < 2^31.
+__device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, int phi) {
+    const int N = max(acc + bterm, e.floor);
+    const int x = ((N >> e.sh) & 1) | phi;
+    return min(max((N + e.hm1 + x) >> e.sh, e.lo), e.hi);
 }
 
 // Two codes in [-512, 511] as a packed fp16 pair: 1536 + c has the bit pattern 0x6600 + c (the
 // binade [1024, 2048) has unit spacing), and one packed subtraction of 1536 leaves c exactly.
 __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
-    const uint32_t bits = (uint32_t)(0x6600 + c0) | ((uint32_t)(0x6600 + c1) << 16);
+    // 0x6600 + c0 >= 0x6400 never borrows from the high half
+    const uint32_t bits = (uint32_t)c1 * 65536u + (uint32_t)c0 + 0x66006600u;
     const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&bits), __halves2half2(__ushort_as_half(0x6600),
                                                                                         __ushort_as_half(0x6600)));
     return *reinterpret_cast<const uint32_t*>(&h);
@@ -359,14 +364,19 @@ __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
 // ------------------------------------------------------------------ kernel
 template <int BN, typename ACC>
 __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+    constexpr int TC_STAGES = tc_stages(BN);
+    constexpr int TC_LAG = tc_lag(BN);
+    static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
     constexpr int EPI_WARPS = tc_epi_warps(BN);
     constexpr int EPI_THREADS = 32 * EPI_WARPS;
     constexpr int MMA_WARP = 4 + EPI_WARPS;
+    constexpr int CPW = (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
     constexpr int B_BYTES = BN * TC_BK * 2;
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
-    // two fp32 accumulator buffers + integer running sums, rounded up to a power of two
-    constexpr uint32_t USED_COLS = 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
+    // fp32 accumulator buffers + integer running sums, rounded up to a power of two (BN = 256: two
+    // buffers without running sums, or one buffer with them)
+    constexpr uint32_t USED_COLS = BN == 256 ? 512u : 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
     constexpr uint32_t TMEM_COLS = USED_COLS <= 256 ? 256u : 512u;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -420,7 +430,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         if (threadIdx.x == 0) {
             const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * 128);
             const int per_img = P.tiles_p * P.tiles_q;
-            uint32_t it = 0;
+            uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
                 const int tm = t / P.tiles_n, tn = t % P.tiles_n;
@@ -429,8 +439,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 for (int gi = 0; gi < P.n_groups && ok; ++gi) {
                     const TcGroup g = P.g[gi];
                     for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                        const int stage = it % TC_STAGES;
-                        if (!wait_bounded(empty0 + 8 * stage, ((it / TC_STAGES) & 1) ^ 1, abort, P.status)) {
+                        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
                             ok = false;
                             break;
                         }
@@ -443,6 +452,10 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                     g.a_plane, fb);
                         tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, f, tn * BN, g.w_plane, fb);
                         ++it;
+                        if (++stage == TC_STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
                     }
                 }
             }
@@ -538,28 +551,29 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     } else if (warp < MMA_WARP) {
         // ============================================================ epilogue
         // Warp w drains TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the quadrant a warp may access) and
-        // the 32-column chunk cb = (w - 4) / 4 of every accumulator.
+        // the 32-column chunks cw * CPW .. cw * CPW + CPW - 1, cw = (w - 4) / 4, of every accumulator.
         const int quad = warp & 3;
-        const int cb = (warp - 4) >> 2;
+        const int cw = (warp - 4) >> 2;
         const int row = quad * 32 + lane;
         const bool leader = threadIdx.x == 128;  // waits for and issues the tile's TMA stores
+        const int nbuf = P.nbuf;
         uint32_t gcount = 0;
         bool ok = true;
-        // Integer running sums of a tile live in TMEM columns [2 BN, 2 BN + BN * words), words = 1
-        // (int32) or 2 (int64 as lo / hi column blocks), so the drain keeps few registers.
+        // Integer running sums of a tile live in TMEM after the accumulator buffers: columns
+        // [nbuf BN, nbuf BN + BN * words), words = 1 (int32) or 2 (int64 as lo / hi column blocks).
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
-        const uint32_t run_col = 2 * BN + cb * 32;
+        const uint32_t run_base = (uint32_t)(nbuf * BN);
         const Epi32 e32 = make_epi32(a);
         uint32_t u = 0;  // tiles written through the staging buffer so far
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             const long long m = tile_row(P, tm, row);  // -1: row outside the output
-            const int k0 = tn * BN + cb * 32;
             for (int gi = 0; gi < P.n_groups; ++gi) {
                 const int shift = P.g[gi].shift;
                 const bool first = gi == 0, last = gi == P.n_groups - 1;
-                const uint32_t buf = gcount & 1;
-                if (!wait_bounded(accfull0 + 8 * buf, (gcount >> 1) & 1, abort, P.status)) {
+                const uint32_t buf = nbuf == 2 ? (gcount & 1) : 0;
+                const uint32_t par = nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
+                if (!wait_bounded(accfull0 + 8 * buf, par, abort, P.status)) {
                     ok = false;
                     break;
                 }
@@ -575,90 +589,103 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                         break;
                     }
                 }
-                ACC acc[32];
-                {
-                    float f[32];
-                    tmem_ld32(lane_base + buf * BN + cb * 32, f);
+#pragma unroll 1
+                for (int c = 0; c < CPW; ++c) {
+                    const int cb = cw * CPW + c;
+                    const int k0 = tn * BN + cb * 32;
+                    const uint32_t run_col = run_base + cb * 32;
+                    ACC acc[32];
+                    {
+                        float f[32];
+                        tmem_ld32(lane_base + buf * BN + cb * 32, f);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) acc[j] = ((ACC)__float2int_rn(f[j])) << shift;
-                }
-                if (sizeof(ACC) == 8) {
-                    // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
+                        for (int j = 0; j < 32; ++j) acc[j] = ((ACC)__float2int_rn(f[j])) << shift;
+                    }
+                    if (sizeof(ACC) == 8) {
+                        // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
 #pragma unroll
-                    for (int hf = 0; hf < 2; ++hf) {
-                        uint32_t lo[16], hi[16];
-                        if (!first) {
-                            tmem_ld16u(lane_base + run_col + 16 * hf, lo);
-                            tmem_ld16u(lane_base + run_col + BN + 16 * hf, hi);
+                        for (int hf = 0; hf < 2; ++hf) {
+                            uint32_t lo[16], hi[16];
+                            if (!first) {
+                                tmem_ld16u(lane_base + run_col + 16 * hf, lo);
+                                tmem_ld16u(lane_base + run_col + BN + 16 * hf, hi);
 #pragma unroll
-                            for (int j = 0; j < 16; ++j)
-                                acc[16 * hf + j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
-                        }
-                        if (!last) {
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                lo[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
-                                hi[j] = (uint32_t)((unsigned long long)acc[16 * hf + j] >> 32);
+                                for (int j = 0; j < 16; ++j)
+                                    acc[16 * hf + j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
                             }
-                            tmem_st16u(lane_base + run_col + 16 * hf, lo);
-                            tmem_st16u(lane_base + run_col + BN + 16 * hf, hi);
-                        }
-                    }
-                } else {
-                    if (!first) {
-                        uint32_t lo[32];
-                        tmem_ld32u(lane_base + run_col, lo);
+                            if (!last) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
-                    }
-                    if (!last) {
-                        uint32_t lo[32];
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) lo[j] = (uint32_t)(unsigned long long)acc[j];
-                        tmem_st32u(lane_base + run_col, lo);
-                    }
-                }
-                // the accumulator buffer is free for the next group's MMAs
-                tc_fence_before();
-                mbar_arrive(accempty0 + 8 * buf);
-                ++gcount;
-                if (!last) continue;
-                if (P.fast_store) {
-                    // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
-                    uint32_t w[16];
-                    if (sizeof(ACC) == 4 && a.v32) {
-#pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            int c2[2];
-#pragma unroll
-                            for (int h = 0; h < 2; ++h) {
-                                const int k = k0 + 2 * j + h;
-                                const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
-                                                   (b & e32.fmask) != 0);
+                                for (int j = 0; j < 16; ++j) {
+                                    lo[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
+                                    hi[j] = (uint32_t)((unsigned long long)acc[16 * hf + j] >> 32);
+                                }
+                                tmem_st16u(lane_base + run_col + 16 * hf, lo);
+                                tmem_st16u(lane_base + run_col + BN + 16 * hf, hi);
                             }
-                            w[j] = pack_codes_f16(c2[0], c2[1]);
                         }
                     } else {
+                        if (!first) {
+                            uint32_t lo[32];
+                            tmem_ld32u(lane_base + run_col, lo);
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            int c2[2];
+                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
+                        }
+                        if (!last) {
+                            uint32_t lo[32];
 #pragma unroll
-                            for (int h = 0; h < 2; ++h) {
-                                const int k = k0 + 2 * j + h;
-                                const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                c2[h] = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j + h], b));
-                            }
-                            w[j] = pack_codes_f16(c2[0], c2[1]);
+                            for (int j = 0; j < 32; ++j) lo[j] = (uint32_t)(unsigned long long)acc[j];
+                            tmem_st32u(lane_base + run_col, lo);
                         }
                     }
-                    unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int chunk = (cb & 1) * 4 + q;
-                        *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
-                            make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                    if (c == CPW - 1) {
+                        // every chunk of this warp is out of the accumulator buffer: free it for the
+                        // next group's MMAs before the final arithmetic
+                        tc_fence_before();
+                        mbar_arrive(accempty0 + 8 * buf);
                     }
+                    if (!last) continue;
+                    if (P.fast_store) {
+                        // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
+                        uint32_t w[16];
+                        if (sizeof(ACC) == 4 && a.v32) {
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                int c2[2];
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    const int k = k0 + 2 * j + h;
+                                    const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                    c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
+                                                       (b & e32.fmask) != 0 ? 1 : 0);
+                                }
+                                w[j] = pack_codes_f16(c2[0], c2[1]);
+                            }
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                int c2[2];
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    const int k = k0 + 2 * j + h;
+                                    const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                    c2[h] = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j + h], b));
+                                }
+                                w[j] = pack_codes_f16(c2[0], c2[1]);
+                            }
+                        }
+                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int chunk = (cb & 1) * 4 + q;
+                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                        }
+                    } else if (m >= 0) {
+                        epilogue_block32<ACC>(a, m, k0, acc);
+                    }
+                }
+                ++gcount;
+                if (last && P.fast_store) {
                     // make the staging writes visible to the async proxy, then one thread stores the tile
                     fence_proxy_async();
                     mbar_arrive(stg_full);
@@ -681,40 +708,47 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                         bulk_commit();
                     }
                     ++u;
-                } else if (m >= 0) {
-                    epilogue_block32<ACC>(a, m, k0, acc);
                 }
             }
         }
         if (leader) bulk_wait0();  // every output store has completed
     } else if (lane == 0) {
         // ============================================================ MMA issue (one thread of MMA_WARP)
-        uint32_t it = 0, gcount = 0;
+        // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
+        // (address >> 4, 14 bits) without carry since shared addresses stay below 256 KB.
+        const uint64_t adesc0 = make_sdesc(smem_u32(sA)), bdesc0 = make_sdesc(smem_u32(sB));
+        uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             for (int gi = 0; gi < P.n_groups && ok; ++gi) {
                 const TcGroup g = P.g[gi];
-                const uint32_t buf = gcount & 1;
-                if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status)) {
+                const uint32_t buf = P.nbuf == 2 ? (gcount & 1) : 0;
+                const uint32_t par = P.nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
+                if (!wait_bounded(accempty0 + 8 * buf, par ^ 1, abort, P.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + buf * BN;
+                uint32_t accum = 0;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                    const int stage = it % TC_STAGES;
-                    if (!wait_bounded(full0 + 8 * stage, (it / TC_STAGES) & 1, abort, P.status)) {
+                    if (!wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t aS = smem_u32(sA + stage * A_BYTES), bS = smem_u32(sB + stage * B_BYTES);
+                    const uint64_t ad = adesc0 + (uint64_t)((stage * A_BYTES) >> 4);
+                    const uint64_t bd = bdesc0 + (uint64_t)((stage * B_BYTES) >> 4);
 #pragma unroll
-                    for (int kk = 0; kk < TC_BK / 16; ++kk)
-                        tc_mma(d, make_sdesc(aS + kk * 32), make_sdesc(bS + kk * 32), IDESC,
-                               (kb > g.kb0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < TC_BK / 16; ++kk) {
+                        tc_mma(d, ad + 2 * kk, bd + 2 * kk, IDESC, accum);
+                        accum = 1;
+                    }
                     tc_commit(empty0 + 8 * stage);
-                    ++it;
+                    if (++stage == TC_STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
                 }
                 if (!ok) break;
                 tc_commit(accfull0 + 8 * buf);
@@ -738,17 +772,30 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
 int g_num_sms = 0;
 std::mutex g_tc_mu;
 
-// FXPQ_CONV_PATH=tc_rows keeps every layer on 128-row tiles (both tilings are exact; the switch
-// lets tests compare them on the same shapes).
-bool patch_enabled() {
+// FXPQ_CONV_PATH picks among exact alternatives so that tests can compare them on the same shapes:
+// "tc_rows" keeps every layer on 128-row tiles, "tc_bn128" never takes 256-column tiles and
+// "tc_bn256" takes them wherever the layer allows (by default they also need enough tiles to keep
+// every SM busy).
+bool conv_path_is(const char* name) {
     const char* e = getenv("FXPQ_CONV_PATH");
-    return !(e && strcmp(e, "tc_rows") == 0);
+    return e && strcmp(e, name) == 0;
 }
-bool g_tc_attr_set[2] = {false, false};
+bool g_tc_attr_set = false;
+
+int num_sms() {
+    std::lock_guard<std::mutex> lk(g_tc_mu);
+    if (g_num_sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_num_sms <= 0) g_num_sms = 1;
+    }
+    return g_num_sms;
+}
 
 template <int BN>
 constexpr size_t tc_smem_bytes() {
-    return 1024 + TC_STAGES * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
+    return 1024 + tc_stages(BN) * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
 }
 
 // Largest |limb| of a format's codes: the only plane (k <= 8) or the hi / lo limb (k > 8).
@@ -776,7 +823,11 @@ bool plan_tc(const ConvArgs& a, const fxpq_conv_desc& d, TcParams& P, bool& acc6
             const long long bound = limb_max(d.fmt_x, ia) * limb_max(d.fmt_w, iw);
             if (bound == 0) continue;
             const long long kmax = ((1LL << 24) - 1) / bound;  // taps per exact fp32 group
-            const int kb_per = (int)(kmax / TC_BK);
+            int kb_per = (int)(kmax / TC_BK);
+            // every partial sum of channel o is at most max|x limb| * sum_taps |w[o]| <= max|x| * w_l1:
+            // below 2^24 the whole reduction is one exact group
+            if (d.w_l1 > 0 && d.w_l1 < (1LL << 24) && pw == 1 && limb_max(d.fmt_x, ia) * d.w_l1 < (1LL << 24))
+                kb_per = n_kb;
             if (kb_per < 1) return false;
             const int shift = 8 * ((pa - 1 - ia) + (pw - 1 - iw));
             shifted |= shift > 0;
@@ -786,8 +837,10 @@ bool plan_tc(const ConvArgs& a, const fxpq_conv_desc& d, TcParams& P, bool& acc6
             }
         }
     P.n_groups = ng;
-    const double total = ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed) * ldexp(1.0, d.fmt_w.bits - d.fmt_w.is_signed) *
-                         (double)a.R * a.S * a.Cp;
+    double total = ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed) * ldexp(1.0, d.fmt_w.bits - d.fmt_w.is_signed) *
+                   (double)a.R * a.S * a.Cp;
+    if (d.w_l1 > 0 && pw == 1)
+        total = fmin(total, ldexp(1.0, d.fmt_x.bits - d.fmt_x.is_signed) * (double)d.w_l1);
     acc64 = shifted || total >= ldexp(1.0, 31) - 1.0;
     P.status = status_ptr();
     return ng > 0;
@@ -821,8 +874,20 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     TcParams P;
     bool acc64 = false;
     if (!plan_tc(a, d, P, acc64)) return FXPQ_OK;
-    // 64-column tiles for int64 sums and for layers with at most 64 output channels
-    const int BN = (acc64 || a.K <= 64) ? 64 : 128;
+    const int sms = num_sms();
+    // 64-column tiles for int64 sums and for layers with at most 64 output channels; 256-column tiles
+    // (one MMA instruction covers twice the work of a 128-column one, which hides its issue cost) for
+    // wide layers with enough tiles
+    int BN = 128;
+    const long long row_tiles_est = (a.M + TC_BM - 1) / TC_BM;
+    if (acc64 || a.K <= 64)
+        BN = 64;
+    else if (a.K > 128 && !conv_path_is("tc_bn128") &&
+             (conv_path_is("tc_bn256") || (a.K % 256 == 0 && row_tiles_est * (a.K / 256) >= sms)))
+        BN = 256;
+    // BN = 256 fills TMEM with two accumulator buffers; with several exact groups per tile it keeps one
+    // buffer and the integer running sums
+    P.nbuf = (BN == 256 && P.n_groups > 1) ? 1 : 2;
     {
         EncodeTiledFn enc = encode_tiled();
         if (!enc) return FXPQ_OK;  // no tensor-map encoder: the CUDA-core kernel runs instead
@@ -836,7 +901,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             return FXPQ_OK;
         // patch tiles for stride-1 layers whose taps are whole 64-channel blocks
         P.patch = 0;
-        if (a.stride == 1 && P.cp64 && a.P > 0 && a.Q > 0 && a.N > 0 && patch_enabled()) {
+        if (a.stride == 1 && P.cp64 && a.P > 0 && a.Q > 0 && a.N > 0 && !conv_path_is("tc_rows")) {
             int best_tw = 0, best_th = 0;
             long long best = 0;
             for (int tw = a.Q < TC_BM ? a.Q : TC_BM; tw >= 1; --tw) {
@@ -897,30 +962,28 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     }
     {
         std::lock_guard<std::mutex> lk(g_tc_mu);
-        if (g_num_sms == 0) {
-            int dev = 0;
-            cudaGetDevice(&dev);
-            cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-            if (g_num_sms <= 0) g_num_sms = 1;
-        }
-        if (!g_tc_attr_set[0]) {
+        if (!g_tc_attr_set) {
             if (cudaFuncSetAttribute(conv_tc_kernel<64, long long>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<64, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<128, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)tc_smem_bytes<128>()) != cudaSuccess)
+                                     (int)tc_smem_bytes<128>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<256>()) != cudaSuccess)
                 return FXPQ_ERR_CUDA;
-            g_tc_attr_set[0] = true;
+            g_tc_attr_set = true;
         }
     }
-    const int grid = P.n_tiles < g_num_sms ? P.n_tiles : g_num_sms;
+    const int grid = P.n_tiles < sms ? P.n_tiles : sms;
     if (acc64)
         conv_tc_kernel<64, long long><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 64)
         conv_tc_kernel<64, int><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
-    else
+    else if (BN == 128)
         conv_tc_kernel<128, int><<<grid, tc_threads(128), tc_smem_bytes<128>(), st>>>(P);
+    else
+        conv_tc_kernel<256, int><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
     launched = true;
     return after_launch("conv_tc");
 }

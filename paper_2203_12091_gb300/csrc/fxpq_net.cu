@@ -135,6 +135,7 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
                 d.fmt_w = o.fmt_w;
                 d.fmt_b = o.fmt_b;
                 d.fmt_y = o.fmt_y;
+                d.w_l1 = o.w_l1;
                 int32_t scale = 0;
                 st = fxpq_conv_fwd(&d, ptr(o.src0), o.d_w, o.d_bias, last ? (void*)d_logits : ptr(o.dst), &scale,
                                    nullptr, 0, stream);

@@ -85,6 +85,38 @@ __global__ void quantize_images_kernel(const float* __restrict__ x, int N, int C
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
 
+// max over rows of sum |code|: one block per row (grid-stride over rows), 8 codes per 16-byte load
+__global__ void code_l1max_kernel(const uint4* __restrict__ codes, long long rows, long long L8,
+                                  unsigned long long* __restrict__ out) {
+    __shared__ long long red[32];
+    for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
+        const uint4* row = codes + r * L8;
+        long long sum = 0;
+        for (long long i = threadIdx.x; i < L8; i += blockDim.x) {
+            const uint4 v = __ldg(row + i);
+            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            int part = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const __half2 h = *reinterpret_cast<const __half2*>(&w[j]);
+                part += abs(__half2int_rn(__low2half(h))) + abs(__half2int_rn(__high2half(h)));
+            }
+            sum += part;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sum;
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            long long t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+            if (threadIdx.x == 0) atomicMax(out, (unsigned long long)t);
+        }
+        __syncthreads();
+    }
+}
+
 }  // namespace
 
 static QParams make_qparams(const fxpq_fmt& f) {
@@ -169,4 +201,16 @@ extern "C" fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, in
                                                                                 planes_of(f), p,
                                                                                 static_cast<__half*>(d_y));
     return after_launch("quantize_images");
+}
+
+extern "C" fxpq_status fxpq_code_l1max(const void* d_codes, int64_t rows, int64_t L, int64_t* d_out, void* stream) {
+    if (rows < 0 || L < 0 || (L % 8) || !d_out || !aligned(d_out, 8)) return FXPQ_ERR_INVALID_ARG;
+    if (rows > 0 && L > 0 && (!d_codes || !aligned(d_codes, 16))) return FXPQ_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (cudaMemsetAsync(d_out, 0, sizeof(int64_t), s) != cudaSuccess) return FXPQ_ERR_CUDA;
+    if (rows == 0 || L == 0) return FXPQ_OK;
+    const int grid = rows < 4096 ? (int)rows : 4096;
+    code_l1max_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4*>(d_codes), rows, L / 8,
+                                           reinterpret_cast<unsigned long long*>(d_out));
+    return after_launch("code_l1max");
 }

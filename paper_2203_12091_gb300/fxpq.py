@@ -53,6 +53,13 @@ def fxpq_quantize_rows(x, rows: int, C: int, f: Fmt, Cp: int, out, stream=None):
     return out
 
 
+def fxpq_code_l1max(codes, rows: int, L_: int, out, stream=None):
+    """max_r sum_j |codes[r, j]| of a one-plane fp16 code tensor [rows, L_] into the int64 device
+    tensor `out` (one element)."""
+    L.check("fxpq_code_l1max", L.lib().fxpq_code_l1max(_p(codes), rows, L_, _p(out), _s(stream)))
+    return out
+
+
 def fxpq_quantize_images(x_nchw, f: Fmt, c_pad: int, out, stream=None):
     N, C, H, W = x_nchw.shape
     L.check("fxpq_quantize_images",
@@ -94,9 +101,9 @@ def fxpq_fl_init(stats: Stats, bits: int, strategy: int) -> Fmt:
 
 
 # ------------------------------------------------------------------------------ C-Blocks
-def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy) -> L.ConvDesc:
+def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy, w_l1=0) -> L.ConvDesc:
     return L.ConvDesc(N, H, W, C, Cp, K, R, S, stride, pad, int(relu), out_mode, fx, fw,
-                      fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0))
+                      fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0), int(w_l1))
 
 
 def fxpq_conv_fwd(desc: L.ConvDesc, x, w, bias, y, stream=None) -> int:

@@ -76,6 +76,7 @@ class QNet:
         self.cp_in = pad8(cin)
         self.fmts = {}
         self.q = {}  # name -> (weight fp16 codes, bias int32 codes)
+        self.w_l1 = {}  # conv name -> max over output channels of sum |weight code| (0: unknown)
         self.names = ["input"] + [L_["name"] for L_ in layers]
         self.slot = {nm: i for i, nm in enumerate(self.names)}
         self.shapes = {}
@@ -121,6 +122,10 @@ class QNet:
         for (nm, key), f in zip(owners, search_fmts(searches, stream)):
             self.fmts[nm][key] = f
         rcodes = {}
+        # per conv layer: the largest L1 norm of an output channel's one-plane weight codes (lets the
+        # tensor-core contraction plan longer exact fp32 groups), read back with the avg-pool codes
+        conv_names = [L_["name"] for L_ in self.layers if L_["type"] == "conv"]
+        l1 = torch.zeros(max(1, len(conv_names)), dtype=torch.int64, device=dev)
         for i, L_ in enumerate(self.layers):
             nm = L_["name"]
             if L_["type"] == "conv":
@@ -130,6 +135,8 @@ class QNet:
                 fw, fb = self.fmts[nm]["w"], self.fmts[nm]["b"]
                 wq = torch.empty(K * R * R * Cp * F.planes(fw), dtype=torch.float16, device=dev)
                 F.fxpq_quantize_rows(w.reshape(-1, C), K * R * R, C, fw, Cp, wq, stream)
+                if F.planes(fw) == 1:
+                    F.fxpq_code_l1max(wq, K, R * R * Cp, l1[conv_names.index(nm):], stream)
                 bq = torch.empty(K, dtype=torch.int32, device=dev)
                 F.fxpq_quantize(b, fb, F.DT_I32, bq, stream)
                 self.q[nm] = (wq, bq)
@@ -137,6 +144,8 @@ class QNet:
                 rc = torch.empty(1, dtype=torch.int32, device=dev)
                 F.fxpq_quantize(recips[nm], self.fmts[nm]["r"], F.DT_I32, rc, stream)
                 rcodes[nm] = rc
+        l1_host = l1.cpu().tolist()
+        self.w_l1 = {nm: int(l1_host[j]) for j, nm in enumerate(conv_names)}
         for nm, rc in rcodes.items():
             self.q[nm] = (None, int(rc.item()))
         self.shapes = shapes
@@ -160,7 +169,7 @@ class QNet:
             sH, sW, sCp = self.shapes[src]
             wq, bq = self.q[nm]
             d = F.conv_desc(N, sH, sW, sCp, sCp, L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], L_["relu"],
-                            out_mode, fx, self.fmts[nm]["w"], self.fmts[nm]["b"], fy)
+                            out_mode, fx, self.fmts[nm]["w"], self.fmts[nm]["b"], fy, self.w_l1.get(nm, 0))
             s = F.fxpq_conv_fwd(d, x, wq, bq, y, stream)
         elif L_["type"] == "maxpool":
             src = self._src(i, L_)
@@ -236,6 +245,7 @@ class QNet:
                 o.fmt_y = self.fmts[nm].get("a", L.Fmt(8, 1, 0))
                 o.d_w = self.q[nm][0].data_ptr()
                 o.d_bias = self.q[nm][1].data_ptr()
+                o.w_l1 = self.w_l1.get(nm, 0)
             elif L_["type"] == "maxpool":
                 o.op = L.OP_MAXPOOL
                 o.src0 = self.slot[self._src(i, L_)]

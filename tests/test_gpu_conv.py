@@ -9,10 +9,11 @@ import oracle
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(scope="module", params=["tc", "tc_rows", "simt"])
+@pytest.fixture(scope="module", params=["tc", "tc_rows", "tc_bn256", "simt"])
 def F(request):
     """Runs every case on the tensor-core kernel (default: patch tiles where the layer allows
-    them), on the tensor-core kernel with 128-row tiles only, and on the CUDA-core kernel."""
+    them), on the tensor-core kernel with 128-row tiles only, on the tensor-core kernel with
+    256-column tiles wherever K > 128, and on the CUDA-core kernel."""
     import os
     import __graft_entry__ as g
     g.build()
@@ -46,7 +47,7 @@ def to_f16_planes(codes, k, Cp):
     return torch.from_numpy(np.stack([hi, lo]).astype(np.float16)).cuda()
 
 
-def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp):
+def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0):
     N, H, W, C = x.shape
     K, R, S, _ = w.shape
     P = (H + 2 * pad - R) // stride + 1
@@ -60,7 +61,7 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp):
         y = torch.empty(N * P * Q * K, dtype=torch.int64, device="cuda")
     else:
         y = torch.empty(N * P * Q * K, dtype=torch.float32, device="cuda")
-    d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy)
+    d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy, w_l1)
     s = F.fxpq_conv_fwd(d, xd, wd, bd, y)
     torch.cuda.synchronize()
     assert F.fxpq_get_device_status() == 0
@@ -108,11 +109,17 @@ CASES = [
     (1, 16, 64, 64, 3, 1, 1, (16, 1, 12), (16, 1, 14), (16, 20), True, 0, (16, 0, 9)),   # two limbs, two planes out
     (2, 16, 64, 40, 3, 1, 1, (5, 1, 2), (4, 1, 3), (16, 9), False, 0, (6, 1, 1)),        # bias finer than acc
     (1, 16, 256, 128, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),      # several exact groups
+    # K > 128: 256-column tiles under tc_bn256 (one exact group: two accumulator buffers; several:
+    # one buffer plus integer running sums)
+    (2, 8, 64, 256, 3, 1, 1, (6, 0, 2), (6, 1, 5), (16, 12), True, 0, (8, 0, 3)),
+    (1, 16, 256, 256, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),
+    (2, 9, 16, 264, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),        # ragged K, row tiles
+    (2, 8, 64, 256, 3, 1, 1, (8, 0, 4), (8, 1, 7), None, True, 2, None),               # fp32 image
+    (2, 8, 64, 256, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), False, 1, None),          # int64 accumulators
 ]
 
 
-@pytest.mark.parametrize("case", CASES)
-def test_conv_parity(F, case):
+def run_case(F, case, use_l1=False):
     N, H, C, K, R, st, pad, tx, tw, tb, relu, mode, ty = case
     rng = np.random.default_rng(H * 131 + K)
     fx, fw = F.fmt(*tx), F.fmt(*tw)
@@ -120,14 +127,41 @@ def test_conv_parity(F, case):
     fy = F.fmt(*ty) if ty else None
     x = rand_codes(rng, (N, H, H, C), tx[0], tx[1])
     w = rand_codes(rng, (K, R, R, C), tw[0], tw[1])
-    # realistic weight magnitudes: mostly small codes
     w = np.where(rng.random(w.shape) < 0.8, w // 4, w)
     b = rand_codes(rng, (K,), tb[0], 1) if tb else None
     Cp = (C + 7) // 8 * 8
-    got, s = run_conv(F, x, fx, w, fw, b, fb, st, pad, relu, mode, fy, Cp)
+    w_l1 = int(np.abs(w).reshape(K, -1).sum(axis=1).max()) if use_l1 else 0
+    got, s = run_conv(F, x, fx, w, fw, b, fb, st, pad, relu, mode, fy, Cp, w_l1)
     want, ws = oracle_conv(x, fx, w, fw, b, fb, st, pad, relu, mode, fy)
     assert s == ws
     assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("case", [c for c in CASES if c[8][0] <= 8])
+def test_conv_parity_l1_bound(F, case):
+    """The weight-code L1 bound lets the tensor-core path take the whole reduction as one exact
+    fp32 group (and a 32-bit epilogue) where the wordlength bound alone would split it."""
+    run_case(F, case, use_l1=True)
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_conv_parity(F, case):
+    run_case(F, case)
+
+
+def test_code_l1max(F):
+    """max over rows of sum |code| on one-plane fp16 codes, against numpy; the zero-row case."""
+    rng = np.random.default_rng(11)
+    for rows, L_, lo, hi in ((37, 8 * 163, -128, 127), (1, 8, 0, 255), (300, 4608, -8, 7)):
+        c = rng.integers(lo, hi + 1, size=(rows, L_))
+        c[rows // 2, :] = hi if abs(hi) > abs(lo) else lo  # the extreme row
+        d = torch.from_numpy(c.astype(np.float16)).cuda()
+        out = torch.full((1,), -1, dtype=torch.int64, device="cuda")
+        F.fxpq_code_l1max(d, rows, L_, out)
+        assert int(out.item()) == int(np.abs(c).sum(axis=1).max())
+    out = torch.full((1,), -1, dtype=torch.int64, device="cuda")
+    F.fxpq_code_l1max(torch.empty(8, dtype=torch.float16, device="cuda"), 0, 8, out)
+    assert int(out.item()) == 0
 
 
 def test_gemm_entry_point(F):
