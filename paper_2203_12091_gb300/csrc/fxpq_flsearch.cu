@@ -119,6 +119,24 @@ struct KeyInfo {
     unsigned validR, validRb;  // bit jj set: slot jj (j = jj - 1) is needed for this key
 };
 
+// Boundary sums of a narrow wordlength range (at most two boundary positions j = jb_lo, jb_lo + 1):
+// per position the remainder mask and modulus of y's fraction and the saturation threshold of M.
+struct RbC {
+    unsigned mask[2], full[2], thr[2];
+};
+
+__device__ __forceinline__ RbC make_rbc(const FsParams& P) {
+    RbC c;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int j = min(P.jb_lo + i, 15);  // j in [0, 15]; a position past jb_hi is never flushed
+        c.full[i] = 1u << (23 - j);
+        c.mask[i] = c.full[i] - 1u;
+        c.thr[i] = ((2u << j) - 1u) << (23 - j);
+    }
+    return c;
+}
+
 __device__ __forceinline__ KeyInfo key_info(int key, const FsParams& P) {
     KeyInfo k;
     k.sg = key >> 8;
@@ -138,26 +156,56 @@ __device__ __forceinline__ KeyInfo key_info(int key, const FsParams& P) {
     return k;
 }
 
-// Per-lane accumulators of the warp's current key; NS slots cover j = -1 .. NS-2.
-template <int NS>
+// Per-lane accumulators of the warp's current key; NS slots cover j = -1 .. NS-2.  Boundary sums:
+// NRB = NS slots indexed like r (any wordlength range), or NRB = 2 slots for j = jb_lo, jb_lo + 1.
+template <int NS, int NRB>
 struct Acc {
     u64 r[NS];
-    u64 rb[NS];
+    u64 rb[NRB];
     u64 s1, s2;
     unsigned n;
 };
 
-template <int NS>
-__device__ __forceinline__ void acc_zero(Acc<NS>& a) {
+template <int NS, int NRB>
+__device__ __forceinline__ void acc_zero(Acc<NS, NRB>& a) {
 #pragma unroll
-    for (int jj = 0; jj < NS; ++jj) a.r[jj] = a.rb[jj] = 0ull;
+    for (int jj = 0; jj < NS; ++jj) a.r[jj] = 0ull;
+#pragma unroll
+    for (int i = 0; i < NRB; ++i) a.rb[i] = 0ull;
     a.s1 = a.s2 = 0ull;
     a.n = 0u;
 }
 
+// Narrow wordlength range: every remainder slot is computed without branches (slots the key does not
+// use are never flushed).  The rounding error's magnitude is min(t, 2^p - t) for the fraction t of y
+// in units of 2^-p, whichever way a tie rounds, so the parity of y's integer part is not needed.
+template <int NS>
+__device__ __forceinline__ void acc_add_narrow(Acc<NS, 2>& a, unsigned M, bool rb_on, const RbC& c) {
+    a.n += 1u;
+    a.s1 += M;
+    a.s2 += (u64)M * M;
+#pragma unroll
+    for (int jj = 0; jj < NS; ++jj) {
+        const unsigned full = 1u << (24 - jj);  // p = 23 - j bits below y's binary point
+        const unsigned t = M & (full - 1u);
+        const unsigned r = min(t, full - t);
+        a.r[jj] += (u64)r * r;
+    }
+    if (rb_on) {
+        // boundary: saturated iff M >= thr, error (M - thr) u_E; otherwise the rounding error
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const unsigned t = M & c.mask[i];
+            const unsigned r = min(t, c.full[i] - t);
+            const unsigned rb = M >= c.thr[i] ? M - c.thr[i] : r;
+            a.rb[i] += (u64)rb * rb;
+        }
+    }
+}
+
 // Add one element (significand M of the warp's current key) to this lane's accumulators.
 template <int NS>
-__device__ __forceinline__ void acc_add(Acc<NS>& a, unsigned M, const KeyInfo& k) {
+__device__ __forceinline__ void acc_add(Acc<NS, NS>& a, unsigned M, const KeyInfo& k) {
     a.n += 1u;
     a.s1 += M;
     a.s2 += (u64)M * M;
@@ -181,8 +229,8 @@ __device__ __forceinline__ void acc_add(Acc<NS>& a, unsigned M, const KeyInfo& k
     }
 }
 
-template <int NS>
-__device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS>& a, int key, const KeyInfo& k, const FsParams& P,
+template <int NS, int NRB>
+__device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS, NRB>& a, int key, const KeyInfo& k, const FsParams& P,
                                           unsigned lane) {
     const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
     const u64 s1 = warp_sum64(a.s1), s2 = warp_sum64(a.s2);
@@ -198,9 +246,19 @@ __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS>& a, int key, const
             const u64 v = warp_sum64(a.r[jj]);
             if (lane == 0) sadd64(sm.r[k.sg][jj][fi], v);
         }
-        if ((k.validRb >> jj) & 1u) {
-            const u64 v = warp_sum64(a.rb[jj]);
+        if (NRB == NS && ((k.validRb >> jj) & 1u)) {
+            const u64 v = warp_sum64(a.rb[jj < NRB ? jj : 0]);
             if (lane == 0) sadd64(sm.rb[jj][fi], v);
+        }
+    }
+    if (NRB == 2) {
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int jj = P.jb_lo + i + 1;
+            if (jj < NJ && ((k.validRb >> jj) & 1u)) {
+                const u64 v = warp_sum64(a.rb[i]);
+                if (lane == 0) sadd64(sm.rb[jj][jj - 1 - k.E - P.fl_lo], v);
+            }
         }
     }
 }
@@ -229,7 +287,7 @@ __device__ __forceinline__ void load16(const FsParams& P, long long tb, int sub,
     }
 }
 
-template <bool VEC, int NS>
+template <bool VEC, int NS, int NRB>
 __global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams P) {
     extern __shared__ __align__(16) unsigned char fs_smem_raw[];
     FsSmem& sm = *reinterpret_cast<FsSmem*>(fs_smem_raw);
@@ -247,6 +305,7 @@ __global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams 
 
     const long long start = (long long)blockIdx.x * P.chunk;
     const long long end = min(start + (long long)P.chunk, P.n);
+    const RbC rbc = make_rbc(P);
     for (long long tb = start; tb < end; tb += TILE) {
         // ---- A+B: read the tile (16 elements per thread per sub-round), stats, key histogram
         for (int sub = 0; sub < TILE / 4096; ++sub) {
@@ -316,7 +375,7 @@ __global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams 
         const int L = (int)sm.live;
         const int per = ((L + FS_WARPS * 32 - 1) / (FS_WARPS * 32)) * 32;
         const int w0 = (int)warp * per, w1 = min(w0 + per, L);
-        Acc<NS> acc;
+        Acc<NS, NRB> acc;
         acc_zero(acc);
         int ck = -1;
         KeyInfo ki;
@@ -341,7 +400,12 @@ __global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams 
                     ck = kk;
                     ki = key_info(ck, P);
                 }
-                if ((in >> lane) & 1u) acc_add(acc, M, ki);
+                if ((in >> lane) & 1u) {
+                    if constexpr (NRB == 2)
+                        acc_add_narrow(acc, M, ki.validRb != 0u, rbc);
+                    else
+                        acc_add(acc, M, ki);
+                }
                 rem &= ~in;
             }
         }
@@ -627,10 +691,12 @@ void st_attr_once() {
     std::lock_guard<std::mutex> lk(g_fs_attr_mu);
     if (g_fs_attr_done) return;
     const int sb = (int)sizeof(FsSmem);
-    cudaFuncSetAttribute(fl_search_bins_kernel<true, 10>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<false, 10>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<true, 10, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<false, 10, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
     g_fs_attr_done = true;
 }
 }  // namespace
@@ -676,17 +742,23 @@ extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_si
     if (n > 0) {
         const int grid = (int)((n + chunk - 1) / chunk);
         const bool vec = aligned(d_x, 16);
-        const bool small = k_hi <= 9;  // slots j = -1 .. k_hi - 1 suffice
+        const bool small = k_hi <= 9;                     // slots j = -1 .. k_hi - 1 suffice
+        const bool narrow = P.jb_hi - P.jb_lo + 1 <= 2;  // at most two boundary positions
         st_attr_once();
         const size_t sb = sizeof(FsSmem);
-        if (vec && small)
-            fl_search_bins_kernel<true, 10><<<grid, FS_THREADS, sb, s>>>(P);
-        else if (vec)
-            fl_search_bins_kernel<true, NJ><<<grid, FS_THREADS, sb, s>>>(P);
-        else if (small)
-            fl_search_bins_kernel<false, 10><<<grid, FS_THREADS, sb, s>>>(P);
-        else
-            fl_search_bins_kernel<false, NJ><<<grid, FS_THREADS, sb, s>>>(P);
+#define FXPQ_FS_LAUNCH(V)                                                       \
+    if (narrow && small)                                                        \
+        fl_search_bins_kernel<V, 10, 2><<<grid, FS_THREADS, sb, s>>>(P);        \
+    else if (narrow)                                                            \
+        fl_search_bins_kernel<V, NJ, 2><<<grid, FS_THREADS, sb, s>>>(P);        \
+    else                                                                        \
+        fl_search_bins_kernel<V, NJ, NJ><<<grid, FS_THREADS, sb, s>>>(P);
+        if (vec) {
+            FXPQ_FS_LAUNCH(true)
+        } else {
+            FXPQ_FS_LAUNCH(false)
+        }
+#undef FXPQ_FS_LAUNCH
         const fxpq_status st = after_launch("fl_search_bins");
         if (st != FXPQ_OK) return st;
     }
