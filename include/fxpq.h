@@ -106,7 +106,8 @@ FXPQ_API fxpq_status fxpq_code_l1max(const void* d_codes, int64_t rows, int64_t 
 
 /* Quantize + transpose + pack fp32 images NCHW -> NHWC fp16 code tensor with the channel count
  * padded to c_pad (a multiple of 8, >= C) with zero codes: the FxP-QLayer inserted at the input
- * of the network (Sec. IV-A.2).  d_y holds planes x [N, H, W, c_pad] fp16 values. */
+ * of the network (Sec. IV-A.2).  d_y (16-byte aligned) holds planes x [N, H, W, c_pad] fp16
+ * values. */
 FXPQ_API fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, int32_t C, int32_t H, int32_t W,
                                  fxpq_fmt f, int32_t c_pad, void* d_y, void* stream);
 

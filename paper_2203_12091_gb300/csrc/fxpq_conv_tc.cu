@@ -220,68 +220,32 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
                  : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-}
-
-__device__ __forceinline__ void tmem_ld32u(uint32_t taddr, uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_ld16u(uint32_t taddr, uint32_t (&r)[16]) {
+// Loads / stores without their completion wait, so that several TMEM accesses share one round trip.
+// After tmem_wait_ld(), reg_fence() on each loaded array orders every use of its registers after the
+// wait (the empty asm redefines them).
+__device__ __forceinline__ void tmem_ld16_nw(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
         "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
-
-__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t (&r)[16]) {
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void reg_fence(uint32_t (&r)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
+}
+__device__ __forceinline__ void tmem_st16_nw(uint32_t taddr, const uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
         "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
         "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
         "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
         : "memory");
-    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
-
-__device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t (&r)[32]) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
-        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]),
-        "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
-        "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
-        : "memory");
-    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
 // Final epilogue of 32 consecutive output channels k0.. of row m (generic outputs: two-plane codes,
 // int64 accumulators, fp32 calibration images): bias alignment, ReLU, FxP-QLayer.
 template <typename ACC>
@@ -594,24 +558,31 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     const int cb = cw * CPW + c;
                     const int k0 = tn * BN + cb * 32;
                     const uint32_t run_col = run_base + cb * 32;
+                    // One TMEM round trip per load batch: the fp32 group sums and, after the first group,
+                    // the integer running sums are loaded together; the running-sum stores share one
+                    // completion wait.
                     ACC acc[32];
-                    {
-                        float f[32];
-                        tmem_ld32(lane_base + buf * BN + cb * 32, f);
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) acc[j] = ((ACC)__float2int_rn(f[j])) << shift;
-                    }
                     if (sizeof(ACC) == 8) {
                         // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
 #pragma unroll
                         for (int hf = 0; hf < 2; ++hf) {
-                            uint32_t lo[16], hi[16];
+                            uint32_t f16[16], lo[16], hi[16];
+                            tmem_ld16_nw(lane_base + buf * BN + cb * 32 + 16 * hf, f16);
                             if (!first) {
-                                tmem_ld16u(lane_base + run_col + 16 * hf, lo);
-                                tmem_ld16u(lane_base + run_col + BN + 16 * hf, hi);
+                                tmem_ld16_nw(lane_base + run_col + 16 * hf, lo);
+                                tmem_ld16_nw(lane_base + run_col + BN + 16 * hf, hi);
+                            }
+                            tmem_wait_ld();
+                            reg_fence(f16);
+                            if (!first) {
+                                reg_fence(lo);
+                                reg_fence(hi);
+                            }
 #pragma unroll
-                                for (int j = 0; j < 16; ++j)
-                                    acc[16 * hf + j] += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
+                            for (int j = 0; j < 16; ++j) {
+                                ACC v = ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << shift;
+                                if (!first) v += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
+                                acc[16 * hf + j] = v;
                             }
                             if (!last) {
 #pragma unroll
@@ -619,23 +590,34 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                     lo[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
                                     hi[j] = (uint32_t)((unsigned long long)acc[16 * hf + j] >> 32);
                                 }
-                                tmem_st16u(lane_base + run_col + 16 * hf, lo);
-                                tmem_st16u(lane_base + run_col + BN + 16 * hf, hi);
+                                tmem_st16_nw(lane_base + run_col + 16 * hf, lo);
+                                tmem_st16_nw(lane_base + run_col + BN + 16 * hf, hi);
                             }
                         }
+                        if (!last) tmem_wait_st();
                     } else {
-                        if (!first) {
-                            uint32_t lo[32];
-                            tmem_ld32u(lane_base + run_col, lo);
+                        // int32 running sums, 16-column halves (keeps the live registers low)
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) acc[j] += (ACC)(int)lo[j];
-                        }
-                        if (!last) {
-                            uint32_t lo[32];
+                        for (int hf = 0; hf < 2; ++hf) {
+                            uint32_t f16[16], run[16];
+                            tmem_ld16_nw(lane_base + buf * BN + cb * 32 + 16 * hf, f16);
+                            if (!first) tmem_ld16_nw(lane_base + run_col + 16 * hf, run);
+                            tmem_wait_ld();
+                            reg_fence(f16);
+                            if (!first) reg_fence(run);
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) lo[j] = (uint32_t)(unsigned long long)acc[j];
-                            tmem_st32u(lane_base + run_col, lo);
+                            for (int j = 0; j < 16; ++j) {
+                                ACC v = ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << shift;
+                                if (!first) v += (ACC)(int)run[j];
+                                acc[16 * hf + j] = v;
+                            }
+                            if (!last) {
+#pragma unroll
+                                for (int j = 0; j < 16; ++j) run[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
+                                tmem_st16_nw(lane_base + run_col + 16 * hf, run);
+                            }
                         }
+                        if (!last) tmem_wait_st();
                     }
                     if (c == CPW - 1) {
                         // every chunk of this warp is out of the accumulator buffer: free it for the

@@ -68,18 +68,73 @@ __global__ void quantize_rows_f16_kernel(const float* __restrict__ x, long long 
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
 
-// NCHW fp32 -> NHWC fp16 codes, channels padded to Cp; one thread per pixel
+// Unpadded rows (C == Cp): the tensor is n = rows * C contiguous codes, n % 8 == 0; 8 codes per
+// thread from two 16-byte loads, one 16-byte store per plane.
+__global__ void quantize_rows_vec8_kernel(const float4* __restrict__ x, long long n8, int planes, QParams p,
+                                          uint4* __restrict__ out) {
+    bool bad = false;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += stride) {
+        const float4 a = __ldg(x + 2 * i), b = __ldg(x + 2 * i + 1);
+        const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int c0 = quant1(v[2 * e], p, bad), c1 = quant1(v[2 * e + 1], p, bad);
+            if (planes == 1) {
+                hi[e] = (uint32_t)__half_as_ushort(__int2half_rn(c0)) |
+                        ((uint32_t)__half_as_ushort(__int2half_rn(c1)) << 16);
+            } else {
+                __half h0, l0, h1, l1;
+                split_limbs(c0, h0, l0);
+                split_limbs(c1, h1, l1);
+                hi[e] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+                lo[e] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+            }
+        }
+        out[i] = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        if (planes == 2) out[n8 + i] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    }
+    if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
+}
+
+// NCHW fp32 -> NHWC fp16 codes, channels padded to Cp (a multiple of 8); one thread per pixel, each
+// group of 8 channels written as one 16-byte store per plane
 __global__ void quantize_images_kernel(const float* __restrict__ x, int N, int C, int H, int W, int Cp, int planes,
                                        QParams p, __half* __restrict__ out) {
     bool bad = false;
-    long long npix = (long long)N * H * W;
-    long long stride = (long long)gridDim.x * blockDim.x;
+    const long long hw = (long long)H * W;
+    const long long npix = (long long)N * hw;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    uint4* o = reinterpret_cast<uint4*>(out);
+    const long long plane8 = npix * Cp / 8;  // plane stride in 16-byte units
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < npix; i += stride) {
-        long long n = i / ((long long)H * W);
-        long long hw = i - n * H * W;
-        for (int c = 0; c < Cp; ++c) {
-            int code = c < C ? quant1(x[(n * C + c) * (long long)H * W + hw], p, bad) : 0;
-            code_put(out, i * Cp + c, planes, npix * Cp, code);
+        const long long n = i / hw;
+        const long long pix = i - n * hw;
+        for (int c0 = 0; c0 < Cp; c0 += 8) {
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                int code[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int c = c0 + 2 * e + h;
+                    code[h] = c < C ? quant1(__ldg(x + (n * C + c) * hw + pix), p, bad) : 0;
+                }
+                if (planes == 1) {
+                    hi[e] = (uint32_t)__half_as_ushort(__int2half_rn(code[0])) |
+                            ((uint32_t)__half_as_ushort(__int2half_rn(code[1])) << 16);
+                } else {
+                    __half h0, l0, h1, l1;
+                    split_limbs(code[0], h0, l0);
+                    split_limbs(code[1], h1, l1);
+                    hi[e] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+                    lo[e] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+                }
+            }
+            const long long q = (i * Cp + c0) / 8;
+            o[q] = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+            if (planes == 2) o[plane8 + q] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
     }
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
@@ -185,6 +240,12 @@ extern "C" fxpq_status fxpq_quantize_rows(const float* d_x, int64_t rows, int32_
     if (rows == 0) return FXPQ_OK;
     if (!d_x || !d_y) return FXPQ_ERR_INVALID_ARG;
     QParams p = make_qparams(f);
+    if (C == Cp && aligned(d_x, 16) && aligned(d_y, 16)) {
+        const long long n8 = rows * (long long)C / 8;
+        quantize_rows_vec8_kernel<<<grid_for(n8, 256), 256, 0, as_stream(stream)>>>(
+            reinterpret_cast<const float4*>(d_x), n8, planes_of(f), p, static_cast<uint4*>(d_y));
+        return after_launch("quantize_rows_vec8");
+    }
     quantize_rows_f16_kernel<<<grid_for(rows * Cp, 256), 256, 0, as_stream(stream)>>>(
         d_x, rows, C, Cp, planes_of(f), p, static_cast<__half*>(d_y));
     return after_launch("quantize_rows_f16");
@@ -194,7 +255,7 @@ extern "C" fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, in
                                             fxpq_fmt f, int32_t c_pad, void* d_y, void* stream) {
     if (N < 0 || C < 1 || H < 1 || W < 1 || c_pad < C || (c_pad % 8) || !fmt_ok(f)) return FXPQ_ERR_INVALID_ARG;
     if (N == 0) return FXPQ_OK;
-    if (!d_x_nchw || !d_y) return FXPQ_ERR_INVALID_ARG;
+    if (!d_x_nchw || !d_y || !aligned(d_y, 16)) return FXPQ_ERR_INVALID_ARG;
     QParams p = make_qparams(f);
     long long npix = (long long)N * H * W;
     quantize_images_kernel<<<grid_for(npix, 256), 256, 0, as_stream(stream)>>>(d_x_nchw, N, C, H, W, c_pad,
