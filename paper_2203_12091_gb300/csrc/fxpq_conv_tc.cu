@@ -64,7 +64,9 @@ struct TcParams {
     CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}
     int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
     int nbuf;            // fp32 accumulator buffers in TMEM: 2, or 1 when BN = 256 needs running sums
-    int patch;           // 1: a tile is a TH x TW patch of one image, the A tile comes by TMA
+    int patch;           // a tile is a TH x TW patch of one image and the A tile comes by TMA:
+                         // 1: Cp % 64 == 0 (one 64-channel box per k-block, 128-byte swizzle);
+                         // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle)
     int TH, TW;          // patch shape (TH * TW = 128)
     int tiles_p, tiles_q;  // patches per image along P and Q
     ConvArgs a;
@@ -187,6 +189,17 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
+// Shared-memory matrix descriptor, K-major without swizzle: core matrices of 8 rows x 16 bytes;
+// lbo = bytes between core matrices adjacent in K, sbo = bytes between 8-row groups.
+__device__ __forceinline__ uint64_t make_sdesc_noswz(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1u << 46;  // descriptor version; layout type 0 = no swizzle
+    return d;
+}
+
 __device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr) {
     uint64_t d = 0;
     d |= (uint64_t)((saddr >> 4) & 0x3FFFu);          // start address
@@ -391,8 +404,12 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         // ============================================================ producer, patch tiles
         // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
         // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
+        // Cp == 8: a k-block is 8 taps of 8 channels; tap tl's box {8, TW, TH} lands at byte
+        // 2048 tl of the stage (a 16-byte K column of the no-swizzle layout), and taps past R*S
+        // are boxes wholly outside the tensor (zero filled).
         if (threadIdx.x == 0) {
-            const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * 128);
+            const bool narrow = P.patch == 2;
+            const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
@@ -412,8 +429,18 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                         const int rr = tp / a.S, ss = tp - rr * a.S;
                         const uint32_t fb = full0 + 8 * stage;
                         mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
-                        tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
-                                    g.a_plane, fb);
+                        if (narrow) {
+                            for (int tl = 0; tl < 8; ++tl) {
+                                const int tap = kb * 8 + tl;
+                                const bool in = tap < a.R * a.S;
+                                const int r8 = in ? tap / a.S : 0, s8 = in ? tap - (tap / a.S) * a.S : 0;
+                                tma_load_5d(smem_u32(sA + stage * A_BYTES + tl * 2048), &P.tmap_x, in ? 0 : 8,
+                                            wq0 + s8, hp0 + r8, n_img, g.a_plane, fb);
+                            }
+                        } else {
+                            tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
+                                        g.a_plane, fb);
+                        }
                         tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, f, tn * BN, g.w_plane, fb);
                         ++it;
                         if (++stage == TC_STAGES) {
@@ -698,7 +725,11 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         // ============================================================ MMA issue (one thread of MMA_WARP)
         // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
         // (address >> 4, 14 bits) without carry since shared addresses stay below 256 KB.
-        const uint64_t adesc0 = make_sdesc(smem_u32(sA)), bdesc0 = make_sdesc(smem_u32(sB));
+        // 8-channel patch tiles: no-swizzle A, one 16-element k step = two taps = 4096 bytes
+        const bool narrow_a = P.patch == 2;
+        const uint64_t adesc0 = narrow_a ? make_sdesc_noswz(smem_u32(sA), 2048, 128) : make_sdesc(smem_u32(sA));
+        const uint32_t a_kstep = narrow_a ? 4096u >> 4 : 2u;
+        const uint64_t bdesc0 = make_sdesc(smem_u32(sB));
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
@@ -723,7 +754,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     const uint64_t bd = bdesc0 + (uint64_t)((stage * B_BYTES) >> 4);
 #pragma unroll
                     for (int kk = 0; kk < TC_BK / 16; ++kk) {
-                        tc_mma(d, ad + 2 * kk, bd + 2 * kk, IDESC, accum);
+                        tc_mma(d, ad + a_kstep * kk, bd + 2 * kk, IDESC, accum);
                         accum = 1;
                     }
                     tc_commit(empty0 + 8 * stage);
@@ -881,9 +912,11 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
-        // patch tiles for stride-1 layers whose taps are whole 64-channel blocks
+        // patch tiles for stride-1 layers whose taps are whole 64-channel blocks, or 8-channel inputs
+        // (a k-block of 8 taps)
         P.patch = 0;
-        if (a.stride == 1 && P.cp64 && a.P > 0 && a.Q > 0 && a.N > 0 && !conv_path_is("tc_rows")) {
+        const bool narrow = a.Cp == 8;
+        if (a.stride == 1 && (P.cp64 || narrow) && a.P > 0 && a.Q > 0 && a.N > 0 && !conv_path_is("tc_rows")) {
             int best_tw = 0, best_th = 0;
             long long best = 0;
             for (int tw = a.Q < TC_BM ? a.Q : TC_BM; tw >= 1; --tw) {
@@ -898,12 +931,14 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                                              (cuuint64_t)a.px};
                 const cuuint64_t xstrides[4] = {(cuuint64_t)a.Cp * 2, (cuuint64_t)a.W * a.Cp * 2,
                                                 (cuuint64_t)a.H * a.W * a.Cp * 2, (cuuint64_t)a.x_ps * 2};
-                const cuuint32_t xbox[5] = {(cuuint32_t)TC_BK, (cuuint32_t)best_tw, (cuuint32_t)best_th, 1, 1};
+                const cuuint32_t xbox[5] = {(cuuint32_t)(narrow ? 8 : TC_BK), (cuuint32_t)best_tw,
+                                            (cuuint32_t)best_th, 1, 1};
                 const cuuint32_t es5[5] = {1, 1, 1, 1, 1};
                 if (enc(&P.tmap_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.x), xdims, xstrides,
-                        xbox, es5, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        xbox, es5, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        narrow ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
-                    P.patch = 1;
+                    P.patch = narrow ? 2 : 1;
                     P.TW = best_tw;
                     P.TH = best_th;
                     P.tiles_p = (a.P + best_th - 1) / best_th;

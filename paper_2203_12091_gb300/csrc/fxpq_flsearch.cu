@@ -16,7 +16,7 @@
 // All sums are integers; the finalize kernel adds one candidate's terms in a 768-bit fixed-point
 // accumulator and rounds once.
 //
-// Pass structure (one HBM read of x).  Each block sorts a tile of 16384 elements by (sign, E) in
+// Pass structure (one HBM read of x).  Each block sorts a tile of 8192 elements by (sign, E) in
 // shared memory (histogram, scan, scatter; the scatter re-reads the tile from L2); each warp then
 // walks a contiguous run of the sorted tile, so runs of equal
 // exponent are accumulated in registers (one slot per j = q) and reduced across the warp only when
@@ -38,7 +38,8 @@ constexpr int MAXFL = 32;  // candidates per wordlength
 constexpr int MAXK = 15;   // k in [2, 16]
 constexpr int FS_THREADS = 256;
 constexpr int FS_WARPS = FS_THREADS / 32;
-constexpr int TILE = 16384;  // 64 elements per thread, read in sub-rounds of 16
+constexpr int TILE = 8192;  // 32 elements per thread, read in sub-rounds of 16
+constexpr int FS_BLOCKS_PER_SM = 3;
 constexpr int CHUNK_MAX = 65536;  // per-block element cap: keeps every 64-bit block bin below 2^64
 
 struct FsSmem {
@@ -137,22 +138,22 @@ __device__ __forceinline__ RbC make_rbc(const FsParams& P) {
     return c;
 }
 
+__device__ __forceinline__ unsigned slot_mask(int jlo, int jhi) {
+    // slots jj = j + 1 for j in [jlo, jhi] (empty when jhi < jlo)
+    if (jhi < jlo) return 0u;
+    return ((2u << (jhi + 1)) - 1u) & ~((1u << (jlo + 1)) - 1u);
+}
+
 __device__ __forceinline__ KeyInfo key_info(int key, const FsParams& P) {
     KeyInfo k;
     k.sg = key >> 8;
     const int eb = key & 255;
     k.E = eb ? eb - 127 : -126;
-    k.validR = 0u;
-    k.validRb = 0u;
+    // candidate FL in [fl_lo, fl_lo + nfl) puts j = E + FL in [E + fl_lo, E + fl_lo + nfl - 1]
+    const int cand_lo = k.E + P.fl_lo, cand_hi = k.E + P.fl_lo + P.nfl - 1;
     const int jmax = k.sg ? P.jmax_neg : P.jmax_pos;
-#pragma unroll
-    for (int jj = 0; jj < NJ; ++jj) {
-        const int j = jj - 1;
-        const int fi = j - k.E - P.fl_lo;
-        if (fi < 0 || fi >= P.nfl) continue;
-        if (j <= jmax) k.validR |= 1u << jj;
-        if (k.sg == 0 && j >= P.jb_lo && j <= P.jb_hi) k.validRb |= 1u << jj;
-    }
+    k.validR = slot_mask(max(-1, cand_lo), min(min(jmax, NJ - 2), cand_hi));
+    k.validRb = k.sg == 0 ? slot_mask(max(max(P.jb_lo, 0), cand_lo), min(min(P.jb_hi, NJ - 2), cand_hi)) : 0u;
     return k;
 }
 
@@ -229,26 +230,27 @@ __device__ __forceinline__ void acc_add(Acc<NS, NS>& a, unsigned M, const KeyInf
     }
 }
 
+// Warp totals of the current key's accumulators into the block bins.  The sums are warp-uniform;
+// the shared-memory atomics are spread over the lanes (lane 0: count, 1-2: moments, 3..: slots) so
+// that they do not queue behind one another.
 template <int NS, int NRB>
 __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS, NRB>& a, int key, const KeyInfo& k, const FsParams& P,
                                           unsigned lane) {
     const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
     const u64 s1 = warp_sum64(a.s1), s2 = warp_sum64(a.s2);
-    if (lane == 0) {
-        atomicAdd(&sm.pn[key], n);
-        sadd64(sm.ps1[key], s1);
-        sadd64(sm.ps2[key], s2);
-    }
+    if (lane == 0) atomicAdd(&sm.pn[key], n);
+    if (lane == 1) sadd64(sm.ps1[key], s1);
+    if (lane == 2) sadd64(sm.ps2[key], s2);
 #pragma unroll
     for (int jj = 0; jj < NS; ++jj) {
         const int fi = jj - 1 - k.E - P.fl_lo;
         if ((k.validR >> jj) & 1u) {
             const u64 v = warp_sum64(a.r[jj]);
-            if (lane == 0) sadd64(sm.r[k.sg][jj][fi], v);
+            if (lane == (unsigned)((3 + jj) & 31)) sadd64(sm.r[k.sg][jj][fi], v);
         }
         if (NRB == NS && ((k.validRb >> jj) & 1u)) {
             const u64 v = warp_sum64(a.rb[jj < NRB ? jj : 0]);
-            if (lane == 0) sadd64(sm.rb[jj][fi], v);
+            if (lane == (unsigned)((3 + NS + jj) & 31)) sadd64(sm.rb[jj][fi], v);
         }
     }
     if (NRB == 2) {
@@ -257,7 +259,7 @@ __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS, NRB>& a, int key, 
             const int jj = P.jb_lo + i + 1;
             if (jj < NJ && ((k.validRb >> jj) & 1u)) {
                 const u64 v = warp_sum64(a.rb[i]);
-                if (lane == 0) sadd64(sm.rb[jj][jj - 1 - k.E - P.fl_lo], v);
+                if (lane == (unsigned)((3 + NS + i) & 31)) sadd64(sm.rb[jj][jj - 1 - k.E - P.fl_lo], v);
             }
         }
     }
@@ -288,7 +290,7 @@ __device__ __forceinline__ void load16(const FsParams& P, long long tb, int sub,
 }
 
 template <bool VEC, int NS, int NRB>
-__global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams P) {
+__global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2) fl_search_bins_kernel(FsParams P) {
     extern __shared__ __align__(16) unsigned char fs_smem_raw[];
     FsSmem& sm = *reinterpret_cast<FsSmem*>(fs_smem_raw);
     const unsigned lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
@@ -380,14 +382,26 @@ __global__ void __launch_bounds__(FS_THREADS, 2) fl_search_bins_kernel(FsParams 
         int ck = -1;
         KeyInfo ki;
         ki.sg = 0, ki.E = 0, ki.validR = ki.validRb = 0u;
+        // one step of lookahead: the next group's shared-memory load is in flight while this one is
+        // accumulated
+        float xn = w0 + (int)lane < w1 ? sm.sorted[w0 + lane] : 0.0f;
         for (int pos = w0; pos < w1; pos += 32) {
             const int p = pos + (int)lane;
             const bool live = p < w1;
-            const float xv = live ? sm.sorted[p] : 0.0f;
+            const float xv = xn;
+            xn = p + 32 < w1 ? sm.sorted[p + 32] : 0.0f;
             const int kx = live ? key_of(xv) : NKEY;
             const unsigned u = __float_as_uint(xv);
             const unsigned eb = (u >> 23) & 0xFFu;
             const unsigned M = eb ? ((u & 0x7FFFFFu) | 0x800000u) : (u & 0x7FFFFFu);
+            // common case: every lane is live and continues the current key
+            if (__all_sync(0xFFFFFFFFu, kx == ck)) {
+                if constexpr (NRB == 2)
+                    acc_add_narrow(acc, M, ki.validRb != 0u, rbc);
+                else
+                    acc_add(acc, M, ki);
+                continue;
+            }
             unsigned rem = __ballot_sync(0xFFFFFFFFu, live);
             while (rem) {
                 const int kk = __shfl_sync(0xFFFFFFFFu, kx, __ffs(rem) - 1);
@@ -724,7 +738,10 @@ extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_si
     FsParams P;
     P.x = d_x;
     P.n = n;
-    long long per = (n + 152LL * 4 - 1) / (152LL * 4);
+    // whole waves of resident blocks, each chunk at most CHUNK_MAX elements
+    const long long resident = 152LL * FS_BLOCKS_PER_SM;
+    const long long waves = (n + resident * CHUNK_MAX - 1) / (resident * CHUNK_MAX);
+    const long long per = (n + resident * waves - 1) / (resident * waves);
     long long chunk = (per + TILE - 1) / TILE * TILE;
     if (chunk < TILE) chunk = TILE;
     if (chunk > CHUNK_MAX) chunk = CHUNK_MAX;

@@ -116,6 +116,9 @@ CASES = [
     (2, 9, 16, 264, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),        # ragged K, row tiles
     (2, 8, 64, 256, 3, 1, 1, (8, 0, 4), (8, 1, 7), None, True, 2, None),               # fp32 image
     (2, 8, 64, 256, 3, 1, 1, (8, 0, 4), (8, 1, 7), (16, 15), False, 1, None),          # int64 accumulators
+    # 8-channel stride-1 inputs: patch tiles with one box per tap (VGG conv1_1-like, two limbs)
+    (2, 20, 3, 16, 5, 1, 2, (16, 1, 12), (16, 1, 14), (16, 20), True, 0, (8, 0, 3)),
+    (3, 16, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 14), (16, 22), True, 0, (4, 0, 2)),
 ]
 
 
