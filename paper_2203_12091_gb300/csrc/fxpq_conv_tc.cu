@@ -328,6 +328,37 @@ __device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, in
     return min(max((N + e.hm1 + x) >> e.sh, e.lo), e.hi);
 }
 
+// The same FxP-QLayer on 64-bit values (wide sums, two-limb layers), valid for 1 <= sh <= 62: the
+// bias alignment is v = (acc << dr) + (B << dl) (one of dl, dr is zero), and the code is
+// round_half_even(v / 2^sh) = floor((v + 2^(sh-1) - 1 + ((v >> sh) & 1)) / 2^sh), clipped.  The host
+// keeps |v| < 2^62, so the rounding sum cannot overflow.
+struct Epi64 {
+    int dl, dr, sh;
+    long long hm1, floor;
+    int lo, hi, has_bias, ok;  // ok: 1 <= sh <= 62 (otherwise the generic path runs)
+};
+
+__device__ __forceinline__ Epi64 make_epi64(const ConvArgs& a) {
+    Epi64 e;
+    e.dl = a.delta > 0 ? a.delta : 0;
+    e.dr = a.delta < 0 ? -a.delta : 0;
+    e.sh = a.sh;
+    e.ok = a.sh >= 1 && a.sh <= 62;
+    e.hm1 = e.ok ? (1LL << (a.sh - 1)) - 1 : 0;
+    e.floor = a.relu ? 0LL : LLONG_MIN;
+    e.lo = (int)a.lo;
+    e.hi = (int)a.hi;
+    e.has_bias = a.has_bias;
+    return e;
+}
+
+__device__ __forceinline__ int epi64_code(const Epi64& e, long long acc, int32_t b) {
+    long long v = (acc << e.dr) + ((long long)b << e.dl);
+    v = max(v, e.floor);
+    const long long c = (v + e.hm1 + ((v >> e.sh) & 1)) >> e.sh;
+    return (int)min(max(c, (long long)e.lo), (long long)e.hi);
+}
+
 // Two codes in [-512, 511] as a packed fp16 pair: 1536 + c has the bit pattern 0x6600 + c (the
 // binade [1024, 2048) has unit spacing), and one packed subtraction of 1536 leaves c exactly.
 __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
@@ -554,7 +585,6 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         // [nbuf BN, nbuf BN + BN * words), words = 1 (int32) or 2 (int64 as lo / hi column blocks).
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
         const uint32_t run_base = (uint32_t)(nbuf * BN);
-        const Epi32 e32 = make_epi32(a);
         uint32_t u = 0;  // tiles written through the staging buffer so far
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
@@ -655,7 +685,11 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     if (!last) continue;
                     if (P.fast_store) {
                         // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
+                        // (the epilogue constants are rebuilt here from the parameters rather than kept
+                        // live across the tile loop)
                         uint32_t w[16];
+                        const Epi32 e32 = make_epi32(a);
+                        const Epi64 e64 = make_epi64(a);
                         if (sizeof(ACC) == 4 && a.v32) {
 #pragma unroll
                             for (int j = 0; j < 16; ++j) {
@@ -666,6 +700,18 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                     const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
                                     c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
                                                        (b & e32.fmask) != 0 ? 1 : 0);
+                                }
+                                w[j] = pack_codes_f16(c2[0], c2[1]);
+                            }
+                        } else if (e64.ok) {
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                int c2[2];
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    const int k = k0 + 2 * j + h;
+                                    const int32_t b = (e64.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                    c2[h] = epi64_code(e64, (long long)acc[2 * j + h], b);
                                 }
                                 w[j] = pack_codes_f16(c2[0], c2[1]);
                             }
@@ -898,6 +944,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     else if (a.K > 128 && !conv_path_is("tc_bn128") &&
              (conv_path_is("tc_bn256") || (a.K % 256 == 0 && row_tiles_est * (a.K / 256) >= sms)))
         BN = 256;
+    // too few 128-column tiles to occupy every SM (small batches, FC layers): 64-column tiles double
+    // the CTA count
+    if (BN == 128 && row_tiles_est * ((a.K + 127) / 128) < sms) BN = 64;
     // BN = 256 fills TMEM with two accumulator buffers; with several exact groups per tile it keeps one
     // buffer and the integer running sums
     P.nbuf = (BN == 256 && P.n_groups > 1) ? 1 : 2;
