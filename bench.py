@@ -294,8 +294,10 @@ def run_reference(args):
 
 def run_kernel(args):
     """Single-kernel timing cases (also the targets of the ncu captures summarised in profiles/):
-    conv     : VGG-16 conv3_1-shaped C-Block, batch 64, 56x56x128 -> 256, 3x3 pad 1, 8-bit codes;
-    flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid."""
+    conv     : VGG-16 conv3_1-shaped C-Block, batch 64, 56x56x128 -> 256, 3x3 pad 1, 8-bit codes, with
+               and without the weight-code L1 bound;
+    flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid;
+    forward  : the integer forward of the workload (first plan, calibrated once), fxpq_net_forward alone."""
     import torch
     import __graft_entry__ as g
     g.build()
@@ -341,12 +343,37 @@ def run_kernel(args):
             ms = sum(ts) / len(ts)
             out[name] = {"ms": round(ms, 4), "gelem_s": round(n / (ms / 1e3) / 1e9, 2),
                          "hbm_gbs": round(4 * n / (ms / 1e3) / 1e9, 1)}
+    if args.kernel in ("forward", "all"):
+        # the integer forward of the bench workload alone (one plan, calibrated once): the target of the
+        # per-launch DRAM traffic capture of the conv kernels
+        from paper_2203_12091_gb300.net import QNet
+        wl = WORKLOADS[args.workload]
+        arch, B = wl["arch"], wl["batch"]
+        W = synth.weights(arch, wl["seed"])
+        imgs = torch.from_numpy(synth.images(B, wl["seed"])).cuda()
+        wdev = {nm: (torch.from_numpy(w).cuda(), torch.from_numpy(b).cuda()) for nm, (w, b) in W.items()}
+        plan = synth.bit_plan(arch, wl["plans"][0])
+        q = QNet(synth.ARCHS[arch](), hw=224, cin=3)
+        q._dev = imgs.device
+        q.quantize_params(wdev, plan)
+        q.calibrate(imgs[: wl["calib"]], plan)
+        ts = []
+        for i in range(args.warmup + args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            q.forward(imgs)
+            e1.record()
+            e1.synchronize()
+            if i >= args.warmup:
+                ts.append(e0.elapsed_time(e1))
+        ms = sum(ts) / len(ts)
+        out["forward"] = {"workload": args.workload, "ms": round(ms, 4), "images_s": round(B / (ms / 1e3), 1)}
     print(json.dumps({"kernel_timing": out}))
 
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=["conv", "flsearch", "all"], help="time one kernel case and exit")
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "forward", "all"], help="time one kernel case and exit")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
