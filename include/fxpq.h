@@ -130,6 +130,26 @@ FXPQ_API fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_sign
                            int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
                            fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream);
 
+/* Several independent FL searches (e.g. every weight and bias tensor of a network, Sec. IV-C's
+ * per-data-structure search) in one set of launches: each item has the arguments, results and
+ * limits of fxpq_fl_search.  Every item is validated before the first launch.  The batch runs in
+ * groups of up to 32 items, each group as three kernels on `stream`.
+ * Workspace: fxpq_fl_search_batch_workspace(n_items) bytes, 256-byte aligned; scratch. */
+typedef struct {
+    const float* d_x;      /* device tensor of n fp32 values                                  */
+    int64_t n;
+    int32_t is_signed;     /* 0, 1, or -1 (S = 1 iff min(x) < 0)                              */
+    int32_t k_lo, k_hi;
+    int32_t fl_lo, fl_hi;
+    double* d_err;         /* device double[(k_hi-k_lo+1) * (fl_hi-fl_lo+1)]                  */
+    int32_t* d_best;       /* device int32[k_hi-k_lo+1]                                       */
+    fxpq_stats* d_stats;   /* device fxpq_stats or NULL                                       */
+} fxpq_fl_search_item;
+
+FXPQ_API size_t fxpq_fl_search_batch_workspace(int32_t n_items);
+FXPQ_API fxpq_status fxpq_fl_search_batch(const fxpq_fl_search_item* h_items, int32_t n_items, void* d_ws,
+                                          size_t ws_bytes, void* stream);
+
 /* fxpq_fl_search for callers that cannot allocate device memory -- for instance a plug-in whose
  * host application owns the whole device memory pool, or a latency-critical loop that must never
  * enter the allocator (cudaMalloc may synchronise the device).  The paper has no counterpart: this

@@ -28,6 +28,11 @@ class Stats(ctypes.Structure):
                 ("sum", ctypes.c_double), ("sumsq", ctypes.c_double), ("n", I64)]
 
 
+class FlSearchItem(ctypes.Structure):
+    _fields_ = [("d_x", VP), ("n", I64), ("is_signed", I32), ("k_lo", I32), ("k_hi", I32), ("fl_lo", I32),
+                ("fl_hi", I32), ("d_err", VP), ("d_best", VP), ("d_stats", VP)]
+
+
 class ConvDesc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("Cp", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("out_mode", I32),
@@ -55,6 +60,8 @@ _SIGS = {
     "fxpq_quantize": (I32, [VP, I64, Fmt, I32, VP, VP]),
     "fxpq_quantize_rows": (I32, [VP, I64, I32, Fmt, I32, VP, VP]),
     "fxpq_code_l1max": (I32, [VP, I64, I64, VP, VP]),
+    "fxpq_fl_search_batch_workspace": (SZ, [I32]),
+    "fxpq_fl_search_batch": (I32, [VP, I32, VP, SZ, VP]),
     "fxpq_quantize_images": (I32, [VP, I32, I32, I32, I32, Fmt, I32, VP, VP]),
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),

@@ -60,7 +60,7 @@ struct FsGlobal {
     u64 ps2[NKEY][2];
     u64 r[2][NJ][MAXFL][2];
     u64 rb[NJ][MAXFL][2];
-    unsigned mn, mx, nonfinite, pad;
+    unsigned mn_inv, mx, nonfinite, pad;  // mn_inv = ~(smallest order key); 0: no finite element
     double cells[2][MAXK][MAXFL];
     double stat_sum, stat_sumsq;
 };
@@ -74,6 +74,30 @@ struct FsParams {
     int jb_lo, jb_hi;        // j range of the boundary sum Rb (x >= 0)
     FsGlobal* g;
 };
+
+// A batch of independent searches (one per tensor) run by the same three launches.  Blocks of the
+// bins kernel and warps of the cells kernel are assigned to items by the prefix arrays.
+constexpr int FS_MAX_ITEMS = 32;
+
+struct FsFinal {
+    int S_lo, S_hi;
+    int k_lo, nk;
+    int fl_lo, nfl;
+};
+
+struct FsBatch {
+    int n_items;
+    int blk0[FS_MAX_ITEMS + 1];   // first bins block of each item (bins launches cover item ranges)
+    int cell0[FS_MAX_ITEMS + 1];  // first cell (warp) of each item in the cells launch
+    FsParams p[FS_MAX_ITEMS];
+    FsFinal f[FS_MAX_ITEMS];
+};
+
+__device__ __forceinline__ int batch_item(const int* start, int n, int idx) {
+    int it = 0;
+    while (it + 1 < n && idx >= start[it + 1]) ++it;
+    return it;
+}
 
 __device__ __forceinline__ unsigned order_key(float x) {
     unsigned u = __float_as_uint(x);
@@ -290,7 +314,12 @@ __device__ __forceinline__ void load16(const FsParams& P, long long tb, int sub,
 }
 
 template <bool VEC, int NS, int NRB>
-__global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2) fl_search_bins_kernel(FsParams P) {
+__global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
+    fl_search_bins_kernel(const __grid_constant__ FsBatch B, int item0, int item1) {
+    // this launch covers items [item0, item1); blk0 holds their block offsets relative to the launch
+    const int item = item0 + batch_item(B.blk0 + item0, item1 - item0, (int)blockIdx.x);
+    const FsParams& P = B.p[item];
+    const int blk = (int)blockIdx.x - B.blk0[item];
     extern __shared__ __align__(16) unsigned char fs_smem_raw[];
     FsSmem& sm = *reinterpret_cast<FsSmem*>(fs_smem_raw);
     const unsigned lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
@@ -305,7 +334,7 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2) f
     bool tnf = false;
     const unsigned lt_mask = (1u << lane) - 1u;
 
-    const long long start = (long long)blockIdx.x * P.chunk;
+    const long long start = (long long)blk * P.chunk;
     const long long end = min(start + (long long)P.chunk, P.n);
     const RbC rbc = make_rbc(P);
     for (long long tb = start; tb < end; tb += TILE) {
@@ -450,7 +479,7 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2) f
         gadd128(g->rb[j][f], ((u64)sm.rb[j][f][1] << 32) | sm.rb[j][f][0]);
     }
     if (threadIdx.x == 0) {
-        atomicMin(&g->mn, sm.mn);
+        if (sm.mn != 0xFFFFFFFFu) atomicMax(&g->mn_inv, ~sm.mn);
         atomicMax(&g->mx, sm.mx);
         if (sm.nonfinite) atomicOr(&g->nonfinite, 1u);
     }
@@ -577,12 +606,6 @@ __device__ void big_negate(Big& a) {
     }
 }
 
-struct FsFinal {
-    int S_lo, S_hi;
-    int k_lo, nk;
-    int fl_lo, nfl;
-};
-
 // saturated set with moments (n, s1, s2) at exponent E: s2 2^(2(E-23)) - 2 T s1 2^(E-23-fl) + T^2 n 2^(-2fl)
 __device__ void add_sat(Big& acc, u64 n, U128 s1, U128 s2, int E, int fl, u64 T) {
     big_add(acc, s2, 2 * (E - 23), false);
@@ -593,12 +616,16 @@ __device__ void add_sat(Big& acc, u64 n, U128 s1, U128 s2, int E, int fl, u64 T)
 }
 
 // One warp per candidate cell (plus two cells for the exact stats); lanes split the exponent keys.
-__global__ void fl_search_cells_kernel(FsParams P, FsFinal F) {
+__global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
+    const int gcell = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (gcell >= B.cell0[B.n_items]) return;
+    const int item = batch_item(B.cell0, B.n_items, gcell);
+    const FsParams& P = B.p[item];
+    const FsFinal& F = B.f[item];
+    const int cell = gcell - B.cell0[item];
     const FsGlobal* g = P.g;
     const int lane = threadIdx.x & 31;
-    const int cell = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
-    if (cell >= ncell + 2) return;
     Big acc;
     big_zero(acc);
     if (cell >= ncell) {
@@ -657,12 +684,28 @@ __global__ void fl_search_cells_kernel(FsParams P, FsFinal F) {
     }
 }
 
-__global__ void fl_search_select_kernel(FsParams P, FsFinal F, int is_signed, double* err, int* best,
-                                        fxpq_stats* stats, int* status) {
+// Per-item outputs of the select kernel.
+struct FsOut {
+    double* err;
+    int* best;
+    fxpq_stats* stats;
+    int is_signed;
+};
+struct FsOutBatch {
+    FsOut o[FS_MAX_ITEMS];
+};
+
+// One block per item: per wordlength, the scores and the argmin (exact ties keep the smaller FL).
+__global__ void fl_search_select_kernel(const __grid_constant__ FsBatch B, const __grid_constant__ FsOutBatch O,
+                                        int* status) {
+    const int item = blockIdx.x;
+    const FsParams& P = B.p[item];
+    const FsFinal& F = B.f[item];
+    const FsOut& out = O.o[item];
     const FsGlobal* g = P.g;
-    const float mn = g->mn == 0xFFFFFFFFu ? 0.0f : order_key_inv(g->mn);
+    const float mn = g->mn_inv == 0u ? 0.0f : order_key_inv(~g->mn_inv);
     const float mx = g->mx == 0u ? 0.0f : order_key_inv(g->mx);
-    const int S = is_signed >= 0 ? is_signed : (mn < 0.0f ? 1 : 0);
+    const int S = out.is_signed >= 0 ? out.is_signed : (mn < 0.0f ? 1 : 0);
     const int i = threadIdx.x;
     if (i < F.nk) {
         const int k = F.k_lo + i;
@@ -670,24 +713,24 @@ __global__ void fl_search_select_kernel(FsParams P, FsFinal F, int is_signed, do
         int bf = F.fl_lo;
         for (int fi = 0; fi < F.nfl; ++fi) {
             const double v = g->cells[S][k - 2][fi];
-            err[(long long)i * F.nfl + fi] = v;
+            out.err[(long long)i * F.nfl + fi] = v;
             if (fi == 0 || v < bv) {  // strict: exact ties keep the smaller FL
                 bv = v;
                 bf = F.fl_lo + fi;
             }
         }
-        best[i] = bf;
+        out.best[i] = bf;
     }
     if (i == 0) {
         if (g->nonfinite) latch_status(status, FXPQ_ERR_NONFINITE);
-        if (stats) {
-            stats->min = mn;
-            stats->max = mx;
-            stats->is_signed = S;
-            stats->nonfinite = g->nonfinite ? 1 : 0;
-            stats->sum = g->stat_sum;
-            stats->sumsq = g->stat_sumsq;
-            stats->n = P.n;
+        if (out.stats) {
+            out.stats->min = mn;
+            out.stats->max = mx;
+            out.stats->is_signed = S;
+            out.stats->nonfinite = g->nonfinite ? 1 : 0;
+            out.stats->sum = g->stat_sum;
+            out.stats->sumsq = g->stat_sumsq;
+            out.stats->n = P.n;
         }
     }
 }
@@ -715,83 +758,175 @@ void st_attr_once() {
 }
 }  // namespace
 
-extern "C" size_t fxpq_fl_search_workspace(int64_t n) {
-    (void)n;
-    return (sizeof(FsGlobal) + 255) / 256 * 256;
-}
+namespace {
+constexpr size_t kFsGlobalBytes = (sizeof(FsGlobal) + 255) / 256 * 256;
 
-extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo, int32_t k_hi,
-                                      int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
-                                      fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream) {
+// One search of a batch, prepared on the host.
+struct FsItemHost {
+    FsParams p;
+    FsFinal f;
+    FsOut o;
+    int variant;  // bins kernel instance: bit 0 vec, bit 1 small (k_hi <= 9), bit 2 narrow boundary range
+    int grid;     // bins blocks
+};
+
+fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h) {
+    const int64_t n = it.n;
     if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;
-    if (is_signed < -1 || is_signed > 1) return FXPQ_ERR_INVALID_ARG;
-    if (k_lo < 2 || k_hi > 16 || k_lo > k_hi) return FXPQ_ERR_INVALID_ARG;
-    if (fl_lo < -32 || fl_hi > 40 || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL) return FXPQ_ERR_INVALID_ARG;
-    if (!d_err || !d_best || (n > 0 && !d_x)) return FXPQ_ERR_INVALID_ARG;
-    if (!d_ws || ws_bytes < fxpq_fl_search_workspace(n) || !aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
-    cudaStream_t s = as_stream(stream);
-    FsGlobal* g = static_cast<FsGlobal*>(d_ws);
-    if (cudaMemsetAsync(g, 0, sizeof(FsGlobal), s) != cudaSuccess) return FXPQ_ERR_CUDA;
-    if (cudaMemsetAsync(&g->mn, 0xFF, sizeof(unsigned), s) != cudaSuccess) return FXPQ_ERR_CUDA;
-
-    const int S_lo = is_signed < 0 ? 0 : is_signed, S_hi = is_signed < 0 ? 1 : is_signed;
-    FsParams P;
-    P.x = d_x;
+    if (it.is_signed < -1 || it.is_signed > 1) return FXPQ_ERR_INVALID_ARG;
+    if (it.k_lo < 2 || it.k_hi > 16 || it.k_lo > it.k_hi) return FXPQ_ERR_INVALID_ARG;
+    if (it.fl_lo < -32 || it.fl_hi > 40 || it.fl_lo > it.fl_hi || it.fl_hi - it.fl_lo + 1 > MAXFL)
+        return FXPQ_ERR_INVALID_ARG;
+    if (!it.d_err || !it.d_best || (n > 0 && !it.d_x)) return FXPQ_ERR_INVALID_ARG;
+    const int S_lo = it.is_signed < 0 ? 0 : it.is_signed, S_hi = it.is_signed < 0 ? 1 : it.is_signed;
+    FsParams& P = h.p;
+    P.x = it.d_x;
     P.n = n;
     // whole waves of resident blocks, each chunk at most CHUNK_MAX elements
     const long long resident = 152LL * FS_BLOCKS_PER_SM;
-    const long long waves = (n + resident * CHUNK_MAX - 1) / (resident * CHUNK_MAX);
+    const long long waves = n > 0 ? (n + resident * CHUNK_MAX - 1) / (resident * CHUNK_MAX) : 1;
     const long long per = (n + resident * waves - 1) / (resident * waves);
     long long chunk = (per + TILE - 1) / TILE * TILE;
     if (chunk < TILE) chunk = TILE;
     if (chunk > CHUNK_MAX) chunk = CHUNK_MAX;
     P.chunk = (int)chunk;
-    P.fl_lo = fl_lo;
-    P.nfl = fl_hi - fl_lo + 1;
+    P.fl_lo = it.fl_lo;
+    P.nfl = it.fl_hi - it.fl_lo + 1;
     // x >= 0 rounds (no clip) for q <= t-2 with t = k-1 (S=1) or k (S=0); x < 0 (S=1) for q <= k-2
-    P.jmax_pos = (S_lo == 0) ? k_hi - 2 : k_hi - 3;
-    P.jmax_neg = (S_hi == 1) ? k_hi - 2 : -2;
+    P.jmax_pos = (S_lo == 0) ? it.k_hi - 2 : it.k_hi - 3;
+    P.jmax_neg = (S_hi == 1) ? it.k_hi - 2 : -2;
     // boundary q = t-1 for x >= 0
-    P.jb_lo = (S_hi == 1) ? k_lo - 2 : k_lo - 1;
-    P.jb_hi = (S_lo == 0) ? k_hi - 1 : k_hi - 2;
+    P.jb_lo = (S_hi == 1) ? it.k_lo - 2 : it.k_lo - 1;
+    P.jb_hi = (S_lo == 0) ? it.k_hi - 1 : it.k_hi - 2;
     if (P.jb_lo < 0) P.jb_lo = 0;
     P.g = g;
-    if (n > 0) {
-        const int grid = (int)((n + chunk - 1) / chunk);
-        const bool vec = aligned(d_x, 16);
-        const bool small = k_hi <= 9;                     // slots j = -1 .. k_hi - 1 suffice
-        const bool narrow = P.jb_hi - P.jb_lo + 1 <= 2;  // at most two boundary positions
-        st_attr_once();
-        const size_t sb = sizeof(FsSmem);
-#define FXPQ_FS_LAUNCH(V)                                                       \
-    if (narrow && small)                                                        \
-        fl_search_bins_kernel<V, 10, 2><<<grid, FS_THREADS, sb, s>>>(P);        \
-    else if (narrow)                                                            \
-        fl_search_bins_kernel<V, NJ, 2><<<grid, FS_THREADS, sb, s>>>(P);        \
-    else                                                                        \
-        fl_search_bins_kernel<V, NJ, NJ><<<grid, FS_THREADS, sb, s>>>(P);
-        if (vec) {
-            FXPQ_FS_LAUNCH(true)
-        } else {
-            FXPQ_FS_LAUNCH(false)
-        }
-#undef FXPQ_FS_LAUNCH
-        const fxpq_status st = after_launch("fl_search_bins");
-        if (st != FXPQ_OK) return st;
+    h.f.S_lo = S_lo;
+    h.f.S_hi = S_hi;
+    h.f.k_lo = it.k_lo;
+    h.f.nk = it.k_hi - it.k_lo + 1;
+    h.f.fl_lo = it.fl_lo;
+    h.f.nfl = P.nfl;
+    h.o.err = it.d_err;
+    h.o.best = it.d_best;
+    h.o.stats = it.d_stats;
+    h.o.is_signed = it.is_signed;
+    h.grid = (int)((n + chunk - 1) / chunk);
+    h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0);
+    return FXPQ_OK;
+}
+
+void fs_bins_launch(int variant, int grid, const FsBatch& B, int i0, int i1, cudaStream_t s) {
+    const size_t sb = sizeof(FsSmem);
+    const bool vec = variant & 1, small = variant & 2, narrow = variant & 4;
+#define FXPQ_FS_LAUNCH(V)                                                                \
+    if (narrow && small)                                                                 \
+        fl_search_bins_kernel<V, 10, 2><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);         \
+    else if (narrow)                                                                     \
+        fl_search_bins_kernel<V, NJ, 2><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);         \
+    else                                                                                 \
+        fl_search_bins_kernel<V, NJ, NJ><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);
+    if (vec) {
+        FXPQ_FS_LAUNCH(true)
+    } else {
+        FXPQ_FS_LAUNCH(false)
     }
-    FsFinal F;
-    F.S_lo = S_lo;
-    F.S_hi = S_hi;
-    F.k_lo = k_lo;
-    F.nk = k_hi - k_lo + 1;
-    F.fl_lo = fl_lo;
-    F.nfl = P.nfl;
-    const int ncell = (S_hi - S_lo + 1) * F.nk * F.nfl + 2;
-    fl_search_cells_kernel<<<(ncell + 3) / 4, 128, 0, s>>>(P, F);
+#undef FXPQ_FS_LAUNCH
+}
+
+// Runs up to FS_MAX_ITEMS prepared searches whose bins live at g[0..n): one clear, one bins launch
+// per run of items sharing a kernel instance (items are ordered by instance), one cells launch, one
+// select launch.
+fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
+    if (n == 0) return FXPQ_OK;
+    if (cudaMemsetAsync(g, 0, kFsGlobalBytes * n, s) != cudaSuccess) return FXPQ_ERR_CUDA;
+    // order by kernel instance (stable), each item keeping its own bins
+    int order[FS_MAX_ITEMS];
+    int m = 0;
+    for (int v = 0; v < 8; ++v)
+        for (int i = 0; i < n; ++i)
+            if (h[i].variant == v) order[m++] = i;
+    FsBatch B;
+    FsOutBatch O;
+    B.n_items = n;
+    int cells = 0;
+    for (int j = 0; j < n; ++j) {
+        const FsItemHost& it = h[order[j]];
+        B.p[j] = it.p;
+        B.p[j].g = reinterpret_cast<FsGlobal*>(reinterpret_cast<char*>(g) + kFsGlobalBytes * order[j]);
+        B.f[j] = it.f;
+        O.o[j] = it.o;
+        B.cell0[j] = cells;
+        cells += (it.f.S_hi - it.f.S_lo + 1) * it.f.nk * it.f.nfl + 2;
+    }
+    B.cell0[n] = cells;
+    st_attr_once();
+    for (int j0 = 0; j0 < n;) {
+        const int v = h[order[j0]].variant;
+        int j1 = j0, blocks = 0;
+        while (j1 < n && h[order[j1]].variant == v) {
+            B.blk0[j1] = blocks;  // relative to this launch
+            blocks += h[order[j1]].grid;
+            ++j1;
+        }
+        B.blk0[j1] = blocks;
+        if (blocks > 0) {
+            fs_bins_launch(v, blocks, B, j0, j1, s);
+            const fxpq_status st = after_launch("fl_search_bins");
+            if (st != FXPQ_OK) return st;
+        }
+        j0 = j1;
+    }
+    fl_search_cells_kernel<<<(cells + 3) / 4, 128, 0, s>>>(B);
     fxpq_status st = after_launch("fl_search_cells");
     if (st != FXPQ_OK) return st;
-    fl_search_select_kernel<<<1, 32, 0, s>>>(P, F, is_signed, d_err, d_best, d_stats, status_ptr());
+    fl_search_select_kernel<<<n, 32, 0, s>>>(B, O, status_ptr());
     return after_launch("fl_search_select");
+}
+}  // namespace
+
+extern "C" size_t fxpq_fl_search_workspace(int64_t n) {
+    (void)n;
+    return kFsGlobalBytes;
+}
+
+extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo, int32_t k_hi,
+                                      int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
+                                      fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream) {
+    const fxpq_fl_search_item it = {d_x, n, is_signed, k_lo, k_hi, fl_lo, fl_hi, d_err, d_best, d_stats};
+    FsItemHost h;
+    const fxpq_status st = fs_prepare(it, static_cast<FsGlobal*>(d_ws), h);
+    if (st != FXPQ_OK) return st;
+    if (!d_ws || ws_bytes < fxpq_fl_search_workspace(n) || !aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
+    return fs_run(&h, 1, static_cast<FsGlobal*>(d_ws), as_stream(stream));
+}
+
+extern "C" size_t fxpq_fl_search_batch_workspace(int32_t n_items) {
+    return n_items > 0 ? kFsGlobalBytes * (size_t)n_items : 0;
+}
+
+extern "C" fxpq_status fxpq_fl_search_batch(const fxpq_fl_search_item* h_items, int32_t n_items, void* d_ws,
+                                            size_t ws_bytes, void* stream) {
+    if (n_items < 0 || (n_items > 0 && !h_items)) return FXPQ_ERR_INVALID_ARG;
+    if (n_items == 0) return FXPQ_OK;
+    if (!d_ws || ws_bytes < fxpq_fl_search_batch_workspace(n_items) || !aligned(d_ws, 256))
+        return FXPQ_ERR_WORKSPACE;
+    FsItemHost h[FS_MAX_ITEMS];
+    FsGlobal* g = static_cast<FsGlobal*>(d_ws);
+    // validate everything before the first launch
+    for (int i = 0; i < n_items; ++i) {
+        FsItemHost tmp;
+        const fxpq_status st = fs_prepare(h_items[i], g, tmp);
+        if (st != FXPQ_OK) return st;
+    }
+    cudaStream_t s = as_stream(stream);
+    for (int i0 = 0; i0 < n_items; i0 += FS_MAX_ITEMS) {
+        const int m = n_items - i0 < FS_MAX_ITEMS ? n_items - i0 : FS_MAX_ITEMS;
+        FsGlobal* gi = reinterpret_cast<FsGlobal*>(reinterpret_cast<char*>(g) + kFsGlobalBytes * i0);
+        for (int i = 0; i < m; ++i) fs_prepare(h_items[i0 + i], gi, h[i]);
+        const fxpq_status st = fs_run(h, m, gi, s);
+        if (st != FXPQ_OK) return st;
+    }
+    return FXPQ_OK;
 }
 
 extern "C" fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32_t strategy, fxpq_fmt* h_out) {

@@ -90,6 +90,17 @@ def fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, s
     return err.view(nk, nfl), best, stats
 
 
+def fxpq_fl_search_batch_workspace(n_items: int) -> int:
+    return L.lib().fxpq_fl_search_batch_workspace(n_items)
+
+
+def fxpq_fl_search_batch(items, ws, stream=None):
+    """items: list of L.FlSearchItem (device pointers filled in).  ws: a device workspace tensor."""
+    arr = (L.FlSearchItem * len(items))(*items)
+    L.check("fxpq_fl_search_batch", L.lib().fxpq_fl_search_batch(
+        ctypes.cast(arr, ctypes.c_void_p), len(items), _p(ws), ws.numel() * ws.element_size(), _s(stream)))
+
+
 def stats_from_device(stats_bytes) -> Stats:
     return Stats.from_buffer_copy(bytes(stats_bytes.cpu().numpy().tobytes()))
 

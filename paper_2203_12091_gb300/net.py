@@ -33,7 +33,7 @@ def pad8(c: int) -> int:
 
 
 def search_fmts(items, stream=None):
-    """FL searches at one wordlength each, launched back to back; one device-to-host read at the end.
+    """FL searches at one wordlength each, as one batch (fxpq_fl_search_batch); one device-to-host read.
 
     items: list of (tensor, k).  Returns the chosen (k, S, FL) per item (sign strategy of Sec. IV-A.3)."""
     if not items:
@@ -43,16 +43,14 @@ def search_fmts(items, stream=None):
     stride = 64  # bytes per result record: int32 best FL at 0, fxpq_stats at 8
     res = torch.empty(len(items) * stride, dtype=torch.uint8, device=dev)
     err = torch.empty(len(items) * nfl, dtype=torch.float64, device=dev)
-    ws = F.workspace(F.fxpq_fl_search_workspace(0), dev)
-    lib = L.lib()
-    s = F._s(stream)
+    ws = F.workspace(F.fxpq_fl_search_batch_workspace(len(items)), dev)
     base = res.data_ptr()
+    batch = []
     for i, (x, k) in enumerate(items):
         x = x.reshape(-1)
-        L.check("fxpq_fl_search", lib.fxpq_fl_search(
-            ctypes.c_void_p(x.data_ptr()), x.numel(), -1, k, k, FL_LO, FL_HI,
-            ctypes.c_void_p(err.data_ptr() + 8 * nfl * i), ctypes.c_void_p(base + stride * i),
-            ctypes.c_void_p(base + stride * i + 8), ctypes.c_void_p(ws.data_ptr()), ws.numel(), s))
+        batch.append(L.FlSearchItem(x.data_ptr(), x.numel(), -1, k, k, FL_LO, FL_HI, err.data_ptr() + 8 * nfl * i,
+                                    base + stride * i, base + stride * i + 8))
+    F.fxpq_fl_search_batch(batch, ws, stream)
     host = bytes(res.cpu().numpy().tobytes())
     out = []
     for i, (_, k) in enumerate(items):

@@ -3,6 +3,8 @@
 Integer outputs (codes, chosen FL) must be identical; the L2 scores are the exact sums rounded
 once on both sides, so they are compared for equality (the stated 1e-5 relative tolerance is
 checked as well, as the contract)."""
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -156,3 +158,41 @@ def test_fl_search_config_large_sampled(F, n):
         assert g[k - 2, fl + 8] == oracle.l2_error(x, k, 1, fl)
     assert s.sumsq == oracle.exact_sum(x.astype(np.float64) ** 2)
     assert s.min == float(x.min()) and s.max == float(x.max())
+
+
+def test_fl_search_batch_matches_oracle(F):
+    """A batch mixing sizes (0 to 300k), wordlength ranges (one k, several k, the full sweep), fixed
+    and automatic signedness and an unaligned tensor: every item equals the oracle's search, and
+    more than 32 items run as several groups."""
+    import paper_2203_12091_gb300._lib as L
+    specs = []
+    for i in range(37):
+        dist = ("normal", "laplace", "relu_normal")[i % 3]
+        n = (0, 1, 17, 1023, 4097, 70001, 300000)[i % 7]
+        klo, khi = ((8, 8), (4, 4), (16, 16), (2, 16), (3, 9), (12, 13))[i % 6]
+        S = (-1, 0, 1)[i % 3] if i % 5 else -1
+        fllo, flhi = ((-8, 23), (0, 15), (-32, -1))[i % 3]
+        specs.append((synth.sweep_tensor(dist, n, 100 + i), S, klo, khi, fllo, flhi, i % 4 == 3))
+    items, keep = [], []
+    for x, S, klo, khi, fllo, flhi, unaligned in specs:
+        xd = torch.from_numpy(np.concatenate([np.zeros(1, np.float32), x])).cuda()
+        xd = xd[1:] if unaligned else xd[1:].clone()
+        nk, nfl = khi - klo + 1, flhi - fllo + 1
+        err = torch.empty(nk * nfl, dtype=torch.float64, device="cuda")
+        best = torch.empty(nk, dtype=torch.int32, device="cuda")
+        st = torch.empty(ctypes.sizeof(L.Stats), dtype=torch.uint8, device="cuda")
+        keep.append((xd, err, best, st))
+        items.append(L.FlSearchItem(xd.data_ptr(), x.size, S, klo, khi, fllo, flhi, err.data_ptr(), best.data_ptr(),
+                                    st.data_ptr()))
+    ws = torch.empty(F.fxpq_fl_search_batch_workspace(len(items)), dtype=torch.uint8, device="cuda")
+    F.fxpq_fl_search_batch(items, ws)
+    torch.cuda.synchronize()
+    assert F.fxpq_get_device_status() == 0
+    for (x, S, klo, khi, fllo, flhi, _), (xd, err, best, st) in zip(specs, keep):
+        oerr, obest, oS, ost = oracle.fl_search(x, S, klo, khi, fllo, flhi)
+        assert np.array_equal(best.cpu().numpy(), obest)
+        assert np.array_equal(err.cpu().numpy(), oerr.reshape(-1))
+        s = F.stats_from_device(st)
+        assert s.is_signed == oS and s.n == x.size
+        if x.size:
+            assert s.min == ost["min"] and s.max == ost["max"] and s.sum == ost["sum"] and s.sumsq == ost["sumsq"]
