@@ -97,6 +97,35 @@ FXPQ_API fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int3
 FXPQ_API fxpq_status fxpq_quantize_rows(const float* d_x, int64_t rows, int32_t C, fxpq_fmt f, int32_t Cp, void* d_y,
                                void* stream);
 
+/* Parameter quantization in one launch, with formats that stay on the device: each item's S and
+ * FL are read from device memory (typically the d_stats / d_best results of fxpq_fl_search_batch),
+ * so no host round trip separates the FL search from the quantization (Sec. IV-C: weights and
+ * biases are quantized with the FL the search picked).  Item kinds:
+ *   FXPQ_QB_ROWS_F16: `rows` rows of C fp32 values -> fp16 code planes [rows, Cp] (as
+ *                     fxpq_quantize_rows); with d_l1 (bits <= 8) the largest L1 norm over groups
+ *                     of rows_per_group consecutive rows (an output channel of KRSC weights:
+ *                     rows_per_group = R*S) is atomically max-ed into *d_l1 (initialise it).
+ *                     C == Cp needs d_x and d_out 16-byte aligned; rows % rows_per_group == 0.
+ *   FXPQ_QB_FLAT_I32: `rows` fp32 values -> int32 codes (biases, the avg-pool reciprocal).
+ * Non-finite inputs latch FXPQ_ERR_NONFINITE and produce code 0.  Not part of the paper's
+ * statement beyond Q itself: it batches Eq. fp_k_bit_quantization over many tensors. */
+enum { FXPQ_QB_ROWS_F16 = 0, FXPQ_QB_FLAT_I32 = 1 };
+typedef struct {
+    const float* d_x;
+    void* d_out;
+    int32_t kind;             /* FXPQ_QB_*                                                     */
+    int32_t bits;             /* k (2..16)                                                     */
+    int64_t rows;             /* ROWS_F16: rows of C values; FLAT_I32: element count           */
+    int32_t C, Cp;            /* ROWS_F16 geometry                                             */
+    int32_t rows_per_group;   /* ROWS_F16: rows per L1 group                                   */
+    int32_t reserved;
+    const int32_t* d_fl;      /* device int32: FL                                              */
+    const fxpq_stats* d_stats; /* device: is_signed gives S                                    */
+    int64_t* d_l1;            /* ROWS_F16, bits <= 8: L1 bound output, or NULL                 */
+} fxpq_quantize_item;
+
+FXPQ_API fxpq_status fxpq_quantize_batch(const fxpq_quantize_item* h_items, int32_t n_items, void* stream);
+
 /* Largest L1 norm over the rows of a one-plane fp16 code tensor [rows, L] (fmt.bits <= 8):
  * *d_out = max_r sum_j |code[r, j]| as an int64 on the device (0 when rows == 0).  For KRSC
  * weights with L = R*S*Cp it is the w_l1 bound of fxpq_conv_desc.  Exact integer arithmetic;

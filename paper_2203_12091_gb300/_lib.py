@@ -33,6 +33,11 @@ class FlSearchItem(ctypes.Structure):
                 ("fl_hi", I32), ("d_err", VP), ("d_best", VP), ("d_stats", VP)]
 
 
+class QuantizeItem(ctypes.Structure):
+    _fields_ = [("d_x", VP), ("d_out", VP), ("kind", I32), ("bits", I32), ("rows", I64), ("C", I32), ("Cp", I32),
+                ("rows_per_group", I32), ("reserved", I32), ("d_fl", VP), ("d_stats", VP), ("d_l1", VP)]
+
+
 class ConvDesc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("Cp", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("out_mode", I32),
@@ -54,6 +59,7 @@ class Net(ctypes.Structure):
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_NONFINITE, ERR_TIMEOUT, ERR_CUDA, ERR_WORKSPACE, ERR_RANGE = range(8)
 DT_I8, DT_U8, DT_I16, DT_U16, DT_I32, DT_F16 = range(6)
 OUT_CODES, OUT_ACC64, OUT_F32 = range(3)
+QB_ROWS_F16, QB_FLAT_I32 = range(2)
 OP_CONV, OP_MAXPOOL, OP_ELTWISE, OP_AVGPOOL = range(4)
 
 _SIGS = {
@@ -62,6 +68,7 @@ _SIGS = {
     "fxpq_code_l1max": (I32, [VP, I64, I64, VP, VP]),
     "fxpq_fl_search_batch_workspace": (SZ, [I32]),
     "fxpq_fl_search_batch": (I32, [VP, I32, VP, SZ, VP]),
+    "fxpq_quantize_batch": (I32, [VP, I32, VP]),
     "fxpq_quantize_images": (I32, [VP, I32, I32, I32, I32, Fmt, I32, VP, VP]),
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),

@@ -172,6 +172,108 @@ __global__ void code_l1max_kernel(const uint4* __restrict__ codes, long long row
     }
 }
 
+// ------------------------------------------------------------------------------------------
+// Batched parameter quantization with device-resident formats
+// ------------------------------------------------------------------------------------------
+constexpr int QB_MAX = 32;
+constexpr int QB_FLAT_UNIT = 4096;  // elements per block of a flat item
+
+struct QbItem {
+    const float* x;
+    void* out;
+    long long* l1;
+    const int* fl;
+    const fxpq_stats* st;
+    long long rows;
+    int C, Cp, rpg, bits, kind;
+};
+
+struct QbBatch {
+    int n;
+    int unit0[QB_MAX + 1];  // first block of each item
+    QbItem it[QB_MAX];
+    int* status;
+};
+
+// One block per work unit: an output-channel group (rpg rows) of a row item, or QB_FLAT_UNIT elements of
+// a flat item.  The format (k from the item, S and FL from the device) is read once per block.
+__global__ void __launch_bounds__(256) quantize_batch_kernel(const __grid_constant__ QbBatch B) {
+    int item = 0;
+    while (item + 1 < B.n && (int)blockIdx.x >= B.unit0[item + 1]) ++item;
+    const QbItem& I = B.it[item];
+    const long long u = (long long)blockIdx.x - B.unit0[item];
+    const int fl = *I.fl;
+    const int S = I.st->is_signed;
+    QParams p;
+    p.scale = __int_as_float((127 + fl) << 23);  // 2^fl, fl in [-32, 40]
+    p.lo = S ? -(float)(1 << (I.bits - 1)) : 0.0f;
+    p.hi = (float)((1 << (I.bits - S)) - 1);
+    p.status = B.status;
+    bool bad = false;
+    if (I.kind == FXPQ_QB_FLAT_I32) {
+        const long long e0 = u * QB_FLAT_UNIT;
+        const long long e1 = min(e0 + QB_FLAT_UNIT, I.rows);
+        int32_t* out = static_cast<int32_t*>(I.out);
+        for (long long e = e0 + threadIdx.x; e < e1; e += blockDim.x) out[e] = quant1(__ldg(I.x + e), p, bad);
+    } else {
+        const int planes = I.bits > 8 ? 2 : 1;
+        const long long r0 = u * I.rpg;
+        const long long total = I.rows * (long long)I.Cp;  // plane stride
+        long long l1 = 0;
+        if (I.C == I.Cp) {
+            // unpadded rows: 8 codes per step, one 16-byte store per plane
+            const long long n8 = (long long)I.rpg * I.Cp / 8, b8 = r0 * I.Cp / 8;
+            const float4* x4 = reinterpret_cast<const float4*>(I.x);
+            uint4* o = static_cast<uint4*>(I.out);
+            for (long long i = threadIdx.x; i < n8; i += blockDim.x) {
+                const float4 a = __ldg(x4 + 2 * (b8 + i)), b = __ldg(x4 + 2 * (b8 + i) + 1);
+                const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int c0 = quant1(v[2 * e], p, bad), c1 = quant1(v[2 * e + 1], p, bad);
+                    l1 += abs(c0) + abs(c1);
+                    if (planes == 1) {
+                        hi[e] = (uint32_t)__half_as_ushort(__int2half_rn(c0)) |
+                                ((uint32_t)__half_as_ushort(__int2half_rn(c1)) << 16);
+                    } else {
+                        __half h0, l0, h1, l1h;
+                        split_limbs(c0, h0, l0);
+                        split_limbs(c1, h1, l1h);
+                        hi[e] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+                        lo[e] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1h) << 16);
+                    }
+                }
+                o[b8 + i] = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                if (planes == 2) o[total / 8 + b8 + i] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+        } else {
+            __half* out = static_cast<__half*>(I.out);
+            const long long n = (long long)I.rpg * I.Cp;
+            for (long long i = threadIdx.x; i < n; i += blockDim.x) {
+                const long long r = r0 + i / I.Cp;
+                const int c = (int)(i % I.Cp);
+                const int code = c < I.C ? quant1(__ldg(I.x + r * I.C + c), p, bad) : 0;
+                l1 += abs(code);
+                code_put(out, r * I.Cp + c, planes, total, code);
+            }
+        }
+        if (I.l1 && planes == 1) {
+            __shared__ long long red[8];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+            if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = l1;
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                long long t = 0;
+                for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+                atomicMax(reinterpret_cast<unsigned long long*>(I.l1), (unsigned long long)t);
+            }
+        }
+    }
+    if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
+}
+
 }  // namespace
 
 static QParams make_qparams(const fxpq_fmt& f) {
@@ -274,4 +376,56 @@ extern "C" fxpq_status fxpq_code_l1max(const void* d_codes, int64_t rows, int64_
     code_l1max_kernel<<<grid, 256, 0, s>>>(static_cast<const uint4*>(d_codes), rows, L / 8,
                                            reinterpret_cast<unsigned long long*>(d_out));
     return after_launch("code_l1max");
+}
+
+extern "C" fxpq_status fxpq_quantize_batch(const fxpq_quantize_item* h_items, int32_t n_items, void* stream) {
+    if (n_items < 0 || (n_items > 0 && !h_items)) return FXPQ_ERR_INVALID_ARG;
+    for (int i = 0; i < n_items; ++i) {
+        const fxpq_quantize_item& it = h_items[i];
+        if (it.bits < 2 || it.bits > 16 || it.rows < 0 || !it.d_fl || !it.d_stats) return FXPQ_ERR_INVALID_ARG;
+        if (it.rows > 0 && (!it.d_x || !it.d_out)) return FXPQ_ERR_INVALID_ARG;
+        if (it.kind == FXPQ_QB_FLAT_I32) {
+            if (it.d_l1) return FXPQ_ERR_INVALID_ARG;
+        } else if (it.kind == FXPQ_QB_ROWS_F16) {
+            if (it.C < 1 || it.Cp < it.C || (it.Cp % 8) || it.rows_per_group < 1 || it.rows % it.rows_per_group)
+                return FXPQ_ERR_INVALID_ARG;
+            if (it.C == it.Cp && (!aligned(it.d_x, 16) || !aligned(it.d_out, 16))) return FXPQ_ERR_INVALID_ARG;
+            if (it.d_l1 && (it.bits > 8 || !aligned(it.d_l1, 8))) return FXPQ_ERR_INVALID_ARG;
+        } else {
+            return FXPQ_ERR_INVALID_ARG;
+        }
+    }
+    cudaStream_t s = as_stream(stream);
+    for (int i0 = 0; i0 < n_items; i0 += QB_MAX) {
+        const int m = n_items - i0 < QB_MAX ? n_items - i0 : QB_MAX;
+        QbBatch B;
+        B.n = m;
+        B.status = status_ptr();
+        long long units = 0;
+        for (int i = 0; i < m; ++i) {
+            const fxpq_quantize_item& it = h_items[i0 + i];
+            QbItem& q = B.it[i];
+            q.x = it.d_x;
+            q.out = it.d_out;
+            q.l1 = reinterpret_cast<long long*>(it.d_l1);
+            q.fl = it.d_fl;
+            q.st = it.d_stats;
+            q.rows = it.rows;
+            q.C = it.C;
+            q.Cp = it.Cp;
+            q.rpg = it.rows_per_group;
+            q.bits = it.bits;
+            q.kind = it.kind;
+            B.unit0[i] = (int)units;
+            units += it.kind == FXPQ_QB_FLAT_I32 ? (it.rows + QB_FLAT_UNIT - 1) / QB_FLAT_UNIT
+                                                 : it.rows / it.rows_per_group;
+            if (units > (1LL << 30)) return FXPQ_ERR_INVALID_ARG;
+        }
+        B.unit0[m] = (int)units;
+        if (units == 0) continue;
+        quantize_batch_kernel<<<(unsigned)units, 256, 0, s>>>(B);
+        const fxpq_status st = after_launch("quantize_batch");
+        if (st != FXPQ_OK) return st;
+    }
+    return FXPQ_OK;
 }

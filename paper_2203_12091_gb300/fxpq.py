@@ -101,6 +101,13 @@ def fxpq_fl_search_batch(items, ws, stream=None):
         ctypes.cast(arr, ctypes.c_void_p), len(items), _p(ws), ws.numel() * ws.element_size(), _s(stream)))
 
 
+def fxpq_quantize_batch(items, stream=None):
+    """items: list of L.QuantizeItem (device pointers filled in)."""
+    arr = (L.QuantizeItem * len(items))(*items)
+    L.check("fxpq_quantize_batch", L.lib().fxpq_quantize_batch(ctypes.cast(arr, ctypes.c_void_p), len(items),
+                                                                _s(stream)))
+
+
 def stats_from_device(stats_bytes) -> Stats:
     return Stats.from_buffer_copy(bytes(stats_bytes.cpu().numpy().tobytes()))
 

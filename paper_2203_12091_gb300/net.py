@@ -32,16 +32,14 @@ def pad8(c: int) -> int:
     return (c + 7) // 8 * 8
 
 
-def search_fmts(items, stream=None):
-    """FL searches at one wordlength each, as one batch (fxpq_fl_search_batch); one device-to-host read.
+REC = 64  # bytes per search result record: int32 best FL at 0, fxpq_stats at 8
 
-    items: list of (tensor, k).  Returns the chosen (k, S, FL) per item (sign strategy of Sec. IV-A.3)."""
-    if not items:
-        return []
+
+def launch_searches(items, res, stream=None):
+    """FL searches at one wordlength each, as one batch (fxpq_fl_search_batch), results into the device
+    uint8 buffer `res` (REC bytes per item); nothing is read back."""
     dev = items[0][0].device
     nfl = FL_HI - FL_LO + 1
-    stride = 64  # bytes per result record: int32 best FL at 0, fxpq_stats at 8
-    res = torch.empty(len(items) * stride, dtype=torch.uint8, device=dev)
     err = torch.empty(len(items) * nfl, dtype=torch.float64, device=dev)
     ws = F.workspace(F.fxpq_fl_search_batch_workspace(len(items)), dev)
     base = res.data_ptr()
@@ -49,15 +47,29 @@ def search_fmts(items, stream=None):
     for i, (x, k) in enumerate(items):
         x = x.reshape(-1)
         batch.append(L.FlSearchItem(x.data_ptr(), x.numel(), -1, k, k, FL_LO, FL_HI, err.data_ptr() + 8 * nfl * i,
-                                    base + stride * i, base + stride * i + 8))
+                                    base + REC * i, base + REC * i + 8))
     F.fxpq_fl_search_batch(batch, ws, stream)
-    host = bytes(res.cpu().numpy().tobytes())
+
+
+def decode_fmts(host: bytes, ks):
+    """The chosen (k, S, FL) per search from the read-back result records (sign strategy of Sec. IV-A.3)."""
     out = []
-    for i, (_, k) in enumerate(items):
-        best = int.from_bytes(host[stride * i:stride * i + 4], "little", signed=True)
-        st = L.Stats.from_buffer_copy(host[stride * i + 8:stride * i + 8 + ctypes.sizeof(L.Stats)])
+    for i, k in enumerate(ks):
+        best = int.from_bytes(host[REC * i:REC * i + 4], "little", signed=True)
+        st = L.Stats.from_buffer_copy(host[REC * i + 8:REC * i + 8 + ctypes.sizeof(L.Stats)])
         out.append(F.fmt(k, st.is_signed, best))
     return out
+
+
+def search_fmts(items, stream=None):
+    """FL searches at one wordlength each, as one batch; one device-to-host read.
+
+    items: list of (tensor, k).  Returns the chosen (k, S, FL) per item."""
+    if not items:
+        return []
+    res = torch.empty(len(items) * REC, dtype=torch.uint8, device=items[0][0].device)
+    launch_searches(items, res, stream)
+    return decode_fmts(bytes(res.cpu().numpy().tobytes()), [k for _, k in items])
 
 
 def search_fmt(x: torch.Tensor, k: int, stream=None) -> L.Fmt:
@@ -87,7 +99,8 @@ class QNet:
     def quantize_params(self, weights_dev, plan, stream=None):
         """weights_dev: name -> (fp32 KRSC weight, fp32 bias) device tensors; plan: wordlengths.
 
-        Every parameter's FL search is launched first (one read-back), then every quantization."""
+        Every parameter's FL search runs as one batch, every quantization as one launch reading the
+        chosen formats on the device, and one read-back returns the formats and the L1 bounds."""
         shapes = {"input": (self.hw, self.hw, self.cp_in)}
         searches, owners = [], []
         dev = next(iter(weights_dev.values()))[0].device
@@ -117,35 +130,46 @@ class QNet:
                 searches.append((r, plan[nm]["r"]))
                 owners.append((nm, "r"))
                 shapes[nm] = (1, 1, Cp)
-        for (nm, key), f in zip(owners, search_fmts(searches, stream)):
-            self.fmts[nm][key] = f
-        rcodes = {}
-        # per conv layer: the largest L1 norm of an output channel's one-plane weight codes (lets the
-        # tensor-core contraction plan longer exact fp32 groups), read back with the avg-pool codes
+        # One buffer read back once: the search records, then the weight-code L1 bounds (int64 per
+        # conv layer), then the avg-pool reciprocal codes (int32).  The quantization reads each
+        # tensor's S and FL from the search records on the device (fxpq_quantize_batch).
         conv_names = [L_["name"] for L_ in self.layers if L_["type"] == "conv"]
-        l1 = torch.zeros(max(1, len(conv_names)), dtype=torch.int64, device=dev)
+        avg_names = [L_["name"] for L_ in self.layers if L_["type"] == "avgpool"]
+        n_s = len(searches)
+        off_l1 = n_s * REC
+        off_rc = off_l1 + 8 * len(conv_names)
+        buf = torch.zeros(off_rc + 4 * len(avg_names) + 8, dtype=torch.uint8, device=dev)
+        launch_searches(searches, buf, stream)
+        base = buf.data_ptr()
+        rec = {key: base + REC * i for i, key in enumerate(owners)}
+        items = []
         for i, L_ in enumerate(self.layers):
             nm = L_["name"]
             if L_["type"] == "conv":
                 w, b = weights_dev[nm]
                 K, R, _, C = w.shape
                 Cp = shapes[self._src(i, L_)][2]
-                fw, fb = self.fmts[nm]["w"], self.fmts[nm]["b"]
-                wq = torch.empty(K * R * R * Cp * F.planes(fw), dtype=torch.float16, device=dev)
-                F.fxpq_quantize_rows(w.reshape(-1, C), K * R * R, C, fw, Cp, wq, stream)
-                if F.planes(fw) == 1:
-                    F.fxpq_code_l1max(wq, K, R * R * Cp, l1[conv_names.index(nm):], stream)
+                kw, kb = plan[nm]["w"], plan[nm]["b"]
+                wq = torch.empty(K * R * R * Cp * (2 if kw > 8 else 1), dtype=torch.float16, device=dev)
                 bq = torch.empty(K, dtype=torch.int32, device=dev)
-                F.fxpq_quantize(b, fb, F.DT_I32, bq, stream)
+                l1p = base + off_l1 + 8 * conv_names.index(nm) if kw <= 8 else None
+                items.append(L.QuantizeItem(w.data_ptr(), wq.data_ptr(), L.QB_ROWS_F16, kw, K * R * R, C, Cp, R * R, 0,
+                                            rec[(nm, "w")], rec[(nm, "w")] + 8, l1p))
+                items.append(L.QuantizeItem(b.data_ptr(), bq.data_ptr(), L.QB_FLAT_I32, kb, K, 0, 0, 1, 0,
+                                            rec[(nm, "b")], rec[(nm, "b")] + 8, None))
                 self.q[nm] = (wq, bq)
             elif L_["type"] == "avgpool":
-                rc = torch.empty(1, dtype=torch.int32, device=dev)
-                F.fxpq_quantize(recips[nm], self.fmts[nm]["r"], F.DT_I32, rc, stream)
-                rcodes[nm] = rc
-        l1_host = l1.cpu().tolist()
-        self.w_l1 = {nm: int(l1_host[j]) for j, nm in enumerate(conv_names)}
-        for nm, rc in rcodes.items():
-            self.q[nm] = (None, int(rc.item()))
+                items.append(L.QuantizeItem(recips[nm].data_ptr(), base + off_rc + 4 * avg_names.index(nm),
+                                            L.QB_FLAT_I32, plan[nm]["r"], 1, 0, 0, 1, 0,
+                                            rec[(nm, "r")], rec[(nm, "r")] + 8, None))
+        F.fxpq_quantize_batch(items, stream)
+        host = bytes(buf.cpu().numpy().tobytes())
+        for (nm, key), f in zip(owners, decode_fmts(host, [k for _, k in searches])):
+            self.fmts[nm][key] = f
+        self.w_l1 = {nm: int.from_bytes(host[off_l1 + 8 * j:off_l1 + 8 * j + 8], "little", signed=True)
+                     for j, nm in enumerate(conv_names)}
+        for j, nm in enumerate(avg_names):
+            self.q[nm] = (None, int.from_bytes(host[off_rc + 4 * j:off_rc + 4 * j + 4], "little", signed=True))
         self.shapes = shapes
 
     # ------------------------------------------------------------------ one C-Block on device tensors

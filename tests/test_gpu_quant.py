@@ -196,3 +196,53 @@ def test_fl_search_batch_matches_oracle(F):
         assert s.is_signed == oS and s.n == x.size
         if x.size:
             assert s.min == ost["min"] and s.max == ost["max"] and s.sum == ost["sum"] and s.sumsq == ost["sumsq"]
+
+
+def test_quantize_batch_device_formats(F):
+    """fxpq_quantize_batch reads S and FL from device memory: rows items (one and two planes, padded
+    and unpadded channels, with and without the L1 bound) and flat int32 items equal the oracle's
+    quantizer; the L1 bound equals the largest per-output-channel sum of |code|."""
+    import paper_2203_12091_gb300._lib as L
+    rng = np.random.default_rng(5)
+    cases = [  # kind, k, S, fl, K, RS, C, Cp, want_l1
+        ("rows", 8, 1, 9, 64, 9, 64, 64, True),
+        ("rows", 5, 1, 6, 32, 9, 3, 8, True),
+        ("rows", 16, 1, 14, 16, 9, 8, 8, False),
+        ("rows", 12, 0, 7, 8, 1, 40, 40, False),
+        ("flat", 16, 1, 20, 1000, 0, 0, 0, False),
+        ("flat", 7, 0, 3, 1, 0, 0, 0, False),
+    ]
+    fmt_buf = torch.zeros(len(cases) * 64, dtype=torch.uint8, device="cuda")
+    host_fmt = bytearray(len(cases) * 64)
+    items, keep = [], []
+    l1 = torch.zeros(len(cases), dtype=torch.int64, device="cuda")
+    for i, (kind, k, S, fl, K, RS, C, Cp, want_l1) in enumerate(cases):
+        host_fmt[64 * i:64 * i + 4] = int(fl).to_bytes(4, "little", signed=True)
+        st = L.Stats(0.0, 0.0, S, 0, 0.0, 0.0, 0)
+        host_fmt[64 * i + 8:64 * i + 8 + ctypes.sizeof(L.Stats)] = bytes(st)
+        if kind == "rows":
+            x = (rng.standard_normal((K * RS, C)) * 2.0 ** (-fl + k - 3)).astype(np.float32)
+            out = torch.empty(K * RS * Cp * (2 if k > 8 else 1), dtype=torch.float16, device="cuda")
+        else:
+            x = (rng.standard_normal(K) * 2.0 ** (-fl + k - 2)).astype(np.float32)
+            out = torch.empty(K, dtype=torch.int32, device="cuda")
+        xd = torch.from_numpy(x).cuda()
+        keep.append((xd, out, x))
+        base = fmt_buf.data_ptr() + 64 * i
+        items.append(L.QuantizeItem(xd.data_ptr(), out.data_ptr(), L.QB_ROWS_F16 if kind == "rows" else L.QB_FLAT_I32,
+                                    k, K * RS if kind == "rows" else K, C, Cp, max(RS, 1), 0, base, base + 8,
+                                    l1.data_ptr() + 8 * i if want_l1 else None))
+    fmt_buf.copy_(torch.frombuffer(host_fmt, dtype=torch.uint8))
+    F.fxpq_quantize_batch(items)
+    torch.cuda.synchronize()
+    assert F.fxpq_get_device_status() == 0
+    l1h = l1.cpu().numpy()
+    for i, ((kind, k, S, fl, K, RS, C, Cp, want_l1), (xd, out, x)) in enumerate(zip(cases, keep)):
+        want = np.asarray(oracle.quantize(x, k, S, fl)).reshape(x.shape)
+        if kind == "rows":
+            got = F.codes_to_int(out.cpu(), F.fmt(k, S, fl), (K * RS, Cp)).numpy()
+            assert np.array_equal(got[:, :C], want) and np.all(got[:, C:] == 0)
+            if want_l1:
+                assert l1h[i] == np.abs(want).reshape(K, -1).sum(axis=1).max()
+        else:
+            assert np.array_equal(out.cpu().numpy(), want)
