@@ -317,6 +317,23 @@ FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_imag
                              int64_t* d_logits, int32_t* h_logits_scale, void* d_ws, size_t ws_bytes,
                              void* stream);
 
+/* Calibration of the activation formats in the forward optimizer's order (Sec. IV-C; reading 9 of
+ * the design notes): the input FxP-QLayer's FL is searched on the fp32 calibration images, then
+ * layer by layer, with every earlier layer already quantized, the FL of each op's output QLayer is
+ * searched on the fp32 nearest-even image of its exact C-Block output (conv: one contraction to
+ * int64 values, the QLayer applied twice; eltwise / avg-pool: their F32 and CODES modes).  S is
+ * picked from the data (Sec. IV-A.3); FLs in [fl_lo, fl_hi], exact ties to the smaller FL.
+ *   h_net: every parameter quantized (d_w, d_bias, fmt_w, fmt_b, recip_code, w_l1); fmt_in.bits and
+ *          each op's fmt_y.bits give the wordlengths (their S and FL are ignored);
+ *   h_fmt_in: the chosen input format; h_fmt_y[n_ops]: each op's output format (a max-pool passes
+ *          its input's on; the last op's entry is copied unchanged).
+ * The host waits for each search (one device-to-host read per QLayer).  Workspace:
+ * fxpq_net_calibrate_workspace(h_net, n_calib) bytes, 256-byte aligned. */
+FXPQ_API size_t fxpq_net_calibrate_workspace(const fxpq_net* h_net, int32_t n_calib);
+FXPQ_API fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_calib_nchw, int32_t n_calib,
+                                        int32_t fl_lo, int32_t fl_hi, fxpq_fmt* h_fmt_in, fxpq_fmt* h_fmt_y,
+                                        void* d_ws, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the latched device status (FXPQ_OK if none). */
 FXPQ_API fxpq_status fxpq_get_device_status(void* stream);
 

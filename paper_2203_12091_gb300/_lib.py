@@ -69,6 +69,8 @@ _SIGS = {
     "fxpq_fl_search_batch_workspace": (SZ, [I32]),
     "fxpq_fl_search_batch": (I32, [VP, I32, VP, SZ, VP]),
     "fxpq_quantize_batch": (I32, [VP, I32, VP]),
+    "fxpq_net_calibrate_workspace": (SZ, [VP, I32]),
+    "fxpq_net_calibrate": (I32, [VP, VP, I32, I32, I32, VP, VP, VP, SZ, VP]),
     "fxpq_quantize_images": (I32, [VP, I32, I32, I32, I32, Fmt, I32, VP, VP]),
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),

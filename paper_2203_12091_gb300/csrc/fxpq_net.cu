@@ -1,6 +1,7 @@
 // fxpq_net.cu -- integer-only network forward (Sec. IV-A.2: FxP-QLayers as vertices, C-Blocks as
 // edges).  Host-side driver: derives every slot's shape, carves the slots out of the caller's
 // workspace, and launches the C-Block kernels in order on the caller's stream.
+#include <cstring>
 #include <vector>
 
 #include "fxpq_common.cuh"
@@ -158,6 +159,162 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
                 st = FXPQ_ERR_INVALID_ARG;
         }
         if (st != FXPQ_OK) return st;
+    }
+    return FXPQ_OK;
+}
+
+// ------------------------------------------------------------------------------------------
+// Calibration of the activation formats (Sec. IV-C: the forward optimizer visits the layers in
+// order; every earlier layer is already quantized when a layer's output FL is searched).
+// ------------------------------------------------------------------------------------------
+namespace {
+
+struct CalibLayout {
+    std::vector<Slot> slots;
+    size_t slots_bytes = 0, acc_off = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, total = 0;
+};
+
+fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
+    fxpq_status st = plan_net(net, n, L.slots, L.slots_bytes);
+    if (st != FXPQ_OK) return st;
+    // largest per-op output (elements) for the int64 contraction values and their fp32 image
+    size_t max_out = 1;
+    for (int i = 0; i < net->n_ops - 1; ++i) {
+        const fxpq_op_desc& o = net->ops[i];
+        const Slot& d = L.slots[o.dst];
+        const size_t e = (size_t)n * d.H * d.W * d.Cp;
+        if (e > max_out) max_out = e;
+    }
+    const size_t img = (size_t)n * net->C * net->H * net->W;
+    L.acc_off = L.slots_bytes;
+    L.f32_off = L.acc_off + align256(max_out * sizeof(int64_t));
+    L.fls_off = L.f32_off + align256((max_out > img ? max_out : img) * sizeof(float));
+    L.rec_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
+    L.err_off = L.rec_off + 256;
+    L.total = L.err_off + align256(32 * sizeof(double));
+    return FXPQ_OK;
+}
+
+// FL search of one fp32 tensor at wordlength k, S picked from the data; waits for the result.
+fxpq_status calib_search(const float* d_x, int64_t n, int k, int fl_lo, int fl_hi, char* base, const CalibLayout& L,
+                         cudaStream_t s, fxpq_fmt& out) {
+    int32_t* d_best = reinterpret_cast<int32_t*>(base + L.rec_off);
+    fxpq_stats* d_stats = reinterpret_cast<fxpq_stats*>(base + L.rec_off + 64);
+    fxpq_status st = fxpq_fl_search(d_x, n, -1, k, k, fl_lo, fl_hi, reinterpret_cast<double*>(base + L.err_off),
+                                    d_best, d_stats, base + L.fls_off, fxpq_fl_search_workspace(n), s);
+    if (st != FXPQ_OK) return st;
+    unsigned char rec[64 + sizeof(fxpq_stats)];
+    if (cudaMemcpyAsync(rec, base + L.rec_off, sizeof(rec), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return FXPQ_ERR_CUDA;
+    int32_t best;
+    fxpq_stats stats;
+    memcpy(&best, rec, sizeof(best));
+    memcpy(&stats, rec + 64, sizeof(stats));
+    out.bits = k;
+    out.is_signed = stats.is_signed;
+    out.fl = best;
+    return FXPQ_OK;
+}
+
+}  // namespace
+
+extern "C" size_t fxpq_net_calibrate_workspace(const fxpq_net* h_net, int32_t n_calib) {
+    CalibLayout L;
+    if (plan_calib(h_net, n_calib, L) != FXPQ_OK) return 0;
+    return L.total + 256;
+}
+
+extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_calib_nchw, int32_t n_calib,
+                                          int32_t fl_lo, int32_t fl_hi, fxpq_fmt* h_fmt_in, fxpq_fmt* h_fmt_y,
+                                          void* d_ws, size_t ws_bytes, void* stream) {
+    CalibLayout L;
+    fxpq_status st = plan_calib(h_net, n_calib, L);
+    if (st != FXPQ_OK) return st;
+    if (n_calib < 1 || !d_calib_nchw || !h_fmt_in || !h_fmt_y) return FXPQ_ERR_INVALID_ARG;
+    if (fl_lo < -32 || fl_hi > 40 || fl_lo > fl_hi || fl_hi - fl_lo > 31) return FXPQ_ERR_INVALID_ARG;
+    if (!d_ws || ws_bytes < L.total || !fxpq::aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
+    cudaStream_t s = fxpq::as_stream(stream);
+    char* base = static_cast<char*>(d_ws);
+    auto ptr = [&](int slot) { return static_cast<void*>(base + L.slots[slot].offset); };
+    int64_t* acc = reinterpret_cast<int64_t*>(base + L.acc_off);
+    float* f32 = reinterpret_cast<float*>(base + L.f32_off);
+    std::vector<fxpq_fmt> fmt(h_net->n_slots, fxpq_fmt{0, 0, 0});
+
+    // input FxP-QLayer: FL search on the fp32 images, then the codes
+    const int64_t n_img = (int64_t)n_calib * h_net->C * h_net->H * h_net->W;
+    st = calib_search(d_calib_nchw, n_img, h_net->fmt_in.bits, fl_lo, fl_hi, base, L, s, fmt[0]);
+    if (st != FXPQ_OK) return st;
+    *h_fmt_in = fmt[0];
+    st = fxpq_quantize_images(d_calib_nchw, n_calib, h_net->C, h_net->H, h_net->W, fmt[0], h_net->Cp_in, ptr(0), s);
+    if (st != FXPQ_OK) return st;
+
+    for (int i = 0; i < h_net->n_ops; ++i) {
+        const fxpq_op_desc& o = h_net->ops[i];
+        h_fmt_y[i] = o.fmt_y;
+        if (o.last) break;  // the logits layer has no QLayer to calibrate
+        const Slot& s0 = L.slots[o.src0];
+        const Slot& d = L.slots[o.dst];
+        const int64_t n_out = (int64_t)n_calib * d.H * d.W * d.Cp;
+        fxpq_fmt fy{o.fmt_y.bits, 0, 0};
+        switch (o.op) {
+            case FXPQ_OP_MAXPOOL:
+                fy = fmt[o.src0];  // no QLayer follows a max-pool
+                st = fxpq_maxpool(ptr(o.src0), n_calib, s0.H, s0.W, s0.Cp, fmt[o.src0], o.R, o.stride, o.pad,
+                                  ptr(o.dst), s);
+                break;
+            case FXPQ_OP_CONV: {
+                // one contraction with exact int64 values; the QLayer runs twice (fp32 image for the
+                // search, then the codes)
+                fxpq_conv_desc cd;
+                cd.N = n_calib;
+                cd.H = s0.H;
+                cd.W = s0.W;
+                cd.C = s0.Cp;
+                cd.Cp = s0.Cp;
+                cd.K = o.K;
+                cd.R = o.R;
+                cd.S = o.S;
+                cd.stride = o.stride;
+                cd.pad = o.pad;
+                cd.relu = o.relu;
+                cd.out_mode = FXPQ_OUT_ACC64;
+                cd.fmt_x = fmt[o.src0];
+                cd.fmt_w = o.fmt_w;
+                cd.fmt_b = o.fmt_b;
+                cd.fmt_y = fy;
+                cd.w_l1 = o.w_l1;
+                int32_t sc = 0;
+                st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, nullptr, 0, s);
+                if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_F32, fy, f32, s);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_CODES, fy, ptr(o.dst), s);
+                break;
+            }
+            case FXPQ_OP_ELTWISE: {
+                const int64_t npix = (int64_t)n_calib * s0.H * s0.W;
+                st = fxpq_eltwise(ptr(o.src0), fmt[o.src0], ptr(o.src1), fmt[o.src1], npix, s0.Cp, o.relu, FXPQ_OUT_F32,
+                                  fy, f32, nullptr, s);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK)
+                    st = fxpq_eltwise(ptr(o.src0), fmt[o.src0], ptr(o.src1), fmt[o.src1], npix, s0.Cp, o.relu,
+                                      FXPQ_OUT_CODES, fy, ptr(o.dst), nullptr, s);
+                break;
+            }
+            case FXPQ_OP_AVGPOOL:
+                st = fxpq_avgpool(ptr(o.src0), n_calib, s0.H, s0.W, s0.Cp, fmt[o.src0], o.recip_code, o.fmt_w,
+                                  FXPQ_OUT_F32, fy, f32, nullptr, s);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK)
+                    st = fxpq_avgpool(ptr(o.src0), n_calib, s0.H, s0.W, s0.Cp, fmt[o.src0], o.recip_code, o.fmt_w,
+                                      FXPQ_OUT_CODES, fy, ptr(o.dst), nullptr, s);
+                break;
+            default:
+                st = FXPQ_ERR_INVALID_ARG;
+        }
+        if (st != FXPQ_OK) return st;
+        fmt[o.dst] = fy;
+        h_fmt_y[i] = fy;
     }
     return FXPQ_OK;
 }

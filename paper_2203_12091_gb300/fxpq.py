@@ -108,6 +108,20 @@ def fxpq_quantize_batch(items, stream=None):
                                                                 _s(stream)))
 
 
+def fxpq_net_calibrate_workspace(net, n_calib: int) -> int:
+    return L.lib().fxpq_net_calibrate_workspace(ctypes.byref(net), n_calib)
+
+
+def fxpq_net_calibrate(net, calib_nchw, n_calib: int, fl_lo: int, fl_hi: int, ws, stream=None):
+    """Returns (input format, [output format per op])."""
+    fin = Fmt()
+    fys = (Fmt * net.n_ops)()
+    L.check("fxpq_net_calibrate", L.lib().fxpq_net_calibrate(
+        ctypes.byref(net), _p(calib_nchw), n_calib, fl_lo, fl_hi, ctypes.byref(fin), ctypes.cast(fys, ctypes.c_void_p),
+        _p(ws), ws.numel(), _s(stream)))
+    return fin, list(fys)
+
+
 def stats_from_device(stats_bytes) -> Stats:
     return Stats.from_buffer_copy(bytes(stats_bytes.cpu().numpy().tobytes()))
 

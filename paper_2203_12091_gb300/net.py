@@ -213,39 +213,22 @@ class QNet:
 
     # ------------------------------------------------------------------ calibration (Sec. IV-C order)
     def calibrate(self, calib_images, plan, stream=None):
+        """Activation formats in the forward optimizer's order, by fxpq_net_calibrate on the op list (the
+        planned wordlengths in, the searched S and FL out); then the final op list."""
         self._dev = calib_images.device
         N = calib_images.shape[0]
-        fin = search_fmt(calib_images, plan["input"], stream)
-        self.fmts["input"] = {"a": fin}
-        x0 = torch.empty(N * self.hw * self.hw * self.cp_in * F.planes(fin), dtype=torch.float16, device=self._dev)
-        F.fxpq_quantize_images(calib_images, fin, self.cp_in, x0, stream)
-        env = {"input": (x0, fin)}
         last = len(self.layers) - 1
+        self.fmts["input"] = {"a": F.fmt(plan["input"], 0, 0)}
         for i, L_ in enumerate(self.layers):
-            nm = L_["name"]
-            if i == last:
-                break
-            if L_["type"] == "maxpool":
-                src = self._src(i, L_)
-                self.fmts[nm]["a"] = env[src][1]
-                y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
-                env[nm] = (y, env[src][1])
-                continue
-            if L_["type"] == "conv":
-                # one contraction: exact C-Block values, then the FxP-QLayer twice (fp32 image for the
-                # FL search, then the codes in the chosen format)
-                acc, s = self.run_layer(i, env, N, F.OUT_ACC64, stream)
-                v = torch.empty(acc.numel(), dtype=torch.float32, device=self._dev)
-                F.fxpq_qlayer(acc, s, F.OUT_F32, None, v, stream)
-                fa = search_fmt(v, plan[nm]["a"], stream)
-                y = torch.empty(acc.numel() * F.planes(fa), dtype=torch.float16, device=self._dev)
-                F.fxpq_qlayer(acc, s, F.OUT_CODES, fa, y, stream)
-                self.fmts[nm]["a"] = fa
-            else:
-                v, _ = self.run_layer(i, env, N, F.OUT_F32, stream)
-                self.fmts[nm]["a"] = search_fmt(v, plan[nm]["a"], stream)
-                y, _ = self.run_layer(i, env, N, F.OUT_CODES, stream)
-            env[nm] = (y, self.fmts[nm]["a"])
+            if i < last and L_["type"] != "maxpool":
+                self.fmts[L_["name"]]["a"] = F.fmt(plan[L_["name"]]["a"], 0, 0)
+        self._build_ops()
+        ws = F.workspace(F.fxpq_net_calibrate_workspace(self.net, N), self._dev)
+        fin, fys = F.fxpq_net_calibrate(self.net, calib_images, N, FL_LO, FL_HI, ws, stream)
+        self.fmts["input"]["a"] = fin
+        for i, L_ in enumerate(self.layers):
+            if i < last:
+                self.fmts[L_["name"]]["a"] = fys[i]
         self._build_ops()
         return self.fmts
 
