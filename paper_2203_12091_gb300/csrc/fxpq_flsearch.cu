@@ -332,7 +332,6 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     if (threadIdx.x == 0) sm.mn = 0xFFFFFFFFu;
     unsigned tmn = 0xFFFFFFFFu, tmx = 0u;
     bool tnf = false;
-    const unsigned lt_mask = (1u << lane) - 1u;
 
     const long long start = (long long)blk * P.chunk;
     const long long end = min(start + (long long)P.chunk, P.n);
@@ -356,9 +355,9 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
                         tmx = max(tmx, ok);
                     }
                 }
-                const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
-                if (key[e] < NKEY && lane == (unsigned)(__ffs(grp) - 1))
-                    atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
+                // per-element shared-memory reduction (no value returned); lanes with equal keys
+                // serialise in the memory pipe instead of a warp-wide match
+                if (key[e] < NKEY) atomicAdd(&sm.cnt[key[e]], 1u);
             }
         }
         __syncthreads();
@@ -393,12 +392,9 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
             load16<VEC>(P, tb, sub, end, v, key);
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-                const unsigned grp = __match_any_sync(0xFFFFFFFFu, (unsigned)key[e]);
-                const unsigned leader = (unsigned)(__ffs(grp) - 1);
-                unsigned base = 0u;
-                if (key[e] < NKEY && lane == leader) base = atomicAdd(&sm.cnt[key[e]], (unsigned)__popc(grp));
-                base = __shfl_sync(0xFFFFFFFFu, base, (int)leader);
-                if (key[e] < NKEY) sm.sorted[base + __popc(grp & lt_mask)] = v[e];
+                // each element takes the next free position of its key (order within a key is
+                // immaterial: every sum is exact)
+                if (key[e] < NKEY) sm.sorted[atomicAdd(&sm.cnt[key[e]], 1u)] = v[e];
             }
         }
         __syncthreads();
