@@ -66,7 +66,12 @@ struct TcParams {
     int nbuf;            // fp32 accumulator buffers in TMEM: 2, or 1 when BN = 256 needs running sums
     int patch;           // a tile is a TH x TW patch of one image and the A tile comes by TMA:
                          // 1: Cp % 64 == 0 (one 64-channel box per k-block, 128-byte swizzle);
-                         // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle)
+                         // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle);
+                         // 3: Cp == 8, window mode (one input window per tile and limb plane, taps as
+                         //    shifted descriptors, weights resident in shared memory)
+    int nacc;            // fp32 accumulators per TMEM buffer (window mode: one per limb pair)
+    int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
+    int win_bytes;       // window mode: bytes of one window (128-byte aligned)
     int TH, TW;          // patch shape (TH * TW = 128)
     int tiles_p, tiles_q;  // patches per image along P and Q
     ConvArgs a;
@@ -384,7 +389,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
     // fp32 accumulator buffers + integer running sums, rounded up to a power of two (BN = 256: two
     // buffers without running sums, or one buffer with them)
-    constexpr uint32_t USED_COLS = BN == 256 ? 512u : 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
+    // (the int64 instance also serves window mode: two buffers of up to four limb-pair accumulators)
+    constexpr uint32_t USED_COLS = (BN == 256 || sizeof(ACC) == 8) ? 512u : 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
     constexpr uint32_t TMEM_COLS = USED_COLS <= 256 ? 256u : 512u;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -400,6 +406,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
     const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue thread
     const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
+    const uint32_t wbar = smem_u32(bars + 2 * TC_STAGES + 9);      // window mode: resident weights loaded
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const ConvArgs& a = P.a;
@@ -418,6 +425,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         mbar_init(done_bar, 1);
         mbar_init(stg_full, EPI_THREADS);
         mbar_init(stg_free, 1);
+        mbar_init(wbar, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -431,7 +439,56 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp < 4 && P.patch) {
+    if (warp < 4 && P.patch == 3) {
+        // ============================================================ producer, window mode
+        // Stride 1, Cp == 8: the weights (per limb plane, kernel row r and tap pair sp, the box
+        // {8 ch, BN out ch, 2 taps}) are loaded once into the B region; per tile, one box per x limb
+        // plane holds the input window of TH + R - 1 rows by TW + S2 - 1 pixels (padding zero filled).
+        if (threadIdx.x == 0) {
+            const int np = P.S2 / 2;
+            const uint32_t wbox = (uint32_t)(BN * 32);
+            mbar_arrive_expect_tx(wbar, (uint32_t)(a.pw * a.R * np) * wbox);
+            for (int iw = 0; iw < a.pw; ++iw)
+                for (int r = 0; r < a.R; ++r)
+                    for (int sp = 0; sp < np; ++sp)
+                        tma_load_5d(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox, &P.tmap_w, 0, 0, 2 * sp,
+                                    r, iw, wbar);
+            const uint32_t win_tx = (uint32_t)(P.WW * P.WH * 16);
+            const int per_img = P.tiles_p * P.tiles_q;
+            uint32_t it = 0, stage = 0, phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+                const int tm = t / P.tiles_n;
+                const int n_img = tm / per_img, r = tm - n_img * per_img;
+                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
+                if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t fb = full0 + 8 * stage;
+                mbar_arrive_expect_tx(fb, (uint32_t)a.px * win_tx);
+                for (int ia = 0; ia < a.px; ++ia)
+                    tma_load_5d(smem_u32(sA + stage * A_BYTES) + (uint32_t)(ia * P.win_bytes), &P.tmap_x, 0, wq0, hp0,
+                                n_img, ia, fb);
+                ++it;
+                if (++stage == TC_STAGES) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            }
+            // bounded wait until the copies of the last stages and the weights have landed
+            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
+            for (uint32_t j = from; j < it; ++j) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
+                       clock64() - t0 < TC_WAIT_CYCLES) {
+                }
+            }
+            const long long t0 = clock64();
+            while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
+            }
+        }
+    } else if (warp < 4 && P.patch) {
         // ============================================================ producer, patch tiles
         // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
         // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
@@ -615,11 +672,105 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     const int cb = cw * CPW + c;
                     const int k0 = tn * BN + cb * 32;
                     const uint32_t run_col = run_base + cb * 32;
+                    if (sizeof(ACC) == 8 && P.patch == 3 && P.nacc == 4 && P.fast_store && a.sh >= 1 && a.sh <= 62) {
+                        // window mode, two-limb x and w, one-plane codes out: each 16-column half goes
+                        // from the four limb accumulators to packed codes before the next is loaded
+                        // (keeps the live 64-bit values to 16)
+                        const Epi64 e64 = make_epi64(a);
+                        const int k0 = tn * BN + cb * 32;
+                        const uint32_t abase = lane_base + buf * (uint32_t)(P.nacc * BN) + cb * 32;
+                        uint32_t w[16];
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf) {
+                            uint32_t fhh[16], fhl[16], flh[16], fll[16];
+                            tmem_ld16_nw(abase + 16 * hf, fhh);
+                            tmem_ld16_nw(abase + (uint32_t)BN + 16 * hf, fhl);
+                            tmem_ld16_nw(abase + (uint32_t)(2 * BN) + 16 * hf, flh);
+                            tmem_ld16_nw(abase + (uint32_t)(3 * BN) + 16 * hf, fll);
+                            tmem_wait_ld();
+                            reg_fence(fhh);
+                            reg_fence(fhl);
+                            reg_fence(flh);
+                            reg_fence(fll);
+                            if (hf == 1 && c == CPW - 1) {
+                                tc_fence_before();
+                                mbar_arrive(accempty0 + 8 * buf);
+                            }
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) {
+                                int c2[2];
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    const int jj = 2 * j + h;
+                                    const int k = k0 + 16 * hf + jj;
+                                    const long long v = ((long long)__float2int_rn(__uint_as_float(fhh[jj])) << 16) +
+                                                        ((long long)(__float2int_rn(__uint_as_float(fhl[jj])) +
+                                                                     __float2int_rn(__uint_as_float(flh[jj])))
+                                                         << 8) +
+                                                        (long long)__float2int_rn(__uint_as_float(fll[jj]));
+                                    const int32_t b = (e64.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                    c2[h] = epi64_code(e64, v, b);
+                                }
+                                w[8 * hf + j] = pack_codes_f16(c2[0], c2[1]);
+                            }
+                        }
+                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int chunk = (cb & 1) * 4 + q;
+                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                        }
+                        continue;
+                    }
                     // One TMEM round trip per load batch: the fp32 group sums and, after the first group,
                     // the integer running sums are loaded together; the running-sum stores share one
                     // completion wait.
                     ACC acc[32];
-                    if (sizeof(ACC) == 8) {
+                    if (sizeof(ACC) == 8 && P.patch == 3) {
+                        // window mode: one accumulator per limb pair (ia, iw), combined with its weight
+                        // 2^(8 ((px-1-ia) + (pw-1-iw))); each is an exact integer below 2^24
+                        const uint32_t abase = lane_base + buf * (uint32_t)(P.nacc * BN) + cb * 32;
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf) {
+                            if (P.nacc == 4) {
+                                // two-limb x and w: the four accumulators share one load round trip;
+                                // v = 2^16 S_hh + 2^8 (S_hl + S_lh) + S_ll, the middle pair summed in 32 bits
+                                uint32_t fhh[16], fhl[16], flh[16], fll[16];
+                                tmem_ld16_nw(abase + 16 * hf, fhh);
+                                tmem_ld16_nw(abase + (uint32_t)BN + 16 * hf, fhl);
+                                tmem_ld16_nw(abase + (uint32_t)(2 * BN) + 16 * hf, flh);
+                                tmem_ld16_nw(abase + (uint32_t)(3 * BN) + 16 * hf, fll);
+                                tmem_wait_ld();
+                                reg_fence(fhh);
+                                reg_fence(fhl);
+                                reg_fence(flh);
+                                reg_fence(fll);
+#pragma unroll
+                                for (int j = 0; j < 16; ++j) {
+                                    const int hh = __float2int_rn(__uint_as_float(fhh[j]));
+                                    const int mid = __float2int_rn(__uint_as_float(fhl[j])) +
+                                                    __float2int_rn(__uint_as_float(flh[j]));
+                                    const int ll = __float2int_rn(__uint_as_float(fll[j]));
+                                    acc[16 * hf + j] = ((ACC)hh << 16) + ((ACC)mid << 8) + (ACC)ll;
+                                }
+                            } else {
+#pragma unroll
+                                for (int j = 0; j < 16; ++j) acc[16 * hf + j] = 0;
+                                for (int ia = 0; ia < a.px; ++ia)
+                                    for (int iw = 0; iw < a.pw; ++iw) {
+                                        uint32_t f16[16];
+                                        tmem_ld16_nw(abase + (uint32_t)((ia * a.pw + iw) * BN) + 16 * hf, f16);
+                                        tmem_wait_ld();
+                                        reg_fence(f16);
+                                        const int sh = 8 * ((a.px - 1 - ia) + (a.pw - 1 - iw));
+#pragma unroll
+                                        for (int j = 0; j < 16; ++j)
+                                            acc[16 * hf + j] += ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << sh;
+                                    }
+                            }
+                        }
+                    } else if (sizeof(ACC) == 8) {
                         // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
 #pragma unroll
                         for (int hf = 0; hf < 2; ++hf) {
@@ -767,6 +918,55 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             }
         }
         if (leader) bulk_wait0();  // every output store has completed
+    } else if (lane == 0 && P.patch == 3) {
+        // ============================================================ MMA issue, window mode
+        // Per tile and limb pair (ia, iw): R * S2/2 MMAs of K = 16 (two taps of 8 channels).  The A
+        // operand of taps (r, 2sp), (r, 2sp + 1) is the window shifted by (r, 2sp) pixels: K-major
+        // without swizzle, the two K core matrices one pixel (16 bytes) apart, the 8-row groups (the
+        // patch rows, TW = 8) one window row apart.  B is the resident box (iw, r, sp).
+        const int np = P.S2 / 2;
+        const uint32_t wbox = (uint32_t)(BN * 32);
+        uint32_t stage = 0, phase = 0, gcount = 0;
+        bool ok = wait_bounded(wbar, 0, abort, P.status);
+        tc_fence_after();
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            const uint32_t buf = gcount & 1;
+            if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
+                !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d0 = tmem + buf * (uint32_t)(P.nacc * BN);
+            const uint32_t wa = smem_u32(sA + stage * A_BYTES);
+            for (int ia = 0; ia < a.px; ++ia)
+                for (int iw = 0; iw < a.pw; ++iw) {
+                    const uint32_t d = d0 + (uint32_t)((ia * a.pw + iw) * BN);
+                    uint32_t accum = 0;
+                    for (int r = 0; r < a.R; ++r)
+                        for (int sp = 0; sp < np; ++sp) {
+                            const uint64_t ad = make_sdesc_noswz(
+                                wa + (uint32_t)(ia * P.win_bytes + (r * P.WW + 2 * sp) * 16), 16, (uint32_t)(P.WW * 16));
+                            const uint64_t bd =
+                                make_sdesc_noswz(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox,
+                                                 (uint32_t)(BN * 16), 128);
+                            tc_mma(d, ad, bd, IDESC, accum);
+                            accum = 1;
+                        }
+                }
+            tc_commit(empty0 + 8 * stage);
+            if (++stage == TC_STAGES) {
+                stage = 0;
+                phase ^= 1;
+            }
+            tc_commit(accfull0 + 8 * buf);
+            ++gcount;
+        }
+        // every MMA issued by this thread has completed once `done` fires
+        tc_commit(done_bar);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
+        }
     } else if (lane == 0) {
         // ============================================================ MMA issue (one thread of MMA_WARP)
         // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
@@ -961,11 +1161,65 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
+        P.patch = 0;
+        P.nacc = 1;
+        // window mode for 8-channel stride-1 layers with at most 64 output channels: 8 x 16 output
+        // patches, one input window per tile and limb plane, weights resident in shared memory, one
+        // exact fp32 accumulator per limb pair (R * S2 * 8 products each)
+        {
+            const int S2 = (a.S + 1) & ~1;
+            const int WW = 8 + S2 - 1, WH = 16 + a.R - 1;
+            const int win_bytes = (WW * WH * 16 + 127) / 128 * 128;
+            bool ok = a.stride == 1 && a.Cp == 8 && a.K <= 64 && a.N > 0 && a.R * S2 <= 16 && WW <= 256 &&
+                      WH <= 256 && a.px * win_bytes <= TC_BM * TC_BK * 2 &&
+                      a.pw * a.R * (S2 / 2) * 64 * 32 <= tc_stages(64) * 64 * TC_BK * 2 && !conv_path_is("tc_rows") &&
+                      !conv_path_is("tc_nowin");
+            for (int ia = 0; ok && ia < a.px; ++ia)
+                for (int iw = 0; iw < a.pw; ++iw)
+                    if ((double)limb_max(d.fmt_x, ia) * limb_max(d.fmt_w, iw) * a.R * S2 * 8 >= 16777216.0) ok = false;
+            if (ok) {
+                const cuuint64_t xdims[5] = {8, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N, (cuuint64_t)a.px};
+                const cuuint64_t xstrides[4] = {16, (cuuint64_t)a.W * 16, (cuuint64_t)a.H * a.W * 16,
+                                                (cuuint64_t)a.x_ps * 2};
+                const cuuint32_t xbox[5] = {8, (cuuint32_t)WW, (cuuint32_t)WH, 1, 1};
+                // weights as {c, out channel, s, r, plane} (strides in that order, not memory order)
+                const cuuint64_t wdims[5] = {8, (cuuint64_t)a.K, (cuuint64_t)a.S, (cuuint64_t)a.R, (cuuint64_t)a.pw};
+                const cuuint64_t wstrides[4] = {(cuuint64_t)a.R * a.S * 16, 16, (cuuint64_t)a.S * 16,
+                                                (cuuint64_t)a.w_ps * 2};
+                const cuuint32_t wbox[5] = {8, 64, 2, 1, 1};
+                const cuuint32_t es5[5] = {1, 1, 1, 1, 1};
+                CUtensorMap mx, mw;
+                if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.x), xdims, xstrides, xbox, es5,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
+                    enc(&mw, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.w), wdims, wstrides, wbox, es5,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
+                    P.tmap_x = mx;
+                    P.tmap_w = mw;
+                    P.patch = 3;
+                    P.TW = 8;
+                    P.TH = 16;
+                    P.tiles_p = (a.P + 15) / 16;
+                    P.tiles_q = (a.Q + 7) / 8;
+                    P.S2 = S2;
+                    P.WW = WW;
+                    P.WH = WH;
+                    P.win_bytes = win_bytes;
+                    P.nacc = a.px * a.pw;
+                    P.n_groups = 1;
+                    P.g[0] = TcGroup{0, 1, 0, 0, 0};
+                    P.nbuf = 2;
+                    BN = 64;
+                    acc64 = true;  // the int64 instance: its TMEM holds two buffers of the limb accumulators
+                }
+            }
+        }
         // patch tiles for stride-1 layers whose taps are whole 64-channel blocks, or 8-channel inputs
         // (a k-block of 8 taps)
-        P.patch = 0;
         const bool narrow = a.Cp == 8;
-        if (a.stride == 1 && (P.cp64 || narrow) && a.P > 0 && a.Q > 0 && a.N > 0 && !conv_path_is("tc_rows")) {
+        if (P.patch == 0 && a.stride == 1 && (P.cp64 || narrow) && a.P > 0 && a.Q > 0 && a.N > 0 &&
+            !conv_path_is("tc_rows")) {
             int best_tw = 0, best_th = 0;
             long long best = 0;
             for (int tw = a.Q < TC_BM ? a.Q : TC_BM; tw >= 1; --tw) {

@@ -119,6 +119,11 @@ CASES = [
     # 8-channel stride-1 inputs: patch tiles with one box per tap (VGG conv1_1-like, two limbs)
     (2, 20, 3, 16, 5, 1, 2, (16, 1, 12), (16, 1, 14), (16, 20), True, 0, (8, 0, 3)),
     (3, 16, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 14), (16, 22), True, 0, (4, 0, 2)),
+    # window mode (8 stored channels, stride 1, K <= 64): ragged patches, 1x1 taps, one plane, ACC64
+    (2, 20, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 13), (16, 21), True, 0, (8, 0, 3)),
+    (2, 12, 8, 24, 1, 1, 0, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),
+    (1, 19, 5, 40, 3, 1, 1, (7, 1, 3), (6, 1, 6), (16, 12), False, 0, (8, 1, 2)),
+    (2, 17, 3, 32, 3, 1, 1, (16, 1, 11), (16, 1, 14), (16, 22), True, 1, None),
 ]
 
 
