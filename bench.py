@@ -297,6 +297,7 @@ def run_kernel(args):
     conv     : VGG-16 conv3_1-shaped C-Block, batch 64, 56x56x128 -> 256, 3x3 pad 1, 8-bit codes, with
                and without the weight-code L1 bound;
     flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid;
+    quantize : Q of 64M N(0,1) fp32 values to int8 codes and to an fp16 code tensor (HBM-bound);
     forward  : the integer forward of the workload (first plan, calibrated once), fxpq_net_forward alone."""
     import torch
     import __graft_entry__ as g
@@ -343,6 +344,25 @@ def run_kernel(args):
             ms = sum(ts) / len(ts)
             out[name] = {"ms": round(ms, 4), "gelem_s": round(n / (ms / 1e3) / 1e9, 2),
                          "hbm_gbs": round(4 * n / (ms / 1e3) / 1e9, 1)}
+    if args.kernel in ("quantize", "all"):
+        # Q on 64M fp32 values: 4 B read + 1 B (int8 codes) or 2 B (fp16 code tensor) written per value
+        n = 1 << 26
+        x = torch.from_numpy(synth.normal(n, 2)).cuda()
+        hbm = measured_peaks()[0]
+        for name, dt, bw in (("quantize_i8", F.DT_I8, 1), ("quantize_f16", F.DT_F16, 2)):
+            y = torch.empty(n * bw, dtype=torch.uint8, device="cuda")
+            ts = []
+            for i in range(args.warmup + args.steps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                F.fxpq_quantize(x, F.fmt(8, 1, 5), dt, y)
+                e1.record()
+                e1.synchronize()
+                if i >= args.warmup:
+                    ts.append(e0.elapsed_time(e1))
+            ms = sum(ts) / len(ts)
+            gbs = (4 + bw) * n / (ms / 1e3) / 1e9
+            out[name] = {"ms": round(ms, 4), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 3)}
     if args.kernel in ("forward", "all"):
         # the integer forward of the bench workload alone (one plan, calibrated once): the target of the
         # per-launch DRAM traffic capture of the conv kernels
@@ -373,7 +393,8 @@ def run_kernel(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=["conv", "flsearch", "forward", "all"], help="time one kernel case and exit")
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "forward", "all"],
+                    help="time one kernel case and exit")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)

@@ -222,14 +222,42 @@ def add_bias(acc, s_acc: int, bias, fl_b: int):
     return (acc << np.int64(-d)) + b, fl_b
 
 
-def cblock(acc, s_acc: int, bias, fl_b, relu: bool):
-    """C-Block output before its FxP-QLayer: MAC result + aligned bias, then ReLU.
-    Returns (int64 value, its scale exponent)."""
+def scale_layer(v, s_v: int, scale, fl_scale: int, shift, fl_shift: int):
+    """Scale layer on integers (Sec. IV-A.1, Eq. BatchNorm: BN(A) = aleph1 * A + aleph2, with aleph1 and
+    aleph2 quantized like weights and biases; Sec. IV-B: an integer multiplier and accumulator).  The
+    per-channel (last axis) product aleph1_code * v has scale s_v + FL_aleph1; aleph2 is aligned to it
+    like a bias (add_bias, with the same reading when its FL is finer).  Returns (value, scale)."""
+    v = np.asarray(v, dtype=np.int64)
+    m = np.asarray(scale, dtype=np.int64)
+    _check_range(v, 62 - int(np.max(np.abs(m), initial=0)).bit_length())
+    p = v * m
+    s_p = s_v + fl_scale
+    if shift is None:
+        return p, s_p
+    return add_bias(p, s_p, shift, fl_shift)
+
+
+def cblock(acc, s_acc: int, bias, fl_b, relu: bool, scale=None, fl_scale: int = 0, shift=None, fl_shift: int = 0):
+    """C-Block output before its FxP-QLayer: MAC result + aligned bias, the optional Scale layer
+    (CONV-Scale-ReLU, Sec. IV-B), then ReLU.  Returns (int64 value, its scale exponent)."""
     if bias is not None:
         acc, s_acc = add_bias(acc, s_acc, bias, fl_b)
+    if scale is not None:
+        acc, s_acc = scale_layer(acc, s_acc, scale, fl_scale, shift, fl_shift)
     if relu:
         acc = np.maximum(acc, 0)
     return acc, s_acc
+
+
+def bn_to_scale(gamma, beta, mean, var, eps=1e-5):
+    """Preprocessor (Sec. IV-A.1, Eq. BatchNorm_s1_s2): a BN layer becomes a Scale layer with
+    aleph1 = gamma / sqrt(var + eps) and aleph2 = beta - gamma * mean / sqrt(var + eps), in fp32 in that
+    order of operations."""
+    g, b, mu, v = (np.asarray(t, dtype=np.float32) for t in (gamma, beta, mean, var))
+    r = np.sqrt(v + np.float32(eps))
+    a1 = (g / r).astype(np.float32)
+    a2 = (b - (g * mu) / r).astype(np.float32)
+    return a1, a2
 
 
 def maxpool(x_nhwc, k: int, stride: int, pad: int) -> np.ndarray:

@@ -266,6 +266,52 @@ def test_bias_alignment_preserves_value():
             assert Fraction(vv, 2 ** s2) == Fraction(a, 2 ** s) + Fraction(bb, 2 ** flb)
 
 
+def test_scale_layer_cblock_equals_exact_bn_value():
+    """CONV-Scale-ReLU (Sec. IV-B): the integer C-Block value times 2^-s equals, as an exact rational,
+    relu(aleph1 * (acc 2^-s_acc + B 2^-FL_b) + aleph2) for every alignment case of both additions."""
+    rng = np.random.default_rng(18)
+    K = 7
+    acc = rng.integers(-2 ** 28, 2 ** 28, size=(9, K))
+    b = rng.integers(-2 ** 15, 2 ** 15, size=K)
+    sc = rng.integers(-2 ** 15, 2 ** 15, size=K)
+    sh = rng.integers(-2 ** 15, 2 ** 15, size=K)
+    for s_acc, flb, fls, flh, relu in [(12, 4, 14, 20, True), (12, 18, 9, 3, False), (5, 5, 15, 30, True),
+                                       (10, 2, 0, 22, False)]:
+        v, s = oracle.cblock(acc, s_acc, b, flb, relu, scale=sc, fl_scale=fls, shift=sh, fl_shift=flh)
+        for i in range(acc.shape[0]):
+            for k in range(K):
+                x = Fraction(int(acc[i, k]), 2 ** s_acc) + Fraction(int(b[k]), 2 ** flb)
+                y = Fraction(int(sc[k]), 2 ** fls) * x + Fraction(int(sh[k]), 2 ** flh)
+                if relu:
+                    y = max(y, Fraction(0))
+                assert Fraction(int(v[i, k]), 2 ** s) == y
+        # and the FxP-QLayer of it equals Q of the exact value
+        q = oracle.requant(v, s, 8, 1, 3)
+        for i in range(acc.shape[0]):
+            for k in range(K):
+                yv = Fraction(int(v[i, k]), 2 ** s) * 8
+                fl, cl = yv.numerator // yv.denominator, yv - yv.numerator // yv.denominator
+                r = fl + (1 if cl > Fraction(1, 2) or (cl == Fraction(1, 2) and fl % 2) else 0)
+                assert q[i, k] == min(max(r, -128), 127)
+
+
+def test_bn_to_scale_matches_the_formula():
+    """Eq. BatchNorm_s1_s2: aleph1 = gamma / sqrt(var + eps), aleph2 = beta - gamma mean / sqrt(var + eps),
+    within fp32 rounding of the float64 formula, and BN(a) = aleph1 a + aleph2."""
+    rng = np.random.default_rng(19)
+    g = rng.uniform(0.5, 2.0, 64).astype(np.float32)
+    be = rng.normal(0, 0.5, 64).astype(np.float32)
+    mu = rng.normal(0, 1, 64).astype(np.float32)
+    var = rng.uniform(0.1, 4.0, 64).astype(np.float32)
+    a1, a2 = oracle.bn_to_scale(g, be, mu, var)
+    r64 = np.sqrt(var.astype(np.float64) + 1e-5)
+    np.testing.assert_allclose(a1, g / r64, rtol=4e-7)
+    np.testing.assert_allclose(a2, be - g * mu.astype(np.float64) / r64, rtol=1e-5, atol=1e-6)
+    x = rng.normal(0, 1, 64)
+    bn = g * (x - mu) / r64 + be
+    np.testing.assert_allclose(a1 * x + a2, bn, rtol=1e-5, atol=1e-5)
+
+
 def test_maxpool_matches_window_max():
     rng = np.random.default_rng(9)
     x = rng.integers(0, 256, size=(2, 13, 11, 5))
