@@ -34,7 +34,20 @@ WORKLOADS = {
     "vgg16": {"arch": "vgg16", "batch": 64, "seed": 7, "plans": list(range(7, 39)), "calib": 8},
     "alexnet": {"arch": "alexnet", "batch": 256, "seed": 5, "plans": [5], "calib": 8},
     "resnet18": {"arch": "resnet18", "batch": 128, "seed": 6, "plans": [6], "calib": 8},
+    # ResNet-18 with its BN layers kept as Scale layers (bias-free convs), the paper's form
+    "resnet18_bn": {"arch": "resnet18_bn", "batch": 128, "seed": 6, "plans": [6], "calib": 8},
 }
+
+
+def device_params(arch, seed, dev):
+    """Seeded fp32 parameters on the device: conv name -> (weight, bias or None), BN conv name ->
+    (gamma, beta, mean, var)."""
+    import torch
+    W = synth.weights(arch, seed)
+    wdev = {nm: (torch.from_numpy(w).to(dev), None if b is None else torch.from_numpy(b).to(dev))
+            for nm, (w, b) in W.items()}
+    bn = {nm: tuple(torch.from_numpy(t).to(dev) for t in v) for nm, v in synth.bn_params(arch, seed + 100).items()}
+    return wdev, bn
 L2_BYTES = 129 * 1024 * 1024
 
 
@@ -115,10 +128,9 @@ def run_fxpq(args):
     wl = WORKLOADS[args.workload]
     arch, B = wl["arch"], wl["batch"]
     layers = synth.ARCHS[arch]()
-    W = synth.weights(arch, wl["seed"])
     imgs_np = synth.images(B, wl["seed"] + 1000 * rank)
     plans = [synth.bit_plan(arch, s) for s in wl["plans"]]
-    wdev = {nm: (torch.from_numpy(w).to(dev), torch.from_numpy(b).to(dev)) for nm, (w, b) in W.items()}
+    wdev, bndev = device_params(arch, wl["seed"], dev)
     imgs = torch.from_numpy(imgs_np).to(dev)
     pinned = torch.from_numpy(imgs_np).pin_memory()
     stream = torch.cuda.current_stream(dev)
@@ -128,7 +140,7 @@ def run_fxpq(args):
         q = QNet(layers, hw=224, cin=3)
         q._dev = dev
         plan = plans[(i + rank) % len(plans)]
-        q.quantize_params(wdev, plan)
+        q.quantize_params(wdev, plan, None, bndev)
         q.calibrate(images[: wl["calib"]], plan)
         logits, s = q.forward(images)
         return q, logits, s
@@ -254,10 +266,11 @@ def oracle_step(workload, n_images=1):
     arch = wl["arch"]
     layers = synth.ARCHS[arch]()
     W = synth.weights(arch, wl["seed"])
+    bn = synth.bn_params(arch, wl["seed"] + 100)
     imgs = synth.images(n_images, wl["seed"])
     plan = synth.bit_plan(arch, wl["plans"][0])
     t0 = time.perf_counter()
-    fm, qp = onet.calibrate(layers, W, imgs[:1], plan)
+    fm, qp = onet.calibrate(layers, W, imgs[:1], plan, bn)
     onet.forward(layers, fm, qp, imgs)
     return time.perf_counter() - t0
 
@@ -369,13 +382,12 @@ def run_kernel(args):
         from paper_2203_12091_gb300.net import QNet
         wl = WORKLOADS[args.workload]
         arch, B = wl["arch"], wl["batch"]
-        W = synth.weights(arch, wl["seed"])
         imgs = torch.from_numpy(synth.images(B, wl["seed"])).cuda()
-        wdev = {nm: (torch.from_numpy(w).cuda(), torch.from_numpy(b).cuda()) for nm, (w, b) in W.items()}
+        wdev, bndev = device_params(arch, wl["seed"], imgs.device)
         plan = synth.bit_plan(arch, wl["plans"][0])
         q = QNet(synth.ARCHS[arch](), hw=224, cin=3)
         q._dev = imgs.device
-        q.quantize_params(wdev, plan)
+        q.quantize_params(wdev, plan, None, bndev)
         q.calibrate(imgs[: wl["calib"]], plan)
         ts = []
         for i in range(args.warmup + args.steps):

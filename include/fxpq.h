@@ -224,6 +224,12 @@ FXPQ_API fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32
 /* most max|x code| * w_l1, which lets the tensor-core path keep longer reductions in exact    */
 /* fp32 groups and the epilogue in 32-bit arithmetic.  A value below the true norm voids the  */
 /* exactness guarantee; not part of the paper (an implementation bound).                      */
+/* Scale layer (optional; Sec. IV-A.1: a BN layer rewritten as aleph1 * A + aleph2, its two    */
+/* per-channel parameters quantized like weights and biases; Sec. IV-B: integer multiply and  */
+/* accumulate in the C-Block): when d_scale != NULL, after the bias alignment the value v of  */
+/* scale s becomes v * aleph1_code[o] of scale s + fmt_scale.fl, and aleph2_code[o] is aligned  */
+/* to it like the bias (delta2 = that scale - fmt_shift.fl, the same two cases); ReLU and the  */
+/* FxP-QLayer follow.  d_scale and d_shift are int32 code arrays [K], both set or both NULL.   */
 /* ---------------------------------------------------------------------------------------- */
 enum { FXPQ_OUT_CODES = 0, FXPQ_OUT_ACC64 = 1, FXPQ_OUT_F32 = 2 };
 
@@ -236,6 +242,9 @@ typedef struct {
     int32_t out_mode;          /* FXPQ_OUT_*                                                 */
     fxpq_fmt fmt_x, fmt_w, fmt_b, fmt_y;
     int64_t w_l1;              /* optional weight-code L1 bound (see above), 0 = none        */
+    fxpq_fmt fmt_scale, fmt_shift;  /* Scale layer aleph1 / aleph2 formats (if d_scale)      */
+    const int32_t* d_scale;    /* Scale layer aleph1 codes [K], or NULL (no Scale layer)     */
+    const int32_t* d_shift;    /* Scale layer aleph2 codes [K] (NULL iff d_scale is NULL)    */
 } fxpq_conv_desc;
 
 FXPQ_API size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc);
@@ -278,6 +287,15 @@ FXPQ_API fxpq_status fxpq_avgpool(const void* d_x, int32_t N, int32_t H, int32_t
                          int32_t recip_code, fxpq_fmt fmt_recip, int32_t out_mode, fxpq_fmt fmt_y,
                          void* d_y, int32_t* h_out_scale, void* stream);
 
+/* BN -> Scale preprocessing (Sec. IV-A.1, the BatchNorm rewrite): per channel,
+ *   aleph1 = gamma / sqrt(var + eps),  aleph2 = beta - (gamma * mean) / sqrt(var + eps),
+ * each operation one correctly rounded fp32 step in that order.  Inputs: fp32 device arrays of n
+ * channels (running statistics and the affine parameters); outputs: fp32 device arrays of n, which
+ * the FL search and fxpq_quantize turn into the Scale layer's codes.  eps >= 0. */
+FXPQ_API fxpq_status fxpq_bn_to_scale(const float* d_gamma, const float* d_beta, const float* d_mean,
+                                      const float* d_var, int64_t n, float eps, float* d_aleph1, float* d_aleph2,
+                                      void* stream);
+
 /* ---------------------------------------------------------------------------------------- */
 /* Network forward (Sec. IV-A.2: FxP-QLayers as vertices, C-Blocks as edges).                */
 /* A network is a list of ops over numbered tensor slots; slot 0 is the input image codes.   */
@@ -301,6 +319,9 @@ typedef struct {
     const void* d_w;         /* conv: fp16 code tensor KRSC [K, R, S, Cp_in]                 */
     const int32_t* d_bias;   /* conv: int32 bias codes [K] or NULL                           */
     int64_t w_l1;            /* conv: optional weight-code L1 bound (fxpq_conv_desc.w_l1)    */
+    fxpq_fmt fmt_scale, fmt_shift;  /* conv: Scale layer formats (fxpq_conv_desc)            */
+    const int32_t* d_scale;  /* conv: Scale layer aleph1 codes [K] or NULL                   */
+    const int32_t* d_shift;  /* conv: Scale layer aleph2 codes [K] or NULL                   */
 } fxpq_op_desc;
 
 typedef struct {

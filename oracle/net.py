@@ -14,12 +14,15 @@ Readings of the paper used here (each is listed with its reason in the design doc):
 * The sign strategy is Sec. IV-A.3's: S = 1 iff the smallest value is negative.
 * The AVG-POOL reciprocal 1/(patch size) is a 16-bit unsigned parameter whose FL is searched
   like any other parameter.
+* A BN layer after a conv is rewritten as a Scale layer (Sec. IV-A.1): aleph1 and aleph2 come from
+  bn_to_scale in fp32 and are then searched and quantized like weights and biases (aleph1 after
+  the weights, aleph2 after it); the C-Block applies them after the (absent) bias and before ReLU.
 """
 from __future__ import annotations
 
 import numpy as np
 
-from . import (avgpool_global, cblock, conv2d, eltwise_add, fl_search, maxpool, quantize,
+from . import (avgpool_global, bn_to_scale, cblock, conv2d, eltwise_add, fl_search, maxpool, quantize,
                requant, to_f32)
 
 FL_LO, FL_HI = -8, 23
@@ -48,12 +51,17 @@ def _layer_pass(layers, i, L, env, fmts, qparams, calibrating: bool, plan):
     if L["type"] == "conv":
         src = L.get("src") or prev
         x, fx = env[src]
-        wq, bq = qparams[name]
-        fw, fb = fmts[name]["w"], fmts[name]["b"]
+        wq, bq = qparams[name][:2]
+        fw, fb = fmts[name]["w"], fmts[name].get("b", (0, 0, 0))
         if x.ndim == 2:
             x = x.reshape(x.shape[0], 1, 1, -1)
         acc = conv2d(x, wq, L["stride"], L["pad"])
-        v, s = cblock(acc, fx[2] + fw[2], bq, fb[2], L["relu"])
+        if L.get("bn"):
+            sq, hq = qparams[name][2:]
+            v, s = cblock(acc, fx[2] + fw[2], bq, fb[2], L["relu"], scale=sq, fl_scale=fmts[name]["s"][2],
+                          shift=hq, fl_shift=fmts[name]["h"][2])
+        else:
+            v, s = cblock(acc, fx[2] + fw[2], bq, fb[2], L["relu"])
         if _is_last(layers, i):
             env[name] = (v.reshape(v.shape[0], -1), ("logits", None, s))
             return
@@ -80,8 +88,10 @@ def _layer_pass(layers, i, L, env, fmts, qparams, calibrating: bool, plan):
     env[name] = (requant(v, s, k, S, fl), fmts[name]["a"])
 
 
-def quantize_params(layers, weights, plan):
-    """Weights then bias of every conv/FC layer: FL search at the planned wordlength, then Q."""
+def quantize_params(layers, weights, plan, bn=None):
+    """Weights then bias of every conv/FC layer: FL search at the planned wordlength, then Q.  A conv
+    with a BN layer (bn[name] = (gamma, beta, mean, var)) has no bias; its Scale parameters aleph1
+    ("s") and aleph2 ("h") follow the weights.  qparams[name] = (W, B or None[, aleph1, aleph2])."""
     fmts, qparams = {}, {}
     for L in layers:
         nm = L["name"]
@@ -89,15 +99,26 @@ def quantize_params(layers, weights, plan):
         if L["type"] == "conv":
             w, b = weights[nm]
             fw = search_fmt(w, plan[nm]["w"])
-            fb = search_fmt(b, plan[nm]["b"])
-            fmts[nm]["w"], fmts[nm]["b"] = fw, fb
-            qparams[nm] = (quantize(w, *fw).reshape(w.shape), quantize(b, *fb))
+            fmts[nm]["w"] = fw
+            qw = quantize(w, *fw).reshape(w.shape)
+            if b is not None:
+                fb = search_fmt(b, plan[nm]["b"])
+                fmts[nm]["b"] = fb
+                qparams[nm] = (qw, quantize(b, *fb))
+            else:
+                qparams[nm] = (qw, None)
+            if L.get("bn"):
+                a1, a2 = bn_to_scale(*bn[nm])
+                fs = search_fmt(a1, plan[nm]["s"])
+                fh = search_fmt(a2, plan[nm]["h"])
+                fmts[nm]["s"], fmts[nm]["h"] = fs, fh
+                qparams[nm] = qparams[nm] + (quantize(a1, *fs), quantize(a2, *fh))
     return fmts, qparams
 
 
-def calibrate(layers, weights, calib_images_nchw, plan):
+def calibrate(layers, weights, calib_images_nchw, plan, bn=None):
     """Forward-optimizer-order calibration on a slice.  Returns (fmts, qparams)."""
-    fmts, qparams = quantize_params(layers, weights, plan)
+    fmts, qparams = quantize_params(layers, weights, plan, bn)
     fmts["input"] = search_fmt(calib_images_nchw, plan["input"])
     env = {"input": (images_to_codes(calib_images_nchw, fmts["input"]), fmts["input"])}
     for i, L in enumerate(layers):

@@ -41,13 +41,15 @@ class QuantizeItem(ctypes.Structure):
 class ConvDesc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("Cp", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("out_mode", I32),
-                ("fmt_x", Fmt), ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("w_l1", I64)]
+                ("fmt_x", Fmt), ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("w_l1", I64),
+                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
 
 
 class OpDesc(ctypes.Structure):
     _fields_ = [("op", I32), ("src0", I32), ("src1", I32), ("dst", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("last", I32), ("recip_code", I32),
-                ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("d_w", VP), ("d_bias", VP), ("w_l1", I64)]
+                ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("d_w", VP), ("d_bias", VP), ("w_l1", I64),
+                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
 
 
 class Net(ctypes.Structure):
@@ -75,6 +77,7 @@ _SIGS = {
     "fxpq_fl_search_workspace": (SZ, [I64]),
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),
     "fxpq_fl_search_noalloc": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP]),
+    "fxpq_bn_to_scale": (I32, [VP, VP, VP, VP, I64, ctypes.c_float, VP, VP, VP]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),
     "fxpq_conv_workspace": (SZ, [ctypes.POINTER(ConvDesc)]),
     "fxpq_conv_fwd": (I32, [ctypes.POINTER(ConvDesc), VP, VP, VP, VP, ctypes.POINTER(I32), VP, SZ, VP]),

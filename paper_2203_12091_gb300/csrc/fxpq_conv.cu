@@ -153,6 +153,31 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
             s = d.fmt_b.fl;
         }
     }
+    a.has_scale = d.d_scale != nullptr;
+    a.scale = d.d_scale;
+    a.shift = d.d_shift;
+    a.delta2 = 0;
+    if (a.has_scale) {
+        // v * aleph1 at scale s + fl_aleph1, then aleph2 aligned like the bias
+        if (!d.d_shift || !fmt_ok(d.fmt_scale, 32) || !fmt_ok(d.fmt_shift, 32)) return FXPQ_ERR_INVALID_ARG;
+        const double mb = ldexp(1.0, d.fmt_scale.bits - d.fmt_scale.is_signed);
+        const double hb = ldexp(1.0, d.fmt_shift.bits - d.fmt_shift.is_signed);
+        const double pbound = vbound * mb;
+        if (pbound >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+        s += d.fmt_scale.fl;
+        a.delta2 = s - d.fmt_shift.fl;
+        if (a.delta2 >= 0) {
+            if (a.delta2 > 40 || hb * ldexp(1.0, a.delta2) + pbound >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+            vbound = pbound + hb * ldexp(1.0, a.delta2);
+        } else {
+            if (-a.delta2 > 40 || pbound * ldexp(1.0, -a.delta2) + hb >= ldexp(1.0, 62)) return FXPQ_ERR_RANGE;
+            vbound = pbound * ldexp(1.0, -a.delta2) + hb;
+            s = d.fmt_shift.fl;
+        }
+    } else if (d.d_shift) {
+        return FXPQ_ERR_INVALID_ARG;
+    }
+    (void)vbound;
     a.s_out = s;
     a.has_bias = bias != nullptr;
     a.v32 = 0;
@@ -171,7 +196,7 @@ fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, con
         a.bsh = a.delta;
         a.sh32 = s_acc - d.fmt_y.fl;
         const double nbound = bound + (a.delta >= 0 ? bb * ldexp(1.0, a.delta) : bb * ldexp(1.0, a.delta) + 1.0);
-        a.v32 = (a.sh32 >= 1 && a.sh32 <= 30 && nbound + ldexp(1.0, a.sh32 - 1) < two31 && a.delta >= -30 &&
+        a.v32 = (!a.has_scale && a.sh32 >= 1 && a.sh32 <= 30 && nbound + ldexp(1.0, a.sh32 - 1) < two31 && a.delta >= -30 &&
                  a.delta <= 30)
                     ? 1
                     : 0;
@@ -233,7 +258,7 @@ extern "C" fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_
                                  const int32_t* d_bias, fxpq_fmt fmt_b, int32_t M, int32_t N, int32_t Kdim,
                                  int32_t relu, int32_t out_mode, fxpq_fmt fmt_y, void* d_y, int32_t* h_out_scale,
                                  void* d_ws, size_t ws_bytes, void* stream) {
-    fxpq_conv_desc d;
+    fxpq_conv_desc d = {};
     d.N = M;
     d.H = d.W = 1;
     d.C = Kdim;

@@ -23,10 +23,17 @@ struct ConvArgs {
     int v32;           // 1: qlayer_code32 applies (the host checked its 32-bit bounds)
     int bsh;           // bias shift of the 32-bit path (= delta)
     int sh32;          // right shift of the 32-bit path, relative to the accumulator's scale
+    const int32_t* scale;  // Scale layer aleph1 codes [K] (has_scale)
+    const int32_t* shift;  // Scale layer aleph2 codes [K]
+    int has_scale;
+    int delta2;        // aleph2 alignment: (scale after the bias) + fl_aleph1 - fl_aleph2
 };
 
-// Bias alignment (B << delta, or the accumulator shifted left when delta < 0) and ReLU: the C-Block
-// output before its FxP-QLayer, in units of 2^-s_out.
+// Bias alignment (B << delta, or the accumulator shifted left when delta < 0), the Scale layer
+// (v * aleph1, then aleph2 aligned the same way) and ReLU: the C-Block output before its FxP-QLayer,
+// in units of 2^-s_out.  SC = false compiles the Scale layer out (for kernels the host launches only
+// for layers without one).
+template <bool SC = true>
 __device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long long v, int32_t bias) {
     if (a.has_bias) {
         const long long b = bias;
@@ -34,6 +41,14 @@ __device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long
             v += b << a.delta;
         else
             v = (v << (-a.delta)) + b;
+    }
+    if (SC && a.has_scale) {
+        v *= (long long)__ldg(a.scale + k);
+        const long long h = __ldg(a.shift + k);
+        if (a.delta2 >= 0)
+            v += h << a.delta2;
+        else
+            v = (v << (-a.delta2)) + h;
     }
     if (a.relu && v < 0) v = 0;
     return v;

@@ -1,1032 +1,12 @@
-// fxpq_conv_tc.cu -- the C-Block contraction (Sec. IV-B) on the 5th-generation tensor cores.
-//
-// Implicit GEMM: rows = output pixels (N*P*Q), columns = output channels K, reduction over the
-// flattened (r, s, c) taps of one code plane.  Operands are fp16 values that are exact integer
-// codes (|code| <= 255 per limb), multiplied by tcgen05.mma .kind::f16 into fp32 TMEM
-// accumulators.  fp32 accumulation is exact while every partial sum stays below 2^24, so the host
-// splits the reduction into groups ("chunks") whose worst-case magnitude max|a| * max|w| * K_chunk
-// is below 2^24; after each group the epilogue warps drain the accumulator, convert it to an
-// integer (exact) and add it, shifted by the limb weight (0, 8 or 16 bits), into integer running
-// sums.  The same grouping carries the two-limb split of 9..16-bit codes
-// (v = 256 * v_hi + v_lo): one pass per (A limb, W limb) pair.
-//
-// CTA (one per SM, persistent over tiles): 9 warps.
-//   warps 0-3  producers, into 128-byte swizzled K-major shared-memory stages.  The B tile
-//              (BN channels x 64 taps) always comes by TMA.  The A tile takes one of two forms:
-//              row tiles (128 consecutive output pixels): cp.async gather by 128 threads, with
-//              zero fill for padding and ragged edges;
-//              patch tiles (stride 1, Cp % 64 == 0): a TH x TW patch of output pixels of one
-//              image, whose input window for one tap and 64 channels is a single 5-D TMA box
-//              (the hardware zero-fills the padding); one thread issues both copies.
-//   warp  4-7  epilogue: drain TMEM (tcgen05.ld), integer running sums, final bias / ReLU /
-//              FxP-QLayer (shared with the CUDA-core kernel).
-//   warp  8    TMEM allocation and the single MMA-issuing thread.
-// Every wait is bounded: on expiry the kernel latches FXPQ_ERR_TIMEOUT, stops issuing work,
-// drains its own copies and MMAs, frees TMEM and returns.
-#include <cuda.h>  // CUtensorMap and its enums (the encoder is fetched through the runtime)
-#include <climits>
-#include <cstdlib>
-#include <cstring>
-#include <mutex>
-
-#include "fxpq_common.cuh"
-#include "fxpq_conv.cuh"
+// fxpq_conv_tc.cu -- host side of the tensor-core C-Block (planning, tensor maps, launch) and the
+// kernels without a Scale layer; the kernel itself is in fxpq_conv_tc.cuh.
+#include "fxpq_conv_tc.cuh"
 
 namespace fxpq {
 
+using namespace tc;
+
 namespace {
-
-constexpr int TC_BM = 128;
-constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
-// Pipeline depth: 6 stages of 32 KB (BN <= 128) or 3 of 48 KB (BN = 256, whose 64 KB output staging
-// leaves no room for a fourth).
-__host__ __device__ constexpr int tc_stages(int BN) { return BN == 256 ? 3 : 6; }
-// Row-tile producers arrive on a stage this many k-blocks after issuing its copies (cp.async groups
-// in flight).  It must stay below the stage count: a producer waiting for a stage to be consumed
-// must already have arrived on it.
-__host__ __device__ constexpr int tc_lag(int BN) { return tc_stages(BN) - 1 < 3 ? tc_stages(BN) - 1 : 3; }
-// Warps: 4 producers, epilogue warps (four per 32-column chunk group: one per TMEM lane quadrant;
-// BN / 8 of them up to 16, each then draining BN / 128 chunks), one MMA / TMEM-allocation warp.
-__host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8 < 16 ? BN / 8 : 16; }
-__host__ __device__ constexpr int tc_threads(int BN) { return (5 + tc_epi_warps(BN)) * 32; }
-constexpr int TC_MAX_GROUPS = 64;
-constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
-
-struct TcGroup {
-    int kb0, kb1;          // k-block range within a plane
-    int a_plane, w_plane;  // limb planes (0 = hi or the only plane, 1 = lo)
-    int shift;             // weight of this pass: 0, 8 or 16 bits
-};
-
-struct TcParams {
-    CUtensorMap tmap_w;  // weights as [planes][K][R*S*Cp] fp16, box {64, BN, 1}, 128-byte swizzle
-    CUtensorMap tmap_y;  // output codes: [M][K] box {64, 128} (linear tiles) or [N][P][Q][K] box {64, TW, TH, 1}
-    CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}
-    int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
-    int nbuf;            // fp32 accumulator buffers in TMEM: 2, or 1 when BN = 256 needs running sums
-    int patch;           // a tile is a TH x TW patch of one image and the A tile comes by TMA:
-                         // 1: Cp % 64 == 0 (one 64-channel box per k-block, 128-byte swizzle);
-                         // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle);
-                         // 3: Cp == 8, window mode (one input window per tile and limb plane, taps as
-                         //    shifted descriptors, weights resident in shared memory)
-    int nacc;            // fp32 accumulators per TMEM buffer (window mode: one per limb pair)
-    int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
-    int win_bytes;       // window mode: bytes of one window (128-byte aligned)
-    int TH, TW;          // patch shape (TH * TW = 128)
-    int tiles_p, tiles_q;  // patches per image along P and Q
-    ConvArgs a;
-    int RSC;       // R * S * Cp: reduction length of one plane
-    int tiles_m, tiles_n, n_tiles;
-    int n_groups;
-    int cp64;      // Cp % 64 == 0: a k-block never straddles a tap
-    int* status;
-    TcGroup g[TC_MAX_GROUPS];
-};
-
-// ------------------------------------------------------------------ PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-// 2-D tiled TMA store from shared memory (bulk-group completion).
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int y, uint32_t src) {
-    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(x), "r"(y), "r"(src)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
-__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, int x, int y, int z, int w, uint32_t src) {
-    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(x), "r"(y), "r"(z), "r"(w), "r"(src)
-                 : "memory");
-}
-
-// 5-D tiled TMA load completing on mbarrier `bar` (coordinates innermost first; out-of-range
-// positions, e.g. the convolution's padding, read as zero).
-__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
-                                            int c4, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
-        "%5, %6}], [%7];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar)
-        : "memory");
-}
-
-// Output row (linear index into N*P*Q, or -1 when outside the map) of tile row i.
-__device__ __forceinline__ long long tile_row(const TcParams& P, int tm, int i) {
-    if (!P.patch) {
-        const long long m = (long long)tm * 128 + i;
-        return m < P.a.M ? m : -1;
-    }
-    if (i >= P.TH * P.TW) return -1;
-    const int per_img = P.tiles_p * P.tiles_q;
-    const int n = tm / per_img, r = tm - n * per_img;
-    const int p = (r / P.tiles_q) * P.TH + i / P.TW, q = (r % P.tiles_q) * P.TW + i % P.TW;
-    if (p >= P.a.P || q >= P.a.Q) return -1;
-    return ((long long)n * P.a.P + p) * P.a.Q + q;
-}
-
-// 3-D tiled TMA load (coordinates innermost first) completing on mbarrier `bar`.
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
-        "[%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
-        : "memory");
-}
-
-// Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
-// timeout status, sets the CTA abort flag) if it gave up or another role already aborted.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort) return false;
-        if (clock64() - t0 > TC_WAIT_CYCLES) {
-            *abort = 1;
-            latch_status(status, FXPQ_ERR_TIMEOUT);
-            return false;
-        }
-    }
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
-// Shared-memory matrix descriptor, K-major without swizzle: core matrices of 8 rows x 16 bytes;
-// lbo = bytes between core matrices adjacent in K, sbo = bytes between 8-row groups.
-__device__ __forceinline__ uint64_t make_sdesc_noswz(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
-    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-    d |= (uint64_t)1u << 46;  // descriptor version; layout type 0 = no swizzle
-    return d;
-}
-
-__device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr) {
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);          // start address
-    d |= (uint64_t)1u << 16;                          // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(1024u >> 4) << 32;                // stride byte offset: 8 rows x 128 B
-    d |= (uint64_t)1u << 46;                          // descriptor version
-    d |= (uint64_t)2u << 61;                          // SWIZZLE_128B
-    return d;
-}
-
-// Instruction descriptor, kind::f16: fp16 A and B (K-major), fp32 accumulator, M x N.
-__host__ __device__ constexpr uint32_t make_idesc(int M, int N) {
-    return (1u << 4)                        // D format F32
-           | (0u << 7) | (0u << 10)         // A, B format F16
-           | ((uint32_t)(N >> 3) << 17)     // N / 8
-           | ((uint32_t)(M >> 4) << 24);    // M / 16
-}
-
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                       uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
-}
-
-// Loads / stores without their completion wait, so that several TMEM accesses share one round trip.
-// After tmem_wait_ld(), reg_fence() on each loaded array orders every use of its registers after the
-// wait (the empty asm redefines them).
-__device__ __forceinline__ void tmem_ld16_nw(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void reg_fence(uint32_t (&r)[N]) {
-#pragma unroll
-    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
-}
-__device__ __forceinline__ void tmem_st16_nw(uint32_t taddr, const uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
-        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
-        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
-        : "memory");
-}
-// Final epilogue of 32 consecutive output channels k0.. of row m (generic outputs: two-plane codes,
-// int64 accumulators, fp32 calibration images): bias alignment, ReLU, FxP-QLayer.
-template <typename ACC>
-__device__ __forceinline__ void epilogue_block32(const ConvArgs& a, long long m, int k0, const ACC (&acc)[32]) {
-    if (a.out_mode == FXPQ_OUT_CODES) {
-        __half* y = static_cast<__half*>(a.y);
-        const long long base = m * a.K + k0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int k = k0 + j;
-            if (k < a.K) {
-                const int32_t b = a.has_bias ? __ldg(a.bias + k) : 0;
-                code_put(y, base + j, a.py, a.M * a.K, qlayer_code(a, cblock_value(a, k, (long long)acc[j], b)));
-            }
-        }
-    } else if (a.out_mode == FXPQ_OUT_ACC64) {
-        long long* y = static_cast<long long*>(a.y) + m * a.K + k0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int k = k0 + j;
-            if (k < a.K) y[j] = cblock_value(a, k, (long long)acc[j], a.has_bias ? __ldg(a.bias + k) : 0);
-        }
-    } else {
-        float* y = static_cast<float*>(a.y) + m * a.K + k0;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int k = k0 + j;
-            if (k < a.K)
-                y[j] = __ll2float_rn(cblock_value(a, k, (long long)acc[j], a.has_bias ? __ldg(a.bias + k) : 0)) *
-                       a.f32_scale;
-        }
-    }
-}
-
-// Uniform constants of the 32-bit FxP-QLayer epilogue (the same arithmetic as qlayer_code32, with
-// the bias alignment split into a left and a right shift so that it has no branches).
-struct Epi32 {
-    int bsl, bsr, fmask;  // bias term (b << bsl) >> bsr; fraction bits b & fmask (bias finer than acc)
-    int sh, hm1;          // requantizing right shift and 2^(sh-1) - 1
-    int floor;            // 0 with ReLU, INT_MIN without
-    int lo, hi;
-    int has_bias;
-};
-
-__device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
-    Epi32 e;
-    e.bsl = a.bsh > 0 ? a.bsh : 0;
-    e.bsr = a.bsh < 0 ? -a.bsh : 0;
-    e.fmask = (1 << e.bsr) - 1;
-    e.sh = a.sh32;
-    e.hm1 = (1 << (a.sh32 - 1)) - 1;
-    e.floor = a.relu ? 0 : INT_MIN;
-    e.lo = (int)a.lo;
-    e.hi = (int)a.hi;
-    e.has_bias = a.has_bias;
-    return e;
-}
-
-// One code: N = acc + aligned bias; ReLU; N / 2^sh rounded half to even, then clipped.  With
-// q = floor(N / 2^sh) and x = (q & 1) | phi, floor((N + 2^(sh-1) - 1 + x) / 2^sh) is q + 1 exactly
-// when the remainder is above one half, or equal to it with q odd or phi set (phi: the bias had
-// nonzero bits below the accumulator's scale, so the true value lies above the tie).  After a ReLU
-// clamp N = 0 and the sum stays below 2^sh whatever phi is.  The host keeps |N| + 2^(sh-1) < 2^31.
-__device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, int phi) {
-    const int N = max(acc + bterm, e.floor);
-    const int x = ((N >> e.sh) & 1) | phi;
-    return min(max((N + e.hm1 + x) >> e.sh, e.lo), e.hi);
-}
-
-// The same FxP-QLayer on 64-bit values (wide sums, two-limb layers), valid for 1 <= sh <= 62: the
-// bias alignment is v = (acc << dr) + (B << dl) (one of dl, dr is zero), and the code is
-// round_half_even(v / 2^sh) = floor((v + 2^(sh-1) - 1 + ((v >> sh) & 1)) / 2^sh), clipped.  The host
-// keeps |v| < 2^62, so the rounding sum cannot overflow.
-struct Epi64 {
-    int dl, dr, sh;
-    long long hm1, floor;
-    int lo, hi, has_bias, ok;  // ok: 1 <= sh <= 62 (otherwise the generic path runs)
-};
-
-__device__ __forceinline__ Epi64 make_epi64(const ConvArgs& a) {
-    Epi64 e;
-    e.dl = a.delta > 0 ? a.delta : 0;
-    e.dr = a.delta < 0 ? -a.delta : 0;
-    e.sh = a.sh;
-    e.ok = a.sh >= 1 && a.sh <= 62;
-    e.hm1 = e.ok ? (1LL << (a.sh - 1)) - 1 : 0;
-    e.floor = a.relu ? 0LL : LLONG_MIN;
-    e.lo = (int)a.lo;
-    e.hi = (int)a.hi;
-    e.has_bias = a.has_bias;
-    return e;
-}
-
-__device__ __forceinline__ int epi64_code(const Epi64& e, long long acc, int32_t b) {
-    long long v = (acc << e.dr) + ((long long)b << e.dl);
-    v = max(v, e.floor);
-    const long long c = (v + e.hm1 + ((v >> e.sh) & 1)) >> e.sh;
-    return (int)min(max(c, (long long)e.lo), (long long)e.hi);
-}
-
-// Two codes in [-512, 511] as a packed fp16 pair: 1536 + c has the bit pattern 0x6600 + c (the
-// binade [1024, 2048) has unit spacing), and one packed subtraction of 1536 leaves c exactly.
-__device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
-    // 0x6600 + c0 >= 0x6400 never borrows from the high half
-    const uint32_t bits = (uint32_t)c1 * 65536u + (uint32_t)c0 + 0x66006600u;
-    const __half2 h = __hsub2(*reinterpret_cast<const __half2*>(&bits), __halves2half2(__ushort_as_half(0x6600),
-                                                                                        __ushort_as_half(0x6600)));
-    return *reinterpret_cast<const uint32_t*>(&h);
-}
-
-// ------------------------------------------------------------------ kernel
-template <int BN, typename ACC>
-__global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
-    constexpr int TC_STAGES = tc_stages(BN);
-    constexpr int TC_LAG = tc_lag(BN);
-    static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
-    constexpr int EPI_WARPS = tc_epi_warps(BN);
-    constexpr int EPI_THREADS = 32 * EPI_WARPS;
-    constexpr int MMA_WARP = 4 + EPI_WARPS;
-    constexpr int CPW = (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
-    constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
-    constexpr int B_BYTES = BN * TC_BK * 2;
-    constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
-    // fp32 accumulator buffers + integer running sums, rounded up to a power of two (BN = 256: two
-    // buffers without running sums, or one buffer with them)
-    // (the int64 instance also serves window mode: two buffers of up to four limb-pair accumulators)
-    constexpr uint32_t USED_COLS = (BN == 256 || sizeof(ACC) == 8) ? 512u : 2 * BN + BN * (uint32_t)(sizeof(ACC) / 4);
-    constexpr uint32_t TMEM_COLS = USED_COLS <= 256 ? 256u : 512u;
-    extern __shared__ unsigned char smem_raw[];
-    unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    unsigned char* sA = base;
-    unsigned char* sB = base + TC_STAGES * A_BYTES;
-    unsigned char* sO = sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of [128 rows][64 codes]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2);
-    // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
-    volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
-    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + TC_STAGES);
-    const uint32_t accfull0 = smem_u32(bars + 2 * TC_STAGES), accempty0 = smem_u32(bars + 2 * TC_STAGES + 2);
-    const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
-    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue thread
-    const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
-    const uint32_t wbar = smem_u32(bars + 2 * TC_STAGES + 9);      // window mode: resident weights loaded
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const ConvArgs& a = P.a;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < TC_STAGES; ++s) {
-            // patch tiles: one expect_tx arrival for both TMAs; row tiles: 128 producer arrivals +
-            // the weight TMA's expect_tx
-            mbar_init(full0 + 8 * s, P.patch ? 1 : 128 + 1);
-            mbar_init(empty0 + 8 * s, 1);
-        }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(accfull0 + 8 * b, 1);
-            mbar_init(accempty0 + 8 * b, EPI_THREADS);
-        }
-        mbar_init(done_bar, 1);
-        mbar_init(stg_full, EPI_THREADS);
-        mbar_init(stg_free, 1);
-        mbar_init(wbar, 1);
-        *abort = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (warp == MMA_WARP) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(TMEM_COLS));
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
-
-    if (warp < 4 && P.patch == 3) {
-        // ============================================================ producer, window mode
-        // Stride 1, Cp == 8: the weights (per limb plane, kernel row r and tap pair sp, the box
-        // {8 ch, BN out ch, 2 taps}) are loaded once into the B region; per tile, one box per x limb
-        // plane holds the input window of TH + R - 1 rows by TW + S2 - 1 pixels (padding zero filled).
-        if (threadIdx.x == 0) {
-            const int np = P.S2 / 2;
-            const uint32_t wbox = (uint32_t)(BN * 32);
-            mbar_arrive_expect_tx(wbar, (uint32_t)(a.pw * a.R * np) * wbox);
-            for (int iw = 0; iw < a.pw; ++iw)
-                for (int r = 0; r < a.R; ++r)
-                    for (int sp = 0; sp < np; ++sp)
-                        tma_load_5d(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox, &P.tmap_w, 0, 0, 2 * sp,
-                                    r, iw, wbar);
-            const uint32_t win_tx = (uint32_t)(P.WW * P.WH * 16);
-            const int per_img = P.tiles_p * P.tiles_q;
-            uint32_t it = 0, stage = 0, phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-                const int tm = t / P.tiles_n;
-                const int n_img = tm / per_img, r = tm - n_img * per_img;
-                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
-                if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t fb = full0 + 8 * stage;
-                mbar_arrive_expect_tx(fb, (uint32_t)a.px * win_tx);
-                for (int ia = 0; ia < a.px; ++ia)
-                    tma_load_5d(smem_u32(sA + stage * A_BYTES) + (uint32_t)(ia * P.win_bytes), &P.tmap_x, 0, wq0, hp0,
-                                n_img, ia, fb);
-                ++it;
-                if (++stage == TC_STAGES) {
-                    stage = 0;
-                    phase ^= 1;
-                }
-            }
-            // bounded wait until the copies of the last stages and the weights have landed
-            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
-            for (uint32_t j = from; j < it; ++j) {
-                const long long t0 = clock64();
-                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
-                       clock64() - t0 < TC_WAIT_CYCLES) {
-                }
-            }
-            const long long t0 = clock64();
-            while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
-            }
-        }
-    } else if (warp < 4 && P.patch) {
-        // ============================================================ producer, patch tiles
-        // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
-        // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
-        // Cp == 8: a k-block is 8 taps of 8 channels; tap tl's box {8, TW, TH} lands at byte
-        // 2048 tl of the stage (a 16-byte K column of the no-swizzle layout), and taps past R*S
-        // are boxes wholly outside the tensor (zero filled).
-        if (threadIdx.x == 0) {
-            const bool narrow = P.patch == 2;
-            const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
-            const int per_img = P.tiles_p * P.tiles_q;
-            uint32_t it = 0, stage = 0, phase = 0;
-            bool ok = true;
-            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-                const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-                const int n_img = tm / per_img, r = tm - n_img * per_img;
-                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
-                for (int gi = 0; gi < P.n_groups && ok; ++gi) {
-                    const TcGroup g = P.g[gi];
-                    for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
-                            ok = false;
-                            break;
-                        }
-                        const int f = kb * TC_BK;
-                        const int tp = f / a.Cp, cc = f - tp * a.Cp;
-                        const int rr = tp / a.S, ss = tp - rr * a.S;
-                        const uint32_t fb = full0 + 8 * stage;
-                        mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
-                        if (narrow) {
-                            for (int tl = 0; tl < 8; ++tl) {
-                                const int tap = kb * 8 + tl;
-                                const bool in = tap < a.R * a.S;
-                                const int r8 = in ? tap / a.S : 0, s8 = in ? tap - (tap / a.S) * a.S : 0;
-                                tma_load_5d(smem_u32(sA + stage * A_BYTES + tl * 2048), &P.tmap_x, in ? 0 : 8,
-                                            wq0 + s8, hp0 + r8, n_img, g.a_plane, fb);
-                            }
-                        } else {
-                            tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
-                                        g.a_plane, fb);
-                        }
-                        tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, f, tn * BN, g.w_plane, fb);
-                        ++it;
-                        if (++stage == TC_STAGES) {
-                            stage = 0;
-                            phase ^= 1;
-                        }
-                    }
-                }
-            }
-            // bounded wait until the copies of the last stages have landed
-            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
-            for (uint32_t j = from; j < it; ++j) {
-                const long long t0 = clock64();
-                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
-                       clock64() - t0 < TC_WAIT_CYCLES) {
-                }
-            }
-        }
-    } else if (warp < 4) {
-        // ============================================================ producers, row tiles
-        // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
-        // threads cover one 128-byte row, so every warp instruction reads four whole rows.
-        const int c = threadIdx.x & 7;
-        const int r0 = threadIdx.x >> 3;  // 0..15
-        constexpr int AR = TC_BM / 16;    // A rows per thread
-        const __half* xb = a.x;
-        uint32_t it = 0;
-        bool ok = true;
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-            const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            long long rowoff[AR];  // element offset of the (r, s) = (0, 0) tap of each row (may be negative)
-            int p0[AR], q0[AR];
-#pragma unroll
-            for (int i = 0; i < AR; ++i) {
-                const long long m = (long long)tm * TC_BM + r0 + 16 * i;
-                const long long mm = m < a.M ? m : 0;
-                const int n_img = (int)(mm / ((long long)a.P * a.Q));
-                const int pq = (int)(mm - (long long)n_img * a.P * a.Q);
-                p0[i] = (pq / a.Q) * a.stride - a.pad;
-                q0[i] = (pq % a.Q) * a.stride - a.pad;
-                if (m >= a.M) p0[i] = -(1 << 20);  // rows past the end read zeros
-                rowoff[i] = (((long long)n_img * a.H + p0[i]) * a.W + q0[i]) * a.Cp;
-            }
-            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
-                const TcGroup g = P.g[gi];
-                const __half* xp = xb + (long long)g.a_plane * a.x_ps;
-                for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                    const int stage = it % TC_STAGES;
-                    const uint32_t ph = (it / TC_STAGES) & 1;
-                    if (!wait_bounded(empty0 + 8 * stage, ph ^ 1, abort, P.status)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t dA = smem_u32(sA + stage * A_BYTES);
-                    if (threadIdx.x == 0) {  // the weight tile: one TMA, zero-filled past K and R*S*Cp
-                        mbar_arrive_expect_tx(full0 + 8 * stage, (uint32_t)B_BYTES);
-                        tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, kb * TC_BK, tn * BN, g.w_plane,
-                                    full0 + 8 * stage);
-                    }
-                    const int f = kb * TC_BK + 8 * c;  // this thread's chunk of the flattened (r, s, c) index
-                    const bool fvalid = f < P.RSC;
-                    const int tp = f / a.Cp;
-                    const int cc = f - tp * a.Cp;
-                    const int rr = tp / a.S, ss = tp - rr * a.S;
-                    const long long toff = ((long long)rr * a.W + ss) * a.Cp + cc;
-#pragma unroll
-                    for (int i = 0; i < AR; ++i) {
-                        const int row = r0 + 16 * i;
-                        const int h = p0[i] + rr, w = q0[i] + ss;
-                        const bool v = fvalid && (unsigned)h < (unsigned)a.H && (unsigned)w < (unsigned)a.W;
-                        const __half* src = v ? xp + rowoff[i] + toff : xb;
-                        cp_async16(dA + row * 128 + (uint32_t)((c ^ (row & 7)) << 4), src, v ? 16u : 0u);
-                    }
-                    cp_async_commit();
-                    if (it >= TC_LAG) {
-                        cp_async_wait<TC_LAG>();
-                        fence_proxy_async();
-                        mbar_arrive(full0 + 8 * ((it - TC_LAG) % TC_STAGES));
-                    }
-                    ++it;
-                }
-            }
-        }
-        cp_async_wait<0>();
-        fence_proxy_async();
-        const uint32_t first = it >= TC_LAG ? it - TC_LAG : 0;
-        for (uint32_t j = first; j < it; ++j) mbar_arrive(full0 + 8 * (j % TC_STAGES));
-        if (threadIdx.x == 0) {
-            // Every weight TMA this thread issued has landed once its stage's phase completes (the MMA
-            // thread already waited for them unless the kernel aborted): bounded wait on the last ones.
-            const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
-            for (uint32_t j = from; j < it; ++j) {
-                const long long t0 = clock64();
-                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
-                       clock64() - t0 < TC_WAIT_CYCLES) {
-                }
-            }
-        }
-    } else if (warp < MMA_WARP) {
-        // ============================================================ epilogue
-        // Warp w drains TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the quadrant a warp may access) and
-        // the 32-column chunks cw * CPW .. cw * CPW + CPW - 1, cw = (w - 4) / 4, of every accumulator.
-        const int quad = warp & 3;
-        const int cw = (warp - 4) >> 2;
-        const int row = quad * 32 + lane;
-        const bool leader = threadIdx.x == 128;  // waits for and issues the tile's TMA stores
-        const int nbuf = P.nbuf;
-        uint32_t gcount = 0;
-        bool ok = true;
-        // Integer running sums of a tile live in TMEM after the accumulator buffers: columns
-        // [nbuf BN, nbuf BN + BN * words), words = 1 (int32) or 2 (int64 as lo / hi column blocks).
-        const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
-        const uint32_t run_base = (uint32_t)(nbuf * BN);
-        uint32_t u = 0;  // tiles written through the staging buffer so far
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-            const int tm = t / P.tiles_n, tn = t % P.tiles_n;
-            const long long m = tile_row(P, tm, row);  // -1: row outside the output
-            for (int gi = 0; gi < P.n_groups; ++gi) {
-                const int shift = P.g[gi].shift;
-                const bool first = gi == 0, last = gi == P.n_groups - 1;
-                const uint32_t buf = nbuf == 2 ? (gcount & 1) : 0;
-                const uint32_t par = nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
-                if (!wait_bounded(accfull0 + 8 * buf, par, abort, P.status)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                if (last && P.fast_store && u > 0) {
-                    // the previous tile's TMA store must have read the staging buffer
-                    if (leader) {
-                        bulk_wait_read0();
-                        mbar_arrive(stg_free);
-                    }
-                    if (!wait_bounded(stg_free, (u - 1) & 1, abort, P.status)) {
-                        ok = false;
-                        break;
-                    }
-                }
-#pragma unroll 1
-                for (int c = 0; c < CPW; ++c) {
-                    const int cb = cw * CPW + c;
-                    const int k0 = tn * BN + cb * 32;
-                    const uint32_t run_col = run_base + cb * 32;
-                    if (sizeof(ACC) == 8 && P.patch == 3 && P.nacc == 4 && P.fast_store && a.sh >= 1 && a.sh <= 62) {
-                        // window mode, two-limb x and w, one-plane codes out: each 16-column half goes
-                        // from the four limb accumulators to packed codes before the next is loaded
-                        // (keeps the live 64-bit values to 16)
-                        const Epi64 e64 = make_epi64(a);
-                        const int k0 = tn * BN + cb * 32;
-                        const uint32_t abase = lane_base + buf * (uint32_t)(P.nacc * BN) + cb * 32;
-                        uint32_t w[16];
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf) {
-                            uint32_t fhh[16], fhl[16], flh[16], fll[16];
-                            tmem_ld16_nw(abase + 16 * hf, fhh);
-                            tmem_ld16_nw(abase + (uint32_t)BN + 16 * hf, fhl);
-                            tmem_ld16_nw(abase + (uint32_t)(2 * BN) + 16 * hf, flh);
-                            tmem_ld16_nw(abase + (uint32_t)(3 * BN) + 16 * hf, fll);
-                            tmem_wait_ld();
-                            reg_fence(fhh);
-                            reg_fence(fhl);
-                            reg_fence(flh);
-                            reg_fence(fll);
-                            if (hf == 1 && c == CPW - 1) {
-                                tc_fence_before();
-                                mbar_arrive(accempty0 + 8 * buf);
-                            }
-#pragma unroll
-                            for (int j = 0; j < 8; ++j) {
-                                int c2[2];
-#pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    const int jj = 2 * j + h;
-                                    const int k = k0 + 16 * hf + jj;
-                                    const long long v = ((long long)__float2int_rn(__uint_as_float(fhh[jj])) << 16) +
-                                                        ((long long)(__float2int_rn(__uint_as_float(fhl[jj])) +
-                                                                     __float2int_rn(__uint_as_float(flh[jj])))
-                                                         << 8) +
-                                                        (long long)__float2int_rn(__uint_as_float(fll[jj]));
-                                    const int32_t b = (e64.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                    c2[h] = epi64_code(e64, v, b);
-                                }
-                                w[8 * hf + j] = pack_codes_f16(c2[0], c2[1]);
-                            }
-                        }
-                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int chunk = (cb & 1) * 4 + q;
-                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
-                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-                        }
-                        continue;
-                    }
-                    // One TMEM round trip per load batch: the fp32 group sums and, after the first group,
-                    // the integer running sums are loaded together; the running-sum stores share one
-                    // completion wait.
-                    ACC acc[32];
-                    if (sizeof(ACC) == 8 && P.patch == 3) {
-                        // window mode: one accumulator per limb pair (ia, iw), combined with its weight
-                        // 2^(8 ((px-1-ia) + (pw-1-iw))); each is an exact integer below 2^24
-                        const uint32_t abase = lane_base + buf * (uint32_t)(P.nacc * BN) + cb * 32;
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf) {
-                            if (P.nacc == 4) {
-                                // two-limb x and w: the four accumulators share one load round trip;
-                                // v = 2^16 S_hh + 2^8 (S_hl + S_lh) + S_ll, the middle pair summed in 32 bits
-                                uint32_t fhh[16], fhl[16], flh[16], fll[16];
-                                tmem_ld16_nw(abase + 16 * hf, fhh);
-                                tmem_ld16_nw(abase + (uint32_t)BN + 16 * hf, fhl);
-                                tmem_ld16_nw(abase + (uint32_t)(2 * BN) + 16 * hf, flh);
-                                tmem_ld16_nw(abase + (uint32_t)(3 * BN) + 16 * hf, fll);
-                                tmem_wait_ld();
-                                reg_fence(fhh);
-                                reg_fence(fhl);
-                                reg_fence(flh);
-                                reg_fence(fll);
-#pragma unroll
-                                for (int j = 0; j < 16; ++j) {
-                                    const int hh = __float2int_rn(__uint_as_float(fhh[j]));
-                                    const int mid = __float2int_rn(__uint_as_float(fhl[j])) +
-                                                    __float2int_rn(__uint_as_float(flh[j]));
-                                    const int ll = __float2int_rn(__uint_as_float(fll[j]));
-                                    acc[16 * hf + j] = ((ACC)hh << 16) + ((ACC)mid << 8) + (ACC)ll;
-                                }
-                            } else {
-#pragma unroll
-                                for (int j = 0; j < 16; ++j) acc[16 * hf + j] = 0;
-                                for (int ia = 0; ia < a.px; ++ia)
-                                    for (int iw = 0; iw < a.pw; ++iw) {
-                                        uint32_t f16[16];
-                                        tmem_ld16_nw(abase + (uint32_t)((ia * a.pw + iw) * BN) + 16 * hf, f16);
-                                        tmem_wait_ld();
-                                        reg_fence(f16);
-                                        const int sh = 8 * ((a.px - 1 - ia) + (a.pw - 1 - iw));
-#pragma unroll
-                                        for (int j = 0; j < 16; ++j)
-                                            acc[16 * hf + j] += ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << sh;
-                                    }
-                            }
-                        }
-                    } else if (sizeof(ACC) == 8) {
-                        // int64 running sums in 16-column halves (lo and hi words in separate column blocks)
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf) {
-                            uint32_t f16[16], lo[16], hi[16];
-                            tmem_ld16_nw(lane_base + buf * BN + cb * 32 + 16 * hf, f16);
-                            if (!first) {
-                                tmem_ld16_nw(lane_base + run_col + 16 * hf, lo);
-                                tmem_ld16_nw(lane_base + run_col + BN + 16 * hf, hi);
-                            }
-                            tmem_wait_ld();
-                            reg_fence(f16);
-                            if (!first) {
-                                reg_fence(lo);
-                                reg_fence(hi);
-                            }
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                ACC v = ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << shift;
-                                if (!first) v += (ACC)(((unsigned long long)hi[j] << 32) | lo[j]);
-                                acc[16 * hf + j] = v;
-                            }
-                            if (!last) {
-#pragma unroll
-                                for (int j = 0; j < 16; ++j) {
-                                    lo[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
-                                    hi[j] = (uint32_t)((unsigned long long)acc[16 * hf + j] >> 32);
-                                }
-                                tmem_st16_nw(lane_base + run_col + 16 * hf, lo);
-                                tmem_st16_nw(lane_base + run_col + BN + 16 * hf, hi);
-                            }
-                        }
-                        if (!last) tmem_wait_st();
-                    } else {
-                        // int32 running sums, 16-column halves (keeps the live registers low)
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf) {
-                            uint32_t f16[16], run[16];
-                            tmem_ld16_nw(lane_base + buf * BN + cb * 32 + 16 * hf, f16);
-                            if (!first) tmem_ld16_nw(lane_base + run_col + 16 * hf, run);
-                            tmem_wait_ld();
-                            reg_fence(f16);
-                            if (!first) reg_fence(run);
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                ACC v = ((ACC)__float2int_rn(__uint_as_float(f16[j]))) << shift;
-                                if (!first) v += (ACC)(int)run[j];
-                                acc[16 * hf + j] = v;
-                            }
-                            if (!last) {
-#pragma unroll
-                                for (int j = 0; j < 16; ++j) run[j] = (uint32_t)(unsigned long long)acc[16 * hf + j];
-                                tmem_st16_nw(lane_base + run_col + 16 * hf, run);
-                            }
-                        }
-                        if (!last) tmem_wait_st();
-                    }
-                    if (c == CPW - 1) {
-                        // every chunk of this warp is out of the accumulator buffer: free it for the
-                        // next group's MMAs before the final arithmetic
-                        tc_fence_before();
-                        mbar_arrive(accempty0 + 8 * buf);
-                    }
-                    if (!last) continue;
-                    if (P.fast_store) {
-                        // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
-                        // (the epilogue constants are rebuilt here from the parameters rather than kept
-                        // live across the tile loop)
-                        uint32_t w[16];
-                        const Epi32 e32 = make_epi32(a);
-                        const Epi64 e64 = make_epi64(a);
-                        if (sizeof(ACC) == 4 && a.v32) {
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                int c2[2];
-#pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    const int k = k0 + 2 * j + h;
-                                    const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                    c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
-                                                       (b & e32.fmask) != 0 ? 1 : 0);
-                                }
-                                w[j] = pack_codes_f16(c2[0], c2[1]);
-                            }
-                        } else if (e64.ok) {
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                int c2[2];
-#pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    const int k = k0 + 2 * j + h;
-                                    const int32_t b = (e64.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                    c2[h] = epi64_code(e64, (long long)acc[2 * j + h], b);
-                                }
-                                w[j] = pack_codes_f16(c2[0], c2[1]);
-                            }
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                int c2[2];
-#pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    const int k = k0 + 2 * j + h;
-                                    const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                    c2[h] = qlayer_code(a, cblock_value(a, k, (long long)acc[2 * j + h], b));
-                                }
-                                w[j] = pack_codes_f16(c2[0], c2[1]);
-                            }
-                        }
-                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int chunk = (cb & 1) * 4 + q;
-                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
-                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-                        }
-                    } else if (m >= 0) {
-                        epilogue_block32<ACC>(a, m, k0, acc);
-                    }
-                }
-                ++gcount;
-                if (last && P.fast_store) {
-                    // make the staging writes visible to the async proxy, then one thread stores the tile
-                    fence_proxy_async();
-                    mbar_arrive(stg_full);
-                    if (leader) {
-                        if (!wait_bounded(stg_full, u & 1, abort, P.status)) {
-                            ok = false;
-                            break;
-                        }
-                        if (P.patch) {
-                            const int per_img = P.tiles_p * P.tiles_q;
-                            const int n_img = tm / per_img, r = tm - n_img * per_img;
-                            for (int hb = 0; hb < BN / 64; ++hb)
-                                tma_store_4d(&P.tmap_y, tn * BN + hb * 64, (r % P.tiles_q) * P.TW,
-                                             (r / P.tiles_q) * P.TH, n_img, smem_u32(sO + hb * (TC_BM * 128)));
-                        } else {
-                            for (int hb = 0; hb < BN / 64; ++hb)
-                                tma_store_2d(&P.tmap_y, tn * BN + hb * 64, tm * TC_BM,
-                                             smem_u32(sO + hb * (TC_BM * 128)));
-                        }
-                        bulk_commit();
-                    }
-                    ++u;
-                }
-            }
-        }
-        if (leader) bulk_wait0();  // every output store has completed
-    } else if (lane == 0 && P.patch == 3) {
-        // ============================================================ MMA issue, window mode
-        // Per tile and limb pair (ia, iw): R * S2/2 MMAs of K = 16 (two taps of 8 channels).  The A
-        // operand of taps (r, 2sp), (r, 2sp + 1) is the window shifted by (r, 2sp) pixels: K-major
-        // without swizzle, the two K core matrices one pixel (16 bytes) apart, the 8-row groups (the
-        // patch rows, TW = 8) one window row apart.  B is the resident box (iw, r, sp).
-        const int np = P.S2 / 2;
-        const uint32_t wbox = (uint32_t)(BN * 32);
-        uint32_t stage = 0, phase = 0, gcount = 0;
-        bool ok = wait_bounded(wbar, 0, abort, P.status);
-        tc_fence_after();
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-            const uint32_t buf = gcount & 1;
-            if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
-                !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            const uint32_t d0 = tmem + buf * (uint32_t)(P.nacc * BN);
-            const uint32_t wa = smem_u32(sA + stage * A_BYTES);
-            for (int ia = 0; ia < a.px; ++ia)
-                for (int iw = 0; iw < a.pw; ++iw) {
-                    const uint32_t d = d0 + (uint32_t)((ia * a.pw + iw) * BN);
-                    uint32_t accum = 0;
-                    for (int r = 0; r < a.R; ++r)
-                        for (int sp = 0; sp < np; ++sp) {
-                            const uint64_t ad = make_sdesc_noswz(
-                                wa + (uint32_t)(ia * P.win_bytes + (r * P.WW + 2 * sp) * 16), 16, (uint32_t)(P.WW * 16));
-                            const uint64_t bd =
-                                make_sdesc_noswz(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox,
-                                                 (uint32_t)(BN * 16), 128);
-                            tc_mma(d, ad, bd, IDESC, accum);
-                            accum = 1;
-                        }
-                }
-            tc_commit(empty0 + 8 * stage);
-            if (++stage == TC_STAGES) {
-                stage = 0;
-                phase ^= 1;
-            }
-            tc_commit(accfull0 + 8 * buf);
-            ++gcount;
-        }
-        // every MMA issued by this thread has completed once `done` fires
-        tc_commit(done_bar);
-        const long long t0 = clock64();
-        while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
-        }
-    } else if (lane == 0) {
-        // ============================================================ MMA issue (one thread of MMA_WARP)
-        // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
-        // (address >> 4, 14 bits) without carry since shared addresses stay below 256 KB.
-        // 8-channel patch tiles: no-swizzle A, one 16-element k step = two taps = 4096 bytes
-        const bool narrow_a = P.patch == 2;
-        const uint64_t adesc0 = narrow_a ? make_sdesc_noswz(smem_u32(sA), 2048, 128) : make_sdesc(smem_u32(sA));
-        const uint32_t a_kstep = narrow_a ? 4096u >> 4 : 2u;
-        const uint64_t bdesc0 = make_sdesc(smem_u32(sB));
-        uint32_t stage = 0, phase = 0, gcount = 0;
-        bool ok = true;
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
-                const TcGroup g = P.g[gi];
-                const uint32_t buf = P.nbuf == 2 ? (gcount & 1) : 0;
-                const uint32_t par = P.nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
-                if (!wait_bounded(accempty0 + 8 * buf, par ^ 1, abort, P.status)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t d = tmem + buf * BN;
-                uint32_t accum = 0;
-                for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                    if (!wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t ad = adesc0 + (uint64_t)((stage * A_BYTES) >> 4);
-                    const uint64_t bd = bdesc0 + (uint64_t)((stage * B_BYTES) >> 4);
-#pragma unroll
-                    for (int kk = 0; kk < TC_BK / 16; ++kk) {
-                        tc_mma(d, ad + a_kstep * kk, bd + 2 * kk, IDESC, accum);
-                        accum = 1;
-                    }
-                    tc_commit(empty0 + 8 * stage);
-                    if (++stage == TC_STAGES) {
-                        stage = 0;
-                        phase ^= 1;
-                    }
-                }
-                if (!ok) break;
-                tc_commit(accfull0 + 8 * buf);
-                ++gcount;
-            }
-        }
-        // every MMA issued by this thread has completed once `done` fires
-        tc_commit(done_bar);
-        const long long t0 = clock64();
-        while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == MMA_WARP) {
-        tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS));
-    }
-}
 
 int g_num_sms = 0;
 std::mutex g_tc_mu;
@@ -1052,10 +32,6 @@ int num_sms() {
     return g_num_sms;
 }
 
-template <int BN>
-constexpr size_t tc_smem_bytes() {
-    return 1024 + tc_stages(BN) * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
-}
 
 // Largest |limb| of a format's codes: the only plane (k <= 8) or the hi / lo limb (k > 8).
 long long limb_max(const fxpq_fmt& f, int plane) {
@@ -1283,27 +259,29 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     {
         std::lock_guard<std::mutex> lk(g_tc_mu);
         if (!g_tc_attr_set) {
-            if (cudaFuncSetAttribute(conv_tc_kernel<64, long long>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            if (cudaFuncSetAttribute(conv_tc_kernel<64, long long, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
-                cudaFuncSetAttribute(conv_tc_kernel<64, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                cudaFuncSetAttribute(conv_tc_kernel<64, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
-                cudaFuncSetAttribute(conv_tc_kernel<128, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                cudaFuncSetAttribute(conv_tc_kernel<128, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<128>()) != cudaSuccess ||
-                cudaFuncSetAttribute(conv_tc_kernel<256, int>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<256>()) != cudaSuccess)
                 return FXPQ_ERR_CUDA;
             g_tc_attr_set = true;
         }
     }
     const int grid = P.n_tiles < sms ? P.n_tiles : sms;
+    launched = true;
+    if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);
     if (acc64)
-        conv_tc_kernel<64, long long><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
+        conv_tc_kernel<64, long long, false><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 64)
-        conv_tc_kernel<64, int><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
+        conv_tc_kernel<64, int, false><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 128)
-        conv_tc_kernel<128, int><<<grid, tc_threads(128), tc_smem_bytes<128>(), st>>>(P);
+        conv_tc_kernel<128, int, false><<<grid, tc_threads(128), tc_smem_bytes<128>(), st>>>(P);
     else
-        conv_tc_kernel<256, int><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
+        conv_tc_kernel<256, int, false><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
     launched = true;
     return after_launch("conv_tc");
 }

@@ -119,7 +119,7 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
         const bool last = o.last != 0;
         switch (o.op) {
             case FXPQ_OP_CONV: {
-                fxpq_conv_desc d;
+                fxpq_conv_desc d = {};
                 d.N = batch;
                 d.H = s0.H;
                 d.W = s0.W;
@@ -137,6 +137,10 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
                 d.fmt_b = o.fmt_b;
                 d.fmt_y = o.fmt_y;
                 d.w_l1 = o.w_l1;
+                d.fmt_scale = o.fmt_scale;
+                d.fmt_shift = o.fmt_shift;
+                d.d_scale = o.d_scale;
+                d.d_shift = o.d_shift;
                 int32_t scale = 0;
                 st = fxpq_conv_fwd(&d, ptr(o.src0), o.d_w, o.d_bias, last ? (void*)d_logits : ptr(o.dst), &scale,
                                    nullptr, 0, stream);
@@ -266,7 +270,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
             case FXPQ_OP_CONV: {
                 // one contraction with exact int64 values; the QLayer runs twice (fp32 image for the
                 // search, then the codes)
-                fxpq_conv_desc cd;
+                fxpq_conv_desc cd = {};
                 cd.N = n_calib;
                 cd.H = s0.H;
                 cd.W = s0.W;
@@ -284,6 +288,10 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.fmt_b = o.fmt_b;
                 cd.fmt_y = fy;
                 cd.w_l1 = o.w_l1;
+                cd.fmt_scale = o.fmt_scale;
+                cd.fmt_shift = o.fmt_shift;
+                cd.d_scale = o.d_scale;
+                cd.d_shift = o.d_shift;
                 int32_t sc = 0;
                 st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, nullptr, 0, s);
                 if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_F32, fy, f32, s);

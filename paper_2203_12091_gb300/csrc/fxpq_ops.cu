@@ -228,3 +228,36 @@ extern "C" fxpq_status fxpq_qlayer(const int64_t* d_v, int64_t n, int32_t s, int
     qlayer_kernel<<<grid_for(n), 256, 0, as_stream(stream)>>>(reinterpret_cast<const long long*>(d_v), n, o, d_y);
     return after_launch("qlayer");
 }
+
+// ---------------------------------------------------------------- BN -> Scale (Sec. IV-A.1)
+namespace fxpq {
+namespace {
+
+// aleph1 = gamma / r and aleph2 = beta - (gamma * mean) / r with r = sqrt(var + eps), every step one
+// correctly rounded fp32 operation (the _rn intrinsics are IEEE round-to-nearest-even, so the
+// result does not depend on contraction into fused multiply-adds).
+__global__ void bn_to_scale_kernel(const float* __restrict__ g, const float* __restrict__ b,
+                                   const float* __restrict__ mu, const float* __restrict__ var, long long n, float eps,
+                                   float* __restrict__ a1, float* __restrict__ a2) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const float r = __fsqrt_rn(__fadd_rn(var[i], eps));
+    a1[i] = __fdiv_rn(g[i], r);
+    a2[i] = __fsub_rn(b[i], __fdiv_rn(__fmul_rn(g[i], mu[i]), r));
+}
+
+}  // namespace
+}  // namespace fxpq
+
+extern "C" fxpq_status fxpq_bn_to_scale(const float* d_gamma, const float* d_beta, const float* d_mean,
+                                        const float* d_var, int64_t n, float eps, float* d_aleph1, float* d_aleph2,
+                                        void* stream) {
+    using namespace fxpq;
+    if (n < 0 || !(eps >= 0.0f)) return FXPQ_ERR_INVALID_ARG;
+    if (n == 0) return FXPQ_OK;
+    if (!d_gamma || !d_beta || !d_mean || !d_var || !d_aleph1 || !d_aleph2) return FXPQ_ERR_INVALID_ARG;
+    const int T = 256;
+    bn_to_scale_kernel<<<(unsigned)((n + T - 1) / T), T, 0, as_stream(stream)>>>(d_gamma, d_beta, d_mean, d_var, n,
+                                                                                 eps, d_aleph1, d_aleph2);
+    return after_launch("bn_to_scale");
+}

@@ -132,10 +132,22 @@ def fxpq_fl_init(stats: Stats, bits: int, strategy: int) -> Fmt:
     return out
 
 
+def fxpq_bn_to_scale(gamma, beta, mean, var, eps, aleph1, aleph2, stream=None):
+    """BN -> Scale layer parameters (fp32 device tensors of one length)."""
+    L.check("fxpq_bn_to_scale", L.lib().fxpq_bn_to_scale(_p(gamma), _p(beta), _p(mean), _p(var), gamma.numel(),
+                                                          float(eps), _p(aleph1), _p(aleph2), _s(stream)))
+    return aleph1, aleph2
+
+
 # ------------------------------------------------------------------------------ C-Blocks
-def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy, w_l1=0) -> L.ConvDesc:
+def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy, w_l1=0,
+              scale=None, fmt_scale=None, shift=None, fmt_shift=None) -> L.ConvDesc:
+    """C-Block descriptor.  scale / shift: int32 aleph1 / aleph2 code tensors [K] of a Scale layer (both
+    or neither; the caller keeps them alive while the descriptor is used)."""
     return L.ConvDesc(N, H, W, C, Cp, K, R, S, stride, pad, int(relu), out_mode, fx, fw,
-                      fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0), int(w_l1))
+                      fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0), int(w_l1),
+                      fmt_scale if fmt_scale is not None else Fmt(16, 1, 0),
+                      fmt_shift if fmt_shift is not None else Fmt(16, 1, 0), _p(scale), _p(shift))
 
 
 def fxpq_conv_fwd(desc: L.ConvDesc, x, w, bias, y, stream=None) -> int:

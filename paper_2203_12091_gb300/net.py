@@ -2,12 +2,16 @@
 activation formats, and the op list handed to ``fxpq_net_forward`` (Sec. IV-A.2).
 
 A layer list is a list of dicts (the format the workload generators produce):
-  {"type": "conv", "name", "C", "K", "R", "stride", "pad", "relu", "src"}   (FC = conv over the map)
+  {"type": "conv", "name", "C", "K", "R", "stride", "pad", "relu", "src"[, "bn"]}   (FC = conv over the map)
   {"type": "maxpool", "name", "k", "stride", "pad"}
   {"type": "eltwise", "name", "a", "b", "relu"}
   {"type": "avgpool", "name", "src"}
 ``src`` (or ``a``/``b``) names the producing layer; ``None`` means the previous layer, and
 "input" is the network input.  The last layer must be a conv/FC: it has no FxP-QLayer.
+
+A conv with "bn" is followed by a BatchNorm layer, which becomes a Scale layer (Sec. IV-A.1): its
+aleph1 / aleph2 are computed by ``fxpq_bn_to_scale``, searched and quantized like weights and biases,
+and applied in the conv's epilogue.
 
 Calibration follows the forward optimizer's order (Sec. IV-C): layer by layer, weights' FL, then
 bias FL, then the output activation FL; each FL comes from ``fxpq_fl_search`` at the planned
@@ -26,6 +30,7 @@ from . import _lib as L
 from . import fxpq as F
 
 FL_LO, FL_HI = -8, 23
+BN_EPS = 1e-5  # the BatchNorm epsilon of the rewritten layers (Caffe's and torchvision's default)
 
 
 def pad8(c: int) -> int:
@@ -85,7 +90,8 @@ class QNet:
         self.hw, self.cin = hw, cin
         self.cp_in = pad8(cin)
         self.fmts = {}
-        self.q = {}  # name -> (weight fp16 codes, bias int32 codes)
+        self.q = {}  # name -> (weight fp16 codes, bias int32 codes or None)
+        self.qs = {}  # BN conv name -> (aleph1 int32 codes, aleph2 int32 codes)
         self.w_l1 = {}  # conv name -> max over output channels of sum |weight code| (0: unknown)
         self.names = ["input"] + [L_["name"] for L_ in layers]
         self.slot = {nm: i for i, nm in enumerate(self.names)}
@@ -96,15 +102,16 @@ class QNet:
         s = L_.get(key)
         return s if s is not None else (self.names[i] if i > 0 else "input")
 
-    def quantize_params(self, weights_dev, plan, stream=None):
-        """weights_dev: name -> (fp32 KRSC weight, fp32 bias) device tensors; plan: wordlengths.
+    def quantize_params(self, weights_dev, plan, stream=None, bn_dev=None):
+        """weights_dev: name -> (fp32 KRSC weight, fp32 bias or None) device tensors; plan: wordlengths;
+        bn_dev: BN conv name -> (gamma, beta, running mean, running variance) fp32 device tensors.
 
         Every parameter's FL search runs as one batch, every quantization as one launch reading the
         chosen formats on the device, and one read-back returns the formats and the L1 bounds."""
         shapes = {"input": (self.hw, self.hw, self.cp_in)}
         searches, owners = [], []
         dev = next(iter(weights_dev.values()))[0].device
-        recips = {}
+        recips, alephs = {}, {}
         for i, L_ in enumerate(self.layers):
             nm = L_["name"]
             self.fmts.setdefault(nm, {})
@@ -113,8 +120,18 @@ class QNet:
                 w, b = weights_dev[nm]
                 K, R, _, C = w.shape
                 assert C <= Cp
-                searches += [(w, plan[nm]["w"]), (b, plan[nm]["b"])]
-                owners += [(nm, "w"), (nm, "b")]
+                searches.append((w, plan[nm]["w"]))
+                owners.append((nm, "w"))
+                if b is not None:
+                    searches.append((b, plan[nm]["b"]))
+                    owners.append((nm, "b"))
+                if L_.get("bn"):
+                    a1 = torch.empty(K, dtype=torch.float32, device=dev)
+                    a2 = torch.empty(K, dtype=torch.float32, device=dev)
+                    F.fxpq_bn_to_scale(*bn_dev[nm], BN_EPS, a1, a2, stream)
+                    alephs[nm] = (a1, a2)
+                    searches += [(a1, plan[nm]["s"]), (a2, plan[nm]["h"])]
+                    owners += [(nm, "s"), (nm, "h")]
                 P = (H + 2 * L_["pad"] - R) // L_["stride"] + 1
                 shapes[nm] = (P, P, K)
             elif L_["type"] == "maxpool":
@@ -149,15 +166,25 @@ class QNet:
                 w, b = weights_dev[nm]
                 K, R, _, C = w.shape
                 Cp = shapes[self._src(i, L_)][2]
-                kw, kb = plan[nm]["w"], plan[nm]["b"]
+                kw, kb = plan[nm]["w"], plan[nm].get("b")
                 wq = torch.empty(K * R * R * Cp * (2 if kw > 8 else 1), dtype=torch.float16, device=dev)
-                bq = torch.empty(K, dtype=torch.int32, device=dev)
                 l1p = base + off_l1 + 8 * conv_names.index(nm) if kw <= 8 else None
                 items.append(L.QuantizeItem(w.data_ptr(), wq.data_ptr(), L.QB_ROWS_F16, kw, K * R * R, C, Cp, R * R, 0,
                                             rec[(nm, "w")], rec[(nm, "w")] + 8, l1p))
-                items.append(L.QuantizeItem(b.data_ptr(), bq.data_ptr(), L.QB_FLAT_I32, kb, K, 0, 0, 1, 0,
-                                            rec[(nm, "b")], rec[(nm, "b")] + 8, None))
+                bq = None
+                if b is not None:
+                    bq = torch.empty(K, dtype=torch.int32, device=dev)
+                    items.append(L.QuantizeItem(b.data_ptr(), bq.data_ptr(), L.QB_FLAT_I32, kb, K, 0, 0, 1, 0,
+                                                rec[(nm, "b")], rec[(nm, "b")] + 8, None))
                 self.q[nm] = (wq, bq)
+                if nm in alephs:
+                    codes = []
+                    for key, t in zip(("s", "h"), alephs[nm]):
+                        c = torch.empty(K, dtype=torch.int32, device=dev)
+                        items.append(L.QuantizeItem(t.data_ptr(), c.data_ptr(), L.QB_FLAT_I32, plan[nm][key], K, 0, 0,
+                                                    1, 0, rec[(nm, key)], rec[(nm, key)] + 8, None))
+                        codes.append(c)
+                    self.qs[nm] = tuple(codes)
             elif L_["type"] == "avgpool":
                 items.append(L.QuantizeItem(recips[nm].data_ptr(), base + off_rc + 4 * avg_names.index(nm),
                                             L.QB_FLAT_I32, plan[nm]["r"], 1, 0, 0, 1, 0,
@@ -190,8 +217,10 @@ class QNet:
             x, fx = env[src]
             sH, sW, sCp = self.shapes[src]
             wq, bq = self.q[nm]
+            sq, hq = self.qs.get(nm, (None, None))
             d = F.conv_desc(N, sH, sW, sCp, sCp, L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], L_["relu"],
-                            out_mode, fx, self.fmts[nm]["w"], self.fmts[nm]["b"], fy, self.w_l1.get(nm, 0))
+                            out_mode, fx, self.fmts[nm]["w"], self.fmts[nm].get("b"), fy, self.w_l1.get(nm, 0),
+                            scale=sq, fmt_scale=self.fmts[nm].get("s"), shift=hq, fmt_shift=self.fmts[nm].get("h"))
             s = F.fxpq_conv_fwd(d, x, wq, bq, y, stream)
         elif L_["type"] == "maxpool":
             src = self._src(i, L_)
@@ -246,11 +275,14 @@ class QNet:
                 o.op = L.OP_CONV
                 o.src0 = self.slot[self._src(i, L_)]
                 o.K, o.R, o.S, o.stride, o.pad, o.relu = L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], int(L_["relu"])
-                o.fmt_w, o.fmt_b = self.fmts[nm]["w"], self.fmts[nm]["b"]
+                o.fmt_w, o.fmt_b = self.fmts[nm]["w"], self.fmts[nm].get("b", L.Fmt(32, 1, 0))
                 o.fmt_y = self.fmts[nm].get("a", L.Fmt(8, 1, 0))
                 o.d_w = self.q[nm][0].data_ptr()
-                o.d_bias = self.q[nm][1].data_ptr()
+                o.d_bias = self.q[nm][1].data_ptr() if self.q[nm][1] is not None else None
                 o.w_l1 = self.w_l1.get(nm, 0)
+                if nm in self.qs:
+                    o.fmt_scale, o.fmt_shift = self.fmts[nm]["s"], self.fmts[nm]["h"]
+                    o.d_scale, o.d_shift = self.qs[nm][0].data_ptr(), self.qs[nm][1].data_ptr()
             elif L_["type"] == "maxpool":
                 o.op = L.OP_MAXPOOL
                 o.src0 = self.slot[self._src(i, L_)]
@@ -306,12 +338,15 @@ class QNet:
         return env
 
 
-def build_qnet(layers, weights_np, calib_images, plan, device="cuda", stream=None):
-    """Quantize parameters and calibrate on `calib_images` (fp32 NCHW device tensor)."""
-    wdev = {nm: (torch.from_numpy(w).to(device), torch.from_numpy(b).to(device)) for nm, (w, b) in weights_np.items()}
+def build_qnet(layers, weights_np, calib_images, plan, device="cuda", stream=None, bn_np=None):
+    """Quantize parameters and calibrate on `calib_images` (fp32 NCHW device tensor).  bn_np: BN conv
+    name -> (gamma, beta, mean, var) fp32 arrays (layers with "bn")."""
+    wdev = {nm: (torch.from_numpy(w).to(device), None if b is None else torch.from_numpy(b).to(device))
+            for nm, (w, b) in weights_np.items()}
+    bn_dev = {nm: tuple(torch.from_numpy(t).to(device) for t in v) for nm, v in (bn_np or {}).items()}
     q = QNet(layers, hw=calib_images.shape[-1], cin=calib_images.shape[1])
     q._dev = torch.device(device)
-    q.quantize_params(wdev, plan, stream)
+    q.quantize_params(wdev, plan, stream, bn_dev)
     q.calibrate(calib_images, plan, stream)
     q.weights_dev = wdev
     return q

@@ -85,11 +85,12 @@ def vgg16():
     return L
 
 
-def resnet18():
-    """ResNet-18 (torchvision topology), BN folded into each conv as a bias.  Stage 1 uses identity
-    shortcuts; stages 2-4 open with a 1x1/2 downsample shortcut.  Every conv output, and every
-    residual add (+ReLU), is a C-Block followed by a QLayer; MAX-POOL has none; the global AVG-POOL
-    multiplies by the quantized reciprocal 1/49."""
+def resnet18(bn: bool = False):
+    """ResNet-18 (torchvision topology), BN folded into each conv as a bias, or (bn=True) kept as a
+    Scale layer after a bias-free conv (the Caffe ResNet form: CONV, BatchNorm, Scale, ReLU).  Stage 1
+    uses identity shortcuts; stages 2-4 open with a 1x1/2 downsample shortcut.  Every conv output,
+    and every residual add (+ReLU), is a C-Block followed by a QLayer; MAX-POOL has none; the global
+    AVG-POOL multiplies by the quantized reciprocal 1/49."""
     L = [_conv("conv1", 3, 64, 7, 2, 3), {"type": "maxpool", "name": "pool1", "k": 3, "stride": 2, "pad": 1}]
     cin = 64
     prev = "pool1"
@@ -107,16 +108,25 @@ def resnet18():
             L.append({"type": "eltwise", "name": pfx, "a": pfx + "_branch2b", "b": short, "relu": True})
             prev = pfx
             cin = c
+    if bn:
+        for layer in L:
+            if layer["type"] == "conv":
+                layer["bn"] = True
     L.append({"type": "avgpool", "name": "pool5", "src": prev})
     L.append(_conv("fc", 512, 1000, 1, 1, 0, relu=False, src="pool5"))
     return L
 
 
-ARCHS = {"alexnet": alexnet, "vgg16": vgg16, "resnet18": resnet18}
+def resnet18_bn():
+    return resnet18(bn=True)
+
+
+ARCHS = {"alexnet": alexnet, "vgg16": vgg16, "resnet18": resnet18, "resnet18_bn": resnet18_bn}
 
 
 def weights(arch: str, seed: int):
-    """He-normal fp32 weights (std sqrt(2 / (C*R*R))) in KRSC and N(0, 0.01) biases, per conv/FC layer."""
+    """He-normal fp32 weights (std sqrt(2 / (C*R*R))) in KRSC and N(0, 0.01) biases, per conv/FC layer;
+    a conv followed by a BN layer has no bias (None)."""
     g = _gen(seed)
     out = {}
     for L in ARCHS[arch]():
@@ -124,8 +134,29 @@ def weights(arch: str, seed: int):
             continue
         fan_in = L["C"] * L["R"] * L["R"]
         w = torch.randn(L["K"], L["R"], L["R"], L["C"], generator=g, dtype=torch.float32) * float(np.sqrt(2.0 / fan_in))
+        if L.get("bn"):
+            out[L["name"]] = (w.numpy(), None)
+            continue
         b = torch.randn(L["K"], generator=g, dtype=torch.float32) * 0.01
         out[L["name"]] = (w.numpy(), b.numpy())
+    return out
+
+
+def bn_params(arch: str, seed: int):
+    """Per BN layer (a conv with "bn"): fp32 (gamma, beta, running mean, running variance) of its K
+    channels, drawn as gamma ~ U(0.5, 1.5), beta ~ N(0, 0.2), mean ~ N(0, 0.2), var ~ U(0.5, 2.0)
+    (no trained statistics exist; these keep the per-channel gain aleph1 within about [0.35, 2.1])."""
+    g = _gen(seed)
+    out = {}
+    for L in ARCHS[arch]():
+        if L["type"] != "conv" or not L.get("bn"):
+            continue
+        K = L["K"]
+        gamma = torch.rand(K, generator=g, dtype=torch.float32) + 0.5
+        beta = torch.randn(K, generator=g, dtype=torch.float32) * 0.2
+        mean = torch.randn(K, generator=g, dtype=torch.float32) * 0.2
+        var = torch.rand(K, generator=g, dtype=torch.float32) * 1.5 + 0.5
+        out[L["name"]] = tuple(t.numpy() for t in (gamma, beta, mean, var))
     return out
 
 
@@ -135,6 +166,8 @@ def bit_plan(arch: str, seed: int):
     alexnet : 8-bit weights and activations (input included), 16-bit biases.
     resnet18: weight bits drawn from {3..8}, activation bits from {4..8} (seeded), 16-bit biases,
               16-bit unsigned AVG-POOL reciprocal.
+    resnet18_bn: resnet18's draws; each BN layer's Scale parameters aleph1 ("s") and aleph2 ("h")
+              16-bit (the C-Block's 16-bit multiplier, Sec. IV-B) in place of the bias.
     vgg16   : first and last layers 16-bit (input image, conv1_1 weights, fc7 output and fc8 weights),
               every other weight / activation drawn from {4..8} (seeded), 16-bit biases.
     Returns {"input": a_bits, layer_name: {"w": .., "b": .., "a": ..}} where "a" is the wordlength of
@@ -152,11 +185,12 @@ def bit_plan(arch: str, seed: int):
                 if L["name"] != "fc8":
                     plan[L["name"]]["a"] = 8
         return plan
-    if arch == "resnet18":
+    if arch in ("resnet18", "resnet18_bn"):
         plan["input"] = int(rng.integers(4, 9))
         for L in layers:
             if L["type"] == "conv":
-                plan[L["name"]] = {"w": int(rng.integers(3, 9)), "b": 16}
+                plan[L["name"]] = {"w": int(rng.integers(3, 9))}
+                plan[L["name"]].update({"s": 16, "h": 16} if L.get("bn") else {"b": 16})
                 if L["name"] != "fc":
                     plan[L["name"]]["a"] = int(rng.integers(4, 9))
             elif L["type"] in ("eltwise", "avgpool"):

@@ -108,3 +108,32 @@ def test_status_strings(lib):
     for c in range(8):
         assert lib.fxpq_status_string(c)
     assert lib.fxpq_launch_count() >= 0
+
+
+def test_struct_layout_matches_header(tmp_path):
+    """Every ctypes mirror of a header struct has the C compiler's size and field offsets."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no host C compiler")
+    mirrors = {"fxpq_fmt": L.Fmt, "fxpq_stats": L.Stats, "fxpq_fl_search_item": L.FlSearchItem,
+               "fxpq_quantize_item": L.QuantizeItem, "fxpq_conv_desc": L.ConvDesc, "fxpq_op_desc": L.OpDesc,
+               "fxpq_net": L.Net}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "fxpq.h"', "int main(void) {"]
+    for cname, py in mirrors.items():
+        lines.append(f'printf("{cname} sizeof %zu\\n", sizeof({cname}));')
+        for f, _ in py._fields_:
+            lines.append(f'printf("{cname} {f} %zu\\n", offsetof({cname}, {f}));')
+    lines += ["return 0; }"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.dirname(HDR), str(src), "-o", str(exe)], check=True)
+    got = {}
+    for ln in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.splitlines():
+        c, f, v = ln.split()
+        got[(c, f)] = int(v)
+    for cname, py in mirrors.items():
+        assert got[(cname, "sizeof")] == ctypes.sizeof(py), cname
+        for f, _ in py._fields_:
+            assert got[(cname, f)] == getattr(py, f).offset, (cname, f)

@@ -47,7 +47,7 @@ def to_f16_planes(codes, k, Cp):
     return torch.from_numpy(np.stack([hi, lo]).astype(np.float16)).cuda()
 
 
-def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0):
+def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0, scale=None):
     N, H, W, C = x.shape
     K, R, S, _ = w.shape
     P = (H + 2 * pad - R) // stride + 1
@@ -61,7 +61,13 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0):
         y = torch.empty(N * P * Q * K, dtype=torch.int64, device="cuda")
     else:
         y = torch.empty(N * P * Q * K, dtype=torch.float32, device="cuda")
-    d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy, w_l1)
+    sd = hd = fs = fh = None
+    if scale is not None:
+        m, fs, h, fh = scale
+        sd = torch.from_numpy(m.astype(np.int32)).cuda()
+        hd = torch.from_numpy(h.astype(np.int32)).cuda()
+    d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy, w_l1,
+                    scale=sd, fmt_scale=fs, shift=hd, fmt_shift=fh)
     s = F.fxpq_conv_fwd(d, xd, wd, bd, y)
     torch.cuda.synchronize()
     assert F.fxpq_get_device_status() == 0
@@ -70,9 +76,14 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0):
     return y.cpu().numpy().reshape(N, P, Q, K), s
 
 
-def oracle_conv(x, fx, w, fw, b, fb, stride, pad, relu, mode, fy):
+def oracle_conv(x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, scale=None):
     acc = oracle.conv2d(x, w, stride, pad)
-    v, s = oracle.cblock(acc, fx.fl + fw.fl, b, fb.fl if fb is not None else 0, relu)
+    if scale is None:
+        v, s = oracle.cblock(acc, fx.fl + fw.fl, b, fb.fl if fb is not None else 0, relu)
+    else:
+        m, fs, h, fh = scale
+        v, s = oracle.cblock(acc, fx.fl + fw.fl, b, fb.fl if fb is not None else 0, relu,
+                             scale=m, fl_scale=fs.fl, shift=h, fl_shift=fh.fl)
     if mode == 0:
         return oracle.requant(v, s, fy.bits, fy.is_signed, fy.fl), s
     if mode == 1:
@@ -254,3 +265,42 @@ def test_avgpool_parity(F, bits):
     v, ws = oracle.avgpool_global(x, 4, rc, 21)
     assert s == ws
     assert np.array_equal(F.codes_to_int(y.cpu(), fy, (N, C)).numpy(), oracle.requant(v, ws, 8, 0, 5))
+
+
+# Scale layer cases: a CASES geometry, then (k, FL) of aleph1 and of aleph2 (both signed)
+SCALE_CASES = [
+    (CASES[0], (16, 14), (16, 12)),     # 8-bit, bias; 64-bit epilogue with the Scale layer
+    (CASES[8], (16, 13), (16, 10)),     # no bias (ResNet-style conv), fp32 calibration image
+    (CASES[7], (12, 9), (16, 30)),      # ACC64; aleph2 finer than the product (delta2 < 0)
+    (CASES[10], (16, 14), (16, 12)),    # requantizing left shift and saturation
+    (CASES[12], (8, 5), (16, 3)),       # bias finer than the accumulator, then the Scale layer
+    (CASES[16], (16, 14), (16, 11)),    # patch tiles
+    (CASES[22], (16, 15), (16, 13)),    # two limbs in, two planes out
+    (CASES[25], (16, 14), (16, 12)),    # 256-column tiles
+    (CASES[32], (16, 14), (16, 12)),    # window mode, two-limb fast epilogue
+    (CASES[35], (16, 14), (16, 12)),    # window mode, ACC64
+]
+
+
+@pytest.mark.parametrize("sc", SCALE_CASES)
+def test_conv_scale_layer_parity(F, sc):
+    """CONV (+bias) -> Scale (aleph1, aleph2) -> ReLU -> FxP-QLayer (Sec. IV-A.1, IV-B), bit-exact."""
+    case, (ks, fls), (kh, flh) = sc
+    N, H, C, K, R, st, pad, tx, tw, tb, relu, mode, ty = case
+    rng = np.random.default_rng(H * 131 + K + 7)
+    fx, fw = F.fmt(*tx), F.fmt(*tw)
+    fb = F.fmt(tb[0], 1, tb[1]) if tb else None
+    fy = F.fmt(*ty) if ty else None
+    x = rand_codes(rng, (N, H, H, C), tx[0], tx[1])
+    w = rand_codes(rng, (K, R, R, C), tw[0], tw[1])
+    w = np.where(rng.random(w.shape) < 0.8, w // 4, w)
+    b = rand_codes(rng, (K,), tb[0], 1) if tb else None
+    m = rand_codes(rng, (K,), ks, 1)
+    h = rand_codes(rng, (K,), kh, 1)
+    scale = (m, F.fmt(ks, 1, fls), h, F.fmt(kh, 1, flh))
+    Cp = (C + 7) // 8 * 8
+    got, s = run_conv(F, x, fx, w, fw, b, fb, st, pad, relu, mode, fy, Cp, scale=scale)
+    want, ws = oracle_conv(x, fx, w, fw, b, fb, st, pad, relu, mode, fy,
+                           scale=(m, scale[1], h, scale[3]))
+    assert s == ws
+    assert np.array_equal(got, want)

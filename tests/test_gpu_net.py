@@ -76,10 +76,11 @@ def _workload(NET, arch, batch, seed, plan_seed=None, calib=8, sample=(0, -1)):
     L = synth.ARCHS[arch]()
     W = synth.weights(arch, seed)
     plan = synth.bit_plan(arch, seed if plan_seed is None else plan_seed)
+    bn = synth.bn_params(arch, seed + 100)
     imgs = synth.images(batch, seed)
     dimgs = torch.from_numpy(imgs).cuda()
-    q = NET.build_qnet(L, W, dimgs[:calib], plan)
-    fm, qp = onet.calibrate(L, W, imgs[:calib], plan)
+    q = NET.build_qnet(L, W, dimgs[:calib], plan, bn_np=bn)
+    fm, qp = onet.calibrate(L, W, imgs[:calib], plan, bn)
     fmts_equal(q.fmts, fm)
     logits, s = q.forward(dimgs)
     torch.cuda.synchronize()
@@ -99,6 +100,31 @@ def test_alexnet_batch256(NET):
 
 def test_resnet18_batch128(NET):
     _workload(NET, "resnet18", 128, 6)
+
+
+def test_resnet18_bn_batch128(NET):
+    """ResNet-18 with its BN layers kept as Scale layers (bias-free convs, aleph1 / aleph2 applied in the
+    conv epilogue before ReLU), the paper's own form of the network."""
+    _workload(NET, "resnet18_bn", 128, 6)
+
+
+def test_bn_to_scale_bit_exact(NET):
+    """fxpq_bn_to_scale against the oracle's fp32 formula, bit for bit (every step correctly rounded)."""
+    from oracle import bn_to_scale
+    from paper_2203_12091_gb300 import fxpq as F
+    rng = np.random.default_rng(31)
+    n = 10007
+    g = rng.uniform(-2, 2, n).astype(np.float32)
+    b = rng.normal(0, 1, n).astype(np.float32)
+    mu = rng.normal(0, 3, n).astype(np.float32)
+    var = np.concatenate([rng.uniform(0, 5, n - 3), [0.0, 1e-30, 1e6]]).astype(np.float32)
+    d = [torch.from_numpy(t).cuda() for t in (g, b, mu, var)]
+    a1 = torch.empty(n, dtype=torch.float32, device="cuda")
+    a2 = torch.empty(n, dtype=torch.float32, device="cuda")
+    F.fxpq_bn_to_scale(*d, NET.BN_EPS, a1, a2)
+    w1, w2 = bn_to_scale(g, b, mu, var, NET.BN_EPS)
+    assert np.array_equal(a1.cpu().numpy().view(np.uint32), w1.view(np.uint32))
+    assert np.array_equal(a2.cpu().numpy().view(np.uint32), w2.view(np.uint32))
 
 
 @pytest.mark.parametrize("plan_seed", [7, 38])

@@ -430,3 +430,59 @@ def test_architecture_size_pins():
     assert 15.3e9 <= synth.macs_per_image("vgg16") <= 15.5e9
     assert abs(synth.macs_per_image("resnet18") - 1.8e9) < 0.05e9
     assert sum(1 for L in synth.vgg16() if L["type"] == "conv") == 16
+
+
+def _bn_net(with_bn: bool):
+    layers = [
+        {"type": "conv", "name": "c1", "C": 3, "K": 8, "R": 3, "stride": 1, "pad": 1, "relu": True, "src": None},
+        {"type": "conv", "name": "c2", "C": 8, "K": 8, "R": 3, "stride": 1, "pad": 1, "relu": False, "src": None},
+        {"type": "conv", "name": "fc", "C": 8, "K": 4, "R": 6, "stride": 1, "pad": 0, "relu": False, "src": None},
+    ]
+    if with_bn:
+        layers[0]["bn"] = layers[1]["bn"] = True
+    return layers
+
+
+def test_scale_layer_with_unit_gain_is_the_folded_bias_net():
+    """Special case of the BN rewrite (Sec. IV-A.1): with gamma = sqrt(var + eps) (so aleph1 = 1 exactly,
+    quantized to code 1 at FL 0) and mean = 0 (aleph2 = beta), a bias-free CONV -> Scale -> ReLU network
+    is the folded network CONV(+bias beta) -> ReLU, bit for bit: same formats, same codes, same logits."""
+    rng = np.random.default_rng(21)
+    folded, withbn = _bn_net(False), _bn_net(True)
+    W, Wbn, bn = {}, {}, {}
+    for L in folded:
+        fan = L["C"] * L["R"] ** 2
+        w = (rng.standard_normal((L["K"], L["R"], L["R"], L["C"])) * np.sqrt(2 / fan)).astype(np.float32)
+        b = (rng.standard_normal(L["K"]) * 0.05).astype(np.float32)
+        W[L["name"]] = (w, b)
+        if L["name"] == "fc":
+            Wbn["fc"] = (w, b)
+            continue
+        Wbn[L["name"]] = (w, None)
+        var = rng.uniform(0.5, 2.0, L["K"]).astype(np.float32)
+        gamma = np.sqrt(var + np.float32(1e-5)).astype(np.float32)
+        bn[L["name"]] = (gamma, b, np.zeros(L["K"], np.float32), var)
+    a1, a2 = oracle.bn_to_scale(*bn["c1"])
+    assert np.all(a1 == 1.0) and np.array_equal(a2, W["c1"][1])
+    plan = {"input": 8, "c1": {"w": 6, "b": 16, "s": 16, "h": 16, "a": 7},
+            "c2": {"w": 7, "b": 16, "s": 16, "h": 16, "a": 8}, "fc": {"w": 8, "b": 16}}
+    imgs = synth.images(3, 5, hw=6)
+    f0, q0 = onet.calibrate(folded, W, imgs, plan)
+    f1, q1 = onet.calibrate(withbn, Wbn, imgs, plan, bn)
+    for nm in ("c1", "c2"):
+        assert f1[nm]["s"] == (16, 0, 0) and np.all(q1[nm][2] == 1)
+        assert f1[nm]["h"] == f0[nm]["b"] and np.array_equal(q1[nm][3], q0[nm][1])
+        assert f1[nm]["a"] == f0[nm]["a"]
+    l0, s0 = onet.forward(folded, f0, q0, imgs)
+    l1, s1 = onet.forward(withbn, f1, q1, imgs)
+    assert s0 == s1 and np.array_equal(l0, l1)
+
+
+def test_scale_layer_gain_applies_before_relu_and_requant():
+    """A Scale layer with gain -1 (gamma = -sqrt(var + eps)) and no shift flips the sign of the conv value
+    before ReLU: the C-Block output equals relu(-conv), not -relu(conv)."""
+    rng = np.random.default_rng(22)
+    acc = rng.integers(-2 ** 20, 2 ** 20, size=(5, 4))
+    v, s = oracle.cblock(acc, 10, None, 0, True, scale=np.full(4, -1), fl_scale=0, shift=np.zeros(4, np.int64),
+                         fl_shift=0)
+    assert s == 10 and np.array_equal(v, np.maximum(-acc, 0))
