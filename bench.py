@@ -376,6 +376,28 @@ def run_kernel(args):
             ms = sum(ts) / len(ts)
             gbs = (4 + bw) * n / (ms / 1e3) / 1e9
             out[name] = {"ms": round(ms, 4), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 3)}
+    if args.kernel in ("quantize", "all"):
+        # packed k-bit storage of 64M 4-bit codes: 2 B read + 0.5 B written per code (pack), the reverse
+        # for unpack
+        n = 1 << 26
+        f4 = F.fmt(4, 1, 0)
+        codes = torch.randint(-8, 8, (n,), dtype=torch.int32, device="cuda").to(torch.float16)
+        words = torch.empty(F.packed_words(n, f4), dtype=torch.int32, device="cuda")
+        hbm = measured_peaks()[0]
+        for name, fn in (("pack_k4", lambda: F.fxpq_pack_codes(codes, n, f4, words)),
+                         ("unpack_k4", lambda: F.fxpq_unpack_codes(words, n, f4, codes))):
+            ts = []
+            for i in range(args.warmup + args.steps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                fn()
+                e1.record()
+                e1.synchronize()
+                if i >= args.warmup:
+                    ts.append(e0.elapsed_time(e1))
+            ms = sum(ts) / len(ts)
+            gbs = 2.5 * n / (ms / 1e3) / 1e9
+            out[name] = {"ms": round(ms, 4), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 3)}
     if args.kernel in ("forward", "all"):
         # the integer forward of the bench workload alone (one plan, calibrated once): the target of the
         # per-launch DRAM traffic capture of the conv kernels
@@ -389,6 +411,7 @@ def run_kernel(args):
         q._dev = imgs.device
         q.quantize_params(wdev, plan, None, bndev)
         q.calibrate(imgs[: wl["calib"]], plan)
+        out["memory"] = {k: round(v, 3) for k, v in q.memory().items()}
         ts = []
         for i in range(args.warmup + args.steps):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)

@@ -287,6 +287,17 @@ FXPQ_API fxpq_status fxpq_avgpool(const void* d_x, int32_t N, int32_t H, int32_t
                          int32_t recip_code, fxpq_fmt fmt_recip, int32_t out_mode, fxpq_fmt fmt_y,
                          void* d_y, int32_t* h_out_scale, void* stream);
 
+/* Packed k-bit code storage (the footprint of Sec. V-E.2's memory model: k bits per code, Eq. mfp).
+ * Codes are taken in groups of 32 (the last zero-padded); group g occupies k = fmt.bits uint32 words,
+ * word g*k + b holding bit b of the k-bit two's-complement field of code 32g + i at bit i (a bit-plane
+ * layout: a warp packs a group with k ballots and unpacks it with k shuffles).  Unpacking sign-extends
+ * when fmt.is_signed.  d_codes: fp16 code tensor of n codes (plane-major when fmt.bits > 8), 2-byte
+ * aligned; d_words: ceil(n / 32) * fmt.bits words, 4-byte aligned.  Codes outside fmt's range are
+ * truncated to their low k bits (they cannot come from the quantizer). */
+FXPQ_API fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt fmt, uint32_t* d_words, void* stream);
+FXPQ_API fxpq_status fxpq_unpack_codes(const uint32_t* d_words, int64_t n, fxpq_fmt fmt, void* d_codes,
+                                       void* stream);
+
 /* BN -> Scale preprocessing (Sec. IV-A.1, the BatchNorm rewrite): per channel,
  *   aleph1 = gamma / sqrt(var + eps),  aleph2 = beta - (gamma * mean) / sqrt(var + eps),
  * each operation one correctly rounded fp32 step in that order.  Inputs: fp32 device arrays of n
@@ -334,6 +345,16 @@ typedef struct {
 } fxpq_net;
 
 FXPQ_API size_t fxpq_net_workspace(const fxpq_net* h_net, int32_t batch);
+
+/* Memory requirement of one inference (Sec. V-E.2, Eq. mfp, RW_R and RO_R), a host computation on the
+ * op list: MFP = nu * k / 2^23 MB for nu elements at k bits (k = 32 for every data-structure when
+ * fp32 != 0, the FP32 baseline).  *h_rw_mb = the largest, over ops, of the footprint of the op's input
+ * activations (both operands of an eltwise) plus its output activations, per image, with the true
+ * channel counts (net->C for the input; the last op's output, which has no FxP-QLayer, at 32 bits);
+ * *h_ro_mb = the sum over conv ops of the weights (K*R*S*C), the bias (K, when d_bias) and the Scale
+ * layer's aleph1 and aleph2 (K each, when d_scale) at their formats' bits.  The compression rates are
+ * ratios of the two calls (fp32 = 1 over fp32 = 0).  No device access. */
+FXPQ_API fxpq_status fxpq_net_memory(const fxpq_net* h_net, int32_t fp32, double* h_rw_mb, double* h_ro_mb);
 FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_images_nchw, int32_t batch,
                              int64_t* d_logits, int32_t* h_logits_scale, void* d_ws, size_t ws_bytes,
                              void* stream);

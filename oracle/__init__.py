@@ -21,6 +21,9 @@ Everything here is the paper's definition written out plainly:
   ReLU, then the FxP-QLayer's right shift with round-half-even and clip.
 * MAX-POOL without a QLayer, AVG-POOL with the reciprocal quantized like a
   parameter, Eltwise add with FL alignment (Sec. IV-A.2).
+* Scale layer (BN rewritten as aleph1 * A + aleph2, Sec. IV-A.1) in the C-Block.
+* Memory model MFP / RW_R / RO_R / COMP (Sec. V-E.2) and the packed k-bit code
+  storage whose footprint it counts.
 
 Parity status of every function is pinned by ``tests/test_oracle_pins.py``.
 """
@@ -306,6 +309,68 @@ def to_f32(v, s: int) -> np.ndarray:
     v = np.asarray(v, dtype=np.int64)
     _check_range(v, 53)
     return (v.astype(np.float64) * (2.0 ** -s)).astype(np.float32)
+
+
+# --------------------------------------------------------------------------
+# Memory model and packed code storage (Sec. V-E.2, Eq. mfp, RW_R, RO_R, compression)
+# --------------------------------------------------------------------------
+def mfp(nu: int, k) -> float:
+    """Memory footprint in MB of a data-structure of nu elements at k bits (k = 32 for FP32)."""
+    return nu * k / 2.0 ** 23
+
+
+def rw_r(layers, act_elems, act_bits) -> float:
+    """Read-write requirement: the largest, over layers l, of the footprints of l's input activations
+    (every layer feeding it; the network input for the first) plus l's own output activations.
+    act_elems / act_bits: name -> elements per image / bits ("input" included)."""
+    best = 0.0
+    prev = "input"
+    for L in layers:
+        if L["type"] == "eltwise":
+            inputs = [L["a"], L["b"]]
+        else:
+            inputs = [L.get("src") or prev]
+        v = sum(mfp(act_elems[i], act_bits[i]) for i in inputs) + mfp(act_elems[L["name"]], act_bits[L["name"]])
+        best = max(best, v)
+        prev = L["name"]
+    return best
+
+
+def ro_r(params) -> float:
+    """Read-only requirement: the sum of the footprints of every layer's parameters.
+    params: list of (elements, bits) pairs (weights and biases of each layer with parameters)."""
+    return sum(mfp(nu, k) for nu, k in params)
+
+
+def pack_codes(codes, k: int) -> np.ndarray:
+    """Packed storage of k-bit codes (1 <= k <= 16), k bits per code: the codes are taken in groups of 32
+    (the last group zero-padded) and group g occupies k uint32 words, word g*k + b holding bit b of the
+    k-bit two's-complement field of code 32g + i at bit i."""
+    c = np.asarray(codes, dtype=np.int64).reshape(-1)
+    ng = (c.size + 31) // 32
+    out = np.zeros(ng * k, dtype=np.uint32)
+    for e in range(c.size):
+        field = int(c[e]) & ((1 << k) - 1)
+        g, i = divmod(e, 32)
+        for b in range(k):
+            if (field >> b) & 1:
+                out[g * k + b] |= np.uint32(1 << i)
+    return out
+
+
+def unpack_codes(words, n: int, k: int, S: int) -> np.ndarray:
+    """Inverse of pack_codes: n codes, sign-extended from k bits when S = 1."""
+    w = np.asarray(words, dtype=np.uint32)
+    out = np.zeros(n, dtype=np.int64)
+    for e in range(n):
+        g, i = divmod(e, 32)
+        field = 0
+        for b in range(k):
+            field |= ((int(w[g * k + b]) >> i) & 1) << b
+        if S and field >= 1 << (k - 1):
+            field -= 1 << k
+        out[e] = field
+    return out
 
 
 # --------------------------------------------------------------------------

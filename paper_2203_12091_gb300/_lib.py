@@ -78,6 +78,9 @@ _SIGS = {
     "fxpq_fl_search": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP, SZ, VP]),
     "fxpq_fl_search_noalloc": (I32, [VP, I64, I32, I32, I32, I32, I32, VP, VP, VP, VP]),
     "fxpq_bn_to_scale": (I32, [VP, VP, VP, VP, I64, ctypes.c_float, VP, VP, VP]),
+    "fxpq_pack_codes": (I32, [VP, I64, Fmt, VP, VP]),
+    "fxpq_unpack_codes": (I32, [VP, I64, Fmt, VP, VP]),
+    "fxpq_net_memory": (I32, [ctypes.POINTER(Net), I32, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),
     "fxpq_conv_workspace": (SZ, [ctypes.POINTER(ConvDesc)]),
     "fxpq_conv_fwd": (I32, [ctypes.POINTER(ConvDesc), VP, VP, VP, VP, ctypes.POINTER(I32), VP, SZ, VP]),

@@ -10,6 +10,7 @@ namespace {
 
 struct Slot {
     int H = 0, W = 0, Cp = 0;
+    int C = 0;  // true channel count (Cp without the padding)
     fxpq_fmt fmt{0, 0, 0};
     bool defined = false;
     size_t offset = 0, bytes = 0;
@@ -26,6 +27,7 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
     slots[0].H = net->H;
     slots[0].W = net->W;
     slots[0].Cp = net->Cp_in;
+    slots[0].C = net->C;
     slots[0].fmt = net->fmt_in;
     slots[0].defined = true;
     for (int i = 0; i < net->n_ops; ++i) {
@@ -42,6 +44,7 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
                 out.H = (s0.H + 2 * o.pad - o.R) / o.stride + 1;
                 out.W = (s0.W + 2 * o.pad - o.S) / o.stride + 1;
                 out.Cp = o.K;
+                out.C = o.K;
                 out.fmt = o.fmt_y;
                 if (last) break;
                 if (!fxpq::fmt_ok(o.fmt_y) || (o.K % 8)) return FXPQ_ERR_INVALID_ARG;
@@ -52,6 +55,7 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
                 out.H = (s0.H + 2 * o.pad - o.R) / o.stride + 1;
                 out.W = (s0.W + 2 * o.pad - o.R) / o.stride + 1;
                 out.Cp = s0.Cp;
+                out.C = s0.C;
                 out.fmt = s0.fmt;
                 break;
             case FXPQ_OP_ELTWISE: {
@@ -65,6 +69,7 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
             case FXPQ_OP_AVGPOOL:
                 out.H = out.W = 1;
                 out.Cp = s0.Cp;
+                out.C = s0.C;
                 out.fmt = o.fmt_y;
                 break;
             default:
@@ -89,6 +94,40 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
 }
 
 }  // namespace
+
+extern "C" fxpq_status fxpq_net_memory(const fxpq_net* h_net, int32_t fp32, double* h_rw_mb, double* h_ro_mb) {
+    std::vector<Slot> slots;
+    size_t total = 0;
+    fxpq_status st = plan_net(h_net, 0, slots, total);
+    if (st != FXPQ_OK) return st;
+    if (!h_rw_mb || !h_ro_mb) return FXPQ_ERR_INVALID_ARG;
+    // MFP(d) = nu * k / 2^23 MB, k = 32 for FP32
+    auto mfp = [fp32](double nu, int bits) { return nu * (fp32 ? 32 : bits) / 8388608.0; };
+    auto act = [&](const Slot& s) { return mfp((double)s.H * s.W * s.C, s.fmt.bits); };
+    double rw = 0.0, ro = 0.0;
+    for (int i = 0; i < h_net->n_ops; ++i) {
+        const fxpq_op_desc& o = h_net->ops[i];
+        const Slot& s0 = slots[o.src0];
+        double in = act(s0);
+        if (o.op == FXPQ_OP_ELTWISE) in += act(slots[o.src1]);
+        double out;
+        if (o.last) {
+            const int P = (s0.H + 2 * o.pad - o.R) / o.stride + 1, Q = (s0.W + 2 * o.pad - o.S) / o.stride + 1;
+            out = (double)P * Q * o.K * 32 / 8388608.0;  // the last layer has no FxP-QLayer
+        } else {
+            out = act(slots[o.dst]);
+        }
+        if (in + out > rw) rw = in + out;
+        if (o.op == FXPQ_OP_CONV) {
+            ro += mfp((double)o.K * o.R * o.S * s0.C, o.fmt_w.bits);
+            if (o.d_bias) ro += mfp(o.K, o.fmt_b.bits);
+            if (o.d_scale) ro += mfp(o.K, o.fmt_scale.bits) + mfp(o.K, o.fmt_shift.bits);
+        }
+    }
+    *h_rw_mb = rw;
+    *h_ro_mb = ro;
+    return FXPQ_OK;
+}
 
 extern "C" size_t fxpq_net_workspace(const fxpq_net* h_net, int32_t batch) {
     std::vector<Slot> slots;

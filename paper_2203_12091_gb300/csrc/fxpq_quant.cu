@@ -53,6 +53,46 @@ __global__ void quantize_vec4_kernel(const float4* __restrict__ x, long long n4,
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
 
+// Storage bits of one code: the integer itself, or (F16) the bit pattern of its fp16 value.
+template <typename S, bool F16>
+__device__ __forceinline__ S code_bits(int c) {
+    if (F16) return (S)__half_as_ushort(__int2half_rn(c));
+    return (S)c;
+}
+
+// Flat quantization, 16 codes per thread and iteration: four 16-byte loads issued together, the
+// codes packed into sizeof(S) 16-byte stores.  x and out 16-byte aligned; the n % 16 tail is done
+// element by element by the first threads of the grid.
+template <typename S, bool F16>
+__global__ void quantize_vec16_kernel(const float* __restrict__ x, long long n, QParams p, S* __restrict__ out) {
+    bool bad = false;
+    const long long n16 = n / 16;
+    const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    const float4* x4 = reinterpret_cast<const float4*>(x);
+    uint4* o4 = reinterpret_cast<uint4*>(out);
+    for (long long i = tid; i < n16; i += stride) {
+        float4 v[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v[j] = __ldg(x4 + 4 * i + j);
+        union {
+            S s[16];
+            uint4 u[sizeof(S)];
+        } pk;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            pk.s[4 * j + 0] = code_bits<S, F16>(quant1(v[j].x, p, bad));
+            pk.s[4 * j + 1] = code_bits<S, F16>(quant1(v[j].y, p, bad));
+            pk.s[4 * j + 2] = code_bits<S, F16>(quant1(v[j].z, p, bad));
+            pk.s[4 * j + 3] = code_bits<S, F16>(quant1(v[j].w, p, bad));
+        }
+#pragma unroll
+        for (int q = 0; q < (int)sizeof(S); ++q) o4[sizeof(S) * i + q] = pk.u[q];
+    }
+    for (long long i = 16 * n16 + tid; i < n; i += stride) out[i] = code_bits<S, F16>(quant1(__ldg(x + i), p, bad));
+    if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
+}
+
 // rows x C fp32 -> fp16 code tensor: planes of [rows, Cp] (hi plane, then lo plane when k > 8)
 __global__ void quantize_rows_f16_kernel(const float* __restrict__ x, long long rows, int C, int Cp, int planes,
                                          QParams p, __half* __restrict__ out) {
@@ -274,7 +314,68 @@ __global__ void __launch_bounds__(256) quantize_batch_kernel(const __grid_consta
     if (bad) latch_status(p.status, FXPQ_ERR_NONFINITE);
 }
 
+// ------------------------------------------------------------------------------------------
+// Packed k-bit code storage: bit-plane words per group of 32 codes (see fxpq_pack_codes)
+// ------------------------------------------------------------------------------------------
+constexpr int PACK_G = 4;  // groups per warp and iteration (their code loads are issued together)
+
+__global__ void pack_codes_kernel(const __half* __restrict__ codes, long long n, int k, int planes,
+                                  uint32_t* __restrict__ words) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const long long ng = (n + 31) / 32;
+    const uint32_t mask = (1u << k) - 1;
+    for (long long g0 = warp * PACK_G; g0 < ng; g0 += nwarps * PACK_G) {
+        uint32_t f[PACK_G];
+#pragma unroll
+        for (int j = 0; j < PACK_G; ++j) {
+            const long long e = (g0 + j) * 32 + lane;
+            f[j] = e < n ? (uint32_t)code_get(codes, e, planes, n) & mask : 0u;
+        }
+#pragma unroll
+        for (int j = 0; j < PACK_G; ++j) {
+            if (g0 + j >= ng) break;
+            uint32_t mine = 0;
+#pragma unroll
+            for (int b = 0; b < 16; ++b) {
+                if (b >= k) break;
+                const uint32_t w = __ballot_sync(0xffffffffu, (f[j] >> b) & 1u);
+                if (lane == b) mine = w;
+            }
+            if (lane < k) words[(g0 + j) * k + lane] = mine;
+        }
+    }
+}
+
+__global__ void unpack_codes_kernel(const uint32_t* __restrict__ words, long long n, int k, int is_signed,
+                                    int planes, __half* __restrict__ codes) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const long long ng = (n + 31) / 32;
+    for (long long g0 = warp * PACK_G; g0 < ng; g0 += nwarps * PACK_G) {
+        uint32_t w[PACK_G];
+#pragma unroll
+        for (int j = 0; j < PACK_G; ++j) w[j] = (g0 + j < ng && lane < k) ? __ldg(words + (g0 + j) * k + lane) : 0u;
+#pragma unroll
+        for (int j = 0; j < PACK_G; ++j) {
+            if (g0 + j >= ng) break;
+            int field = 0;
+#pragma unroll
+            for (int b = 0; b < 16; ++b) {
+                if (b >= k) break;
+                field |= (int)((__shfl_sync(0xffffffffu, w[j], b) >> lane) & 1u) << b;
+            }
+            if (is_signed && (field >> (k - 1))) field -= 1 << k;  // sign extension of the k-bit field
+            const long long e = (g0 + j) * 32 + lane;
+            if (e < n) code_put(codes, e, planes, n, field);
+        }
+    }
+}
+
 }  // namespace
+
 
 static QParams make_qparams(const fxpq_fmt& f) {
     QParams p;
@@ -313,10 +414,39 @@ extern "C" fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, in
     cudaStream_t s = as_stream(stream);
     QParams p = make_qparams(f);
     const int T = 256;
+    const bool al16 = aligned(d_x, 16) && aligned(d_codes, 16);
     if (dtype == FXPQ_DT_F16) {
-        quantize_rows_f16_kernel<<<grid_for(n, T), T, 0, s>>>(d_x, 1, (int)n, (int)n, planes_of(f), p,
+        if (planes_of(f) == 1 && al16) {
+            quantize_vec16_kernel<uint16_t, true><<<grid_for((n + 15) / 16, T), T, 0, s>>>(
+                d_x, n, p, static_cast<uint16_t*>(d_codes));
+            return after_launch("quantize_f16");
+        }
+        if (al16 && n % 8 == 0) {
+            quantize_rows_vec8_kernel<<<grid_for(n / 8, T), T, 0, s>>>(reinterpret_cast<const float4*>(d_x), n / 8,
+                                                                      planes_of(f), p, static_cast<uint4*>(d_codes));
+            return after_launch("quantize_rows_vec8");
+        }
+        // unaligned: one code per row of one channel
+        quantize_rows_f16_kernel<<<grid_for(n, T), T, 0, s>>>(d_x, n, 1, 1, planes_of(f), p,
                                                               static_cast<__half*>(d_codes));
         return after_launch("quantize_rows_f16");
+    }
+    if (al16) {
+        const int g = grid_for((n + 15) / 16, T);
+        switch (dtype) {
+            case FXPQ_DT_I8:
+            case FXPQ_DT_U8:
+                quantize_vec16_kernel<uint8_t, false><<<g, T, 0, s>>>(d_x, n, p, static_cast<uint8_t*>(d_codes));
+                break;
+            case FXPQ_DT_I16:
+            case FXPQ_DT_U16:
+                quantize_vec16_kernel<uint16_t, false><<<g, T, 0, s>>>(d_x, n, p, static_cast<uint16_t*>(d_codes));
+                break;
+            default:
+                quantize_vec16_kernel<uint32_t, false><<<g, T, 0, s>>>(d_x, n, p, static_cast<uint32_t*>(d_codes));
+                break;
+        }
+        return after_launch("quantize_vec16");
     }
     bool vec = aligned(d_x, 16) && (n % 4 == 0);
 #define FXPQ_Q_LAUNCH(TYPE)                                                                                       \
@@ -428,4 +558,28 @@ extern "C" fxpq_status fxpq_quantize_batch(const fxpq_quantize_item* h_items, in
         if (st != FXPQ_OK) return st;
     }
     return FXPQ_OK;
+}
+
+extern "C" fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt fmt, uint32_t* d_words,
+                                       void* stream) {
+    if (n < 0 || !fmt_ok(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
+        return FXPQ_ERR_INVALID_ARG;
+    if (n == 0) return FXPQ_OK;
+    const long long ng = (n + 31) / 32;
+    const int T = 256;
+    pack_codes_kernel<<<grid_for((ng + PACK_G - 1) / PACK_G * 32, T), T, 0, as_stream(stream)>>>(
+        static_cast<const __half*>(d_codes), n, fmt.bits, planes_of(fmt), d_words);
+    return after_launch("pack_codes");
+}
+
+extern "C" fxpq_status fxpq_unpack_codes(const uint32_t* d_words, int64_t n, fxpq_fmt fmt, void* d_codes,
+                                         void* stream) {
+    if (n < 0 || !fmt_ok(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
+        return FXPQ_ERR_INVALID_ARG;
+    if (n == 0) return FXPQ_OK;
+    const long long ng = (n + 31) / 32;
+    const int T = 256;
+    unpack_codes_kernel<<<grid_for((ng + PACK_G - 1) / PACK_G * 32, T), T, 0, as_stream(stream)>>>(
+        d_words, n, fmt.bits, fmt.is_signed, planes_of(fmt), static_cast<__half*>(d_codes));
+    return after_launch("unpack_codes");
 }

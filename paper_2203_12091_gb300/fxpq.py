@@ -132,6 +132,28 @@ def fxpq_fl_init(stats: Stats, bits: int, strategy: int) -> Fmt:
     return out
 
 
+def fxpq_pack_codes(codes, n: int, f: Fmt, words, stream=None):
+    """fp16 code tensor of n codes -> packed k-bit words (ceil(n / 32) * f.bits uint32)."""
+    L.check("fxpq_pack_codes", L.lib().fxpq_pack_codes(_p(codes), n, f, _p(words), _s(stream)))
+    return words
+
+
+def fxpq_unpack_codes(words, n: int, f: Fmt, codes, stream=None):
+    L.check("fxpq_unpack_codes", L.lib().fxpq_unpack_codes(_p(words), n, f, _p(codes), _s(stream)))
+    return codes
+
+
+def packed_words(n: int, f: Fmt) -> int:
+    return (n + 31) // 32 * f.bits
+
+
+def fxpq_net_memory(net, fp32: bool):
+    """(RW_R, RO_R) in MB of one inference of the op list (Sec. V-E.2); host-only."""
+    rw, ro = ctypes.c_double(0), ctypes.c_double(0)
+    L.check("fxpq_net_memory", L.lib().fxpq_net_memory(ctypes.byref(net), int(fp32), ctypes.byref(rw), ctypes.byref(ro)))
+    return rw.value, ro.value
+
+
 def fxpq_bn_to_scale(gamma, beta, mean, var, eps, aleph1, aleph2, stream=None):
     """BN -> Scale layer parameters (fp32 device tensors of one length)."""
     L.check("fxpq_bn_to_scale", L.lib().fxpq_bn_to_scale(_p(gamma), _p(beta), _p(mean), _p(var), gamma.numel(),

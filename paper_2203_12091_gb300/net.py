@@ -304,6 +304,14 @@ class QNet:
                          self.fmts["input"]["a"], ctypes.cast(ops, ctypes.POINTER(L.OpDesc)))
         self.n_classes = self.layers[-1]["K"]
 
+    def memory(self):
+        """Memory requirement of one inference (Sec. V-E.2): RW_R / RO_R in MB for the FxP network and
+        its FP32 baseline, and the compression rates COMP_Act and COMP_Model."""
+        rw_q, ro_q = F.fxpq_net_memory(self.net, False)
+        rw_f, ro_f = F.fxpq_net_memory(self.net, True)
+        return {"rw_mb": rw_q, "ro_mb": ro_q, "rw_fp32_mb": rw_f, "ro_fp32_mb": ro_f,
+                "comp_act": rw_f / rw_q, "comp_model": ro_f / ro_q}
+
     def workspace_bytes(self, batch: int) -> int:
         return F.fxpq_net_workspace(self.net, batch)
 

@@ -137,3 +137,52 @@ def test_struct_layout_matches_header(tmp_path):
         assert got[(cname, "sizeof")] == ctypes.sizeof(py), cname
         for f, _ in py._fields_:
             assert got[(cname, f)] == getattr(py, f).offset, (cname, f)
+
+
+@pytest.mark.parametrize("arch", ["vgg16", "resnet18_bn", "alexnet"])
+def test_net_memory_matches_oracle(lib, arch):
+    """fxpq_net_memory (host-only) against the oracle's RW_R / RO_R on a workload's bit plan."""
+    import torch
+    import synth
+    from paper_2203_12091_gb300 import fxpq as F
+    from paper_2203_12091_gb300.net import QNet
+    layers = synth.ARCHS[arch]()
+    plan = synth.bit_plan(arch, 3)
+    q = QNet(layers)
+    dummy = torch.zeros(8)
+    q.fmts["input"] = {"a": F.fmt(plan["input"], 1, 0)}
+    bits = {"input": plan["input"]}
+    params = []
+    prev = "input"
+    for i, Lr in enumerate(layers):
+        nm = Lr["name"]
+        p = plan.get(nm, {})
+        f = q.fmts.setdefault(nm, {})
+        last = i == len(layers) - 1
+        if "a" in p:
+            f["a"] = F.fmt(p["a"], 1, 0)
+        if Lr["type"] == "conv":
+            f["w"] = F.fmt(p["w"], 1, 0)
+            params.append((Lr["K"] * Lr["R"] * Lr["R"] * Lr["C"], p["w"]))
+            if "b" in p:
+                f["b"] = F.fmt(p["b"], 1, 0)
+                params.append((Lr["K"], p["b"]))
+            q.q[nm] = (dummy, dummy if "b" in p else None)
+            if Lr.get("bn"):
+                f["s"], f["h"] = F.fmt(p["s"], 1, 0), F.fmt(p["h"], 1, 0)
+                q.qs[nm] = (dummy, dummy)
+                params += [(Lr["K"], p["s"]), (Lr["K"], p["h"])]
+        elif Lr["type"] == "avgpool":
+            f["r"] = F.fmt(p["r"], 0, 0)
+            q.q[nm] = (None, 1)
+        bits[nm] = 32 if last else (bits[Lr.get("src") or prev] if Lr["type"] == "maxpool" else p["a"])
+        prev = nm
+    q._build_ops()
+    rw, ro = F.fxpq_net_memory(q.net, False)
+    rw32, ro32 = F.fxpq_net_memory(q.net, True)
+    from tests.test_oracle_pins import _act_elems
+    elems = _act_elems(layers)
+    assert rw == pytest.approx(oracle.rw_r(layers, elems, bits), rel=1e-12)
+    assert ro == pytest.approx(oracle.ro_r(params), rel=1e-12)
+    assert rw32 == pytest.approx(oracle.rw_r(layers, elems, {nm: 32 for nm in bits}), rel=1e-12)
+    assert ro32 == pytest.approx(oracle.ro_r([(n, 32) for n, _ in params]), rel=1e-12)

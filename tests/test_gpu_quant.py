@@ -52,6 +52,23 @@ def test_quantize_parity(F, n, k, S, fl, dt):
     assert np.array_equal(out.cpu().numpy()[:n].astype(np.int64), want)
 
 
+@pytest.mark.parametrize("n", [0, 5, 4097, 1 << 20])
+@pytest.mark.parametrize("k,S,fl", [(8, 1, 5), (6, 0, 2), (12, 1, 9), (16, 0, 14)])
+@pytest.mark.parametrize("offset", [0, 1])
+def test_quantize_f16_flat(F, n, k, S, fl, offset):
+    """fxpq_quantize to an fp16 code tensor (plane-major when k > 8), 16-byte aligned (vector path) and
+    4-byte aligned (scalar path)."""
+    x = _adv(n + k + 100, max(n + offset, 1))
+    xd = torch.from_numpy(x).cuda()[offset:offset + n]
+    f = F.fmt(k, S, fl)
+    out = torch.empty(max(n, 1) * F.planes(f), dtype=torch.float16, device="cuda")
+    F.fxpq_quantize(xd, f, F.DT_F16, out)
+    torch.cuda.synchronize()
+    want = oracle.quantize(x[offset:offset + n], k, S, fl)
+    got = F.codes_to_int(out[: n * F.planes(f)].cpu(), f, (n,)).numpy()
+    assert np.array_equal(got, want)
+
+
 def test_quantize_unaligned_and_nonfinite(F):
     x = _adv(5, 999)
     xd = torch.from_numpy(x).cuda()
@@ -246,3 +263,51 @@ def test_quantize_batch_device_formats(F):
                 assert l1h[i] == np.abs(want).reshape(K, -1).sum(axis=1).max()
         else:
             assert np.array_equal(out.cpu().numpy(), want)
+
+
+def _f16_codes(c, k):
+    """fp16 code tensor of a flat code array (plane-major hi / lo limbs when k > 8)."""
+    c = np.asarray(c, dtype=np.int64)
+    if k <= 8:
+        return torch.from_numpy(c.astype(np.float16)).cuda()
+    hi = c >> 8
+    return torch.from_numpy(np.concatenate([hi, c - (hi << 8)]).astype(np.float16)).cuda()
+
+
+@pytest.mark.parametrize("k,S", [(2, 1), (3, 0), (4, 1), (5, 1), (8, 0), (8, 1), (11, 1), (16, 0), (16, 1)])
+@pytest.mark.parametrize("n", [0, 1, 31, 33, 1000])
+def test_pack_unpack_parity(F, k, S, n):
+    """fxpq_pack_codes word for word against the oracle's packed layout; fxpq_unpack_codes restores the
+    codes (sign-extended when S = 1)."""
+    rng = np.random.default_rng(k * 100 + n + S)
+    c = rng.integers(oracle.qmin(k, S), oracle.qmax(k, S) + 1, size=n)
+    c[: min(2, n)] = [oracle.qmin(k, S), oracle.qmax(k, S)][: min(2, n)]
+    f = F.fmt(k, S, 0)
+    nw = F.packed_words(n, f)
+    words = torch.full((max(nw, 1),), 0x5A5A5A5A, dtype=torch.int32, device="cuda")
+    F.fxpq_pack_codes(_f16_codes(c, k) if n else torch.empty(1, dtype=torch.float16, device="cuda"), n, f, words)
+    torch.cuda.synchronize()
+    got = words.cpu().numpy().view(np.uint32)[:nw]
+    assert np.array_equal(got, oracle.pack_codes(c, k))
+    out = torch.empty(max(n, 1) * F.planes(f), dtype=torch.float16, device="cuda")
+    F.fxpq_unpack_codes(words, n, f, out)
+    assert np.array_equal(F.codes_to_int(out[: n * F.planes(f)].cpu(), f, (n,)).numpy(), c)
+
+
+@pytest.mark.parametrize("k,S", [(4, 1), (12, 1)])
+def test_pack_unpack_large_sampled(F, k, S):
+    """64M + 5 codes: the round trip is exact everywhere and sampled groups match the oracle's words."""
+    n = (1 << 26) + 5
+    rng = np.random.default_rng(k)
+    c = rng.integers(oracle.qmin(k, S), oracle.qmax(k, S) + 1, size=n)
+    f = F.fmt(k, S, 0)
+    words = torch.empty(F.packed_words(n, f), dtype=torch.int32, device="cuda")
+    F.fxpq_pack_codes(_f16_codes(c, k), n, f, words)
+    out = torch.empty(n * F.planes(f), dtype=torch.float16, device="cuda")
+    F.fxpq_unpack_codes(words, n, f, out)
+    assert np.array_equal(F.codes_to_int(out.cpu(), f, (n,)).numpy(), c)
+    w = words.cpu().numpy().view(np.uint32)
+    ng = (n + 31) // 32
+    for g in list(rng.integers(0, ng, size=40)) + [ng - 1]:
+        seg = c[32 * g: 32 * g + 32]
+        assert np.array_equal(w[g * k:(g + 1) * k], oracle.pack_codes(seg, k)), g

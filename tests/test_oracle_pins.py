@@ -486,3 +486,79 @@ def test_scale_layer_gain_applies_before_relu_and_requant():
     v, s = oracle.cblock(acc, 10, None, 0, True, scale=np.full(4, -1), fl_scale=0, shift=np.zeros(4, np.int64),
                          fl_shift=0)
     assert s == 10 and np.array_equal(v, np.maximum(-acc, 0))
+
+
+def test_memory_footprint_closed_forms():
+    """Eq. mfp: nu * k / 2^23 MB, so 2^20 8-bit codes are exactly 1 MB and FP32 over k bits is 32 / k."""
+    assert oracle.mfp(2 ** 20, 8) == 1.0
+    assert oracle.mfp(2 ** 23, 1) == 1.0
+    for k in range(2, 17):
+        assert oracle.mfp(12345, 32) / oracle.mfp(12345, k) == pytest.approx(32 / k, rel=1e-15)
+
+
+def _act_elems(layers, hw=224, cin=3):
+    """Output elements per image of every layer (true channels), by plain shape propagation."""
+    shapes = {"input": (hw, cin)}
+    prev = "input"
+    for L in layers:
+        src = L.get("src") or prev
+        h, c = shapes[L["a"] if L["type"] == "eltwise" else src]
+        if L["type"] == "conv":
+            shapes[L["name"]] = ((h + 2 * L["pad"] - L["R"]) // L["stride"] + 1, L["K"])
+        elif L["type"] == "maxpool":
+            shapes[L["name"]] = ((h + 2 * L["pad"] - L["k"]) // L["stride"] + 1, c)
+        elif L["type"] == "avgpool":
+            shapes[L["name"]] = (1, c)
+        else:
+            shapes[L["name"]] = (h, c)
+        prev = L["name"]
+    return {nm: h * h * c for nm, (h, c) in shapes.items()}
+
+
+def test_memory_model_vgg16_fp32_textbook_figures():
+    """VGG-16 in FP32: RO_R is its textbook 138,357,544 parameters at 32 bits; RW_R is conv1_2's input
+    plus output (two 224 x 224 x 64 maps), the largest pair of any layer."""
+    layers = synth.vgg16()
+    elems = _act_elems(layers)
+    rw = oracle.rw_r(layers, elems, {nm: 32 for nm in elems})
+    assert rw == pytest.approx(2 * 224 * 224 * 64 * 32 / 2 ** 23, rel=1e-15)
+    params = []
+    for L in layers:
+        if L["type"] == "conv":
+            params += [(L["K"] * L["R"] * L["R"] * L["C"], 32), (L["K"], 32)]
+    assert sum(n for n, _ in params) == 138357544
+    assert oracle.ro_r(params) == pytest.approx(138357544 * 32 / 2 ** 23, rel=1e-15)
+
+
+def test_memory_model_resnet18_residual_inputs():
+    """ResNet-18: an eltwise layer reads both its operands (Sec. V-E.2); in FP32 the largest read-write pair
+    is pool1 (conv1's 112 x 112 x 64 output in, 56 x 56 x 64 out), above any residual add's three maps."""
+    layers = synth.resnet18()
+    elems = _act_elems(layers)
+    bits = {nm: 32 for nm in elems}
+    assert oracle.rw_r(layers, elems, bits) == pytest.approx((112 * 112 * 64 + 56 * 56 * 64) * 32 / 2 ** 23)
+    # an eltwise alone: its two inputs and its output
+    one = [L for L in layers if L["name"] == "res1a"]
+    assert oracle.rw_r(one, elems, bits) == pytest.approx(3 * 56 * 56 * 64 * 32 / 2 ** 23)
+
+
+def test_pack_codes_worked_example_and_round_trip():
+    """Packed k-bit storage: signed 3-bit codes (1, -1, 2) are the fields 001, 111, 010, so the bit-0 word
+    is 0b011 = 3, the bit-1 word 0b110 = 6 and the bit-2 word 0b010 = 2; every code of every format
+    survives the round trip, and the footprint is ceil(n / 32) * k words."""
+    w = oracle.pack_codes([1, -1, 2], 3)
+    assert w.tolist() == [3, 6, 2]
+    assert oracle.unpack_codes(w, 3, 3, 1).tolist() == [1, -1, 2]
+    rng = np.random.default_rng(41)
+    for k in (2, 3, 5, 8, 11, 16):
+        for S in (0, 1):
+            n = 70
+            c = rng.integers(oracle.qmin(k, S), oracle.qmax(k, S) + 1, size=n)
+            c[:2] = [oracle.qmin(k, S), oracle.qmax(k, S)]
+            words = oracle.pack_codes(c, k)
+            assert words.size == 3 * k
+            assert np.array_equal(oracle.unpack_codes(words, n, k, S), c)
+            # bit b of the stream counts the codes whose field has bit b set
+            for b in range(k):
+                ones = sum(bin(int(x)).count("1") for x in words[b::k])
+                assert ones == sum(((int(v) & ((1 << k) - 1)) >> b) & 1 for v in c)
