@@ -68,7 +68,9 @@ def _L():
         lib.ora_l2_error.restype = ctypes.c_double
         lib.ora_exact_sum.argtypes = [f64p, L]
         lib.ora_exact_sum.restype = ctypes.c_double
-        lib.ora_fl_search.argtypes = [f32p, L, I, I, I, I, I, f64p, i32p, f64p]
+        lib.ora_l1_error.argtypes = [f32p, L, I, I, I]
+        lib.ora_l1_error.restype = ctypes.c_double
+        lib.ora_fl_search.argtypes = [f32p, L, I, I, I, I, I, f64p, i32p, f64p, I]
         lib.ora_fl_search.restype = I
         lib.ora_conv2d.argtypes = [i32p, I, I, I, I, i32p, I, I, I, I, I, I, I, i64p]
         lib.ora_conv2d.restype = None
@@ -94,11 +96,21 @@ def qmax(k: int, S: int) -> int:
 
 
 def quantize(x, k: int, S: int, fl: int) -> np.ndarray:
-    """Eq. (fp_k_bit_quantization): codes of fp32 ``x`` in S(alpha, FL) / U(alpha, FL), k = alpha + FL."""
+    """Eq. (fp_k_bit_quantization): codes of fp32 ``x`` in S(alpha, FL) / U(alpha, FL), k = alpha + FL.
+    k = 1 with S = 1 is the binary quantizer of Eq. (fp_1_bit_quantization): -1 for x < 0, else 0."""
     x = np.ascontiguousarray(x, dtype=np.float32).reshape(-1)
     out = np.empty(x.size, dtype=np.int32)
     _L().ora_quantize(_p(x, ctypes.c_float), x.size, k, S, fl, _p(out, ctypes.c_int32))
     return out.astype(np.int64)
+
+
+def value(codes, k: int, S: int, fl: int) -> np.ndarray:
+    """The values codes stand for (fp64, exact): code * 2^-FL, or for the binary quantizer (k = 1,
+    S = 1) the decoded sign, 0 -> +1 and -1 -> -1, times 2^-FL (Eq. fp_1_bit_quantization)."""
+    c = np.asarray(codes, dtype=np.int64)
+    if k == 1 and S == 1:
+        c = 2 * c + 1
+    return np.ldexp(c.astype(np.float64), -fl)
 
 
 def l2_error(x, k: int, S: int, fl: int) -> float:
@@ -107,13 +119,20 @@ def l2_error(x, k: int, S: int, fl: int) -> float:
     return float(_L().ora_l2_error(_p(x, ctypes.c_float), x.size, k, S, fl))
 
 
+def l1_error(x, k: int, S: int, fl: int) -> float:
+    """Eq. (MAE) as a sum: sum |X - X~| (the MAE is this over N), exact sum rounded once."""
+    x = np.ascontiguousarray(x, dtype=np.float32).reshape(-1)
+    return float(_L().ora_l1_error(_p(x, ctypes.c_float), x.size, k, S, fl))
+
+
 def exact_sum(v) -> float:
     v = np.ascontiguousarray(v, dtype=np.float64).reshape(-1)
     return float(_L().ora_exact_sum(_p(v, ctypes.c_double), v.size))
 
 
-def fl_search(x, S: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int):
-    """Score every (k, FL) candidate by Eq. (DSB_QE); argmin FL per k (ties -> smallest FL).
+def fl_search(x, S: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, score: str = "l2"):
+    """Score every (k, FL) candidate by Eq. (DSB_QE) (score "l2") or by the L1 error of Eq. (MAE) as a
+    sum (score "l1"); argmin FL per k (ties -> smallest FL).
 
     S = -1 selects the sign strategy of Sec. IV-A.3 (S = 1 iff min(X) < 0).
     Returns (err[nk, nfl] float64, best_fl[nk] int32, S_used, stats dict).
@@ -124,7 +143,8 @@ def fl_search(x, S: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int):
     best = np.empty(nk, dtype=np.int32)
     st = np.empty(4, dtype=np.float64)
     s_used = _L().ora_fl_search(_p(x, ctypes.c_float), x.size, S, k_lo, k_hi, fl_lo, fl_hi,
-                                _p(err, ctypes.c_double), _p(best, ctypes.c_int32), _p(st, ctypes.c_double))
+                                _p(err, ctypes.c_double), _p(best, ctypes.c_int32), _p(st, ctypes.c_double),
+                                {"l2": 0, "l1": 1}[score])
     stats = {"min": st[0], "max": st[1], "sum": st[2], "sumsq": st[3], "n": x.size}
     return err.reshape(nk, nfl), best, int(s_used), stats
 

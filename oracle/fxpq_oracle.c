@@ -141,14 +141,23 @@ static double round_half_even(double y) {
     return (fmod(f, 2.0) == 0.0) ? f : f + 1.0;
 }
 
-/* Eq. (fp_k_bit_quantization) + Eq. (clip) for one element */
+/* Eq. (fp_k_bit_quantization) + Eq. (clip) for one element; a signed 1-bit data-structure takes the
+ * binary quantizer of Eq. (fp_1_bit_quantization): -1 for x < 0, 0 otherwise */
 static int64_t ora_q1(float x, int k, int S, int beta) {
+    if (k == 1 && S == 1) return x < 0.0f ? -1 : 0;
     double y = ldexp((double)x, beta); /* exact in double */
     double m = round_half_even(y);
     double lo = (double)ora_qmin(k, S), hi = (double)ora_qmax(k, S);
     if (m < lo) m = lo;
     if (m > hi) m = hi;
     return (int64_t)m;
+}
+
+/* the value a code stands for: code * 2^-beta, or for the binary quantizer the decoded sign
+ * (0 -> +1, -1 -> -1) times 2^-beta */
+static double ora_value(int64_t code, int k, int S, int beta) {
+    if (k == 1 && S == 1) return ldexp((double)(2 * code + 1), -beta);
+    return ldexp((double)code, -beta);
 }
 
 void ora_quantize(const float* x, int64_t n, int k, int S, int beta, int32_t* codes) {
@@ -161,10 +170,29 @@ double ora_l2_error(const float* x, int64_t n, int k, int S, int beta) {
     ka_zero(&acc);
     for (int64_t i = 0; i < n; ++i) {
         double xi = (double)x[i];
-        double c = ldexp((double)ora_q1(x[i], k, S, beta), -beta); /* value of the code */
+        double c = ora_value(ora_q1(x[i], k, S, beta), k, S, beta); /* value of the code */
         ka_add(&acc, xi * xi);        /* exact: 48-bit product        */
         ka_add(&acc, -2.0 * xi * c);  /* exact: 24 x 17-bit product   */
         ka_add(&acc, c * c);          /* exact: 17 x 17-bit product   */
+    }
+    return ka_to_double(&acc);
+}
+
+/* Eq. (MAE) without the 1/N: sum_i |x_i - value_i|, exact then rounded once.  Both x_i and the value
+ * are exact doubles, so the sign of each difference is decided exactly and each is added with it. */
+double ora_l1_error(const float* x, int64_t n, int k, int S, int beta) {
+    ka_t acc;
+    ka_zero(&acc);
+    for (int64_t i = 0; i < n; ++i) {
+        double xi = (double)x[i];
+        double c = ora_value(ora_q1(x[i], k, S, beta), k, S, beta);
+        if (xi >= c) {
+            ka_add(&acc, xi);
+            ka_add(&acc, -c);
+        } else {
+            ka_add(&acc, c);
+            ka_add(&acc, -xi);
+        }
     }
     return ka_to_double(&acc);
 }
@@ -181,14 +209,15 @@ double ora_exact_sum(const double* v, int64_t n) {
 /*
  * FL search over a grid of candidates: for every wordlength k in [k_lo,k_hi]
  * and fractional length beta in [fl_lo, fl_hi], L(X; k, beta, S) by
- * Eq. (DSB_QE); best[k] = the beta with the smallest L, exact ties going to
+ * Eq. (DSB_QE) (score 0) or the L1 error of Eq. (MAE) as a sum (score 1); best[k] = the beta with the
+ * smallest score, exact ties going to
  * the smallest beta.  err is row-major [k][beta].
  * S = -1 picks the sign strategy by Sec. IV-A.3: S = 1 iff min(X) < 0.
  * stats = {min, max, sum, sumsq} (sum and sumsq exact, rounded once).
  * Returns the S used.
  */
 int ora_fl_search(const float* x, int64_t n, int S, int k_lo, int k_hi, int fl_lo, int fl_hi,
-                  double* err, int32_t* best, double* stats) {
+                  double* err, int32_t* best, double* stats, int score) {
     float mn = INFINITY, mx = -INFINITY;
     ka_t s1, s2;
     ka_zero(&s1);
@@ -206,7 +235,8 @@ int ora_fl_search(const float* x, int64_t n, int S, int k_lo, int k_hi, int fl_l
     /* every candidate is scored independently (OpenMP only spreads the candidates) */
 #pragma omp parallel for schedule(dynamic, 1)
     for (int c = 0; c < nk * nfl; ++c)
-        err[c] = ora_l2_error(x, n, k_lo + c / nfl, S, fl_lo + c % nfl);
+        err[c] = score == 1 ? ora_l1_error(x, n, k_lo + c / nfl, S, fl_lo + c % nfl)
+                            : ora_l2_error(x, n, k_lo + c / nfl, S, fl_lo + c % nfl);
     for (int k = k_lo; k <= k_hi; ++k) {
         double bestv = INFINITY;
         int bestfl = fl_lo;

@@ -562,3 +562,61 @@ def test_pack_codes_worked_example_and_round_trip():
             for b in range(k):
                 ones = sum(bin(int(x)).count("1") for x in words[b::k])
                 assert ones == sum(((int(v) & ((1 << k) - 1)) >> b) & 1 for v in c)
+
+
+# ---------------------------------------------------------------- score variants: binary quantizer, L1
+def frac_val(x, k, S, fl):
+    """Exact value of Q(x): code * 2^-FL, or for the signed 1-bit binary quantizer the decoded sign."""
+    if k == 1 and S == 1:
+        return (Fraction(-1) if F(x) < 0 else Fraction(1)) * Fraction(2) ** (-fl)
+    return Fraction(frac_q(x, k, S, fl)) * Fraction(2) ** (-fl)
+
+
+def test_binary_quantizer_worked_example():
+    """Eq. fp_1_bit_quantization: -1 for x < 0, 0 for x >= 0 (-0.0 included); decoded 0 -> +1, so the values
+    are +-2^-FL and the L2 / L1 errors are sums of (|x| - 2^-FL)^2 / ||x| - 2^-FL|."""
+    x = np.array([-0.5, -0.0, 0.0, 3.0, -1e-30, 0.25], np.float32)
+    assert oracle.quantize(x, 1, 1, 2).tolist() == [-1, 0, 0, 0, -1, 0]
+    assert oracle.value(oracle.quantize(x, 1, 1, 2), 1, 1, 2).tolist() == [-0.25, 0.25, 0.25, 0.25, -0.25, 0.25]
+    c = Fraction(1, 4)
+    want2 = sum((abs(F(v)) - c) ** 2 for v in x)
+    want1 = sum(abs(abs(F(v)) - c) for v in x)
+    assert oracle.l2_error(x, 1, 1, 2) == float(want2)
+    assert oracle.l1_error(x, 1, 1, 2) == float(want1)
+
+
+def test_l1_bruteforce_all_candidates_and_argmin():
+    """The L1 score (Eq. MAE without the 1/N) of every (k, FL), k = 1..16 and both sign strategies, against
+    an exact Fraction brute force; argmin ties go to the smallest FL."""
+    for seed in (23, 24):
+        xs = _adversarial(seed, 10)[:16]
+        for S in (1, 0):
+            err, best, s_used, _ = oracle.fl_search(xs, S, 1, 16, -8, 23, score="l1")
+            assert s_used == S
+            for ki, k in enumerate(range(1, 17)):
+                exact = [sum(abs(F(x) - frac_val(x, k, S, fl)) for x in xs) for fl in range(-8, 24)]
+                assert err[ki].tolist() == [float(e) for e in exact], (k, S)
+                assert best[ki] == -8 + exact.index(min(exact))
+
+
+def test_l2_one_bit_row_bruteforce():
+    """The k = 1 row of the L2 search: the binary quantizer for S = 1, the two levels {0, 1} for S = 0."""
+    xs = _adversarial(25, 10)[:16]
+    for S in (1, 0):
+        err, best, _, _ = oracle.fl_search(xs, S, 1, 1, -8, 23)
+        exact = [sum((F(x) - frac_val(x, 1, S, fl)) ** 2 for x in xs) for fl in range(-8, 24)]
+        assert err[0].tolist() == [float(e) for e in exact]
+
+
+def test_l1_closed_forms_and_cauchy_schwarz():
+    """L1 is zero on the grid, |x - Q(x)| for one element, and L1^2 <= n * L2 (Cauchy-Schwarz)."""
+    codes = np.arange(-128, 128)
+    for fl in (-3, 0, 5):
+        assert oracle.l1_error((codes * 2.0 ** -fl).astype(np.float32), 8, 1, fl) == 0.0
+    for x in (0.3, -0.7, 5.25, -100.0):
+        for k, S, fl in ((8, 1, 4), (2, 0, 1), (1, 1, 3)):
+            assert oracle.l1_error(np.array([x], np.float32), k, S, fl) == float(abs(F(np.float32(x)) - frac_val(np.float32(x), k, S, fl)))
+    xs = _adversarial(26, 200)
+    for k, fl in ((4, 2), (8, 6), (1, 0)):
+        l1, l2 = oracle.l1_error(xs, k, 1, fl), oracle.l2_error(xs, k, 1, fl)
+        assert l1 * l1 <= xs.size * l2 * (1 + 1e-12)
