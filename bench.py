@@ -309,7 +309,8 @@ def run_kernel(args):
     """Single-kernel timing cases (also the targets of the ncu captures summarised in profiles/):
     conv     : VGG-16 conv3_1-shaped C-Block, batch 64, 56x56x128 -> 256, 3x3 pad 1, 8-bit codes, with
                and without the weight-code L1 bound;
-    flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid;
+    flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid, with
+               the L2 score and with the L1 score (k = 1..16 for the sweep);
     quantize : Q of 64M N(0,1) fp32 values to int8 codes and to an fp16 code tensor (HBM-bound);
     forward  : the integer forward of the workload (first plan, calibrated once), fxpq_net_forward alone."""
     import torch
@@ -344,12 +345,13 @@ def run_kernel(args):
     if args.kernel in ("flsearch", "all"):
         n = 1 << 26
         x = torch.from_numpy(synth.normal(n, 2)).cuda()
-        for name, (klo, khi) in (("flsearch_k8", (8, 8)), ("flsearch_sweep", (2, 16))):
+        for name, (klo, khi, score) in (("flsearch_k8", (8, 8, "l2")), ("flsearch_sweep", (2, 16, "l2")),
+                                        ("flsearch_k8_l1", (8, 8, "l1")), ("flsearch_sweep_l1", (1, 16, "l1"))):
             ts = []
             for i in range(args.warmup + args.steps):
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record()
-                F.fl_search(x, -1, klo, khi, -8, 23)
+                F.fl_search(x, -1, klo, khi, -8, 23, score=score)
                 e1.record()
                 e1.synchronize()
                 if i >= args.warmup:

@@ -87,6 +87,9 @@ typedef struct {
 /* enough and of the right signedness; F16 writes an fp16 code tensor: plane hi at [0, n) and */
 /* plane lo at [n, 2n) when k > 8).  n may be 0.                                             */
 /* NaN/Inf inputs latch FXPQ_ERR_NONFINITE and produce code 0.                               */
+/* f.bits may be 1: S = 0 gives the levels {0, 1}; S = 1 the binary quantizer of             */
+/* Eq. fp_1_bit_quantization, code -1 for x < 0 and 0 otherwise (-0.0 included), decoded     */
+/* 0 -> +1 before use, so the values are +-2^-fl.  fxpq_pack_codes stores it in one bit.     */
 /* ---------------------------------------------------------------------------------------- */
 FXPQ_API fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int32_t dtype, void* d_codes,
                           void* stream);
@@ -150,7 +153,10 @@ FXPQ_API fxpq_status fxpq_quantize_images(const float* d_x_nchw, int32_t N, int3
 /*   d_best : device int32[k_hi-k_lo+1]: the fl with the smallest L per k, exact ties to the  */
 /*            smallest fl.                                                                   */
 /*   d_stats: device fxpq_stats (may be NULL).                                               */
-/* Limits: 2 <= k_lo <= k_hi <= 16; -32 <= fl_lo <= fl_hi <= 40; fl_hi - fl_lo <= 31;         */
+/* k = 1 with S = 1 scores the binary quantizer of Eq. fp_1_bit_quantization (every value     */
+/* decoded to +-2^-fl: error | |x| - 2^-fl |, zeros included); k = 1 with S = 0 the levels    */
+/* {0, 1}.                                                                                   */
+/* Limits: 1 <= k_lo <= k_hi <= 16; -32 <= fl_lo <= fl_hi <= 40; fl_hi - fl_lo <= 31;         */
 /* 0 <= n <= 2^31.  Non-finite inputs latch FXPQ_ERR_NONFINITE.                              */
 /* Workspace: fxpq_fl_search_workspace() bytes, 256-byte aligned; contents are scratch.       */
 /* ---------------------------------------------------------------------------------------- */
@@ -173,7 +179,11 @@ typedef struct {
     double* d_err;         /* device double[(k_hi-k_lo+1) * (fl_hi-fl_lo+1)]                  */
     int32_t* d_best;       /* device int32[k_hi-k_lo+1]                                       */
     fxpq_stats* d_stats;   /* device fxpq_stats or NULL                                       */
+    int32_t score;         /* FXPQ_SCORE_L2: Eq. DSB_QE; FXPQ_SCORE_L1: sum_i |x_i - Q(x_i)|,   */
+                           /* the L1 error of Eq. MAE times N (same argmin), exact, rounded once */
 } fxpq_fl_search_item;
+
+enum { FXPQ_SCORE_L2 = 0, FXPQ_SCORE_L1 = 1 };
 
 FXPQ_API size_t fxpq_fl_search_batch_workspace(int32_t n_items);
 FXPQ_API fxpq_status fxpq_fl_search_batch(const fxpq_fl_search_item* h_items, int32_t n_items, void* d_ws,

@@ -30,7 +30,7 @@ class Stats(ctypes.Structure):
 
 class FlSearchItem(ctypes.Structure):
     _fields_ = [("d_x", VP), ("n", I64), ("is_signed", I32), ("k_lo", I32), ("k_hi", I32), ("fl_lo", I32),
-                ("fl_hi", I32), ("d_err", VP), ("d_best", VP), ("d_stats", VP)]
+                ("fl_hi", I32), ("d_err", VP), ("d_best", VP), ("d_stats", VP), ("score", I32)]
 
 
 class QuantizeItem(ctypes.Structure):
@@ -60,6 +60,7 @@ class Net(ctypes.Structure):
 # status / dtype / mode constants (mirror of include/fxpq.h)
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_NONFINITE, ERR_TIMEOUT, ERR_CUDA, ERR_WORKSPACE, ERR_RANGE = range(8)
 DT_I8, DT_U8, DT_I16, DT_U16, DT_I32, DT_F16 = range(6)
+SCORE_L2, SCORE_L1 = 0, 1
 OUT_CODES, OUT_ACC64, OUT_F32 = range(3)
 QB_ROWS_F16, QB_FLAT_I32 = range(2)
 OP_CONV, OP_MAXPOOL, OP_ELTWISE, OP_AVGPOOL = range(4)

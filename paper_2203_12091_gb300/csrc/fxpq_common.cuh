@@ -22,6 +22,11 @@ inline bool fmt_ok(const fxpq_fmt& f, int max_bits = 16) {
     return f.bits >= 2 && f.bits <= max_bits && (f.is_signed == 0 || f.is_signed == 1) && f.fl >= -32 &&
            f.fl <= 40;
 }
+// Formats of standalone code tensors may also be 1-bit: the levels {0, 1} (S = 0) or the binary
+// quantizer (S = 1, Eq. fp_1_bit_quantization).
+inline bool fmt_ok1(const fxpq_fmt& f, int max_bits = 16) {
+    return f.bits == 1 ? (f.is_signed == 0 || f.is_signed == 1) && f.fl >= -32 && f.fl <= 40 : fmt_ok(f, max_bits);
+}
 inline int planes_of(const fxpq_fmt& f) { return f.bits > 8 ? 2 : 1; }
 inline int64_t qmin_of(const fxpq_fmt& f) { return f.is_signed ? -(int64_t(1) << (f.bits - 1)) : 0; }
 inline int64_t qmax_of(const fxpq_fmt& f) { return (int64_t(1) << (f.bits - f.is_signed)) - 1; }

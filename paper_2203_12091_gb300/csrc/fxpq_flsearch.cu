@@ -35,7 +35,7 @@ typedef unsigned long long u64;
 constexpr int NKEY = 512;  // key = sign * 256 + biased exponent field (0..254; 255 = non-finite)
 constexpr int NJ = 17;     // j = q in [-1, 15]
 constexpr int MAXFL = 32;  // candidates per wordlength
-constexpr int MAXK = 15;   // k in [2, 16]
+constexpr int MAXK = 16;   // k in [1, 16]
 constexpr int FS_THREADS = 256;
 constexpr int FS_WARPS = FS_THREADS / 32;
 constexpr int TILE = 8192;  // 32 elements per thread, read in sub-rounds of 16
@@ -61,7 +61,8 @@ struct FsGlobal {
     u64 r[2][NJ][MAXFL][2];
     u64 rb[NJ][MAXFL][2];
     unsigned mn_inv, mx, nonfinite, pad;  // mn_inv = ~(smallest order key); 0: no finite element
-    double cells[2][MAXK][MAXFL];
+    u64 nzero;                            // finite zeros (+-0.0): no key, but a binary-quantizer error
+    double cells[2][MAXK][MAXFL];         // [S][k - 1][fl - fl_lo]
     double stat_sum, stat_sumsq;
 };
 
@@ -83,6 +84,7 @@ struct FsFinal {
     int S_lo, S_hi;
     int k_lo, nk;
     int fl_lo, nfl;
+    int l1;  // score: 0 = L2 (Eq. DSB_QE), 1 = L1 (Eq. MAE as a sum)
 };
 
 struct FsBatch {
@@ -204,7 +206,8 @@ __device__ __forceinline__ void acc_zero(Acc<NS, NRB>& a) {
 // Narrow wordlength range: every remainder slot is computed without branches (slots the key does not
 // use are never flushed).  The rounding error's magnitude is min(t, 2^p - t) for the fraction t of y
 // in units of 2^-p, whichever way a tie rounds, so the parity of y's integer part is not needed.
-template <int NS>
+// L1: first powers of the remainders (the L1 score), otherwise squares.
+template <int NS, bool L1>
 __device__ __forceinline__ void acc_add_narrow(Acc<NS, 2>& a, unsigned M, bool rb_on, const RbC& c) {
     a.n += 1u;
     a.s1 += M;
@@ -214,7 +217,7 @@ __device__ __forceinline__ void acc_add_narrow(Acc<NS, 2>& a, unsigned M, bool r
         const unsigned full = 1u << (24 - jj);  // p = 23 - j bits below y's binary point
         const unsigned t = M & (full - 1u);
         const unsigned r = min(t, full - t);
-        a.r[jj] += (u64)r * r;
+        a.r[jj] += L1 ? (u64)r : (u64)r * r;
     }
     if (rb_on) {
         // boundary: saturated iff M >= thr, error (M - thr) u_E; otherwise the rounding error
@@ -223,13 +226,13 @@ __device__ __forceinline__ void acc_add_narrow(Acc<NS, 2>& a, unsigned M, bool r
             const unsigned t = M & c.mask[i];
             const unsigned r = min(t, c.full[i] - t);
             const unsigned rb = M >= c.thr[i] ? M - c.thr[i] : r;
-            a.rb[i] += (u64)rb * rb;
+            a.rb[i] += L1 ? (u64)rb : (u64)rb * rb;
         }
     }
 }
 
 // Add one element (significand M of the warp's current key) to this lane's accumulators.
-template <int NS>
+template <int NS, bool L1>
 __device__ __forceinline__ void acc_add(Acc<NS, NS>& a, unsigned M, const KeyInfo& k) {
     a.n += 1u;
     a.s1 += M;
@@ -243,12 +246,12 @@ __device__ __forceinline__ void acc_add(Acc<NS, NS>& a, unsigned M, const KeyInf
             const unsigned odd = (M >> p) & 1u;
             const bool up = (t + odd) > (1u << (p - 1));
             const unsigned r = up ? (1u << p) - t : t;
-            if ((k.validR >> jj) & 1u) a.r[jj] += (u64)r * r;
+            if ((k.validR >> jj) & 1u) a.r[jj] += L1 ? (u64)r : (u64)r * r;
             if (j >= 0 && ((k.validRb >> jj) & 1u)) {
                 // boundary t' = j + 1: saturated iff M >= (2^(j+1) - 1) 2^(23-j)
                 const unsigned thr = ((2u << j) - 1u) << (23 - j);
                 const unsigned rb = M >= thr ? M - thr : r;
-                a.rb[jj] += (u64)rb * rb;
+                a.rb[jj] += L1 ? (u64)rb : (u64)rb * rb;
             }
         }
     }
@@ -313,7 +316,7 @@ __device__ __forceinline__ void load16(const FsParams& P, long long tb, int sub,
     }
 }
 
-template <bool VEC, int NS, int NRB>
+template <bool VEC, int NS, int NRB, bool L1>
 __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     fl_search_bins_kernel(const __grid_constant__ FsBatch B, int item0, int item1) {
     // this launch covers items [item0, item1); blk0 holds their block offsets relative to the launch
@@ -331,6 +334,7 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     __syncthreads();
     if (threadIdx.x == 0) sm.mn = 0xFFFFFFFFu;
     unsigned tmn = 0xFFFFFFFFu, tmx = 0u;
+    unsigned tz = 0u;  // finite zeros
     bool tnf = false;
 
     const long long start = (long long)blk * P.chunk;
@@ -353,6 +357,7 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
                         const unsigned ok = order_key(v[e]);
                         tmn = min(tmn, ok);
                         tmx = max(tmx, ok);
+                        tz += (u & 0x7FFFFFFFu) == 0u ? 1u : 0u;
                     }
                 }
                 // per-element shared-memory reduction (no value returned); lanes with equal keys
@@ -422,9 +427,9 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
             // common case: every lane is live and continues the current key
             if (__all_sync(0xFFFFFFFFu, kx == ck)) {
                 if constexpr (NRB == 2)
-                    acc_add_narrow(acc, M, ki.validRb != 0u, rbc);
+                    acc_add_narrow<NS, L1>(acc, M, ki.validRb != 0u, rbc);
                 else
-                    acc_add(acc, M, ki);
+                    acc_add<NS, L1>(acc, M, ki);
                 continue;
             }
             unsigned rem = __ballot_sync(0xFFFFFFFFu, live);
@@ -441,9 +446,9 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
                 }
                 if ((in >> lane) & 1u) {
                     if constexpr (NRB == 2)
-                        acc_add_narrow(acc, M, ki.validRb != 0u, rbc);
+                        acc_add_narrow<NS, L1>(acc, M, ki.validRb != 0u, rbc);
                     else
-                        acc_add(acc, M, ki);
+                        acc_add<NS, L1>(acc, M, ki);
                 }
                 rem &= ~in;
             }
@@ -456,6 +461,10 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     atomicMin(&sm.mn, tmn);
     atomicMax(&sm.mx, tmx);
     if (tnf) sm.nonfinite = 1u;
+    {
+        const unsigned zw = __reduce_add_sync(0xFFFFFFFFu, tz);
+        if (lane == 0 && zw) atomicAdd(&P.g->nzero, (u64)zw);
+    }
     __syncthreads();
 
     // ---- block bins -> exact workspace bins
@@ -634,32 +643,62 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             else
                 big_add(acc, ld128(g->ps1[key]), E - 23, (key >> 8) != 0);
         }
+    } else if (F.k_lo == 1 && F.S_lo + cell / (F.nk * F.nfl) == 1 && (cell % (F.nk * F.nfl)) / F.nfl == 0) {
+        // k = 1, S = 1: the binary quantizer (Eq. fp_1_bit_quantization), every value decoded to
+        // +-c with c = 2^-fl, so the error of x is | |x| - c |: from the moments alone, zeros included
+        const int fl = F.fl_lo + cell % F.nfl;
+        if (lane == 0) {
+            const U128 nz{g->nzero, 0ull};
+            big_add(acc, nz, F.l1 ? -fl : -2 * fl, false);
+        }
+        for (int key = lane; key < NKEY; key += 32) {
+            const u64 n = g->pn[key];
+            if (!n) continue;
+            const int eb = key & 255, E = eb ? eb - 127 : -126;
+            const U128 s1 = ld128(g->ps1[key]), s2 = ld128(g->ps2[key]);
+            if (!F.l1) {
+                add_sat(acc, n, s1, s2, E, fl, 1ull);  // sum (|x| - c)^2
+            } else {
+                // |x| >= 2^E >= c when E >= -fl, else |x| < 2^(E+1) <= c
+                const bool above = E >= -fl;
+                big_add(acc, s1, E - 23, !above);
+                big_add(acc, U128{n, 0ull}, -fl, above);
+            }
+        }
     } else {
         const int S = F.S_lo + cell / (F.nk * F.nfl);
         const int rem = cell % (F.nk * F.nfl);
         const int k = F.k_lo + rem / F.nfl;
         const int fi = rem % F.nfl;
         const int fl = F.fl_lo + fi;
+        // L2 terms weigh u_E^2 = 2^(2(E-23)), L1 terms u_E = 2^(E-23)
+        const int pw = F.l1 ? 1 : 2;
         for (int key = lane; key < NKEY; key += 32) {
             const u64 n = g->pn[key];
             if (!n) continue;
             const int sg = key >> 8, eb = key & 255, E = eb ? eb - 127 : -126;
             const U128 s1 = ld128(g->ps1[key]), s2 = ld128(g->ps2[key]);
-            if (sg == 1 && S == 0) {  // clipped to code 0: error x^2
-                big_add(acc, s2, 2 * (E - 23), false);
+            if (sg == 1 && S == 0) {  // clipped to code 0: error |x|
+                big_add(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
                 continue;
             }
             const int t = (sg == 0) ? (S ? k - 1 : k) : (k - 1);
             const u64 T = (sg == 0) ? ((1ull << t) - 1ull) : (1ull << t);
             const int q = E + fl;
-            if (q >= t)
-                add_sat(acc, n, s1, s2, E, fl, T);
-            else if (sg == 0 && q == t - 1)
-                big_add(acc, ld128(g->rb[q + 1][fi]), 2 * (E - 23), false);
-            else if (q <= -2)
-                big_add(acc, s2, 2 * (E - 23), false);
-            else
-                big_add(acc, ld128(g->r[sg][q + 1][fi]), 2 * (E - 23), false);
+            if (q >= t) {
+                if (F.l1) {  // |x| >= T 2^-fl: sum |x| - n T 2^-fl
+                    big_add(acc, s1, E - 23, false);
+                    big_add(acc, U128{n * T, 0ull}, -fl, true);
+                } else {
+                    add_sat(acc, n, s1, s2, E, fl, T);
+                }
+            } else if (sg == 0 && q == t - 1) {
+                big_add(acc, ld128(g->rb[q + 1][fi]), pw * (E - 23), false);
+            } else if (q <= -2) {
+                big_add(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
+            } else {
+                big_add(acc, ld128(g->r[sg][q + 1][fi]), pw * (E - 23), false);
+            }
         }
     }
 #pragma unroll
@@ -676,7 +715,7 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
     } else {
         const int S = F.S_lo + cell / (F.nk * F.nfl);
         const int rem = cell % (F.nk * F.nfl);
-        gw->cells[S][F.k_lo + rem / F.nfl - 2][rem % F.nfl] = big_to_double(acc);
+        gw->cells[S][F.k_lo + rem / F.nfl - 1][rem % F.nfl] = big_to_double(acc);
     }
 }
 
@@ -708,7 +747,7 @@ __global__ void fl_search_select_kernel(const __grid_constant__ FsBatch B, const
         double bv = 0.0;
         int bf = F.fl_lo;
         for (int fi = 0; fi < F.nfl; ++fi) {
-            const double v = g->cells[S][k - 2][fi];
+            const double v = g->cells[S][k - 1][fi];
             out.err[(long long)i * F.nfl + fi] = v;
             if (fi == 0 || v < bv) {  // strict: exact ties keep the smaller FL
                 bv = v;
@@ -744,12 +783,15 @@ void st_attr_once() {
     std::lock_guard<std::mutex> lk(g_fs_attr_mu);
     if (g_fs_attr_done) return;
     const int sb = (int)sizeof(FsSmem);
-    cudaFuncSetAttribute(fl_search_bins_kernel<true, 10, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<true, NJ, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<false, 10, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
-    cudaFuncSetAttribute(fl_search_bins_kernel<false, NJ, NJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+#define FXPQ_FS_ATTR(V, L1)                                                                                      \
+    cudaFuncSetAttribute(fl_search_bins_kernel<V, 10, 2, L1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb); \
+    cudaFuncSetAttribute(fl_search_bins_kernel<V, NJ, 2, L1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb); \
+    cudaFuncSetAttribute(fl_search_bins_kernel<V, NJ, NJ, L1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sb);
+    FXPQ_FS_ATTR(true, false)
+    FXPQ_FS_ATTR(false, false)
+    FXPQ_FS_ATTR(true, true)
+    FXPQ_FS_ATTR(false, true)
+#undef FXPQ_FS_ATTR
     g_fs_attr_done = true;
 }
 }  // namespace
@@ -762,7 +804,8 @@ struct FsItemHost {
     FsParams p;
     FsFinal f;
     FsOut o;
-    int variant;  // bins kernel instance: bit 0 vec, bit 1 small (k_hi <= 9), bit 2 narrow boundary range
+    int variant;  // bins kernel instance: bit 0 vec, bit 1 small (k_hi <= 9), bit 2 narrow boundary range,
+                  // bit 3 L1 score
     int grid;     // bins blocks
 };
 
@@ -770,7 +813,8 @@ fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h
     const int64_t n = it.n;
     if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;
     if (it.is_signed < -1 || it.is_signed > 1) return FXPQ_ERR_INVALID_ARG;
-    if (it.k_lo < 2 || it.k_hi > 16 || it.k_lo > it.k_hi) return FXPQ_ERR_INVALID_ARG;
+    if (it.k_lo < 1 || it.k_hi > 16 || it.k_lo > it.k_hi) return FXPQ_ERR_INVALID_ARG;
+    if (it.score != FXPQ_SCORE_L2 && it.score != FXPQ_SCORE_L1) return FXPQ_ERR_INVALID_ARG;
     if (it.fl_lo < -32 || it.fl_hi > 40 || it.fl_lo > it.fl_hi || it.fl_hi - it.fl_lo + 1 > MAXFL)
         return FXPQ_ERR_INVALID_ARG;
     if (!it.d_err || !it.d_best || (n > 0 && !it.d_x)) return FXPQ_ERR_INVALID_ARG;
@@ -802,29 +846,35 @@ fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h
     h.f.nk = it.k_hi - it.k_lo + 1;
     h.f.fl_lo = it.fl_lo;
     h.f.nfl = P.nfl;
+    h.f.l1 = it.score == FXPQ_SCORE_L1 ? 1 : 0;
     h.o.err = it.d_err;
     h.o.best = it.d_best;
     h.o.stats = it.d_stats;
     h.o.is_signed = it.is_signed;
     h.grid = (int)((n + chunk - 1) / chunk);
-    h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0);
+    h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0) |
+                (h.f.l1 ? 8 : 0);
     return FXPQ_OK;
 }
 
 void fs_bins_launch(int variant, int grid, const FsBatch& B, int i0, int i1, cudaStream_t s) {
     const size_t sb = sizeof(FsSmem);
-    const bool vec = variant & 1, small = variant & 2, narrow = variant & 4;
-#define FXPQ_FS_LAUNCH(V)                                                                \
+    const bool vec = variant & 1, small = variant & 2, narrow = variant & 4, l1 = variant & 8;
+#define FXPQ_FS_LAUNCH(V, L1)                                                            \
     if (narrow && small)                                                                 \
-        fl_search_bins_kernel<V, 10, 2><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);         \
+        fl_search_bins_kernel<V, 10, 2, L1><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);     \
     else if (narrow)                                                                     \
-        fl_search_bins_kernel<V, NJ, 2><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);         \
+        fl_search_bins_kernel<V, NJ, 2, L1><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);     \
     else                                                                                 \
-        fl_search_bins_kernel<V, NJ, NJ><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);
-    if (vec) {
-        FXPQ_FS_LAUNCH(true)
+        fl_search_bins_kernel<V, NJ, NJ, L1><<<grid, FS_THREADS, sb, s>>>(B, i0, i1);
+    if (vec && !l1) {
+        FXPQ_FS_LAUNCH(true, false)
+    } else if (!l1) {
+        FXPQ_FS_LAUNCH(false, false)
+    } else if (vec) {
+        FXPQ_FS_LAUNCH(true, true)
     } else {
-        FXPQ_FS_LAUNCH(false)
+        FXPQ_FS_LAUNCH(false, true)
     }
 #undef FXPQ_FS_LAUNCH
 }
@@ -838,7 +888,7 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
     // order by kernel instance (stable), each item keeping its own bins
     int order[FS_MAX_ITEMS];
     int m = 0;
-    for (int v = 0; v < 8; ++v)
+    for (int v = 0; v < 16; ++v)
         for (int i = 0; i < n; ++i)
             if (h[i].variant == v) order[m++] = i;
     FsBatch B;
@@ -888,7 +938,7 @@ extern "C" size_t fxpq_fl_search_workspace(int64_t n) {
 extern "C" fxpq_status fxpq_fl_search(const float* d_x, int64_t n, int32_t is_signed, int32_t k_lo, int32_t k_hi,
                                       int32_t fl_lo, int32_t fl_hi, double* d_err, int32_t* d_best,
                                       fxpq_stats* d_stats, void* d_ws, size_t ws_bytes, void* stream) {
-    const fxpq_fl_search_item it = {d_x, n, is_signed, k_lo, k_hi, fl_lo, fl_hi, d_err, d_best, d_stats};
+    const fxpq_fl_search_item it = {d_x, n, is_signed, k_lo, k_hi, fl_lo, fl_hi, d_err, d_best, d_stats, FXPQ_SCORE_L2};
     FsItemHost h;
     const fxpq_status st = fs_prepare(it, static_cast<FsGlobal*>(d_ws), h);
     if (st != FXPQ_OK) return st;
@@ -981,8 +1031,8 @@ extern "C" fxpq_status fxpq_fl_search_noalloc(const float* d_x, int64_t n, int32
                                               int32_t k_hi, int32_t fl_lo, int32_t fl_hi, double* d_err,
                                               int32_t* d_best, fxpq_stats* d_stats, void* stream) {
     if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;  // the largest tensor the bins can hold
-    if (k_lo < 2 || k_hi > 16 || k_lo > k_hi || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL)
-        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 15 x 32
+    if (k_lo < 1 || k_hi > 16 || k_lo > k_hi || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL)
+        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 16 x 32
     if (fxpq_fl_search_workspace(n) > kFlSearchStaticBytes) return FXPQ_ERR_WORKSPACE;
     void* scratch = nullptr;
     const fxpq_status st = fl_search_scratch_ptr(&scratch);

@@ -13,6 +13,7 @@ namespace {
 struct QParams {
     float scale;  // 2^fl (exact power of two; fl in [-32, 40])
     float lo, hi; // Qmin, Qmax as floats (exact, |.| <= 2^16)
+    int binary;   // signed 1-bit: the binary quantizer (Eq. fp_1_bit_quantization)
     int* status;
 };
 
@@ -21,6 +22,7 @@ __device__ __forceinline__ int quant1(float x, const QParams& p, bool& bad) {
         bad = true;
         return 0;
     }
+    if (p.binary) return x < 0.0f ? -1 : 0;  // -0.0 is not below zero
     // x * 2^fl is exact unless it overflows (then it saturates) or falls below 2^-126 (then it
     // rounds to 0 either way); rintf rounds half to even.
     float y = rintf(x * p.scale);
@@ -248,6 +250,7 @@ __global__ void __launch_bounds__(256) quantize_batch_kernel(const __grid_consta
     p.scale = __int_as_float((127 + fl) << 23);  // 2^fl, fl in [-32, 40]
     p.lo = S ? -(float)(1 << (I.bits - 1)) : 0.0f;
     p.hi = (float)((1 << (I.bits - S)) - 1);
+    p.binary = 0;  // batch items have k >= 2
     p.status = B.status;
     bool bad = false;
     if (I.kind == FXPQ_QB_FLAT_I32) {
@@ -382,6 +385,7 @@ static QParams make_qparams(const fxpq_fmt& f) {
     p.scale = ldexpf(1.0f, f.fl);
     p.lo = (float)qmin_of(f);
     p.hi = (float)qmax_of(f);
+    p.binary = f.bits == 1 && f.is_signed == 1;
     p.status = status_ptr();
     return p;
 }
@@ -399,7 +403,7 @@ using namespace fxpq;
 
 extern "C" fxpq_status fxpq_quantize(const float* d_x, int64_t n, fxpq_fmt f, int32_t dtype, void* d_codes,
                                      void* stream) {
-    if (n < 0 || (n > 0 && (!d_x || !d_codes)) || !fmt_ok(f, 32)) return FXPQ_ERR_INVALID_ARG;
+    if (n < 0 || (n > 0 && (!d_x || !d_codes)) || !fmt_ok1(f, 32)) return FXPQ_ERR_INVALID_ARG;
     if (f.bits > 16 && dtype != FXPQ_DT_I32) return FXPQ_ERR_INVALID_ARG;
     switch (dtype) {
         case FXPQ_DT_I8: if (!(f.is_signed && f.bits <= 8)) return FXPQ_ERR_INVALID_ARG; break;
@@ -562,7 +566,7 @@ extern "C" fxpq_status fxpq_quantize_batch(const fxpq_quantize_item* h_items, in
 
 extern "C" fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt fmt, uint32_t* d_words,
                                        void* stream) {
-    if (n < 0 || !fmt_ok(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
+    if (n < 0 || !fmt_ok1(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
         return FXPQ_ERR_INVALID_ARG;
     if (n == 0) return FXPQ_OK;
     const long long ng = (n + 31) / 32;
@@ -574,7 +578,7 @@ extern "C" fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt 
 
 extern "C" fxpq_status fxpq_unpack_codes(const uint32_t* d_words, int64_t n, fxpq_fmt fmt, void* d_codes,
                                          void* stream) {
-    if (n < 0 || !fmt_ok(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
+    if (n < 0 || !fmt_ok1(fmt) || (n > 0 && (!d_codes || !d_words)) || !aligned(d_words, 4))
         return FXPQ_ERR_INVALID_ARG;
     if (n == 0) return FXPQ_OK;
     const long long ng = (n + 31) / 32;

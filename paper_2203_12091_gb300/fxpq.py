@@ -78,15 +78,21 @@ def fxpq_fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: i
                                    _p(stats), _p(ws), ws.numel(), _s(stream)))
 
 
-def fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, stream=None):
-    """Allocate the outputs and run fxpq_fl_search.  Returns device (err[nk, nfl], best[nk], stats bytes)."""
+def fl_search(x, is_signed: int, k_lo: int, k_hi: int, fl_lo: int, fl_hi: int, stream=None, score: str = "l2"):
+    """Allocate the outputs and run fxpq_fl_search (score "l2"), or a one-item fxpq_fl_search_batch with
+    the L1 score (score "l1").  Returns device (err[nk, nfl], best[nk], stats bytes)."""
     nk, nfl = k_hi - k_lo + 1, fl_hi - fl_lo + 1
     dev = x.device
     err = torch.empty(nk * nfl, dtype=torch.float64, device=dev)
     best = torch.empty(nk, dtype=torch.int32, device=dev)
     stats = torch.empty(ctypes.sizeof(Stats), dtype=torch.uint8, device=dev)
-    ws = workspace(fxpq_fl_search_workspace(x.numel()), dev)
-    fxpq_fl_search(x, is_signed, k_lo, k_hi, fl_lo, fl_hi, err, best, stats, ws, stream)
+    if score == "l2":
+        ws = workspace(fxpq_fl_search_workspace(x.numel()), dev)
+        fxpq_fl_search(x, is_signed, k_lo, k_hi, fl_lo, fl_hi, err, best, stats, ws, stream)
+    else:
+        item = L.FlSearchItem(x.data_ptr(), x.numel(), is_signed, k_lo, k_hi, fl_lo, fl_hi, err.data_ptr(),
+                              best.data_ptr(), stats.data_ptr(), {"l1": L.SCORE_L1}[score])
+        fxpq_fl_search_batch([item], workspace(fxpq_fl_search_batch_workspace(1), dev), stream)
     return err.view(nk, nfl), best, stats
 
 

@@ -51,7 +51,7 @@ def test_host_validation_rejects_bad_arguments(lib):
     ws = lib.fxpq_fl_search_workspace(100)
     assert ws > 0 and ws % 256 == 0
     # k out of range, FL span too wide, missing outputs, workspace too small / misaligned
-    assert lib.fxpq_fl_search(p, 100, -1, 1, 8, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_fl_search(p, 100, -1, 0, 8, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
     assert lib.fxpq_fl_search(p, 100, -1, 2, 17, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
     assert lib.fxpq_fl_search(p, 100, -1, 2, 8, -8, 24, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
     assert lib.fxpq_fl_search(p, 100, 2, 2, 8, 0, 10, p, p, None, p, ws, None) == L.ERR_INVALID_ARG
@@ -186,3 +186,24 @@ def test_net_memory_matches_oracle(lib, arch):
     assert ro == pytest.approx(oracle.ro_r(params), rel=1e-12)
     assert rw32 == pytest.approx(oracle.rw_r(layers, elems, {nm: 32 for nm in bits}), rel=1e-12)
     assert ro32 == pytest.approx(oracle.ro_r([(n, 32) for n, _ in params]), rel=1e-12)
+
+
+def test_new_entry_points_reject_bad_arguments(lib):
+    """Every rejected call returns before any launch (no device is touched)."""
+    p = ctypes.c_void_p(256)
+    assert lib.fxpq_pack_codes(p, 10, L.Fmt(0, 1, 0), p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_pack_codes(p, 10, L.Fmt(17, 1, 0), p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_pack_codes(p, -1, L.Fmt(4, 1, 0), p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_pack_codes(p, 10, L.Fmt(4, 1, 0), ctypes.c_void_p(258), None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_unpack_codes(p, 10, L.Fmt(4, 2, 0), p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_unpack_codes(None, 10, L.Fmt(4, 1, 0), p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_bn_to_scale(p, p, p, p, -1, 1e-5, p, p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_bn_to_scale(p, p, p, p, 8, -1.0, p, p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_bn_to_scale(p, None, p, p, 8, 1e-5, p, p, None) == L.ERR_INVALID_ARG
+    assert lib.fxpq_quantize(p, 4, L.Fmt(1, 2, 0), L.DT_I8, p, None) == L.ERR_INVALID_ARG
+    item = L.FlSearchItem(256, 100, -1, 1, 8, 0, 10, 256, 256, None, 2)  # unknown score
+    ws = lib.fxpq_fl_search_batch_workspace(1)
+    arr = (L.FlSearchItem * 1)(item)
+    assert lib.fxpq_fl_search_batch(ctypes.cast(arr, ctypes.c_void_p), 1, p, ws, None) == L.ERR_INVALID_ARG
+    rw, ro = ctypes.c_double(), ctypes.c_double()
+    assert lib.fxpq_net_memory(None, 0, ctypes.byref(rw), ctypes.byref(ro)) == L.ERR_INVALID_ARG

@@ -102,10 +102,10 @@ def test_quantize_rows_and_images(F, k, C, Cp):
     assert np.array_equal(got[..., :3], want) and np.all(got[..., 3:] == 0)
 
 
-def _check_search(F, x, S, klo, khi, fllo, flhi):
-    err, best, st = F.fl_search(torch.from_numpy(x).cuda(), S, klo, khi, fllo, flhi)
+def _check_search(F, x, S, klo, khi, fllo, flhi, score="l2"):
+    err, best, st = F.fl_search(torch.from_numpy(x).cuda(), S, klo, khi, fllo, flhi, score=score)
     torch.cuda.synchronize()
-    oerr, obest, oS, ost = oracle.fl_search(x, S, klo, khi, fllo, flhi)
+    oerr, obest, oS, ost = oracle.fl_search(x, S, klo, khi, fllo, flhi, score=score)
     g = err.cpu().numpy()
     assert np.array_equal(best.cpu().numpy(), obest)
     np.testing.assert_allclose(g, oerr, rtol=RTOL, atol=0)
@@ -133,6 +133,46 @@ def test_fl_search_small_sizes_and_ranges(F, dist, n):
     _check_search(F, x, 1, 8, 8, 0, 15)
     _check_search(F, x, -1, 3, 9, -32, -1)
     _check_search(F, x, -1, 13, 16, 9, 40)
+
+
+@pytest.mark.parametrize("score", ["l2", "l1"])
+@pytest.mark.parametrize("seed", [4, 5])
+def test_fl_search_scores_with_one_bit_rows(F, score, seed):
+    """Both scores over k = 1..16 (k = 1: the binary quantizer for S = 1, the levels {0, 1} for S = 0),
+    exact zeros included, bit-identical to the oracle."""
+    x = _adv(seed, 3000)
+    x[::97] = 0.0
+    x[5] = -0.0
+    _check_search(F, x, -1, 1, 16, -8, 23, score)
+    _check_search(F, np.abs(x), -1, 1, 16, -8, 23, score)
+    _check_search(F, x, 0, 1, 16, -8, 23, score)
+    _check_search(F, x, 1, 1, 1, -8, 23, score)
+
+
+@pytest.mark.parametrize("dist", ["normal", "laplace", "relu_normal"])
+@pytest.mark.parametrize("n", [0, 1, 1023, 70001])
+def test_fl_search_l1_sizes_and_ranges(F, dist, n):
+    x = synth.sweep_tensor(dist, n, 17 + n)
+    _check_search(F, x, -1, 1, 16, -8, 23, "l1")
+    _check_search(F, x, 1, 8, 8, 0, 15, "l1")
+    _check_search(F, x, -1, 13, 16, 9, 40, "l1")
+
+
+def test_quantize_binary(F):
+    """The binary quantizer: -1 for x < 0, 0 otherwise (-0.0 included), to int8 and to an fp16 code tensor."""
+    x = _adv(9, 5000)
+    x[:3] = [-0.0, 0.0, -1e-45]
+    xd = torch.from_numpy(x).cuda()
+    want = oracle.quantize(x, 1, 1, 3)
+    o8 = torch.empty(x.size, dtype=torch.int8, device="cuda")
+    F.fxpq_quantize(xd, F.fmt(1, 1, 3), F.DT_I8, o8)
+    assert np.array_equal(o8.cpu().numpy().astype(np.int64), want)
+    o16 = torch.empty(x.size, dtype=torch.float16, device="cuda")
+    F.fxpq_quantize(xd, F.fmt(1, 1, 3), F.DT_F16, o16)
+    assert np.array_equal(o16.cpu().numpy().astype(np.int64), want)
+    words = torch.empty(F.packed_words(x.size, F.fmt(1, 1, 3)), dtype=torch.int32, device="cuda")
+    F.fxpq_pack_codes(o16, x.size, F.fmt(1, 1, 3), words)
+    assert np.array_equal(words.cpu().numpy().view(np.uint32), oracle.pack_codes(want, 1))
 
 
 def test_fl_search_ties_pick_smallest_fl(F):
@@ -175,6 +215,20 @@ def test_fl_search_config_large_sampled(F, n):
         assert g[k - 2, fl + 8] == oracle.l2_error(x, k, 1, fl)
     assert s.sumsq == oracle.exact_sum(x.astype(np.float64) ** 2)
     assert s.min == float(x.min()) and s.max == float(x.max())
+
+
+def test_fl_search_l1_large_sampled(F):
+    """16M Laplace values, k = 1..16 with the L1 score: sampled cells (the k = 1 binary row included)
+    recomputed by the oracle one by one, argmin against the GPU's own scores."""
+    n = 1 << 24
+    x = synth.sweep_tensor("laplace", n, 3)
+    err, best, st = F.fl_search(torch.from_numpy(x).cuda(), -1, 1, 16, -8, 23, score="l1")
+    g = err.cpu().numpy()
+    b = best.cpu().numpy()
+    for ki in range(16):
+        assert b[ki] == -8 + int(np.argmin(g[ki]))
+    for k, fl in [(1, int(b[0])), (1, -8), (8, int(b[7])), (3, 2), (16, 23)]:
+        assert g[k - 1, fl + 8] == oracle.l1_error(x, k, 1, fl)
 
 
 def test_fl_search_batch_matches_oracle(F):
