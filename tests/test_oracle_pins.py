@@ -620,3 +620,107 @@ def test_l1_closed_forms_and_cauchy_schwarz():
     for k, fl in ((4, 2), (8, 6), (1, 0)):
         l1, l2 = oracle.l1_error(xs, k, 1, fl), oracle.l2_error(xs, k, 1, fl)
         assert l1 * l1 <= xs.size * l2 * (1 + 1e-12)
+
+
+# ---------------------------------------------------------------- forward optimizer (Alg. 1, cost F)
+from oracle import qopt  # noqa: E402
+
+
+def test_qparams_opt_hand_traced_search():
+    """Alg. 1 on the convex cost (FL - 7)^2 from FL 4 with K = 1: direction -1 tries 3 and stops; direction
+    +1 improves at 5, 6, 7 (each success extends the limit by one), tries 8 and stops."""
+    calls = []
+
+    def cost(fl):
+        calls.append(fl)
+        return float((fl - 7) ** 2)
+
+    best, c, trace = qopt.qparams_opt(cost, 4, K=1)
+    assert (best, c) == (7, 0.0)
+    assert trace == [(4, 9.0), (3, 16.0), (5, 4.0), (6, 1.0), (7, 0.0), (8, 1.0)]
+    # K = 2 also looks two steps to the left without an improvement; a tie is not an improvement
+    best, c, trace = qopt.qparams_opt(lambda fl: float(abs(fl - 4) // 2), 4, K=2)
+    assert best == 4 and [f for f, _ in trace] == [4, 3, 2, 5, 6]
+
+
+def test_unclass_and_mispred_hand_example():
+    """Eqs. unclassified_samples / mispredicted_classes: sample 0 ties two classes, sample 1 none, sample 2
+    ties all three: UnClass = 2/3, MisPred = (1 + 0 + 2) / (3 * 3)."""
+    lg = np.array([[1.0, 1.0, 0.0], [2.0, 0.0, 0.0], [5.0, 5.0, 5.0]])
+    assert qopt.ties(lg).tolist() == [2, 1, 3]
+    uc, mp = qopt.unclass_mispred(lg)
+    assert uc == pytest.approx(2 / 3) and mp == pytest.approx(3 / 9)
+
+
+def test_fp_conv_equals_integer_conv_on_integer_data():
+    rng = np.random.default_rng(51)
+    x = rng.integers(-20, 20, size=(2, 7, 6, 5))
+    w = rng.integers(-9, 9, size=(4, 3, 3, 5))
+    for st, pad in ((1, 1), (2, 0)):
+        assert np.array_equal(qopt.f_conv(x, w, None, st, pad, False), oracle.conv2d(x, w, st, pad).astype(np.float64))
+
+
+def _qopt_tiny():
+    layers = [
+        {"type": "conv", "name": "c1", "C": 3, "K": 8, "R": 3, "stride": 1, "pad": 1, "relu": True, "src": None},
+        {"type": "maxpool", "name": "p1", "k": 2, "stride": 2, "pad": 0},
+        {"type": "conv", "name": "c2", "C": 8, "K": 8, "R": 3, "stride": 1, "pad": 1, "relu": False, "src": "p1"},
+        {"type": "eltwise", "name": "e", "a": "c2", "b": "p1", "relu": True},
+        {"type": "avgpool", "name": "gap", "src": "e"},
+        {"type": "conv", "name": "fc", "C": 8, "K": 10, "R": 1, "stride": 1, "pad": 0, "relu": False, "src": "gap"},
+    ]
+    rng = np.random.default_rng(52)
+    W = {}
+    for L in layers:
+        if L["type"] == "conv":
+            fan = L["C"] * L["R"] ** 2
+            W[L["name"]] = ((rng.standard_normal((L["K"], L["R"], L["R"], L["C"])) * np.sqrt(2 / fan)).astype(np.float32),
+                            (rng.standard_normal(L["K"]) * 0.05).astype(np.float32))
+    plan = {"input": 6, "c1": {"w": 5, "b": 8, "a": 5}, "c2": {"w": 4, "b": 8, "a": 6}, "e": {"a": 5},
+            "gap": {"a": 6, "r": 16}, "fc": {"w": 6, "b": 8}}
+    return layers, W, plan, synth.images(4, 53, hw=8)
+
+
+def test_mixed_forward_fully_fixed_point_equals_integer_network():
+    """With every data-structure fixed point, the mixed forward's logits equal the integer network's (oracle
+    net) at the same formats, value for value; pi sums to one per layer."""
+    layers, W, plan, imgs = _qopt_tiny()
+    net = qopt.Net(layers, W, imgs, plan)
+    last = net.order[-1]
+    net_fmts = {"input": net.fmt[("input", "a")]}
+    for L in layers:
+        nm = L["name"]
+        d = {}
+        for j in ("w", "b", "a"):
+            if (nm, j) in net.fmt:
+                d[j] = net.fmt[(nm, j)]
+        if L["type"] == "avgpool":
+            d["r"] = net._recip(nm, 16)[0]
+        net_fmts[nm] = d
+    for ds in net.order[:-1]:
+        net.done.add(ds)
+    X, logits = net.forward(last, net.fmt[last][2])
+    qparams = {}
+    for L in layers:
+        if L["type"] == "conv":
+            nm = L["name"]
+            qparams[nm] = (oracle.quantize(W[nm][0], *net_fmts[nm]["w"]).reshape(W[nm][0].shape),
+                           oracle.quantize(W[nm][1], *net_fmts[nm]["b"]))
+    want, s = onet.forward(layers, net_fmts, qparams, imgs)
+    assert np.array_equal(logits, want.astype(np.float64) * 2.0 ** -s)
+    # the importance weights of a layer's data-structures sum to one
+    sts = [qopt.ds_stats(X[("c1", j)][0], j == "a") for j in ("a", "w", "b")]
+    den = sum(s_ * n for s_, n, _ in sts)
+    assert sum(s_ * n / den for s_, n, _ in sts) == pytest.approx(1.0)
+
+
+def test_forward_optimizer_cost_is_zero_for_on_grid_data():
+    """L is zero for data on the grid, so E vanishes for a data-structure whose every term is exact: a
+    network of one 1x1 conv with power-of-two weights and integer images has E = 0 for its bias."""
+    layers = [{"type": "conv", "name": "fc", "C": 3, "K": 4, "R": 1, "stride": 1, "pad": 0, "relu": False, "src": None}]
+    W = {"fc": (np.array([1, 0.5, -2, 0.25] * 3, np.float32).reshape(4, 1, 1, 3), np.array([1, 2, 3, 4], np.float32))}
+    imgs = np.random.default_rng(54).integers(-3, 4, size=(2, 3, 2, 2)).astype(np.float32)
+    net = qopt.Net(layers, W, imgs, {"input": 8, "fc": {"w": 8, "b": 8}})
+    F_, E, uc, mp = net.cost(("fc", "b"), net.fmt[("fc", "b")][2])
+    assert E == 0.0
+    assert F_ == uc + mp
