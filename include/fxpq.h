@@ -386,6 +386,54 @@ FXPQ_API fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_ca
                                         int32_t fl_lo, int32_t fl_hi, fxpq_fmt* h_fmt_in, fxpq_fmt* h_fmt_y,
                                         void* d_ws, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------------------- */
+/* Forward optimizer support (Sec. IV-C, Alg. 1 QParamsOpt and its cost F of                */
+/* Eq. quantization_parameters_optimization).  While one data-structure's QPs are searched,  */
+/* every data-structure after it is FP32: these are the FP32 layers, the conversions between */
+/* the two worlds, and the statistics the cost reads.  FP32 tensors are NHWC with the true    */
+/* channel count (no padding).                                                               */
+/* ---------------------------------------------------------------------------------------- */
+typedef struct {
+    int32_t N, H, W, C;        /* input geometry                                             */
+    int32_t K, R, S;           /* output channels, window                                    */
+    int32_t stride, pad;
+    int32_t relu;
+} fxpq_conv_f32_desc;
+
+/* y[n,p,q,o] = relu?(sum_{r,s,c} x[n, p*st+r-pad, q*st+s-pad, c] * w[o,r,s,c] + bias[o]) in fp32
+ * (fused multiply-adds, taps outside the map are zero); w KRSC fp32 [K,R,S,C], bias [K] or NULL. */
+FXPQ_API fxpq_status fxpq_conv_f32(const fxpq_conv_f32_desc* h_desc, const float* d_x, const float* d_w,
+                                   const float* d_bias, float* d_y, void* stream);
+/* k x k max-pool (taps outside the map ignored), element-wise add (+ ReLU), global average pool
+ * (fp32 sum over H x W divided by H W); fp32 NHWC. */
+FXPQ_API fxpq_status fxpq_maxpool_f32(const float* d_x, int32_t N, int32_t H, int32_t W, int32_t C, int32_t k,
+                                      int32_t stride, int32_t pad, float* d_y, void* stream);
+FXPQ_API fxpq_status fxpq_eltwise_f32(const float* d_a, const float* d_b, int64_t n, int32_t relu, float* d_y,
+                                      void* stream);
+FXPQ_API fxpq_status fxpq_avgpool_f32(const float* d_x, int32_t N, int32_t H, int32_t W, int32_t C, float* d_y,
+                                      void* stream);
+/* fp32 images NCHW -> NHWC (the FP32 network's input). */
+FXPQ_API fxpq_status fxpq_nchw_to_nhwc_f32(const float* d_x, int32_t N, int32_t C, int32_t H, int32_t W, float* d_y,
+                                           void* stream);
+/* Values of an fp16 code tensor [npix, Cp] (planes per fmt.bits) as fp32 [npix, C]: code * 2^-fl
+ * (the binary quantizer's codes decoded 0 -> +1 first); exact. */
+FXPQ_API fxpq_status fxpq_dequantize(const void* d_codes, int64_t npix, int32_t Cp, int32_t C, fxpq_fmt fmt,
+                                     float* d_y, void* stream);
+/* In place on fp32 [npix, K]: y += bias[k] (bias may be NULL), then ReLU if relu: the FP32 bias of a
+ * layer whose weights are already fixed point (the contraction ran in FXPQ_OUT_F32 mode). */
+FXPQ_API fxpq_status fxpq_bias_relu_f32(float* d_y, int64_t npix, int32_t K, const float* d_bias, int32_t relu,
+                                        void* stream);
+/* Statistics of one data-structure of n_samples x nu fp32 values, the terms of Eq. CPB_QE: d_out
+ * (device double[3 + 2 n_samples]) = { L = sum (x - Q(x; fmt))^2 (Eq. DSB_QE, fp64 sums), min, max,
+ * then per sample sum x, sum x^2 } (the dispersion of Eq. importance follows on the host).  d_ws:
+ * 8 bytes of device scratch.  n_samples <= 65535. */
+FXPQ_API fxpq_status fxpq_ds_stats(const float* d_x, int32_t n_samples, int64_t nu, fxpq_fmt fmt, double* d_out,
+                                   void* d_ws, void* stream);
+/* |C_i| of Eqs. unclassified_samples / mispredicted_classes: per sample the number of classes whose
+ * logit equals the largest.  Logits [N, C]: fp32, or exact int64 C-Block values when is_int64. */
+FXPQ_API fxpq_status fxpq_top1_ties(const void* d_logits, int32_t is_int64, int32_t N, int32_t C,
+                                    int32_t* d_counts, void* stream);
+
 /* Synchronises `stream`, returns and clears the latched device status (FXPQ_OK if none). */
 FXPQ_API fxpq_status fxpq_get_device_status(void* stream);
 

@@ -52,6 +52,11 @@ class OpDesc(ctypes.Structure):
                 ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
 
 
+class ConvF32Desc(ctypes.Structure):
+    _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("K", I32), ("R", I32), ("S", I32),
+                ("stride", I32), ("pad", I32), ("relu", I32)]
+
+
 class Net(ctypes.Structure):
     _fields_ = [("n_ops", I32), ("n_slots", I32), ("C", I32), ("H", I32), ("W", I32), ("Cp_in", I32),
                 ("fmt_in", Fmt), ("ops", ctypes.POINTER(OpDesc))]
@@ -82,6 +87,15 @@ _SIGS = {
     "fxpq_pack_codes": (I32, [VP, I64, Fmt, VP, VP]),
     "fxpq_unpack_codes": (I32, [VP, I64, Fmt, VP, VP]),
     "fxpq_net_memory": (I32, [ctypes.POINTER(Net), I32, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
+    "fxpq_conv_f32": (I32, [ctypes.POINTER(ConvF32Desc), VP, VP, VP, VP, VP]),
+    "fxpq_maxpool_f32": (I32, [VP, I32, I32, I32, I32, I32, I32, I32, VP, VP]),
+    "fxpq_eltwise_f32": (I32, [VP, VP, I64, I32, VP, VP]),
+    "fxpq_avgpool_f32": (I32, [VP, I32, I32, I32, I32, VP, VP]),
+    "fxpq_dequantize": (I32, [VP, I64, I32, I32, Fmt, VP, VP]),
+    "fxpq_bias_relu_f32": (I32, [VP, I64, I32, VP, I32, VP]),
+    "fxpq_ds_stats": (I32, [VP, I32, I64, Fmt, VP, VP, VP]),
+    "fxpq_top1_ties": (I32, [VP, I32, I32, I32, VP, VP]),
+    "fxpq_nchw_to_nhwc_f32": (I32, [VP, I32, I32, I32, I32, VP, VP]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),
     "fxpq_conv_workspace": (SZ, [ctypes.POINTER(ConvDesc)]),
     "fxpq_conv_fwd": (I32, [ctypes.POINTER(ConvDesc), VP, VP, VP, VP, ctypes.POINTER(I32), VP, SZ, VP]),

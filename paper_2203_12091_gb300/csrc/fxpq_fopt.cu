@@ -1,0 +1,369 @@
+// fxpq_fopt.cu -- the forward optimizer's FP32 side (Sec. IV-C, Alg. 1 and its cost F): while one
+// data-structure's QPs are searched, every later layer runs in FP32, and the cost needs each
+// data-structure's quantization error, range and dispersion and the logits' top-1 ties.
+//   conv / max-pool / eltwise / global avg-pool in fp32 (NHWC, true channel counts);
+//   code tensors -> fp32 values; fp32 bias + ReLU after an integer contraction;
+//   per-data-structure statistics (L of Eq. DSB_QE at one format, min, max, per-sample moments);
+//   top-1 tie counts of logits (fp32 or exact int64).
+#include <math.h>
+
+#include "fxpq_common.cuh"
+
+namespace fxpq {
+namespace {
+
+// ------------------------------------------------------------------ fp32 implicit-GEMM convolution
+// Tile 64 output pixels x 64 output channels, 16 reduction steps per stage, 256 threads with 4 x 4
+// outputs each.  x: [N, H, W, C]; w: [K, R*S*C] (KRSC); y: [N, P, Q, K].
+constexpr int CF_BM = 64, CF_BN = 64, CF_BK = 16;
+
+struct ConvF32Args {
+    const float* x;
+    const float* w;
+    const float* bias;
+    float* y;
+    int N, H, W, C, K, R, S, stride, pad, P, Q, relu;
+    long long M;
+};
+
+__global__ void __launch_bounds__(256) conv_f32_kernel(const ConvF32Args a) {
+    __shared__ float sa[CF_BK][CF_BM + 4];
+    __shared__ float sb[CF_BK][CF_BN + 4];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const long long m0 = (long long)blockIdx.x * CF_BM;
+    const int n0 = blockIdx.y * CF_BN;
+    const int RSC = a.R * a.S * a.C;
+    // the A element this thread stages: pixel row (threadIdx.x / 4) and reduction columns 4 * (tid % 4) ..
+    const int lr = threadIdx.x >> 2, lk = (threadIdx.x & 3) * 4;
+    const long long m = m0 + lr;
+    int pn = 0, pp = 0, pq = 0;
+    if (m < a.M) {
+        pn = (int)(m / ((long long)a.P * a.Q));
+        const int rem = (int)(m - (long long)pn * a.P * a.Q);
+        pp = rem / a.Q;
+        pq = rem - pp * a.Q;
+    }
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < RSC; k0 += CF_BK) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int kk = k0 + lk + e;
+            float v = 0.0f;
+            if (m < a.M && kk < RSC) {
+                const int c = kk % a.C, rs = kk / a.C;
+                const int s = rs % a.S, r = rs / a.S;
+                const int h = pp * a.stride + r - a.pad, ww = pq * a.stride + s - a.pad;
+                if (h >= 0 && h < a.H && ww >= 0 && ww < a.W) v = a.x[(((long long)pn * a.H + h) * a.W + ww) * a.C + c];
+            }
+            sa[lk + e][lr] = v;
+            const int o = n0 + lr;
+            sb[lk + e][lr] = (o < a.K && kk < RSC) ? a.w[(long long)o * RSC + kk] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < CF_BK; ++kk) {
+            float av[4], bv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) av[i] = sa[kk][ty * 4 + i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) bv[j] = sb[kk][tx * 4 + j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const long long mm = m0 + ty * 4 + i;
+        if (mm >= a.M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int o = n0 + tx * 4 + j;
+            if (o >= a.K) continue;
+            float v = acc[i][j];
+            if (a.bias) v += a.bias[o];
+            if (a.relu) v = fmaxf(v, 0.0f);
+            a.y[mm * a.K + o] = v;
+        }
+    }
+}
+
+__global__ void maxpool_f32_kernel(const float* __restrict__ x, int N, int H, int W, int C, int k, int stride, int pad,
+                                   int P, int Q, float* __restrict__ y) {
+    const long long total = (long long)N * P * Q * C;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        const long long pix = i / C;
+        const int q = (int)(pix % Q), p = (int)((pix / Q) % P);
+        const long long n = pix / ((long long)P * Q);
+        float best = -INFINITY;
+        for (int r = 0; r < k; ++r) {
+            const int h = p * stride + r - pad;
+            if (h < 0 || h >= H) continue;
+            for (int s = 0; s < k; ++s) {
+                const int w = q * stride + s - pad;
+                if (w >= 0 && w < W) best = fmaxf(best, x[((n * H + h) * W + w) * C + c]);
+            }
+        }
+        y[i] = best;
+    }
+}
+
+__global__ void eltwise_f32_kernel(const float* __restrict__ a, const float* __restrict__ b, long long n, int relu,
+                                   float* __restrict__ y) {
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const float v = a[i] + b[i];
+        y[i] = relu ? fmaxf(v, 0.0f) : v;
+    }
+}
+
+// one thread per (n, c): the mean over H x W (sum in fp32, then divided by H W)
+__global__ void avgpool_f32_kernel(const float* __restrict__ x, int N, int HW, int C, float* __restrict__ y) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (long long)N * C) return;
+    const long long n = i / C;
+    const int c = (int)(i % C);
+    float s = 0.0f;
+    for (int p = 0; p < HW; ++p) s += x[(n * HW + p) * C + c];
+    y[i] = s / (float)HW;
+}
+
+// fp16 code tensor [npix, Cp] (planes) -> fp32 values [npix, C]; the binary quantizer's codes decode
+// 0 -> +1, -1 -> -1
+__global__ void dequantize_kernel(const __half* __restrict__ codes, long long npix, int Cp, int C, int planes, float scale,
+                                  int binary, float* __restrict__ y) {
+    const long long total = npix * C;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+        const long long pix = i / C;
+        const int c = (int)(i - pix * C);
+        int code = code_get(codes, pix * Cp + c, planes, npix * Cp);
+        if (binary) code = 2 * code + 1;
+        y[i] = (float)code * scale;  // exact: |code| < 2^17 and scale a power of two
+    }
+}
+
+__global__ void bias_relu_f32_kernel(float* __restrict__ y, long long npix, int K, const float* __restrict__ bias,
+                                     int relu) {
+    const long long total = npix * K;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+        float v = y[i];
+        if (bias) v += bias[i % K];
+        y[i] = relu ? fmaxf(v, 0.0f) : v;
+    }
+}
+
+__device__ __forceinline__ unsigned ord_key(float x) {
+    const unsigned u = __float_as_uint(x);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Statistics of one data-structure of n_samples x nu fp32 values under format (k, S, fl):
+// out[0] += sum (x - Q(x))^2, out[3 + 2 s] += sum x and out[4 + 2 s] += sum x^2 of sample s; the
+// smallest and largest values as order keys in keys[0], keys[1] (ds_stats_finish_kernel converts
+// them into out[1], out[2]).  Blocks never straddle samples: grid.y = sample.
+__global__ void ds_stats_kernel(const float* __restrict__ x, long long nu, int k, int S, int fl, double* out,
+                                unsigned* keys) {
+    const int s = blockIdx.y;
+    const float* xs = x + (long long)s * nu;
+    const double scale = ldexp(1.0, fl), inv = ldexp(1.0, -fl);
+    const double lo = S ? -ldexp(1.0, k - 1) : 0.0, hi = ldexp(1.0, k - S) - 1.0;
+    const bool binary = k == 1 && S == 1;
+    double l2 = 0.0, s1 = 0.0, s2 = 0.0;
+    unsigned mn = 0xFFFFFFFFu, mx = 0u;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nu; i += (long long)gridDim.x * blockDim.x) {
+        const float v = xs[i];
+        const double d = (double)v;
+        double q;
+        if (binary) {
+            q = v < 0.0f ? -inv : inv;
+        } else {
+            q = fmin(fmax(nearbyint(d * scale), lo), hi) * inv;  // round half to even, clip
+        }
+        const double e = d - q;
+        l2 += e * e;
+        s1 += d;
+        s2 += d * d;
+        const unsigned key = ord_key(v);
+        mn = min(mn, key);
+        mx = max(mx, key);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        l2 += __shfl_xor_sync(0xFFFFFFFFu, l2, off);
+        s1 += __shfl_xor_sync(0xFFFFFFFFu, s1, off);
+        s2 += __shfl_xor_sync(0xFFFFFFFFu, s2, off);
+        mn = min(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, off));
+        mx = max(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, off));
+    }
+    if ((threadIdx.x & 31) == 0) {
+        atomicAdd(out, l2);
+        atomicAdd(out + 3 + 2 * s, s1);
+        atomicAdd(out + 4 + 2 * s, s2);
+        atomicMin(keys, mn);
+        atomicMax(keys + 1, mx);
+    }
+}
+
+__global__ void ds_stats_init_kernel(unsigned* keys) {
+    keys[0] = 0xFFFFFFFFu;
+    keys[1] = 0u;
+}
+
+__global__ void ds_stats_finish_kernel(double* out, const unsigned* keys) {
+    const unsigned kmn = keys[0], kmx = keys[1];
+    const unsigned umn = (kmn & 0x80000000u) ? (kmn & 0x7FFFFFFFu) : ~kmn;
+    const unsigned umx = (kmx & 0x80000000u) ? (kmx & 0x7FFFFFFFu) : ~kmx;
+    out[1] = (double)__uint_as_float(umn);
+    out[2] = (double)__uint_as_float(umx);
+}
+
+// one warp per sample: the number of classes whose logit equals the sample's largest
+template <typename T>
+__global__ void top1_ties_kernel(const T* __restrict__ logits, int N, int C, int32_t* __restrict__ counts) {
+    const int n = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (n >= N) return;
+    const T* row = logits + (long long)n * C;
+    T best = row[0];
+    for (int c = lane; c < C; c += 32) best = row[c] > best ? row[c] : best;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const T o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
+        best = o > best ? o : best;
+    }
+    int cnt = 0;
+    for (int c = lane; c < C; c += 32) cnt += row[c] == best ? 1 : 0;
+    cnt = __reduce_add_sync(0xFFFFFFFFu, (unsigned)cnt);
+    if (lane == 0) counts[n] = cnt;
+}
+
+__global__ void nchw_to_nhwc_kernel(const float* __restrict__ x, int N, int C, int HW, float* __restrict__ y) {
+    const long long total = (long long)N * C * HW;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(i % C);
+        const long long pix = i / C;  // n * HW + p
+        const long long n = pix / HW;
+        y[i] = x[(n * C + c) * HW + (pix - n * HW)];
+    }
+}
+
+int grid_of(long long work) {
+    long long b = (work + 255) / 256;
+    if (b < 1) b = 1;
+    if (b > 152LL * 16) b = 152LL * 16;
+    return (int)b;
+}
+
+}  // namespace
+}  // namespace fxpq
+
+using namespace fxpq;
+
+extern "C" fxpq_status fxpq_conv_f32(const fxpq_conv_f32_desc* h_desc, const float* d_x, const float* d_w,
+                                     const float* d_bias, float* d_y, void* stream) {
+    if (!h_desc) return FXPQ_ERR_INVALID_ARG;
+    const fxpq_conv_f32_desc& d = *h_desc;
+    if (d.N < 0 || d.H < 1 || d.W < 1 || d.C < 1 || d.K < 1 || d.R < 1 || d.S < 1 || d.stride < 1 || d.pad < 0)
+        return FXPQ_ERR_INVALID_ARG;
+    const int P = (d.H + 2 * d.pad - d.R) / d.stride + 1, Q = (d.W + 2 * d.pad - d.S) / d.stride + 1;
+    if (P < 1 || Q < 1) return FXPQ_ERR_INVALID_ARG;
+    if (d.N > 0 && (!d_x || !d_w || !d_y)) return FXPQ_ERR_INVALID_ARG;
+    ConvF32Args a{d_x, d_w, d_bias, d_y, d.N, d.H, d.W, d.C, d.K, d.R, d.S, d.stride, d.pad, P, Q, d.relu ? 1 : 0,
+                  (long long)d.N * P * Q};
+    if (a.M == 0) return FXPQ_OK;
+    dim3 grid((unsigned)((a.M + CF_BM - 1) / CF_BM), (unsigned)((d.K + CF_BN - 1) / CF_BN));
+    conv_f32_kernel<<<grid, 256, 0, as_stream(stream)>>>(a);
+    return after_launch("conv_f32");
+}
+
+extern "C" fxpq_status fxpq_maxpool_f32(const float* d_x, int32_t N, int32_t H, int32_t W, int32_t C, int32_t k,
+                                        int32_t stride, int32_t pad, float* d_y, void* stream) {
+    if (N < 0 || H < 1 || W < 1 || C < 1 || k < 1 || stride < 1 || pad < 0 || pad >= k) return FXPQ_ERR_INVALID_ARG;
+    const int P = (H + 2 * pad - k) / stride + 1, Q = (W + 2 * pad - k) / stride + 1;
+    if (P < 1 || Q < 1 || (N > 0 && (!d_x || !d_y))) return FXPQ_ERR_INVALID_ARG;
+    const long long total = (long long)N * P * Q * C;
+    if (total == 0) return FXPQ_OK;
+    maxpool_f32_kernel<<<grid_of(total), 256, 0, as_stream(stream)>>>(d_x, N, H, W, C, k, stride, pad, P, Q, d_y);
+    return after_launch("maxpool_f32");
+}
+
+extern "C" fxpq_status fxpq_eltwise_f32(const float* d_a, const float* d_b, int64_t n, int32_t relu, float* d_y,
+                                        void* stream) {
+    if (n < 0 || (n > 0 && (!d_a || !d_b || !d_y))) return FXPQ_ERR_INVALID_ARG;
+    if (n == 0) return FXPQ_OK;
+    eltwise_f32_kernel<<<grid_of(n), 256, 0, as_stream(stream)>>>(d_a, d_b, n, relu, d_y);
+    return after_launch("eltwise_f32");
+}
+
+extern "C" fxpq_status fxpq_avgpool_f32(const float* d_x, int32_t N, int32_t H, int32_t W, int32_t C, float* d_y,
+                                        void* stream) {
+    if (N < 0 || H < 1 || W < 1 || C < 1 || (N > 0 && (!d_x || !d_y))) return FXPQ_ERR_INVALID_ARG;
+    const long long total = (long long)N * C;
+    if (total == 0) return FXPQ_OK;
+    avgpool_f32_kernel<<<(unsigned)((total + 255) / 256), 256, 0, as_stream(stream)>>>(d_x, N, H * W, C, d_y);
+    return after_launch("avgpool_f32");
+}
+
+extern "C" fxpq_status fxpq_dequantize(const void* d_codes, int64_t npix, int32_t Cp, int32_t C, fxpq_fmt fmt,
+                                       float* d_y, void* stream) {
+    if (npix < 0 || C < 1 || Cp < C || !fmt_ok1(fmt) || (npix > 0 && (!d_codes || !d_y))) return FXPQ_ERR_INVALID_ARG;
+    if (npix == 0) return FXPQ_OK;
+    dequantize_kernel<<<grid_of(npix * C), 256, 0, as_stream(stream)>>>(
+        static_cast<const __half*>(d_codes), npix, Cp, C, planes_of(fmt), ldexpf(1.0f, -fmt.fl),
+        fmt.bits == 1 && fmt.is_signed == 1, d_y);
+    return after_launch("dequantize");
+}
+
+extern "C" fxpq_status fxpq_bias_relu_f32(float* d_y, int64_t npix, int32_t K, const float* d_bias, int32_t relu,
+                                          void* stream) {
+    if (npix < 0 || K < 1 || (npix > 0 && !d_y)) return FXPQ_ERR_INVALID_ARG;
+    if (npix == 0) return FXPQ_OK;
+    bias_relu_f32_kernel<<<grid_of(npix * K), 256, 0, as_stream(stream)>>>(d_y, npix, K, d_bias, relu);
+    return after_launch("bias_relu_f32");
+}
+
+extern "C" fxpq_status fxpq_ds_stats(const float* d_x, int32_t n_samples, int64_t nu, fxpq_fmt fmt, double* d_out,
+                                     void* d_ws, void* stream) {
+    if (n_samples < 1 || n_samples > 65535 || nu < 1 || !fmt_ok1(fmt, 32) || !d_x || !d_out || !d_ws)
+        return FXPQ_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (cudaMemsetAsync(d_out, 0, sizeof(double) * (3 + 2 * (size_t)n_samples), s) != cudaSuccess) return FXPQ_ERR_CUDA;
+    ds_stats_init_kernel<<<1, 1, 0, s>>>(static_cast<unsigned*>(d_ws));
+    fxpq_status st = after_launch("ds_stats_init");
+    if (st != FXPQ_OK) return st;
+    long long bx = (nu + 255) / 256;
+    const long long cap = (152LL * 8 + n_samples - 1) / n_samples;
+    if (bx > cap) bx = cap;
+    if (bx < 1) bx = 1;
+    ds_stats_kernel<<<dim3((unsigned)bx, (unsigned)n_samples), 256, 0, s>>>(d_x, nu, fmt.bits, fmt.is_signed, fmt.fl,
+                                                                          d_out, static_cast<unsigned*>(d_ws));
+    st = after_launch("ds_stats");
+    if (st != FXPQ_OK) return st;
+    ds_stats_finish_kernel<<<1, 1, 0, s>>>(d_out, static_cast<const unsigned*>(d_ws));
+    return after_launch("ds_stats_finish");
+}
+
+extern "C" fxpq_status fxpq_top1_ties(const void* d_logits, int32_t is_int64, int32_t N, int32_t C, int32_t* d_counts,
+                                      void* stream) {
+    if (N < 0 || C < 1 || (N > 0 && (!d_logits || !d_counts))) return FXPQ_ERR_INVALID_ARG;
+    if (N == 0) return FXPQ_OK;
+    const unsigned blocks = (unsigned)((N + 7) / 8);
+    if (is_int64)
+        top1_ties_kernel<long long><<<blocks, 256, 0, as_stream(stream)>>>(static_cast<const long long*>(d_logits), N, C,
+                                                                           d_counts);
+    else
+        top1_ties_kernel<float><<<blocks, 256, 0, as_stream(stream)>>>(static_cast<const float*>(d_logits), N, C,
+                                                                       d_counts);
+    return after_launch("top1_ties");
+}
+
+extern "C" fxpq_status fxpq_nchw_to_nhwc_f32(const float* d_x, int32_t N, int32_t C, int32_t H, int32_t W, float* d_y,
+                                             void* stream) {
+    if (N < 0 || C < 1 || H < 1 || W < 1 || (N > 0 && (!d_x || !d_y))) return FXPQ_ERR_INVALID_ARG;
+    const long long total = (long long)N * C * H * W;
+    if (total == 0) return FXPQ_OK;
+    nchw_to_nhwc_kernel<<<grid_of(total), 256, 0, as_stream(stream)>>>(d_x, N, C, H * W, d_y);
+    return after_launch("nchw_to_nhwc");
+}

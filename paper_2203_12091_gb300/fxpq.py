@@ -160,6 +160,55 @@ def fxpq_net_memory(net, fp32: bool):
     return rw.value, ro.value
 
 
+# ------------------------------------------------------------------------------ forward optimizer support
+def fxpq_conv_f32(N, H, W, C, K, R, S, stride, pad, relu, x, w, bias, y, stream=None):
+    d = L.ConvF32Desc(N, H, W, C, K, R, S, stride, pad, int(relu))
+    L.check("fxpq_conv_f32", L.lib().fxpq_conv_f32(ctypes.byref(d), _p(x), _p(w), _p(bias), _p(y), _s(stream)))
+    return y
+
+
+def fxpq_maxpool_f32(x, N, H, W, C, k, stride, pad, y, stream=None):
+    L.check("fxpq_maxpool_f32", L.lib().fxpq_maxpool_f32(_p(x), N, H, W, C, k, stride, pad, _p(y), _s(stream)))
+    return y
+
+
+def fxpq_eltwise_f32(a, b, n, relu, y, stream=None):
+    L.check("fxpq_eltwise_f32", L.lib().fxpq_eltwise_f32(_p(a), _p(b), n, int(relu), _p(y), _s(stream)))
+    return y
+
+
+def fxpq_avgpool_f32(x, N, H, W, C, y, stream=None):
+    L.check("fxpq_avgpool_f32", L.lib().fxpq_avgpool_f32(_p(x), N, H, W, C, _p(y), _s(stream)))
+    return y
+
+
+def fxpq_nchw_to_nhwc_f32(x, N, C, H, W, y, stream=None):
+    L.check("fxpq_nchw_to_nhwc_f32", L.lib().fxpq_nchw_to_nhwc_f32(_p(x), N, C, H, W, _p(y), _s(stream)))
+    return y
+
+
+def fxpq_dequantize(codes, npix, Cp, C, f: Fmt, y, stream=None):
+    L.check("fxpq_dequantize", L.lib().fxpq_dequantize(_p(codes), npix, Cp, C, f, _p(y), _s(stream)))
+    return y
+
+
+def fxpq_bias_relu_f32(y, npix, K, bias, relu, stream=None):
+    L.check("fxpq_bias_relu_f32", L.lib().fxpq_bias_relu_f32(_p(y), npix, K, _p(bias), int(relu), _s(stream)))
+    return y
+
+
+def fxpq_ds_stats(x, n_samples, nu, f: Fmt, out, ws, stream=None):
+    """out: device float64[3 + 2 n_samples]; ws: 8 bytes of device scratch."""
+    L.check("fxpq_ds_stats", L.lib().fxpq_ds_stats(_p(x), n_samples, nu, f, _p(out), _p(ws), _s(stream)))
+    return out
+
+
+def fxpq_top1_ties(logits, N, C, counts, stream=None):
+    is64 = 1 if logits.dtype == torch.int64 else 0
+    L.check("fxpq_top1_ties", L.lib().fxpq_top1_ties(_p(logits), is64, N, C, _p(counts), _s(stream)))
+    return counts
+
+
 def fxpq_bn_to_scale(gamma, beta, mean, var, eps, aleph1, aleph2, stream=None):
     """BN -> Scale layer parameters (fp32 device tensors of one length)."""
     L.check("fxpq_bn_to_scale", L.lib().fxpq_bn_to_scale(_p(gamma), _p(beta), _p(mean), _p(var), gamma.numel(),

@@ -118,6 +118,7 @@ def test_struct_layout_matches_header(tmp_path):
         pytest.skip("no host C compiler")
     mirrors = {"fxpq_fmt": L.Fmt, "fxpq_stats": L.Stats, "fxpq_fl_search_item": L.FlSearchItem,
                "fxpq_quantize_item": L.QuantizeItem, "fxpq_conv_desc": L.ConvDesc, "fxpq_op_desc": L.OpDesc,
+               "fxpq_conv_f32_desc": L.ConvF32Desc,
                "fxpq_net": L.Net}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "fxpq.h"', "int main(void) {"]
     for cname, py in mirrors.items():
