@@ -312,6 +312,8 @@ def run_kernel(args):
     flsearch : FL search over 64M N(0,1) fp32 values, one wordlength (k=8) and the full 15 x 32 grid, with
                the L2 score and with the L1 score (k = 1..16 for the sweep);
     quantize : Q of 64M N(0,1) fp32 values to int8 codes and to an fp16 code tensor (HBM-bound);
+    fopt     : the forward optimizer (Alg. 1, cost F) on ResNet-18 with 8 calibration images, and its fp32
+               convolution;
     forward  : the integer forward of the workload (first plan, calibrated once), fxpq_net_forward alone."""
     import torch
     import __graft_entry__ as g
@@ -400,6 +402,52 @@ def run_kernel(args):
             ms = sum(ts) / len(ts)
             gbs = 2.5 * n / (ms / 1e3) / 1e9
             out[name] = {"ms": round(ms, 4), "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 3)}
+    if args.kernel in ("fopt", "all"):
+        # the forward optimizer (Alg. 1 with the cost F) on ResNet-18, 8 calibration images at 224 x 224:
+        # the first 12 data-structures, every candidate's cost over the whole network
+        from paper_2203_12091_gb300.fopt import ForwardOptimizer
+        wdev, _ = device_params("resnet18", 6, torch.device("cuda"))
+        imgs = torch.from_numpy(synth.images(8, 6)).cuda()
+        plan = synth.bit_plan("resnet18", 6)
+        t0 = time.perf_counter()
+        fo = ForwardOptimizer(synth.resnet18(), wdev, imgs, plan)
+        torch.cuda.synchronize()
+        t_init = time.perf_counter() - t0
+        n_eval = [0]
+        cost0 = fo.cost
+
+        def counted(cur, fl):
+            n_eval[0] += 1
+            return cost0(cur, fl)
+
+        fo.cost = counted
+        t0 = time.perf_counter()
+        res = fo.run(1, 12)
+        torch.cuda.synchronize()
+        dt = time.perf_counter() - t0
+        out["fopt"] = {"workload": "resnet18 224x224, 8 calibration images, K=1, first 12 data-structures",
+                       "init_s": round(t_init, 3), "s": round(dt, 3), "cost_evals": n_eval[0],
+                       "ms_per_cost_eval": round(1e3 * dt / max(n_eval[0], 1), 2),
+                       "data_structures_s": round(len(res) / dt, 2)}
+        # the fp32 convolution of the FP32 side on a ResNet-18 stage-2 shape: 8 x 56 x 56 x 64 -> 64, 3 x 3
+        N, H, C, K = 8, 56, 64, 64
+        x = torch.randn(N * H * H * C, device="cuda")
+        w = torch.randn(K * 9 * C, device="cuda")
+        y = torch.empty(N * H * H * K, device="cuda")
+        ts = []
+        for i in range(args.warmup + args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            F.fxpq_conv_f32(N, H, H, C, K, 3, 3, 1, 1, True, x, w, None, y)
+            e1.record()
+            e1.synchronize()
+            if i >= args.warmup:
+                ts.append(e0.elapsed_time(e1))
+        ms = sum(ts) / len(ts)
+        tf = 2.0 * N * H * H * K * 9 * C / (ms / 1e3) / 1e12
+        peak = 152 * 128 * 2 * 2.07e9 / 1e12  # fp32 FMA lanes x 2 FLOP x max SM clock
+        out["conv_f32"] = {"ms": round(ms, 4), "tflops": round(tf, 2), "peak_fp32_tflops": round(peak, 1),
+                           "frac": round(tf / peak, 3)}
     if args.kernel in ("forward", "all"):
         # the integer forward of the bench workload alone (one plan, calibrated once): the target of the
         # per-launch DRAM traffic capture of the conv kernels
@@ -430,7 +478,7 @@ def run_kernel(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "forward", "all"],
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "fopt", "forward", "all"],
                     help="time one kernel case and exit")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)

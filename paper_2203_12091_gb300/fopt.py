@@ -90,12 +90,7 @@ class ForwardOptimizer:
     def _stats(self, x, n_samples, nu, fmt):
         out = self._stats_out[: 3 + 2 * n_samples]
         F.fxpq_ds_stats(x, n_samples, nu, fmt, out, self._stats_ws, self.stream)
-        h = out.cpu().tolist()
-        sig = 0.0
-        for s in range(n_samples):
-            m1, m2 = h[3 + 2 * s] / nu, h[4 + 2 * s] / nu
-            sig += math.sqrt(max(m2 - m1 * m1, 0.0))
-        return {"L": h[0], "min": h[1], "max": h[2], "sigma": sig / n_samples, "nu": nu}
+        return _decode(out.cpu().tolist(), 0, n_samples, nu)
 
     # ------------------------------------------------------------------ helpers
     def _src(self, i, L_):
@@ -290,23 +285,38 @@ class ForwardOptimizer:
         """F = E + UnClass + MisPred for cur at FL cand_fl: (F, E, UnClass, MisPred)."""
         X, logits = self.forward(cur, cand_fl)
         start = self.names.index(cur[0])
-        E = 0.0
+        # every statistic and the tie counts into one device buffer, read back once
+        layers = []
+        off = 0
         for nm in self.names[start:]:
             terms = [(j, X[(nm, j)]) for j in ("a", "w", "b") if (nm, j) in X]
-            if not terms:
-                continue
-            st = {j: self._stats(t.reshape(-1), n_s, nu, f) for j, (t, f, n_s, nu) in terms}
+            if terms:
+                layers.append([(j, t, f, n_s, nu, off + 0) for j, (t, f, n_s, nu) in terms])
+                for _, _, _, n_s, _, _ in layers[-1]:
+                    off += 3 + 2 * n_s
+        n_cls = self.layers[-1]["K"]
+        buf = torch.empty(off + self.N, dtype=torch.float64, device=self.dev)
+        o = 0
+        for terms in layers:
+            for i, (j, t, f, n_s, nu, _) in enumerate(terms):
+                terms[i] = (j, t, f, n_s, nu, o)
+                F.fxpq_ds_stats(t.reshape(-1), n_s, nu, f, buf[o:o + 3 + 2 * n_s], self._stats_ws, self.stream)
+                o += 3 + 2 * n_s
+        counts = buf[off:].view(torch.int32)[: self.N]
+        F.fxpq_top1_ties(logits, self.N, n_cls, counts, self.stream)
+        hb = buf.cpu()
+        h = hb[:off].tolist()
+        E = 0.0
+        for terms in layers:
+            st = {j: _decode(h, o, n_s, nu) for j, _, _, n_s, nu, o in terms}
             den = sum(v["sigma"] * v["nu"] for v in st.values())
-            for j, _ in terms:
+            for j, *_ in terms:
                 v = st[j]
                 R = v["max"] - v["min"]
                 if den == 0.0 or R == 0.0:
                     continue
                 E += (v["sigma"] * v["nu"] / den) * v["L"] / R
-        n_cls = self.layers[-1]["K"]
-        counts = self._empty(self.N, torch.int32)
-        F.fxpq_top1_ties(logits, self.N, n_cls, counts, self.stream)
-        c = counts.cpu()
+        c = hb[off:].view(torch.int32)[: self.N]
         uc = float((c > 1).sum()) / self.N
         mp = float((c - 1).sum()) / (self.N * n_cls)
         return E + uc + mp, E, uc, mp
@@ -343,3 +353,12 @@ class ForwardOptimizer:
 
 def env_size(v):
     return v.H * v.W * v.C
+
+
+def _decode(h, o, n_samples, nu):
+    """L, range ends and the mean per-sample dispersion (Eq. importance) of one fxpq_ds_stats record."""
+    sig = 0.0
+    for s in range(n_samples):
+        m1, m2 = h[o + 3 + 2 * s] / nu, h[o + 4 + 2 * s] / nu
+        sig += math.sqrt(max(m2 - m1 * m1, 0.0))
+    return {"L": h[o], "min": h[o + 1], "max": h[o + 2], "sigma": sig / n_samples, "nu": nu}
