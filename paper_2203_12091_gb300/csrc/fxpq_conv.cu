@@ -101,7 +101,39 @@ __global__ void __launch_bounds__(NT) conv_simt_kernel(ConvArgs a) {
     }
 }
 
+template <typename ACC>
+__global__ void splitk_reduce_kernel(const ConvArgs a, const ACC* __restrict__ part, int ks) {
+    const long long total = a.M * a.K;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        long long v = 0;
+        for (int s = 0; s < ks; ++s) v += (long long)part[s * total + i];
+        cblock_epilogue_store(a, i / a.K, (int)(i % a.K), v);
+    }
+}
+
 }  // namespace
+
+fxpq_status launch_splitk_reduce(const ConvArgs& a, const void* part, int ks, bool acc64, cudaStream_t st) {
+    const long long total = a.M * a.K;
+    long long blocks = (total + 255) / 256;
+    if (blocks > 152LL * 8) blocks = 152LL * 8;
+    if (blocks < 1) blocks = 1;
+    if (acc64)
+        splitk_reduce_kernel<long long><<<(unsigned)blocks, 256, 0, st>>>(a, static_cast<const long long*>(part), ks);
+    else
+        splitk_reduce_kernel<int><<<(unsigned)blocks, 256, 0, st>>>(a, static_cast<const int*>(part), ks);
+    return after_launch("splitk_reduce");
+}
+
+// At most 16 shares of int64 sums, for layers whose M x K outputs are small enough for the split to pay
+// (it is taken only when the tiles cannot occupy the SMs); capped at 64 MiB.
+size_t conv_split_ws_bytes(long long M, int K) {
+    const size_t one = (size_t)M * (size_t)K * sizeof(long long);
+    const size_t cap = (size_t)64 << 20;
+    if (M <= 0 || K <= 0 || 2 * one > cap) return 0;
+    return 16 * one < cap ? 16 * one : cap;
+}
 
 // Host-side planning shared by conv and gemm: fills ConvArgs, checks the integer bounds.
 fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, const int32_t* bias, void* y,
@@ -216,12 +248,13 @@ static bool tc_path_enabled() {
     return !(e && strcmp(e, "simt") == 0);
 }
 
-fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st) {
+fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st, void* ws,
+                        size_t ws_bytes) {
     const long long M = (long long)a.N * a.P * a.Q;
     if (M == 0) return FXPQ_OK;
     if (tc_path_enabled()) {
         bool launched = false;
-        fxpq_status s = launch_conv_tc(a, d, st, launched);
+        fxpq_status s = launch_conv_tc(a, d, st, launched, ws, ws_bytes);
         if (s != FXPQ_OK || launched) return s;
     }
     dim3 grid((unsigned)((M + TM - 1) / TM), (unsigned)((a.K + TN - 1) / TN));
@@ -237,21 +270,23 @@ fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64,
 using namespace fxpq;
 
 extern "C" size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc) {
-    (void)h_desc;
-    return 0;
+    if (!h_desc || h_desc->N < 1 || h_desc->stride < 1 || h_desc->R < 1 || h_desc->S < 1) return 0;
+    const int P = (h_desc->H + 2 * h_desc->pad - h_desc->R) / h_desc->stride + 1;
+    const int Q = (h_desc->W + 2 * h_desc->pad - h_desc->S) / h_desc->stride + 1;
+    if (P < 1 || Q < 1) return 0;
+    return conv_split_ws_bytes((long long)h_desc->N * P * Q, h_desc->K);
 }
 
 extern "C" fxpq_status fxpq_conv_fwd(const fxpq_conv_desc* h_desc, const void* d_x, const void* d_w,
                                      const int32_t* d_bias, void* d_y, int32_t* h_out_scale, void* d_ws,
                                      size_t ws_bytes, void* stream) {
-    (void)d_ws;
-    (void)ws_bytes;
     if (!h_desc) return FXPQ_ERR_INVALID_ARG;
+    if (d_ws && !aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
     ConvArgs a;
     bool need64 = false;
     fxpq_status st = plan_conv(*h_desc, d_x, d_w, d_bias, d_y, a, h_out_scale, need64);
     if (st != FXPQ_OK) return st;
-    return launch_conv(a, *h_desc, need64, as_stream(stream));
+    return launch_conv(a, *h_desc, need64, as_stream(stream), d_ws, d_ws ? ws_bytes : 0);
 }
 
 extern "C" fxpq_status fxpq_gemm(const void* d_x, fxpq_fmt fmt_x, const void* d_w, fxpq_fmt fmt_w,

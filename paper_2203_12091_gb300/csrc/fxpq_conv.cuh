@@ -117,8 +117,16 @@ __device__ __forceinline__ void cblock_epilogue_store(const ConvArgs& a, long lo
 
 fxpq_status plan_conv(const fxpq_conv_desc& d, const void* x, const void* w, const int32_t* bias, void* y,
                       ConvArgs& a, int32_t* out_scale, bool& need64);
-fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st);
-// Tensor-core path; sets launched = false when the shape needs the CUDA-core kernel instead.
-fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched);
+fxpq_status launch_conv(const ConvArgs& a, const fxpq_conv_desc& d, bool need64, cudaStream_t st, void* ws,
+                        size_t ws_bytes);
+// Tensor-core path; sets launched = false when the shape needs the CUDA-core kernel instead.  ws (may be
+// null): scratch for the split reduction of layers with too few tiles for the SMs.
+fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched, void* ws,
+                           size_t ws_bytes);
+// Adds the ks integer shares part[s][M][K] (int32, or int64 when acc64) of a split reduction and applies
+// the C-Block epilogue (cblock_epilogue_store) to every output.
+fxpq_status launch_splitk_reduce(const ConvArgs& a, const void* part, int ks, bool acc64, cudaStream_t st);
+// Scratch bytes a conv may use for its split reduction (0: never split).
+size_t conv_split_ws_bytes(long long M, int K);
 
 }  // namespace fxpq

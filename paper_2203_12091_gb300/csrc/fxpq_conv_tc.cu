@@ -1,5 +1,7 @@
 // fxpq_conv_tc.cu -- host side of the tensor-core C-Block (planning, tensor maps, launch) and the
 // kernels without a Scale layer; the kernel itself is in fxpq_conv_tc.cuh.
+#include <algorithm>
+
 #include "fxpq_conv_tc.cuh"
 
 namespace fxpq {
@@ -104,7 +106,8 @@ EncodeTiledFn encode_tiled() {
 }
 }  // namespace
 
-fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched) {
+fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStream_t st, bool& launched, void* ws,
+                           size_t ws_bytes) {
     launched = false;
     TcParams P;
     bool acc64 = false;
@@ -256,6 +259,48 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         launched = true;
         return FXPQ_OK;
     }
+    // Split reduction for layers whose tiles cannot occupy the SMs (FC layers, small batches) and whose
+    // reduction is long: ks units share every tile's k-blocks (share s of every exact group), and their
+    // exact integer sums meet in the workspace.
+    P.ksplit = 1;
+    P.part = nullptr;
+    P.gs[0] = 0;
+    P.gs[1] = P.n_groups;
+    if (P.patch != 3 && ws && P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
+        const int ng = P.n_groups;
+        int min_len = 1 << 30;
+        for (int gi = 0; gi < ng; ++gi) min_len = std::min(min_len, P.g[gi].kb1 - P.g[gi].kb0);
+        const size_t share = (size_t)a.M * a.K * (acc64 ? sizeof(long long) : sizeof(int));
+        const int cap = std::min(sms / P.n_tiles, (int)std::min<size_t>(ws_bytes / share, TC_MAX_SPLIT));
+        // long groups: each share takes a sub-range of every group (at least four k-blocks); many short
+        // groups (two-limb layers): each share takes whole groups
+        const int ks_sub = std::min(cap, std::min(min_len / 4, TC_MAX_GROUPS / ng));
+        const int ks_whole = std::min(cap, ng);
+        if (ks_sub >= 2 && ks_sub >= ks_whole) {
+            TcGroup g0[TC_MAX_GROUPS];
+            for (int gi = 0; gi < ng; ++gi) g0[gi] = P.g[gi];
+            for (int s = 0; s < ks_sub; ++s) {
+                for (int gi = 0; gi < ng; ++gi) {
+                    const int len = g0[gi].kb1 - g0[gi].kb0;
+                    TcGroup g = g0[gi];
+                    g.kb0 = g0[gi].kb0 + (int)((long long)len * s / ks_sub);
+                    g.kb1 = g0[gi].kb0 + (int)((long long)len * (s + 1) / ks_sub);
+                    P.g[s * ng + gi] = g;
+                }
+                P.gs[s] = s * ng;
+            }
+            P.gs[ks_sub] = ks_sub * ng;
+            P.ksplit = ks_sub;
+        } else if (ks_whole >= 2) {
+            for (int s = 0; s <= ks_whole; ++s) P.gs[s] = (int)((long long)ng * s / ks_whole);
+            P.ksplit = ks_whole;
+        }
+        if (P.ksplit > 1) {
+            P.part = ws;
+            P.fast_store = 0;
+        }
+    }
+    P.n_units = P.n_tiles * P.ksplit;
     {
         std::lock_guard<std::mutex> lk(g_tc_mu);
         if (!g_tc_attr_set) {
@@ -271,9 +316,13 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             g_tc_attr_set = true;
         }
     }
-    const int grid = P.n_tiles < sms ? P.n_tiles : sms;
+    const int grid = P.n_units < sms ? P.n_units : sms;
     launched = true;
-    if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);
+    if (a.has_scale) {
+        const fxpq_status s = launch_conv_tc_scaled(P, BN, acc64, grid, st);
+        if (s != FXPQ_OK || P.ksplit == 1) return s;
+        return launch_splitk_reduce(a, P.part, P.ksplit, acc64, st);
+    }
     if (acc64)
         conv_tc_kernel<64, long long, false><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 64)
@@ -283,7 +332,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     else
         conv_tc_kernel<256, int, false><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
     launched = true;
-    return after_launch("conv_tc");
+    const fxpq_status s = after_launch("conv_tc");
+    if (s != FXPQ_OK || P.ksplit == 1) return s;
+    return launch_splitk_reduce(a, P.part, P.ksplit, acc64, st);
 }
 
 }  // namespace fxpq

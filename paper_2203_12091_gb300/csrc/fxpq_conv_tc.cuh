@@ -60,6 +60,7 @@ constexpr size_t tc_smem_bytes() {
     return 1024 + tc_stages(BN) * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
 }
 constexpr int TC_MAX_GROUPS = 64;
+constexpr int TC_MAX_SPLIT = 16;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
 
 struct TcGroup {
@@ -88,6 +89,13 @@ struct TcParams {
     int RSC;       // R * S * Cp: reduction length of one plane
     int tiles_m, tiles_n, n_tiles;
     int n_groups;
+    // Split reduction: every tile's reduction is shared by ksplit work units, unit share s taking the
+    // groups g[gs[s]] .. g[gs[s + 1] - 1] (sub-ranges of every exact group, or whole groups); a unit
+    // writes its exact integer sums to part[s][M][K] (ACC) and a second kernel adds the shares and
+    // applies the epilogue.  Without a split, gs = {0, n_groups}.
+    int ksplit, n_units;
+    int gs[TC_MAX_SPLIT + 1];
+    void* part;
     int cp64;      // Cp % 64 == 0: a k-block never straddles a tap
     int* status;
     TcGroup g[TC_MAX_GROUPS];
@@ -478,7 +486,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+                const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+                (void)sp;
                 const int tm = t / P.tiles_n;
                 const int n_img = tm / per_img, r = tm - n_img * per_img;
                 const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
@@ -522,11 +532,13 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+                const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+                (void)sp;
                 const int tm = t / P.tiles_n, tn = t % P.tiles_n;
                 const int n_img = tm / per_img, r = tm - n_img * per_img;
                 const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
-                for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+                for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
                     const TcGroup g = P.g[gi];
                     for (int kb = g.kb0; kb < g.kb1; ++kb) {
                         if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
@@ -578,7 +590,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const __half* xb = a.x;
         uint32_t it = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            (void)sp;
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             long long rowoff[AR];  // element offset of the (r, s) = (0, 0) tap of each row (may be negative)
             int p0[AR], q0[AR];
@@ -593,7 +607,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 if (m >= a.M) p0[i] = -(1 << 20);  // rows past the end read zeros
                 rowoff[i] = (((long long)n_img * a.H + p0[i]) * a.W + q0[i]) * a.Cp;
             }
-            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+            for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const __half* xp = xb + (long long)g.a_plane * a.x_ps;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
@@ -664,12 +678,14 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
         const uint32_t run_base = (uint32_t)(nbuf * BN);
         uint32_t u = 0;  // tiles written through the staging buffer so far
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            (void)sp;
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             const long long m = tile_row(P, tm, row);  // -1: row outside the output
-            for (int gi = 0; gi < P.n_groups; ++gi) {
+            for (int gi = P.gs[sp]; gi < P.gs[sp + 1]; ++gi) {
                 const int shift = P.g[gi].shift;
-                const bool first = gi == 0, last = gi == P.n_groups - 1;
+                const bool first = gi == P.gs[sp], last = gi == P.gs[sp + 1] - 1;
                 const uint32_t buf = nbuf == 2 ? (gcount & 1) : 0;
                 const uint32_t par = nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
                 if (!wait_bounded(accfull0 + 8 * buf, par, abort, P.status)) {
@@ -856,6 +872,16 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                         mbar_arrive(accempty0 + 8 * buf);
                     }
                     if (!last) continue;
+                    if (P.ksplit > 1) {
+                        // one share of the reduction: its exact integer sums go to the partial buffer
+                        if (m >= 0) {
+                            ACC* dst = static_cast<ACC*>(P.part) + ((long long)sp * a.M + m) * a.K + k0;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)
+                                if (k0 + j < a.K) dst[j] = acc[j];
+                        }
+                        continue;
+                    }
                     if (P.fast_store) {
                         // 32 one-plane codes -> 4 swizzled 16-byte chunks of this row in the staging buffer
                         // (the epilogue constants are rebuilt here from the parameters rather than kept
@@ -952,7 +978,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = wait_bounded(wbar, 0, abort, P.status);
         tc_fence_after();
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            (void)sp;
             const uint32_t buf = gcount & 1;
             if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
                 !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
@@ -1001,8 +1029,10 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const uint64_t bdesc0 = make_sdesc(smem_u32(sB));
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
-            for (int gi = 0; gi < P.n_groups && ok; ++gi) {
+        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
+            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            (void)sp;
+            for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const uint32_t buf = P.nbuf == 2 ? (gcount & 1) : 0;
                 const uint32_t par = P.nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);

@@ -5,6 +5,7 @@
 #include <vector>
 
 #include "fxpq_common.cuh"
+#include "fxpq_conv.cuh"
 
 namespace {
 
@@ -93,6 +94,20 @@ fxpq_status plan_net(const fxpq_net* net, int32_t batch, std::vector<Slot>& slot
     return FXPQ_OK;
 }
 
+// Largest split-reduction scratch any conv op of the list may use at this batch.
+size_t net_conv_ws(const fxpq_net* net, const std::vector<Slot>& slots, int32_t batch) {
+    size_t m = 0;
+    for (int i = 0; i < net->n_ops; ++i) {
+        const fxpq_op_desc& o = net->ops[i];
+        if (o.op != FXPQ_OP_CONV) continue;
+        const Slot& s0 = slots[o.src0];
+        const int P = (s0.H + 2 * o.pad - o.R) / o.stride + 1, Q = (s0.W + 2 * o.pad - o.S) / o.stride + 1;
+        const size_t b = fxpq::conv_split_ws_bytes((long long)batch * P * Q, o.K);
+        if (b > m) m = b;
+    }
+    return align256(m);
+}
+
 }  // namespace
 
 extern "C" fxpq_status fxpq_net_memory(const fxpq_net* h_net, int32_t fp32, double* h_rw_mb, double* h_ro_mb) {
@@ -133,7 +148,7 @@ extern "C" size_t fxpq_net_workspace(const fxpq_net* h_net, int32_t batch) {
     std::vector<Slot> slots;
     size_t total = 0;
     if (plan_net(h_net, batch, slots, total) != FXPQ_OK) return 0;
-    return total + 256;
+    return total + net_conv_ws(h_net, slots, batch) + 256;
 }
 
 extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_images_nchw, int32_t batch,
@@ -148,6 +163,9 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
     char* base = static_cast<char*>(d_ws);
     auto ptr = [&](int slot) { return static_cast<void*>(base + slots[slot].offset); };
     if (batch == 0) return FXPQ_OK;
+    // the convs' split-reduction scratch follows the slots when the caller provided it
+    const size_t cws = net_conv_ws(h_net, slots, batch);
+    void* conv_ws = (cws && ws_bytes >= total + cws) ? static_cast<void*>(base + total) : nullptr;
 
     st = fxpq_quantize_images(d_images_nchw, batch, h_net->C, h_net->H, h_net->W, h_net->fmt_in, h_net->Cp_in, ptr(0),
                               stream);
@@ -182,7 +200,7 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
                 d.d_shift = o.d_shift;
                 int32_t scale = 0;
                 st = fxpq_conv_fwd(&d, ptr(o.src0), o.d_w, o.d_bias, last ? (void*)d_logits : ptr(o.dst), &scale,
-                                   nullptr, 0, stream);
+                                   conv_ws, conv_ws ? cws : 0, stream);
                 if (last && h_logits_scale) *h_logits_scale = scale;
                 break;
             }
@@ -214,7 +232,8 @@ namespace {
 
 struct CalibLayout {
     std::vector<Slot> slots;
-    size_t slots_bytes = 0, acc_off = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, total = 0;
+    size_t slots_bytes = 0, acc_off = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, cws_off = 0, cws = 0,
+           total = 0;
 };
 
 fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
@@ -234,7 +253,9 @@ fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
     L.fls_off = L.f32_off + align256((max_out > img ? max_out : img) * sizeof(float));
     L.rec_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
     L.err_off = L.rec_off + 256;
-    L.total = L.err_off + align256(32 * sizeof(double));
+    L.cws_off = L.err_off + align256(32 * sizeof(double));
+    L.cws = net_conv_ws(net, L.slots, n);
+    L.total = L.cws_off + L.cws;
     return FXPQ_OK;
 }
 
@@ -332,7 +353,8 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.d_scale = o.d_scale;
                 cd.d_shift = o.d_shift;
                 int32_t sc = 0;
-                st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, nullptr, 0, s);
+                st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, L.cws ? base + L.cws_off : nullptr,
+                                   L.cws, s);
                 if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_F32, fy, f32, s);
                 if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
                 if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_CODES, fy, ptr(o.dst), s);

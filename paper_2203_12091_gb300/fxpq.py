@@ -227,18 +227,26 @@ def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, 
                       fmt_shift if fmt_shift is not None else Fmt(16, 1, 0), _p(scale), _p(shift))
 
 
-def fxpq_conv_fwd(desc: L.ConvDesc, x, w, bias, y, stream=None) -> int:
+def fxpq_conv_workspace(desc: L.ConvDesc) -> int:
+    return L.lib().fxpq_conv_workspace(ctypes.byref(desc))
+
+
+def fxpq_conv_fwd(desc: L.ConvDesc, x, w, bias, y, stream=None, ws=None) -> int:
+    """ws: optional device workspace (fxpq_conv_workspace bytes) for the split reduction of layers with
+    too few tiles for the SMs."""
     scale = L.I32(0)
     L.check("fxpq_conv_fwd", L.lib().fxpq_conv_fwd(ctypes.byref(desc), _p(x), _p(w), _p(bias), _p(y),
-                                                   ctypes.byref(scale), None, 0, _s(stream)))
+                                                   ctypes.byref(scale), _p(ws),
+                                                   0 if ws is None else ws.numel() * ws.element_size(), _s(stream)))
     return scale.value
 
 
-def fxpq_gemm(x, fx, w, fw, bias, fb, M, N, Kdim, relu, out_mode, fy, y, stream=None) -> int:
+def fxpq_gemm(x, fx, w, fw, bias, fb, M, N, Kdim, relu, out_mode, fy, y, stream=None, ws=None) -> int:
     scale = L.I32(0)
     L.check("fxpq_gemm", L.lib().fxpq_gemm(_p(x), fx, _p(w), fw, _p(bias), fb if fb is not None else Fmt(32, 1, 0),
                                            M, N, Kdim, int(relu), out_mode, fy if fy is not None else Fmt(8, 1, 0),
-                                           _p(y), ctypes.byref(scale), None, 0, _s(stream)))
+                                           _p(y), ctypes.byref(scale), _p(ws),
+                                           0 if ws is None else ws.numel() * ws.element_size(), _s(stream)))
     return scale.value
 
 

@@ -221,7 +221,10 @@ class QNet:
             d = F.conv_desc(N, sH, sW, sCp, sCp, L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], L_["relu"],
                             out_mode, fx, self.fmts[nm]["w"], self.fmts[nm].get("b"), fy, self.w_l1.get(nm, 0),
                             scale=sq, fmt_scale=self.fmts[nm].get("s"), shift=hq, fmt_shift=self.fmts[nm].get("h"))
-            s = F.fxpq_conv_fwd(d, x, wq, bq, y, stream)
+            nws = F.fxpq_conv_workspace(d)
+            if nws and (getattr(self, "_cws", None) is None or self._cws.numel() < nws):
+                self._cws = torch.empty(nws, dtype=torch.uint8, device=self._dev)
+            s = F.fxpq_conv_fwd(d, x, wq, bq, y, stream, ws=self._cws if nws else None)
         elif L_["type"] == "maxpool":
             src = self._src(i, L_)
             x, fx = env[src]

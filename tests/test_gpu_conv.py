@@ -68,7 +68,9 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0, sc
         hd = torch.from_numpy(h.astype(np.int32)).cuda()
     d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy, w_l1,
                     scale=sd, fmt_scale=fs, shift=hd, fmt_shift=fh)
-    s = F.fxpq_conv_fwd(d, xd, wd, bd, y)
+    nws = F.fxpq_conv_workspace(d)
+    ws = torch.empty(nws, dtype=torch.uint8, device="cuda") if nws else None
+    s = F.fxpq_conv_fwd(d, xd, wd, bd, y, ws=ws)
     torch.cuda.synchronize()
     assert F.fxpq_get_device_status() == 0
     if mode == F.OUT_CODES:
@@ -135,6 +137,13 @@ CASES = [
     (2, 12, 8, 24, 1, 1, 0, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),
     (1, 19, 5, 40, 3, 1, 1, (7, 1, 3), (6, 1, 6), (16, 12), False, 0, (8, 1, 2)),
     (2, 17, 3, 32, 3, 1, 1, (16, 1, 11), (16, 1, 14), (16, 22), True, 1, None),
+    # FC-like layers (few output rows, long reductions): the split reduction across SMs, one- and
+    # two-limb, every output mode, with biases coarser and finer than the accumulator
+    (3, 7, 512, 200, 7, 1, 0, (8, 0, 4), (6, 1, 8), (16, 15), True, 0, (8, 0, 3)),
+    (2, 7, 512, 96, 7, 1, 0, (8, 0, 4), (16, 1, 15), (16, 22), False, 1, None),
+    (5, 1, 4096, 136, 1, 1, 0, (5, 0, 2), (7, 1, 9), (16, 8), False, 2, None),
+    (4, 1, 4096, 1000, 1, 1, 0, (16, 0, 12), (16, 1, 18), (16, 20), False, 1, None),
+    (9, 3, 512, 64, 3, 1, 0, (7, 0, 3), (5, 1, 6), (16, 4), True, 0, (6, 0, 1)),
 ]
 
 
@@ -279,6 +288,8 @@ SCALE_CASES = [
     (CASES[25], (16, 14), (16, 12)),    # 256-column tiles
     (CASES[32], (16, 14), (16, 12)),    # window mode, two-limb fast epilogue
     (CASES[35], (16, 14), (16, 12)),    # window mode, ACC64
+    (CASES[36], (16, 14), (16, 12)),    # split reduction
+    (CASES[39], (16, 13), (16, 10)),    # split reduction, two limbs, ACC64
 ]
 
 
