@@ -266,7 +266,8 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     P.part = nullptr;
     P.gs[0] = 0;
     P.gs[1] = P.n_groups;
-    if (P.patch != 3 && ws && P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
+    // (64-column tiles only, without a Scale layer: the instantiations that carry the split)
+    if (P.patch != 3 && BN == 64 && !a.has_scale && ws && P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
         const int ng = P.n_groups;
         int min_len = 1 << 30;
         for (int gi = 0; gi < ng; ++gi) min_len = std::min(min_len, P.g[gi].kb1 - P.g[gi].kb0);
@@ -306,6 +307,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         if (!g_tc_attr_set) {
             if (cudaFuncSetAttribute(conv_tc_kernel<64, long long, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<64, long long, false, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<64>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<64, int, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<64>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<64, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<64>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<128, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -318,12 +323,12 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     }
     const int grid = P.n_units < sms ? P.n_units : sms;
     launched = true;
-    if (a.has_scale) {
-        const fxpq_status s = launch_conv_tc_scaled(P, BN, acc64, grid, st);
-        if (s != FXPQ_OK || P.ksplit == 1) return s;
-        return launch_splitk_reduce(a, P.part, P.ksplit, acc64, st);
-    }
-    if (acc64)
+    if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);  // never split
+    if (P.ksplit > 1 && acc64)
+        conv_tc_kernel<64, long long, false, true><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
+    else if (P.ksplit > 1)
+        conv_tc_kernel<64, int, false, true><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
+    else if (acc64)
         conv_tc_kernel<64, long long, false><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (BN == 64)
         conv_tc_kernel<64, int, false><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);

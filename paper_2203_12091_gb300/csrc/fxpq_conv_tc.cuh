@@ -404,7 +404,9 @@ __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
 }
 
 // ------------------------------------------------------------------ kernel
-template <int BN, typename ACC, bool SC>
+// SPLIT: the instantiation that runs split reductions (P.ksplit >= 1, unit share ranges P.gs); without it
+// the unit loop is the tile loop and every tile takes all P.n_groups groups.
+template <int BN, typename ACC, bool SC, bool SPLIT = false>
 __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
     constexpr int TC_STAGES = tc_stages(BN);
     constexpr int TC_LAG = tc_lag(BN);
@@ -486,8 +488,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
-            for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-                const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+                const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
                 (void)sp;
                 const int tm = t / P.tiles_n;
                 const int n_img = tm / per_img, r = tm - n_img * per_img;
@@ -532,13 +534,13 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
             bool ok = true;
-            for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-                const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+            for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+                const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
                 (void)sp;
                 const int tm = t / P.tiles_n, tn = t % P.tiles_n;
                 const int n_img = tm / per_img, r = tm - n_img * per_img;
                 const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
-                for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
+                for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups) && ok; ++gi) {
                     const TcGroup g = P.g[gi];
                     for (int kb = g.kb0; kb < g.kb1; ++kb) {
                         if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
@@ -590,8 +592,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const __half* xb = a.x;
         uint32_t it = 0;
         bool ok = true;
-        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+        for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+            const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
             (void)sp;
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             long long rowoff[AR];  // element offset of the (r, s) = (0, 0) tap of each row (may be negative)
@@ -607,7 +609,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 if (m >= a.M) p0[i] = -(1 << 20);  // rows past the end read zeros
                 rowoff[i] = (((long long)n_img * a.H + p0[i]) * a.W + q0[i]) * a.Cp;
             }
-            for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
+            for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups) && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const __half* xp = xb + (long long)g.a_plane * a.x_ps;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
@@ -678,14 +680,15 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
         const uint32_t run_base = (uint32_t)(nbuf * BN);
         uint32_t u = 0;  // tiles written through the staging buffer so far
-        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+        for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+            const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
             (void)sp;
             const int tm = t / P.tiles_n, tn = t % P.tiles_n;
             const long long m = tile_row(P, tm, row);  // -1: row outside the output
-            for (int gi = P.gs[sp]; gi < P.gs[sp + 1]; ++gi) {
+            const int g_lo = SPLIT ? P.gs[sp] : 0, g_hi = SPLIT ? P.gs[sp + 1] : P.n_groups;
+            for (int gi = g_lo; gi < g_hi; ++gi) {
                 const int shift = P.g[gi].shift;
-                const bool first = gi == P.gs[sp], last = gi == P.gs[sp + 1] - 1;
+                const bool first = gi == g_lo, last = gi == g_hi - 1;
                 const uint32_t buf = nbuf == 2 ? (gcount & 1) : 0;
                 const uint32_t par = nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
                 if (!wait_bounded(accfull0 + 8 * buf, par, abort, P.status)) {
@@ -872,7 +875,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                         mbar_arrive(accempty0 + 8 * buf);
                     }
                     if (!last) continue;
-                    if (P.ksplit > 1) {
+                    if (SPLIT && P.ksplit > 1) {
                         // one share of the reduction: its exact integer sums go to the partial buffer
                         if (m >= 0) {
                             ACC* dst = static_cast<ACC*>(P.part) + ((long long)sp * a.M + m) * a.K + k0;
@@ -978,8 +981,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = wait_bounded(wbar, 0, abort, P.status);
         tc_fence_after();
-        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+        for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+            const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
             (void)sp;
             const uint32_t buf = gcount & 1;
             if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
@@ -1029,10 +1032,10 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         const uint64_t bdesc0 = make_sdesc(smem_u32(sB));
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = true;
-        for (int ut = blockIdx.x; ut < P.n_units && ok; ut += gridDim.x) {
-            const int t = ut / P.ksplit, sp = ut - t * P.ksplit;
+        for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
+            const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
             (void)sp;
-            for (int gi = P.gs[sp]; gi < P.gs[sp + 1] && ok; ++gi) {
+            for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups) && ok; ++gi) {
                 const TcGroup g = P.g[gi];
                 const uint32_t buf = P.nbuf == 2 ? (gcount & 1) : 0;
                 const uint32_t par = P.nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);

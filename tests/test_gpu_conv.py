@@ -144,6 +144,11 @@ CASES = [
     (5, 1, 4096, 136, 1, 1, 0, (5, 0, 2), (7, 1, 9), (16, 8), False, 2, None),
     (4, 1, 4096, 1000, 1, 1, 0, (16, 0, 12), (16, 1, 18), (16, 20), False, 1, None),
     (9, 3, 512, 64, 3, 1, 0, (7, 0, 3), (5, 1, 6), (16, 4), True, 0, (6, 0, 1)),
+    # window mode, two limbs, one-plane codes: the 32-bit epilogue (shift >= 17, bias not finer), its
+    # shift-17 edge and no ReLU with signed codes, and the 64-bit fallback for a finer bias
+    (2, 20, 3, 48, 3, 1, 1, (16, 1, 9), (16, 1, 12), (16, 18), False, 0, (6, 1, 2)),
+    (1, 18, 3, 64, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 17), True, 0, (8, 0, 2)),
+    (2, 20, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 13), (16, 30), False, 0, (8, 1, 3)),
 ]
 
 
