@@ -41,6 +41,9 @@ constexpr int FS_WARPS = FS_THREADS / 32;
 constexpr int TILE = 8192;  // 32 elements per thread, read in sub-rounds of 16
 constexpr int FS_BLOCKS_PER_SM = 3;
 constexpr int CHUNK_MAX = 65536;  // per-block element cap: keeps every 64-bit block bin below 2^64
+// Phase E balances the warps' shares of the sorted tile by elements plus this many per key they touch
+// (a key change costs the warp a flush of its accumulators, about as long as this many elements).
+constexpr unsigned FS_FLUSH_ELEMS = 128;
 
 struct FsSmem {
     float sorted[TILE];
@@ -51,6 +54,7 @@ struct FsSmem {
     unsigned r[2][NJ][MAXFL][2];
     unsigned rb[NJ][MAXFL][2];
     unsigned mn, mx, nonfinite, live;
+    unsigned wbeg[FS_WARPS + 1];  // phase E: warp w walks sorted[wbeg[w], wbeg[w + 1])
 };
 
 // Workspace: exact 128-bit bins as {lo, hi}, then per-candidate scores.
@@ -257,38 +261,94 @@ __device__ __forceinline__ void acc_add(Acc<NS, NS>& a, unsigned M, const KeyInf
     }
 }
 
-// Warp totals of the current key's accumulators into the block bins.  The sums are warp-uniform;
-// the shared-memory atomics are spread over the lanes (lane 0: count, 1-2: moments, 3..: slots) so
-// that they do not queue behind one another.
+// Sum of 16 per-lane 64-bit values over the warp, scattered: on return v[0] of lanes 2 i and 2 i + 1
+// holds the total of value i.  Four halving exchange stages (each lane keeps the half selected by one
+// of its lane bits and adds its partner's copy of it), then one pairwise add.
+__device__ __forceinline__ void warp_reduce_scatter16(u64 (&v)[16], unsigned lane) {
+#pragma unroll
+    for (int st = 0; st < 4; ++st) {
+        const int half = 8 >> st;
+        const unsigned o = 16u >> st;
+        const bool b = (lane & o) != 0u;
+#pragma unroll
+        for (int i = 0; i < half; ++i) {
+            const u64 mine = b ? v[half + i] : v[i];
+            const u64 other = b ? v[i] : v[half + i];
+            v[i] = mine + __shfl_xor_sync(0xFFFFFFFFu, other, o);
+        }
+    }
+    v[0] += __shfl_xor_sync(0xFFFFFFFFu, v[0], 1);
+}
+
+// Warp totals of the current key's accumulators into the block bins.
+// Narrow ranges (NRB = 2): the values (count, moments, remainder slots, boundary sums) are reduced in
+// groups of 16 by exchange stages, and each even lane adds one total into its bin.  Wide ranges: every
+// total by warp reductions first (independent, they pipeline), then one round of shared-memory
+// atomics, value v by lane v % 32 (a second value per lane past 32).
 template <int NS, int NRB>
 __device__ __forceinline__ void acc_flush(FsSmem& sm, Acc<NS, NRB>& a, int key, const KeyInfo& k, const FsParams& P,
                                           unsigned lane) {
-    const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
-    const u64 s1 = warp_sum64(a.s1), s2 = warp_sum64(a.s2);
-    if (lane == 0) atomicAdd(&sm.pn[key], n);
-    if (lane == 1) sadd64(sm.ps1[key], s1);
-    if (lane == 2) sadd64(sm.ps2[key], s2);
+    if constexpr (NRB == 2) {
+        constexpr int NV = 3 + NS + 2;  // count, s1, s2, r[0 .. NS), rb[0 .. 2)
+        constexpr int NG = (NV + 15) / 16;
 #pragma unroll
-    for (int jj = 0; jj < NS; ++jj) {
-        const int fi = jj - 1 - k.E - P.fl_lo;
-        if ((k.validR >> jj) & 1u) {
-            const u64 v = warp_sum64(a.r[jj]);
-            if (lane == (unsigned)((3 + jj) & 31)) sadd64(sm.r[k.sg][jj][fi], v);
-        }
-        if (NRB == NS && ((k.validRb >> jj) & 1u)) {
-            const u64 v = warp_sum64(a.rb[jj < NRB ? jj : 0]);
-            if (lane == (unsigned)((3 + NS + jj) & 31)) sadd64(sm.rb[jj][fi], v);
-        }
-    }
-    if (NRB == 2) {
+        for (int grp = 0; grp < NG; ++grp) {
+            u64 v[16];
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
-            const int jj = P.jb_lo + i + 1;
-            if (jj < NJ && ((k.validRb >> jj) & 1u)) {
-                const u64 v = warp_sum64(a.rb[i]);
-                if (lane == (unsigned)((3 + NS + i) & 31)) sadd64(sm.rb[jj][jj - 1 - k.E - P.fl_lo], v);
+            for (int i = 0; i < 16; ++i) {
+                const int idx = 16 * grp + i;
+                v[i] = idx == 0 ? (u64)a.n
+                                : idx == 1 ? a.s1
+                                           : idx == 2 ? a.s2
+                                                      : idx < 3 + NS ? a.r[(idx - 3) < NS ? idx - 3 : 0]
+                                                                     : idx < NV ? a.rb[(idx - 3 - NS) & 1] : 0ull;
+            }
+            warp_reduce_scatter16(v, lane);
+            const int idx = 16 * grp + (int)(lane >> 1);
+            if ((lane & 1u) || idx >= NV) continue;
+            const u64 tot = v[0];
+            if (idx == 0) {
+                atomicAdd(&sm.pn[key], (unsigned)tot);
+            } else if (idx == 1) {
+                sadd64(sm.ps1[key], tot);
+            } else if (idx == 2) {
+                sadd64(sm.ps2[key], tot);
+            } else if (idx < 3 + NS) {
+                const int jj = idx - 3;
+                if ((k.validR >> jj) & 1u) sadd64(sm.r[k.sg][jj][jj - 1 - k.E - P.fl_lo], tot);
+            } else {
+                const int jj = P.jb_lo + (idx - 3 - NS) + 1;
+                if (jj < NJ && ((k.validRb >> jj) & 1u)) sadd64(sm.rb[jj][jj - 1 - k.E - P.fl_lo], tot);
             }
         }
+    } else {
+        const unsigned n = __reduce_add_sync(0xFFFFFFFFu, a.n);
+        u64 v0 = 0ull, v1 = 0ull;  // this lane's totals
+        unsigned o0 = 0u, o1 = 0u;  // and the byte offsets of their {lo, hi} bins in sm (0: none)
+        char* const base = reinterpret_cast<char*>(&sm);
+        auto take = [&](int idx, u64 v, unsigned* d) {
+            if (lane == (unsigned)(idx & 31)) {
+                const unsigned off = (unsigned)(reinterpret_cast<char*>(d) - base);
+                if (idx < 32) {
+                    v0 = v;
+                    o0 = off;
+                } else {
+                    v1 = v;
+                    o1 = off;
+                }
+            }
+        };
+        take(1, warp_sum64(a.s1), sm.ps1[key]);
+        take(2, warp_sum64(a.s2), sm.ps2[key]);
+#pragma unroll
+        for (int jj = 0; jj < NS; ++jj) {
+            const int fi = jj - 1 - k.E - P.fl_lo;
+            if ((k.validR >> jj) & 1u) take(3 + jj, warp_sum64(a.r[jj]), sm.r[k.sg][jj][fi]);
+            if ((k.validRb >> jj) & 1u) take(3 + NS + jj, warp_sum64(a.rb[jj < NRB ? jj : 0]), sm.rb[jj][fi]);
+        }
+        if (lane == 0) atomicAdd(&sm.pn[key], n);
+        if (o0) sadd64(reinterpret_cast<unsigned*>(base + o0), v0);
+        if (o1) sadd64(reinterpret_cast<unsigned*>(base + o1), v1);
     }
 }
 
@@ -382,12 +442,41 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
                 if (lane >= (unsigned)off) incl += o;
             }
             unsigned run = incl - s;
+            const unsigned first = run;  // sorted position of this lane's first key
 #pragma unroll
             for (int i = 0; i < NKEY / 32; ++i) {
                 sm.cnt[lane * (NKEY / 32) + i] = run;
                 run += loc[i];
             }
             if (lane == 31) sm.live = incl;
+            // the warps' shares of phase E: equal in elements plus FS_FLUSH_ELEMS per key present
+            unsigned e = 0;
+#pragma unroll
+            for (int i = 0; i < NKEY / 32; ++i) e += loc[i] + (loc[i] ? FS_FLUSH_ELEMS : 0u);
+            unsigned eincl = e;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const unsigned o = __shfl_up_sync(0xFFFFFFFFu, eincl, off);
+                if (lane >= (unsigned)off) eincl += o;
+            }
+            const unsigned eexcl = eincl - e, etot = __shfl_sync(0xFFFFFFFFu, eincl, 31);
+            const unsigned total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+            if (lane < FS_WARPS) sm.wbeg[lane] = 0u;
+            if (lane == 0) sm.wbeg[FS_WARPS] = total;
+            __syncwarp();
+            // every lane checks its own keys against the FS_WARPS - 1 boundaries (each falls in one key)
+            unsigned ec = eexcl, pos = first;
+#pragma unroll
+            for (int i = 0; i < NKEY / 32; ++i) {
+                const unsigned ke = loc[i] + (loc[i] ? FS_FLUSH_ELEMS : 0u);
+#pragma unroll
+                for (int w = 1; w < FS_WARPS; ++w) {
+                    const unsigned T = (unsigned)(((unsigned long long)etot * (unsigned)w) / FS_WARPS);
+                    if (T >= ec && T < ec + ke) sm.wbeg[w] = pos + min(T - ec, loc[i]);
+                }
+                ec += ke;
+                pos += loc[i];
+            }
         }
         __syncthreads();
         // ---- D: scatter into key order (the tile is read again; it is L2-resident)
@@ -404,9 +493,7 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
         }
         __syncthreads();
         // ---- E: each warp walks a contiguous run of the sorted tile
-        const int L = (int)sm.live;
-        const int per = ((L + FS_WARPS * 32 - 1) / (FS_WARPS * 32)) * 32;
-        const int w0 = (int)warp * per, w1 = min(w0 + per, L);
+        const int w0 = (int)sm.wbeg[warp], w1 = (int)sm.wbeg[warp + 1];
         Acc<NS, NRB> acc;
         acc_zero(acc);
         int ck = -1;
