@@ -13,9 +13,11 @@ namespace fxpq {
 namespace {
 
 // ------------------------------------------------------------------ fp32 implicit-GEMM convolution
-// Tile 64 output pixels x 64 output channels, 16 reduction steps per stage, 256 threads with 4 x 4
-// outputs each.  x: [N, H, W, C]; w: [K, R*S*C] (KRSC); y: [N, P, Q, K].
-constexpr int CF_BM = 64, CF_BN = 64, CF_BK = 16;
+// Tile 128 output pixels x BN output channels (BN = 128 for wide layers, 64 otherwise), 8 reduction
+// steps per stage (double-buffered shared memory), 256 threads with 8 x BN/16 outputs each (64 or 32
+// FMAs per 16 or 12 shared-memory words).  x: [N, H, W, C]; w: [K, R*S*C] (KRSC); y: [N, P, Q, K].
+// When C % 8 == 0 a stage's 8 reduction steps are 8 channels of one tap, loaded as float4.
+constexpr int CF_BM = 128, CF_BK = 8;
 
 struct ConvF32Args {
     const float* x;
@@ -26,12 +28,134 @@ struct ConvF32Args {
     long long M;
 };
 
+template <int CF_BN>
 __global__ void __launch_bounds__(256) conv_f32_kernel(const ConvF32Args a) {
-    __shared__ float sa[CF_BK][CF_BM + 4];
-    __shared__ float sb[CF_BK][CF_BN + 4];
+    constexpr int TN = CF_BN / 16;  // output channels per thread
+    __shared__ __align__(16) float sa[2][CF_BK][CF_BM];
+    __shared__ __align__(16) float sb[2][CF_BK][CF_BN];
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const long long m0 = (long long)blockIdx.x * CF_BM;
     const int n0 = blockIdx.y * CF_BN;
+    const int RSC = a.R * a.S * a.C;
+    // staging: thread t loads row t / 2 of the A tile (and of the B tile when BN = 128; rows t / 4 with
+    // two columns each when BN = 64), reduction columns 4 (t % 2) .. + 3
+    const int lr = threadIdx.x >> 1, lk = (threadIdx.x & 1) * 4;
+    const int br = CF_BN == 128 ? lr : (threadIdx.x >> 2), bk = CF_BN == 128 ? lk : (threadIdx.x & 3) * 2;
+    const long long m = m0 + lr;
+    const bool mok = m < a.M;
+    int pn = 0, pp = 0, pq = 0;
+    if (mok) {
+        pn = (int)(m / ((long long)a.P * a.Q));
+        const int rem = (int)(m - (long long)pn * a.P * a.Q);
+        pp = rem / a.Q;
+        pq = rem - pp * a.Q;
+    }
+    const int o = n0 + br;
+    const bool ook = o < a.K;
+    const bool vecA = (a.C % 8) == 0, vecB = (RSC % 4) == 0;
+    float ra[4], rb[4];
+    auto load = [&](int k0) {
+        if (vecA) {
+            const int rs = k0 / a.C, c = k0 - rs * a.C + lk;
+            const int s = rs % a.S, r = rs / a.S;
+            const int h = pp * a.stride + r - a.pad, ww = pq * a.stride + s - a.pad;
+            if (mok && k0 < RSC && h >= 0 && h < a.H && ww >= 0 && ww < a.W) {
+                const float4 v =
+                    *reinterpret_cast<const float4*>(a.x + (((long long)pn * a.H + h) * a.W + ww) * a.C + c);
+                ra[0] = v.x, ra[1] = v.y, ra[2] = v.z, ra[3] = v.w;
+            } else {
+                ra[0] = ra[1] = ra[2] = ra[3] = 0.0f;
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int kk = k0 + lk + e;
+                float v = 0.0f;
+                if (mok && kk < RSC) {
+                    const int c = kk % a.C, rs = kk / a.C;
+                    const int s = rs % a.S, r = rs / a.S;
+                    const int h = pp * a.stride + r - a.pad, ww = pq * a.stride + s - a.pad;
+                    if (h >= 0 && h < a.H && ww >= 0 && ww < a.W)
+                        v = a.x[(((long long)pn * a.H + h) * a.W + ww) * a.C + c];
+                }
+                ra[e] = v;
+            }
+        }
+        const int kb = k0 + bk;
+        constexpr int NB = CF_BN == 128 ? 4 : 2;
+        if (CF_BN == 128 && vecB && ook && kb + 3 < RSC) {
+            const float4 v = *reinterpret_cast<const float4*>(a.w + (long long)o * RSC + kb);
+            rb[0] = v.x, rb[1] = v.y, rb[2] = v.z, rb[3] = v.w;
+        } else {
+#pragma unroll
+            for (int e = 0; e < NB; ++e) rb[e] = (ook && kb + e < RSC) ? a.w[(long long)o * RSC + kb + e] : 0.0f;
+        }
+    };
+    auto store = [&](int buf) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sa[buf][lk + e][lr] = ra[e];
+#pragma unroll
+        for (int e = 0; e < (CF_BN == 128 ? 4 : 2); ++e) sb[buf][bk + e][br] = rb[e];
+    };
+    float acc[8][TN];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) acc[i][j] = 0.0f;
+    load(0);
+    store(0);
+    __syncthreads();
+    int buf = 0;
+    for (int k0 = 0; k0 < RSC; k0 += CF_BK) {
+        const bool more = k0 + CF_BK < RSC;
+        if (more) load(k0 + CF_BK);  // next stage's global loads in flight during this stage's FMAs
+#pragma unroll
+        for (int kk = 0; kk < CF_BK; ++kk) {
+            const float4 a0 = *reinterpret_cast<const float4*>(&sa[buf][kk][ty * 8]);
+            const float4 a1 = *reinterpret_cast<const float4*>(&sa[buf][kk][ty * 8 + 4]);
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            float bv[TN];
+#pragma unroll
+            for (int q = 0; q < TN / 4; ++q) {
+                const float4 b = *reinterpret_cast<const float4*>(&sb[buf][kk][tx * TN + 4 * q]);
+                bv[4 * q] = b.x, bv[4 * q + 1] = b.y, bv[4 * q + 2] = b.z, bv[4 * q + 3] = b.w;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+        if (more) {
+            store(buf ^ 1);
+            __syncthreads();
+            buf ^= 1;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const long long mm = m0 + ty * 8 + i;
+        if (mm >= a.M) continue;
+#pragma unroll
+        for (int j = 0; j < TN; ++j) {
+            const int oo = n0 + tx * TN + j;
+            if (oo >= a.K) continue;
+            float v = acc[i][j];
+            if (a.bias) v += a.bias[oo];
+            if (a.relu) v = fmaxf(v, 0.0f);
+            a.y[mm * a.K + oo] = v;
+        }
+    }
+}
+
+// Small layers (too few 128-row tiles to occupy the SMs): 64 x 64 tiles, 4 x 4 outputs per thread.
+constexpr int SF_BM = 64, SF_BN = 64, SF_BK = 16;
+
+__global__ void __launch_bounds__(256) conv_f32_small_kernel(const ConvF32Args a) {
+    __shared__ float sa[SF_BK][SF_BM + 4];
+    __shared__ float sb[SF_BK][SF_BN + 4];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const long long m0 = (long long)blockIdx.x * SF_BM;
+    const int n0 = blockIdx.y * SF_BN;
     const int RSC = a.R * a.S * a.C;
     // the A element this thread stages: pixel row (threadIdx.x / 4) and reduction columns 4 * (tid % 4) ..
     const int lr = threadIdx.x >> 2, lk = (threadIdx.x & 3) * 4;
@@ -44,7 +168,7 @@ __global__ void __launch_bounds__(256) conv_f32_kernel(const ConvF32Args a) {
         pq = rem - pp * a.Q;
     }
     float acc[4][4] = {};
-    for (int k0 = 0; k0 < RSC; k0 += CF_BK) {
+    for (int k0 = 0; k0 < RSC; k0 += SF_BK) {
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const int kk = k0 + lk + e;
@@ -61,7 +185,7 @@ __global__ void __launch_bounds__(256) conv_f32_kernel(const ConvF32Args a) {
         }
         __syncthreads();
 #pragma unroll
-        for (int kk = 0; kk < CF_BK; ++kk) {
+        for (int kk = 0; kk < SF_BK; ++kk) {
             float av[4], bv[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) av[i] = sa[kk][ty * 4 + i];
@@ -273,8 +397,17 @@ extern "C" fxpq_status fxpq_conv_f32(const fxpq_conv_f32_desc* h_desc, const flo
     ConvF32Args a{d_x, d_w, d_bias, d_y, d.N, d.H, d.W, d.C, d.K, d.R, d.S, d.stride, d.pad, P, Q, d.relu ? 1 : 0,
                   (long long)d.N * P * Q};
     if (a.M == 0) return FXPQ_OK;
-    dim3 grid((unsigned)((a.M + CF_BM - 1) / CF_BM), (unsigned)((d.K + CF_BN - 1) / CF_BN));
-    conv_f32_kernel<<<grid, 256, 0, as_stream(stream)>>>(a);
+    const long long big = ((a.M + CF_BM - 1) / CF_BM) * ((d.K + (d.K >= 128 ? 127 : 63)) / (d.K >= 128 ? 128 : 64));
+    if (big < 152) {
+        dim3 grid((unsigned)((a.M + SF_BM - 1) / SF_BM), (unsigned)((d.K + SF_BN - 1) / SF_BN));
+        conv_f32_small_kernel<<<grid, 256, 0, as_stream(stream)>>>(a);
+    } else if (d.K >= 128) {
+        dim3 grid((unsigned)((a.M + CF_BM - 1) / CF_BM), (unsigned)((d.K + 127) / 128));
+        conv_f32_kernel<128><<<grid, 256, 0, as_stream(stream)>>>(a);
+    } else {
+        dim3 grid((unsigned)((a.M + CF_BM - 1) / CF_BM), (unsigned)((d.K + 63) / 64));
+        conv_f32_kernel<64><<<grid, 256, 0, as_stream(stream)>>>(a);
+    }
     return after_launch("conv_f32");
 }
 
