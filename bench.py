@@ -110,6 +110,22 @@ def measured_peaks():
     return 6800.0, 1900.0, 1700.0, "fallback"
 
 
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's mean step time: every rank times the same number of steps after one barrier."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, batch: int, t_max_ms: float) -> float:
+    """Whole-job images/s: every rank evaluates its own batch (replicas, weak scaling) in t_max."""
+    return world * batch / (t_max_ms / 1e3)
+
+
 # ----------------------------------------------------------------------------- GPU arm
 def run_fxpq(args):
     import torch
@@ -167,12 +183,8 @@ def run_fxpq(args):
     torch.cuda.synchronize()
     launches = F.fxpq_launch_count() - launches0
     ms = sum(times) / len(times)
-    t_max = ms
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_max = float(t.item())
-    value = world * B / (t_max / 1e3)
+    t_max = max_over_ranks(ms, world, dev)
+    value = job_throughput(world, B, t_max)
 
     # ---- end to end through the public API: pinned host images in, logits out, every step
     e2e_times = []

@@ -130,3 +130,50 @@ def test_bn_to_scale_bit_exact(NET):
 @pytest.mark.parametrize("plan_seed", [7, 38])
 def test_vgg16_batch64_plans(NET, plan_seed):
     _workload(NET, "vgg16", 64, 7, plan_seed=plan_seed, sample=(0,))
+
+
+def test_single_conv_workload_end_to_end(NET):
+    """The single-conv workload (batch 8, 64 -> 64 channels, 32 x 32 maps, 3 x 3, stride 1, pad 1): He-normal
+    weights, ReLU(N(0,1)) inputs, N(0, 0.01) biases, 8-bit weights and activations with FL searched over
+    0..15 (16-bit bias), the output requantized to 8 bits with its FL searched on the exact C-Block output.
+    Every format and every code equals the oracle's."""
+    import oracle
+    from paper_2203_12091_gb300 import fxpq as F
+    N, H, C, K = 8, 32, 64, 64
+    g = torch.Generator().manual_seed(91)
+    x = torch.relu(torch.randn(N, H, H, C, generator=g)).numpy()
+    w = (torch.randn(K, 3, 3, C, generator=g) * np.sqrt(2.0 / (9 * C))).numpy().astype(np.float32)
+    b = (torch.randn(K, generator=g) * 0.01).numpy().astype(np.float32)
+    fmt_gpu, fmt_ora = {}, {}
+    for nm, t, k in (("x", x, 8), ("w", w, 8), ("b", b, 16)):
+        err, best, st = F.fl_search(torch.from_numpy(t).cuda().reshape(-1), -1, k, k, 0, 15)
+        S = F.stats_from_device(st).is_signed
+        fmt_gpu[nm] = F.fmt(k, S, int(best.cpu()[0]))
+        _, obest, oS, _ = oracle.fl_search(t.reshape(-1), -1, k, k, 0, 15)
+        fmt_ora[nm] = (k, oS, int(obest[0]))
+        assert fmt_gpu[nm].tup() == fmt_ora[nm], nm
+    xq = torch.empty(N * H * H * C, dtype=torch.float16, device="cuda")
+    F.fxpq_quantize_rows(torch.from_numpy(x).cuda(), N * H * H, C, fmt_gpu["x"], C, xq)
+    wq = torch.empty(K * 9 * C, dtype=torch.float16, device="cuda")
+    F.fxpq_quantize_rows(torch.from_numpy(w).cuda(), K * 9, C, fmt_gpu["w"], C, wq)
+    bq = torch.empty(K, dtype=torch.int32, device="cuda")
+    F.fxpq_quantize(torch.from_numpy(b).cuda(), fmt_gpu["b"], F.DT_I32, bq)
+    # the exact C-Block output's fp32 image, its FL search, then the codes
+    f32 = torch.empty(N * H * H * K, dtype=torch.float32, device="cuda")
+    d = F.conv_desc(N, H, H, C, C, K, 3, 3, 1, 1, True, F.OUT_F32, fmt_gpu["x"], fmt_gpu["w"], fmt_gpu["b"], None)
+    F.fxpq_conv_fwd(d, xq, wq, bq, f32)
+    _, ybest, yst = F.fl_search(f32, -1, 8, 8, 0, 15)
+    fy = F.fmt(8, F.stats_from_device(yst).is_signed, int(ybest.cpu()[0]))
+    y = torch.empty(N * H * H * K, dtype=torch.float16, device="cuda")
+    d = F.conv_desc(N, H, H, C, C, K, 3, 3, 1, 1, True, F.OUT_CODES, fmt_gpu["x"], fmt_gpu["w"], fmt_gpu["b"], fy)
+    F.fxpq_conv_fwd(d, xq, wq, bq, y)
+    torch.cuda.synchronize()
+    qx = oracle.quantize(x, *fmt_ora["x"]).reshape(x.shape)
+    qw = oracle.quantize(w, *fmt_ora["w"]).reshape(w.shape)
+    qb = oracle.quantize(b, *fmt_ora["b"])
+    v, s = oracle.cblock(oracle.conv2d(qx, qw, 1, 1), fmt_ora["x"][2] + fmt_ora["w"][2], qb, fmt_ora["b"][2], True)
+    assert np.array_equal(f32.cpu().numpy().reshape(v.shape), oracle.to_f32(v, s))
+    _, oyb, oyS, _ = oracle.fl_search(oracle.to_f32(v, s).reshape(-1), -1, 8, 8, 0, 15)
+    assert fy.tup() == (8, oyS, int(oyb[0]))
+    want = oracle.requant(v, s, 8, oyS, int(oyb[0]))
+    assert np.array_equal(F.codes_to_int(y.cpu(), fy, (N, H, H, K)).numpy(), want)
