@@ -149,7 +149,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             const int S2 = (a.S + 1) & ~1;
             const int WW = 8 + S2 - 1, WH = 16 + a.R - 1;
             const int win_bytes = (WW * WH * 16 + 127) / 128 * 128;
-            bool ok = a.stride == 1 && a.Cp == 8 && a.K <= 64 && a.N > 0 && a.R * S2 <= 16 && WW <= 256 &&
+            bool ok = a.stride == 1 && a.Cp == 8 && a.K <= 64 && a.N > 0 && a.R * S2 <= 16 && 8 * WW <= 256 &&
                       WH <= 256 && a.px * win_bytes <= TC_BM * TC_BK * 2 &&
                       a.pw * a.R * (S2 / 2) * 64 * 32 <= tc_stages(64) * 64 * TC_BK * 2 && !conv_path_is("tc_rows") &&
                       !conv_path_is("tc_nowin");
@@ -157,10 +157,11 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 for (int iw = 0; iw < a.pw; ++iw)
                     if ((double)limb_max(d.fmt_x, ia) * limb_max(d.fmt_w, iw) * a.R * S2 * 8 >= 16777216.0) ok = false;
             if (ok) {
-                const cuuint64_t xdims[5] = {8, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N, (cuuint64_t)a.px};
-                const cuuint64_t xstrides[4] = {16, (cuuint64_t)a.W * 16, (cuuint64_t)a.H * a.W * 16,
-                                                (cuuint64_t)a.x_ps * 2};
-                const cuuint32_t xbox[5] = {8, (cuuint32_t)WW, (cuuint32_t)WH, 1, 1};
+                // the input as [planes][N][H][W * 8]: one window row (WW pixels of 8 channels) is a single
+                // 16 WW-byte run of the box rather than WW 16-byte rows
+                const cuuint64_t xdims[4] = {(cuuint64_t)a.W * 8, (cuuint64_t)a.H, (cuuint64_t)a.N, (cuuint64_t)a.px};
+                const cuuint64_t xstrides[3] = {(cuuint64_t)a.W * 16, (cuuint64_t)a.H * a.W * 16, (cuuint64_t)a.x_ps * 2};
+                const cuuint32_t xbox[4] = {(cuuint32_t)(8 * WW), (cuuint32_t)WH, 1, 1};
                 // weights as {c, out channel, s, r, plane} (strides in that order, not memory order)
                 const cuuint64_t wdims[5] = {8, (cuuint64_t)a.K, (cuuint64_t)a.S, (cuuint64_t)a.R, (cuuint64_t)a.pw};
                 const cuuint64_t wstrides[4] = {(cuuint64_t)a.R * a.S * 16, 16, (cuuint64_t)a.S * 16,
@@ -168,7 +169,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 const cuuint32_t wbox[5] = {8, 64, 2, 1, 1};
                 const cuuint32_t es5[5] = {1, 1, 1, 1, 1};
                 CUtensorMap mx, mw;
-                if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.x), xdims, xstrides, xbox, es5,
+                if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<__half*>(a.x), xdims, xstrides, xbox, es5,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
                     enc(&mw, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 5, const_cast<__half*>(a.w), wdims, wstrides, wbox, es5,

@@ -72,7 +72,8 @@ struct TcGroup {
 struct TcParams {
     CUtensorMap tmap_w;  // weights as [planes][K][R*S*Cp] fp16, box {64, BN, 1}, 128-byte swizzle
     CUtensorMap tmap_y;  // output codes: [M][K] box {64, 128} (linear tiles) or [N][P][Q][K] box {64, TW, TH, 1}
-    CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}
+    CUtensorMap tmap_x;  // patch tiles: activations [planes][N][H][W][Cp], box {64, TW, TH, 1, 1}; window mode:
+                         // [planes][N][H][W * 8], box {8 WW, WH, 1, 1} (a window row is one 16 WW-byte run)
     int fast_store;      // 1: one-plane codes staged in shared memory and written by TMA stores
     int nbuf;            // fp32 accumulator buffers in TMEM: 2, or 1 when BN = 256 needs running sums
     int patch;           // a tile is a TH x TW patch of one image and the A tile comes by TMA:
@@ -156,6 +157,16 @@ __device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap* map
         "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
         "%5, %6}], [%7];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar)
+        : "memory");
+}
+
+// 4-D tiled TMA load (coordinates innermost first) completing on mbarrier `bar`.
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
+        "%5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
         : "memory");
 }
 
@@ -435,7 +446,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + TC_STAGES);
     const uint32_t accfull0 = smem_u32(bars + 2 * TC_STAGES), accempty0 = smem_u32(bars + 2 * TC_STAGES + 2);
     const uint32_t done_bar = smem_u32(bars + 2 * TC_STAGES + 4);
-    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue thread
+    const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue warp
     const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
     const uint32_t wbar = smem_u32(bars + 2 * TC_STAGES + 9);      // window mode: resident weights loaded
 
@@ -444,17 +455,17 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < TC_STAGES; ++s) {
-            // patch tiles: one expect_tx arrival for both TMAs; row tiles: 128 producer arrivals +
-            // the weight TMA's expect_tx
-            mbar_init(full0 + 8 * s, P.patch ? 1 : 128 + 1);
+            // patch tiles: one expect_tx arrival for both TMAs; row tiles: one arrival per producer
+            // warp + the weight TMA's expect_tx
+            mbar_init(full0 + 8 * s, P.patch ? 1 : 4 + 1);
             mbar_init(empty0 + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accfull0 + 8 * b, 1);
-            mbar_init(accempty0 + 8 * b, EPI_THREADS);
+            mbar_init(accempty0 + 8 * b, EPI_WARPS);  // one arrival per epilogue warp
         }
         mbar_init(done_bar, 1);
-        mbar_init(stg_full, EPI_THREADS);
+        mbar_init(stg_full, EPI_WARPS);
         mbar_init(stg_free, 1);
         mbar_init(wbar, 1);
         *abort = 0;
@@ -500,8 +511,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 }
                 const uint32_t fb = full0 + 8 * stage;
                 mbar_arrive_expect_tx(fb, (uint32_t)a.px * win_tx);
+                // (pixels and channels of a row are one inner dimension: x = 8 * pixel, a multiple of 8)
                 for (int ia = 0; ia < a.px; ++ia)
-                    tma_load_5d(smem_u32(sA + stage * A_BYTES) + (uint32_t)(ia * P.win_bytes), &P.tmap_x, 0, wq0, hp0,
+                    tma_load_4d(smem_u32(sA + stage * A_BYTES) + (uint32_t)(ia * P.win_bytes), &P.tmap_x, 8 * wq0, hp0,
                                 n_img, ia, fb);
                 ++it;
                 if (++stage == TC_STAGES) {
@@ -641,9 +653,11 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     }
                     cp_async_commit();
                     if (it >= TC_LAG) {
+                        // this warp's copies of stage it - TC_LAG have landed: one arrival for the warp
                         cp_async_wait<TC_LAG>();
                         fence_proxy_async();
-                        mbar_arrive(full0 + 8 * ((it - TC_LAG) % TC_STAGES));
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(full0 + 8 * ((it - TC_LAG) % TC_STAGES));
                     }
                     ++it;
                 }
@@ -651,8 +665,10 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         }
         cp_async_wait<0>();
         fence_proxy_async();
+        __syncwarp();
         const uint32_t first = it >= TC_LAG ? it - TC_LAG : 0;
-        for (uint32_t j = first; j < it; ++j) mbar_arrive(full0 + 8 * (j % TC_STAGES));
+        if (lane == 0)
+            for (uint32_t j = first; j < it; ++j) mbar_arrive(full0 + 8 * (j % TC_STAGES));
         if (threadIdx.x == 0) {
             // Every weight TMA this thread issued has landed once its stage's phase completes (the MMA
             // thread already waited for them unless the kernel aborted): bounded wait on the last ones.
@@ -734,7 +750,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                             reg_fence(fll);
                             if (hf == 1 && c == CPW - 1) {
                                 tc_fence_before();
-                                mbar_arrive(accempty0 + 8 * buf);
+                                __syncwarp();
+                                if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
                             }
 #pragma unroll
                             for (int j = 0; j < 8; ++j) {
@@ -870,9 +887,11 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     }
                     if (c == CPW - 1) {
                         // every chunk of this warp is out of the accumulator buffer: free it for the
-                        // next group's MMAs before the final arithmetic
+                        // next group's MMAs before the final arithmetic (one arrival per warp: same-address
+                        // arrivals of every thread serialise)
                         tc_fence_before();
-                        mbar_arrive(accempty0 + 8 * buf);
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
                     }
                     if (!last) continue;
                     if (SPLIT && P.ksplit > 1) {
@@ -946,7 +965,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 if (last && P.fast_store) {
                     // make the staging writes visible to the async proxy, then one thread stores the tile
                     fence_proxy_async();
-                    mbar_arrive(stg_full);
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(stg_full);
                     if (leader) {
                         if (!wait_bounded(stg_full, u & 1, abort, P.status)) {
                             ok = false;
