@@ -62,6 +62,7 @@ constexpr size_t tc_smem_bytes() {
 constexpr int TC_MAX_GROUPS = 64;
 constexpr int TC_MAX_SPLIT = 16;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
+constexpr int TC_PRODUCERS = 2;  // TMA-issuing threads of patch tiles (lane 0 of warps 0, 1)
 
 struct TcGroup {
     int kb0, kb1;          // k-block range within a plane
@@ -540,11 +541,14 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         // Cp == 8: a k-block is 8 taps of 8 channels; tap tl's box {8, TW, TH} lands at byte
         // 2048 tl of the stage (a 16-byte K column of the no-swizzle layout), and taps past R*S
         // are boxes wholly outside the tensor (zero filled).
-        if (threadIdx.x == 0) {
+        if (lane == 0 && warp < TC_PRODUCERS) {
+            // k-block it is issued by producer it % TC_PRODUCERS (lane 0 of warps 0 .. TC_PRODUCERS - 1): one
+            // thread's latency per k-block (barrier wait, two TMA instructions) would bound the stage rate
+            const int me = warp;
             const bool narrow = P.patch == 2;
             const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
             const int per_img = P.tiles_p * P.tiles_q;
-            uint32_t it = 0, stage = 0, phase = 0;
+            uint32_t it = 0;
             bool ok = true;
             for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
                 const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
@@ -554,33 +558,43 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
                 for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups) && ok; ++gi) {
                     const TcGroup g = P.g[gi];
-                    for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
-                            ok = false;
-                            break;
-                        }
-                        const int f = kb * TC_BK;
-                        const int tp = f / a.Cp, cc = f - tp * a.Cp;
-                        const int rr = tp / a.S, ss = tp - rr * a.S;
-                        const uint32_t fb = full0 + 8 * stage;
-                        mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
-                        if (narrow) {
-                            for (int tl = 0; tl < 8; ++tl) {
-                                const int tap = kb * 8 + tl;
-                                const bool in = tap < a.R * a.S;
-                                const int r8 = in ? tap / a.S : 0, s8 = in ? tap - (tap / a.S) * a.S : 0;
-                                tma_load_5d(smem_u32(sA + stage * A_BYTES + tl * 2048), &P.tmap_x, in ? 0 : 8,
-                                            wq0 + s8, hp0 + r8, n_img, g.a_plane, fb);
+                    // tap (rr, ss) and channel offset cc of the group's first k-block, then stepped by
+                    // TC_BK channels (Cp % 64 == 0: a k-block never straddles a tap)
+                    const int tp0 = g.kb0 * TC_BK / a.Cp;
+                    int cc = g.kb0 * TC_BK - tp0 * a.Cp;
+                    int rr = tp0 / a.S, ss = tp0 - rr * a.S;
+                    for (int kb = g.kb0; kb < g.kb1; ++kb, ++it) {
+                        if ((int)(it % TC_PRODUCERS) == me) {
+                            const uint32_t stage = it % TC_STAGES, phase = (it / TC_STAGES) & 1;
+                            if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
+                                ok = false;
+                                break;
                             }
-                        } else {
-                            tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
-                                        g.a_plane, fb);
+                            const uint32_t fb = full0 + 8 * stage;
+                            mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
+                            if (narrow) {
+                                for (int tl = 0; tl < 8; ++tl) {
+                                    const int tap = kb * 8 + tl;
+                                    const bool in = tap < a.R * a.S;
+                                    const int r8 = in ? tap / a.S : 0, s8 = in ? tap - (tap / a.S) * a.S : 0;
+                                    tma_load_5d(smem_u32(sA + stage * A_BYTES + tl * 2048), &P.tmap_x, in ? 0 : 8,
+                                                wq0 + s8, hp0 + r8, n_img, g.a_plane, fb);
+                                }
+                            } else {
+                                tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
+                                            g.a_plane, fb);
+                            }
+                            tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, kb * TC_BK, tn * BN, g.w_plane, fb);
                         }
-                        tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, f, tn * BN, g.w_plane, fb);
-                        ++it;
-                        if (++stage == TC_STAGES) {
-                            stage = 0;
-                            phase ^= 1;
+                        if (!narrow) {
+                            cc += TC_BK;
+                            if (cc >= a.Cp) {
+                                cc = 0;
+                                if (++ss == a.S) {
+                                    ss = 0;
+                                    ++rr;
+                                }
+                            }
                         }
                     }
                 }
