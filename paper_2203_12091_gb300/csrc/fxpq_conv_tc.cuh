@@ -62,7 +62,11 @@ constexpr size_t tc_smem_bytes() {
 constexpr int TC_MAX_GROUPS = 64;
 constexpr int TC_MAX_SPLIT = 16;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
-constexpr int TC_PRODUCERS = 2;  // TMA-issuing threads of patch tiles (lane 0 of warps 0, 1)
+// TMA-issuing threads of patch tiles (lane 0 of warps 0 .. n-1).  Producer p issues the k-blocks of the
+// stages s with s % n == p, so every use of a stage comes from one thread, in order: a thread that waited
+// on a stage another thread refills could pass a parity wait one phase early (the barrier two phases
+// behind reads as complete).  Hence n divides the stage count.
+__host__ __device__ constexpr int tc_producers(int BN) { return tc_stages(BN) % 2 == 0 ? 2 : tc_stages(BN); }
 
 struct TcGroup {
     int kb0, kb1;          // k-block range within a plane
@@ -423,6 +427,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     constexpr int TC_STAGES = tc_stages(BN);
     constexpr int TC_LAG = tc_lag(BN);
     static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
+    constexpr int TC_PRODUCERS = tc_producers(BN);
+    static_assert(TC_STAGES % TC_PRODUCERS == 0 && TC_PRODUCERS <= 4,
+                  "each stage must have one producer thread among warps 0..3");
     constexpr int EPI_WARPS = tc_epi_warps(BN);
     constexpr int EPI_THREADS = 32 * EPI_WARPS;
     constexpr int MMA_WARP = 4 + EPI_WARPS;
@@ -542,8 +549,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         // 2048 tl of the stage (a 16-byte K column of the no-swizzle layout), and taps past R*S
         // are boxes wholly outside the tensor (zero filled).
         if (lane == 0 && warp < TC_PRODUCERS) {
-            // k-block it is issued by producer it % TC_PRODUCERS (lane 0 of warps 0 .. TC_PRODUCERS - 1): one
-            // thread's latency per k-block (barrier wait, two TMA instructions) would bound the stage rate
+            // k-block it goes to producer (it % TC_STAGES) % TC_PRODUCERS: one thread's latency per k-block
+            // (barrier wait, two TMA instructions) would bound the stage rate
             const int me = warp;
             const bool narrow = P.patch == 2;
             const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
@@ -564,7 +571,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     int cc = g.kb0 * TC_BK - tp0 * a.Cp;
                     int rr = tp0 / a.S, ss = tp0 - rr * a.S;
                     for (int kb = g.kb0; kb < g.kb1; ++kb, ++it) {
-                        if ((int)(it % TC_PRODUCERS) == me) {
+                        if ((int)((it % TC_STAGES) % TC_PRODUCERS) == me) {
                             const uint32_t stage = it % TC_STAGES, phase = (it / TC_STAGES) & 1;
                             if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
                                 ok = false;
