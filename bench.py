@@ -236,7 +236,11 @@ def run_fxpq(args):
 
 
 def conv_roofline(q, imgs, F, stream, iters=3):
-    """Average conv launch time over `iters` op-by-op forwards (CUDA events on the launching stream)."""
+    """Average conv launch time over `iters` op-by-op forwards (CUDA events on the launching stream).
+
+    A short device-side sleep is queued ahead of each timed conv, so that the host's argument
+    preparation overlaps it and the events bracket the conv kernel(s) alone rather than the host gap
+    before the launch."""
     import torch
     env0 = None
     tot_ms, flops, n = 0.0, 0, 0
@@ -252,6 +256,7 @@ def conv_roofline(q, imgs, F, stream, iters=3):
             mode = F.OUT_ACC64 if i == last else F.OUT_CODES
             if L_["type"] == "conv":
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda._sleep(400_000)  # ~0.2 ms at 2 GHz: longer than the host work of run_layer
                 e0.record(stream)
                 y, s = q.run_layer(i, env, N, mode)
                 e1.record(stream)
