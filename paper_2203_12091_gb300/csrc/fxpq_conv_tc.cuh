@@ -63,9 +63,10 @@ constexpr int TC_MAX_GROUPS = 64;
 constexpr int TC_MAX_SPLIT = 16;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
 // TMA-issuing threads of patch tiles (lane 0 of warps 0 .. n-1).  Producer p issues the k-blocks of the
-// stages s with s % n == p, so every use of a stage comes from one thread, in order: a thread that waited
-// on a stage another thread refills could pass a parity wait one phase early (the barrier two phases
-// behind reads as complete).  Hence n divides the stage count.
+// stages s with s % n == p (n divides the stage count), so every use of a stage comes from one thread, in
+// order, and its parity wait on the stage's `empty` barrier is never more than one phase ahead of it.
+// (A parity wait two phases ahead reads as complete: with k-blocks dealt round-robin, more producers
+// than stages could refill a stage before its data was consumed.)
 __host__ __device__ constexpr int tc_producers(int BN) { return tc_stages(BN) % 2 == 0 ? 2 : tc_stages(BN); }
 
 struct TcGroup {
