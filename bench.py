@@ -217,9 +217,7 @@ def run_fxpq(args):
             "value": round(value, 2), "unit": "images/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(t_max, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "int (exact integer codes; fp16-valued operands)", "data": "synthetic",
-            "config": {"workload": f"{arch} batch {B}, {len(plans)} candidate plans, calib slice {wl['calib']}",
-                       "model": arch, "global_batch": B * world, "seq_len": None, "parallelism": f"replicas x{world}",
-                       "l2": "flushed between timed steps (2x L2 buffer written)"},
+            "config": workload_config(args.workload, world),
             "e2e": {"value": round(world * B / e2e_s, 2), "unit": "images/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": int(launches),
@@ -300,6 +298,14 @@ def cpu_baseline(workload):
                       f"1-image slice, forward of 1 image ({t:.1f} s)"}
 
 
+def workload_config(workload, world):
+    """The bench line's `config` (both arms): the workload and how it is laid out over the ranks."""
+    wl = WORKLOADS[workload]
+    return {"workload": f"{wl['arch']} batch {wl['batch']}, {len(wl['plans'])} candidate plans, calib slice {wl['calib']}",
+            "model": wl["arch"], "global_batch": wl["batch"] * world, "seq_len": None,
+            "parallelism": f"replicas x{world}", "l2": "flushed between timed steps (2x L2 buffer written)"}
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -314,10 +320,11 @@ def run_reference(args):
         "value": v, "unit": "images/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(t * 1e3, 1), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int64 (exact)", "data": "synthetic",
-        "config": {"workload": args.workload, "model": args.workload, "global_batch": 1, "seq_len": None,
-                   "parallelism": "cpu"},
+        "config": workload_config(args.workload, world),
         "cpu_baseline": {"value": v, "unit": "images/s", "cores": cores, "kind": "oracle",
-                         "sample": "one candidate plan on 1 image (calibration slice of 1 image)"},
+                         "sample": f"{args.workload}, rank 0 on the host cores: per step one candidate plan -- "
+                                   "parameter FL search + quantize, calibration on a 1-image slice, forward of "
+                                   "1 image"},
         "e2e": {"value": v, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
