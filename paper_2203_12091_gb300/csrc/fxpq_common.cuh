@@ -37,8 +37,9 @@ __device__ __forceinline__ void latch_status(int* st, int code) {
     if (st) atomicCAS(st, 0, code);
 }
 
-// Round half to even of v / 2^sh for sh >= 1 (exact, int64): the FxP-QLayer's shift.
-__device__ __forceinline__ long long rne_shift(long long v, int sh) {
+// Round half to even of v / 2^sh for sh >= 1 (exact, int64): the FxP-QLayer's shift.  (Host-callable
+// like the rest of the epilogue arithmetic, so that the CPU tests can run it.)
+__host__ __device__ __forceinline__ long long rne_shift(long long v, int sh) {
     long long q = v >> sh;  // floor (arithmetic shift)
     unsigned long long rem = (unsigned long long)(v - (q << sh));
     unsigned long long half = 1ull << (sh - 1);
@@ -47,7 +48,7 @@ __device__ __forceinline__ long long rne_shift(long long v, int sh) {
 }
 
 // value * 2^(fl_out - s) rounded half-even, clipped to [lo, hi]  (sh = s - fl_out)
-__device__ __forceinline__ long long requant_value(long long v, int sh, long long lo, long long hi) {
+__host__ __device__ __forceinline__ long long requant_value(long long v, int sh, long long lo, long long hi) {
     long long q;
     if (sh > 0)
         q = rne_shift(v, sh);

@@ -34,7 +34,7 @@ struct ConvArgs {
 // in units of 2^-s_out.  SC = false compiles the Scale layer out (for kernels the host launches only
 // for layers without one).
 template <bool SC = true>
-__device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long long v, int32_t bias) {
+__host__ __device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long long v, int32_t bias) {
     if (a.has_bias) {
         const long long b = bias;
         if (a.delta >= 0)
@@ -42,20 +42,22 @@ __device__ __forceinline__ long long cblock_value(const ConvArgs& a, int k, long
         else
             v = (v << (-a.delta)) + b;
     }
-    if (SC && a.has_scale) {
-        v *= (long long)__ldg(a.scale + k);
-        const long long h = __ldg(a.shift + k);
-        if (a.delta2 >= 0)
-            v += h << a.delta2;
-        else
-            v = (v << (-a.delta2)) + h;
+    if constexpr (SC) {
+        if (a.has_scale) {
+            v *= (long long)__ldg(a.scale + k);
+            const long long h = __ldg(a.shift + k);
+            if (a.delta2 >= 0)
+                v += h << a.delta2;
+            else
+                v = (v << (-a.delta2)) + h;
+        }
     }
     if (a.relu && v < 0) v = 0;
     return v;
 }
 
 // FxP-QLayer: v * 2^(fl_y - s_out) rounded half to even on the dropped bits, clipped to fmt_y.
-__device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
+__host__ __device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
     long long q;
     if (a.sh > 0) {
         q = rne_shift(v, a.sh);
@@ -79,7 +81,7 @@ __device__ __forceinline__ int qlayer_code(const ConvArgs& a, long long v) {
 // 0 <= phi < 1, floor((N + phi) / 2^sh32) = N >> sh32, and against half = 2^(sh32-1) the remainder
 // (N mod 2^sh32) + phi is above half iff rem > half or (rem == half and phi > 0), a tie iff
 // rem == half and phi == 0.  ReLU: N + phi < 0 iff N < 0.
-__device__ __forceinline__ int qlayer_code32(const ConvArgs& a, int acc, int32_t bias) {
+__host__ __device__ __forceinline__ int qlayer_code32(const ConvArgs& a, int acc, int32_t bias) {
     int N = acc;
     bool phi = false;
     if (a.has_bias) {

@@ -343,7 +343,7 @@ struct Epi32 {
     int has_bias;
 };
 
-__device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
+__host__ __device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
     Epi32 e;
     e.bsl = a.bsh > 0 ? a.bsh : 0;
     e.bsr = a.bsh < 0 ? -a.bsh : 0;
@@ -362,7 +362,7 @@ __device__ __forceinline__ Epi32 make_epi32(const ConvArgs& a) {
 // when the remainder is above one half, or equal to it with q odd or phi set (phi: the bias had
 // nonzero bits below the accumulator's scale, so the true value lies above the tie).  After a ReLU
 // clamp N = 0 and the sum stays below 2^sh whatever phi is.  The host keeps |N| + 2^(sh-1) < 2^31.
-__device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, int phi) {
+__host__ __device__ __forceinline__ int epi32_code(const Epi32& e, int acc, int bterm, int phi) {
     const int N = max(acc + bterm, e.floor);
     const int x = ((N >> e.sh) & 1) | phi;
     return min(max((N + e.hm1 + x) >> e.sh, e.lo), e.hi);
@@ -380,7 +380,7 @@ struct Epi64 {
     int dl2, dr2;
 };
 
-__device__ __forceinline__ Epi64 make_epi64(const ConvArgs& a) {
+__host__ __device__ __forceinline__ Epi64 make_epi64(const ConvArgs& a) {
     Epi64 e;
     e.dl = a.delta > 0 ? a.delta : 0;
     e.dr = a.delta < 0 ? -a.delta : 0;
@@ -398,7 +398,7 @@ __device__ __forceinline__ Epi64 make_epi64(const ConvArgs& a) {
 
 // m, h: aleph1 and aleph2 codes of the channel (read only when SC)
 template <bool SC>
-__device__ __forceinline__ int epi64_code(const Epi64& e, long long acc, int32_t b, int32_t m, int32_t h) {
+__host__ __device__ __forceinline__ int epi64_code(const Epi64& e, long long acc, int32_t b, int32_t m, int32_t h) {
     long long v = (acc << e.dr) + ((long long)b << e.dl);
     if (SC) v = ((v * (long long)m) << e.dr2) + ((long long)h << e.dl2);
     v = max(v, e.floor);
