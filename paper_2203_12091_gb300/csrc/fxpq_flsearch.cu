@@ -23,6 +23,8 @@
 // the exponent changes.  Block totals go to the workspace bins with integer atomics.
 #include <math.h>
 
+#include <algorithm>
+
 #include <mutex>
 
 #include "fxpq_common.cuh"
@@ -57,17 +59,23 @@ struct FsSmem {
     unsigned wbeg[FS_WARPS + 1];  // phase E: warp w walks sorted[wbeg[w], wbeg[w + 1])
 };
 
-// Workspace: exact 128-bit bins as {lo, hi}, then per-candidate scores.
+// Workspace: exact bins, then per-candidate scores.  A sum bin is three 64-bit words w0, w1, w2 that
+// stand for w0 + w1 2^32 + w2 2^64 (w2 two's complement): every contribution is split into 32-bit
+// limbs and added with plain (non-returning) atomics, so no carry has to be propagated between
+// words, and the sum of at most 2^32 limbs stays below 2^64 in every word.
 struct FsGlobal {
     u64 pn[NKEY];
-    u64 ps1[NKEY][2];
-    u64 ps2[NKEY][2];
-    u64 r[2][NJ][MAXFL][2];
-    u64 rb[NJ][MAXFL][2];
+    u64 ps1[NKEY][3];
+    u64 ps2[NKEY][3];
+    u64 r[2][NJ][MAXFL][3];
+    u64 rb[NJ][MAXFL][3];
     unsigned mn_inv, mx, nonfinite, pad;  // mn_inv = ~(smallest order key); 0: no finite element
     u64 nzero;                            // finite zeros (+-0.0): no key, but a binary-quantizer error
     double cells[2][MAXK][MAXFL];         // [S][k - 1][fl - fl_lo]
     double stat_sum, stat_sumsq;
+    // Exact sums of squares by biased exponent eb, weight 2^(2(eb - 150)), that belong to every L2
+    // cell and to the sum of squares but to no key's moments (the histogram kernel's sum of L^2)
+    u64 cband[256][3];
 };
 
 struct FsParams {
@@ -77,6 +85,11 @@ struct FsParams {
     int fl_lo, nfl;
     int jmax_pos, jmax_neg;  // largest j whose remainder sum R is needed (x >= 0 / x < 0)
     int jb_lo, jb_hi;        // j range of the boundary sum Rb (x >= 0)
+    // histogram kernel (fxpq_flsearch_hist.cuh): split bit s, the window's lowest biased exponent and
+    // its keys per sign
+    int hs_s;
+    int hs_eb_lo;
+    int hs_w;
     FsGlobal* g;
 };
 
@@ -124,10 +137,21 @@ __device__ __forceinline__ void sadd64(unsigned* p, u64 v) {
     if (hi) atomicAdd(p + 1, hi);
 }
 
-__device__ __forceinline__ void gadd128(u64* p, u64 v) {
+// v into a three-limb sum bin (v >= 0)
+__device__ __forceinline__ void gaddL(u64* p, u64 v) {
     if (!v) return;
-    const u64 old = atomicAdd(p, v);
-    if (old + v < old) atomicAdd(p + 1, 1ull);
+    atomicAdd(p, v & 0xFFFFFFFFull);
+    if (v >> 32) atomicAdd(p + 1, v >> 32);
+}
+// v (two's complement, |v| < 2^95) into a three-limb sum bin
+__device__ __forceinline__ void gaddLs(u64* p, __int128 v) {
+    if (!v) return;
+    const unsigned __int128 w = (unsigned __int128)v;
+    const u64 l0 = (u64)w & 0xFFFFFFFFull, l1 = (u64)(w >> 32) & 0xFFFFFFFFull;
+    const long long l2 = (long long)(v >> 64);
+    if (l0) atomicAdd(p, l0);
+    if (l1) atomicAdd(p + 1, l1);
+    if (l2) atomicAdd(p + 2, (u64)l2);
 }
 
 // Sum of a per-lane value v < 2^63 over the full warp (three 21-bit pieces, exact).
@@ -559,16 +583,16 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     for (int i = threadIdx.x; i < NKEY; i += FS_THREADS) {
         if (!sm.pn[i]) continue;
         atomicAdd(&g->pn[i], (u64)sm.pn[i]);
-        gadd128(g->ps1[i], ((u64)sm.ps1[i][1] << 32) | sm.ps1[i][0]);
-        gadd128(g->ps2[i], ((u64)sm.ps2[i][1] << 32) | sm.ps2[i][0]);
+        gaddL(g->ps1[i], ((u64)sm.ps1[i][1] << 32) | sm.ps1[i][0]);
+        gaddL(g->ps2[i], ((u64)sm.ps2[i][1] << 32) | sm.ps2[i][0]);
     }
     for (int i = threadIdx.x; i < 2 * NJ * MAXFL; i += FS_THREADS) {
         const int s = i / (NJ * MAXFL), j = (i / MAXFL) % NJ, f = i % MAXFL;
-        gadd128(g->r[s][j][f], ((u64)sm.r[s][j][f][1] << 32) | sm.r[s][j][f][0]);
+        gaddL(g->r[s][j][f], ((u64)sm.r[s][j][f][1] << 32) | sm.r[s][j][f][0]);
     }
     for (int i = threadIdx.x; i < NJ * MAXFL; i += FS_THREADS) {
         const int j = i / MAXFL, f = i % MAXFL;
-        gadd128(g->rb[j][f], ((u64)sm.rb[j][f][1] << 32) | sm.rb[j][f][0]);
+        gaddL(g->rb[j][f], ((u64)sm.rb[j][f][1] << 32) | sm.rb[j][f][0]);
     }
     if (threadIdx.x == 0) {
         if (sm.mn != 0xFFFFFFFFu) atomicMax(&g->mn_inv, ~sm.mn);
@@ -577,11 +601,18 @@ __global__ void __launch_bounds__(FS_THREADS, NRB == 2 ? FS_BLOCKS_PER_SM : 2)
     }
 }
 
+}  // namespace
+}  // namespace fxpq
+
+#include "fxpq_flsearch_hist.cuh"
+
+namespace fxpq {
+namespace {
+
 // ------------------------------------------------------------------ exact finalize
 struct U128 {
     u64 lo, hi;
 };
-__device__ __forceinline__ U128 ld128(const u64* p) { return U128{p[0], p[1]}; }
 // (a * m) for a 128-bit a and 64-bit m: the callers' bounds keep the product below 2^128
 __device__ __forceinline__ U128 mul128_64(U128 a, u64 m) {
     U128 r;
@@ -637,6 +668,16 @@ __device__ void big_add(Big& a, U128 v, int e, bool neg) {
             if (i - wi >= 2 && borrow == 0ull) break;
         }
     }
+}
+
+// a += (neg ? -1 : 1) * m * 2^e * (the three-limb bin at p).  The top limb is signed: the histogram
+// kernel's remainder sums leave out the sum of L^2 that its exponent band carries, so one key's
+// share of a cell may be negative.
+__device__ __forceinline__ void big_add_L3(Big& a, const u64* p, int e, bool neg, u64 m = 1ull) {
+    big_add(a, mul128_64(U128{p[0], 0ull}, m), e, neg);
+    big_add(a, mul128_64(U128{p[1], 0ull}, m), e + 32, neg);
+    const long long w2 = (long long)p[2];
+    if (w2) big_add(a, mul128_64(U128{w2 < 0 ? (u64)(-w2) : (u64)w2, 0ull}, m), e + 64, neg != (w2 < 0));
 }
 
 // a += (the big number held by lane `src_lane`), modulo 2^768 (warp-collective)
@@ -699,10 +740,10 @@ __device__ void big_negate(Big& a) {
 }
 
 // saturated set with moments (n, s1, s2) at exponent E: s2 2^(2(E-23)) - 2 T s1 2^(E-23-fl) + T^2 n 2^(-2fl)
-__device__ void add_sat(Big& acc, u64 n, U128 s1, U128 s2, int E, int fl, u64 T) {
-    big_add(acc, s2, 2 * (E - 23), false);
+__device__ void add_sat(Big& acc, u64 n, const u64* s1, const u64* s2, int E, int fl, u64 T) {
+    big_add_L3(acc, s2, 2 * (E - 23), false);
     if (T) {
-        big_add(acc, mul128_64(s1, 2ull * T), E - 23 - fl, true);
+        big_add_L3(acc, s1, E - 23 - fl, true, 2ull * T);
         big_add(acc, mul128_64(U128{n, 0ull}, T * T), -2 * fl, false);
     }
 }
@@ -720,15 +761,19 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
     const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
     Big acc;
     big_zero(acc);
+    // the exponent-indexed sums of squares that belong to every L2 cell and to the sum of squares
+    const bool with_band = cell == ncell + 1 || (cell < ncell && !F.l1);
+    if (with_band)
+        for (int eb = lane; eb < 256; eb += 32) big_add_L3(acc, g->cband[eb], 2 * (eb - 150), false);
     if (cell >= ncell) {
         const bool sq = cell == ncell + 1;
         for (int key = lane; key < NKEY; key += 32) {
             if (!g->pn[key]) continue;
             const int eb = key & 255, E = eb ? eb - 127 : -126;
             if (sq)
-                big_add(acc, ld128(g->ps2[key]), 2 * (E - 23), false);
+                big_add_L3(acc, g->ps2[key], 2 * (E - 23), false);
             else
-                big_add(acc, ld128(g->ps1[key]), E - 23, (key >> 8) != 0);
+                big_add_L3(acc, g->ps1[key], E - 23, (key >> 8) != 0);
         }
     } else if (F.k_lo == 1 && F.S_lo + cell / (F.nk * F.nfl) == 1 && (cell % (F.nk * F.nfl)) / F.nfl == 0) {
         // k = 1, S = 1: the binary quantizer (Eq. fp_1_bit_quantization), every value decoded to
@@ -742,13 +787,14 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             const u64 n = g->pn[key];
             if (!n) continue;
             const int eb = key & 255, E = eb ? eb - 127 : -126;
-            const U128 s1 = ld128(g->ps1[key]), s2 = ld128(g->ps2[key]);
+            const u64* s1 = g->ps1[key];
+            const u64* s2 = g->ps2[key];
             if (!F.l1) {
                 add_sat(acc, n, s1, s2, E, fl, 1ull);  // sum (|x| - c)^2
             } else {
                 // |x| >= 2^E >= c when E >= -fl, else |x| < 2^(E+1) <= c
                 const bool above = E >= -fl;
-                big_add(acc, s1, E - 23, !above);
+                big_add_L3(acc, s1, E - 23, !above);
                 big_add(acc, U128{n, 0ull}, -fl, above);
             }
         }
@@ -764,9 +810,10 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             const u64 n = g->pn[key];
             if (!n) continue;
             const int sg = key >> 8, eb = key & 255, E = eb ? eb - 127 : -126;
-            const U128 s1 = ld128(g->ps1[key]), s2 = ld128(g->ps2[key]);
+            const u64* s1 = g->ps1[key];
+            const u64* s2 = g->ps2[key];
             if (sg == 1 && S == 0) {  // clipped to code 0: error |x|
-                big_add(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
+                big_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
                 continue;
             }
             const int t = (sg == 0) ? (S ? k - 1 : k) : (k - 1);
@@ -774,17 +821,17 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             const int q = E + fl;
             if (q >= t) {
                 if (F.l1) {  // |x| >= T 2^-fl: sum |x| - n T 2^-fl
-                    big_add(acc, s1, E - 23, false);
+                    big_add_L3(acc, s1, E - 23, false);
                     big_add(acc, U128{n * T, 0ull}, -fl, true);
                 } else {
                     add_sat(acc, n, s1, s2, E, fl, T);
                 }
             } else if (sg == 0 && q == t - 1) {
-                big_add(acc, ld128(g->rb[q + 1][fi]), pw * (E - 23), false);
+                big_add_L3(acc, g->rb[q + 1][fi], pw * (E - 23), false);
             } else if (q <= -2) {
-                big_add(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
+                big_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
             } else {
-                big_add(acc, ld128(g->r[sg][q + 1][fi]), pw * (E - 23), false);
+                big_add_L3(acc, g->r[sg][q + 1][fi], pw * (E - 23), false);
             }
         }
     }
@@ -879,6 +926,11 @@ void st_attr_once() {
     FXPQ_FS_ATTR(true, true)
     FXPQ_FS_ATTR(false, true)
 #undef FXPQ_FS_ATTR
+    const int hb = (int)HS_SMEM;
+    cudaFuncSetAttribute(fl_search_hist_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, hb);
+    cudaFuncSetAttribute(fl_search_hist_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, hb);
+    cudaFuncSetAttribute(fl_search_hist_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, hb);
+    cudaFuncSetAttribute(fl_search_hist_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, hb);
     g_fs_attr_done = true;
 }
 }  // namespace
@@ -892,9 +944,26 @@ struct FsItemHost {
     FsFinal f;
     FsOut o;
     int variant;  // bins kernel instance: bit 0 vec, bit 1 small (k_hi <= 9), bit 2 narrow boundary range,
-                  // bit 3 L1 score
+                  // bit 3 L1 score, bit 4 the histogram kernel (then bits 1-2 are clear)
     int grid;     // bins blocks
 };
+
+// The histogram kernel serves a search when every slot it needs has j <= 7: split bit
+// s = min(16, 22 - jneed) >= 15.  Window: the exponents E with a needed slot for some candidate FL,
+// E in [-1 - fl_hi, jneed - fl_lo]; below it every candidate rounds to zero, above it every one
+// saturates.  Both signs take the same window and split (negative keys of an unsigned-only search
+// need their moments alone).
+bool hs_configure(FsParams& P, int S_hi) {
+    const int fl_hi = P.fl_lo + P.nfl - 1;
+    const int jneed = max(max(P.jmax_pos, P.jb_hi), S_hi == 1 ? P.jmax_neg : -1);
+    if (jneed > 7) return false;
+    P.hs_s = min(16, 22 - max(jneed, -1));
+    const int e_lo = -1 - fl_hi, e_hi = max(jneed, -1) - P.fl_lo;
+    P.hs_eb_lo = e_lo + 127;
+    P.hs_w = e_hi - e_lo + 1;
+    // every window exponent is a normal one (fl in [-32, 40], j <= 7)
+    return P.hs_eb_lo >= 1 && P.hs_eb_lo + P.hs_w - 1 <= 254;
+}
 
 fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h) {
     const int64_t n = it.n;
@@ -941,10 +1010,38 @@ fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h
     h.grid = (int)((n + chunk - 1) / chunk);
     h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0) |
                 (h.f.l1 ? 8 : 0);
+    if (hs_configure(P, S_hi) && hs_fits(P)) {
+        // one block per SM, whole iterations per block except the last, at most HS_CHUNK_MAX each
+        const long long waves = n > 0 ? (n + 152LL * HS_CHUNK_MAX - 1) / (152LL * HS_CHUNK_MAX) : 1;
+        long long per = (n + 152 * waves - 1) / (152 * waves);
+        per = (per + HS_ITER - 1) / HS_ITER * HS_ITER;
+        if (per < HS_CHUNK_MIN) per = HS_CHUNK_MIN;
+        if (per > HS_CHUNK_MAX) per = HS_CHUNK_MAX;
+        P.chunk = (int)per;
+        h.grid = n > 0 ? (int)((n + per - 1) / per) : 0;
+        h.variant = 16 | (aligned(it.d_x, 16) ? 1 : 0) | (h.f.l1 ? 8 : 0);
+    } else {
+        P.hs_s = 16;
+        P.hs_eb_lo = 0;
+        P.hs_w = 0;
+    }
     return FXPQ_OK;
 }
 
 void fs_bins_launch(int variant, int grid, const FsBatch& B, int i0, int i1, cudaStream_t s) {
+    if (variant & 16) {
+        const size_t hb = HS_SMEM;
+        const bool vec = variant & 1, l1 = variant & 8;
+        if (vec && !l1)
+            fl_search_hist_kernel<true, false><<<grid, HS_T, hb, s>>>(B, i0, i1);
+        else if (!l1)
+            fl_search_hist_kernel<false, false><<<grid, HS_T, hb, s>>>(B, i0, i1);
+        else if (vec)
+            fl_search_hist_kernel<true, true><<<grid, HS_T, hb, s>>>(B, i0, i1);
+        else
+            fl_search_hist_kernel<false, true><<<grid, HS_T, hb, s>>>(B, i0, i1);
+        return;
+    }
     const size_t sb = sizeof(FsSmem);
     const bool vec = variant & 1, small = variant & 2, narrow = variant & 4, l1 = variant & 8;
 #define FXPQ_FS_LAUNCH(V, L1)                                                            \
@@ -975,7 +1072,7 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
     // order by kernel instance (stable), each item keeping its own bins
     int order[FS_MAX_ITEMS];
     int m = 0;
-    for (int v = 0; v < 16; ++v)
+    for (int v = 0; v < 32; ++v)
         for (int i = 0; i < n; ++i)
             if (h[i].variant == v) order[m++] = i;
     FsBatch B;
