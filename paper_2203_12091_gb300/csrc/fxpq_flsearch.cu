@@ -69,7 +69,8 @@ struct FsGlobal {
     u64 ps2[NKEY][3];
     u64 r[2][NJ][MAXFL][3];
     u64 rb[NJ][MAXFL][3];
-    unsigned mn_inv, mx, nonfinite, pad;  // mn_inv = ~(smallest order key); 0: no finite element
+    unsigned mn_inv, mx, nonfinite, fin_done;  // mn_inv = ~(smallest order key), 0: no finite element;
+                                               // fin_done: finalize blocks done
     u64 nzero;                            // finite zeros (+-0.0): no key, but a binary-quantizer error
     double cells[2][MAXK][MAXFL];         // [S][k - 1][fl - fl_lo]
     double stat_sum, stat_sumsq;
@@ -107,7 +108,8 @@ struct FsFinal {
 struct FsBatch {
     int n_items;
     int blk0[FS_MAX_ITEMS + 1];   // first bins block of each item (bins launches cover item ranges)
-    int cell0[FS_MAX_ITEMS + 1];  // first cell (warp) of each item in the cells launch
+    int cell0[FS_MAX_ITEMS + 1];  // first cell of each item in the finalize launch
+    int fin0[FS_MAX_ITEMS + 1];   // first finalize block of each item
     FsParams p[FS_MAX_ITEMS];
     FsFinal f[FS_MAX_ITEMS];
 };
@@ -680,21 +682,6 @@ __device__ __forceinline__ void big_add_L3(Big& a, const u64* p, int e, bool neg
     if (w2) big_add(a, mul128_64(U128{w2 < 0 ? (u64)(-w2) : (u64)w2, 0ull}, m), e + 64, neg != (w2 < 0));
 }
 
-// a += (the big number held by lane `src_lane`), modulo 2^768 (warp-collective)
-__device__ __forceinline__ void big_add_from_lane(Big& a, int off) {
-    u64 carry = 0ull;
-#pragma unroll
-    for (int i = 0; i < BW; ++i) {
-        const u64 o = __shfl_down_sync(0xFFFFFFFFu, a.w[i], off);
-        const u64 t = a.w[i] + o;
-        const u64 c1 = t < o;
-        const u64 t2 = t + carry;
-        const u64 c2 = t2 < t;
-        a.w[i] = t2;
-        carry = c1 | c2;
-    }
-}
-
 __device__ u64 big_bits64(const Big& a, int pos) {  // bits [pos, pos + 64), zero below bit 0
     const int wi = pos >= 0 ? (pos >> 6) : -((-pos + 63) >> 6);
     const int b = pos - wi * 64;
@@ -748,32 +735,73 @@ __device__ void add_sat(Big& acc, u64 n, const u64* s1, const u64* s2, int E, in
     }
 }
 
-// One warp per candidate cell (plus two cells for the exact stats); lanes split the exponent keys.
-__global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
-    const int gcell = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (gcell >= B.cell0[B.n_items]) return;
-    const int item = batch_item(B.cell0, B.n_items, gcell);
-    const FsParams& P = B.p[item];
-    const FsFinal& F = B.f[item];
-    const int cell = gcell - B.cell0[item];
-    const FsGlobal* g = P.g;
-    const int lane = threadIdx.x & 31;
-    const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
-    Big acc;
+// ------------------------------------------------------------------ finalize: scores, argmin, stats
+constexpr int FIN_T = 256;  // threads per finalize block; one block per cell
+
+// The keys with elements and the non-zero exponent sums of squares of one item, staged per block;
+// after the scoring, the lanes' 768-bit sums (word-major) reuse the moments' storage.
+struct FinSmem {
+    unsigned nkey, nband, last;
+    unsigned key[NKEY];
+    u64 n[NKEY];
+    union {
+        struct {
+            u64 s1[NKEY][3];
+            u64 s2[NKEY][3];
+        } m;
+        u64 col[BW][FIN_T];
+    } u;
+    u64 part[BW][FIN_T / 16][2];  // column sums of 16 lanes: low word, carries
+    unsigned beb[256];
+    u64 band[256][3];
+};
+static_assert(sizeof(u64) * BW * FIN_T <= sizeof(u64) * NKEY * 6, "column buffer fits the moments' storage");
+
+__device__ void fin_stage(FinSmem& sm, const FsGlobal* g) {
+    if (threadIdx.x == 0) sm.nkey = sm.nband = 0u;
+    __syncthreads();
+    for (int key = threadIdx.x; key < NKEY; key += blockDim.x) {
+        const u64 n = g->pn[key];
+        if (!n) continue;
+        const unsigned i = atomicAdd(&sm.nkey, 1u);
+        sm.key[i] = (unsigned)key;
+        sm.n[i] = n;
+#pragma unroll
+        for (int w = 0; w < 3; ++w) {
+            sm.u.m.s1[i][w] = g->ps1[key][w];
+            sm.u.m.s2[i][w] = g->ps2[key][w];
+        }
+    }
+    for (int eb = threadIdx.x; eb < 256; eb += blockDim.x) {
+        const u64 a = g->cband[eb][0], b = g->cband[eb][1], c = g->cband[eb][2];
+        if (!(a | b | c)) continue;
+        const unsigned i = atomicAdd(&sm.nband, 1u);
+        sm.beb[i] = (unsigned)eb;
+        sm.band[i][0] = a;
+        sm.band[i][1] = b;
+        sm.band[i][2] = c;
+    }
+    __syncthreads();
+}
+
+// The exact value of one cell (candidate (S, k, FL), or the two stats cells) in a warp's Big: lanes
+// split the staged keys, then the warp sums its lanes.
+__device__ void fin_cell(Big& acc, const FinSmem& sm, const FsGlobal* g, const FsFinal& F, int cell, int ncell,
+                         int lane, int nlanes) {
     big_zero(acc);
     // the exponent-indexed sums of squares that belong to every L2 cell and to the sum of squares
     const bool with_band = cell == ncell + 1 || (cell < ncell && !F.l1);
     if (with_band)
-        for (int eb = lane; eb < 256; eb += 32) big_add_L3(acc, g->cband[eb], 2 * (eb - 150), false);
+        for (unsigned i = lane; i < sm.nband; i += nlanes) big_add_L3(acc, sm.band[i], 2 * ((int)sm.beb[i] - 150), false);
     if (cell >= ncell) {
         const bool sq = cell == ncell + 1;
-        for (int key = lane; key < NKEY; key += 32) {
-            if (!g->pn[key]) continue;
+        for (unsigned i = lane; i < sm.nkey; i += nlanes) {
+            const int key = (int)sm.key[i];
             const int eb = key & 255, E = eb ? eb - 127 : -126;
             if (sq)
-                big_add_L3(acc, g->ps2[key], 2 * (E - 23), false);
+                big_add_L3(acc, sm.u.m.s2[i], 2 * (E - 23), false);
             else
-                big_add_L3(acc, g->ps1[key], E - 23, (key >> 8) != 0);
+                big_add_L3(acc, sm.u.m.s1[i], E - 23, (key >> 8) != 0);
         }
     } else if (F.k_lo == 1 && F.S_lo + cell / (F.nk * F.nfl) == 1 && (cell % (F.nk * F.nfl)) / F.nfl == 0) {
         // k = 1, S = 1: the binary quantizer (Eq. fp_1_bit_quantization), every value decoded to
@@ -783,18 +811,16 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             const U128 nz{g->nzero, 0ull};
             big_add(acc, nz, F.l1 ? -fl : -2 * fl, false);
         }
-        for (int key = lane; key < NKEY; key += 32) {
-            const u64 n = g->pn[key];
-            if (!n) continue;
+        for (unsigned i = lane; i < sm.nkey; i += nlanes) {
+            const int key = (int)sm.key[i];
+            const u64 n = sm.n[i];
             const int eb = key & 255, E = eb ? eb - 127 : -126;
-            const u64* s1 = g->ps1[key];
-            const u64* s2 = g->ps2[key];
             if (!F.l1) {
-                add_sat(acc, n, s1, s2, E, fl, 1ull);  // sum (|x| - c)^2
+                add_sat(acc, n, sm.u.m.s1[i], sm.u.m.s2[i], E, fl, 1ull);  // sum (|x| - c)^2
             } else {
                 // |x| >= 2^E >= c when E >= -fl, else |x| < 2^(E+1) <= c
                 const bool above = E >= -fl;
-                big_add_L3(acc, s1, E - 23, !above);
+                big_add_L3(acc, sm.u.m.s1[i], E - 23, !above);
                 big_add(acc, U128{n, 0ull}, -fl, above);
             }
         }
@@ -806,12 +832,12 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
         const int fl = F.fl_lo + fi;
         // L2 terms weigh u_E^2 = 2^(2(E-23)), L1 terms u_E = 2^(E-23)
         const int pw = F.l1 ? 1 : 2;
-        for (int key = lane; key < NKEY; key += 32) {
-            const u64 n = g->pn[key];
-            if (!n) continue;
+        for (unsigned i = lane; i < sm.nkey; i += nlanes) {
+            const int key = (int)sm.key[i];
+            const u64 n = sm.n[i];
             const int sg = key >> 8, eb = key & 255, E = eb ? eb - 127 : -126;
-            const u64* s1 = g->ps1[key];
-            const u64* s2 = g->ps2[key];
+            const u64* s1 = sm.u.m.s1[i];
+            const u64* s2 = sm.u.m.s2[i];
             if (sg == 1 && S == 0) {  // clipped to code 0: error |x|
                 big_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
                 continue;
@@ -835,25 +861,9 @@ __global__ void fl_search_cells_kernel(const __grid_constant__ FsBatch B) {
             }
         }
     }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) big_add_from_lane(acc, off);
-    if (lane != 0) return;
-    FsGlobal* gw = P.g;
-    if (cell == ncell) {
-        const bool neg = (long long)acc.w[BW - 1] < 0;
-        if (neg) big_negate(acc);
-        const double v = big_to_double(acc);
-        gw->stat_sum = neg ? -v : v;
-    } else if (cell == ncell + 1) {
-        gw->stat_sumsq = big_to_double(acc);
-    } else {
-        const int S = F.S_lo + cell / (F.nk * F.nfl);
-        const int rem = cell % (F.nk * F.nfl);
-        gw->cells[S][F.k_lo + rem / F.nfl - 1][rem % F.nfl] = big_to_double(acc);
-    }
 }
 
-// Per-item outputs of the select kernel.
+// Per-item outputs.
 struct FsOut {
     double* err;
     int* best;
@@ -864,41 +874,113 @@ struct FsOutBatch {
     FsOut o[FS_MAX_ITEMS];
 };
 
-// One block per item: per wordlength, the scores and the argmin (exact ties keep the smaller FL).
-__global__ void fl_search_select_kernel(const __grid_constant__ FsBatch B, const __grid_constant__ FsOutBatch O,
-                                        int* status) {
-    const int item = blockIdx.x;
+// Finalize: one block per cell of one item (the cells of every S, k, FL, then the two stats cells).
+// Every thread scores its share of the staged keys, and the block adds the lanes' 768-bit sums by
+// columns of words with one carry pass; the item's last block to finish (completion ticket) writes
+// the scores, the argmin per wordlength (exact ties keep the smaller FL) and the stats.
+__global__ void __launch_bounds__(FIN_T) fl_search_final_kernel(const __grid_constant__ FsBatch B,
+                                                                 const __grid_constant__ FsOutBatch O, int* status) {
+    const int item = batch_item(B.fin0, B.n_items, (int)blockIdx.x);
     const FsParams& P = B.p[item];
     const FsFinal& F = B.f[item];
     const FsOut& out = O.o[item];
-    const FsGlobal* g = P.g;
+    FsGlobal* g = P.g;
+    __shared__ FinSmem sm;
+    const int cell = (int)blockIdx.x - B.fin0[item];
+    const int nblk = B.fin0[item + 1] - B.fin0[item];
+    const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
+    const int tid = (int)threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    fin_stage(sm, g);
+    {
+        Big acc;
+        fin_cell(acc, sm, g, F, cell, ncell, tid, FIN_T);
+        __syncthreads();  // the moments' storage becomes the column buffer
+#pragma unroll
+        for (int w = 0; w < BW; ++w) sm.u.col[w][tid] = acc.w[w];
+    }
+    __syncthreads();
+    if (tid < BW * 16) {  // 16-lane column sums of each word: the low word and its carries
+        const int w = tid >> 4, j = tid & 15;
+        u64 lo = 0ull, c = 0ull;
+        for (int l = 0; l < 16; ++l) {
+            const u64 v = sm.u.col[w][16 * j + l];
+            lo += v;
+            c += lo < v ? 1ull : 0ull;
+        }
+        sm.part[w][j][0] = lo;
+        sm.part[w][j][1] = c;
+    }
+    __syncthreads();
+    if (tid < BW) {  // whole columns: the low word and the carry into the next word
+        u64 lo = 0ull, c = 0ull;
+        for (int j = 0; j < 16; ++j) {
+            lo += sm.part[tid][j][0];
+            c += (lo < sm.part[tid][j][0] ? 1ull : 0ull) + sm.part[tid][j][1];
+        }
+        sm.part[tid][0][0] = lo;
+        sm.part[tid][1][1] = c;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        Big acc;
+        u64 cin = 0ull;
+        for (int w = 0; w < BW; ++w) {  // modulo 2^768: the carry out of the top word drops
+            const u64 lo = sm.part[w][0][0] + cin;
+            acc.w[w] = lo;
+            cin = sm.part[w][1][1] + (lo < cin ? 1ull : 0ull);
+        }
+        if (cell == ncell) {
+            const bool neg = (long long)acc.w[BW - 1] < 0;
+            if (neg) big_negate(acc);
+            const double v = big_to_double(acc);
+            g->stat_sum = neg ? -v : v;
+        } else if (cell == ncell + 1) {
+            g->stat_sumsq = big_to_double(acc);
+        } else {
+            const int S = F.S_lo + cell / (F.nk * F.nfl);
+            const int rem = cell % (F.nk * F.nfl);
+            g->cells[S][F.k_lo + rem / F.nfl - 1][rem % F.nfl] = big_to_double(acc);
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        sm.last = atomicAdd(&g->fin_done, 1u) == (unsigned)(nblk - 1) ? 1u : 0u;
+    }
+    __syncthreads();
+    if (!sm.last) return;
+    __threadfence();
     const float mn = g->mn_inv == 0u ? 0.0f : order_key_inv(~g->mn_inv);
     const float mx = g->mx == 0u ? 0.0f : order_key_inv(g->mx);
     const int S = out.is_signed >= 0 ? out.is_signed : (mn < 0.0f ? 1 : 0);
-    const int i = threadIdx.x;
-    if (i < F.nk) {
+    for (int i = warp; i < F.nk; i += FIN_T / 32) {  // one warp per wordlength, one lane per FL
         const int k = F.k_lo + i;
-        double bv = 0.0;
-        int bf = F.fl_lo;
-        for (int fi = 0; fi < F.nfl; ++fi) {
-            const double v = g->cells[S][k - 1][fi];
-            out.err[(long long)i * F.nfl + fi] = v;
-            if (fi == 0 || v < bv) {  // strict: exact ties keep the smaller FL
-                bv = v;
-                bf = F.fl_lo + fi;
+        double v = __longlong_as_double(0x7FF0000000000000ll);
+        if (lane < F.nfl) {
+            v = __ldcg(&g->cells[S][k - 1][lane]);
+            out.err[(long long)i * F.nfl + lane] = v;
+        }
+        int bf = lane;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const double ov = __shfl_down_sync(0xFFFFFFFFu, v, off);
+            const int of = __shfl_down_sync(0xFFFFFFFFu, bf, off);
+            if (ov < v || (ov == v && of < bf)) {  // exact ties keep the smaller FL
+                v = ov;
+                bf = of;
             }
         }
-        out.best[i] = bf;
+        if (lane == 0) out.best[i] = F.fl_lo + bf;
     }
-    if (i == 0) {
+    if (threadIdx.x == 0) {
         if (g->nonfinite) latch_status(status, FXPQ_ERR_NONFINITE);
         if (out.stats) {
             out.stats->min = mn;
             out.stats->max = mx;
             out.stats->is_signed = S;
             out.stats->nonfinite = g->nonfinite ? 1 : 0;
-            out.stats->sum = g->stat_sum;
-            out.stats->sumsq = g->stat_sumsq;
+            out.stats->sum = __ldcg(&g->stat_sum);
+            out.stats->sumsq = __ldcg(&g->stat_sumsq);
             out.stats->n = P.n;
         }
     }
@@ -1078,7 +1160,7 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
     FsBatch B;
     FsOutBatch O;
     B.n_items = n;
-    int cells = 0;
+    int cells = 0, fblocks = 0;
     for (int j = 0; j < n; ++j) {
         const FsItemHost& it = h[order[j]];
         B.p[j] = it.p;
@@ -1086,9 +1168,13 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
         B.f[j] = it.f;
         O.o[j] = it.o;
         B.cell0[j] = cells;
-        cells += (it.f.S_hi - it.f.S_lo + 1) * it.f.nk * it.f.nfl + 2;
+        B.fin0[j] = fblocks;
+        const int nc = (it.f.S_hi - it.f.S_lo + 1) * it.f.nk * it.f.nfl + 2;
+        cells += nc;
+        fblocks += nc;  // one finalize block per cell
     }
     B.cell0[n] = cells;
+    B.fin0[n] = fblocks;
     st_attr_once();
     for (int j0 = 0; j0 < n;) {
         const int v = h[order[j0]].variant;
@@ -1106,11 +1192,8 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
         }
         j0 = j1;
     }
-    fl_search_cells_kernel<<<(cells + 3) / 4, 128, 0, s>>>(B);
-    fxpq_status st = after_launch("fl_search_cells");
-    if (st != FXPQ_OK) return st;
-    fl_search_select_kernel<<<n, 32, 0, s>>>(B, O, status_ptr());
-    return after_launch("fl_search_select");
+    fl_search_final_kernel<<<fblocks, FIN_T, 0, s>>>(B, O, status_ptr());
+    return after_launch("fl_search_final");
 }
 }  // namespace
 
@@ -1216,7 +1299,7 @@ extern "C" fxpq_status fxpq_fl_search_noalloc(const float* d_x, int64_t n, int32
                                               int32_t* d_best, fxpq_stats* d_stats, void* stream) {
     if (n < 0 || n > (int64_t(1) << 31)) return FXPQ_ERR_INVALID_ARG;  // the largest tensor the bins can hold
     if (k_lo < 1 || k_hi > 16 || k_lo > k_hi || fl_lo > fl_hi || fl_hi - fl_lo + 1 > MAXFL)
-        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 16 x 32
+        return FXPQ_ERR_INVALID_ARG;  // the largest candidate grid the array holds: 16 x 32 (k in [1, 16])
     if (fxpq_fl_search_workspace(n) > kFlSearchStaticBytes) return FXPQ_ERR_WORKSPACE;
     void* scratch = nullptr;
     const fxpq_status st = fl_search_scratch_ptr(&scratch);

@@ -279,13 +279,19 @@ __device__ void hs_convert_key(const FsParams& P, const unsigned* smem, const u6
                 // g = Hf = 2^HB + h: the rounding bit is the implicit one, A = 2^HB - 1 - h
 #pragma unroll
                 for (int i = 0; i < NE; ++i) hs_term<L1>(X, Y, (unsigned)(nH - 1 - ((int)lane + 32 * i)), 1u, n[i], sl[i], s);
-            } else if (pb >= 5) {
+            } else if (pb >= 6) {
+                // entry i holds g = lane + 32 i: its rounding bit (bit pb - 1 >= 5) is bit pb - 6 of i
 #pragma unroll
                 for (int i = 0; i < ((1 << pb) >> 5); ++i) {
-                    unsigned A, b;
-                    hs_round(lane + 32u * i, pb, A, b);
+                    const unsigned b = ((unsigned)i >> (pb - 6)) & 1u;
+                    const unsigned m = (1u << (pb - 1)) - 1u;
+                    const unsigned A = ((lane + 32u * i) & m) ^ (b ? m : 0u);
                     hs_term<L1>(X, Y, A, b, n[i], sl[i], s);
                 }
+            } else if (pb == 5) {
+                unsigned A, b;
+                hs_round(lane, pb, A, b);
+                hs_term<L1>(X, Y, A, b, n[0], sl[0], s);
             } else if (lane < (1u << pb)) {
                 unsigned A, b;
                 hs_round(lane, pb, A, b);
