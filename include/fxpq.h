@@ -194,8 +194,8 @@ FXPQ_API fxpq_status fxpq_fl_search_batch(const fxpq_fl_search_item* h_items, in
  * enter the allocator (cudaMalloc may synchronise the device).  The paper has no counterpart: this
  * is a deployment variant of fxpq_fl_search with the same arguments, results and limits, minus
  * the workspace.  It allocates nothing.  Its scratch is a file-scope device array of about
- * 53 KiB inside libfxpq.so that every GPU which loads the library holds until the process exits.
- *   - Limits: n <= 2^31 elements and at most 15 x 32 candidates (k in [2,16], fl_hi-fl_lo <= 31);
+ * 81 KiB inside libfxpq.so that every GPU which loads the library holds until the process exits.
+ *   - Limits: n <= 2^31 elements and at most 16 x 32 candidates (k in [1,16], fl_hi-fl_lo <= 31);
  *     larger requests return FXPQ_ERR_INVALID_ARG before any launch.
  *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
  *     that device current; make that first call before any stream capture begins.
@@ -369,8 +369,9 @@ FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_imag
                              int64_t* d_logits, int32_t* h_logits_scale, void* d_ws, size_t ws_bytes,
                              void* stream);
 
-/* Calibration of the activation formats in the forward optimizer's order (Sec. IV-C; reading 9 of
- * the design notes): the input FxP-QLayer's FL is searched on the fp32 calibration images, then
+/* Calibration of the activation formats in the forward optimizer's order (Sec. IV-C, which does not
+ * say where activation FLs come from; here they are searched on a calibration slice and then
+ * frozen): the input FxP-QLayer's FL is searched on the fp32 calibration images, then
  * layer by layer, with every earlier layer already quantized, the FL of each op's output QLayer is
  * searched on the fp32 nearest-even image of its exact C-Block output (conv: one contraction to
  * int64 values, the QLayer applied twice; eltwise / avg-pool: their F32 and CODES modes).  S is

@@ -2,7 +2,8 @@
 
 TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).
 
-Readings of the paper used here (each is listed with its reason in the design doc):
+Readings of the paper used here, where it is silent or ambiguous (the CUDA path follows the same
+readings):
 
 * FxP-QLayers sit after the input and after every C-Block output, not after MAX-POOL and
   not after the last layer (Sec. IV-A.2).

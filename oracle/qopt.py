@@ -5,7 +5,8 @@ TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).  Plain numpy in float64; 
 network are evaluated in float64 here (the GPU evaluates them in fp32; the tests compare within a
 tolerance).
 
-Readings of the paper used here (each is listed with its reason in the design doc):
+Readings of the paper used here, where it is silent or ambiguous (the CUDA path follows the same
+readings):
 
 * Data-structures: the network input's activations ("input", a only), then per layer in order its
   weights w, bias b (conv/FC only) and output activations a (not for MAX-POOL, which has no QLayer,

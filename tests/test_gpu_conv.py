@@ -320,3 +320,71 @@ def test_conv_scale_layer_parity(F, sc):
                            scale=(m, scale[1], h, scale[3]))
     assert s == ws
     assert np.array_equal(got, want)
+
+
+# ---------------------------------------------------------------- exactness at the fp32 group bound
+def _edge_case(kind, K):
+    """Codes that drive every exact fp32 group of the tensor-core path to its planner bound, with odd
+    partial sums (an accumulator that dropped low bits would change them).
+
+    "wordlength": 8-bit unsigned x = 255, 8-bit signed w = -128 or 127: the bound alone makes groups of
+      512 taps (255 * 128 * 512 = 16,711,680 < 2^24), and one weight per channel is nudged by one so
+      that every group sum is odd.
+    "limbs": 16-bit codes whose low limbs are all 255: lo x lo products of 65,025 in groups of 256
+      taps (16,646,400).
+    "l1": 8-bit unsigned x = 255 with sum |w[o]| = 65,793, so that max|x| * w_l1 = 2^24 - 1: the L1
+      bound makes the whole reduction one group and channels of one sign reach exactly +-(2^24 - 1).
+    """
+    N, H, C, R = 2, 5, 64, 3  # 3 x 3 taps over 64 channels: 576 taps per output, no padding
+    taps = R * R * C
+    rng = np.random.default_rng({"wordlength": 1, "limbs": 2, "l1": 3}[kind] * 100 + K)
+    if kind == "limbs":
+        hi_x = rng.integers(-100, 100, size=(N, H, H, C))
+        x = hi_x * 256 + 255
+        hi_w = rng.integers(-100, 100, size=(K, taps))
+        lo_w = np.full((K, taps), 255)
+        lo_w[:, [0, 256, 512]] = 254  # one even product per 256-tap group: odd group sums
+        w = (hi_w * 256 + lo_w).reshape(K, R, R, C)
+        return x, (16, 1, 12), w, (16, 1, 14), (16, 1, 20)
+    x = np.full((N, H, H, C), 255)
+    x[0, 0, 0, :5] = [254, 253, 1, 0, 128]  # a few other codes so the rows differ
+    if kind == "wordlength":
+        sign = np.where(np.arange(K) % 2 == 0, -1, 1)
+        w = np.where(sign[:, None] < 0, -128, 127) * np.ones((K, taps), np.int64)
+        w[:, 7] -= sign  # -127 / 126: odd group sums
+        return x, (8, 0, 4), w.reshape(K, R, R, C), (8, 1, 7), (16, 1, 15)
+    # l1: per channel sum |w| = 65793 = 513 * 128 + 63 * 2 + 3, one sign per channel
+    mag = np.concatenate([np.full(513, 128), np.full(62, 2), [5]])
+    assert mag.sum() == 65793 and mag.size == taps
+    w = np.empty((K, taps), np.int64)
+    for o in range(K):
+        m = rng.permutation(mag)
+        w[o] = -m if o % 3 == 0 else np.minimum(m, 127)
+    # positive channels cannot reach 128: keep them at 127 (their bound is then lower); the negative
+    # channels carry the exact 2^24 - 1 sums
+    return x, (8, 0, 4), w.reshape(K, R, R, C), (8, 1, 7), (16, 1, 15)
+
+
+@pytest.mark.parametrize("kind", ["wordlength", "limbs", "l1"])
+@pytest.mark.parametrize("K,mode", [(64, 1), (128, 1), (256, 1), (128, 0)])
+def test_conv_exact_at_group_bound(F, kind, K, mode):
+    x, tx, w, tw, tb = _edge_case(kind, K)
+    fx, fw = F.fmt(*tx), F.fmt(*tw)
+    fb = F.fmt(tb[0], 1, tb[1])
+    b = np.zeros(K, np.int64)
+    b[::5] = 3
+    fy = F.fmt(8, 1, -12) if mode == 0 else None
+    Cp = x.shape[-1]
+    w_l1 = int(np.abs(w).reshape(K, -1).sum(axis=1).max()) if kind == "l1" else 0
+    if kind == "l1":
+        assert 255 * w_l1 == 2 ** 24 - 1
+    got, s = run_conv(F, x, fx, w, fw, b, fb, 1, 0, False, mode, fy, Cp, w_l1)
+    want, ws = oracle_conv(x, fx, w, fw, b, fb, 1, 0, False, mode, fy)
+    assert s == ws
+    assert np.array_equal(got, want)
+    if mode == 1:
+        acc = oracle.conv2d(x, w, 1, 0)
+        if kind == "l1":
+            assert np.abs(acc).max() == 2 ** 24 - 1  # the exact edge is reached
+        if kind == "wordlength":
+            assert np.any(acc % 2 == 1) and np.abs(acc).max() > 2 ** 24  # odd sums; the full reduction exceeds one group

@@ -410,8 +410,10 @@ def test_tiny_network_layers_equal_quantized_exact_reals():
     acc = oracle.conv2d(x, qp["c1"][0], 1, 1)
     v, s = oracle.cblock(acc, fx[2] + fmts["c1"]["w"][2], qp["c1"][1], fmts["c1"]["b"][2], True)
     vf = oracle.to_f32(v, s)
-    errs = [frac_l2(vf.ravel()[:64], 5, 0, fl) for fl in range(-8, 24)]  # sub-sample sanity: finite & ordered
-    assert all(e >= 0 for e in errs)
+    k, S, fl_c = fmts["c1"]["a"]
+    assert S == (1 if vf.min() < 0 else 0)  # sign strategy of Sec. IV-A.3
+    errs = [frac_l2(vf.ravel(), k, S, fl) for fl in range(-8, 24)]  # exact L of every candidate FL
+    assert fl_c == -8 + min(range(32), key=lambda i: (errs[i], i))  # smallest L, exact ties to the smaller FL
 
 
 # ---------------------------------------------------------------- architecture size pins
@@ -724,3 +726,115 @@ def test_forward_optimizer_cost_is_zero_for_on_grid_data():
     F_, E, uc, mp = net.cost(("fc", "b"), net.fmt[("fc", "b")][2])
     assert E == 0.0
     assert F_ == uc + mp
+
+
+# ---------------------------------------------------------------- forward optimizer: E, pi, sigma, R
+def _pop_sigma(vals):
+    """Population standard deviation from the exact mean and variance (Fractions), then one sqrt."""
+    fr = [F(v) for v in vals]
+    m = sum(fr) / len(fr)
+    return float(sum((v - m) ** 2 for v in fr) / len(fr)) ** 0.5
+
+
+def test_ds_stats_population_sigma_and_per_sample_activations():
+    """Eq. importance's sigma is the population deviation; activations take it per sample (averaged over
+    the calibration samples) with nu the per-sample size; Eq. data_range's R = max - min."""
+    s, n, R = qopt.ds_stats(np.array([1.0, 2.0, 3.0, 6.0]), per_sample=False)
+    assert s == pytest.approx(3.5 ** 0.5, rel=1e-15) and n == 4 and R == 5.0  # sample deviation: sqrt(14/3)
+    s, n, R = qopt.ds_stats(np.array([[0.0, 2.0], [1.0, 5.0]]), per_sample=True)
+    assert s == pytest.approx(1.5, rel=1e-15) and n == 2 and R == 5.0  # per-tensor: sqrt(3.5), nu 4
+
+
+def _two_layer_net():
+    """conv c1 (1x1, 1 -> 2 channels, no ReLU) then fc (1x1 over 2x2 maps of 2 channels -> 2 classes),
+    hand-sized weights, two 2x2 single-channel images."""
+    layers = [{"type": "conv", "name": "c1", "C": 1, "K": 2, "R": 1, "stride": 1, "pad": 0, "relu": False, "src": None},
+              {"type": "conv", "name": "fc", "C": 2, "K": 2, "R": 2, "stride": 1, "pad": 0, "relu": False, "src": None}]
+    W = {"c1": (np.array([0.8125, -0.40625], np.float32).reshape(2, 1, 1, 1), np.array([0.1, -0.3], np.float32)),
+         "fc": (np.array([0.3, -0.7, 0.45, 0.2, -0.15, 0.6, 0.05, -0.35,
+                          0.25, 0.5, -0.6, 0.1, 0.7, -0.2, 0.35, 0.15], np.float32).reshape(2, 2, 2, 2),
+                np.array([0.02, -0.01], np.float32))}
+    imgs = np.array([[[[1.3, -0.7], [0.4, 2.1]]], [[[-1.6, 0.9], [0.25, -0.45]]]], np.float32)
+    plan = {"input": 6, "c1": {"w": 4, "b": 5, "a": 5}, "fc": {"w": 5, "b": 6}}
+    return layers, W, imgs, plan
+
+
+def _fq(v, fmt):
+    k, S, fl = fmt
+    return Fraction(frac_q(v, k, S, fl)) * Fraction(2) ** (-fl)
+
+
+def _term(vals, fmt, per_sample, nsamp):
+    """(sigma * nu, L / R) of one data-structure straight from Eqs. importance, DSB_QE and data_range."""
+    flat = [float(v) for v in np.asarray(vals, np.float64).ravel()]
+    if per_sample:
+        m = len(flat) // nsamp
+        sig = sum(_pop_sigma(flat[i * m:(i + 1) * m]) for i in range(nsamp)) / nsamp
+        nu = m
+    else:
+        sig, nu = _pop_sigma(flat), len(flat)
+    L = sum((F(v) - _fq(v, fmt)) ** 2 for v in flat)
+    R = F(max(flat)) - F(min(flat))
+    return sig * nu, (float(L / R) if R else 0.0)
+
+
+def _E(layer_terms):
+    """Eq. CPB_QE: per layer, pi_j = sigma_j nu_j / sum (sigma nu), E = sum pi_j L_j / R_j."""
+    E = 0.0
+    for terms in layer_terms:
+        den = sum(sn for sn, _ in terms)
+        E += sum(sn / den * lr for sn, lr in terms)
+    return E
+
+
+def test_cost_E_from_the_equations_with_a_later_layer_fp32():
+    """E for c1's weights at candidate FLs: the input is fixed point (optimized before), c1's weights take
+    the candidate, c1's bias and activations and all of fc are FP32 -- and each term's L is taken under
+    its own QPs (candidate, or the initial QPs of the preprocessor)."""
+    layers, W, imgs, plan = _two_layer_net()
+    net = qopt.Net(layers, W, imgs, plan)
+    x = np.transpose(imgs.astype(np.float64), (0, 2, 3, 1))  # NHWC, one channel
+    fin = net.fmt[("input", "a")]
+    xq = [[_fq(v, fin) for v in img.ravel()] for img in x]
+    w1, b1 = W["c1"]
+    for cand in (net.fmt[("c1", "w")][2] - 1, net.fmt[("c1", "w")][2], net.fmt[("c1", "w")][2] + 2):
+        fw = (net.fmt[("c1", "w")][0], net.fmt[("c1", "w")][1], cand)
+        wq = [_fq(v, fw) for v in w1.ravel()]
+        # c1's output (FP32 bias, no ReLU): sample-major, pixel, channel
+        y = [[float(xq[n][p] * wq[c] + F(b1[c])) for p in range(4) for c in range(2)] for n in range(2)]
+        c1_terms = [_term(y, net.fmt[("c1", "a")], True, 2), _term(w1, fw, False, 1),
+                    _term(b1, net.fmt[("c1", "b")], False, 1)]
+        fc_terms = [_term(W["fc"][0], net.fmt[("fc", "w")], False, 1), _term(W["fc"][1], net.fmt[("fc", "b")], False, 1)]
+        want = _E([c1_terms, fc_terms])
+        _, E, _, _ = net.cost(("c1", "w"), cand)
+        assert E == pytest.approx(want, rel=1e-12)
+
+
+def test_cost_E_in_a_mixed_state_with_a_quantized_prefix():
+    """E for fc's weights once input, c1's w, b and a are fixed point at their QPs: only layer fc's terms
+    count, fc's input is c1's quantized output, and fc's bias keeps its initial QPs (FP32 values)."""
+    layers, W, imgs, plan = _two_layer_net()
+    net = qopt.Net(layers, W, imgs, plan)
+    for ds in net.order[:4]:
+        net.done.add(ds)
+    cur = ("fc", "w")
+    assert net.order[4] == cur
+    for cand in (net.fmt[cur][2], net.fmt[cur][2] + 1):
+        fw = (net.fmt[cur][0], net.fmt[cur][1], cand)
+        _, E, uc, mp = net.cost(cur, cand)
+        want = _E([[_term(W["fc"][0], fw, False, 1), _term(W["fc"][1], net.fmt[("fc", "b")], False, 1)]])
+        assert E == pytest.approx(want, rel=1e-12)
+    # the logits of this forward: quantized input, c1 weights, bias and output, candidate fc weights
+    x = np.transpose(imgs.astype(np.float64), (0, 2, 3, 1))
+    fin, f1w, f1b, f1a = (net.fmt[d] for d in net.order[:4])
+    fw = net.fmt[cur]
+    w1, b1 = W["c1"]
+    wf, bf = W["fc"]
+    logits = []
+    for n in range(2):
+        h = [[_fq(_fq(x[n].ravel()[p], fin) * _fq(w1.ravel()[c], f1w) + _fq(b1[c], f1b), f1a) for c in range(2)]
+             for p in range(4)]
+        logits.append([sum(h[p][c] * _fq(wf[o].reshape(4, 2)[p, c], fw) for p in range(4) for c in range(2)) + F(bf[o])
+                       for o in range(2)])
+    X, lg = net.forward(cur, fw[2])
+    assert np.array_equal(lg, np.array([[float(v) for v in row] for row in logits]))

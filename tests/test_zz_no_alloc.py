@@ -27,7 +27,9 @@ def test_noalloc_fl_search_matches_workspace_version_twice():
     from paper_2203_12091_gb300 import _lib as L
     lib = L.lib()
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
-    cases = [("normal", 1 << 20, 2, -1, 2, 16, -8, 23), ("laplace", 300001, 3, 1, 4, 9, -2, 21)]
+    # the sorting kernel (k up to 16, k = 1 rows included) and the histogram kernel (k <= 8)
+    cases = [("normal", 1 << 20, 2, -1, 2, 16, -8, 23), ("laplace", 300001, 3, 1, 4, 9, -2, 21),
+             ("normal", 50000, 5, -1, 1, 16, -8, 23), ("relu_normal", 70001, 4, -1, 1, 8, -8, 23)]
     for dist, n, seed, S, klo, khi, fllo, flhi in cases:
         x = torch.from_numpy(synth.sweep_tensor(dist, n, seed)).cuda()
         nk, nfl = khi - klo + 1, flhi - fllo + 1
