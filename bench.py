@@ -15,6 +15,7 @@ Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a bound
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
 import statistics
@@ -59,47 +60,66 @@ def dist_env():
 
 
 class ClockSampler:
-    """nvidia-smi samples during the timed region (SM clock, max clock, throttle reasons)."""
+    """nvidia-smi samples during the timed region (SM clock, max clock, throttle reasons): one
+    streaming nvidia-smi process (-lms 25), started ahead of the region; only the samples stamped
+    inside the region are kept."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
-        self.samples = []
-        self._stop = threading.Event()
+        self.samples = []  # (monotonic time, fields)
+        self._p = None
         self._t = None
+        self.t0 = self.t1 = None
 
     def _run(self):
-        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
-             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-             "clocks_event_reasons.sw_power_cap")
-        while not self._stop.is_set():
-            try:
-                out = subprocess.run(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}", "--format=csv,noheader,nounits"],
-                                     capture_output=True, text=True, timeout=5).stdout.strip()
-                if out:
-                    self.samples.append([s.strip() for s in out.split(",")])
-            except Exception:
-                pass
-            self._stop.wait(0.2)
+        for line in self._p.stdout:
+            f = [x.strip() for x in line.strip().split(",")]
+            if len(f) >= 7:
+                self.samples.append((time.monotonic(), f))
 
     def __enter__(self):
-        self._t = threading.Thread(target=self._run, daemon=True)
-        self._t.start()
+        try:
+            self._p = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                        "--format=csv,noheader,nounits", "-lms", "25"],
+                                       stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+            deadline = time.monotonic() + 3.0
+            while not self.samples and time.monotonic() < deadline:
+                time.sleep(0.01)
+        except Exception:
+            self._p = None
+        self.t0 = time.monotonic()
         return self
 
     def __exit__(self, *a):
-        self._stop.set()
+        self.t1 = time.monotonic()
+        time.sleep(0.05)  # let the sample that straddles the end arrive
+        if self._p:
+            self._p.terminate()
+            try:
+                self._p.wait(timeout=5)
+            except Exception:
+                self._p.kill()
         if self._t:
-            self._t.join(timeout=10)
+            self._t.join(timeout=5)
 
     def summary(self):
-        if not self.samples:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm = [float(s[0]) for s in self.samples if s[0].replace(".", "").isdigit()]
-        mx = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        inside = [f for t, f in self.samples if self.t0 <= t <= self.t1 + 0.03]
+        if not inside:  # a region shorter than the sampling interval: the nearest samples
+            inside = [f for t, f in self.samples[-2:]]
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        sm = [float(s[0]) for s in inside if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in inside if s[1].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for s in self.samples for i in range(4) if len(s) > 3 + i and s[3 + i] == "Active"})
+        reasons = sorted({names[i] for s in inside for i in range(4) if len(s) > 3 + i and s[3 + i] == "Active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(self.samples)}
+                "reasons": reasons, "samples": len(inside)}
 
 
 def measured_peaks():
@@ -236,9 +256,9 @@ def run_fxpq(args):
 def conv_roofline(q, imgs, F, stream, iters=3):
     """Average conv launch time over `iters` op-by-op forwards (CUDA events on the launching stream).
 
-    A short device-side sleep is queued ahead of each timed conv, so that the host's argument
-    preparation overlaps it and the events bracket the conv kernel(s) alone rather than the host gap
-    before the launch."""
+    A device-side sleep of about 1 ms is queued ahead of each timed conv, so that the host's argument
+    preparation (workspace queries, tensor-map encoding, the split reduction's workspace) overlaps it
+    and the events bracket the conv kernel(s) alone rather than the host gap before the launch."""
     import torch
     env0 = None
     tot_ms, flops, n = 0.0, 0, 0
@@ -254,7 +274,7 @@ def conv_roofline(q, imgs, F, stream, iters=3):
             mode = F.OUT_ACC64 if i == last else F.OUT_CODES
             if L_["type"] == "conv":
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                torch.cuda._sleep(400_000)  # ~0.2 ms at 2 GHz: longer than the host work of run_layer
+                torch.cuda._sleep(2_000_000)  # ~1 ms at 2 GHz: longer than the host work of run_layer
                 e0.record(stream)
                 y, s = q.run_layer(i, env, N, mode)
                 e1.record(stream)
@@ -270,6 +290,181 @@ def conv_roofline(q, imgs, F, stream, iters=3):
         del env0
         env0 = env
     return tot_ms, flops, n
+
+
+# ----------------------------------------------------------------------------- configs 1 and 2
+CONFIG1 = {"N": 8, "H": 32, "C": 64, "K": 64, "R": 3}  # 3x3 conv, stride 1, pad 1, 8-bit w/a, FL in 0..15
+
+
+def config1_inputs():
+    """The single-conv workload: ReLU(N(0,1)) NHWC inputs, He-normal KRSC weights (std sqrt(2/576)),
+    N(0, 0.01) biases, seeded."""
+    c = CONFIG1
+    x = np.maximum(synth.normal(c["N"] * c["H"] * c["H"] * c["C"], 1), np.float32(0)).reshape(c["N"], c["H"], c["H"], c["C"])
+    w = synth.normal(c["K"] * c["R"] * c["R"] * c["C"], 2, std=float(np.sqrt(2.0 / (c["R"] * c["R"] * c["C"])))).reshape(
+        c["K"], c["R"], c["R"], c["C"])
+    b = synth.normal(c["K"], 3, std=0.01)
+    return x, w, b
+
+
+def oracle_config1():
+    """The oracle running the single-conv workload: FL searches of x, w (k = 8, FL 0..15) and b (k = 16,
+    FL -8..23), quantization, the C-Block to its fp32 image, the output FL search, the requantized codes."""
+    import oracle
+    x, w, b = config1_inputs()
+    t0 = time.perf_counter()
+    fmts = []
+    for t, k, lo, hi in ((x, 8, 0, 15), (w, 8, 0, 15), (b, 16, -8, 23)):
+        _, best, S, _ = oracle.fl_search(t, -1, k, k, lo, hi)
+        fmts.append((k, S, int(best[0])))
+    (kx, Sx, flx), (kw, Sw, flw), (kb, Sb, flb) = fmts
+    xq, wq, bq = oracle.quantize(x, kx, Sx, flx), oracle.quantize(w, kw, Sw, flw), oracle.quantize(b, kb, Sb, flb)
+    acc = oracle.conv2d(xq.reshape(x.shape), wq.reshape(w.shape), 1, 1)
+    v, sc = oracle.cblock(acc, flx + flw, bq, flb, True)
+    _, best, Sy, _ = oracle.fl_search(oracle.to_f32(v, sc), -1, 8, 8, 0, 15)
+    oracle.requant(v, sc, 8, Sy, int(best[0]))
+    return time.perf_counter() - t0
+
+
+def oracle_config2(n, sweep):
+    import oracle
+    x = synth.sweep_tensor("normal", n, 2)
+    t0 = time.perf_counter()
+    if sweep:
+        oracle.fl_search(x, -1, 2, 16, -8, 23)
+    else:
+        oracle.fl_search(x, -1, 8, 8, -8, 23)
+    return time.perf_counter() - t0
+
+
+def oracle_job(spec):
+    """Time one oracle job (run in a subprocess with OMP_NUM_THREADS set by the caller)."""
+    kind, *a = spec.split(":")
+    if kind == "config1":
+        t = oracle_config1()
+    else:
+        t = oracle_config2(int(a[0]), a[1] == "sweep")
+    print(json.dumps({"oracle_s": t}))
+
+
+def timed_oracle(spec, threads):
+    """Seconds of an oracle job on `threads` host cores (a subprocess, so that OpenMP reads its count)."""
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads))
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-job", spec], capture_output=True,
+                       text=True, env=env, timeout=900)
+    return json.loads(r.stdout.strip().splitlines()[-1])["oracle_s"]
+
+
+def bench_config1(args, F):
+    """The single-conv workload end to end on the GPU (FL searches of x, w and b as one batch, their
+    quantization, the C-Block's fp32 image and its FL search, the requantized codes) and the final
+    C-Block alone; the oracle on the same workload on one and on all host cores."""
+    import torch
+    import paper_2203_12091_gb300._lib as L
+    c = CONFIG1
+    x, w, b = config1_inputs()
+    xd, wd, bd = (torch.from_numpy(np.ascontiguousarray(t)).cuda().reshape(-1) for t in (x, w, b))
+    dev = xd.device
+    N, H, C, K, R = c["N"], c["H"], c["C"], c["K"], c["R"]
+    REC = 64
+    res = torch.empty(3 * REC, dtype=torch.uint8, device=dev)
+    err = torch.empty(3 * 32, dtype=torch.float64, device=dev)
+    ws = F.workspace(F.fxpq_fl_search_batch_workspace(3), dev)
+    xq = torch.empty(xd.numel(), dtype=torch.float16, device=dev)
+    wq = torch.empty(wd.numel(), dtype=torch.float16, device=dev)
+    bq = torch.empty(K, dtype=torch.int32, device=dev)
+    y32 = torch.empty(N * H * H * K, dtype=torch.float32, device=dev)
+    y = torch.empty(N * H * H * K, dtype=torch.float16, device=dev)
+    flops = 2 * N * H * H * K * C * R * R
+
+    def search(items):
+        batch = [L.FlSearchItem(t.data_ptr(), t.numel(), -1, k, k, lo, hi, err.data_ptr() + 8 * 32 * i,
+                                res.data_ptr() + REC * i, res.data_ptr() + REC * i + 8)
+                 for i, (t, k, lo, hi) in enumerate(items)]
+        F.fxpq_fl_search_batch(batch, ws)
+        host = bytes(res.cpu().numpy().tobytes())
+        out = []
+        for i, (t, k, lo, hi) in enumerate(items):
+            best = int.from_bytes(host[REC * i:REC * i + 4], "little", signed=True)
+            st = L.Stats.from_buffer_copy(host[REC * i + 8:REC * i + 8 + ctypes.sizeof(L.Stats)])
+            out.append(F.fmt(k, st.is_signed, best))
+        return out
+
+    state = {}
+
+    def step():
+        fx, fw, fb = search([(xd, 8, 0, 15), (wd, 8, 0, 15), (bd, 16, -8, 23)])
+        F.fxpq_quantize(xd, fx, F.DT_F16, xq)
+        F.fxpq_quantize(wd, fw, F.DT_F16, wq)
+        F.fxpq_quantize(bd, fb, F.DT_I32, bq)
+        d32 = F.conv_desc(N, H, H, C, C, K, R, R, 1, 1, True, F.OUT_F32, fx, fw, fb, F.fmt(8, 0, 0))
+        F.fxpq_conv_fwd(d32, xq, wq, bq, y32)
+        (fy,) = search([(y32, 8, 0, 15)])
+        d = F.conv_desc(N, H, H, C, C, K, R, R, 1, 1, True, F.OUT_CODES, fx, fw, fb, fy)
+        F.fxpq_conv_fwd(d, xq, wq, bq, y)
+        state["d"] = d
+
+    def timeit(fn):
+        ts = []
+        for i in range(args.warmup + args.steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            e1.synchronize()
+            if i >= args.warmup:
+                ts.append(e0.elapsed_time(e1))
+        return sum(ts) / len(ts)
+
+    ms_step = timeit(step)
+    d = state["d"]
+    ms_conv = timeit(lambda: F.fxpq_conv_fwd(d, xq, wq, bq, y))
+    hbm, bf16, _, src = measured_peaks()
+    t1 = timed_oracle("config1", 1)
+    tn = timed_oracle("config1", os.cpu_count() or 1)
+    return {"config1": {
+        "workload": "3x3 conv, batch 8, 64->64 channels, 32x32 maps, 8-bit w/a (FL 0..15), 16-bit bias, 8-bit output",
+        "step_ms": round(ms_step, 4), "conv_us": round(ms_conv * 1e3, 2),
+        "conv_tops": round(flops / (ms_conv / 1e3) / 1e12, 2), "conv_frac_peak": round(flops / (ms_conv / 1e3) / 1e12 / bf16, 4),
+        "peak_tflops": bf16, "peak_source": src,
+        "oracle_step_s_1_thread": round(t1, 3), "oracle_step_s_all_cores": round(tn, 3), "host_cores": os.cpu_count()}}
+
+
+def bench_config2(args, F):
+    """The FL-search sweep workload: per size (1M, 16M, 64M) and distribution (N(0,1), Laplace(0, 0.1),
+    ReLU(N(0,1))) the single-wordlength search (k = 8, FL -8..23), the full 15 x 32 grid (k 2..16) and the
+    quantization to int8 codes; the oracle on 1M (row and grid) and 16M (row) values."""
+    import torch
+    hbm, _, _, src = measured_peaks()
+    rows = []
+    for n in (1 << 20, 1 << 24, 1 << 26):
+        for dist in ("normal", "laplace", "relu_normal"):
+            x = torch.from_numpy(synth.sweep_tensor(dist, n, 2)).cuda()
+            y = torch.empty(n, dtype=torch.int8, device="cuda")
+            r = {"n": n, "dist": dist}
+            for name, fn in (("row_k8", lambda: F.fl_search(x, -1, 8, 8, -8, 23)),
+                             ("grid_k2_16", lambda: F.fl_search(x, -1, 2, 16, -8, 23)),
+                             ("quantize_i8", lambda: F.fxpq_quantize(x, F.fmt(8, 1, 5), F.DT_I8, y))):
+                ts = []
+                for i in range(args.warmup + args.steps):
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                    fn()
+                    e1.record()
+                    e1.synchronize()
+                    if i >= args.warmup:
+                        ts.append(e0.elapsed_time(e1))
+                ms = sum(ts) / len(ts)
+                nbytes = (5 if name == "quantize_i8" else 4) * n
+                r[name] = {"ms": round(ms, 4), "gelem_s": round(n / (ms / 1e3) / 1e9, 1),
+                           "gbs": round(nbytes / (ms / 1e3) / 1e9, 1), "frac_hbm": round(nbytes / (ms / 1e3) / 1e9 / hbm, 3)}
+            rows.append(r)
+    cores = os.cpu_count() or 1
+    orc = {"row_1M_s_1_thread": round(timed_oracle(f"config2:{1 << 20}:row", 1), 3),
+           "row_1M_s_all_cores": round(timed_oracle(f"config2:{1 << 20}:row", cores), 3),
+           "grid_1M_s_all_cores": round(timed_oracle(f"config2:{1 << 20}:sweep", cores), 3),
+           "row_16M_s_all_cores": round(timed_oracle(f"config2:{1 << 24}:row", cores), 3), "host_cores": cores}
+    return {"config2": {"rows": rows, "hbm_gbs": hbm, "peak_source": src, "oracle": orc}}
 
 
 # ----------------------------------------------------------------------------- CPU oracle arm
@@ -472,6 +667,10 @@ def run_kernel(args):
         peak = 152 * 128 * 2 * 2.07e9 / 1e12  # fp32 FMA lanes x 2 FLOP x max SM clock
         out["conv_f32"] = {"ms": round(ms, 4), "tflops": round(tf, 2), "peak_fp32_tflops": round(peak, 1),
                            "frac": round(tf / peak, 3)}
+    if args.kernel in ("config1", "all"):
+        out.update(bench_config1(args, F))
+    if args.kernel in ("config2", "all"):
+        out.update(bench_config2(args, F))
     if args.kernel in ("forward", "all"):
         # the integer forward of the bench workload alone (one plan, calibrated once): the target of the
         # per-launch DRAM traffic capture of the conv kernels
@@ -502,8 +701,9 @@ def run_kernel(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "fopt", "forward", "all"],
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "fopt", "forward", "config1", "config2", "all"],
                     help="time one kernel case and exit")
+    ap.add_argument("--oracle-job", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
@@ -511,7 +711,9 @@ def main():
     ap.add_argument("--workload", default="vgg16", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle cpu_baseline leg")
     args = ap.parse_args()
-    if args.kernel:
+    if args.oracle_job:
+        oracle_job(args.oracle_job)
+    elif args.kernel:
         run_kernel(args)
     elif args.impl == "reference":
         run_reference(args)
