@@ -424,12 +424,46 @@ FXPQ_API fxpq_status fxpq_dequantize(const void* d_codes, int64_t npix, int32_t 
  * layer whose weights are already fixed point (the contraction ran in FXPQ_OUT_F32 mode). */
 FXPQ_API fxpq_status fxpq_bias_relu_f32(float* d_y, int64_t npix, int32_t K, const float* d_bias, int32_t relu,
                                         void* stream);
-/* Statistics of one data-structure of n_samples x nu fp32 values, the terms of Eq. CPB_QE: d_out
- * (device double[3 + 2 n_samples]) = { L = sum (x - Q(x; fmt))^2 (Eq. DSB_QE, fp64 sums), min, max,
- * then per sample sum x, sum x^2 } (the dispersion of Eq. importance follows on the host).  d_ws:
- * 8 bytes of device scratch.  n_samples <= 65535. */
-FXPQ_API fxpq_status fxpq_ds_stats(const float* d_x, int32_t n_samples, int64_t nu, fxpq_fmt fmt, double* d_out,
-                                   void* d_ws, void* stream);
+/* Statistics of data-structures, the terms of Eq. CPB_QE (Sec. IV-C), many in one set of launches.
+ * Item i: n_samples x nu fp32 values (sample-major) and the QPs under which its error is taken; its
+ * record d_out (device double[3 + 2 n_samples]) receives
+ *   { L = sum (x - Q(x; fmt))^2 (Eq. DSB_QE, fp64), min, max,
+ *     then per sample its mean and its sum of squared deviations from that mean }
+ * so that the population deviation of Eq. importance is sqrt(M2 / nu), free of the cancellation
+ * of the one-pass form.  Each sum is formed in a fixed order (deterministic, no floating-point
+ * atomics).  Items <= 4096, n_samples <= 65535, nu >= 1.  Workspace:
+ * fxpq_ds_stats_batch_workspace(items) bytes, 256-byte aligned, scratch. */
+typedef struct {
+    const float* d_x;   /* device fp32 values, n_samples x nu                                    */
+    double* d_out;      /* device record, double[3 + 2 n_samples]                                 */
+    int64_t nu;         /* values per sample                                                     */
+    int32_t n_samples;  /* samples (1 for a parameter tensor)                                    */
+    fxpq_fmt fmt;       /* the QPs of the error L (k = 1..32; k = 1, S = 1 the binary quantizer)  */
+} fxpq_ds_item;
+FXPQ_API size_t fxpq_ds_stats_batch_workspace(const fxpq_ds_item* h_items, int32_t n_items);
+FXPQ_API fxpq_status fxpq_ds_stats_batch(const fxpq_ds_item* h_items, int32_t n_items, void* d_ws, size_t ws_bytes,
+                                         void* stream);
+
+/* The cost F = E + UnClass + MisPred of Alg. 1 (Eq. quantization_parameters_optimization) for
+ * n_cand candidates at once, on the device.  Term t of candidate c is the fxpq_ds_stats_batch record
+ * at d_stats + c * cand_stride + h_terms[t].offset; terms of one layer (equal .layer) share the
+ * normaliser of Eq. importance:
+ *   sigma_t = mean over samples of sqrt(M2_s / nu), pi_t = sigma_t nu_t / sum over the layer of sigma nu,
+ *   E = sum_t pi_t L_t / R_t  (Eq. CPB_QE; R = max - min, Eq. data_range; a term with R = 0 or a
+ *       layer with sum sigma nu = 0 adds nothing).
+ * d_ties: per candidate N counts |C_i| (fxpq_top1_ties), candidate c at d_ties + c * N:
+ *   UnClass = #{i : |C_i| > 1} / N, MisPred = sum (|C_i| - 1) / (N n_classes)
+ * (Eqs. unclassified_samples, mispredicted_classes).  d_cost: device double[n_cand][4] =
+ * { F, E, UnClass, MisPred }.  n_terms <= 512. */
+typedef struct {
+    int64_t offset;     /* the term's record, in doubles from the candidate's base               */
+    int64_t nu;         /* values per sample                                                     */
+    int32_t n_samples;
+    int32_t layer;      /* terms with equal layer share the importance normaliser                 */
+} fxpq_cost_term;
+FXPQ_API fxpq_status fxpq_fopt_cost(const double* d_stats, int64_t cand_stride, const fxpq_cost_term* h_terms,
+                                    int32_t n_terms, const int32_t* d_ties, int32_t N, int32_t n_classes,
+                                    int32_t n_cand, double* d_cost, void* stream);
 /* |C_i| of Eqs. unclassified_samples / mispredicted_classes: per sample the number of classes whose
  * logit equals the largest.  Logits [N, C]: fp32, or exact int64 C-Block values when is_int64. */
 FXPQ_API fxpq_status fxpq_top1_ties(const void* d_logits, int32_t is_int64, int32_t N, int32_t C,

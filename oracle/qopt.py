@@ -284,22 +284,24 @@ class Net:
 
 
 def qparams_opt(cost_fn, init: int, K: int = 1):
-    """Alg. 1 around the initial FL `init` with cost_fn(FL) -> F: returns (best FL, best cost, trace
-    [(FL, cost)] in evaluation order)."""
-    best_fl, cost_best = init, cost_fn(init)
-    trace = [(init, cost_best)]
-    for i in (-1, +1):
-        k, j = 1, 0
-        while k <= K + j:
-            fl = init + i * k
-            if fl < FL_MIN or fl > FL_MAX:
-                break
+    """Alg. 1 around the initial FL `init` with cost_fn(FL) -> F (Sec. IV-C): the FL moves away from init in
+    each direction at a fixed wordlength; a candidate is accepted only when its cost is strictly below the
+    best so far, and each acceptance lets its direction go one step beyond the K steps it always takes;
+    FLs outside [FL_MIN, FL_MAX] end a direction.  Returns (best FL, best cost, [(FL, cost)] in the order
+    visited)."""
+    best_fl, best = init, cost_fn(init)
+    trace = [(init, best)]
+    for d in (-1, 1):
+        steps, k = K, 1
+        while k <= steps and FL_MIN <= init + d * k <= FL_MAX:
+            fl = init + d * k
             c = cost_fn(fl)
             trace.append((fl, c))
-            if c < cost_best:
-                cost_best, best_fl, j = c, fl, j + 1
+            if c < best:
+                best, best_fl = c, fl
+                steps += 1
             k += 1
-    return best_fl, cost_best, trace
+    return best_fl, best, trace
 
 
 def forward_optimize(net: Net, K: int = 1, upto=None):

@@ -52,6 +52,14 @@ class OpDesc(ctypes.Structure):
                 ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
 
 
+class DsItem(ctypes.Structure):
+    _fields_ = [("d_x", VP), ("d_out", VP), ("nu", I64), ("n_samples", I32), ("fmt", Fmt)]
+
+
+class CostTerm(ctypes.Structure):
+    _fields_ = [("offset", I64), ("nu", I64), ("n_samples", I32), ("layer", I32)]
+
+
 class ConvF32Desc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32)]
@@ -93,7 +101,9 @@ _SIGS = {
     "fxpq_avgpool_f32": (I32, [VP, I32, I32, I32, I32, VP, VP]),
     "fxpq_dequantize": (I32, [VP, I64, I32, I32, Fmt, VP, VP]),
     "fxpq_bias_relu_f32": (I32, [VP, I64, I32, VP, I32, VP]),
-    "fxpq_ds_stats": (I32, [VP, I32, I64, Fmt, VP, VP, VP]),
+    "fxpq_ds_stats_batch_workspace": (SZ, [VP, I32]),
+    "fxpq_ds_stats_batch": (I32, [VP, I32, VP, SZ, VP]),
+    "fxpq_fopt_cost": (I32, [VP, I64, VP, I32, VP, I32, I32, I32, VP, VP]),
     "fxpq_top1_ties": (I32, [VP, I32, I32, I32, VP, VP]),
     "fxpq_nchw_to_nhwc_f32": (I32, [VP, I32, I32, I32, I32, VP, VP]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),

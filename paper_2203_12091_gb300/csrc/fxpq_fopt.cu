@@ -283,64 +283,208 @@ __device__ __forceinline__ unsigned ord_key(float x) {
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Statistics of one data-structure of n_samples x nu fp32 values under format (k, S, fl):
-// out[0] += sum (x - Q(x))^2, out[3 + 2 s] += sum x and out[4 + 2 s] += sum x^2 of sample s; the
-// smallest and largest values as order keys in keys[0], keys[1] (ds_stats_finish_kernel converts
-// them into out[1], out[2]).  Blocks never straddle samples: grid.y = sample.
-__global__ void ds_stats_kernel(const float* __restrict__ x, long long nu, int k, int S, int fl, double* out,
-                                unsigned* keys) {
-    const int s = blockIdx.y;
-    const float* xs = x + (long long)s * nu;
-    const double scale = ldexp(1.0, fl), inv = ldexp(1.0, -fl);
-    const double lo = S ? -ldexp(1.0, k - 1) : 0.0, hi = ldexp(1.0, k - S) - 1.0;
-    const bool binary = k == 1 && S == 1;
-    double l2 = 0.0, s1 = 0.0, s2 = 0.0;
+// ---------------------------------------------------------------- data-structure statistics (batched)
+// Items of fxpq_ds_stats_batch, split into work units of DS_CHUNK values of one sample each; the unit
+// prefix of each item sits in the kernel parameters.  Three passes: per-unit sums; per-unit sums of
+// squared deviations from the sample mean (the mean from the first pass's sums, in unit order), the
+// quantization error and the extremes; per-item records from the units in order.  No floating-point
+// atomics: every total is formed in a fixed order.
+constexpr int DS_MAX_ITEMS = 128;  // items per launch group
+constexpr long long DS_CHUNK = 1 << 16;
+constexpr int DS_T = 256;
+
+struct DsItemDev {
+    const float* x;
+    double* out;
+    long long nu;
+    int n_samples, k, S, fl;
+    int chunks;  // units per sample
+    int unit0;   // first unit of the item (within its launch group)
+};
+struct DsBatchDev {
+    int n;
+    DsItemDev it[DS_MAX_ITEMS];
+    int unit_end;  // units of the launch group
+};
+
+// Per-unit scratch of one launch group.
+struct DsUnit {
+    double sum, m2, l2;
+    unsigned mn, mx;
+};
+
+__device__ __forceinline__ int ds_item_of(const DsBatchDev& B, int u) {
+    int lo = 0, hi = B.n - 1;  // last item whose unit0 <= u
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (B.it[mid].unit0 <= u) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ double ds_block_sum(double v, double* red) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, off);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    double t = 0.0;
+    if (threadIdx.x == 0)
+        for (int i = 0; i < DS_T / 32; ++i) t += red[i];  // fixed order
+    return t;  // valid in thread 0
+}
+
+__global__ void __launch_bounds__(DS_T) ds_sum_kernel(const __grid_constant__ DsBatchDev B, DsUnit* units) {
+    __shared__ double red[DS_T / 32];
+    const int u = blockIdx.x;
+    const DsItemDev& it = B.it[ds_item_of(B, u)];
+    const int rel = u - it.unit0, s = rel / it.chunks, c = rel % it.chunks;
+    const float* xs = it.x + (long long)s * it.nu;
+    const long long i0 = (long long)c * DS_CHUNK, i1 = min(i0 + DS_CHUNK, it.nu);
+    double acc = 0.0;
+    for (long long i = i0 + threadIdx.x; i < i1; i += DS_T) acc += (double)xs[i];
+    const double t = ds_block_sum(acc, red);
+    if (threadIdx.x == 0) units[u].sum = t;
+}
+
+__global__ void __launch_bounds__(DS_T) ds_dev_kernel(const __grid_constant__ DsBatchDev B, DsUnit* units) {
+    __shared__ double red[DS_T / 32];
+    __shared__ unsigned kmn, kmx;
+    const int u = blockIdx.x;
+    const DsItemDev& it = B.it[ds_item_of(B, u)];
+    const int rel = u - it.unit0, s = rel / it.chunks, c = rel % it.chunks;
+    const float* xs = it.x + (long long)s * it.nu;
+    const long long i0 = (long long)c * DS_CHUNK, i1 = min(i0 + DS_CHUNK, it.nu);
+    // the sample mean from the first pass's unit sums, in unit order
+    const int first = it.unit0 + s * it.chunks;
+    double sum = 0.0;
+    for (int v = 0; v < it.chunks; ++v) sum += units[first + v].sum;
+    const double mean = sum / (double)it.nu;
+    const double scale = ldexp(1.0, it.fl), inv = ldexp(1.0, -it.fl);
+    const double lo = it.S ? -ldexp(1.0, it.k - 1) : 0.0, hi = ldexp(1.0, it.k - it.S) - 1.0;
+    const bool binary = it.k == 1 && it.S == 1;
+    double m2 = 0.0, l2 = 0.0;
     unsigned mn = 0xFFFFFFFFu, mx = 0u;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nu; i += (long long)gridDim.x * blockDim.x) {
+    for (long long i = i0 + threadIdx.x; i < i1; i += DS_T) {
         const float v = xs[i];
         const double d = (double)v;
-        double q;
-        if (binary) {
-            q = v < 0.0f ? -inv : inv;
-        } else {
-            q = fmin(fmax(nearbyint(d * scale), lo), hi) * inv;  // round half to even, clip
-        }
-        const double e = d - q;
+        const double q = binary ? (v < 0.0f ? -inv : inv) : fmin(fmax(nearbyint(d * scale), lo), hi) * inv;
+        const double e = d - q, dv = d - mean;
         l2 += e * e;
-        s1 += d;
-        s2 += d * d;
+        m2 += dv * dv;
         const unsigned key = ord_key(v);
         mn = min(mn, key);
         mx = max(mx, key);
     }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        l2 += __shfl_xor_sync(0xFFFFFFFFu, l2, off);
-        s1 += __shfl_xor_sync(0xFFFFFFFFu, s1, off);
-        s2 += __shfl_xor_sync(0xFFFFFFFFu, s2, off);
-        mn = min(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, off));
-        mx = max(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, off));
+    if (threadIdx.x == 0) {
+        kmn = 0xFFFFFFFFu;
+        kmx = 0u;
     }
+    const double tm2 = ds_block_sum(m2, red);
+    const double tl2 = ds_block_sum(l2, red);
+    mn = __reduce_min_sync(0xFFFFFFFFu, mn);
+    mx = __reduce_max_sync(0xFFFFFFFFu, mx);
     if ((threadIdx.x & 31) == 0) {
-        atomicAdd(out, l2);
-        atomicAdd(out + 3 + 2 * s, s1);
-        atomicAdd(out + 4 + 2 * s, s2);
-        atomicMin(keys, mn);
-        atomicMax(keys + 1, mx);
+        atomicMin(&kmn, mn);
+        atomicMax(&kmx, mx);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        units[u].m2 = tm2;
+        units[u].l2 = tl2;
+        units[u].mn = kmn;
+        units[u].mx = kmx;
     }
 }
 
-__global__ void ds_stats_init_kernel(unsigned* keys) {
-    keys[0] = 0xFFFFFFFFu;
-    keys[1] = 0u;
+__device__ __forceinline__ float ds_key_value(unsigned k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
-__global__ void ds_stats_finish_kernel(double* out, const unsigned* keys) {
-    const unsigned kmn = keys[0], kmx = keys[1];
-    const unsigned umn = (kmn & 0x80000000u) ? (kmn & 0x7FFFFFFFu) : ~kmn;
-    const unsigned umx = (kmx & 0x80000000u) ? (kmx & 0x7FFFFFFFu) : ~kmx;
-    out[1] = (double)__uint_as_float(umn);
-    out[2] = (double)__uint_as_float(umx);
+// One thread per item: its record from its units, in unit order.
+__global__ void ds_finish_kernel(const __grid_constant__ DsBatchDev B, const DsUnit* units) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= B.n) return;
+    const DsItemDev& it = B.it[i];
+    double l2 = 0.0;
+    unsigned mn = 0xFFFFFFFFu, mx = 0u;
+    for (int s = 0; s < it.n_samples; ++s) {
+        double sum = 0.0, m2 = 0.0;
+        for (int c = 0; c < it.chunks; ++c) {
+            const DsUnit& q = units[it.unit0 + s * it.chunks + c];
+            sum += q.sum;
+            m2 += q.m2;
+            l2 += q.l2;
+            mn = min(mn, q.mn);
+            mx = max(mx, q.mx);
+        }
+        it.out[3 + 2 * s] = sum / (double)it.nu;
+        it.out[4 + 2 * s] = m2;
+    }
+    it.out[0] = l2;
+    it.out[1] = (double)ds_key_value(mn);
+    it.out[2] = (double)ds_key_value(mx);
+}
+
+// ---------------------------------------------------------------- the cost F of Alg. 1
+constexpr int COST_MAX_TERMS = 512;
+struct CostTermDev {
+    long long offset, nu;
+    int n_samples, layer;
+};
+struct CostTerms {
+    int n;
+    CostTermDev t[COST_MAX_TERMS];
+};
+
+// One block per candidate; thread 0 adds the terms in order (a few dozen per network).
+__global__ void fopt_cost_kernel(const double* __restrict__ stats, long long cand_stride,
+                                 const __grid_constant__ CostTerms T, const int* __restrict__ ties, int N,
+                                 int n_classes, double* __restrict__ cost) {
+    const int c = blockIdx.x;
+    const double* base = stats + (long long)c * cand_stride;
+    __shared__ unsigned n_tied, extra;
+    if (threadIdx.x == 0) n_tied = extra = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        const int k = ties[(long long)c * N + i];
+        if (k > 1) atomicAdd(&n_tied, 1u);
+        atomicAdd(&extra, (unsigned)(k - 1));
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    double E = 0.0;
+    int t0 = 0;
+    while (t0 < T.n) {
+        int t1 = t0;
+        double den = 0.0;
+        while (t1 < T.n && T.t[t1].layer == T.t[t0].layer) {  // one layer: sum of sigma nu
+            const CostTermDev& q = T.t[t1];
+            const double* r = base + q.offset;
+            double sig = 0.0;
+            for (int s = 0; s < q.n_samples; ++s) sig += sqrt(r[4 + 2 * s] / (double)q.nu);
+            den += sig / q.n_samples * (double)q.nu;
+            ++t1;
+        }
+        if (den > 0.0) {
+            for (int t = t0; t < t1; ++t) {
+                const CostTermDev& q = T.t[t];
+                const double* r = base + q.offset;
+                const double R = r[2] - r[1];
+                if (R == 0.0) continue;
+                double sig = 0.0;
+                for (int s = 0; s < q.n_samples; ++s) sig += sqrt(r[4 + 2 * s] / (double)q.nu);
+                E += (sig / q.n_samples * (double)q.nu / den) * r[0] / R;
+            }
+        }
+        t0 = t1;
+    }
+    const double uc = (double)n_tied / N, mp = (double)extra / ((double)N * n_classes);
+    cost[4 * c + 0] = E + uc + mp;
+    cost[4 * c + 1] = E;
+    cost[4 * c + 2] = uc;
+    cost[4 * c + 3] = mp;
 }
 
 // one warp per sample: the number of classes whose logit equals the sample's largest
@@ -457,25 +601,87 @@ extern "C" fxpq_status fxpq_bias_relu_f32(float* d_y, int64_t npix, int32_t K, c
     return after_launch("bias_relu_f32");
 }
 
-extern "C" fxpq_status fxpq_ds_stats(const float* d_x, int32_t n_samples, int64_t nu, fxpq_fmt fmt, double* d_out,
-                                     void* d_ws, void* stream) {
-    if (n_samples < 1 || n_samples > 65535 || nu < 1 || !fmt_ok1(fmt, 32) || !d_x || !d_out || !d_ws)
-        return FXPQ_ERR_INVALID_ARG;
+namespace {
+// Units of one item (DS_CHUNK values of one sample each), or -1 for an invalid item.
+long long ds_units(const fxpq_ds_item& it) {
+    if (it.n_samples < 1 || it.n_samples > 65535 || it.nu < 1 || !fxpq::fmt_ok1(it.fmt, 32) || !it.d_x || !it.d_out)
+        return -1;
+    return (long long)it.n_samples * ((it.nu + DS_CHUNK - 1) / DS_CHUNK);
+}
+}  // namespace
+
+extern "C" size_t fxpq_ds_stats_batch_workspace(const fxpq_ds_item* h_items, int32_t n_items) {
+    if (n_items < 1 || n_items > 4096 || !h_items) return 0;
+    long long most = 0;  // the largest launch group's units
+    for (int i0 = 0; i0 < n_items; i0 += DS_MAX_ITEMS) {
+        long long u = 0;
+        for (int i = i0; i < n_items && i < i0 + DS_MAX_ITEMS; ++i) {
+            const long long v = ds_units(h_items[i]);
+            if (v < 0) return 0;
+            u += v;
+        }
+        most = u > most ? u : most;
+    }
+    return ((size_t)most * sizeof(DsUnit) + 255) / 256 * 256;
+}
+
+extern "C" fxpq_status fxpq_ds_stats_batch(const fxpq_ds_item* h_items, int32_t n_items, void* d_ws, size_t ws_bytes,
+                                           void* stream) {
+    if (n_items < 1 || n_items > 4096 || !h_items) return FXPQ_ERR_INVALID_ARG;
+    for (int i = 0; i < n_items; ++i)
+        if (ds_units(h_items[i]) < 0) return FXPQ_ERR_INVALID_ARG;
+    const size_t need = fxpq_ds_stats_batch_workspace(h_items, n_items);
+    if (!d_ws || ws_bytes < need || !aligned(d_ws, 256)) return FXPQ_ERR_WORKSPACE;
     cudaStream_t s = as_stream(stream);
-    if (cudaMemsetAsync(d_out, 0, sizeof(double) * (3 + 2 * (size_t)n_samples), s) != cudaSuccess) return FXPQ_ERR_CUDA;
-    ds_stats_init_kernel<<<1, 1, 0, s>>>(static_cast<unsigned*>(d_ws));
-    fxpq_status st = after_launch("ds_stats_init");
-    if (st != FXPQ_OK) return st;
-    long long bx = (nu + 255) / 256;
-    const long long cap = (152LL * 8 + n_samples - 1) / n_samples;
-    if (bx > cap) bx = cap;
-    if (bx < 1) bx = 1;
-    ds_stats_kernel<<<dim3((unsigned)bx, (unsigned)n_samples), 256, 0, s>>>(d_x, nu, fmt.bits, fmt.is_signed, fmt.fl,
-                                                                          d_out, static_cast<unsigned*>(d_ws));
-    st = after_launch("ds_stats");
-    if (st != FXPQ_OK) return st;
-    ds_stats_finish_kernel<<<1, 1, 0, s>>>(d_out, static_cast<const unsigned*>(d_ws));
-    return after_launch("ds_stats_finish");
+    DsUnit* units = static_cast<DsUnit*>(d_ws);
+    for (int i0 = 0; i0 < n_items; i0 += DS_MAX_ITEMS) {
+        DsBatchDev B;
+        B.n = 0;
+        long long u = 0;
+        for (int i = i0; i < n_items && i < i0 + DS_MAX_ITEMS; ++i) {
+            const fxpq_ds_item& h = h_items[i];
+            DsItemDev& d = B.it[B.n++];
+            d.x = h.d_x;
+            d.out = h.d_out;
+            d.nu = h.nu;
+            d.n_samples = h.n_samples;
+            d.k = h.fmt.bits;
+            d.S = h.fmt.is_signed;
+            d.fl = h.fmt.fl;
+            d.chunks = (int)((h.nu + DS_CHUNK - 1) / DS_CHUNK);
+            d.unit0 = (int)u;
+            u += ds_units(h);
+        }
+        if (u > 0x7FFFFFFFLL) return FXPQ_ERR_INVALID_ARG;
+        B.unit_end = (int)u;
+        ds_sum_kernel<<<(unsigned)u, DS_T, 0, s>>>(B, units);
+        fxpq_status st = after_launch("ds_sum");
+        if (st != FXPQ_OK) return st;
+        ds_dev_kernel<<<(unsigned)u, DS_T, 0, s>>>(B, units);
+        st = after_launch("ds_dev");
+        if (st != FXPQ_OK) return st;
+        ds_finish_kernel<<<(B.n + 127) / 128, 128, 0, s>>>(B, units);
+        st = after_launch("ds_finish");
+        if (st != FXPQ_OK) return st;
+    }
+    return FXPQ_OK;
+}
+
+extern "C" fxpq_status fxpq_fopt_cost(const double* d_stats, int64_t cand_stride, const fxpq_cost_term* h_terms,
+                                      int32_t n_terms, const int32_t* d_ties, int32_t N, int32_t n_classes,
+                                      int32_t n_cand, double* d_cost, void* stream) {
+    if (n_terms < 0 || n_terms > COST_MAX_TERMS || (n_terms > 0 && !h_terms) || N < 1 || n_classes < 1 || n_cand < 1 ||
+        cand_stride < 0 || !d_stats || !d_ties || !d_cost)
+        return FXPQ_ERR_INVALID_ARG;
+    CostTerms T;
+    T.n = n_terms;
+    for (int i = 0; i < n_terms; ++i) {
+        const fxpq_cost_term& h = h_terms[i];
+        if (h.offset < 0 || h.nu < 1 || h.n_samples < 1) return FXPQ_ERR_INVALID_ARG;
+        T.t[i] = CostTermDev{h.offset, h.nu, h.n_samples, h.layer};
+    }
+    fopt_cost_kernel<<<n_cand, 128, 0, as_stream(stream)>>>(d_stats, cand_stride, T, d_ties, N, n_classes, d_cost);
+    return after_launch("fopt_cost");
 }
 
 extern "C" fxpq_status fxpq_top1_ties(const void* d_logits, int32_t is_int64, int32_t N, int32_t C, int32_t* d_counts,

@@ -7,15 +7,15 @@ point at its chosen QPs, d takes the candidate, and every later one is FP32: the
 integer C-Blocks (fxpq_conv_fwd, fxpq_eltwise, fxpq_avgpool, fxpq_maxpool) up to the point where FP32
 takes over (fxpq_dequantize), then the FP32 layers (fxpq_conv_f32, ...).  E sums, over the
 data-structures of layers l, l+1, ..., the importance pi (Eq. importance) times the quantization
-error L (Eq. DSB_QE) over the range R (Eq. data_range), each from fxpq_ds_stats on the data-structure's
-FP32 values in that forward; UnClass and MisPred count top-1 ties of the logits (fxpq_top1_ties).
-The initial QPs come from the preprocessor (Eq. initial_quantization_parameters, fxpq_fl_init) on the
-ranges of the FP32 network.  Every arithmetic step runs in libfxpq.so; this module sequences the calls
-and combines a handful of per-data-structure scalars on the host.
+error L (Eq. DSB_QE) over the range R (Eq. data_range), from the statistics of the data-structure's
+FP32 values in that forward (fxpq_ds_stats_batch); UnClass and MisPred count top-1 ties of the logits
+(fxpq_top1_ties); fxpq_fopt_cost forms F on the device.  The candidates of one data-structure share
+their forward: the layers before its layer run once, its layer once per candidate, every later layer
+once over the candidates stacked along the batch.  The initial QPs come from the preprocessor (Eq.
+initial_quantization_parameters, fxpq_fl_init) on the ranges of the FP32 network.  Every arithmetic
+step runs in libfxpq.so; this module sequences the calls and reads back one cost per candidate.
 """
 from __future__ import annotations
-
-import math
 
 import torch
 
@@ -68,11 +68,13 @@ class ForwardOptimizer:
         F.fxpq_nchw_to_nhwc_f32(self.x0, self.N, self.cin, self.hw, self.hw, self.x0_nhwc, stream)
         self.order = data_structures(layers)
         self.names = ["input"] + [L_["name"] for L_ in layers]
-        self._stats_out = torch.empty(3 + 2 * max(self.N, 1), dtype=torch.float64, device=self.dev)
-        self._stats_ws = torch.empty(2, dtype=torch.int32, device=self.dev)
         self._recip = {}
         self.fmt = {}
+        # initial QPs (preprocessor) from the ranges of the FP32 network: one statistics batch, one read-back
         acts = self._fp32_forward()
+        items, ks, off = [], [], 0
+        rec = torch.empty(sum(3 + 2 * (self.N if j == "a" else 1) for _, j in self.order), dtype=torch.float64,
+                          device=self.dev)
         for nm, j in self.order:
             if j == "a":
                 x = acts[nm].t
@@ -82,15 +84,14 @@ class ForwardOptimizer:
                 x = self.W[nm][0] if j == "w" else self.W[nm][1]
                 k = plan[nm][j]
                 n_s, nu = 1, x.numel()
-            st = self._stats(x.reshape(-1), n_s, nu, F.fmt(k, 1, 0))
-            stats = L.Stats(st["min"], st["max"], 0, 0, 0.0, 0.0, x.numel())
+            items.append((x.reshape(-1), n_s, nu, F.fmt(k, 1, 0), rec[off:off + 3 + 2 * n_s]))
+            ks.append((off, k, x.numel()))
+            off += 3 + 2 * n_s
+        F.fxpq_ds_stats_batch(items, stream)
+        h = rec.cpu().tolist()
+        for (nm, j), (o, k, n) in zip(self.order, ks):
+            stats = L.Stats(h[o + 1], h[o + 2], 0, 0, 0.0, 0.0, n)
             self.fmt[(nm, j)] = F.fxpq_fl_init(stats, k, STRATEGY[strategy])
-
-    # ------------------------------------------------------------------ device statistics
-    def _stats(self, x, n_samples, nu, fmt):
-        out = self._stats_out[: 3 + 2 * n_samples]
-        F.fxpq_ds_stats(x, n_samples, nu, fmt, out, self._stats_ws, self.stream)
-        return _decode(out.cpu().tolist(), 0, n_samples, nu)
 
     # ------------------------------------------------------------------ helpers
     def _src(self, i, L_):
@@ -100,12 +101,23 @@ class ForwardOptimizer:
     def _empty(self, n, dtype=torch.float32):
         return torch.empty(max(n, 1), dtype=dtype, device=self.dev)
 
-    def _to_f(self, v):
+    def _to_f(self, v, nb=None):
         if isinstance(v, _F):
             return v
-        y = self._empty(self.N * v.H * v.W * v.C)
-        F.fxpq_dequantize(v.t, self.N * v.H * v.W, v.Cp, v.C, v.fmt, y, self.stream)
+        nb = self.N if nb is None else nb
+        y = self._empty(nb * v.H * v.W * v.C)
+        F.fxpq_dequantize(v.t, nb * v.H * v.W, v.Cp, v.C, v.fmt, y, self.stream)
         return _F(y, v.H, v.W, v.C)
+
+    def _stack(self, entries):
+        """One FP32 entry holding the given entries (each over the N calibration samples) one after the other
+        along the batch: candidate c's samples are rows c N .. (c + 1) N - 1."""
+        fs = [self._to_f(e) for e in entries]
+        n = fs[0].t.numel()
+        y = self._empty(n * len(fs))
+        for c, f in enumerate(fs):
+            y[c * n:(c + 1) * n].copy_(f.t[:n])  # device-to-device copies
+        return _F(y, fs[0].H, fs[0].W, fs[0].C)
 
     def _recip_of(self, nm, hw):
         if nm not in self._recip:
@@ -131,95 +143,138 @@ class ForwardOptimizer:
     def _fp32_forward(self):
         env = {"input": _F(self.x0_nhwc, self.hw, self.hw, self.cin)}
         for i, L_ in enumerate(self.layers):
-            env[L_["name"]] = self._f_layer(i, L_, env, None)
+            env[L_["name"]] = self._f_layer(i, L_, env)
         return env
 
-    def _f_layer(self, i, L_, env, wq_override):
-        """One layer in FP32 on FP32 inputs (dequantized where needed)."""
+    def _f_layer(self, i, L_, env, nb=None):
+        """One layer in FP32 on FP32 inputs (dequantized where needed), over nb samples (N by default)."""
         nm, typ = L_["name"], L_["type"]
+        N = self.N if nb is None else nb
         if typ == "conv":
-            x = self._to_f(env[self._src(i, L_)])
+            x = self._to_f(env[self._src(i, L_)], N)
             w, b = self.W[nm]
             K, R = L_["K"], L_["R"]
             P = (x.H + 2 * L_["pad"] - R) // L_["stride"] + 1
-            y = self._empty(self.N * P * P * K)
-            F.fxpq_conv_f32(self.N, x.H, x.W, x.C, K, R, R, L_["stride"], L_["pad"], L_["relu"], x.t, w, b, y,
+            y = self._empty(N * P * P * K)
+            F.fxpq_conv_f32(N, x.H, x.W, x.C, K, R, R, L_["stride"], L_["pad"], L_["relu"], x.t, w, b, y,
                             self.stream)
             return _F(y, P, P, K)
         if typ == "maxpool":
-            x = self._to_f(env[self._src(i, L_)])
+            x = self._to_f(env[self._src(i, L_)], N)
             P = (x.H + 2 * L_["pad"] - L_["k"]) // L_["stride"] + 1
-            y = self._empty(self.N * P * P * x.C)
-            F.fxpq_maxpool_f32(x.t, self.N, x.H, x.W, x.C, L_["k"], L_["stride"], L_["pad"], y, self.stream)
+            y = self._empty(N * P * P * x.C)
+            F.fxpq_maxpool_f32(x.t, N, x.H, x.W, x.C, L_["k"], L_["stride"], L_["pad"], y, self.stream)
             return _F(y, P, P, x.C)
         if typ == "eltwise":
-            a, b = self._to_f(env[L_["a"]]), self._to_f(env[L_["b"]])
-            y = self._empty(self.N * a.H * a.W * a.C)
-            F.fxpq_eltwise_f32(a.t, b.t, self.N * a.H * a.W * a.C, L_["relu"], y, self.stream)
+            a, b = self._to_f(env[L_["a"]], N), self._to_f(env[L_["b"]], N)
+            y = self._empty(N * a.H * a.W * a.C)
+            F.fxpq_eltwise_f32(a.t, b.t, N * a.H * a.W * a.C, L_["relu"], y, self.stream)
             return _F(y, a.H, a.W, a.C)
-        x = self._to_f(env[self._src(i, L_)])  # avgpool
-        y = self._empty(self.N * x.C)
-        F.fxpq_avgpool_f32(x.t, self.N, x.H, x.W, x.C, y, self.stream)
+        x = self._to_f(env[self._src(i, L_)], N)  # avgpool
+        y = self._empty(N * x.C)
+        F.fxpq_avgpool_f32(x.t, N, x.H, x.W, x.C, y, self.stream)
         return _F(y, 1, 1, x.C)
 
     # ------------------------------------------------------------------ the mixed forward
-    def forward(self, cur, cand_fl):
-        """Forward of the calibration slice while data-structure cur = (name, j) takes FL cand_fl.
-        Returns (X: data-structure -> (fp32 device values, fmt, n_samples, nu) for the cost, logits)."""
+    def _q_input(self, f):
+        cp = pad8(self.cin)
+        t = self._empty(self.N * self.hw * self.hw * cp * F.planes(f), torch.float16)
+        F.fxpq_quantize_images(self.x0, f, cp, t, self.stream)
+        return _Q(t, f, self.hw, self.hw, self.cin, cp)
+
+    def _fixed_layer(self, i, L_, env):
+        """A layer before the current data-structure's: every data-structure of it is fixed point."""
+        nm = L_["name"]
+        if L_["type"] == "maxpool":
+            src = env[self._src(i, L_)]
+            P = (src.H + 2 * L_["pad"] - L_["k"]) // L_["stride"] + 1
+            y = self._empty(self.N * P * P * src.Cp * F.planes(src.fmt), torch.float16)
+            F.fxpq_maxpool(src.t, self.N, src.H, src.W, src.Cp, src.fmt, L_["k"], L_["stride"], L_["pad"], y,
+                           self.stream)
+            return _Q(y, src.fmt, P, P, src.C, src.Cp)
+        if L_["type"] == "conv":
+            return self._conv_q(i, L_, env, lambda ds: self.fmt[ds], lambda ds: True, False)[0]
+        return self._other_q(i, L_, env, self.fmt[(nm, "a")])[0]
+
+    def _forward_candidates(self, cur, fls):
+        """The calibration slice through the mixed network for each candidate FL of cur (Sec. IV-C: the
+        data-structures optimized before cur fixed point, cur at the candidate, every later one FP32).
+
+        The layers before cur's layer are the same for every candidate and run once; cur's layer runs
+        once per candidate; every later layer runs once over the candidates stacked along the batch.
+        Returns (terms: per candidate {data-structure: (fp32 values, fmt, n_samples, nu)}, stacked
+        logits [n_cand N, classes] (fp32, or exact int64 when cur's layer is the last one))."""
+        N, nc = self.N, len(fls)
         pos = self.order.index(cur)
         fixed = set(self.order[:pos])
+        cl = self.names.index(cur[0]) - 1  # cur's layer; -1: the input QLayer
 
-        def fmt_of(ds):
-            if ds == cur:
-                f = self.fmt[ds]
-                return F.fmt(f.bits, f.is_signed, cand_fl)
-            return self.fmt[ds]
+        def fmt_for(fl):
+            def fmt_of(ds):
+                if ds == cur:
+                    f = self.fmt[ds]
+                    return F.fmt(f.bits, f.is_signed, fl)
+                return self.fmt[ds]
+            return fmt_of
 
         def is_q(ds):
             return ds in fixed or ds == cur
 
-        X = {}
-        if is_q(("input", "a")):
-            f = fmt_of(("input", "a"))
-            cp = pad8(self.cin)
-            t = self._empty(self.N * self.hw * self.hw * cp * F.planes(f), torch.float16)
-            F.fxpq_quantize_images(self.x0, f, cp, t, self.stream)
-            env = {"input": _Q(t, f, self.hw, self.hw, self.cin, cp)}
-        else:
-            env = {"input": _F(self.x0_nhwc, self.hw, self.hw, self.cin)}
-        X[("input", "a")] = (self.x0_nhwc, fmt_of(("input", "a")), self.N, self.hw * self.hw * self.cin)
+        terms = [dict() for _ in range(nc)]
+        env = {}
         logits = None
-        for i, L_ in enumerate(self.layers):
-            nm, typ = L_["name"], L_["type"]
-            last = i == len(self.layers) - 1
-            if typ == "conv":
-                X[(nm, "w")] = (self.W[nm][0], fmt_of((nm, "w")), 1, self.W[nm][0].numel())
-                X[(nm, "b")] = (self.W[nm][1], fmt_of((nm, "b")), 1, self.W[nm][1].numel())
-            qa = (nm, "a") in self.fmt
-            if typ == "maxpool":
-                src = env[self._src(i, L_)]
-                if isinstance(src, _Q):
-                    P = (src.H + 2 * L_["pad"] - L_["k"]) // L_["stride"] + 1
-                    y = self._empty(self.N * P * P * src.Cp * F.planes(src.fmt), torch.float16)
-                    F.fxpq_maxpool(src.t, self.N, src.H, src.W, src.Cp, src.fmt, L_["k"], L_["stride"], L_["pad"], y,
-                                   self.stream)
-                    env[nm] = _Q(y, src.fmt, P, P, src.C, src.Cp)
+        if cl < 0:
+            outs = [self._q_input(fmt_for(fl)(cur)) for fl in fls]
+            for c, fl in enumerate(fls):
+                terms[c][cur] = (self.x0_nhwc, fmt_for(fl)(cur), N, self.hw * self.hw * self.cin)
+            stacked = {"input": self._stack(outs)}
+        else:
+            env["input"] = self._q_input(self.fmt[("input", "a")])
+            for i in range(cl):
+                env[self.layers[i]["name"]] = self._fixed_layer(i, self.layers[i], env)
+            L_ = self.layers[cl]
+            nm = L_["name"]
+            last = cl == len(self.layers) - 1
+            outs, lgs = [], []
+            for c, fl in enumerate(fls):
+                fo = fmt_for(fl)
+                if L_["type"] == "conv":
+                    y, xa, lg = self._conv_q(cl, L_, env, fo, is_q, last)
+                    terms[c][(nm, "w")] = (self.W[nm][0], fo((nm, "w")), 1, self.W[nm][0].numel())
+                    terms[c][(nm, "b")] = (self.W[nm][1], fo((nm, "b")), 1, self.W[nm][1].numel())
                 else:
-                    env[nm] = self._f_layer(i, L_, env, None)
-                continue
-            if typ == "conv" and is_q((nm, "w")):
-                env[nm], xa, lg = self._conv_q(i, L_, env, fmt_of, is_q, last)
-            elif typ in ("eltwise", "avgpool") and qa and is_q((nm, "a")):
-                env[nm], xa = self._other_q(i, L_, env, fmt_of((nm, "a")))
-                lg = None
-            else:
-                y = self._f_layer(i, L_, env, None)
-                env[nm], xa, lg = y, y.t, (y.t if last else None)
+                    y, xa = self._other_q(cl, L_, env, fo((nm, "a")))
+                    lg = None
+                if last:
+                    lgs.append(lg)
+                else:
+                    terms[c][(nm, "a")] = (xa, fo((nm, "a")), N, env_size(y))
+                    outs.append(y)
             if last:
-                logits = lg
-            else:
-                X[(nm, "a")] = (xa, fmt_of((nm, "a")), self.N, env_size(env[nm]))
-        return X, logits
+                n = lgs[0].numel()
+                logits = torch.empty(n * nc, dtype=lgs[0].dtype, device=self.dev)
+                for c, lg in enumerate(lgs):
+                    logits[c * n:(c + 1) * n].copy_(lg.reshape(-1)[:n])
+                return terms, logits
+            stacked = {nm: self._stack(outs)}
+        # every later layer in FP32 over the stacked batch; an entry of the prefix is repeated on first use
+        senv = _Stacked(self, env, nc, stacked)
+        for i in range(cl + 1, len(self.layers)):
+            L_ = self.layers[i]
+            nm = L_["name"]
+            y = self._f_layer(i, L_, senv, N * nc)
+            senv[nm] = y
+            n = N * env_size(y)
+            if L_["type"] == "conv":
+                for c in range(nc):
+                    terms[c][(nm, "w")] = (self.W[nm][0], self.fmt[(nm, "w")], 1, self.W[nm][0].numel())
+                    terms[c][(nm, "b")] = (self.W[nm][1], self.fmt[(nm, "b")], 1, self.W[nm][1].numel())
+            if i == len(self.layers) - 1:
+                logits = y.t
+            elif L_["type"] != "maxpool":
+                for c in range(nc):
+                    terms[c][(nm, "a")] = (y.t[c * n:(c + 1) * n], self.fmt[(nm, "a")], N, env_size(y))
+        return terms, logits
 
     def _conv_q(self, i, L_, env, fmt_of, is_q, last):
         """A conv whose weights are fixed point: (output entry, FP32 values of its C-Block output, logits)."""
@@ -281,63 +336,62 @@ class ForwardOptimizer:
         return _Q(codes, fy, H, H, C, Cp), xf
 
     # ------------------------------------------------------------------ the cost
-    def cost(self, cur, cand_fl):
-        """F = E + UnClass + MisPred for cur at FL cand_fl: (F, E, UnClass, MisPred)."""
-        X, logits = self.forward(cur, cand_fl)
+    def costs(self, cur, fls):
+        """(F, E, UnClass, MisPred) for each candidate FL of data-structure cur (Eq.
+        quantization_parameters_optimization): the candidates' mixed forwards together, the statistics of
+        every term of layers cur's and later (Eq. CPB_QE) in one batch, the tie counts of the logits, and
+        every candidate's cost on the device; one read-back."""
+        terms, logits = self._forward_candidates(cur, fls)
+        nc = len(fls)
         start = self.names.index(cur[0])
-        # every statistic and the tie counts into one device buffer, read back once
-        layers = []
+        layout = []  # (data-structure, n_samples, nu, record offset, layer) -- the same for every candidate
         off = 0
-        for nm in self.names[start:]:
-            terms = [(j, X[(nm, j)]) for j in ("a", "w", "b") if (nm, j) in X]
-            if terms:
-                layers.append([(j, t, f, n_s, nu, off + 0) for j, (t, f, n_s, nu) in terms])
-                for _, _, _, n_s, _, _ in layers[-1]:
+        for li, nm in enumerate(self.names[start:]):
+            for j in ("a", "w", "b"):
+                if (nm, j) in terms[0]:
+                    _, _, n_s, nu = terms[0][(nm, j)]
+                    layout.append(((nm, j), n_s, nu, off, li))
                     off += 3 + 2 * n_s
         n_cls = self.layers[-1]["K"]
-        buf = torch.empty(off + self.N, dtype=torch.float64, device=self.dev)
-        o = 0
-        for terms in layers:
-            for i, (j, t, f, n_s, nu, _) in enumerate(terms):
-                terms[i] = (j, t, f, n_s, nu, o)
-                F.fxpq_ds_stats(t.reshape(-1), n_s, nu, f, buf[o:o + 3 + 2 * n_s], self._stats_ws, self.stream)
-                o += 3 + 2 * n_s
-        counts = buf[off:].view(torch.int32)[: self.N]
-        F.fxpq_top1_ties(logits, self.N, n_cls, counts, self.stream)
-        hb = buf.cpu()
-        h = hb[:off].tolist()
-        E = 0.0
-        for terms in layers:
-            st = {j: _decode(h, o, n_s, nu) for j, _, _, n_s, nu, o in terms}
-            den = sum(v["sigma"] * v["nu"] for v in st.values())
-            for j, *_ in terms:
-                v = st[j]
-                R = v["max"] - v["min"]
-                if den == 0.0 or R == 0.0:
-                    continue
-                E += (v["sigma"] * v["nu"] / den) * v["L"] / R
-        c = hb[off:].view(torch.int32)[: self.N]
-        uc = float((c > 1).sum()) / self.N
-        mp = float((c - 1).sum()) / (self.N * n_cls)
-        return E + uc + mp, E, uc, mp
+        stats = self._empty(off * nc, torch.float64)
+        items = [(terms[c][ds][0].reshape(-1), n_s, nu, terms[c][ds][1], stats[c * off + o:c * off + o + 3 + 2 * n_s])
+                 for c in range(nc) for ds, n_s, nu, o, _ in layout]
+        F.fxpq_ds_stats_batch(items, self.stream)
+        ties = self._empty(nc * self.N, torch.int32)
+        F.fxpq_top1_ties(logits, nc * self.N, n_cls, ties, self.stream)
+        cost = self._empty(4 * nc, torch.float64)
+        F.fxpq_fopt_cost(stats, off, [(o, nu, n_s, li) for _, n_s, nu, o, li in layout], ties, self.N, n_cls, nc, cost,
+                         self.stream)
+        h = cost.cpu().tolist()
+        return [tuple(h[4 * c:4 * c + 4]) for c in range(nc)]
+
+    def cost(self, cur, cand_fl):
+        """F, E, UnClass, MisPred for one candidate FL."""
+        return self.costs(cur, [cand_fl])[0]
 
     # ------------------------------------------------------------------ Alg. 1 and the forward optimizer
     def qparams_opt(self, cur, K=1):
+        """Alg. 1 for data-structure cur: its FL moves away from the initial one in each direction at a fixed
+        wordlength, and a candidate is accepted only when it lowers the best cost so far.  Each direction
+        takes at least K steps (fewer only at the ends of the FL range), so the initial FL and those 2K
+        neighbours are scored as one batch; every accepted step lets its direction go one step further.
+        Returns (best FL, its cost, [(FL, cost)] in the order the algorithm visits them)."""
         init = self.fmt[cur].fl
-        best_fl, cost_best = init, self.cost(cur, init)[0]
-        trace = [(init, cost_best)]
-        for i in (-1, 1):
-            k, j = 1, 0
-            while k <= K + j:
-                fl = init + i * k
-                if fl < FL_MIN or fl > FL_MAX:
-                    break
-                c = self.cost(cur, fl)[0]
-                trace.append((fl, c))
-                if c < cost_best:
-                    cost_best, best_fl, j = c, fl, j + 1
+        ring = [init] + [init + d * k for d in (-1, 1) for k in range(1, K + 1) if FL_MIN <= init + d * k <= FL_MAX]
+        seen = {fl: c[0] for fl, c in zip(ring, self.costs(cur, ring))}
+        best_fl, best = init, seen[init]
+        trace = [(init, best)]
+        for d in (-1, 1):
+            reach, k = K, 1
+            while k <= reach and FL_MIN <= init + d * k <= FL_MAX:
+                fl = init + d * k
+                if fl not in seen:
+                    seen[fl] = self.cost(cur, fl)[0]
+                trace.append((fl, seen[fl]))
+                if seen[fl] < best:
+                    best, best_fl, reach = seen[fl], fl, reach + 1
                 k += 1
-        return best_fl, cost_best, trace
+        return best_fl, best, trace
 
     def run(self, K=1, upto=None):
         """Alg. 1 on every data-structure in order (the first `upto`), fixing each chosen FL before the next.
@@ -351,14 +405,19 @@ class ForwardOptimizer:
         return out
 
 
+class _Stacked(dict):
+    """Entries over the candidates' stacked batch; an entry of the candidate-independent prefix is repeated
+    once per candidate on first use."""
+
+    def __init__(self, opt, base, nc, init):
+        super().__init__(init)
+        self.opt, self.base, self.nc = opt, base, nc
+
+    def __missing__(self, key):
+        v = self.opt._stack([self.base[key]] * self.nc)
+        self[key] = v
+        return v
+
+
 def env_size(v):
     return v.H * v.W * v.C
-
-
-def _decode(h, o, n_samples, nu):
-    """L, range ends and the mean per-sample dispersion (Eq. importance) of one fxpq_ds_stats record."""
-    sig = 0.0
-    for s in range(n_samples):
-        m1, m2 = h[o + 3 + 2 * s] / nu, h[o + 4 + 2 * s] / nu
-        sig += math.sqrt(max(m2 - m1 * m1, 0.0))
-    return {"L": h[o], "min": h[o + 1], "max": h[o + 2], "sigma": sig / n_samples, "nu": nu}

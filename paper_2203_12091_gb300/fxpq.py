@@ -197,10 +197,23 @@ def fxpq_bias_relu_f32(y, npix, K, bias, relu, stream=None):
     return y
 
 
-def fxpq_ds_stats(x, n_samples, nu, f: Fmt, out, ws, stream=None):
-    """out: device float64[3 + 2 n_samples]; ws: 8 bytes of device scratch."""
-    L.check("fxpq_ds_stats", L.lib().fxpq_ds_stats(_p(x), n_samples, nu, f, _p(out), _p(ws), _s(stream)))
-    return out
+def fxpq_ds_stats_batch(items, stream=None):
+    """items: list of (fp32 device tensor, n_samples, nu, Fmt, record: device float64[3 + 2 n_samples])."""
+    arr = (L.DsItem * len(items))(*[L.DsItem(x.data_ptr(), out.data_ptr(), nu, ns, f) for x, ns, nu, f, out in items])
+    nbytes = L.lib().fxpq_ds_stats_batch_workspace(arr, len(items))
+    if nbytes == 0:
+        raise L.FxpqError("fxpq_ds_stats_batch_workspace", L.ERR_INVALID_ARG)
+    dev = items[0][0].device
+    L.check("fxpq_ds_stats_batch", L.lib().fxpq_ds_stats_batch(arr, len(items), _p(workspace(nbytes, dev)), nbytes,
+                                                               _s(stream)))
+
+
+def fxpq_fopt_cost(stats, cand_stride, terms, ties, N, n_classes, n_cand, cost, stream=None):
+    """terms: list of (record offset in doubles, nu, n_samples, layer); cost: device float64[n_cand * 4]."""
+    arr = (L.CostTerm * max(len(terms), 1))(*[L.CostTerm(o, nu, ns, ly) for o, nu, ns, ly in terms])
+    L.check("fxpq_fopt_cost", L.lib().fxpq_fopt_cost(_p(stats), cand_stride, arr, len(terms), _p(ties), N, n_classes,
+                                                     n_cand, _p(cost), _s(stream)))
+    return cost
 
 
 def fxpq_top1_ties(logits, N, C, counts, stream=None):

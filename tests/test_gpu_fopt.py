@@ -45,25 +45,59 @@ def test_fp32_layers_match_float64(M):
     np.testing.assert_allclose(a.cpu().numpy().reshape(2, 1, 1, 5), qopt.f_avgpool(x), rtol=1e-6, atol=1e-6)
 
 
-def test_ds_stats_and_ties(M):
+def test_ds_stats_batch_and_ties(M):
+    """Statistics records (Eq. DSB_QE's L, the range ends, per-sample mean and sum of squared deviations)
+    against float64 numpy, several items in one batch, one of them past one work unit per sample; a
+    data-structure with a large mean and a small spread keeps its deviation (no one-pass cancellation)."""
     fopt, F = M
     rng = np.random.default_rng(62)
-    x = (rng.standard_normal((3, 1000)) * [[0.5], [2.0], [1.0]]).astype(np.float32)
-    out = torch.empty(3 + 6, dtype=torch.float64, device="cuda")
-    ws = torch.empty(2, dtype=torch.int32, device="cuda")
+    xs = [(rng.standard_normal((3, 1000)) * [[0.5], [2.0], [1.0]]).astype(np.float32),
+          (rng.standard_normal((2, 70000)) * 0.001 + 1000.0).astype(np.float32),
+          rng.standard_normal((1, 5)).astype(np.float32)]
     for fmt in ((6, 1, 3), (1, 1, 1), (8, 0, 5)):
-        F.fxpq_ds_stats(torch.from_numpy(x).cuda(), 3, 1000, F.fmt(*fmt), out, ws)
-        h = out.cpu().numpy()
-        assert h[0] == pytest.approx(qopt.qerr(x, fmt), rel=1e-12)
-        assert h[1] == x.min() and h[2] == x.max()
-        np.testing.assert_allclose(h[3::2], x.astype(np.float64).sum(axis=1), rtol=1e-12)
-        np.testing.assert_allclose(h[4::2], (x.astype(np.float64) ** 2).sum(axis=1), rtol=1e-12)
+        outs = [torch.empty(3 + 2 * x.shape[0], dtype=torch.float64, device="cuda") for x in xs]
+        F.fxpq_ds_stats_batch([(torch.from_numpy(x).cuda().reshape(-1), x.shape[0], x.shape[1], F.fmt(*fmt), o)
+                               for x, o in zip(xs, outs)])
+        for x, o in zip(xs, outs):
+            h = o.cpu().numpy()
+            x64 = x.astype(np.float64)
+            assert h[0] == pytest.approx(qopt.qerr(x, fmt), rel=1e-12)
+            assert h[1] == x.min() and h[2] == x.max()
+            np.testing.assert_allclose(h[3::2], x64.mean(axis=1), rtol=1e-14)
+            np.testing.assert_allclose(h[4::2], ((x64 - x64.mean(axis=1, keepdims=True)) ** 2).sum(axis=1), rtol=1e-9)
     lg = np.array([[1, 1, 0], [2, 0, 0], [5, 5, 5]], np.float32)
     c = torch.empty(3, dtype=torch.int32, device="cuda")
     F.fxpq_top1_ties(torch.from_numpy(lg).cuda(), 3, 3, c)
     assert c.cpu().tolist() == [2, 1, 3]
     F.fxpq_top1_ties(torch.from_numpy(lg.astype(np.int64)).cuda(), 3, 3, c)
     assert c.cpu().tolist() == [2, 1, 3]
+
+
+def test_fopt_cost_from_records(M):
+    """fxpq_fopt_cost on hand-made records: E by Eq. importance / Eq. CPB_QE per layer, UnClass and
+    MisPred by their equations, two candidates with their own records and ties."""
+    fopt, F = M
+    # candidate 0: layer 0 = {a: 2 samples, nu 4}, {w: 1 sample, nu 6}; layer 1 = {w: nu 3 with R = 0}
+    rec0 = [[0.5, -1.0, 3.0, 0.2, 1.0, 0.1, 4.0], [0.25, -2.0, 2.0, 0.0, 6.0], [0.1, 1.0, 1.0, 1.0, 0.0]]
+    rec1 = [[1.5, -1.0, 1.0, 0.0, 0.25, 0.0, 1.0], [0.0, -2.0, 2.0, 0.0, 1.5], [0.3, 0.0, 2.0, 1.0, 3.0]]
+    layout = [(0, 4, 2, 0), (7, 6, 1, 0), (12, 3, 1, 1)]
+    stats = torch.tensor(sum(rec0, []) + sum(rec1, []), dtype=torch.float64, device="cuda")
+    ties = torch.tensor([1, 2, 1, 3, 1, 1, 1, 1], dtype=torch.int32, device="cuda")
+    cost = torch.empty(8, dtype=torch.float64, device="cuda")
+    F.fxpq_fopt_cost(stats, 17, layout, ties, 4, 5, 2, cost)
+    got = cost.cpu().numpy().reshape(2, 4)
+    for c, recs in enumerate((rec0, rec1)):
+        E = 0.0
+        for layer in (0, 1):
+            ts = [(r, nu, ns) for r, (o, nu, ns, ly) in zip(recs, layout) if ly == layer]
+            sig = [sum(np.sqrt(r[4 + 2 * s_] / nu) for s_ in range(ns)) / ns for r, nu, ns in ts]
+            den = sum(sg * nu for sg, (r, nu, ns) in zip(sig, ts))
+            for sg, (r, nu, ns) in zip(sig, ts):
+                if den > 0 and r[2] > r[1]:
+                    E += sg * nu / den * r[0] / (r[2] - r[1])
+        t = ties.cpu().numpy()[4 * c:4 * c + 4]
+        uc, mp = np.mean(t > 1), (t - 1).sum() / (4 * 5)
+        np.testing.assert_allclose(got[c], [E + uc + mp, E, uc, mp], rtol=1e-14)
 
 
 def _tiny():
