@@ -472,6 +472,13 @@ FXPQ_API fxpq_status fxpq_top1_ties(const void* d_logits, int32_t is_int64, int3
 /* Synchronises `stream`, returns and clears the latched device status (FXPQ_OK if none). */
 FXPQ_API fxpq_status fxpq_get_device_status(void* stream);
 
+/* Failure-detection check (tests): one thread waits on a shared-memory mbarrier that nothing arrives on,
+ * with the same bounded-wait routine that guards every wait of the tensor-core kernels, given up after
+ * limit_cycles SM clocks (1 .. 10^8).  The routine latches FXPQ_ERR_TIMEOUT in the device status word
+ * and returns, so the next fxpq_get_device_status reports FXPQ_ERR_TIMEOUT (and clears it) and the
+ * context stays usable.  No copy or tensor-memory allocation is involved. */
+FXPQ_API fxpq_status fxpq_selftest_wait_timeout(int64_t limit_cycles, void* stream);
+
 /* Static English description of a status code. */
 FXPQ_API const char* fxpq_status_string(fxpq_status s);
 

@@ -104,6 +104,7 @@ _SIGS = {
     "fxpq_ds_stats_batch_workspace": (SZ, [VP, I32]),
     "fxpq_ds_stats_batch": (I32, [VP, I32, VP, SZ, VP]),
     "fxpq_fopt_cost": (I32, [VP, I64, VP, I32, VP, I32, I32, I32, VP, VP]),
+    "fxpq_selftest_wait_timeout": (I32, [I64, VP]),
     "fxpq_top1_ties": (I32, [VP, I32, I32, I32, VP, VP]),
     "fxpq_nchw_to_nhwc_f32": (I32, [VP, I32, I32, I32, I32, VP, VP]),
     "fxpq_fl_init": (I32, [ctypes.POINTER(Stats), I32, I32, ctypes.POINTER(Fmt)]),

@@ -344,3 +344,25 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
 }
 
 }  // namespace fxpq
+
+// ------------------------------------------------------------------------------------------
+// Failure detection: the kernels' bounded mbarrier wait, run on a barrier that nothing arrives on.
+// ------------------------------------------------------------------------------------------
+namespace {
+__global__ void wait_selftest_kernel(long long limit, int* status) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    abort_flag = 0;
+    const uint32_t b = fxpq::tc::smem_u32(&bar);
+    fxpq::tc::mbar_init(b, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    // phase 0 of the barrier never completes: the wait runs out, latches the status and returns
+    fxpq::tc::wait_bounded_for(b, 0, &abort_flag, status, limit);
+}
+}  // namespace
+
+extern "C" fxpq_status fxpq_selftest_wait_timeout(int64_t limit_cycles, void* stream) {
+    if (limit_cycles < 1 || limit_cycles > 100000000LL) return FXPQ_ERR_INVALID_ARG;
+    wait_selftest_kernel<<<1, 1, 0, fxpq::as_stream(stream)>>>(limit_cycles, fxpq::status_ptr());
+    return fxpq::after_launch("wait_selftest");
+}

@@ -201,18 +201,23 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
 // timeout status, sets the CTA abort flag) if it gave up or another role already aborted.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
+__device__ __forceinline__ bool wait_bounded_for(uint32_t bar, uint32_t parity, volatile int* abort, int* status,
+                                                 long long limit) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort) return false;
-        if (clock64() - t0 > TC_WAIT_CYCLES) {
+        if (clock64() - t0 > limit) {
             *abort = 1;
             latch_status(status, FXPQ_ERR_TIMEOUT);
             return false;
         }
     }
+}
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
+    return wait_bounded_for(bar, parity, abort, status, TC_WAIT_CYCLES);
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {

@@ -388,3 +388,17 @@ def test_conv_exact_at_group_bound(F, kind, K, mode):
             assert np.abs(acc).max() == 2 ** 24 - 1  # the exact edge is reached
         if kind == "wordlength":
             assert np.any(acc % 2 == 1) and np.abs(acc).max() > 2 ** 24  # odd sums; the full reduction exceeds one group
+
+
+def test_bounded_wait_runs_out_and_the_context_stays_usable(F):
+    """A bounded mbarrier wait of the tensor-core kernels given up after a short limit on a barrier that
+    nothing arrives on: FXPQ_ERR_TIMEOUT is latched and read once, and a normal launch afterwards is
+    bit-exact (no fault, no hang)."""
+    from paper_2203_12091_gb300 import _lib as L
+    assert F.fxpq_get_device_status() == 0
+    assert L.lib().fxpq_selftest_wait_timeout(20000, None) == L.OK
+    assert F.fxpq_get_device_status() == L.ERR_TIMEOUT
+    assert F.fxpq_get_device_status() == 0  # read once: the word is cleared
+    run_case(F, CASES[0])
+    run_case(F, CASES[16])  # a patch-tile case on the tensor cores
+    assert F.fxpq_get_device_status() == 0
