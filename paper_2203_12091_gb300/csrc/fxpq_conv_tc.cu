@@ -14,9 +14,10 @@ int g_num_sms = 0;
 std::mutex g_tc_mu;
 
 // FXPQ_CONV_PATH picks among exact alternatives so that tests can compare them on the same shapes:
-// "tc_rows" keeps every layer on 128-row tiles, "tc_bn128" never takes 256-column tiles and
-// "tc_bn256" takes them wherever the layer allows (by default they also need enough tiles to keep
-// every SM busy).
+// "tc_rows" keeps every layer on 128-row tiles gathered by the producer warps, "tc_patch" takes patch tiles wherever the geometry
+// allows them (by default only while they compute few extra rows), "tc_bn128" never takes
+// 256-column tiles and "tc_bn256" takes them wherever the layer allows (by default they also need
+// enough tiles to keep every SM busy).
 bool conv_path_is(const char* name) {
     const char* e = getenv("FXPQ_CONV_PATH");
     return e && strcmp(e, name) == 0;
@@ -141,6 +142,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return FXPQ_OK;
         P.patch = 0;
+        P.rows_tma = 0;
         P.nacc = 1;
         // window mode for 8-channel stride-1 layers with at most 64 output channels: 8 x 16 output
         // patches, one input window per tile and limb plane, weights resident in shared memory, one
@@ -195,10 +197,25 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 }
             }
         }
+        // Layers whose im2col matrix is the stored activations themselves: 1x1 stride-1 convolutions
+        // without padding ([M][Cp] per plane) and kernels covering the whole unpadded map (P = Q = 1,
+        // FC layers: [N][H W Cp]).  A 128-row A tile is then one 2-D box of [M][R S Cp].
+        const bool one_by_one = a.R == 1 && a.S == 1 && a.stride == 1 && a.pad == 0;
+        const bool whole_map = a.R == a.H && a.S == a.W && a.pad == 0 && a.P == 1 && a.Q == 1;
+        if (P.patch == 0 && (one_by_one || whole_map) && a.M > 0 && a.M < (1LL << 31) - TC_BM &&
+            !conv_path_is("tc_rows") && !conv_path_is("tc_patch")) {
+            const cuuint64_t xdims[3] = {(cuuint64_t)P.RSC, (cuuint64_t)a.M, (cuuint64_t)a.px};
+            const cuuint64_t xstrides[2] = {(cuuint64_t)P.RSC * 2, (cuuint64_t)a.x_ps * 2};
+            const cuuint32_t xbox[3] = {(cuuint32_t)TC_BK, (cuuint32_t)TC_BM, 1};
+            if (enc(&P.tmap_x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<__half*>(a.x), xdims, xstrides, xbox, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS)
+                P.rows_tma = 1;
+        }
         // patch tiles for stride-1 layers whose taps are whole 64-channel blocks, or 8-channel inputs
         // (a k-block of 8 taps)
         const bool narrow = a.Cp == 8;
-        if (P.patch == 0 && a.stride == 1 && (P.cp64 || narrow) && a.P > 0 && a.Q > 0 && a.N > 0 &&
+        if (P.patch == 0 && !P.rows_tma && a.stride == 1 && (P.cp64 || narrow) && a.P > 0 && a.Q > 0 && a.N > 0 &&
             !conv_path_is("tc_rows")) {
             int best_tw = 0, best_th = 0;
             long long best = 0;
@@ -207,9 +224,12 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 const long long cost = (long long)((a.P + th - 1) / th) * ((a.Q + tw - 1) / tw);
                 if (best_tw == 0 || cost < best) best = cost, best_tw = tw, best_th = th;
             }
-            // take patches unless they compute clearly more rows than 128-row tiles of N*P*Q would
+            // take patches unless they need more than twice as many tiles as 128-row tiles of N*P*Q:
+            // one TMA box per k-block against 128 gathered rows pays for a good deal of idle MMA rows
+            // (3x3 layers, 14x14 maps: 2 patches of 126 rows per image, 1.3x the row tiles, 1.7-2x
+            // faster; 7x7 maps: 2.6x the row tiles, 6% slower)
             const long long row_tiles = (a.M + TC_BM - 1) / TC_BM;
-            if ((double)a.N * best <= 1.15 * (double)row_tiles + 1e-9) {
+            if ((double)a.N * best <= 2.0 * (double)row_tiles + 1e-9 || conv_path_is("tc_patch")) {
                 const cuuint64_t xdims[5] = {(cuuint64_t)a.Cp, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N,
                                              (cuuint64_t)a.px};
                 const cuuint64_t xstrides[4] = {(cuuint64_t)a.Cp * 2, (cuuint64_t)a.W * a.Cp * 2,

@@ -87,6 +87,10 @@ struct TcParams {
                          // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle);
                          // 3: Cp == 8, window mode (one input window per tile and limb plane, taps as
                          //    shifted descriptors, weights resident in shared memory)
+    int rows_tma;        // 128-row tiles whose A tile is one 2-D TMA box of the activations seen as
+                         // [planes][M][R*S*Cp] (1x1 stride-1 layers without padding, and kernels that
+                         // cover the whole unpadded map: FC layers), box {64, 128, 1}, 128-byte
+                         // swizzle, rows past M and taps past R*S*Cp zero filled
     int nacc;            // fp32 accumulators per TMEM buffer (window mode: one per limb pair)
     int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
     int win_bytes;       // window mode: bytes of one window (128-byte aligned)
@@ -471,7 +475,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         for (int s = 0; s < TC_STAGES; ++s) {
             // patch tiles: one expect_tx arrival for both TMAs; row tiles: one arrival per producer
             // warp + the weight TMA's expect_tx
-            mbar_init(full0 + 8 * s, P.patch ? 1 : 4 + 1);
+            mbar_init(full0 + 8 * s, (P.patch || P.rows_tma) ? 1 : 4 + 1);
             mbar_init(empty0 + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -547,7 +551,7 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
             }
         }
-    } else if (warp < 4 && P.patch) {
+    } else if (warp < 4 && (P.patch || P.rows_tma)) {
         // ============================================================ producer, patch tiles
         // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
         // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
@@ -559,8 +563,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             // (barrier wait, two TMA instructions) would bound the stage rate
             const int me = warp;
             const bool narrow = P.patch == 2;
-            const uint32_t a_bytes = (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
-            const int per_img = P.tiles_p * P.tiles_q;
+            const uint32_t a_bytes = P.rows_tma ? (uint32_t)(TC_BM * 128) : (uint32_t)(P.TH * P.TW * (narrow ? 8 * 16 : 128));
+            const int per_img = P.rows_tma ? 1 : P.tiles_p * P.tiles_q;
             uint32_t it = 0;
             bool ok = true;
             for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
@@ -568,7 +572,8 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                 (void)sp;
                 const int tm = t / P.tiles_n, tn = t % P.tiles_n;
                 const int n_img = tm / per_img, r = tm - n_img * per_img;
-                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
+                const int tq = P.rows_tma ? 1 : P.tiles_q;
+                const int hp0 = (r / tq) * P.TH - a.pad, wq0 = (r % tq) * P.TW - a.pad;
                 for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups) && ok; ++gi) {
                     const TcGroup g = P.g[gi];
                     // tap (rr, ss) and channel offset cc of the group's first k-block, then stepped by
@@ -593,6 +598,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                     tma_load_5d(smem_u32(sA + stage * A_BYTES + tl * 2048), &P.tmap_x, in ? 0 : 8,
                                                 wq0 + s8, hp0 + r8, n_img, g.a_plane, fb);
                                 }
+                            } else if (P.rows_tma) {
+                                tma_load_3d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, kb * TC_BK, tm * TC_BM, g.a_plane,
+                                            fb);
                             } else {
                                 tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
                                             g.a_plane, fb);

@@ -144,6 +144,12 @@ CASES = [
     (5, 1, 4096, 136, 1, 1, 0, (5, 0, 2), (7, 1, 9), (16, 8), False, 2, None),
     (4, 1, 4096, 1000, 1, 1, 0, (16, 0, 12), (16, 1, 18), (16, 20), False, 1, None),
     (9, 3, 512, 64, 3, 1, 0, (7, 0, 3), (5, 1, 6), (16, 4), True, 0, (6, 0, 1)),
+    # 1x1 stride-1 layers without padding: 128-row tiles whose A tile is one 2-D TMA box of [M][Cp]
+    # (ragged M, M below one tile, two-limb activations with int64 sums, 256 output channels)
+    (3, 9, 64, 72, 1, 1, 0, (8, 0, 4), (8, 1, 7), (16, 15), True, 0, (8, 0, 3)),
+    (2, 20, 128, 128, 1, 1, 0, (16, 1, 12), (8, 1, 7), (16, 20), False, 1, None),
+    (1, 11, 192, 256, 1, 1, 0, (7, 0, 3), (6, 1, 6), (16, 12), True, 0, (8, 0, 2)),
+    (2, 13, 40, 24, 1, 1, 0, (8, 0, 4), (8, 1, 7), None, True, 2, None),
     # window mode, two limbs, one-plane codes: the 32-bit epilogue (shift >= 17, bias not finer), its
     # shift-17 edge and no ReLU with signed codes, and the 64-bit fallback for a finer bias
     (2, 20, 3, 48, 3, 1, 1, (16, 1, 9), (16, 1, 12), (16, 18), False, 0, (6, 1, 2)),
@@ -293,6 +299,7 @@ SCALE_CASES = [
     (CASES[25], (16, 14), (16, 12)),    # 256-column tiles
     (CASES[32], (16, 14), (16, 12)),    # window mode, two-limb fast epilogue
     (CASES[35], (16, 14), (16, 12)),    # window mode, ACC64
+    (CASES[41], (16, 14), (16, 12)),    # 1x1: A tiles as 2-D TMA boxes
     (CASES[36], (16, 14), (16, 12)),    # split reduction
     (CASES[39], (16, 13), (16, 10)),    # split reduction, two limbs, ACC64
 ]
