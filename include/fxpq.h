@@ -240,6 +240,13 @@ FXPQ_API fxpq_status fxpq_fl_init(const fxpq_stats* h_stats, int32_t bits, int32
 /* scale s becomes v * aleph1_code[o] of scale s + fmt_scale.fl, and aleph2_code[o] is aligned  */
 /* to it like the bias (delta2 = that scale - fmt_shift.fl, the same two cases); ReLU and the  */
 /* FxP-QLayer follow.  d_scale and d_shift are int32 code arrays [K], both set or both NULL.   */
+/* d_wpacked (optional; Sec. V-E.2: k-bit storage of the read-only data-structures): the       */
+/* weights of d_w, one plane of fmt_w.bits <= 8, as fxpq_pack_weights' tiles.  Layers whose A   */
+/* operand is the stored activations themselves (FC layers: R = H, S = W, pad 0; 1x1 stride-1   */
+/* without padding) and whose output tiles are too few for the SMs (the split reduction) then   */
+/* read k bits per weight from memory instead of a 2-byte fp16 code; other layers ignore it.    */
+/* d_w stays required (every other path reads it); d_wpacked must hold exactly d_w's codes,     */
+/* 16-byte aligned.                                                                             */
 /* ---------------------------------------------------------------------------------------- */
 enum { FXPQ_OUT_CODES = 0, FXPQ_OUT_ACC64 = 1, FXPQ_OUT_F32 = 2 };
 
@@ -255,6 +262,7 @@ typedef struct {
     fxpq_fmt fmt_scale, fmt_shift;  /* Scale layer aleph1 / aleph2 formats (if d_scale)      */
     const int32_t* d_scale;    /* Scale layer aleph1 codes [K], or NULL (no Scale layer)     */
     const int32_t* d_shift;    /* Scale layer aleph2 codes [K] (NULL iff d_scale is NULL)    */
+    const void* d_wpacked;     /* optional: the same weights packed by fxpq_pack_weights, or NULL */
 } fxpq_conv_desc;
 
 FXPQ_API size_t fxpq_conv_workspace(const fxpq_conv_desc* h_desc);
@@ -308,6 +316,20 @@ FXPQ_API fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt fm
 FXPQ_API fxpq_status fxpq_unpack_codes(const uint32_t* d_words, int64_t n, fxpq_fmt fmt, void* d_codes,
                                        void* stream);
 
+/* Packed weights for the contraction (Sec. V-E.2: a data-structure of k-bit values occupies k bits
+ * per value).  d_w: one plane of fp16 weight codes [K][L] (L = R*S*Cp, KRSC order), fmt_w.bits in
+ * [1, 8].  d_packed receives the codes' k-bit two's-complement fields as bit planes of tiles of 256
+ * output channels x 64 reduction steps: words [ceil(L / 64)][K_pad / 256][k][256][2], K_pad = K
+ * rounded up to a multiple of 256; word (kb, t, b, o, h) holds at bit i bit b of the field of code
+ * W[256 t + o][64 kb + 32 h + i] (zero past L and past K).  These are fxpq_pack_codes' words for the
+ * codes rearranged as [ceil(L / 64)][K_pad][64], with each tile's words ordered plane-major.  One tile
+ * is a single contiguous run of 2 KiB per plane, which the contraction copies to shared memory and
+ * expands there.  fxpq_packed_weights_bytes gives the size (k bits per code of the padded tensor);
+ * d_packed 16-byte aligned. */
+FXPQ_API size_t fxpq_packed_weights_bytes(fxpq_fmt fmt_w, int32_t K, int32_t L);
+FXPQ_API fxpq_status fxpq_pack_weights(const void* d_w, fxpq_fmt fmt_w, int32_t K, int32_t L, void* d_packed,
+                                       void* stream);
+
 /* BN -> Scale preprocessing (Sec. IV-A.1, the BatchNorm rewrite): per channel,
  *   aleph1 = gamma / sqrt(var + eps),  aleph2 = beta - (gamma * mean) / sqrt(var + eps),
  * each operation one correctly rounded fp32 step in that order.  Inputs: fp32 device arrays of n
@@ -343,6 +365,7 @@ typedef struct {
     fxpq_fmt fmt_scale, fmt_shift;  /* conv: Scale layer formats (fxpq_conv_desc)            */
     const int32_t* d_scale;  /* conv: Scale layer aleph1 codes [K] or NULL                   */
     const int32_t* d_shift;  /* conv: Scale layer aleph2 codes [K] or NULL                   */
+    const void* d_wpacked;   /* conv: optional packed weights (fxpq_conv_desc.d_wpacked)       */
 } fxpq_op_desc;
 
 typedef struct {

@@ -42,14 +42,14 @@ class ConvDesc(ctypes.Structure):
     _fields_ = [("N", I32), ("H", I32), ("W", I32), ("C", I32), ("Cp", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("out_mode", I32),
                 ("fmt_x", Fmt), ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("w_l1", I64),
-                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
+                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP), ("d_wpacked", VP)]
 
 
 class OpDesc(ctypes.Structure):
     _fields_ = [("op", I32), ("src0", I32), ("src1", I32), ("dst", I32), ("K", I32), ("R", I32), ("S", I32),
                 ("stride", I32), ("pad", I32), ("relu", I32), ("last", I32), ("recip_code", I32),
                 ("fmt_w", Fmt), ("fmt_b", Fmt), ("fmt_y", Fmt), ("d_w", VP), ("d_bias", VP), ("w_l1", I64),
-                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP)]
+                ("fmt_scale", Fmt), ("fmt_shift", Fmt), ("d_scale", VP), ("d_shift", VP), ("d_wpacked", VP)]
 
 
 class DsItem(ctypes.Structure):
@@ -94,6 +94,8 @@ _SIGS = {
     "fxpq_bn_to_scale": (I32, [VP, VP, VP, VP, I64, ctypes.c_float, VP, VP, VP]),
     "fxpq_pack_codes": (I32, [VP, I64, Fmt, VP, VP]),
     "fxpq_unpack_codes": (I32, [VP, I64, Fmt, VP, VP]),
+    "fxpq_packed_weights_bytes": (ctypes.c_size_t, [Fmt, I32, I32]),
+    "fxpq_pack_weights": (I32, [VP, Fmt, I32, I32, VP, VP]),
     "fxpq_net_memory": (I32, [ctypes.POINTER(Net), I32, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
     "fxpq_conv_f32": (I32, [ctypes.POINTER(ConvF32Desc), VP, VP, VP, VP, VP]),
     "fxpq_maxpool_f32": (I32, [VP, I32, I32, I32, I32, I32, I32, I32, VP, VP]),

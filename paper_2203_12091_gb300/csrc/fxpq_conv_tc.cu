@@ -119,11 +119,32 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     // wide layers with enough tiles
     int BN = 128;
     const long long row_tiles_est = (a.M + TC_BM - 1) / TC_BM;
+    // Layers whose im2col matrix is the stored activations themselves: 1x1 stride-1 convolutions
+    // without padding ([M][Cp] per plane) and kernels covering the whole unpadded map (P = Q = 1,
+    // FC layers: [N][H W Cp]).  A 128-row A tile is then one 2-D box of [M][R S Cp].
+    const bool one_by_one = a.R == 1 && a.S == 1 && a.stride == 1 && a.pad == 0;
+    const bool whole_map = a.R == a.H && a.S == a.W && a.pad == 0 && a.P == 1 && a.Q == 1;
+    const bool rows_geom = (one_by_one || whole_map) && a.M > 0 && a.M < (1LL << 31) - TC_BM &&
+                           !conv_path_is("tc_rows") && !conv_path_is("tc_patch");
+    // ... with few row tiles (FC layers at small batches) they take 256-column tiles and a split
+    // reduction fills the SMs: the MMA thread's fixed cost per k-block is then hidden, and the weights
+    // stream at the memory's rate
+    const bool wide_split = rows_geom && !acc64 && !a.has_scale && ws && a.K > 128 && !conv_path_is("tc_bn128") &&
+                            !conv_path_is("tc_nosplit") && row_tiles_est * ((a.K + 255) / 256) * 2 <= sms;
     if (acc64 || a.K <= 64)
         BN = 64;
-    else if (a.K > 128 && !conv_path_is("tc_bn128") &&
-             (conv_path_is("tc_bn256") || (a.K % 256 == 0 && row_tiles_est * (a.K / 256) >= sms)))
+    else if (wide_split || (a.K > 128 && !conv_path_is("tc_bn128") &&
+                            (conv_path_is("tc_bn256") || (a.K % 256 == 0 && row_tiles_est * (a.K / 256) >= sms))))
         BN = 256;
+    // packed k-bit weights (k <= 8, one plane) are read by the 256-column TMA-row instances of the
+    // split (FC) layers, whose weights stream through once; elsewhere every weight tile is expanded
+    // once per row tile and the fp16 codes are read instead
+    P.pk = d.d_wpacked && d.fmt_w.bits <= 8 && BN == 256 && wide_split && (reinterpret_cast<uintptr_t>(d.d_wpacked) & 15) == 0 &&
+           !conv_path_is("tc_nopack");
+    P.wpack = static_cast<const uint32_t*>(d.d_wpacked);
+    P.wk = d.fmt_w.bits;
+    P.wsigned = d.fmt_w.is_signed;
+    P.K_pad = (a.K + 255) / 256 * 256;
     // too few 128-column tiles to occupy every SM (small batches, FC layers): 64-column tiles double
     // the CTA count
     if (BN == 128 && row_tiles_est * ((a.K + 127) / 128) < sms) BN = 64;
@@ -197,13 +218,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 }
             }
         }
-        // Layers whose im2col matrix is the stored activations themselves: 1x1 stride-1 convolutions
-        // without padding ([M][Cp] per plane) and kernels covering the whole unpadded map (P = Q = 1,
-        // FC layers: [N][H W Cp]).  A 128-row A tile is then one 2-D box of [M][R S Cp].
-        const bool one_by_one = a.R == 1 && a.S == 1 && a.stride == 1 && a.pad == 0;
-        const bool whole_map = a.R == a.H && a.S == a.W && a.pad == 0 && a.P == 1 && a.Q == 1;
-        if (P.patch == 0 && (one_by_one || whole_map) && a.M > 0 && a.M < (1LL << 31) - TC_BM &&
-            !conv_path_is("tc_rows") && !conv_path_is("tc_patch")) {
+        if (P.patch == 0 && rows_geom) {
             const cuuint64_t xdims[3] = {(cuuint64_t)P.RSC, (cuuint64_t)a.M, (cuuint64_t)a.px};
             const cuuint64_t xstrides[2] = {(cuuint64_t)P.RSC * 2, (cuuint64_t)a.x_ps * 2};
             const cuuint32_t xbox[3] = {(cuuint32_t)TC_BK, (cuuint32_t)TC_BM, 1};
@@ -249,9 +264,11 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 }
             }
         }
-        // one-plane codes: stage the tile in shared memory and write it with TMA stores
+        if (!P.rows_tma) P.pk = 0;
+        // one-plane codes: stage the tile in shared memory and write it with TMA stores (not with packed
+        // weights, whose staging region holds the packed stages)
         P.fast_store = 0;
-        if (a.out_mode == FXPQ_OUT_CODES && a.py == 1) {
+        if (a.out_mode == FXPQ_OUT_CODES && a.py == 1 && !P.pk) {
             CUresult r;
             if (P.patch) {
                 const cuuint64_t ydims[4] = {(cuuint64_t)a.K, (cuuint64_t)a.Q, (cuuint64_t)a.P, (cuuint64_t)a.N};
@@ -287,8 +304,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     P.part = nullptr;
     P.gs[0] = 0;
     P.gs[1] = P.n_groups;
-    // (64-column tiles only, without a Scale layer: the instantiations that carry the split)
-    if (P.patch != 3 && BN == 64 && !a.has_scale && ws && P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
+    // (64-column tiles, and 256-column TMA-row tiles, without a Scale layer: the instantiations that carry
+    // the split)
+    if (P.patch != 3 && (BN == 64 || (BN == 256 && P.rows_tma && !acc64)) && !a.has_scale && ws &&
+        P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
         const int ng = P.n_groups;
         int min_len = 1 << 30;
         for (int gi = 0; gi < ng; ++gi) min_len = std::min(min_len, P.g[gi].kb1 - P.g[gi].kb0);
@@ -337,7 +356,13 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 cudaFuncSetAttribute(conv_tc_kernel<128, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<128>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<256, int, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)tc_smem_bytes<256>()) != cudaSuccess)
+                                     (int)tc_smem_bytes<256>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<256>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, false, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess)
                 return FXPQ_ERR_CUDA;
             g_tc_attr_set = true;
         }
@@ -345,7 +370,13 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     const int grid = P.n_units < sms ? P.n_units : sms;
     launched = true;
     if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);  // never split
-    if (P.ksplit > 1 && acc64)
+    if (P.pk && P.ksplit > 1)
+        conv_tc_kernel<256, int, false, true, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
+    else if (P.pk)
+        conv_tc_kernel<256, int, false, false, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
+    else if (P.ksplit > 1 && BN == 256)
+        conv_tc_kernel<256, int, false, true><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
+    else if (P.ksplit > 1 && acc64)
         conv_tc_kernel<64, long long, false, true><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);
     else if (P.ksplit > 1)
         conv_tc_kernel<64, int, false, true><<<grid, tc_threads(64), tc_smem_bytes<64>(), st>>>(P);

@@ -54,6 +54,12 @@ __host__ __device__ constexpr int tc_lag(int BN) { return tc_stages(BN) - 1 < 3 
 // BN / 8 of them up to 16, each then draining BN / 128 chunks), one MMA / TMEM-allocation warp.
 __host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8 < 16 ? BN / 8 : 16; }
 __host__ __device__ constexpr int tc_threads(int BN) { return (5 + tc_epi_warps(BN)) * 32; }
+// Packed weights (PK instances, BN = 256 only): the weights arrive as k-bit records (k <= 8) and these
+// extra warps after the MMA warp, with producer warps 1-3, expand every k-block's records into the
+// fp16 B stage.  The packed stages live in the output staging region, which PK layers do not use.
+constexpr int TC_PK_WARPS = 5;
+constexpr int TC_PK_CONVERTERS = 3 + TC_PK_WARPS;  // converter warps
+__host__ __device__ constexpr int tc_threads_pk(int BN, bool pk) { return tc_threads(BN) + (pk ? 32 * TC_PK_WARPS : 0); }
 // Dynamic shared memory: barriers, the stages (A and B tiles), the output staging tile.
 template <int BN>
 constexpr size_t tc_smem_bytes() {
@@ -108,6 +114,11 @@ struct TcParams {
     int gs[TC_MAX_SPLIT + 1];
     void* part;
     int cp64;      // Cp % 64 == 0: a k-block never straddles a tap
+    // Packed weights (pk = 1, one plane of wk <= 8 bits, wsigned): fxpq_pack_weights' tiles, words
+    // [ceil(R*S*Cp / 64)][K_pad / 256][wk][256][2]: word (kb, t, b, o, h) bit i = bit b of code
+    // 64 kb + 32 h + i of output channel 256 t + o.
+    const uint32_t* wpack;
+    int pk, wk, wsigned, K_pad;
     int* status;
     TcGroup g[TC_MAX_GROUPS];
 };
@@ -201,6 +212,87 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
         "[%5];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
         : "memory");
+}
+
+// 1-D bulk copy global -> shared completing on mbarrier `bar` (both addresses 16-byte aligned, bytes a
+// multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+// Bit-plane bytes -> fp16 codes.  (lo, hi): an 8 x 8 bit matrix, byte b = plane b (bytes 0-3 in lo,
+// 4-7 in hi), bit c = code c of eight consecutive codes.  Three delta swaps transpose it (Hacker's
+// Delight, 7-3: byte c then holds code c's k bits).  Signed codes have bit k-1 flipped (`flip`), which
+// maps them to u = code + 2^(k-1) in [0, 2^k); each byte then becomes the fp16 1024 + u (exponent
+// byte 0x64, u in the mantissa) and one half2 subtraction of `off` = 1024 (+ 2^(k-1) if signed)
+// leaves the code itself, exactly.  Returns the 16-byte chunk of the eight fp16 codes.
+__device__ __forceinline__ uint4 planes_to_f16(uint32_t lo, uint32_t hi, uint32_t flip, uint32_t off) {
+    uint32_t t;
+    t = (lo ^ (lo >> 7)) & 0x00AA00AAu;
+    lo ^= t ^ (t << 7);
+    t = (hi ^ (hi >> 7)) & 0x00AA00AAu;
+    hi ^= t ^ (t << 7);
+    t = (lo ^ (lo >> 14)) & 0x0000CCCCu;
+    lo ^= t ^ (t << 14);
+    t = (hi ^ (hi >> 14)) & 0x0000CCCCu;
+    hi ^= t ^ (t << 14);
+    t = (lo ^ (hi << 4)) & 0xF0F0F0F0u;  // the 4 x 4 blocks across the two words
+    lo ^= t;
+    hi ^= t >> 4;
+    lo ^= flip;
+    hi ^= flip;
+    const __half2 o2 = *reinterpret_cast<const __half2*>(&off);
+    uint32_t h[4] = {__byte_perm(lo, 0x64646464u, 0x5140), __byte_perm(lo, 0x64646464u, 0x5342),
+                     __byte_perm(hi, 0x64646464u, 0x5140), __byte_perm(hi, 0x64646464u, 0x5342)};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const __half2 v = __hsub2(*reinterpret_cast<const __half2*>(&h[q]), o2);
+        h[q] = *reinterpret_cast<const uint32_t*>(&v);
+    }
+    return make_uint4(h[0], h[1], h[2], h[3]);
+}
+
+// 4 x 4 byte transpose: out[m] byte b = in[b] byte m.
+__device__ __forceinline__ void byte_transpose4(const uint32_t (&in)[4], uint32_t (&out)[4]) {
+    const uint32_t t0 = __byte_perm(in[0], in[1], 0x5140), t1 = __byte_perm(in[0], in[1], 0x7362);
+    const uint32_t t2 = __byte_perm(in[2], in[3], 0x5140), t3 = __byte_perm(in[2], in[3], 0x7362);
+    out[0] = __byte_perm(t0, t2, 0x5410);
+    out[1] = __byte_perm(t0, t2, 0x7632);
+    out[2] = __byte_perm(t1, t3, 0x5410);
+    out[3] = __byte_perm(t1, t3, 0x7632);
+}
+
+// Expands one k-block's packed tile (`pk`: k bit planes of BN rows x 2 words, word (b, o, h) at
+// 2 (b BN + o) + h, bit i = bit b of code 32 h + i of row o) into the fp16 B stage `sb` (BN rows of
+// 128 bytes, 128-byte swizzle: chunk j of row o at 16 ((j ^ o) & 7)).  Thread tid of nthreads takes
+// rows tid, tid + nthreads, ...: one 8-byte load per plane (consecutive rows: no bank conflicts), then
+// eight chunks.
+template <int BN>
+__device__ __forceinline__ void pk_convert_stage(const uint32_t* pk, unsigned char* sb, int k, uint32_t flip,
+                                                 uint32_t off, int tid, int nthreads) {
+    for (int o = tid; o < BN; o += nthreads) {
+        uint32_t w[2][8];
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            uint2 v = make_uint2(0u, 0u);
+            if (b < k) v = *reinterpret_cast<const uint2*>(pk + 2 * (b * BN + o));
+            w[0][b] = v.x;
+            w[1][b] = v.y;
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            uint32_t lo[4], hi[4];
+            byte_transpose4({w[h][0], w[h][1], w[h][2], w[h][3]}, lo);
+            byte_transpose4({w[h][4], w[h][5], w[h][6], w[h][7]}, hi);
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                const int j = 4 * h + m;
+                *reinterpret_cast<uint4*>(sb + o * 128 + ((j ^ (o & 7)) << 4)) = planes_to_f16(lo[m], hi[m], flip, off);
+            }
+        }
+    }
 }
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
@@ -430,14 +522,51 @@ __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
 }
 
 // ------------------------------------------------------------------ kernel
+// PK converter warp `cid` (of TC_PK_CONVERTERS): walks the same k-block sequence as the issuing thread;
+// for each k-block waits until its A box and packed records have landed (pkfull), expands its share of
+// the records into the B stage, makes the writes visible to the tensor cores' async proxy and arrives
+// on the stage's full barrier (one arrival per warp).
+template <int BN, bool SPLIT>
+__device__ __forceinline__ void pk_convert_loop(const TcParams& P, int cid, int lane, const unsigned char* sP,
+                                                unsigned char* sB, uint32_t pkfull0, uint32_t full0, volatile int* abort) {
+    constexpr int STAGES = tc_stages(BN);
+    constexpr int B_BYTES = BN * TC_BK * 2;
+    const int k = P.wk;
+    const uint32_t flip = P.wsigned ? 0x01010101u * (1u << (k - 1)) : 0u;
+    const uint32_t o1 = 0x6400u + (P.wsigned ? (1u << (k - 1)) : 0u);  // fp16 bits of 1024 (+ 2^(k-1))
+    const uint32_t off = o1 | (o1 << 16);
+    uint32_t it = 0;
+    for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles); ut += gridDim.x) {
+        const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
+        (void)t;
+        (void)sp;
+        for (int gi = SPLIT ? P.gs[sp] : 0; gi < (SPLIT ? P.gs[sp + 1] : P.n_groups); ++gi) {
+            for (int kb = P.g[gi].kb0; kb < P.g[gi].kb1; ++kb, ++it) {
+                const uint32_t stage = it % STAGES, phase = (it / STAGES) & 1;
+                if (!wait_bounded(pkfull0 + 8 * stage, phase, abort, P.status)) return;
+                pk_convert_stage<BN>(reinterpret_cast<const uint32_t*>(sP + stage * (BN * 64)), sB + stage * B_BYTES, k,
+                                     flip, off, cid * 32 + lane, TC_PK_CONVERTERS * 32);
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(full0 + 8 * stage);
+            }
+        }
+    }
+}
+
 // SPLIT: the instantiation that runs split reductions (P.ksplit >= 1, unit share ranges P.gs); without it
 // the unit loop is the tile loop and every tile takes all P.n_groups groups.
-template <int BN, typename ACC, bool SC, bool SPLIT = false>
-__global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+// PK: the instantiation that reads packed k-bit weights (P.pk = 1; BN = 256, TMA A tiles, no output
+// staging): one thread issues every copy and TC_PK_CONVERTERS warps expand the weights.
+template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false>
+__global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
     constexpr int TC_STAGES = tc_stages(BN);
     constexpr int TC_LAG = tc_lag(BN);
     static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
-    constexpr int TC_PRODUCERS = tc_producers(BN);
+    static_assert(!PK || (BN == 256 && sizeof(ACC) == 4 && !SC), "packed weights: 256-column int32 tiles only");
+    static_assert(!PK || TC_STAGES * BN * 64 <= BN * TC_BM * 2, "packed stages must fit the staging region");
+    // PK: one issuing thread (producer warp 0), so its stage waits are in order by construction
+    constexpr int TC_PRODUCERS = PK ? 1 : tc_producers(BN);
     static_assert(TC_STAGES % TC_PRODUCERS == 0 && TC_PRODUCERS <= 4,
                   "each stage must have one producer thread among warps 0..3");
     constexpr int EPI_WARPS = tc_epi_warps(BN);
@@ -467,6 +596,10 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
     const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue warp
     const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
     const uint32_t wbar = smem_u32(bars + 2 * TC_STAGES + 9);      // window mode: resident weights loaded
+    // PK: pkfull[s] completes when stage s's A box and packed weight records have landed; the
+    // converters then fill the B stage and arrive on full[s]
+    const uint32_t pkfull0 = smem_u32(bars + 2 * TC_STAGES + 10);
+    unsigned char* sP = sO;  // PK: packed stages of BN * 64 bytes (k <= 8 words per 32 codes)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const ConvArgs& a = P.a;
@@ -475,8 +608,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
         for (int s = 0; s < TC_STAGES; ++s) {
             // patch tiles: one expect_tx arrival for both TMAs; row tiles: one arrival per producer
             // warp + the weight TMA's expect_tx
-            mbar_init(full0 + 8 * s, (P.patch || P.rows_tma) ? 1 : 4 + 1);
+            mbar_init(full0 + 8 * s, PK ? TC_PK_CONVERTERS : (P.patch || P.rows_tma) ? 1 : 4 + 1);
             mbar_init(empty0 + 8 * s, 1);
+            if (PK) mbar_init(pkfull0 + 8 * s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accfull0 + 8 * b, 1);
@@ -588,8 +722,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                 ok = false;
                                 break;
                             }
-                            const uint32_t fb = full0 + 8 * stage;
-                            mbar_arrive_expect_tx(fb, a_bytes + (uint32_t)B_BYTES);
+                            const uint32_t fb = PK ? pkfull0 + 8 * stage : full0 + 8 * stage;
+                            const uint32_t pk_bytes = PK ? (uint32_t)(BN * 8 * P.wk) : 0u;
+                            mbar_arrive_expect_tx(fb, a_bytes + (PK ? pk_bytes : (uint32_t)B_BYTES));
                             if (narrow) {
                                 for (int tl = 0; tl < 8; ++tl) {
                                     const int tap = kb * 8 + tl;
@@ -605,7 +740,12 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                                 tma_load_5d(smem_u32(sA + stage * A_BYTES), &P.tmap_x, cc, wq0 + ss, hp0 + rr, n_img,
                                             g.a_plane, fb);
                             }
-                            tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, kb * TC_BK, tn * BN, g.w_plane, fb);
+                            if (PK)
+                                bulk_load(smem_u32(sP + stage * (BN * 64)),
+                                          P.wpack + ((size_t)kb * P.K_pad + (size_t)tn * BN) * 2 * P.wk, pk_bytes, fb);
+                            else
+                                tma_load_3d(smem_u32(sB + stage * B_BYTES), &P.tmap_w, kb * TC_BK, tn * BN, g.w_plane,
+                                            fb);
                         }
                         if (!narrow) {
                             cc += TC_BK;
@@ -620,15 +760,18 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
                     }
                 }
             }
-            // bounded wait until the copies of the last stages have landed
+            // bounded wait until the copies of the last stages have landed (PK: on pkfull, which only
+            // the copies complete)
+            const uint32_t drain0 = PK ? pkfull0 : full0;
             const uint32_t from = it >= TC_STAGES ? it - TC_STAGES : 0;
             for (uint32_t j = from; j < it; ++j) {
                 const long long t0 = clock64();
-                while (!mbar_try_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
+                while (!mbar_try_wait(drain0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1) &&
                        clock64() - t0 < TC_WAIT_CYCLES) {
                 }
             }
         }
+        if (PK && warp >= 1) pk_convert_loop<BN, SPLIT>(P, warp - 1, lane, sP, sB, pkfull0, full0, abort);
     } else if (warp < 4) {
         // ============================================================ producers, row tiles
         // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
@@ -1025,6 +1168,9 @@ __global__ void __launch_bounds__(tc_threads(BN), 1) conv_tc_kernel(const __grid
             }
         }
         if (leader) bulk_wait0();  // every output store has completed
+    } else if (PK && warp > MMA_WARP) {
+        // ============================================================ packed-weight converters
+        pk_convert_loop<BN, SPLIT>(P, 3 + (warp - MMA_WARP - 1), lane, sP, sB, pkfull0, full0, abort);
     } else if (lane == 0 && P.patch == 3) {
         // ============================================================ MMA issue, window mode
         // Per tile and limb pair (ia, iw): R * S2/2 MMAs of K = 16 (two taps of 8 channels).  The A

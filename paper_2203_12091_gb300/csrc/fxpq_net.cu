@@ -198,6 +198,7 @@ extern "C" fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_im
                 d.fmt_shift = o.fmt_shift;
                 d.d_scale = o.d_scale;
                 d.d_shift = o.d_shift;
+                d.d_wpacked = o.d_wpacked;
                 int32_t scale = 0;
                 st = fxpq_conv_fwd(&d, ptr(o.src0), o.d_w, o.d_bias, last ? (void*)d_logits : ptr(o.dst), &scale,
                                    conv_ws, conv_ws ? cws : 0, stream);
@@ -352,6 +353,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.fmt_shift = o.fmt_shift;
                 cd.d_scale = o.d_scale;
                 cd.d_shift = o.d_shift;
+                cd.d_wpacked = o.d_wpacked;
                 int32_t sc = 0;
                 st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, L.cws ? base + L.cws_off : nullptr,
                                    L.cws, s);

@@ -377,6 +377,36 @@ __global__ void unpack_codes_kernel(const uint32_t* __restrict__ words, long lon
     }
 }
 
+// Packed weights for the contraction: one warp per 32 codes (kb, o, h), codes W[o][64 kb + 32 h + i]
+// (zero past L and past K); lane i reads code i, lane b < k writes bit plane b to word
+// (((kb * n_ct + o / 256) * k + b) * 256 + o % 256) * 2 + h.
+__global__ void pack_weights_kernel(const __half* __restrict__ w, int K, int L, int K_pad, int k,
+                                    uint32_t* __restrict__ words) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const long long n_kb = (L + 63) / 64;
+    const long long n_rec = n_kb * K_pad * 2;
+    const long long n_ct = K_pad / 256;
+    const uint32_t mask = (1u << k) - 1;
+    for (long long r = warp; r < n_rec; r += nwarps) {
+        const int h = (int)(r & 1);
+        const long long ko = r >> 1;
+        const int o = (int)(ko % K_pad);
+        const long long kb = ko / K_pad;
+        const long long col = kb * 64 + h * 32 + lane;
+        const uint32_t f = (o < K && col < L) ? (uint32_t)__half2int_rn(w[(long long)o * L + col]) & mask : 0u;
+        uint32_t mine = 0;
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            if (b >= k) break;
+            const uint32_t v = __ballot_sync(0xffffffffu, (f >> b) & 1u);
+            if (lane == b) mine = v;
+        }
+        if (lane < k) words[(((kb * n_ct + o / 256) * k + lane) * 256 + o % 256) * 2 + h] = mine;
+    }
+}
+
 }  // namespace
 
 
@@ -574,6 +604,25 @@ extern "C" fxpq_status fxpq_pack_codes(const void* d_codes, int64_t n, fxpq_fmt 
     pack_codes_kernel<<<grid_for((ng + PACK_G - 1) / PACK_G * 32, T), T, 0, as_stream(stream)>>>(
         static_cast<const __half*>(d_codes), n, fmt.bits, planes_of(fmt), d_words);
     return after_launch("pack_codes");
+}
+
+extern "C" size_t fxpq_packed_weights_bytes(fxpq_fmt fmt_w, int32_t K, int32_t L) {
+    if (fmt_w.bits < 1 || fmt_w.bits > 8 || K < 1 || L < 1) return 0;
+    const size_t n_kb = ((size_t)L + 63) / 64, K_pad = ((size_t)K + 255) / 256 * 256;
+    return n_kb * K_pad * 2 * (size_t)fmt_w.bits * 4;
+}
+
+extern "C" fxpq_status fxpq_pack_weights(const void* d_w, fxpq_fmt fmt_w, int32_t K, int32_t L, void* d_packed,
+                                         void* stream) {
+    if (!fmt_ok1(fmt_w) || fmt_w.bits > 8 || K < 1 || L < 1 || !d_w || !d_packed || !aligned(d_packed, 16) ||
+        !aligned(d_w, 2))
+        return FXPQ_ERR_INVALID_ARG;
+    const int K_pad = (K + 255) / 256 * 256;
+    const long long n_rec = ((long long)L + 63) / 64 * K_pad * 2;
+    const int T = 256;
+    pack_weights_kernel<<<grid_for(n_rec * 32, T), T, 0, as_stream(stream)>>>(
+        static_cast<const __half*>(d_w), K, L, K_pad, fmt_w.bits, static_cast<uint32_t*>(d_packed));
+    return after_launch("pack_weights");
 }
 
 extern "C" fxpq_status fxpq_unpack_codes(const uint32_t* d_words, int64_t n, fxpq_fmt fmt, void* d_codes,

@@ -149,6 +149,24 @@ def fxpq_unpack_codes(words, n: int, f: Fmt, codes, stream=None):
     return codes
 
 
+def fxpq_packed_weights_bytes(fw: Fmt, K: int, Lw: int) -> int:
+    return L.lib().fxpq_packed_weights_bytes(fw, K, Lw)
+
+
+def fxpq_pack_weights(w, fw: Fmt, K: int, Lw: int, packed, stream=None):
+    """One plane of fp16 weight codes [K][Lw] (fw.bits <= 8) -> the contraction's packed records."""
+    L.check("fxpq_pack_weights", L.lib().fxpq_pack_weights(_p(w), fw, K, Lw, _p(packed), _s(stream)))
+    return packed
+
+
+def pack_weights(w, fw: Fmt, K: int, Lw: int, stream=None):
+    """Allocates and fills the packed copy of the weights (a uint8 device tensor)."""
+    import torch
+    n = fxpq_packed_weights_bytes(fw, K, Lw)
+    packed = torch.empty(n, dtype=torch.uint8, device=w.device)
+    return fxpq_pack_weights(w, fw, K, Lw, packed, stream)
+
+
 def packed_words(n: int, f: Fmt) -> int:
     return (n + 31) // 32 * f.bits
 
@@ -231,13 +249,14 @@ def fxpq_bn_to_scale(gamma, beta, mean, var, eps, aleph1, aleph2, stream=None):
 
 # ------------------------------------------------------------------------------ C-Blocks
 def conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, out_mode, fx, fw, fb, fy, w_l1=0,
-              scale=None, fmt_scale=None, shift=None, fmt_shift=None) -> L.ConvDesc:
+              scale=None, fmt_scale=None, shift=None, fmt_shift=None, wpacked=None) -> L.ConvDesc:
     """C-Block descriptor.  scale / shift: int32 aleph1 / aleph2 code tensors [K] of a Scale layer (both
-    or neither; the caller keeps them alive while the descriptor is used)."""
+    or neither; the caller keeps them alive while the descriptor is used).  wpacked: optional packed
+    copy of the weights (fxpq_pack_weights)."""
     return L.ConvDesc(N, H, W, C, Cp, K, R, S, stride, pad, int(relu), out_mode, fx, fw,
                       fb if fb is not None else Fmt(32, 1, 0), fy if fy is not None else Fmt(8, 1, 0), int(w_l1),
                       fmt_scale if fmt_scale is not None else Fmt(16, 1, 0),
-                      fmt_shift if fmt_shift is not None else Fmt(16, 1, 0), _p(scale), _p(shift))
+                      fmt_shift if fmt_shift is not None else Fmt(16, 1, 0), _p(scale), _p(shift), _p(wpacked))
 
 
 def fxpq_conv_workspace(desc: L.ConvDesc) -> int:

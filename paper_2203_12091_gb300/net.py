@@ -85,12 +85,18 @@ def search_fmt(x: torch.Tensor, k: int, stream=None) -> L.Fmt:
 class QNet:
     """A quantized network on one device: code tensors, formats, and the fxpq_net op list."""
 
-    def __init__(self, layers, hw=224, cin=3):
+    def __init__(self, layers, hw=224, cin=3, pack_weights=False):
         self.layers = layers
         self.hw, self.cin = hw, cin
         self.cp_in = pad8(cin)
         self.fmts = {}
         self.q = {}  # name -> (weight fp16 codes, bias int32 codes or None)
+        # name -> packed k-bit weights (fxpq_pack_weights) of FC and 1x1 layers with k <= 8, which the
+        # contraction reads instead of the fp16 codes (Sec. V-E.2: k bits per read-only value); built
+        # when pack_weights is set (they halve or better the FC layers' weight reads, while the
+        # in-kernel expansion costs FC time at present)
+        self.qp = {}
+        self.pack_weights = pack_weights
         self.qs = {}  # BN conv name -> (aleph1 int32 codes, aleph2 int32 codes)
         self.w_l1 = {}  # conv name -> max over output channels of sum |weight code| (0: unknown)
         self.names = ["input"] + [L_["name"] for L_ in layers]
@@ -195,6 +201,15 @@ class QNet:
             self.fmts[nm][key] = f
         self.w_l1 = {nm: int.from_bytes(host[off_l1 + 8 * j:off_l1 + 8 * j + 8], "little", signed=True)
                      for j, nm in enumerate(conv_names)}
+        self.qp = {}
+        for i, L_ in enumerate(self.layers):
+            nm = L_["name"]
+            if not self.pack_weights or L_["type"] != "conv" or plan[nm]["w"] > 8:
+                continue
+            H, _, Cp = shapes[self._src(i, L_)]
+            R, st, pad = L_["R"], L_["stride"], L_["pad"]
+            if pad == 0 and ((R == 1 and st == 1) or (R == H and shapes[nm][0] == 1)):
+                self.qp[nm] = F.pack_weights(self.q[nm][0], self.fmts[nm]["w"], L_["K"], R * R * Cp, stream)
         for j, nm in enumerate(avg_names):
             self.q[nm] = (None, int.from_bytes(host[off_rc + 4 * j:off_rc + 4 * j + 4], "little", signed=True))
         self.shapes = shapes
@@ -220,7 +235,8 @@ class QNet:
             sq, hq = self.qs.get(nm, (None, None))
             d = F.conv_desc(N, sH, sW, sCp, sCp, L_["K"], L_["R"], L_["R"], L_["stride"], L_["pad"], L_["relu"],
                             out_mode, fx, self.fmts[nm]["w"], self.fmts[nm].get("b"), fy, self.w_l1.get(nm, 0),
-                            scale=sq, fmt_scale=self.fmts[nm].get("s"), shift=hq, fmt_shift=self.fmts[nm].get("h"))
+                            scale=sq, fmt_scale=self.fmts[nm].get("s"), shift=hq, fmt_shift=self.fmts[nm].get("h"),
+                            wpacked=self.qp.get(nm))
             nws = F.fxpq_conv_workspace(d)
             if nws and (getattr(self, "_cws", None) is None or self._cws.numel() < nws):
                 self._cws = torch.empty(nws, dtype=torch.uint8, device=self._dev)
@@ -283,6 +299,7 @@ class QNet:
                 o.d_w = self.q[nm][0].data_ptr()
                 o.d_bias = self.q[nm][1].data_ptr() if self.q[nm][1] is not None else None
                 o.w_l1 = self.w_l1.get(nm, 0)
+                o.d_wpacked = self.qp[nm].data_ptr() if nm in self.qp else None
                 if nm in self.qs:
                     o.fmt_scale, o.fmt_shift = self.fmts[nm]["s"], self.fmts[nm]["h"]
                     o.d_scale, o.d_shift = self.qs[nm][0].data_ptr(), self.qs[nm][1].data_ptr()
@@ -349,13 +366,14 @@ class QNet:
         return env
 
 
-def build_qnet(layers, weights_np, calib_images, plan, device="cuda", stream=None, bn_np=None):
+def build_qnet(layers, weights_np, calib_images, plan, device="cuda", stream=None, bn_np=None, pack_weights=False):
     """Quantize parameters and calibrate on `calib_images` (fp32 NCHW device tensor).  bn_np: BN conv
-    name -> (gamma, beta, mean, var) fp32 arrays (layers with "bn")."""
+    name -> (gamma, beta, mean, var) fp32 arrays (layers with "bn").  pack_weights: FC layers with
+    k <= 8 read packed k-bit weights."""
     wdev = {nm: (torch.from_numpy(w).to(device), None if b is None else torch.from_numpy(b).to(device))
             for nm, (w, b) in weights_np.items()}
     bn_dev = {nm: tuple(torch.from_numpy(t).to(device) for t in v) for nm, v in (bn_np or {}).items()}
-    q = QNet(layers, hw=calib_images.shape[-1], cin=calib_images.shape[1])
+    q = QNet(layers, hw=calib_images.shape[-1], cin=calib_images.shape[1], pack_weights=pack_weights)
     q._dev = torch.device(device)
     q.quantize_params(wdev, plan, stream, bn_dev)
     q.calibrate(calib_images, plan, stream)

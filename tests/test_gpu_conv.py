@@ -1,5 +1,7 @@
 """GPU parity of the C-Block kernels (conv / FC with the fused epilogue, max-pool, eltwise,
 avg-pool) against the CPU oracle: bit-exact codes, accumulators and fp32 calibration images."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -47,7 +49,9 @@ def to_f16_planes(codes, k, Cp):
     return torch.from_numpy(np.stack([hi, lo]).astype(np.float16)).cuda()
 
 
-def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0, scale=None):
+def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0, scale=None, packed_w=None):
+    """packed_w: one-plane weight codes [K, R, S, C] whose packed records (fxpq_pack_weights) go with the
+    descriptor (normally w itself)."""
     N, H, W, C = x.shape
     K, R, S, _ = w.shape
     P = (H + 2 * pad - R) // stride + 1
@@ -66,8 +70,11 @@ def run_conv(F, x, fx, w, fw, b, fb, stride, pad, relu, mode, fy, Cp, w_l1=0, sc
         m, fs, h, fh = scale
         sd = torch.from_numpy(m.astype(np.int32)).cuda()
         hd = torch.from_numpy(h.astype(np.int32)).cuda()
+    wp = None
+    if packed_w is not None:
+        wp = F.pack_weights(to_f16_planes(packed_w, fw.bits, Cp), fw, K, R * S * Cp)
     d = F.conv_desc(N, H, W, C, Cp, K, R, S, stride, pad, relu, mode, fx, fw, fb, fy, w_l1,
-                    scale=sd, fmt_scale=fs, shift=hd, fmt_shift=fh)
+                    scale=sd, fmt_scale=fs, shift=hd, fmt_shift=fh, wpacked=wp)
     nws = F.fxpq_conv_workspace(d)
     ws = torch.empty(nws, dtype=torch.uint8, device="cuda") if nws else None
     s = F.fxpq_conv_fwd(d, xd, wd, bd, y, ws=ws)
@@ -409,3 +416,80 @@ def test_bounded_wait_runs_out_and_the_context_stays_usable(F):
     run_case(F, CASES[0])
     run_case(F, CASES[16])  # a patch-tile case on the tensor cores
     assert F.fxpq_get_device_status() == 0
+
+
+# ----------------------------------------------------------------------------- packed k-bit weights
+@pytest.mark.parametrize("k,S", [(1, 0), (1, 1), (2, 1), (3, 1), (4, 0), (5, 1), (7, 1), (8, 1), (8, 0)])
+@pytest.mark.parametrize("K,Lw", [(5, 100), (300, 64), (1, 8)])
+def test_pack_weights_layout(F, k, S, K, Lw):
+    """fxpq_pack_weights: the oracle's k-bit packing (Sec. V-E.2) of the codes rearranged as
+    [ceil(L / 64)][K rounded up to 256][64], zero past L and past K, each 256-channel tile's words
+    plane-major."""
+    rng = np.random.default_rng(100 * k + K + Lw + S)
+    c = rand_codes(rng, (K, Lw), k, S)
+    fw = F.fmt(k, S, 3)
+    packed = F.pack_weights(torch.from_numpy(c.astype(np.float16)).cuda(), fw, K, Lw)
+    n_kb, K_pad = (Lw + 63) // 64, (K + 255) // 256 * 256
+    r = np.zeros((n_kb, K_pad, 64), np.int64)
+    for kb in range(n_kb):
+        seg = c[:, 64 * kb:64 * kb + 64]
+        r[kb, :K, :seg.shape[1]] = seg
+    # pack_codes' records (kb, o, h) of k words, then each 256-channel tile's words plane-major
+    want = oracle.pack_codes(r, k).reshape(n_kb, K_pad // 256, 256, 2, k).transpose(0, 1, 4, 2, 3).reshape(-1)
+    assert packed.numel() == F.fxpq_packed_weights_bytes(fw, K, Lw) == want.size * 4
+    assert np.array_equal(packed.cpu().numpy().view(np.uint32), want)
+
+
+PACKED_CASES = [
+    # N, H, C, K, R, (kx,Sx,flx), (kb,flb) or None, relu, mode, (ky,Sy,fly), packed records read: FC layers
+    # (R = H, pad 0) and 1x1 layers; every weight wordlength runs on each
+    (3, 7, 64, 304, 7, (8, 0, 4), (16, 15), True, 0, (8, 0, 3), True),      # FC, ragged K, split reduction
+    (64, 1, 1024, 512, 1, (5, 0, 2), (16, 12), True, 0, (8, 0, 3), True),   # FC at batch 64
+    (2, 9, 64, 272, 1, (8, 0, 4), (16, 15), False, 0, (8, 1, 3), True),     # 1x1, two row tiles, signed out
+    (3, 1, 40, 264, 1, (7, 0, 3), None, True, 2, None, True),               # reduction of 40: a partial k-block
+    (2, 3, 128, 136, 3, (6, 0, 2), (16, 10), False, 1, None, True),         # FC over a 3x3 map, int64 sums out
+    (64, 18, 64, 256, 1, (8, 0, 4), (16, 15), True, 0, (8, 0, 3), False),   # 1x1, enough tiles: fp16 codes read
+]
+# (the C-Block takes weights of 2..16 bits: 1-bit codes exist only as stored tensors)
+PACKED_W = [(2, 1, 2), (2, 0, 1), (3, 1, 3), (4, 1, 5), (4, 0, 4), (5, 1, 6), (6, 1, 7), (7, 1, 8), (8, 1, 9),
+            (8, 0, 8)]
+
+
+@pytest.mark.parametrize("tw", PACKED_W)
+@pytest.mark.parametrize("case", PACKED_CASES)
+def test_conv_packed_weights(F, case, tw):
+    """FC and 1x1 layers with packed k-bit weights (k = 2..8): bit-exact against the oracle and equal to
+    the layer reading fp16 codes.  Then the packed records of a weight tensor with one channel changed go
+    with the original fp16 codes: where the tensor-core path reads the records (layers split across
+    the SMs, on every path but tc_rows and simt) the output follows the changed codes, which shows the
+    kernel consumed them; elsewhere it follows the fp16 codes."""
+    N, H, C, K, R, tx, tb, relu, mode, ty, reads_packed = case
+    rng = np.random.default_rng(H * 7 + K + tw[0] * 31 + tw[1])
+    fx, fw = F.fmt(*tx), F.fmt(*tw)
+    fb = F.fmt(tb[0], 1, tb[1]) if tb else None
+    fy = F.fmt(*ty) if ty else None
+    x = rand_codes(rng, (N, H, H, C), tx[0], tx[1])
+    w = rand_codes(rng, (K, R, R, C), tw[0], tw[1])
+    b = rand_codes(rng, (K,), tb[0], 1) if tb else None
+    Cp = (C + 7) // 8 * 8
+    w_l1 = int(np.abs(w).reshape(K, -1).sum(axis=1).max())
+    want, ws = oracle_conv(x, fx, w, fw, b, fb, 1, 0, relu, mode, fy)
+    got, s = run_conv(F, x, fx, w, fw, b, fb, 1, 0, relu, mode, fy, Cp, w_l1, packed_w=w)
+    assert s == ws
+    assert np.array_equal(got, want)
+    # output channel K-1 set to the largest (else the smallest) code in the packed copy only (the L1
+    # bound passed covers both tensors): its outputs change, and they follow the packed copy wherever
+    # the kernel reads it
+    for code in (oracle.qmax(tw[0], tw[1]), oracle.qmin(tw[0], tw[1])):
+        w2 = w.copy()
+        w2[K - 1] = code
+        want2, _ = oracle_conv(x, fx, w2, fw, b, fb, 1, 0, relu, mode, fy)
+        if not np.array_equal(want2, want):
+            break
+    assert not np.array_equal(want2, want)
+    w_l1_2 = max(w_l1, int(np.abs(w2).reshape(K, -1).sum(axis=1).max()))
+    got2, _ = run_conv(F, x, fx, w, fw, b, fb, 1, 0, relu, mode, fy, Cp, w_l1_2, packed_w=w2)
+    if os.environ.get("FXPQ_CONV_PATH") in ("tc_rows", "simt") or not reads_packed:
+        assert np.array_equal(got2, want)
+    else:
+        assert np.array_equal(got2, want2)

@@ -72,14 +72,16 @@ def test_tiny_residual_net(NET):
         assert np.array_equal(got[..., : oenv[l["name"]][0].shape[-1]], oenv[l["name"]][0]), l["name"]
 
 
-def _workload(NET, arch, batch, seed, plan_seed=None, calib=8, sample=(0, -1)):
+def _workload(NET, arch, batch, seed, plan_seed=None, calib=8, sample=(0, -1), pack=False):
     L = synth.ARCHS[arch]()
     W = synth.weights(arch, seed)
     plan = synth.bit_plan(arch, seed if plan_seed is None else plan_seed)
     bn = synth.bn_params(arch, seed + 100)
     imgs = synth.images(batch, seed)
     dimgs = torch.from_numpy(imgs).cuda()
-    q = NET.build_qnet(L, W, dimgs[:calib], plan, bn_np=bn)
+    q = NET.build_qnet(L, W, dimgs[:calib], plan, bn_np=bn, pack_weights=pack)
+    if pack:
+        assert q.qp, "no layer took packed weights"
     fm, qp = onet.calibrate(L, W, imgs[:calib], plan, bn)
     fmts_equal(q.fmts, fm)
     logits, s = q.forward(dimgs)
@@ -96,6 +98,12 @@ def _workload(NET, arch, batch, seed, plan_seed=None, calib=8, sample=(0, -1)):
 
 def test_alexnet_batch256(NET):
     _workload(NET, "alexnet", 256, 5)
+
+
+def test_alexnet_batch256_packed_fc_weights(NET):
+    """The same workload with its three FC layers' 8-bit weights read as packed 8-bit planes
+    (Sec. V-E.2) by the contraction, calibration included: formats and logits equal the oracle's."""
+    _workload(NET, "alexnet", 256, 5, pack=True)
 
 
 def test_resnet18_batch128(NET):
@@ -130,6 +138,12 @@ def test_bn_to_scale_bit_exact(NET):
 @pytest.mark.parametrize("plan_seed", [7, 38])
 def test_vgg16_batch64_plans(NET, plan_seed):
     _workload(NET, "vgg16", 64, 7, plan_seed=plan_seed, sample=(0,))
+
+
+def test_vgg16_batch64_packed_fc_weights(NET):
+    """VGG-16 with fc6 / fc7 reading packed weights (4..8 bits per the plan; fc8's are 16-bit and stay
+    fp16 code planes)."""
+    _workload(NET, "vgg16", 64, 7, plan_seed=7, sample=(0,), pack=True)
 
 
 def test_single_conv_workload_end_to_end(NET):
