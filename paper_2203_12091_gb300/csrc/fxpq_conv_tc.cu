@@ -17,7 +17,8 @@ std::mutex g_tc_mu;
 // "tc_rows" keeps every layer on 128-row tiles gathered by the producer warps, "tc_patch" takes patch tiles wherever the geometry
 // allows them (by default only while they compute few extra rows), "tc_bn128" never takes
 // 256-column tiles and "tc_bn256" takes them wherever the layer allows (by default they also need
-// enough tiles to keep every SM busy).
+// enough tiles to keep every SM busy), "tc_win64" keeps window mode's two-limb epilogue in 64-bit
+// arithmetic.
 bool conv_path_is(const char* name) {
     const char* e = getenv("FXPQ_CONV_PATH");
     return e && strcmp(e, name) == 0;
@@ -164,6 +165,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             return FXPQ_OK;
         P.patch = 0;
         P.rows_tma = 0;
+        P.w32 = 0;
         P.nacc = 1;
         // window mode for 8-channel stride-1 layers with at most 64 output channels: 8 x 16 output
         // patches, one input window per tile and limb plane, weights resident in shared memory, one
@@ -189,7 +191,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 const cuuint64_t wdims[5] = {8, (cuuint64_t)a.K, (cuuint64_t)a.S, (cuuint64_t)a.R, (cuuint64_t)a.pw};
                 const cuuint64_t wstrides[4] = {(cuuint64_t)a.R * a.S * 16, 16, (cuuint64_t)a.S * 16,
                                                 (cuuint64_t)a.w_ps * 2};
-                const cuuint32_t wbox[5] = {8, 64, 2, 1, 1};
+                const cuuint32_t wbox[5] = {8, 64, 1, 1, 1};  // one tap of one plane
                 const cuuint32_t es5[5] = {1, 1, 1, 1, 1};
                 CUtensorMap mx, mw;
                 if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<__half*>(a.x), xdims, xstrides, xbox, es5,
@@ -215,6 +217,23 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                     P.nbuf = 2;
                     BN = 64;
                     acc64 = true;  // the int64 instance: its TMEM holds two buffers of the limb accumulators
+                    // 32-bit epilogue of two-limb x and w (v = 2^16 T + Lo, see the kernel): every limb
+                    // sum covers R * S2 * 8 products; L = 2^8 (S_hl + S_lh) + S_ll + Lo(B') and T must stay
+                    // below 2^31, the aligned bias must not be finer than the sums (delta >= 0), and
+                    // sh - 16 in [0, 30]; the per-channel bias table takes the last 512 bytes of the B region
+                    if (a.px == 2 && a.pw == 2 && !a.has_scale && a.delta >= 0 && a.out_mode == FXPQ_OUT_CODES &&
+                        a.py == 1 && a.sh >= 16 && a.sh <= 46 &&
+                        a.pw * a.R * (S2 / 2) * 64 * 32 + 512 <= tc_stages(64) * 64 * TC_BK * 2) {
+                        const double taps = (double)a.R * S2 * 8;
+                        const double hh = (double)limb_max(d.fmt_x, 0) * limb_max(d.fmt_w, 0) * taps;
+                        const double hl = (double)limb_max(d.fmt_x, 0) * limb_max(d.fmt_w, 1) * taps;
+                        const double lh = (double)limb_max(d.fmt_x, 1) * limb_max(d.fmt_w, 0) * taps;
+                        const double ll = (double)limb_max(d.fmt_x, 1) * limb_max(d.fmt_w, 1) * taps;
+                        const double bb = a.has_bias ? ldexp(1.0, d.fmt_b.bits - d.fmt_b.is_signed + a.delta) : 0.0;
+                        const double Lb = 256.0 * (hl + lh) + ll + 65536.0;
+                        const double Tb = hh + bb / 65536.0 + 1.0 + Lb / 65536.0 + 1.0;
+                        P.w32 = Lb < ldexp(1.0, 31) && Tb < ldexp(1.0, 31) && !conv_path_is("tc_win64");
+                    }
                 }
             }
         }
@@ -265,6 +284,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             }
         }
         if (!P.rows_tma) P.pk = 0;
+        if (P.w32 && !(a.out_mode == FXPQ_OUT_CODES && a.py == 1)) P.w32 = 0;
         // one-plane codes: stage the tile in shared memory and write it with TMA stores (not with packed
         // weights, whose staging region holds the packed stages)
         P.fast_store = 0;
@@ -289,6 +309,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
             }
             P.fast_store = r == CUDA_SUCCESS;
         }
+        if (!P.fast_store) P.w32 = 0;  // the 32-bit window epilogue writes through the staging tile
     }
     P.tiles_m = P.patch ? a.N * P.tiles_p * P.tiles_q : (int)((a.M + TC_BM - 1) / TC_BM);
     P.tiles_n = (a.K + BN - 1) / BN;
@@ -362,7 +383,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true, true>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<256, int, false, false, true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess)
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<64, long long, false, false, false, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)(tc_smem_bytes<64>() + 64 * TC_BM * 2)) != cudaSuccess)
                 return FXPQ_ERR_CUDA;
             g_tc_attr_set = true;
         }
@@ -370,7 +394,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     const int grid = P.n_units < sms ? P.n_units : sms;
     launched = true;
     if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);  // never split
-    if (P.pk && P.ksplit > 1)
+    if (P.patch == 3 && P.w32)  // window mode, 32-bit two-limb epilogue: its own instance (never split)
+        conv_tc_kernel<64, long long, false, false, false, true>
+            <<<grid, tc_threads_win(), tc_smem_bytes<64>() + 64 * TC_BM * 2, st>>>(P);
+    else if (P.pk && P.ksplit > 1)
         conv_tc_kernel<256, int, false, true, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
     else if (P.pk)
         conv_tc_kernel<256, int, false, false, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);

@@ -60,6 +60,10 @@ __host__ __device__ constexpr int tc_threads(int BN) { return (5 + tc_epi_warps(
 constexpr int TC_PK_WARPS = 5;
 constexpr int TC_PK_CONVERTERS = 3 + TC_PK_WARPS;  // converter warps
 __host__ __device__ constexpr int tc_threads_pk(int BN, bool pk) { return tc_threads(BN) + (pk ? 32 * TC_PK_WARPS : 0); }
+// Window-mode instance (WIN, BN = 64, two-limb x and w, 32-bit epilogue): 16 epilogue warps of 16 columns
+// each and two output staging tiles.
+constexpr int TC_WIN_EPI_WARPS = 16;
+__host__ __device__ constexpr int tc_threads_win() { return (5 + TC_WIN_EPI_WARPS) * 32; }
 // Dynamic shared memory: barriers, the stages (A and B tiles), the output staging tile.
 template <int BN>
 constexpr size_t tc_smem_bytes() {
@@ -99,6 +103,8 @@ struct TcParams {
                          // swizzle, rows past M and taps past R*S*Cp zero filled
     int nacc;            // fp32 accumulators per TMEM buffer (window mode: one per limb pair)
     int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
+    int w32;             // window mode, two-limb x and w, one-plane codes out: the 32-bit epilogue (the
+                         // host proved its bounds; see the epilogue), with m = sh - 16 in [0, 30]
     int win_bytes;       // window mode: bytes of one window (128-byte aligned)
     int TH, TW;          // patch shape (TH * TW = 128)
     int tiles_p, tiles_q;  // patches per image along P and Q
@@ -161,6 +167,7 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int 
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 __device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, int x, int y, int z, int w, uint32_t src) {
@@ -558,8 +565,11 @@ __device__ __forceinline__ void pk_convert_loop(const TcParams& P, int cid, int 
 // the unit loop is the tile loop and every tile takes all P.n_groups groups.
 // PK: the instantiation that reads packed k-bit weights (P.pk = 1; BN = 256, TMA A tiles, no output
 // staging): one thread issues every copy and TC_PK_CONVERTERS warps expand the weights.
-template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false>
-__global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const __grid_constant__ TcParams P) {
+// WIN: the window-mode instance of the 32-bit two-limb epilogue (P.patch == 3, P.w32): 16 epilogue warps and
+// two staging tiles; only window mode's roles are compiled into it.
+template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false, bool WIN = false>
+__global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK), 1)
+    conv_tc_kernel(const __grid_constant__ TcParams P) {
     constexpr int TC_STAGES = tc_stages(BN);
     constexpr int TC_LAG = tc_lag(BN);
     static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
@@ -569,10 +579,11 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
     constexpr int TC_PRODUCERS = PK ? 1 : tc_producers(BN);
     static_assert(TC_STAGES % TC_PRODUCERS == 0 && TC_PRODUCERS <= 4,
                   "each stage must have one producer thread among warps 0..3");
-    constexpr int EPI_WARPS = tc_epi_warps(BN);
+    static_assert(!WIN || (BN == 64 && sizeof(ACC) == 8 && !SC && !SPLIT && !PK), "window instance: BN = 64, int64");
+    constexpr int EPI_WARPS = WIN ? TC_WIN_EPI_WARPS : tc_epi_warps(BN);
     constexpr int EPI_THREADS = 32 * EPI_WARPS;
     constexpr int MMA_WARP = 4 + EPI_WARPS;
-    constexpr int CPW = (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
+    constexpr int CPW = WIN ? 1 : (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
     constexpr int B_BYTES = BN * TC_BK * 2;
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
@@ -586,7 +597,7 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
     unsigned char* sA = base;
     unsigned char* sB = base + TC_STAGES * A_BYTES;
     unsigned char* sO = sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of [128 rows][64 codes]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2 * (WIN ? 2 : 1));  // WIN: two staging tiles
     // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
     volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
@@ -596,6 +607,8 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
     const uint32_t stg_full = smem_u32(bars + 2 * TC_STAGES + 7);  // staging written by every epilogue warp
     const uint32_t stg_free = smem_u32(bars + 2 * TC_STAGES + 8);  // staging read by the previous TMA store
     const uint32_t wbar = smem_u32(bars + 2 * TC_STAGES + 9);      // window mode: resident weights loaded
+    const uint32_t stg_full2 = smem_u32(bars + 2 * TC_STAGES + 10);  // WIN: the second staging tile
+    const uint32_t stg_free2 = smem_u32(bars + 2 * TC_STAGES + 11);
     // PK: pkfull[s] completes when stage s's A box and packed weight records have landed; the
     // converters then fill the B stage and arrive on full[s]
     const uint32_t pkfull0 = smem_u32(bars + 2 * TC_STAGES + 10);
@@ -619,6 +632,10 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
         mbar_init(done_bar, 1);
         mbar_init(stg_full, EPI_WARPS);
         mbar_init(stg_free, 1);
+        if (WIN) {
+            mbar_init(stg_full2, EPI_WARPS);
+            mbar_init(stg_free2, 1);
+        }
         mbar_init(wbar, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -628,6 +645,15 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
                      "r"(TMEM_COLS));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
+    // window mode, 32-bit epilogue: per output channel the aligned bias B' = b 2^delta split as
+    // (B' >> 16, B' & 0xFFFF), in the last 512 bytes of the B region (the resident weights stay below)
+    int2* wtab = reinterpret_cast<int2*>(sB + TC_STAGES * B_BYTES - 512);
+    if (BN == 64 && sizeof(ACC) == 8 && !SC && P.patch == 3 && P.w32 && warp == 1) {
+        for (int k = lane; k < 64; k += 32) {
+            const long long bb = (a.has_bias && k < a.K) ? ((long long)__ldg(a.bias + k) << (a.delta > 0 ? a.delta : 0)) : 0;
+            wtab[k] = make_int2((int)(bb >> 16), (int)(bb & 0xFFFF));
+        }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -635,18 +661,21 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
 
     if (warp < 4 && P.patch == 3) {
         // ============================================================ producer, window mode
-        // Stride 1, Cp == 8: the weights (per limb plane, kernel row r and tap pair sp, the box
-        // {8 ch, BN out ch, 2 taps}) are loaded once into the B region; per tile, one box per x limb
-        // plane holds the input window of TH + R - 1 rows by TW + S2 - 1 pixels (padding zero filled).
+        // Stride 1, Cp == 8: the weights are loaded once into the B region, per kernel row r and tap
+        // pair sp a block of the two taps, each tap the BN output channels of every limb plane in turn
+        // (rows [W_hi | W_lo] of one B operand of N = pw BN: one MMA forms both limb sums of an x limb;
+        // one box {8 ch, BN out ch} per tap and plane, taps past S zero filled); per tile, one box per
+        // x limb plane holds the input window of TH + R - 1 rows by TW + S2 - 1 pixels (padding zero
+        // filled).
         if (threadIdx.x == 0) {
             const int np = P.S2 / 2;
-            const uint32_t wbox = (uint32_t)(BN * 32);
-            mbar_arrive_expect_tx(wbar, (uint32_t)(a.pw * a.R * np) * wbox);
-            for (int iw = 0; iw < a.pw; ++iw)
-                for (int r = 0; r < a.R; ++r)
-                    for (int sp = 0; sp < np; ++sp)
-                        tma_load_5d(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox, &P.tmap_w, 0, 0, 2 * sp,
-                                    r, iw, wbar);
+            const uint32_t tapb = (uint32_t)(BN * 16);  // one tap of one plane
+            mbar_arrive_expect_tx(wbar, (uint32_t)(a.pw * a.R * np * 2) * tapb);
+            for (int r = 0; r < a.R; ++r)
+                for (int t = 0; t < 2 * np; ++t)
+                    for (int iw = 0; iw < a.pw; ++iw)
+                        tma_load_5d(smem_u32(sB) + (uint32_t)(((r * np + t / 2) * 2 + (t & 1)) * a.pw + iw) * tapb,
+                                    &P.tmap_w, 0, 0, t, r, iw, wbar);
             const uint32_t win_tx = (uint32_t)(P.WW * P.WH * 16);
             const int per_img = P.tiles_p * P.tiles_q;
             uint32_t it = 0, stage = 0, phase = 0;
@@ -685,7 +714,7 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
             while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
             }
         }
-    } else if (warp < 4 && (P.patch || P.rows_tma)) {
+    } else if (!WIN && warp < 4 && (P.patch || P.rows_tma)) {
         // ============================================================ producer, patch tiles
         // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
         // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
@@ -772,7 +801,7 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
             }
         }
         if (PK && warp >= 1) pk_convert_loop<BN, SPLIT>(P, warp - 1, lane, sP, sB, pkfull0, full0, abort);
-    } else if (warp < 4) {
+    } else if (!WIN && warp < 4) {
         // ============================================================ producers, row tiles
         // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
         // threads cover one 128-byte row, so every warp instruction reads four whole rows.
@@ -858,6 +887,103 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
                 }
             }
         }
+    } else if (WIN && warp < MMA_WARP) {
+        // ============================================================ epilogue, window instance
+        // Warp w drains TMEM lanes 32 (w % 4) .. + 31 and the 16 columns 16 cw .., cw = (w - 4) / 4, of the
+        // four limb accumulators, with the 32-bit arithmetic of the generic window epilogue below; tile u
+        // goes through staging tile u % 2, whose previous store must have read it (at most the other
+        // tile's store is then in flight).
+        const int quad = warp & 3, cw = (warp - 4) >> 2;
+        const int row = quad * 32 + lane;
+        const bool leader = threadIdx.x == 128;  // waits for and issues the TMA stores
+        const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
+        const int m = a.sh - 16;
+        const int half = m > 0 ? 1 << (m - 1) : 0;
+        const int mmask = (int)((1u << m) - 1u);
+        const int lo = (int)a.lo, hi = (int)a.hi;
+        const int per_img = P.tiles_p * P.tiles_q;
+        bool ok = true;
+        uint32_t u = 0;
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x, ++u) {
+            const uint32_t buf = u & 1;
+            if (!wait_bounded(accfull0 + 8 * buf, (u >> 1) & 1, abort, P.status)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t fhh[16], fhl[16], flh[16], fll[16];
+            const uint32_t abase = lane_base + buf * (uint32_t)(4 * BN) + (uint32_t)(cw * 16);
+            tmem_ld16_nw(abase, fhh);
+            tmem_ld16_nw(abase + (uint32_t)BN, fhl);
+            tmem_ld16_nw(abase + (uint32_t)(2 * BN), flh);
+            tmem_ld16_nw(abase + (uint32_t)(3 * BN), fll);
+            tmem_wait_ld();
+            reg_fence(fhh);
+            reg_fence(fhl);
+            reg_fence(flh);
+            reg_fence(fll);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
+            uint32_t w[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                int c2[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int jj = 2 * j + h;
+                    const int2 bt = wtab[cw * 16 + jj];
+                    const int mid = __float2int_rn(__uint_as_float(fhl[jj])) + __float2int_rn(__uint_as_float(flh[jj]));
+                    const int L = mid * 256 + __float2int_rn(__uint_as_float(fll[jj])) + bt.y;
+                    const int T = __float2int_rn(__uint_as_float(fhh[jj])) + bt.x + (L >> 16);
+                    const int Lo = L & 0xFFFF;
+                    int q, up;
+                    if (m > 0) {
+                        q = T >> m;
+                        const int rem = T & mmask;
+                        up = (rem > half) | ((rem == half) & ((Lo != 0) | (q & 1)));
+                    } else {
+                        q = T;
+                        up = (Lo > 0x8000) | ((Lo == 0x8000) & (q & 1));
+                    }
+                    const int cc = (a.relu && T < 0) ? 0 : q + up;
+                    c2[h] = min(max(cc, lo), hi);
+                }
+                w[j] = pack_codes_f16(c2[0], c2[1]);
+            }
+            const uint32_t sb = u & 1, n = u >> 1;  // staging tile and its use count
+            const uint32_t sfull = sb ? stg_full2 : stg_full, sfree = sb ? stg_free2 : stg_free;
+            if (n > 0) {
+                if (leader) {
+                    bulk_wait_read1();  // the store of tile u - 2 (this staging tile) has read it
+                    mbar_arrive(sfree);
+                }
+                if (!wait_bounded(sfree, (n - 1) & 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+            }
+            unsigned char* sbuf = sO + sb * (TC_BM * 128);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int chunk = cw * 2 + q;
+                *reinterpret_cast<uint4*>(sbuf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                    make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+            }
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(sfull);
+            if (leader) {
+                if (!wait_bounded(sfull, n & 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+                const int n_img = t / per_img, r = t - n_img * per_img;
+                tma_store_4d(&P.tmap_y, 0, (r % P.tiles_q) * P.TW, (r / P.tiles_q) * P.TH, n_img, smem_u32(sbuf));
+                bulk_commit();
+            }
+        }
+        if (leader) bulk_wait0();  // every output store has completed
     } else if (warp < MMA_WARP) {
         // ============================================================ epilogue
         // Warp w drains TMEM lanes 32 (w % 4) .. 32 (w % 4) + 31 (the quadrant a warp may access) and
@@ -906,6 +1032,74 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
                     const int cb = cw * CPW + c;
                     const int k0 = tn * BN + cb * 32;
                     const uint32_t run_col = run_base + cb * 32;
+                    if (BN == 64 && sizeof(ACC) == 8 && !SC && P.patch == 3 && P.w32) {
+                        // window mode, two-limb x and w, 32-bit arithmetic.  With the limb sums S_hh,
+                        // S_mid = S_hl + S_lh, S_ll and the aligned bias B' = 2^16 Bh + Bl (0 <= Bl < 2^16):
+                        //   v = 2^16 S_hh + 2^8 S_mid + S_ll + B' = 2^16 T + Lo,
+                        //   L = 2^8 S_mid + S_ll + Bl,  T = S_hh + Bh + (L >> 16),  Lo = L & 0xFFFF,
+                        // (the host keeps |L| and |T| below 2^31).  With sh = 16 + m, floor(v / 2^sh) =
+                        // T >> m and the remainder is 2^16 (T mod 2^m) + Lo, so round half to even needs
+                        // T mod 2^m against 2^(m-1), and Lo only to tell a tie (Lo = 0) from above it.
+                        // ReLU: v < 0 exactly when T < 0.
+                        const int m = a.sh - 16;
+                        const int half = m > 0 ? 1 << (m - 1) : 0;
+                        const int mmask = (int)((1u << m) - 1u);
+                        const int lo = (int)a.lo, hi = (int)a.hi;
+                        const uint32_t abase = lane_base + buf * (uint32_t)(4 * BN) + cb * 32;
+                        uint32_t w[16];
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf) {
+                            uint32_t fhh[16], fhl[16], flh[16], fll[16];
+                            tmem_ld16_nw(abase + 16 * hf, fhh);
+                            tmem_ld16_nw(abase + (uint32_t)BN + 16 * hf, fhl);
+                            tmem_ld16_nw(abase + (uint32_t)(2 * BN) + 16 * hf, flh);
+                            tmem_ld16_nw(abase + (uint32_t)(3 * BN) + 16 * hf, fll);
+                            tmem_wait_ld();
+                            reg_fence(fhh);
+                            reg_fence(fhl);
+                            reg_fence(flh);
+                            reg_fence(fll);
+                            if (hf == 1 && c == CPW - 1) {
+                                tc_fence_before();
+                                __syncwarp();
+                                if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
+                            }
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) {
+                                int c2[2];
+#pragma unroll
+                                for (int h = 0; h < 2; ++h) {
+                                    const int jj = 2 * j + h;
+                                    const int2 bt = wtab[cb * 32 + 16 * hf + jj];
+                                    const int mid = __float2int_rn(__uint_as_float(fhl[jj])) +
+                                                    __float2int_rn(__uint_as_float(flh[jj]));
+                                    const int L = mid * 256 + __float2int_rn(__uint_as_float(fll[jj])) + bt.y;
+                                    const int T = __float2int_rn(__uint_as_float(fhh[jj])) + bt.x + (L >> 16);
+                                    const int Lo = L & 0xFFFF;
+                                    int q, up;
+                                    if (m > 0) {
+                                        q = T >> m;
+                                        const int rem = T & mmask;
+                                        up = (rem > half) | ((rem == half) & ((Lo != 0) | (q & 1)));
+                                    } else {
+                                        q = T;
+                                        up = (Lo > 0x8000) | ((Lo == 0x8000) & (q & 1));
+                                    }
+                                    int cc = (a.relu && T < 0) ? 0 : q + up;
+                                    c2[h] = min(max(cc, lo), hi);
+                                }
+                                w[8 * hf + j] = pack_codes_f16(c2[0], c2[1]);
+                            }
+                        }
+                        unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int chunk = (cb & 1) * 4 + q;
+                            *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
+                                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                        }
+                        continue;
+                    }
                     if (sizeof(ACC) == 8 && P.patch == 3 && P.nacc == 4 && P.fast_store && a.sh >= 1 && a.sh <= 62) {
                         // window mode, two-limb x and w, one-plane codes out: each 16-column half goes
                         // from the four limb accumulators to packed codes before the next is loaded
@@ -1178,7 +1372,18 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
         // without swizzle, the two K core matrices one pixel (16 bytes) apart, the 8-row groups (the
         // patch rows, TW = 8) one window row apart.  B is the resident box (iw, r, sp).
         const int np = P.S2 / 2;
-        const uint32_t wbox = (uint32_t)(BN * 32);
+        const uint32_t tapb = (uint32_t)(BN * 16);
+        // N = pw BN: the B operand of tap pair (r, sp) holds [W_hi | W_lo] (one plane: N = BN); its K
+        // core matrices (the two taps) are pw BN 16 bytes apart, its 8-row groups 128 bytes apart
+        const uint32_t idesc_w = a.pw == 2 ? make_idesc(TC_BM, 2 * BN) : IDESC;
+        uint64_t bdesc[8];
+        uint32_t aoff[8];  // A start of tap pair (r, sp) in the window, in 16-byte units
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int r = i / np, sp = i - r * np;
+            bdesc[i] = make_sdesc_noswz(smem_u32(sB) + (uint32_t)(i * 2 * a.pw) * tapb, (uint32_t)a.pw * tapb, 128);
+            aoff[i] = (uint32_t)((r * P.WW + 2 * sp) * 16) >> 4;
+        }
         uint32_t stage = 0, phase = 0, gcount = 0;
         bool ok = wait_bounded(wbar, 0, abort, P.status);
         tc_fence_after();
@@ -1194,21 +1399,15 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
             tc_fence_after();
             const uint32_t d0 = tmem + buf * (uint32_t)(P.nacc * BN);
             const uint32_t wa = smem_u32(sA + stage * A_BYTES);
-            for (int ia = 0; ia < a.px; ++ia)
-                for (int iw = 0; iw < a.pw; ++iw) {
-                    const uint32_t d = d0 + (uint32_t)((ia * a.pw + iw) * BN);
-                    uint32_t accum = 0;
-                    for (int r = 0; r < a.R; ++r)
-                        for (int sp = 0; sp < np; ++sp) {
-                            const uint64_t ad = make_sdesc_noswz(
-                                wa + (uint32_t)(ia * P.win_bytes + (r * P.WW + 2 * sp) * 16), 16, (uint32_t)(P.WW * 16));
-                            const uint64_t bd =
-                                make_sdesc_noswz(smem_u32(sB) + (uint32_t)((iw * a.R + r) * np + sp) * wbox,
-                                                 (uint32_t)(BN * 16), 128);
-                            tc_mma(d, ad, bd, IDESC, accum);
-                            accum = 1;
-                        }
-                }
+            for (int ia = 0; ia < a.px; ++ia) {
+                // accumulators (ia, iw) at columns (ia pw + iw) BN: one MMA of N = pw BN fills the pw of them
+                const uint32_t d = d0 + (uint32_t)(ia * a.pw * BN);
+                const uint64_t ad0 = make_sdesc_noswz(wa + (uint32_t)(ia * P.win_bytes), 16, (uint32_t)(P.WW * 16));
+                const int nt = a.R * np;  // <= 8
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    if (i < nt) tc_mma(d, ad0 + (uint64_t)aoff[i], bdesc[i], idesc_w, i > 0 ? 1u : 0u);
+            }
             tc_commit(empty0 + 8 * stage);
             if (++stage == TC_STAGES) {
                 stage = 0;
@@ -1222,7 +1421,7 @@ __global__ void __launch_bounds__(tc_threads_pk(BN, PK), 1) conv_tc_kernel(const
         const long long t0 = clock64();
         while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
         }
-    } else if (lane == 0) {
+    } else if (!WIN && lane == 0) {
         // ============================================================ MMA issue (one thread of MMA_WARP)
         // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
         // (address >> 4, 14 bits) without carry since shared addresses stay below 256 KB.

@@ -162,6 +162,10 @@ CASES = [
     (2, 20, 3, 48, 3, 1, 1, (16, 1, 9), (16, 1, 12), (16, 18), False, 0, (6, 1, 2)),
     (1, 18, 3, 64, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 17), True, 0, (8, 0, 2)),
     (2, 20, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 13), (16, 30), False, 0, (8, 1, 3)),
+    # the 32-bit window epilogue at its smallest shift (16: the tie is decided by the low 16 bits alone),
+    # and one below it (15: the 64-bit path)
+    (1, 16, 3, 32, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 15), False, 0, (8, 1, 3)),
+    (1, 16, 3, 32, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 15), True, 0, (8, 1, 4)),
 ]
 
 
@@ -193,6 +197,23 @@ def test_conv_parity_l1_bound(F, case):
 @pytest.mark.parametrize("case", CASES)
 def test_conv_parity(F, case):
     run_case(F, case)
+
+
+WINDOW_TWO_LIMB = [c for c in CASES if c[2] <= 8 and c[3] <= 64 and c[5] == 1 and c[7][0] > 8 and c[8][0] > 8]
+
+
+@pytest.mark.parametrize("alt", ["tc_win64"])
+@pytest.mark.parametrize("case", WINDOW_TWO_LIMB)
+def test_window_epilogue_alternatives(F, case, alt):
+    """Window mode's two-limb epilogue in its 64-bit form on the same cases as the default (32-bit
+    where the bounds allow)."""
+    if os.environ.get("FXPQ_CONV_PATH") != "tc":
+        pytest.skip("alternative forms of the default tensor-core path")
+    os.environ["FXPQ_CONV_PATH"] = alt
+    try:
+        run_case(F, case)
+    finally:
+        os.environ["FXPQ_CONV_PATH"] = "tc"
 
 
 def test_code_l1max(F):
