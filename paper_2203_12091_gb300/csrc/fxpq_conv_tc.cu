@@ -237,6 +237,42 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                 }
             }
         }
+        // 64-channel window mode (W64 instance) for one-plane stride-1 layers with at most 64 output
+        // channels, kernels up to 3 x 3, a reduction of one exact group and one-plane codes out (VGG
+        // conv1_2): 8 x 16 output patches, the weights resident (one 8 KiB swizzled block per tap), then
+        // two window slots of S copies (shifted by 0 .. S - 1 pixels) of TH + R - 1 rows of 8 pixels
+        if (P.patch == 0 && BN == 64 && a.K <= 64 && !acc64 && a.stride == 1 && a.Cp == 64 && a.px == 1 &&
+            a.pw == 1 && P.n_groups == 1 && a.N > 0 && a.P > 0 && a.Q > 0 && a.R <= 3 && a.S <= 3 &&
+            a.out_mode == FXPQ_OUT_CODES && a.py == 1 && (a.v32 || (a.sh >= 1 && a.sh <= 62)) && !a.has_scale &&
+            !conv_path_is("tc_rows") && !conv_path_is("tc_patch") && !conv_path_is("tc_nowin")) {
+            const int WH = 16 + a.R - 1;
+            const long long slot = (long long)a.S * WH * 1024;
+            const long long wb = (long long)a.R * a.S * 8192;
+            if (wb + 2 * slot <= TC_W64_SO) {
+                const cuuint64_t xdims[4] = {(cuuint64_t)a.Cp, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N};
+                const cuuint64_t xstrides[3] = {(cuuint64_t)a.Cp * 2, (cuuint64_t)a.W * a.Cp * 2,
+                                                (cuuint64_t)a.H * a.W * a.Cp * 2};
+                const cuuint32_t xbox[4] = {64, 8, (cuuint32_t)WH, 1};
+                const cuuint32_t es4[4] = {1, 1, 1, 1};
+                CUtensorMap mx;
+                if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<__half*>(a.x), xdims, xstrides, xbox, es4,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS) {
+                    P.tmap_x = mx;  // the weights keep the tiled map above (box {64, 64}: one tap)
+                    P.patch = 4;
+                    P.TW = 8;
+                    P.TH = 16;
+                    P.tiles_p = (a.P + 15) / 16;
+                    P.tiles_q = (a.Q + 7) / 8;
+                    P.WW = 8;
+                    P.WH = WH;
+                    P.win_bytes = (int)slot;
+                    P.w64_slot0 = (int)wb;
+                    P.w64_slot_stride = (int)slot;
+                    P.nbuf = 2;
+                }
+            }
+        }
         if (P.patch == 0 && rows_geom) {
             const cuuint64_t xdims[3] = {(cuuint64_t)P.RSC, (cuuint64_t)a.M, (cuuint64_t)a.px};
             const cuuint64_t xstrides[2] = {(cuuint64_t)P.RSC * 2, (cuuint64_t)a.x_ps * 2};
@@ -327,7 +363,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     P.gs[1] = P.n_groups;
     // (64-column tiles, and 256-column TMA-row tiles, without a Scale layer: the instantiations that carry
     // the split)
-    if (P.patch != 3 && (BN == 64 || (BN == 256 && P.rows_tma && !acc64)) && !a.has_scale && ws &&
+    if (P.patch != 3 && P.patch != 4 && (BN == 64 || (BN == 256 && P.rows_tma && !acc64)) && !a.has_scale && ws &&
         P.n_tiles * 2 <= sms && !conv_path_is("tc_nosplit")) {
         const int ng = P.n_groups;
         int min_len = 1 << 30;
@@ -386,7 +422,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<64, long long, false, false, false, true>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)(tc_smem_bytes<64>() + 64 * TC_BM * 2)) != cudaSuccess)
+                                     (int)(tc_smem_bytes<64>() + 64 * TC_BM * 2)) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<64, int, false, false, false, false, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_w64()) != cudaSuccess)
                 return FXPQ_ERR_CUDA;
             g_tc_attr_set = true;
         }
@@ -397,6 +435,13 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     if (P.patch == 3 && P.w32)  // window mode, 32-bit two-limb epilogue: its own instance (never split)
         conv_tc_kernel<64, long long, false, false, false, true>
             <<<grid, tc_threads_win(), tc_smem_bytes<64>() + 64 * TC_BM * 2, st>>>(P);
+    else if (P.patch == 4 && P.fast_store)
+        // 64-channel window mode: the instance with its own shared-memory layout and 16 epilogue warps
+        conv_tc_kernel<64, int, false, false, false, false, true><<<grid, tc_threads_win(), tc_smem_w64(), st>>>(P);
+    else if (P.patch == 4) {
+        launched = false;  // no TMA store of the output: the CUDA-core kernel runs instead
+        return FXPQ_OK;
+    }
     else if (P.pk && P.ksplit > 1)
         conv_tc_kernel<256, int, false, true, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
     else if (P.pk)

@@ -63,6 +63,11 @@ __host__ __device__ constexpr int tc_threads_pk(int BN, bool pk) { return tc_thr
 // Window-mode instance (WIN, BN = 64, two-limb x and w, 32-bit epilogue): 16 epilogue warps of 16 columns
 // each and two output staging tiles.
 constexpr int TC_WIN_EPI_WARPS = 16;
+// W64 instance (64-channel window mode) shared memory: resident weights (up to 9 taps of 8 KiB) and two
+// window slots of up to 3 copies of 18 rows x 8 pixels x 128 bytes from the start, the two staging tiles
+// at W64_SO.
+constexpr int TC_W64_SO = 180 * 1024;
+constexpr size_t tc_smem_w64() { return 1024 + TC_W64_SO + 2 * 64 * TC_BM * 2 + 256; }
 __host__ __device__ constexpr int tc_threads_win() { return (5 + TC_WIN_EPI_WARPS) * 32; }
 // Dynamic shared memory: barriers, the stages (A and B tiles), the output staging tile.
 template <int BN>
@@ -97,6 +102,9 @@ struct TcParams {
                          // 2: Cp == 8 (one 8-channel box per tap, 8 taps per k-block, no swizzle);
                          // 3: Cp == 8, window mode (one input window per tile and limb plane, taps as
                          //    shifted descriptors, weights resident in shared memory)
+                         // 4: Cp == 64, window mode of one-plane layers (W64 instance): the 8 x 16 patch's
+                         //    input window, one 128-byte-swizzled TMA box per tile, weights resident,
+                         //    every tap and 16-channel step one shifted swizzled MMA
     int rows_tma;        // 128-row tiles whose A tile is one 2-D TMA box of the activations seen as
                          // [planes][M][R*S*Cp] (1x1 stride-1 layers without padding, and kernels that
                          // cover the whole unpadded map: FC layers), box {64, 128, 1}, 128-byte
@@ -105,7 +113,9 @@ struct TcParams {
     int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
     int w32;             // window mode, two-limb x and w, one-plane codes out: the 32-bit epilogue (the
                          // host proved its bounds; see the epilogue), with m = sh - 16 in [0, 30]
-    int win_bytes;       // window mode: bytes of one window (128-byte aligned)
+    int win_bytes;       // window mode: bytes of one window (128-byte aligned; patch 4: 16-byte aligned)
+    int w64_slot0;       // patch 4: offset of window slot 0 (after the resident weights)
+    int w64_slot_stride; // bytes between the two window slots (S copies of WH KiB)
     int TH, TW;          // patch shape (TH * TW = 128)
     int tiles_p, tiles_q;  // patches per image along P and Q
     ConvArgs a;
@@ -567,8 +577,9 @@ __device__ __forceinline__ void pk_convert_loop(const TcParams& P, int cid, int 
 // staging): one thread issues every copy and TC_PK_CONVERTERS warps expand the weights.
 // WIN: the window-mode instance of the 32-bit two-limb epilogue (P.patch == 3, P.w32): 16 epilogue warps and
 // two staging tiles; only window mode's roles are compiled into it.
-template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false, bool WIN = false>
-__global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK), 1)
+// W64: the same for the 64-channel window mode (P.patch == 4) with one-plane codes out.
+template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false, bool WIN = false, bool W64 = false>
+__global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_pk(BN, PK), 1)
     conv_tc_kernel(const __grid_constant__ TcParams P) {
     constexpr int TC_STAGES = tc_stages(BN);
     constexpr int TC_LAG = tc_lag(BN);
@@ -580,10 +591,12 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
     static_assert(TC_STAGES % TC_PRODUCERS == 0 && TC_PRODUCERS <= 4,
                   "each stage must have one producer thread among warps 0..3");
     static_assert(!WIN || (BN == 64 && sizeof(ACC) == 8 && !SC && !SPLIT && !PK), "window instance: BN = 64, int64");
-    constexpr int EPI_WARPS = WIN ? TC_WIN_EPI_WARPS : tc_epi_warps(BN);
+    static_assert(!W64 || (BN == 64 && sizeof(ACC) == 4 && !SC && !SPLIT && !PK && !WIN), "W64 instance: BN = 64, int32");
+    constexpr bool WEPI = WIN || W64;  // the window instances' epilogue (16 warps, two staging tiles)
+    constexpr int EPI_WARPS = WEPI ? TC_WIN_EPI_WARPS : tc_epi_warps(BN);
     constexpr int EPI_THREADS = 32 * EPI_WARPS;
     constexpr int MMA_WARP = 4 + EPI_WARPS;
-    constexpr int CPW = WIN ? 1 : (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
+    constexpr int CPW = WEPI ? 1 : (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
     constexpr int B_BYTES = BN * TC_BK * 2;
     constexpr uint32_t IDESC = make_idesc(TC_BM, BN);
@@ -596,8 +609,9 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     unsigned char* sA = base;
     unsigned char* sB = base + TC_STAGES * A_BYTES;
-    unsigned char* sO = sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of [128 rows][64 codes]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2 * (WIN ? 2 : 1));  // WIN: two staging tiles
+    unsigned char* sO = W64 ? base + TC_W64_SO : sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of
+                                                                         // [128 rows][64 codes]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2 * (WEPI ? 2 : 1));  // WEPI: two staging tiles
     // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
     volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
@@ -632,7 +646,7 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
         mbar_init(done_bar, 1);
         mbar_init(stg_full, EPI_WARPS);
         mbar_init(stg_free, 1);
-        if (WIN) {
+        if (WEPI) {
             mbar_init(stg_full2, EPI_WARPS);
             mbar_init(stg_free2, 1);
         }
@@ -659,7 +673,49 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp < 4 && P.patch == 3) {
+    if (!WIN && warp < 4 && P.patch == 4) {
+        // ============================================================ producer, 64-channel window mode
+        // The weights, one 128-byte-swizzled box {64 ch, 64 out ch} per tap (8 KiB, the layout of a B
+        // stage), are loaded once to the start of shared memory.  Per tile and tap column s, the input
+        // window of the 16 x 8 patch shifted by s pixels, TH + R - 1 rows of 8 pixels of 64 channels (one
+        // swizzle pattern per row, padding zero filled), is one box into window slot (tile count mod 2):
+        // every tap's A operand then starts on a pattern boundary.
+        if (threadIdx.x == 0) {
+            mbar_arrive_expect_tx(wbar, (uint32_t)(a.R * a.S) * 8192u);
+            for (int t = 0; t < a.R * a.S; ++t)
+                tma_load_3d(smem_u32(sA) + (uint32_t)t * 8192u, &P.tmap_w, t * TC_BK, 0, 0, wbar);
+            const uint32_t copyb = (uint32_t)P.WH * 1024u;
+            const int per_img = P.tiles_p * P.tiles_q;
+            uint32_t it = 0, stage = 0, phase = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+                const int n_img = t / per_img, r = t - n_img * per_img;
+                const int hp0 = (r / P.tiles_q) * P.TH - a.pad, wq0 = (r % P.tiles_q) * P.TW - a.pad;
+                if (!wait_bounded(empty0 + 8 * stage, phase ^ 1, abort, P.status)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t fb = full0 + 8 * stage;
+                mbar_arrive_expect_tx(fb, (uint32_t)a.S * copyb);
+                const uint32_t dst = smem_u32(sA) + (uint32_t)P.w64_slot0 + stage * (uint32_t)P.w64_slot_stride;
+                for (int q = 0; q < a.S; ++q) tma_load_4d(dst + (uint32_t)q * copyb, &P.tmap_x, 0, wq0 + q, hp0, n_img, fb);
+                ++it;
+                if (++stage == 2) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            }
+            const uint32_t from = it >= 2 ? it - 2 : 0;
+            for (uint32_t j = from; j < it; ++j) {
+                const long long t0 = clock64();
+                while (!mbar_try_wait(full0 + 8 * (j % 2), (j / 2) & 1) && clock64() - t0 < TC_WAIT_CYCLES) {
+                }
+            }
+            const long long t0 = clock64();
+            while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
+            }
+        }
+    } else if (!W64 && warp < 4 && P.patch == 3) {
         // ============================================================ producer, window mode
         // Stride 1, Cp == 8: the weights are loaded once into the B region, per kernel row r and tap
         // pair sp a block of the two taps, each tap the BN output channels of every limb plane in turn
@@ -714,7 +770,7 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
             while (!mbar_try_wait(wbar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
             }
         }
-    } else if (!WIN && warp < 4 && (P.patch || P.rows_tma)) {
+    } else if (!WEPI && warp < 4 && (P.patch || P.rows_tma)) {
         // ============================================================ producer, patch tiles
         // Stride 1 and Cp % 64 == 0: the A tile of tap (r, s) and channels c0..c0+63 is the box
         // {64, TW, TH} of the input at (c0, q0 + s - pad, p0 + r - pad); the padding reads as zeros.
@@ -801,7 +857,7 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
             }
         }
         if (PK && warp >= 1) pk_convert_loop<BN, SPLIT>(P, warp - 1, lane, sP, sB, pkfull0, full0, abort);
-    } else if (!WIN && warp < 4) {
+    } else if (!WEPI && warp < 4) {
         // ============================================================ producers, row tiles
         // Thread t copies 16-byte chunk c = t % 8 of rows t/8, t/8 + 16, ...: eight consecutive
         // threads cover one 128-byte row, so every warp instruction reads four whole rows.
@@ -887,10 +943,11 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
                 }
             }
         }
-    } else if (WIN && warp < MMA_WARP) {
-        // ============================================================ epilogue, window instance
-        // Warp w drains TMEM lanes 32 (w % 4) .. + 31 and the 16 columns 16 cw .., cw = (w - 4) / 4, of the
-        // four limb accumulators, with the 32-bit arithmetic of the generic window epilogue below; tile u
+    } else if (WEPI && warp < MMA_WARP) {
+        // ============================================================ epilogue, window instances
+        // Warp w drains TMEM lanes 32 (w % 4) .. + 31 and the 16 columns 16 cw .., cw = (w - 4) / 4: WIN of
+        // the four limb accumulators, with the 32-bit arithmetic of the generic window epilogue below;
+        // W64 of the one int32-exact accumulator, with the FxP-QLayer of the generic epilogue.  Tile u
         // goes through staging tile u % 2, whose previous store must have read it (at most the other
         // tile's store is then in flight).
         const int quad = warp & 3, cw = (warp - 4) >> 2;
@@ -911,23 +968,49 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
                 break;
             }
             tc_fence_after();
-            uint32_t fhh[16], fhl[16], flh[16], fll[16];
-            const uint32_t abase = lane_base + buf * (uint32_t)(4 * BN) + (uint32_t)(cw * 16);
-            tmem_ld16_nw(abase, fhh);
-            tmem_ld16_nw(abase + (uint32_t)BN, fhl);
-            tmem_ld16_nw(abase + (uint32_t)(2 * BN), flh);
-            tmem_ld16_nw(abase + (uint32_t)(3 * BN), fll);
-            tmem_wait_ld();
-            reg_fence(fhh);
-            reg_fence(fhl);
-            reg_fence(flh);
-            reg_fence(fll);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
             uint32_t w[8];
+            if (W64) {
+                uint32_t f[16];
+                tmem_ld16_nw(lane_base + buf * (uint32_t)BN + (uint32_t)(cw * 16), f);
+                tmem_wait_ld();
+                reg_fence(f);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
+                const Epi32 e32 = make_epi32(a);
+                const Epi64 e64 = make_epi64(a);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+                for (int j = 0; j < 8; ++j) {
+                    int c2[2];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int k = cw * 16 + 2 * j + h;
+                        const int acc = __float2int_rn(__uint_as_float(f[2 * j + h]));
+                        const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                        c2[h] = a.v32 ? epi32_code(e32, acc, (b << e32.bsl) >> e32.bsr, (b & e32.fmask) != 0 ? 1 : 0)
+                                      : epi64_code<false>(e64, (long long)acc, b, 0, 0);
+                    }
+                    w[j] = pack_codes_f16(c2[0], c2[1]);
+                }
+            }
+            uint32_t fhh[16], fhl[16], flh[16], fll[16];
+            if (WIN) {
+                const uint32_t abase = lane_base + buf * (uint32_t)(4 * BN) + (uint32_t)(cw * 16);
+                tmem_ld16_nw(abase, fhh);
+                tmem_ld16_nw(abase + (uint32_t)BN, fhl);
+                tmem_ld16_nw(abase + (uint32_t)(2 * BN), flh);
+                tmem_ld16_nw(abase + (uint32_t)(3 * BN), fll);
+                tmem_wait_ld();
+                reg_fence(fhh);
+                reg_fence(fhl);
+                reg_fence(flh);
+                reg_fence(fll);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
+            }
+#pragma unroll
+            for (int j = 0; j < (WIN ? 8 : 0); ++j) {
                 int c2[2];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -1365,7 +1448,50 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
     } else if (PK && warp > MMA_WARP) {
         // ============================================================ packed-weight converters
         pk_convert_loop<BN, SPLIT>(P, 3 + (warp - MMA_WARP - 1), lane, sP, sB, pkfull0, full0, abort);
-    } else if (lane == 0 && P.patch == 3) {
+    } else if (!WIN && lane == 0 && P.patch == 4) {
+        // ============================================================ MMA issue, 64-channel window mode
+        // Per tile, tap (r, s) and 16-channel step kk: one MMA.  A is window copy s from row r: rows 128
+        // bytes apart, the 8-row groups (patch rows, TW = 8) one pattern (1 KiB) apart; B the resident tap
+        // block (a B stage's layout).  One barrier round per tile.
+        const uint32_t copyb = (uint32_t)P.WH * 1024u;
+        uint32_t stage = 0, phase = 0, gcount = 0;
+        bool ok = wait_bounded(wbar, 0, abort, P.status);
+        tc_fence_after();
+        for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
+            const uint32_t buf = gcount & 1;
+            if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
+                !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t wa = smem_u32(sA) + (uint32_t)P.w64_slot0 + stage * (uint32_t)P.w64_slot_stride;
+            const uint32_t d = tmem + buf * BN;
+            uint32_t accum = 0;
+            for (int r = 0; r < a.R; ++r)
+                for (int q = 0; q < a.S; ++q) {
+                    const uint64_t ad = make_sdesc(wa + (uint32_t)q * copyb + (uint32_t)r * 1024u);
+                    const uint64_t bd = make_sdesc(smem_u32(sA) + (uint32_t)(r * a.S + q) * 8192u);
+#pragma unroll
+                    for (int kk = 0; kk < TC_BK / 16; ++kk) {
+                        tc_mma(d, ad + 2 * kk, bd + 2 * kk, IDESC, accum);
+                        accum = 1;
+                    }
+                }
+            tc_commit(empty0 + 8 * stage);
+            if (++stage == 2) {
+                stage = 0;
+                phase ^= 1;
+            }
+            tc_commit(accfull0 + 8 * buf);
+            ++gcount;
+        }
+        // every MMA issued by this thread has completed once `done` fires
+        tc_commit(done_bar);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
+        }
+    } else if (!W64 && lane == 0 && P.patch == 3) {
         // ============================================================ MMA issue, window mode
         // Per tile and limb pair (ia, iw): R * S2/2 MMAs of K = 16 (two taps of 8 channels).  The A
         // operand of taps (r, 2sp), (r, 2sp + 1) is the window shifted by (r, 2sp) pixels: K-major
@@ -1421,7 +1547,7 @@ __global__ void __launch_bounds__(WIN ? tc_threads_win() : tc_threads_pk(BN, PK)
         const long long t0 = clock64();
         while (!mbar_try_wait(done_bar, 0) && clock64() - t0 < TC_WAIT_CYCLES) {
         }
-    } else if (!WIN && lane == 0) {
+    } else if (!WEPI && lane == 0) {
         // ============================================================ MMA issue (one thread of MMA_WARP)
         // Descriptors of stage 0; a stage or a 16-element k step moves the start-address field
         // (address >> 4, 14 bits) without carry since shared addresses stay below 256 KB.

@@ -162,6 +162,12 @@ CASES = [
     (2, 20, 3, 48, 3, 1, 1, (16, 1, 9), (16, 1, 12), (16, 18), False, 0, (6, 1, 2)),
     (1, 18, 3, 64, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 17), True, 0, (8, 0, 2)),
     (2, 20, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 13), (16, 30), False, 0, (8, 1, 3)),
+    # 64-channel window mode (stride 1, one plane, Cp % 16 == 0 and <= 64, K <= 64, one exact group):
+    # ragged maps, every supported Cp, no padding, 2 x 2 taps, every output mode
+    (2, 19, 64, 64, 3, 1, 1, (8, 0, 4), (7, 1, 8), (16, 15), True, 0, (8, 0, 3)),
+    (3, 12, 32, 48, 3, 1, 1, (6, 0, 2), (5, 1, 5), (16, 10), False, 0, (8, 1, 2)),
+    (2, 10, 16, 64, 3, 1, 0, (8, 0, 4), (8, 1, 7), None, True, 2, None),
+    (1, 9, 48, 24, 2, 1, 0, (4, 0, 1), (8, 1, 9), (16, 12), True, 1, None),
     # the 32-bit window epilogue at its smallest shift (16: the tie is decided by the low 16 bits alone),
     # and one below it (15: the 64-bit path)
     (1, 16, 3, 32, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 15), False, 0, (8, 1, 3)),
@@ -328,6 +334,7 @@ SCALE_CASES = [
     (CASES[32], (16, 14), (16, 12)),    # window mode, two-limb fast epilogue
     (CASES[35], (16, 14), (16, 12)),    # window mode, ACC64
     (CASES[41], (16, 14), (16, 12)),    # 1x1: A tiles as 2-D TMA boxes
+    (CASES[48], (16, 14), (16, 12)),    # 64-channel window mode
     (CASES[36], (16, 14), (16, 12)),    # split reduction
     (CASES[39], (16, 13), (16, 10)),    # split reduction, two limbs, ACC64
 ]
