@@ -222,7 +222,7 @@ def run_fxpq(args):
     d2h = host_logits.numel() * 8
 
     # ---- roofline of the dominant kernel (the conv C-Block): op-by-op forward with events per conv
-    conv_ms, conv_flops, nconv = conv_roofline(q, imgs, F, stream)
+    conv_ms, conv_flops, nconv, conv_layers = conv_roofline(q, imgs, F, stream)
     hbm, bf16, bf16s, src = measured_peaks()
     achieved = conv_flops / (conv_ms / 1e3) / 1e12
     traffic = None
@@ -244,7 +244,7 @@ def run_fxpq(args):
             "roofline": {"bound": "tensor", "kernel": "conv C-Block", "achieved": round(achieved, 3),
                          "peak": bf16, "unit": "TFLOP/s", "frac": round(achieved / bf16, 5), "traffic": traffic,
                          "peak_source": f"{src} bf16 dense burst (fp16 operands run at the bf16 rate)",
-                         "conv_launches_timed": nconv},
+                         "conv_launches_timed": nconv, "conv_layers_us": conv_layers},
             "clocks": clk.summary(),
             "cpu_baseline": cpu,
         }
@@ -258,12 +258,18 @@ def conv_roofline(q, imgs, F, stream, iters=3):
 
     A device-side sleep of about 1 ms is queued ahead of each timed conv, so that the host's argument
     preparation (workspace queries, tensor-map encoding, the split reduction's workspace) overlaps it
-    and the events bracket the conv kernel(s) alone rather than the host gap before the launch."""
+    and the events bracket the conv kernel(s) alone rather than the host gap before the launch.  The
+    first forward is not counted (its allocations reach the device).  Returns the total time, the
+    algorithmic FLOPs, the number of timed launches and the per-layer average in microseconds."""
     import torch
-    env0 = None
     tot_ms, flops, n = 0.0, 0, 0
+    per_layer = {}
     N = imgs.shape[0]
+    env = None
     for it in range(iters):
+        # the previous forward's tensors go back to the caching allocator before this one allocates, so
+        # from the second forward on no layer's output allocation reaches the device inside its events
+        env = None
         fin = q.fmts["input"]["a"]
         x0 = torch.empty(N * q.hw * q.hw * q.cp_in * F.planes(fin), dtype=torch.float16, device=imgs.device)
         F.fxpq_quantize_images(imgs, fin, q.cp_in, x0)
@@ -281,15 +287,14 @@ def conv_roofline(q, imgs, F, stream, iters=3):
                 e1.synchronize()
                 if it > 0:
                     tot_ms += e0.elapsed_time(e1)
+                    per_layer[nm] = per_layer.get(nm, 0.0) + e0.elapsed_time(e1) * 1e3 / (iters - 1)
                     H, _, K = q.shapes[nm]
                     flops += 2 * N * H * H * K * L_["C"] * L_["R"] * L_["R"]
                     n += 1
             else:
                 y, s = q.run_layer(i, env, N, mode)
             env[nm] = (y, q.fmts[nm].get("a"))
-        del env0
-        env0 = env
-    return tot_ms, flops, n
+    return tot_ms, flops, n, {k: round(v, 1) for k, v in per_layer.items()}
 
 
 # ----------------------------------------------------------------------------- configs 1 and 2
@@ -668,6 +673,36 @@ def run_kernel(args):
         peak = 152 * 128 * 2 * 2.07e9 / 1e12  # fp32 FMA lanes x 2 FLOP x max SM clock
         out["conv_f32"] = {"ms": round(ms, 4), "tflops": round(tf, 2), "peak_fp32_tflops": round(peak, 1),
                            "frac": round(tf / peak, 3)}
+    if args.kernel in ("fc", "all"):
+        # VGG-16 fc6 at batch 64 (25088 -> 4096: a 7 x 7 kernel over the 7 x 7 map) with k-bit weights read
+        # as fp16 code tensors and as packed k-bit planes (Sec. V-E.2); weight bytes read per launch
+        N, H, C, K = 64, 7, 512, 4096
+        rng = np.random.default_rng(5)
+        x = torch.from_numpy(rng.integers(0, 32, size=(N, H, H, C)).astype(np.float16)).cuda()
+        b = torch.from_numpy(rng.integers(-2 ** 15, 2 ** 15, size=K).astype(np.int32)).cuda()
+        y = torch.empty(N * K, dtype=torch.float16, device="cuda")
+        for kw in (8, 4):
+            wc = rng.integers(-(1 << (kw - 1)), 1 << (kw - 1), size=(K, H, H, C))
+            w = torch.from_numpy(wc.astype(np.float16)).cuda()
+            fw = F.fmt(kw, 1, kw + 4)
+            l1 = int(np.abs(wc).reshape(K, -1).sum(axis=1).max())
+            wp = F.pack_weights(w, fw, K, H * H * C)
+            for name, packed in ((f"fc6_k{kw}_f16", None), (f"fc6_k{kw}_packed", wp)):
+                d = F.conv_desc(N, H, H, C, C, K, H, H, 1, 0, 1, F.OUT_CODES, F.fmt(5, 0, 2), fw, F.fmt(16, 1, 20),
+                                F.fmt(8, 0, 3), l1, wpacked=packed)
+                ws = torch.empty(F.fxpq_conv_workspace(d), dtype=torch.uint8, device="cuda")
+                ts = []
+                for i in range(args.warmup + args.steps):
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                    F.fxpq_conv_fwd(d, x, w, b, y, ws=ws)
+                    e1.record()
+                    e1.synchronize()
+                    if i >= args.warmup:
+                        ts.append(e0.elapsed_time(e1))
+                ms = sum(ts) / len(ts)
+                wbytes = w.numel() * 2 if packed is None else packed.numel()
+                out[name] = {"ms": round(ms, 4), "weight_bytes": wbytes, "weight_gbs": round(wbytes / (ms / 1e3) / 1e9, 1)}
     if args.kernel in ("config1", "all"):
         out.update(bench_config1(args, F))
     if args.kernel in ("config2", "all"):
@@ -702,7 +737,8 @@ def run_kernel(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "fopt", "forward", "config1", "config2", "all"],
+    ap.add_argument("--kernel", choices=["conv", "flsearch", "quantize", "fopt", "forward", "fc", "config1", "config2",
+                                         "all"],
                     help="time one kernel case and exit")
     ap.add_argument("--oracle-job", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--gpus", type=int, default=1)
