@@ -221,7 +221,13 @@ def run_fxpq(args):
     h2d = pinned.numel() * 4
     d2h = host_logits.numel() * 8
 
-    # ---- roofline of the dominant kernel (the conv C-Block): op-by-op forward with events per conv
+    # ---- roofline of the dominant kernel (the conv C-Block): op-by-op forward with events per conv, on
+    # the workload's first plan (the network `--kernel forward` builds, whose conv launches the DRAM
+    # traffic capture profiles; another plan's formats can change a layer's exact groups)
+    q = QNet(layers, hw=224, cin=3)
+    q._dev = dev
+    q.quantize_params(wdev, plans[0], None, bndev)
+    q.calibrate(imgs[: wl["calib"]], plans[0])
     conv_ms, conv_flops, nconv, conv_layers = conv_roofline(q, imgs, F, stream)
     hbm, bf16, bf16s, src = measured_peaks()
     achieved = conv_flops / (conv_ms / 1e3) / 1e12
