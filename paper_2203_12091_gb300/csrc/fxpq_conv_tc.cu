@@ -166,6 +166,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         P.patch = 0;
         P.rows_tma = 0;
         P.w32 = 0;
+        P.wf32 = 0;
         P.nacc = 1;
         // window mode for 8-channel stride-1 layers with at most 64 output channels: 8 x 16 output
         // patches, one input window per tile and limb plane, weights resident in shared memory, one
@@ -221,8 +222,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                     // sum covers R * S2 * 8 products; L = 2^8 (S_hl + S_lh) + S_ll + Lo(B') and T must stay
                     // below 2^31, the aligned bias must not be finer than the sums (delta >= 0), and
                     // sh - 16 in [0, 30]; the per-channel bias table takes the last 512 bytes of the B region
-                    if (a.px == 2 && a.pw == 2 && !a.has_scale && a.delta >= 0 && a.out_mode == FXPQ_OUT_CODES &&
-                        a.py == 1 && a.sh >= 16 && a.sh <= 46 &&
+                    const bool codes32 = a.out_mode == FXPQ_OUT_CODES && a.py == 1 && a.sh >= 16 && a.sh <= 46;
+                    const bool image32 = a.out_mode == FXPQ_OUT_F32 && a.K % 4 == 0;  // the fp32 image
+                    if (a.px == 2 && a.pw == 2 && !a.has_scale && a.delta >= 0 && (codes32 || image32) &&
                         a.pw * a.R * (S2 / 2) * 64 * 32 + 512 <= tc_stages(64) * 64 * TC_BK * 2) {
                         const double taps = (double)a.R * S2 * 8;
                         const double hh = (double)limb_max(d.fmt_x, 0) * limb_max(d.fmt_w, 0) * taps;
@@ -232,7 +234,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                         const double bb = a.has_bias ? ldexp(1.0, d.fmt_b.bits - d.fmt_b.is_signed + a.delta) : 0.0;
                         const double Lb = 256.0 * (hl + lh) + ll + 65536.0;
                         const double Tb = hh + bb / 65536.0 + 1.0 + Lb / 65536.0 + 1.0;
-                        P.w32 = Lb < ldexp(1.0, 31) && Tb < ldexp(1.0, 31) && !conv_path_is("tc_win64");
+                        const bool ok32 = Lb < ldexp(1.0, 31) && Tb < ldexp(1.0, 31) && !conv_path_is("tc_win64");
+                        P.w32 = ok32 && codes32;
+                        P.wf32 = ok32 && image32;
                     }
                 }
             }
@@ -243,7 +247,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         // two window slots of S copies (shifted by 0 .. S - 1 pixels) of TH + R - 1 rows of 8 pixels
         if (P.patch == 0 && BN == 64 && a.K <= 64 && !acc64 && a.stride == 1 && a.Cp == 64 && a.px == 1 &&
             a.pw == 1 && P.n_groups == 1 && a.N > 0 && a.P > 0 && a.Q > 0 && a.R <= 3 && a.S <= 3 &&
-            a.out_mode == FXPQ_OUT_CODES && a.py == 1 && (a.v32 || (a.sh >= 1 && a.sh <= 62)) && !a.has_scale &&
+            ((a.out_mode == FXPQ_OUT_CODES && a.py == 1 && (a.v32 || (a.sh >= 1 && a.sh <= 62))) ||
+             (a.out_mode == FXPQ_OUT_F32 && a.K % 4 == 0)) &&
+            !a.has_scale &&
             !conv_path_is("tc_rows") && !conv_path_is("tc_patch") && !conv_path_is("tc_nowin")) {
             const int WH = 16 + a.R - 1;
             const long long slot = (long long)a.S * WH * 1024;
@@ -321,6 +327,7 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         }
         if (!P.rows_tma) P.pk = 0;
         if (P.w32 && !(a.out_mode == FXPQ_OUT_CODES && a.py == 1)) P.w32 = 0;
+        if (P.wf32 && a.out_mode != FXPQ_OUT_F32) P.wf32 = 0;
         // one-plane codes: stage the tile in shared memory and write it with TMA stores (not with packed
         // weights, whose staging region holds the packed stages)
         P.fast_store = 0;
@@ -432,10 +439,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
     const int grid = P.n_units < sms ? P.n_units : sms;
     launched = true;
     if (a.has_scale) return launch_conv_tc_scaled(P, BN, acc64, grid, st);  // never split
-    if (P.patch == 3 && P.w32)  // window mode, 32-bit two-limb epilogue: its own instance (never split)
+    if (P.patch == 3 && (P.w32 || P.wf32))  // window mode, 32-bit two-limb epilogue: its own instance (never split)
         conv_tc_kernel<64, long long, false, false, false, true>
             <<<grid, tc_threads_win(), tc_smem_bytes<64>() + 64 * TC_BM * 2, st>>>(P);
-    else if (P.patch == 4 && P.fast_store)
+    else if (P.patch == 4 && (P.fast_store || a.out_mode == FXPQ_OUT_F32))
         // 64-channel window mode: the instance with its own shared-memory layout and 16 epilogue warps
         conv_tc_kernel<64, int, false, false, false, false, true><<<grid, tc_threads_win(), tc_smem_w64(), st>>>(P);
     else if (P.patch == 4) {

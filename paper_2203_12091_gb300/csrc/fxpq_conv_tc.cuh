@@ -113,6 +113,7 @@ struct TcParams {
     int WW, WH, S2;      // window mode: window width / height in pixels, taps per row rounded up to even
     int w32;             // window mode, two-limb x and w, one-plane codes out: the 32-bit epilogue (the
                          // host proved its bounds; see the epilogue), with m = sh - 16 in [0, 30]
+    int wf32;            // the same window instance writing the fp32 image of v = 2^16 T + Lo
     int win_bytes;       // window mode: bytes of one window (128-byte aligned; patch 4: 16-byte aligned)
     int w64_slot0;       // patch 4: offset of window slot 0 (after the resident weights)
     int w64_slot_stride; // bytes between the two window slots (S copies of WH KiB)
@@ -451,6 +452,62 @@ __device__ __forceinline__ void epilogue_block32(const ConvArgs& a, long long m,
     }
 }
 
+// The same for fp32-image and int64 outputs through a 2 KiB shared-memory slice of the warp (`wbuf`): every
+// round each lane puts 64 bytes of its row there (16-byte pieces rotated against bank conflicts), then the
+// warp writes 16-byte pieces of whole row segments, eight rows per instruction, rather than 32 rows at one
+// value per lane.  All 32 lanes take part; rows with m < 0 (outside the output) store nothing.  Needs K %
+// 4 == 0 (fp32) or K % 2 == 0 (int64), so that a 16-byte piece is wholly inside or past K.
+template <typename ACC, bool SC>
+__device__ __forceinline__ void epilogue_block32_staged(const ConvArgs& a, long long m, int k0, const ACC (&acc)[32],
+                                                        unsigned char* wbuf, int lane) {
+    const bool f32 = a.out_mode == FXPQ_OUT_F32;
+    const int per = f32 ? 16 : 8;  // values per round: 64 bytes of a row
+#pragma unroll
+    for (int c0 = 0; c0 < 32; c0 += 8) {
+        if (c0 % per) continue;  // fp32 rounds start at 0 and 16
+        uint32_t wv[16];
+        if (f32) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int k = k0 + c0 + j;
+                float v = 0.0f;
+                if (m >= 0 && k < a.K && c0 + j < 32)
+                    v = __ll2float_rn(cblock_value<SC>(a, k, (long long)acc[(c0 + j) & 31], a.has_bias ? __ldg(a.bias + k) : 0)) *
+                        a.f32_scale;
+                wv[j] = __float_as_uint(v);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int k = k0 + c0 + j;
+                long long v = 0;
+                if (m >= 0 && k < a.K) v = cblock_value<SC>(a, k, (long long)acc[c0 + j], a.has_bias ? __ldg(a.bias + k) : 0);
+                wv[2 * j] = (uint32_t)(unsigned long long)v;
+                wv[2 * j + 1] = (uint32_t)((unsigned long long)v >> 32);
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(wbuf + lane * 64 + 16 * (q ^ ((lane >> 1) & 3))) =
+                make_uint4(wv[4 * q], wv[4 * q + 1], wv[4 * q + 2], wv[4 * q + 3]);
+        __syncwarp();
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+            const int r = (lane >> 2) + 8 * it, pc = lane & 3;
+            const long long mr = __shfl_sync(0xffffffffu, m, r);
+            const uint4 v = *reinterpret_cast<const uint4*>(wbuf + r * 64 + 16 * (pc ^ ((r >> 1) & 3)));
+            const int kk = k0 + c0 + pc * (f32 ? 4 : 2);
+            if (mr >= 0 && kk < a.K) {
+                if (f32)
+                    *reinterpret_cast<uint4*>(static_cast<float*>(a.y) + mr * a.K + kk) = v;
+                else
+                    *reinterpret_cast<uint4*>(static_cast<long long*>(a.y) + mr * a.K + kk) = v;
+            }
+        }
+        __syncwarp();
+    }
+}
+
 // Uniform constants of the 32-bit FxP-QLayer epilogue (the same arithmetic as qlayer_code32, with
 // the bias alignment split into a left and a right shift so that it has no branches).
 struct Epi32 {
@@ -662,7 +719,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
     // window mode, 32-bit epilogue: per output channel the aligned bias B' = b 2^delta split as
     // (B' >> 16, B' & 0xFFFF), in the last 512 bytes of the B region (the resident weights stay below)
     int2* wtab = reinterpret_cast<int2*>(sB + TC_STAGES * B_BYTES - 512);
-    if (BN == 64 && sizeof(ACC) == 8 && !SC && P.patch == 3 && P.w32 && warp == 1) {
+    if (BN == 64 && sizeof(ACC) == 8 && !SC && P.patch == 3 && (P.w32 || P.wf32) && warp == 1) {
         for (int k = lane; k < 64; k += 32) {
             const long long bb = (a.has_bias && k < a.K) ? ((long long)__ldg(a.bias + k) << (a.delta > 0 ? a.delta : 0)) : 0;
             wtab[k] = make_int2((int)(bb >> 16), (int)(bb & 0xFFFF));
@@ -959,6 +1016,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
         const int mmask = (int)((1u << m) - 1u);
         const int lo = (int)a.lo, hi = (int)a.hi;
         const int per_img = P.tiles_p * P.tiles_q;
+        const bool f32out = a.out_mode == FXPQ_OUT_F32;  // the fp32 image (calibration) instead of codes
         bool ok = true;
         uint32_t u = 0;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x, ++u) {
@@ -968,7 +1026,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 break;
             }
             tc_fence_after();
-            uint32_t w[8];
+            uint32_t w[16];  // codes: 8 words of fp16 pairs; fp32 image: 16 values
             if (W64) {
                 uint32_t f[16];
                 tmem_ld16_nw(lane_base + buf * (uint32_t)BN + (uint32_t)(cw * 16), f);
@@ -979,8 +1037,17 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
                 const Epi32 e32 = make_epi32(a);
                 const Epi64 e64 = make_epi64(a);
+                if (f32out) {
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
+                    for (int j = 0; j < 16; ++j) {
+                        const int k = cw * 16 + j;
+                        const int acc = __float2int_rn(__uint_as_float(f[j]));
+                        const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                        w[j] = __float_as_uint(__ll2float_rn(cblock_value<false>(a, k, (long long)acc, b)) * a.f32_scale);
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < (f32out ? 0 : 8); ++j) {
                     int c2[2];
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
@@ -1009,8 +1076,20 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 __syncwarp();
                 if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
             }
+            if (WIN && f32out) {
+                // the fp32 nearest-even image of v = 2^16 T + Lo (ReLU: 0 when T < 0), scaled by 2^-s
 #pragma unroll
-            for (int j = 0; j < (WIN ? 8 : 0); ++j) {
+                for (int jj = 0; jj < 16; ++jj) {
+                    const int2 bt = wtab[cw * 16 + jj];
+                    const int mid = __float2int_rn(__uint_as_float(fhl[jj])) + __float2int_rn(__uint_as_float(flh[jj]));
+                    const int L = mid * 256 + __float2int_rn(__uint_as_float(fll[jj])) + bt.y;
+                    const int T = __float2int_rn(__uint_as_float(fhh[jj])) + bt.x + (L >> 16);
+                    const long long v = (a.relu && T < 0) ? 0LL : ((long long)T << 16) + (L & 0xFFFF);
+                    w[jj] = __float_as_uint(__ll2float_rn(v) * a.f32_scale);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < ((WIN && !f32out) ? 8 : 0); ++j) {
                 int c2[2];
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -1033,6 +1112,18 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                     c2[h] = min(max(cc, lo), hi);
                 }
                 w[j] = pack_codes_f16(c2[0], c2[1]);
+            }
+            if (f32out) {
+                // fp32 image out: this row's 16 values are 64 contiguous bytes of the output row
+                const long long mrow = tile_row(P, t, row);
+                if (mrow >= 0) {
+                    float* yp = static_cast<float*>(a.y) + mrow * a.K + cw * 16;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        if (cw * 16 + 4 * q < a.K)
+                            *reinterpret_cast<uint4*>(yp + 4 * q) = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                }
+                continue;
             }
             const uint32_t sb = u & 1, n = u >> 1;  // staging tile and its use count
             const uint32_t sfull = sb ? stg_full2 : stg_full, sfree = sb ? stg_free2 : stg_free;
@@ -1412,6 +1503,9 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                             *reinterpret_cast<uint4*>(half_buf + row * 128 + ((chunk ^ (row & 7)) << 4)) =
                                 make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
                         }
+                    } else if (!PK && (a.out_mode == FXPQ_OUT_F32 ? a.K % 4 == 0 : (a.out_mode == FXPQ_OUT_ACC64 && a.K % 2 == 0))) {
+                        // fp32 / int64 outputs through the warp's 2 KiB of the (unused) staging tile
+                        epilogue_block32_staged<ACC, SC>(a, m, k0, acc, sO + (warp - 4) * 2048, lane);
                     } else if (m >= 0) {
                         epilogue_block32<ACC, SC>(a, m, k0, acc);
                     }

@@ -233,14 +233,13 @@ namespace {
 
 struct CalibLayout {
     std::vector<Slot> slots;
-    size_t slots_bytes = 0, acc_off = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, cws_off = 0, cws = 0,
-           total = 0;
+    size_t slots_bytes = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, cws_off = 0, cws = 0, total = 0;
 };
 
 fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
     fxpq_status st = plan_net(net, n, L.slots, L.slots_bytes);
     if (st != FXPQ_OK) return st;
-    // largest per-op output (elements) for the int64 contraction values and their fp32 image
+    // largest per-op output (elements): the fp32 image of a C-Block output searched by the calibration
     size_t max_out = 1;
     for (int i = 0; i < net->n_ops - 1; ++i) {
         const fxpq_op_desc& o = net->ops[i];
@@ -249,8 +248,7 @@ fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
         if (e > max_out) max_out = e;
     }
     const size_t img = (size_t)n * net->C * net->H * net->W;
-    L.acc_off = L.slots_bytes;
-    L.f32_off = L.acc_off + align256(max_out * sizeof(int64_t));
+    L.f32_off = L.slots_bytes;
     L.fls_off = L.f32_off + align256((max_out > img ? max_out : img) * sizeof(float));
     L.rec_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
     L.err_off = L.rec_off + 256;
@@ -302,7 +300,6 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
     cudaStream_t s = fxpq::as_stream(stream);
     char* base = static_cast<char*>(d_ws);
     auto ptr = [&](int slot) { return static_cast<void*>(base + L.slots[slot].offset); };
-    int64_t* acc = reinterpret_cast<int64_t*>(base + L.acc_off);
     float* f32 = reinterpret_cast<float*>(base + L.f32_off);
     std::vector<fxpq_fmt> fmt(h_net->n_slots, fxpq_fmt{0, 0, 0});
 
@@ -329,8 +326,10 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                                   ptr(o.dst), s);
                 break;
             case FXPQ_OP_CONV: {
-                // one contraction with exact int64 values; the QLayer runs twice (fp32 image for the
-                // search, then the codes)
+                // the contraction writes the fp32 nearest-even image of its exact C-Block output for the
+                // search, then runs again with the searched format to codes (the same exact values both
+                // times: two passes over the codes and weights cost less than an int64 tensor written
+                // once and read twice)
                 fxpq_conv_desc cd = {};
                 cd.N = n_calib;
                 cd.H = s0.H;
@@ -343,7 +342,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.stride = o.stride;
                 cd.pad = o.pad;
                 cd.relu = o.relu;
-                cd.out_mode = FXPQ_OUT_ACC64;
+                cd.out_mode = FXPQ_OUT_F32;
                 cd.fmt_x = fmt[o.src0];
                 cd.fmt_w = o.fmt_w;
                 cd.fmt_b = o.fmt_b;
@@ -355,11 +354,14 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.d_shift = o.d_shift;
                 cd.d_wpacked = o.d_wpacked;
                 int32_t sc = 0;
-                st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, L.cws ? base + L.cws_off : nullptr,
-                                   L.cws, s);
-                if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_F32, fy, f32, s);
+                void* cws = L.cws ? base + L.cws_off : nullptr;
+                st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, f32, &sc, cws, L.cws, s);
                 if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
-                if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_CODES, fy, ptr(o.dst), s);
+                if (st == FXPQ_OK) {
+                    cd.out_mode = FXPQ_OUT_CODES;
+                    cd.fmt_y = fy;
+                    st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, ptr(o.dst), &sc, cws, L.cws, s);
+                }
                 break;
             }
             case FXPQ_OP_ELTWISE: {

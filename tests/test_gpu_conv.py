@@ -168,6 +168,11 @@ CASES = [
     (3, 12, 32, 48, 3, 1, 1, (6, 0, 2), (5, 1, 5), (16, 10), False, 0, (8, 1, 2)),
     (2, 10, 16, 64, 3, 1, 0, (8, 0, 4), (8, 1, 7), None, True, 2, None),
     (1, 9, 48, 24, 2, 1, 0, (4, 0, 1), (8, 1, 9), (16, 12), True, 1, None),
+    # the fp32 image of a C-Block output (calibration) from both window instances: two limbs with and
+    # without ReLU, and the 64-channel window
+    (2, 20, 3, 64, 3, 1, 1, (16, 1, 11), (16, 1, 13), (16, 21), True, 2, None),
+    (1, 18, 3, 48, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 17), False, 2, None),
+    (2, 19, 64, 64, 3, 1, 1, (8, 0, 4), (7, 1, 8), (16, 15), True, 2, None),
     # the 32-bit window epilogue at its smallest shift (16: the tie is decided by the low 16 bits alone),
     # and one below it (15: the 64-bit path)
     (1, 16, 3, 32, 3, 1, 1, (16, 1, 9), (16, 1, 10), (16, 15), False, 0, (8, 1, 3)),
