@@ -404,7 +404,9 @@ FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_imag
  *          each op's fmt_y.bits give the wordlengths (their S and FL are ignored);
  *   h_fmt_in: the chosen input format; h_fmt_y[n_ops]: each op's output format (a max-pool passes
  *          its input's on; the last op's entry is copied unchanged).
- * The host waits for each search (one device-to-host read per QLayer).  Workspace:
+ * The host waits for each search (a stream synchronisation per QLayer; the search writes its result
+ * into a mapped pinned host record that the library allocates once and reuses).  Errors: as the
+ * calls it makes, FXPQ_ERR_CUDA if the host record cannot be allocated.  Workspace:
  * fxpq_net_calibrate_workspace(h_net, n_calib) bytes, 256-byte aligned. */
 FXPQ_API size_t fxpq_net_calibrate_workspace(const fxpq_net* h_net, int32_t n_calib);
 FXPQ_API fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_calib_nchw, int32_t n_calib,

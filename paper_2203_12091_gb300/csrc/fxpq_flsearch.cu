@@ -631,55 +631,48 @@ struct Big {
     u64 w[BW];
 };
 
-__device__ __forceinline__ void big_zero(Big& a) {
-#pragma unroll
-    for (int i = 0; i < BW; ++i) a.w[i] = 0ull;
-}
+// A cell's exact sum is gathered in 24 signed 64-bit columns in shared memory, column c weighing
+// 2^(32 c + BBASE): every term is cut into 32-bit pieces added to their columns (shared-memory
+// atomics, so the lanes of a warp share one set), and one carry pass turns the columns into the
+// 768-bit two's complement value.  A column takes well under 2^31 pieces, so it cannot overflow;
+// pieces above column 23 weigh multiples of 2^(768 + BBASE) and drop, as modulo 2^768 they must.
+constexpr int NCOL = 2 * BW;
 
-// a += (neg ? -1 : 1) * v * 2^e for a 128-bit magnitude v
-__device__ void big_add(Big& a, U128 v, int e, bool neg) {
+// col += (neg ? -1 : 1) * v * 2^e for a 128-bit magnitude v
+__device__ __forceinline__ void col_add(u64* col, U128 v, int e, bool neg) {
     if ((v.lo | v.hi) == 0ull) return;
     const int pos = e - BBASE;
-    const int wi = pos >> 6, b = pos & 63;
-    u64 s[3];
-    s[0] = v.lo << b;
-    s[1] = b ? ((v.hi << b) | (v.lo >> (64 - b))) : v.hi;
-    s[2] = b ? (v.hi >> (64 - b)) : 0ull;
-    if (!neg) {
-        u64 carry = 0ull;
-        for (int i = wi; i < BW; ++i) {
-            const u64 add = (i - wi < 3) ? s[i - wi] : 0ull;
-            const u64 t = a.w[i] + add;
-            const u64 c1 = t < add;
-            const u64 t2 = t + carry;
-            const u64 c2 = t2 < t;
-            a.w[i] = t2;
-            carry = c1 | c2;
-            if (i - wi >= 2 && carry == 0ull) break;
-        }
-    } else {
-        u64 borrow = 0ull;
-        for (int i = wi; i < BW; ++i) {
-            const u64 sub = (i - wi < 3) ? s[i - wi] : 0ull;
-            const u64 t = a.w[i] - sub;
-            const u64 b1 = a.w[i] < sub;
-            const u64 t2 = t - borrow;
-            const u64 b2 = t < borrow;
-            a.w[i] = t2;
-            borrow = b1 | b2;
-            if (i - wi >= 2 && borrow == 0ull) break;
-        }
+    const int ci = pos >> 5;
+    const unsigned b = (unsigned)pos & 31u;
+    const unsigned x0 = (unsigned)v.lo, x1 = (unsigned)(v.lo >> 32), x2 = (unsigned)v.hi,
+                   x3 = (unsigned)(v.hi >> 32);
+    const unsigned c[5] = {x0 << b, __funnelshift_l(x0, x1, b), __funnelshift_l(x1, x2, b),
+                           __funnelshift_l(x2, x3, b), __funnelshift_l(x3, 0u, b)};
+#pragma unroll
+    for (int j = 0; j < 5; ++j)
+        if (c[j] && ci + j < NCOL) atomicAdd(&col[ci + j], neg ? (u64)(-(long long)c[j]) : (u64)c[j]);
+}
+
+// The columns' value as a 768-bit two's complement number.
+__device__ void col_to_big(const u64* col, Big& a) {
+    long long carry = 0;
+#pragma unroll
+    for (int i = 0; i < BW; ++i) {
+        const long long t0 = (long long)col[2 * i] + carry;
+        const long long t1 = (long long)col[2 * i + 1] + (t0 >> 32);
+        carry = t1 >> 32;
+        a.w[i] = (u64)(unsigned)t0 | ((u64)(unsigned)t1 << 32);
     }
 }
 
 // a += (neg ? -1 : 1) * m * 2^e * (the three-limb bin at p).  The top limb is signed: the histogram
 // kernel's remainder sums leave out the sum of L^2 that its exponent band carries, so one key's
 // share of a cell may be negative.
-__device__ __forceinline__ void big_add_L3(Big& a, const u64* p, int e, bool neg, u64 m = 1ull) {
-    big_add(a, mul128_64(U128{p[0], 0ull}, m), e, neg);
-    big_add(a, mul128_64(U128{p[1], 0ull}, m), e + 32, neg);
+__device__ __forceinline__ void col_add_L3(u64* a, const u64* p, int e, bool neg, u64 m = 1ull) {
+    col_add(a, mul128_64(U128{p[0], 0ull}, m), e, neg);
+    col_add(a, mul128_64(U128{p[1], 0ull}, m), e + 32, neg);
     const long long w2 = (long long)p[2];
-    if (w2) big_add(a, mul128_64(U128{w2 < 0 ? (u64)(-w2) : (u64)w2, 0ull}, m), e + 64, neg != (w2 < 0));
+    if (w2) col_add(a, mul128_64(U128{w2 < 0 ? (u64)(-w2) : (u64)w2, 0ull}, m), e + 64, neg != (w2 < 0));
 }
 
 __device__ u64 big_bits64(const Big& a, int pos) {  // bits [pos, pos + 64), zero below bit 0
@@ -727,35 +720,30 @@ __device__ void big_negate(Big& a) {
 }
 
 // saturated set with moments (n, s1, s2) at exponent E: s2 2^(2(E-23)) - 2 T s1 2^(E-23-fl) + T^2 n 2^(-2fl)
-__device__ void add_sat(Big& acc, u64 n, const u64* s1, const u64* s2, int E, int fl, u64 T) {
-    big_add_L3(acc, s2, 2 * (E - 23), false);
+__device__ void add_sat(u64* acc, u64 n, const u64* s1, const u64* s2, int E, int fl, u64 T) {
+    col_add_L3(acc, s2, 2 * (E - 23), false);
     if (T) {
-        big_add_L3(acc, s1, E - 23 - fl, true, 2ull * T);
-        big_add(acc, mul128_64(U128{n, 0ull}, T * T), -2 * fl, false);
+        col_add_L3(acc, s1, E - 23 - fl, true, 2ull * T);
+        col_add(acc, mul128_64(U128{n, 0ull}, T * T), -2 * fl, false);
     }
 }
 
 // ------------------------------------------------------------------ finalize: scores, argmin, stats
-constexpr int FIN_T = 256;  // threads per finalize block; one block per cell
+constexpr int FIN_T = 256;            // threads per finalize block
+constexpr int FIN_WARPS = FIN_T / 32;  // cells per finalize block, one per warp
 
-// The keys with elements and the non-zero exponent sums of squares of one item, staged per block;
-// after the scoring, the lanes' 768-bit sums (word-major) reuse the moments' storage.
+// The keys with elements and the non-zero exponent sums of squares of one item, staged per block,
+// and every warp's column accumulator.
 struct FinSmem {
     unsigned nkey, nband, last;
     unsigned key[NKEY];
     u64 n[NKEY];
-    union {
-        struct {
-            u64 s1[NKEY][3];
-            u64 s2[NKEY][3];
-        } m;
-        u64 col[BW][FIN_T];
-    } u;
-    u64 part[BW][FIN_T / 16][2];  // column sums of 16 lanes: low word, carries
+    u64 s1[NKEY][3];
+    u64 s2[NKEY][3];
     unsigned beb[256];
     u64 band[256][3];
+    u64 col[FIN_WARPS][NCOL];
 };
-static_assert(sizeof(u64) * BW * FIN_T <= sizeof(u64) * NKEY * 6, "column buffer fits the moments' storage");
 
 __device__ void fin_stage(FinSmem& sm, const FsGlobal* g) {
     if (threadIdx.x == 0) sm.nkey = sm.nband = 0u;
@@ -768,8 +756,8 @@ __device__ void fin_stage(FinSmem& sm, const FsGlobal* g) {
         sm.n[i] = n;
 #pragma unroll
         for (int w = 0; w < 3; ++w) {
-            sm.u.m.s1[i][w] = g->ps1[key][w];
-            sm.u.m.s2[i][w] = g->ps2[key][w];
+            sm.s1[i][w] = g->ps1[key][w];
+            sm.s2[i][w] = g->ps2[key][w];
         }
     }
     for (int eb = threadIdx.x; eb < 256; eb += blockDim.x) {
@@ -784,24 +772,23 @@ __device__ void fin_stage(FinSmem& sm, const FsGlobal* g) {
     __syncthreads();
 }
 
-// The exact value of one cell (candidate (S, k, FL), or the two stats cells) in a warp's Big: lanes
-// split the staged keys, then the warp sums its lanes.
-__device__ void fin_cell(Big& acc, const FinSmem& sm, const FsGlobal* g, const FsFinal& F, int cell, int ncell,
+// The exact value of one cell (candidate (S, k, FL), or the two stats cells) added to a warp's
+// columns: the lanes split the staged keys.
+__device__ void fin_cell(u64* acc, const FinSmem& sm, const FsGlobal* g, const FsFinal& F, int cell, int ncell,
                          int lane, int nlanes) {
-    big_zero(acc);
     // the exponent-indexed sums of squares that belong to every L2 cell and to the sum of squares
     const bool with_band = cell == ncell + 1 || (cell < ncell && !F.l1);
     if (with_band)
-        for (unsigned i = lane; i < sm.nband; i += nlanes) big_add_L3(acc, sm.band[i], 2 * ((int)sm.beb[i] - 150), false);
+        for (unsigned i = lane; i < sm.nband; i += nlanes) col_add_L3(acc, sm.band[i], 2 * ((int)sm.beb[i] - 150), false);
     if (cell >= ncell) {
         const bool sq = cell == ncell + 1;
         for (unsigned i = lane; i < sm.nkey; i += nlanes) {
             const int key = (int)sm.key[i];
             const int eb = key & 255, E = eb ? eb - 127 : -126;
             if (sq)
-                big_add_L3(acc, sm.u.m.s2[i], 2 * (E - 23), false);
+                col_add_L3(acc, sm.s2[i], 2 * (E - 23), false);
             else
-                big_add_L3(acc, sm.u.m.s1[i], E - 23, (key >> 8) != 0);
+                col_add_L3(acc, sm.s1[i], E - 23, (key >> 8) != 0);
         }
     } else if (F.k_lo == 1 && F.S_lo + cell / (F.nk * F.nfl) == 1 && (cell % (F.nk * F.nfl)) / F.nfl == 0) {
         // k = 1, S = 1: the binary quantizer (Eq. fp_1_bit_quantization), every value decoded to
@@ -809,19 +796,19 @@ __device__ void fin_cell(Big& acc, const FinSmem& sm, const FsGlobal* g, const F
         const int fl = F.fl_lo + cell % F.nfl;
         if (lane == 0) {
             const U128 nz{g->nzero, 0ull};
-            big_add(acc, nz, F.l1 ? -fl : -2 * fl, false);
+            col_add(acc, nz, F.l1 ? -fl : -2 * fl, false);
         }
         for (unsigned i = lane; i < sm.nkey; i += nlanes) {
             const int key = (int)sm.key[i];
             const u64 n = sm.n[i];
             const int eb = key & 255, E = eb ? eb - 127 : -126;
             if (!F.l1) {
-                add_sat(acc, n, sm.u.m.s1[i], sm.u.m.s2[i], E, fl, 1ull);  // sum (|x| - c)^2
+                add_sat(acc, n, sm.s1[i], sm.s2[i], E, fl, 1ull);  // sum (|x| - c)^2
             } else {
                 // |x| >= 2^E >= c when E >= -fl, else |x| < 2^(E+1) <= c
                 const bool above = E >= -fl;
-                big_add_L3(acc, sm.u.m.s1[i], E - 23, !above);
-                big_add(acc, U128{n, 0ull}, -fl, above);
+                col_add_L3(acc, sm.s1[i], E - 23, !above);
+                col_add(acc, U128{n, 0ull}, -fl, above);
             }
         }
     } else {
@@ -836,10 +823,10 @@ __device__ void fin_cell(Big& acc, const FinSmem& sm, const FsGlobal* g, const F
             const int key = (int)sm.key[i];
             const u64 n = sm.n[i];
             const int sg = key >> 8, eb = key & 255, E = eb ? eb - 127 : -126;
-            const u64* s1 = sm.u.m.s1[i];
-            const u64* s2 = sm.u.m.s2[i];
+            const u64* s1 = sm.s1[i];
+            const u64* s2 = sm.s2[i];
             if (sg == 1 && S == 0) {  // clipped to code 0: error |x|
-                big_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
+                col_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
                 continue;
             }
             const int t = (sg == 0) ? (S ? k - 1 : k) : (k - 1);
@@ -847,17 +834,17 @@ __device__ void fin_cell(Big& acc, const FinSmem& sm, const FsGlobal* g, const F
             const int q = E + fl;
             if (q >= t) {
                 if (F.l1) {  // |x| >= T 2^-fl: sum |x| - n T 2^-fl
-                    big_add_L3(acc, s1, E - 23, false);
-                    big_add(acc, U128{n * T, 0ull}, -fl, true);
+                    col_add_L3(acc, s1, E - 23, false);
+                    col_add(acc, U128{n * T, 0ull}, -fl, true);
                 } else {
                     add_sat(acc, n, s1, s2, E, fl, T);
                 }
             } else if (sg == 0 && q == t - 1) {
-                big_add_L3(acc, g->rb[q + 1][fi], pw * (E - 23), false);
+                col_add_L3(acc, g->rb[q + 1][fi], pw * (E - 23), false);
             } else if (q <= -2) {
-                big_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
+                col_add_L3(acc, F.l1 ? s1 : s2, pw * (E - 23), false);
             } else {
-                big_add_L3(acc, g->r[sg][q + 1][fi], pw * (E - 23), false);
+                col_add_L3(acc, g->r[sg][q + 1][fi], pw * (E - 23), false);
             }
         }
     }
@@ -874,10 +861,11 @@ struct FsOutBatch {
     FsOut o[FS_MAX_ITEMS];
 };
 
-// Finalize: one block per cell of one item (the cells of every S, k, FL, then the two stats cells).
-// Every thread scores its share of the staged keys, and the block adds the lanes' 768-bit sums by
-// columns of words with one carry pass; the item's last block to finish (completion ticket) writes
-// the scores, the argmin per wordlength (exact ties keep the smaller FL) and the stats.
+// Finalize: one warp per cell of one item (the cells of every S, k, FL, then the two stats cells),
+// FIN_WARPS cells per block.  The block stages the item's keys once; each warp's lanes score their
+// share of the keys into the warp's columns, and lane 0 turns them into the exact 768-bit value and
+// its nearest double.  The item's last block to finish (completion ticket) writes the scores, the
+// argmin per wordlength (exact ties keep the smaller FL) and the stats.
 __global__ void __launch_bounds__(FIN_T) fl_search_final_kernel(const __grid_constant__ FsBatch B,
                                                                  const __grid_constant__ FsOutBatch O, int* status) {
     const int item = batch_item(B.fin0, B.n_items, (int)blockIdx.x);
@@ -886,60 +874,32 @@ __global__ void __launch_bounds__(FIN_T) fl_search_final_kernel(const __grid_con
     const FsOut& out = O.o[item];
     FsGlobal* g = P.g;
     __shared__ FinSmem sm;
-    const int cell = (int)blockIdx.x - B.fin0[item];
     const int nblk = B.fin0[item + 1] - B.fin0[item];
     const int ncell = (F.S_hi - F.S_lo + 1) * F.nk * F.nfl;
     const int tid = (int)threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int cell = ((int)blockIdx.x - B.fin0[item]) * FIN_WARPS + warp;
+    u64* col = sm.col[warp];
+    if (lane < NCOL) col[lane] = 0ull;
     fin_stage(sm, g);
-    {
-        Big acc;
-        fin_cell(acc, sm, g, F, cell, ncell, tid, FIN_T);
-        __syncthreads();  // the moments' storage becomes the column buffer
-#pragma unroll
-        for (int w = 0; w < BW; ++w) sm.u.col[w][tid] = acc.w[w];
-    }
-    __syncthreads();
-    if (tid < BW * 16) {  // 16-lane column sums of each word: the low word and its carries
-        const int w = tid >> 4, j = tid & 15;
-        u64 lo = 0ull, c = 0ull;
-        for (int l = 0; l < 16; ++l) {
-            const u64 v = sm.u.col[w][16 * j + l];
-            lo += v;
-            c += lo < v ? 1ull : 0ull;
-        }
-        sm.part[w][j][0] = lo;
-        sm.part[w][j][1] = c;
-    }
-    __syncthreads();
-    if (tid < BW) {  // whole columns: the low word and the carry into the next word
-        u64 lo = 0ull, c = 0ull;
-        for (int j = 0; j < 16; ++j) {
-            lo += sm.part[tid][j][0];
-            c += (lo < sm.part[tid][j][0] ? 1ull : 0ull) + sm.part[tid][j][1];
-        }
-        sm.part[tid][0][0] = lo;
-        sm.part[tid][1][1] = c;
-    }
-    __syncthreads();
-    if (tid == 0) {
-        Big acc;
-        u64 cin = 0ull;
-        for (int w = 0; w < BW; ++w) {  // modulo 2^768: the carry out of the top word drops
-            const u64 lo = sm.part[w][0][0] + cin;
-            acc.w[w] = lo;
-            cin = sm.part[w][1][1] + (lo < cin ? 1ull : 0ull);
-        }
-        if (cell == ncell) {
-            const bool neg = (long long)acc.w[BW - 1] < 0;
-            if (neg) big_negate(acc);
-            const double v = big_to_double(acc);
-            g->stat_sum = neg ? -v : v;
-        } else if (cell == ncell + 1) {
-            g->stat_sumsq = big_to_double(acc);
-        } else {
-            const int S = F.S_lo + cell / (F.nk * F.nfl);
-            const int rem = cell % (F.nk * F.nfl);
-            g->cells[S][F.k_lo + rem / F.nfl - 1][rem % F.nfl] = big_to_double(acc);
+    if (cell < ncell + 2) {  // warp-uniform
+        fin_cell(col, sm, g, F, cell, ncell, lane, 32);
+        __syncwarp();
+        if (lane == 0) {
+            Big acc;
+            col_to_big(col, acc);
+            if (cell == ncell) {
+                const bool neg = (long long)acc.w[BW - 1] < 0;
+                if (neg) big_negate(acc);
+                const double v = big_to_double(acc);
+                g->stat_sum = neg ? -v : v;
+            } else if (cell == ncell + 1) {
+                g->stat_sumsq = big_to_double(acc);
+            } else {
+                const int S = F.S_lo + cell / (F.nk * F.nfl);
+                const int rem = cell % (F.nk * F.nfl);
+                g->cells[S][F.k_lo + rem / F.nfl - 1][rem % F.nfl] = big_to_double(acc);
+            }
+            __threadfence();
         }
     }
     __syncthreads();
@@ -1093,10 +1053,11 @@ fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h
     h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0) |
                 (h.f.l1 ? 8 : 0);
     if (hs_configure(P, S_hi) && hs_fits(P)) {
-        // one block per SM, whole iterations per block except the last, at most HS_CHUNK_MAX each
+        // one block per SM with equal chunks (multiples of 4 elements: 16-byte aligned starts), at
+        // least one float4 per thread and at most HS_CHUNK_MAX elements each
         const long long waves = n > 0 ? (n + 152LL * HS_CHUNK_MAX - 1) / (152LL * HS_CHUNK_MAX) : 1;
         long long per = (n + 152 * waves - 1) / (152 * waves);
-        per = (per + HS_ITER - 1) / HS_ITER * HS_ITER;
+        per = (per + 3) / 4 * 4;
         if (per < HS_CHUNK_MIN) per = HS_CHUNK_MIN;
         if (per > HS_CHUNK_MAX) per = HS_CHUNK_MAX;
         P.chunk = (int)per;
@@ -1171,7 +1132,7 @@ fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
         B.fin0[j] = fblocks;
         const int nc = (it.f.S_hi - it.f.S_lo + 1) * it.f.nk * it.f.nfl + 2;
         cells += nc;
-        fblocks += nc;  // one finalize block per cell
+        fblocks += (nc + FIN_WARPS - 1) / FIN_WARPS;  // one finalize warp per cell
     }
     B.cell0[n] = cells;
     B.fin0[n] = fblocks;

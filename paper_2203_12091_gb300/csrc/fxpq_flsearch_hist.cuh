@@ -47,7 +47,7 @@ namespace {
 constexpr int HS_T = 1024;                 // threads per block (one block per SM)
 constexpr int HS_ITER = 16 * HS_T;         // elements per block iteration (four float4 per thread)
 constexpr int HS_CHUNK_MAX = 1 << 20;      // per-block elements: keeps stripe sums below 2^32
-constexpr int HS_CHUNK_MIN = 2 * HS_ITER;
+constexpr int HS_CHUNK_MIN = 4 * HS_T;  // at least one float4 per thread
 constexpr int HS_STRIPE = 16;              // per-key L^2 bins, by lane % 16
 constexpr unsigned HS_CNT_LIMIT = 65536u;  // a bin this full may have wrapped its 32-bit sum of L
 constexpr int HS_OVF_MAX = HS_CHUNK_MAX / (int)HS_CNT_LIMIT;
@@ -60,7 +60,8 @@ constexpr int HS_O_SL = HS_MAX_BINS + 32;
 constexpr int HS_O_L2LO = 2 * HS_O_SL;
 constexpr int HS_O_L2HI = HS_O_L2LO + 2 * HS_MAX_W * HS_STRIPE;
 constexpr int HS_O_MISC = HS_O_L2HI + 2 * HS_MAX_W * HS_STRIPE;
-constexpr int HS_MISC = 64;  // band, min, max, counters, overflow list and its 64-bit sums
+constexpr int HM_WSUM = 64;  // the warps' band sums (2 x 32 u64)
+constexpr int HS_MISC = HM_WSUM + 4 * (HS_T / 32);  // band, min, max, counters, overflow list and its 64-bit sums
 constexpr size_t HS_SMEM = (size_t)(HS_O_MISC + HS_MISC) * 4u;
 static_assert(HS_O_MISC % 2 == 0, "misc holds 64-bit sums");
 constexpr int HM_BAND = 0, HM_MN = 1, HM_MX = 2, HM_NOVF = 3, HM_COLD = 4, HM_NF = 5, HM_OVF_IDX = 8,
@@ -169,6 +170,13 @@ __device__ __forceinline__ u64 hs_wsum52(u64 v) {
     const unsigned lo = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v & 0x3FFFFFFull));
     const unsigned hi = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v >> 26));
     return (u64)lo + ((u64)hi << 26);
+}
+// Warp sum of per-lane values below 2^63 (three 21-bit pieces), exact in 128 bits.
+__device__ __forceinline__ unsigned __int128 hs_wsum128(u64 v) {
+    const unsigned a = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v & 0x1FFFFFull));
+    const unsigned b = __reduce_add_sync(0xFFFFFFFFu, (unsigned)((v >> 21) & 0x1FFFFFull));
+    const unsigned c = __reduce_add_sync(0xFFFFFFFFu, (unsigned)(v >> 42));
+    return (unsigned __int128)a + ((unsigned __int128)b << 21) + ((unsigned __int128)c << 42);
 }
 // ... of signed per-lane values with |v| < 2^45.
 __device__ __forceinline__ long long hs_wsum_s(long long v) {
@@ -371,6 +379,29 @@ __device__ __forceinline__ void hs_load4(const float* __restrict__ x, long long 
     }
 }
 
+// The same slots as hs_load4 for the block's last, partial iteration: the elements below `end`
+// (bit 4 q + c of the returned mask), zeros elsewhere.
+template <bool VEC>
+__device__ __forceinline__ unsigned hs_load4p(const float* __restrict__ x, long long i0, long long end,
+                                              uint4 (&d)[4]) {
+    unsigned m = 0u;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const long long i = i0 + 4LL * HS_T * q;
+        d[q] = make_uint4(0u, 0u, 0u, 0u);
+        if (VEC && i + 4 <= end) {
+            d[q] = __ldg(reinterpret_cast<const uint4*>(x + i));
+            m |= 0xFu << (4 * q);
+        } else {
+            if (i < end) d[q].x = __float_as_uint(__ldg(x + i)), m |= 1u << (4 * q);
+            if (i + 1 < end) d[q].y = __float_as_uint(__ldg(x + i + 1)), m |= 2u << (4 * q);
+            if (i + 2 < end) d[q].z = __float_as_uint(__ldg(x + i + 2)), m |= 4u << (4 * q);
+            if (i + 3 < end) d[q].w = __float_as_uint(__ldg(x + i + 3)), m |= 8u << (4 * q);
+        }
+    }
+    return m;
+}
+
 template <bool VEC, bool L1>
 __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_constant__ FsBatch B, int item0, int item1) {
     const int item = item0 + batch_item(B.blk0 + item0, item1 - item0, (int)blockIdx.x);
@@ -379,6 +410,7 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
     extern __shared__ __align__(16) unsigned hs_smem[];
     unsigned* misc = hs_smem + HS_O_MISC;
     u64* ovf_sum = reinterpret_cast<u64*>(misc + HM_OVF_SUM);
+    u64* wsum = reinterpret_cast<u64*>(misc + HM_WSUM);
     const unsigned tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
     FsGlobal* g = P.g;
     const HsLayout Ly = hs_layout(P);
@@ -400,6 +432,8 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
 
     const long long start = (long long)blk * P.chunk;
     const long long end = min(start + (long long)P.chunk, P.n);
+    // whole iterations, then at most one partial one
+    const long long nit = end > start ? (end - start + HS_ITER - 1) / HS_ITER : 0;
     const long long nfull = end > start ? (end - start) / HS_ITER : 0;
     HsLane st;
     st.acc0 = st.acc1 = 0ull;
@@ -408,21 +442,23 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
     unsigned nout = 0u;
 
     uint4 va[4], vb[4];
+    unsigned ma = 0xFFFFu;  // valid elements of the first iteration
     const long long t0 = start + 4LL * tid;
-    if (nfull > 0) hs_load4<VEC>(P.x, t0, va);
+    if (nfull > 0)
+        hs_load4<VEC>(P.x, t0, va);
+    else
+        ma = nit > 0 ? hs_load4p<VEC>(P.x, t0, end, va) : 0u;
     // the block's band: up to 16 exponents of the window ending at the largest window exponent of its
     // first iteration
     {
         unsigned m = 0u;
-        if (nfull > 0) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const unsigned w4[4] = {va[q].x, va[q].y, va[q].z, va[q].w};
+        for (int q = 0; q < 4; ++q) {
+            const unsigned w4[4] = {va[q].x, va[q].y, va[q].z, va[q].w};
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const unsigned zw = (w4[c] << 1) - K.eblo24;
-                    if (zw < K.w24) m = max(m, (w4[c] >> 23) & 0xFFu);
-                }
+            for (int c = 0; c < 4; ++c) {
+                const unsigned zw = (w4[c] << 1) - K.eblo24;
+                if (((ma >> (4 * q + c)) & 1u) && zw < K.w24) m = max(m, (w4[c] >> 23) & 0xFFu);
             }
         }
         m = __reduce_max_sync(0xFFFFFFFFu, m);
@@ -440,15 +476,7 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
 
     // One group of 16 elements as a single basic block; the rare ones that need the cold pass are
     // marked in a mask and handled after the group, each at a compile-time register index.
-    auto body = [&](const uint4 (&v)[4]) {
-        unsigned cm = 0u;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            cm |= hs_elem(v[q].x, hs_smem, K, st) ? 1u << (4 * q) : 0u;
-            cm |= hs_elem(v[q].y, hs_smem, K, st) ? 2u << (4 * q) : 0u;
-            cm |= hs_elem(v[q].z, hs_smem, K, st) ? 4u << (4 * q) : 0u;
-            cm |= hs_elem(v[q].w, hs_smem, K, st) ? 8u << (4 * q) : 0u;
-        }
+    auto cold = [&](const uint4 (&v)[4], unsigned cm) {
         if (cm) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -459,6 +487,17 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
             }
         }
     };
+    auto body = [&](const uint4 (&v)[4]) {
+        unsigned cm = 0u;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            cm |= hs_elem(v[q].x, hs_smem, K, st) ? 1u << (4 * q) : 0u;
+            cm |= hs_elem(v[q].y, hs_smem, K, st) ? 2u << (4 * q) : 0u;
+            cm |= hs_elem(v[q].z, hs_smem, K, st) ? 4u << (4 * q) : 0u;
+            cm |= hs_elem(v[q].w, hs_smem, K, st) ? 8u << (4 * q) : 0u;
+        }
+        cold(v, cm);
+    };
     // two buffers in rotation: one iteration of loads in flight (1024 threads x 64 B per SM) while the
     // other is binned
     for (long long it = 0; it < nfull; it += 2) {
@@ -468,10 +507,18 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
         if (it + 2 < nfull) hs_load4<VEC>(P.x, t0 + (it + 2) * HS_ITER, va);
         body(vb);
     }
-    // ragged tail, element by element
-    for (long long i = start + nfull * HS_ITER + tid; i < end; i += HS_T) {
-        const unsigned u = __float_as_uint(__ldg(P.x + i));
-        if (hs_elem(u, hs_smem, K, st)) nout += hs_cold(u, K, hs_smem, g, lane);
+    // the partial iteration (the only one of a chunk below HS_ITER elements): its valid elements
+    if (nit > nfull) {
+        if (nfull > 0) ma = hs_load4p<VEC>(P.x, t0 + nfull * HS_ITER, end, va);
+        unsigned cm = 0u;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if ((ma >> (4 * q)) & 1u) cm |= hs_elem(va[q].x, hs_smem, K, st) ? 1u << (4 * q) : 0u;
+            if ((ma >> (4 * q)) & 2u) cm |= hs_elem(va[q].y, hs_smem, K, st) ? 2u << (4 * q) : 0u;
+            if ((ma >> (4 * q)) & 4u) cm |= hs_elem(va[q].z, hs_smem, K, st) ? 4u << (4 * q) : 0u;
+            if ((ma >> (4 * q)) & 8u) cm |= hs_elem(va[q].w, hs_smem, K, st) ? 8u << (4 * q) : 0u;
+        }
+        cold(va, cm);
     }
 
     // per-lane results: stats, band sums, elements outside the window that were not zeros
@@ -483,11 +530,18 @@ __global__ void __launch_bounds__(HS_T, 1) fl_search_hist_kernel(const __grid_co
             atomicMin(&misc[HM_MN], mn);
             atomicMax(&misc[HM_MX], mx);
             if (no) atomicAdd(&misc[HM_COLD], no);
-            gaddL(g->cband[band], a0);
-            gaddL(g->cband[band + 8u], a1);
+            wsum[warp] = a0;
+            wsum[HS_T / 32 + warp] = a1;
         }
     }
     __syncthreads();
+    if (warp == 0) {  // the block's band sums (< 2^66), one workspace add each
+        const unsigned __int128 b0 = hs_wsum128(wsum[lane]), b1 = hs_wsum128(wsum[HS_T / 32 + lane]);
+        if (lane == 0) {
+            gaddLs(g->cband[band], (__int128)b0);
+            gaddLs(g->cband[band + 8u], (__int128)b1);
+        }
+    }
     if (misc[HM_NF]) {
         // a non-finite value reached the order keys: take min and max again over the finite ones
         __syncthreads();

@@ -2,6 +2,7 @@
 // edges).  Host-side driver: derives every slot's shape, carves the slots out of the caller's
 // workspace, and launches the C-Block kernels in order on the caller's stream.
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "fxpq_common.cuh"
@@ -233,7 +234,7 @@ namespace {
 
 struct CalibLayout {
     std::vector<Slot> slots;
-    size_t slots_bytes = 0, f32_off = 0, fls_off = 0, rec_off = 0, err_off = 0, cws_off = 0, cws = 0, total = 0;
+    size_t slots_bytes = 0, f32_off = 0, fls_off = 0, err_off = 0, cws_off = 0, cws = 0, total = 0;
 };
 
 fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
@@ -250,30 +251,72 @@ fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
     const size_t img = (size_t)n * net->C * net->H * net->W;
     L.f32_off = L.slots_bytes;
     L.fls_off = L.f32_off + align256((max_out > img ? max_out : img) * sizeof(float));
-    L.rec_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
-    L.err_off = L.rec_off + 256;
+    L.err_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
     L.cws_off = L.err_off + align256(32 * sizeof(double));
     L.cws = net_conv_ws(net, L.slots, n);
     L.total = L.cws_off + L.cws;
     return FXPQ_OK;
 }
 
+// Mapped pinned host records: the FL search's final kernel writes the chosen FL and the stats
+// straight into host memory, so that the calibration reads them after a stream synchronisation
+// with no copy in between.  A small pool, one record per running calibration, kept for the
+// process's lifetime.
+struct HostRec {
+    unsigned char* h = nullptr;  // host address
+    unsigned char* d = nullptr;  // its device address
+};
+constexpr size_t kHostRecBytes = 256;
+static_assert(64 + sizeof(fxpq_stats) <= kHostRecBytes, "the record holds the FL and the stats");
+std::mutex g_rec_mu;
+std::vector<HostRec> g_rec_free;
+
+struct HostRecLease {
+    HostRec r;
+    bool ok = false;
+    HostRecLease() {
+        {
+            std::lock_guard<std::mutex> lk(g_rec_mu);
+            if (!g_rec_free.empty()) {
+                r = g_rec_free.back();
+                g_rec_free.pop_back();
+                ok = true;
+                return;
+            }
+        }
+        void* h = nullptr;
+        void* d = nullptr;
+        if (cudaHostAlloc(&h, kHostRecBytes, cudaHostAllocMapped | cudaHostAllocPortable) != cudaSuccess) return;
+        if (cudaHostGetDevicePointer(&d, h, 0) != cudaSuccess) {
+            cudaFreeHost(h);
+            return;
+        }
+        r.h = static_cast<unsigned char*>(h);
+        r.d = static_cast<unsigned char*>(d);
+        ok = true;
+    }
+    ~HostRecLease() {
+        if (!ok) return;
+        std::lock_guard<std::mutex> lk(g_rec_mu);
+        g_rec_free.push_back(r);
+    }
+    HostRecLease(const HostRecLease&) = delete;
+    HostRecLease& operator=(const HostRecLease&) = delete;
+};
+
 // FL search of one fp32 tensor at wordlength k, S picked from the data; waits for the result.
 fxpq_status calib_search(const float* d_x, int64_t n, int k, int fl_lo, int fl_hi, char* base, const CalibLayout& L,
-                         cudaStream_t s, fxpq_fmt& out) {
-    int32_t* d_best = reinterpret_cast<int32_t*>(base + L.rec_off);
-    fxpq_stats* d_stats = reinterpret_cast<fxpq_stats*>(base + L.rec_off + 64);
+                         const HostRec& rec, cudaStream_t s, fxpq_fmt& out) {
+    int32_t* d_best = reinterpret_cast<int32_t*>(rec.d);
+    fxpq_stats* d_stats = reinterpret_cast<fxpq_stats*>(rec.d + 64);
     fxpq_status st = fxpq_fl_search(d_x, n, -1, k, k, fl_lo, fl_hi, reinterpret_cast<double*>(base + L.err_off),
                                     d_best, d_stats, base + L.fls_off, fxpq_fl_search_workspace(n), s);
     if (st != FXPQ_OK) return st;
-    unsigned char rec[64 + sizeof(fxpq_stats)];
-    if (cudaMemcpyAsync(rec, base + L.rec_off, sizeof(rec), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-        cudaStreamSynchronize(s) != cudaSuccess)
-        return FXPQ_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FXPQ_ERR_CUDA;
     int32_t best;
     fxpq_stats stats;
-    memcpy(&best, rec, sizeof(best));
-    memcpy(&stats, rec + 64, sizeof(stats));
+    memcpy(&best, rec.h, sizeof(best));
+    memcpy(&stats, rec.h + 64, sizeof(stats));
     out.bits = k;
     out.is_signed = stats.is_signed;
     out.fl = best;
@@ -301,11 +344,13 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
     char* base = static_cast<char*>(d_ws);
     auto ptr = [&](int slot) { return static_cast<void*>(base + L.slots[slot].offset); };
     float* f32 = reinterpret_cast<float*>(base + L.f32_off);
+    HostRecLease lease;
+    if (!lease.ok) return FXPQ_ERR_CUDA;
     std::vector<fxpq_fmt> fmt(h_net->n_slots, fxpq_fmt{0, 0, 0});
 
     // input FxP-QLayer: FL search on the fp32 images, then the codes
     const int64_t n_img = (int64_t)n_calib * h_net->C * h_net->H * h_net->W;
-    st = calib_search(d_calib_nchw, n_img, h_net->fmt_in.bits, fl_lo, fl_hi, base, L, s, fmt[0]);
+    st = calib_search(d_calib_nchw, n_img, h_net->fmt_in.bits, fl_lo, fl_hi, base, L, lease.r, s, fmt[0]);
     if (st != FXPQ_OK) return st;
     *h_fmt_in = fmt[0];
     st = fxpq_quantize_images(d_calib_nchw, n_calib, h_net->C, h_net->H, h_net->W, fmt[0], h_net->Cp_in, ptr(0), s);
@@ -356,7 +401,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 int32_t sc = 0;
                 void* cws = L.cws ? base + L.cws_off : nullptr;
                 st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, f32, &sc, cws, L.cws, s);
-                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, lease.r, s, fy);
                 if (st == FXPQ_OK) {
                     cd.out_mode = FXPQ_OUT_CODES;
                     cd.fmt_y = fy;
@@ -368,7 +413,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 const int64_t npix = (int64_t)n_calib * s0.H * s0.W;
                 st = fxpq_eltwise(ptr(o.src0), fmt[o.src0], ptr(o.src1), fmt[o.src1], npix, s0.Cp, o.relu, FXPQ_OUT_F32,
                                   fy, f32, nullptr, s);
-                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, lease.r, s, fy);
                 if (st == FXPQ_OK)
                     st = fxpq_eltwise(ptr(o.src0), fmt[o.src0], ptr(o.src1), fmt[o.src1], npix, s0.Cp, o.relu,
                                       FXPQ_OUT_CODES, fy, ptr(o.dst), nullptr, s);
@@ -377,7 +422,7 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
             case FXPQ_OP_AVGPOOL:
                 st = fxpq_avgpool(ptr(o.src0), n_calib, s0.H, s0.W, s0.Cp, fmt[o.src0], o.recip_code, o.fmt_w,
                                   FXPQ_OUT_F32, fy, f32, nullptr, s);
-                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, s, fy);
+                if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, lease.r, s, fy);
                 if (st == FXPQ_OK)
                     st = fxpq_avgpool(ptr(o.src0), n_calib, s0.H, s0.W, s0.Cp, fmt[o.src0], o.recip_code, o.fmt_w,
                                       FXPQ_OUT_CODES, fy, ptr(o.dst), nullptr, s);
