@@ -423,10 +423,10 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
                                      (int)tc_smem_bytes<256>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)tc_smem_bytes<256>()) != cudaSuccess ||
-                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true, true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
-                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, false, true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes<256>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<256, true>()) != cudaSuccess ||
+                cudaFuncSetAttribute(conv_tc_kernel<256, int, false, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)tc_smem_bytes<256, true>()) != cudaSuccess ||
                 cudaFuncSetAttribute(conv_tc_kernel<64, long long, false, false, false, true>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)(tc_smem_bytes<64>() + 64 * TC_BM * 2)) != cudaSuccess ||
@@ -450,9 +450,9 @@ fxpq_status launch_conv_tc(const ConvArgs& a, const fxpq_conv_desc& d, cudaStrea
         return FXPQ_OK;
     }
     else if (P.pk && P.ksplit > 1)
-        conv_tc_kernel<256, int, false, true, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
+        conv_tc_kernel<256, int, false, true, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256, true>(), st>>>(P);
     else if (P.pk)
-        conv_tc_kernel<256, int, false, false, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256>(), st>>>(P);
+        conv_tc_kernel<256, int, false, false, true><<<grid, tc_threads_pk(256, true), tc_smem_bytes<256, true>(), st>>>(P);
     else if (P.ksplit > 1 && BN == 256)
         conv_tc_kernel<256, int, false, true><<<grid, tc_threads(256), tc_smem_bytes<256>(), st>>>(P);
     else if (P.ksplit > 1 && acc64)

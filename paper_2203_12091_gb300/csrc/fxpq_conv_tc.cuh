@@ -43,13 +43,19 @@ namespace tc {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;  // fp16 elements per k-block row = 128 bytes (one swizzle atom row)
-// Pipeline depth: 6 stages of 32 KB (BN <= 128) or 3 of 48 KB (BN = 256, whose 64 KB output staging
-// leaves no room for a fourth).
-__host__ __device__ constexpr int tc_stages(int BN) { return BN == 256 ? 3 : 6; }
+// Pipeline depth: 6 stages of 32 KB (BN <= 128); 4 of 48 KB for BN = 256, whose one-plane codes are
+// stored through per-warp 2 KB slices (no TMA-store staging of the whole tile) so that the output
+// staging keeps only 32 KB; 3 for the packed-weight instance, whose packed stages take the 64 KB
+// staging region.  (The 256-column layers lose about a fifth of their speed from 3 stages to 2: the
+// copies' latency, not the tensor pipe, bounds them at this depth.)
+__host__ __device__ constexpr int tc_stages(int BN, bool PK = false) { return BN == 256 ? (PK ? 3 : 4) : 6; }
+// Output staging bytes: BN / 64 boxes of 128 rows x 128 bytes for the TMA-store epilogue, 32 KB where
+// the codes are stored directly (BN = 256 without packed weights).
+__host__ __device__ constexpr int tc_out_bytes(int BN, bool PK = false) { return (BN == 256 && !PK) ? 32768 : BN * TC_BM * 2; }
 // Row-tile producers arrive on a stage this many k-blocks after issuing its copies (cp.async groups
 // in flight).  It must stay below the stage count: a producer waiting for a stage to be consumed
 // must already have arrived on it.
-__host__ __device__ constexpr int tc_lag(int BN) { return tc_stages(BN) - 1 < 3 ? tc_stages(BN) - 1 : 3; }
+__host__ __device__ constexpr int tc_lag(int BN, bool PK = false) { return tc_stages(BN, PK) - 1 < 3 ? tc_stages(BN, PK) - 1 : 3; }
 // Warps: 4 producers, epilogue warps (four per 32-column chunk group: one per TMEM lane quadrant;
 // BN / 8 of them up to 16, each then draining BN / 128 chunks), one MMA / TMEM-allocation warp.
 __host__ __device__ constexpr int tc_epi_warps(int BN) { return BN / 8 < 16 ? BN / 8 : 16; }
@@ -70,10 +76,12 @@ constexpr int TC_W64_SO = 180 * 1024;
 constexpr size_t tc_smem_w64() { return 1024 + TC_W64_SO + 2 * 64 * TC_BM * 2 + 256; }
 __host__ __device__ constexpr int tc_threads_win() { return (5 + TC_WIN_EPI_WARPS) * 32; }
 // Dynamic shared memory: barriers, the stages (A and B tiles), the output staging tile.
-template <int BN>
+template <int BN, bool PK = false>
 constexpr size_t tc_smem_bytes() {
-    return 1024 + tc_stages(BN) * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + BN * TC_BM * 2 + 256;
+    return 1024 + tc_stages(BN, PK) * (TC_BM * TC_BK * 2 + BN * TC_BK * 2) + tc_out_bytes(BN, PK) + 256;
 }
+static_assert(tc_smem_bytes<256>() <= 232448 && tc_smem_bytes<256, true>() <= 232448 && tc_smem_bytes<128>() <= 232448,
+              "dynamic shared memory within the 227 KB a CTA may use");
 constexpr int TC_MAX_GROUPS = 64;
 constexpr int TC_MAX_SPLIT = 16;
 constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
@@ -82,7 +90,9 @@ constexpr long long TC_WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
 // order, and its parity wait on the stage's `empty` barrier is never more than one phase ahead of it.
 // (A parity wait two phases ahead reads as complete: with k-blocks dealt round-robin, more producers
 // than stages could refill a stage before its data was consumed.)
-__host__ __device__ constexpr int tc_producers(int BN) { return tc_stages(BN) % 2 == 0 ? 2 : tc_stages(BN); }
+__host__ __device__ constexpr int tc_producers(int BN, bool PK = false) {
+    return tc_stages(BN, PK) <= 4 ? tc_stages(BN, PK) : 2;
+}
 
 struct TcGroup {
     int kb0, kb1;          // k-block range within a plane
@@ -154,6 +164,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// The non-blocking probe, for the thread that issues the MMAs: a try_wait there stalls the issuing
+// thread until its queued MMAs have drained (about 230 cycles per k-block of four 128-column MMAs, half
+// the tensor rate), a test_wait costs about 45.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
@@ -315,12 +340,14 @@ __device__ __forceinline__ void pk_convert_stage(const uint32_t* pk, unsigned ch
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
 // timeout status, sets the CTA abort flag) if it gave up or another role already aborted.
+template <bool TEST = false>
 __device__ __forceinline__ bool wait_bounded_for(uint32_t bar, uint32_t parity, volatile int* abort, int* status,
                                                  long long limit) {
-    if (mbar_try_wait(bar, parity)) return true;
+    auto probe = [&]() { return TEST ? mbar_test_wait(bar, parity) : mbar_try_wait(bar, parity); };
+    if (probe()) return true;
     const long long t0 = clock64();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (probe()) return true;
         if (*abort) return false;
         if (clock64() - t0 > limit) {
             *abort = 1;
@@ -332,6 +359,10 @@ __device__ __forceinline__ bool wait_bounded_for(uint32_t bar, uint32_t parity, 
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
     return wait_bounded_for(bar, parity, abort, status, TC_WAIT_CYCLES);
+}
+// the same for the MMA-issuing thread (non-blocking probes)
+__device__ __forceinline__ bool wait_mma(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
+    return wait_bounded_for<true>(bar, parity, abort, status, TC_WAIT_CYCLES);
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
@@ -603,7 +634,7 @@ __device__ __forceinline__ uint32_t pack_codes_f16(int c0, int c1) {
 template <int BN, bool SPLIT>
 __device__ __forceinline__ void pk_convert_loop(const TcParams& P, int cid, int lane, const unsigned char* sP,
                                                 unsigned char* sB, uint32_t pkfull0, uint32_t full0, volatile int* abort) {
-    constexpr int STAGES = tc_stages(BN);
+    constexpr int STAGES = tc_stages(BN, true);
     constexpr int B_BYTES = BN * TC_BK * 2;
     const int k = P.wk;
     const uint32_t flip = P.wsigned ? 0x01010101u * (1u << (k - 1)) : 0u;
@@ -638,13 +669,16 @@ __device__ __forceinline__ void pk_convert_loop(const TcParams& P, int cid, int 
 template <int BN, typename ACC, bool SC, bool SPLIT = false, bool PK = false, bool WIN = false, bool W64 = false>
 __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_pk(BN, PK), 1)
     conv_tc_kernel(const __grid_constant__ TcParams P) {
-    constexpr int TC_STAGES = tc_stages(BN);
-    constexpr int TC_LAG = tc_lag(BN);
+    constexpr int TC_STAGES = tc_stages(BN, PK);
+    constexpr int TC_LAG = tc_lag(BN, PK);
+    // 256-column tiles without packed weights store their one-plane codes with plain stores through
+    // each warp's 2 KB slice of the staging region rather than by TMA stores of a whole staged tile
+    constexpr bool DIRECT = BN == 256 && !PK;
     static_assert(TC_LAG >= 1 && TC_LAG < TC_STAGES, "producer lag must be below the stage count");
     static_assert(!PK || (BN == 256 && sizeof(ACC) == 4 && !SC), "packed weights: 256-column int32 tiles only");
-    static_assert(!PK || TC_STAGES * BN * 64 <= BN * TC_BM * 2, "packed stages must fit the staging region");
+    static_assert(!PK || TC_STAGES * BN * 64 <= tc_out_bytes(BN, PK), "packed stages must fit the staging region");
     // PK: one issuing thread (producer warp 0), so its stage waits are in order by construction
-    constexpr int TC_PRODUCERS = PK ? 1 : tc_producers(BN);
+    constexpr int TC_PRODUCERS = PK ? 1 : tc_producers(BN, PK);
     static_assert(TC_STAGES % TC_PRODUCERS == 0 && TC_PRODUCERS <= 4,
                   "each stage must have one producer thread among warps 0..3");
     static_assert(!WIN || (BN == 64 && sizeof(ACC) == 8 && !SC && !SPLIT && !PK), "window instance: BN = 64, int64");
@@ -652,6 +686,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
     constexpr bool WEPI = WIN || W64;  // the window instances' epilogue (16 warps, two staging tiles)
     constexpr int EPI_WARPS = WEPI ? TC_WIN_EPI_WARPS : tc_epi_warps(BN);
     constexpr int EPI_THREADS = 32 * EPI_WARPS;
+    static_assert(WEPI || tc_out_bytes(BN, PK) >= EPI_WARPS * 2048, "the staged fp32 / int64 epilogue takes 2 KB per warp");
     constexpr int MMA_WARP = 4 + EPI_WARPS;
     constexpr int CPW = WEPI ? 1 : (BN / 32) / (EPI_WARPS / 4);  // 32-column chunks per epilogue warp
     constexpr int A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
@@ -668,7 +703,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
     unsigned char* sB = base + TC_STAGES * A_BYTES;
     unsigned char* sO = W64 ? base + TC_W64_SO : sB + TC_STAGES * B_BYTES;  // output staging: BN/64 halves of
                                                                          // [128 rows][64 codes]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + BN * TC_BM * 2 * (WEPI ? 2 : 1));  // WEPI: two staging tiles
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sO + (WEPI ? 2 * BN * TC_BM * 2 : tc_out_bytes(BN, PK)));  // WEPI: two staging tiles
     // bars: full[STAGES], empty[STAGES], accfull[2], accempty[2], done
     volatile int* abort = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
@@ -1190,7 +1225,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                     break;
                 }
                 tc_fence_after();
-                if (last && P.fast_store && u > 0) {
+                if (!DIRECT && last && P.fast_store && u > 0) {
                     // the previous tile's TMA store must have read the staging buffer
                     if (leader) {
                         bulk_wait_read0();
@@ -1496,6 +1531,29 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                                 w[j] = pack_codes_f16(c2[0], c2[1]);
                             }
                         }
+                        if (DIRECT) {
+                            // through the warp's 2 KB slice of the staging region: each lane puts its row's
+                            // 64 bytes there (16-byte pieces rotated against bank conflicts), then every
+                            // store instruction writes whole 64-byte row segments of eight rows.  One-plane
+                            // codes have K % 8 == 0, so a 16-byte piece lies wholly inside or past K.
+                            unsigned char* wbuf = sO + (warp - 4) * 2048;
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                *reinterpret_cast<uint4*>(wbuf + lane * 64 + 16 * (q ^ ((lane >> 1) & 3))) =
+                                    make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+                            __syncwarp();
+#pragma unroll
+                            for (int it = 0; it < 4; ++it) {
+                                const int r = (lane >> 2) + 8 * it, pc = lane & 3;
+                                const long long mr = __shfl_sync(0xffffffffu, m, r);
+                                const uint4 v = *reinterpret_cast<const uint4*>(wbuf + r * 64 + 16 * (pc ^ ((r >> 1) & 3)));
+                                const int kk = k0 + pc * 8;
+                                if (mr >= 0 && kk < a.K)
+                                    *reinterpret_cast<uint4*>(static_cast<__half*>(a.y) + mr * a.K + kk) = v;
+                            }
+                            __syncwarp();
+                            continue;
+                        }
                         unsigned char* half_buf = sO + (cb >> 1) * (TC_BM * 128);
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {
@@ -1511,7 +1569,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                     }
                 }
                 ++gcount;
-                if (last && P.fast_store) {
+                if (!DIRECT && last && P.fast_store) {
                     // make the staging writes visible to the async proxy, then one thread stores the tile
                     fence_proxy_async();
                     __syncwarp();
@@ -1549,12 +1607,12 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
         // block (a B stage's layout).  One barrier round per tile.
         const uint32_t copyb = (uint32_t)P.WH * 1024u;
         uint32_t stage = 0, phase = 0, gcount = 0;
-        bool ok = wait_bounded(wbar, 0, abort, P.status);
+        bool ok = wait_mma(wbar, 0, abort, P.status);
         tc_fence_after();
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x) {
             const uint32_t buf = gcount & 1;
-            if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
-                !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
+            if (!wait_mma(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
+                !wait_mma(full0 + 8 * stage, phase, abort, P.status)) {
                 ok = false;
                 break;
             }
@@ -1605,14 +1663,14 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
             aoff[i] = (uint32_t)((r * P.WW + 2 * sp) * 16) >> 4;
         }
         uint32_t stage = 0, phase = 0, gcount = 0;
-        bool ok = wait_bounded(wbar, 0, abort, P.status);
+        bool ok = wait_mma(wbar, 0, abort, P.status);
         tc_fence_after();
         for (int ut = blockIdx.x; ut < (SPLIT ? P.n_units : P.n_tiles) && ok; ut += gridDim.x) {
             const int t = SPLIT ? ut / P.ksplit : ut, sp = SPLIT ? ut - t * P.ksplit : 0;
             (void)sp;
             const uint32_t buf = gcount & 1;
-            if (!wait_bounded(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
-                !wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
+            if (!wait_mma(accempty0 + 8 * buf, ((gcount >> 1) & 1) ^ 1, abort, P.status) ||
+                !wait_mma(full0 + 8 * stage, phase, abort, P.status)) {
                 ok = false;
                 break;
             }
@@ -1659,7 +1717,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 const TcGroup g = P.g[gi];
                 const uint32_t buf = P.nbuf == 2 ? (gcount & 1) : 0;
                 const uint32_t par = P.nbuf == 2 ? ((gcount >> 1) & 1) : (gcount & 1);
-                if (!wait_bounded(accempty0 + 8 * buf, par ^ 1, abort, P.status)) {
+                if (!wait_mma(accempty0 + 8 * buf, par ^ 1, abort, P.status)) {
                     ok = false;
                     break;
                 }
@@ -1667,7 +1725,7 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 const uint32_t d = tmem + buf * BN;
                 uint32_t accum = 0;
                 for (int kb = g.kb0; kb < g.kb1; ++kb) {
-                    if (!wait_bounded(full0 + 8 * stage, phase, abort, P.status)) {
+                    if (!wait_mma(full0 + 8 * stage, phase, abort, P.status)) {
                         ok = false;
                         break;
                     }
