@@ -1052,6 +1052,20 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
         const int lo = (int)a.lo, hi = (int)a.hi;
         const int per_img = P.tiles_p * P.tiles_q;
         const bool f32out = a.out_mode == FXPQ_OUT_F32;  // the fp32 image (calibration) instead of codes
+        // W64, 32-bit codes: a thread's 16 output channels are the same in every tile, so their aligned
+        // bias terms and the flags of bias bits below the accumulator's scale are formed once
+        const Epi32 e32w = make_epi32(a);
+        int btw[16];
+        uint32_t phiw = 0u;
+        if (W64) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                const int k = cw * 16 + j;
+                const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                btw[j] = (b << e32w.bsl) >> e32w.bsr;
+                phiw |= ((b & e32w.fmask) != 0 ? 1u : 0u) << j;
+            }
+        }
         bool ok = true;
         uint32_t u = 0;
         for (int t = blockIdx.x; t < P.n_tiles && ok; t += gridDim.x, ++u) {
@@ -1070,8 +1084,6 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(accempty0 + 8 * buf);
-                const Epi32 e32 = make_epi32(a);
-                const Epi64 e64 = make_epi64(a);
                 if (f32out) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
@@ -1081,18 +1093,31 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                         w[j] = __float_as_uint(__ll2float_rn(cblock_value<false>(a, k, (long long)acc, b)) * a.f32_scale);
                     }
                 }
+                if (!f32out && a.v32) {
 #pragma unroll
-                for (int j = 0; j < (f32out ? 0 : 8); ++j) {
-                    int c2[2];
+                    for (int j = 0; j < 8; ++j) {
+                        int c2[2];
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int k = cw * 16 + 2 * j + h;
-                        const int acc = __float2int_rn(__uint_as_float(f[2 * j + h]));
-                        const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                        c2[h] = a.v32 ? epi32_code(e32, acc, (b << e32.bsl) >> e32.bsr, (b & e32.fmask) != 0 ? 1 : 0)
-                                      : epi64_code<false>(e64, (long long)acc, b, 0, 0);
+                        for (int h = 0; h < 2; ++h) {
+                            const int jj = 2 * j + h;
+                            c2[h] = epi32_code(e32w, __float2int_rn(__uint_as_float(f[jj])), btw[jj], (int)((phiw >> jj) & 1u));
+                        }
+                        w[j] = pack_codes_f16(c2[0], c2[1]);
                     }
-                    w[j] = pack_codes_f16(c2[0], c2[1]);
+                } else if (!f32out) {
+                    const Epi64 e64 = make_epi64(a);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        int c2[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const int k = cw * 16 + 2 * j + h;
+                            const int acc = __float2int_rn(__uint_as_float(f[2 * j + h]));
+                            const int32_t b = (a.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                            c2[h] = epi64_code<false>(e64, (long long)acc, b, 0, 0);
+                        }
+                        w[j] = pack_codes_f16(c2[0], c2[1]);
+                    }
                 }
             }
             uint32_t fhh[16], fhl[16], flh[16], fll[16];
