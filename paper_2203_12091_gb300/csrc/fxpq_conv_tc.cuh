@@ -340,14 +340,15 @@ __device__ __forceinline__ void pk_convert_stage(const uint32_t* pk, unsigned ch
 
 // Bounded wait for the phase of `bar` with the given parity.  Returns false (and latches the
 // timeout status, sets the CTA abort flag) if it gave up or another role already aborted.
+// TEST: the first probe does not block (the MMA-issuing thread's fast path); the retries suspend in
+// try_wait rather than spin, which would take issue slots from the epilogue warps.
 template <bool TEST = false>
 __device__ __forceinline__ bool wait_bounded_for(uint32_t bar, uint32_t parity, volatile int* abort, int* status,
                                                  long long limit) {
-    auto probe = [&]() { return TEST ? mbar_test_wait(bar, parity) : mbar_try_wait(bar, parity); };
-    if (probe()) return true;
+    if (TEST ? mbar_test_wait(bar, parity) : mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
-        if (probe()) return true;
+        if (mbar_try_wait(bar, parity)) return true;
         if (*abort) return false;
         if (clock64() - t0 > limit) {
             *abort = 1;
@@ -360,7 +361,7 @@ __device__ __forceinline__ bool wait_bounded_for(uint32_t bar, uint32_t parity, 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
     return wait_bounded_for(bar, parity, abort, status, TC_WAIT_CYCLES);
 }
-// the same for the MMA-issuing thread (non-blocking probes)
+// the same for the MMA-issuing thread (a non-blocking first probe)
 __device__ __forceinline__ bool wait_mma(uint32_t bar, uint32_t parity, volatile int* abort, int* status) {
     return wait_bounded_for<true>(bar, parity, abort, status, TC_WAIT_CYCLES);
 }
@@ -1518,17 +1519,32 @@ __global__ void __launch_bounds__((WIN || W64) ? tc_threads_win() : tc_threads_p
                         const Epi32 e32 = make_epi32(a);
                         const Epi64 e64 = make_epi64(a);
                         if (sizeof(ACC) == 4 && !SC && a.v32) {
+                            // the chunk's 32 biases by 16-byte loads where they are whole and aligned
+                            const bool bvec = e32.has_bias && k0 + 32 <= a.K &&
+                                              (reinterpret_cast<uintptr_t>(a.bias) & 15u) == 0;
 #pragma unroll
-                            for (int j = 0; j < 16; ++j) {
-                                int c2[2];
+                            for (int j4 = 0; j4 < 8; ++j4) {
+                                int bb[4];
+                                if (bvec) {
+                                    const int4 v4 = __ldg(reinterpret_cast<const int4*>(a.bias + k0) + j4);
+                                    bb[0] = v4.x;
+                                    bb[1] = v4.y;
+                                    bb[2] = v4.z;
+                                    bb[3] = v4.w;
+                                } else {
 #pragma unroll
-                                for (int h = 0; h < 2; ++h) {
-                                    const int k = k0 + 2 * j + h;
-                                    const int32_t b = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
-                                    c2[h] = epi32_code(e32, (int)acc[2 * j + h], (b << e32.bsl) >> e32.bsr,
-                                                       (b & e32.fmask) != 0 ? 1 : 0);
+                                    for (int e = 0; e < 4; ++e) {
+                                        const int k = k0 + 4 * j4 + e;
+                                        bb[e] = (e32.has_bias && k < a.K) ? __ldg(a.bias + k) : 0;
+                                    }
                                 }
-                                w[j] = pack_codes_f16(c2[0], c2[1]);
+                                int c4[4];
+#pragma unroll
+                                for (int e = 0; e < 4; ++e)
+                                    c4[e] = epi32_code(e32, (int)acc[4 * j4 + e], (bb[e] << e32.bsl) >> e32.bsr,
+                                                       min(bb[e] & e32.fmask, 1));
+                                w[2 * j4] = pack_codes_f16(c4[0], c4[1]);
+                                w[2 * j4 + 1] = pack_codes_f16(c4[2], c4[3]);
                             }
                         } else if (e64.ok) {
 #pragma unroll
