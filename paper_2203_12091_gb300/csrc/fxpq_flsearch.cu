@@ -1053,11 +1053,13 @@ fxpq_status fs_prepare(const fxpq_fl_search_item& it, FsGlobal* g, FsItemHost& h
     h.variant = (aligned(it.d_x, 16) ? 1 : 0) | (it.k_hi <= 9 ? 2 : 0) | (P.jb_hi - P.jb_lo + 1 <= 2 ? 4 : 0) |
                 (h.f.l1 ? 8 : 0);
     if (hs_configure(P, S_hi) && hs_fits(P)) {
-        // one block per SM with equal chunks (multiples of 4 elements: 16-byte aligned starts), at
-        // least one float4 per thread and at most HS_CHUNK_MAX elements each
+        // one block per SM, at most HS_CHUNK_MAX elements each: whole iterations per block except the
+        // last where a block gets one or more (the partial pass exposes a load latency), else equal
+        // chunks below one iteration (multiples of 4 elements: 16-byte aligned starts), at least one
+        // float4 per thread
         const long long waves = n > 0 ? (n + 152LL * HS_CHUNK_MAX - 1) / (152LL * HS_CHUNK_MAX) : 1;
         long long per = (n + 152 * waves - 1) / (152 * waves);
-        per = (per + 3) / 4 * 4;
+        per = per >= HS_ITER ? (per + HS_ITER - 1) / HS_ITER * HS_ITER : (per + 3) / 4 * 4;
         if (per < HS_CHUNK_MIN) per = HS_CHUNK_MIN;
         if (per > HS_CHUNK_MAX) per = HS_CHUNK_MAX;
         P.chunk = (int)per;
