@@ -397,8 +397,10 @@ FXPQ_API fxpq_status fxpq_net_forward(const fxpq_net* h_net, const float* d_imag
  * frozen): the input FxP-QLayer's FL is searched on the fp32 calibration images, then
  * layer by layer, with every earlier layer already quantized, the FL of each op's output QLayer is
  * searched on the fp32 nearest-even image of its exact C-Block output (conv: the contraction to that
- * image, then again to codes with the searched format; eltwise / avg-pool: their F32 and CODES
- * modes).  S is
+ * image, then again to codes with the searched format, or -- where a time model of output size against
+ * input, weight and contraction work favours it, the FC layers and late 3x3 layers at calibration batch
+ * sizes -- the contraction once to int64 values and fxpq_qlayer to the image and then to the codes;
+ * eltwise / avg-pool: their F32 and CODES modes).  S is
  * picked from the data (Sec. IV-A.3); FLs in [fl_lo, fl_hi], exact ties to the smaller FL.
  *   h_net: every parameter quantized (d_w, d_bias, fmt_w, fmt_b, recip_code, w_l1); fmt_in.bits and
  *          each op's fmt_y.bits give the wordlengths (their S and FL are ignored);

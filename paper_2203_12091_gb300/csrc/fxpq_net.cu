@@ -1,6 +1,7 @@
 // fxpq_net.cu -- integer-only network forward (Sec. IV-A.2: FxP-QLayers as vertices, C-Blocks as
 // edges).  Host-side driver: derives every slot's shape, carves the slots out of the caller's
 // workspace, and launches the C-Block kernels in order on the caller's stream.
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -234,22 +235,43 @@ namespace {
 
 struct CalibLayout {
     std::vector<Slot> slots;
-    size_t slots_bytes = 0, f32_off = 0, fls_off = 0, err_off = 0, cws_off = 0, cws = 0, total = 0;
+    size_t slots_bytes = 0, acc_off = 0, f32_off = 0, fls_off = 0, err_off = 0, cws_off = 0, cws = 0, total = 0;
 };
+
+// The calibration of a contraction's output format needs its exact values twice: as the fp32 image
+// for the FL search and as codes once the format is known.  Either the contraction runs once to int64
+// values and the FxP-QLayer twice from them, or the contraction runs twice (to the fp32 image, then to
+// codes).  The first costs about 30 bytes of traffic per output value and two small launches, the
+// second one more pass over the input codes and weights and the contraction's work: a rough time
+// model (5 TB/s, 1 PFLOP/s, 10 / 8 us of fixed cost) picks the cheaper, so FC layers and the late
+// 3x3 layers at calibration batch sizes take int64 values, and the large early layers the second pass.
+bool calib_acc64(const fxpq_op_desc& o, const Slot& s0, const Slot& d, int32_t n) {
+    if (o.op != FXPQ_OP_CONV) return false;
+    const double n_out = (double)n * d.H * d.W * d.Cp;
+    const double n_in = (double)n * s0.H * s0.W * s0.Cp;
+    const double w_bytes = (double)o.K * o.R * o.S * s0.Cp * 2.0 * (o.fmt_w.bits > 8 ? 2.0 : 1.0);
+    const double flops = 2.0 * (double)n * d.H * d.W * o.K * o.R * o.S * s0.Cp;
+    const double t_pass = std::max(flops / 1e15, (2.0 * n_in + w_bytes + 2.0 * n_out) / 5e12) + 10e-6;
+    const double t_acc = 30.0 * n_out / 5e12 + 8e-6;
+    return t_acc < t_pass;
+}
 
 fxpq_status plan_calib(const fxpq_net* net, int32_t n, CalibLayout& L) {
     fxpq_status st = plan_net(net, n, L.slots, L.slots_bytes);
     if (st != FXPQ_OK) return st;
-    // largest per-op output (elements): the fp32 image of a C-Block output searched by the calibration
-    size_t max_out = 1;
+    // largest per-op output (elements): the fp32 image of a C-Block output searched by the calibration,
+    // and of the contractions that go through int64 values
+    size_t max_out = 1, max_acc = 0;
     for (int i = 0; i < net->n_ops - 1; ++i) {
         const fxpq_op_desc& o = net->ops[i];
         const Slot& d = L.slots[o.dst];
         const size_t e = (size_t)n * d.H * d.W * d.Cp;
         if (e > max_out) max_out = e;
+        if (calib_acc64(o, L.slots[o.src0], d, n) && e > max_acc) max_acc = e;
     }
     const size_t img = (size_t)n * net->C * net->H * net->W;
-    L.f32_off = L.slots_bytes;
+    L.acc_off = L.slots_bytes;
+    L.f32_off = L.acc_off + align256(max_acc * sizeof(int64_t));
     L.fls_off = L.f32_off + align256((max_out > img ? max_out : img) * sizeof(float));
     L.err_off = L.fls_off + align256(fxpq_fl_search_workspace(0));
     L.cws_off = L.err_off + align256(32 * sizeof(double));
@@ -371,10 +393,11 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                                   ptr(o.dst), s);
                 break;
             case FXPQ_OP_CONV: {
-                // the contraction writes the fp32 nearest-even image of its exact C-Block output for the
-                // search, then runs again with the searched format to codes (the same exact values both
-                // times: two passes over the codes and weights cost less than an int64 tensor written
-                // once and read twice)
+                // either the contraction writes the fp32 nearest-even image of its exact C-Block output
+                // for the search, then runs again with the searched format to codes (the same exact
+                // values both times), or it writes the int64 values once and the FxP-QLayer makes the
+                // image and then the codes from them (calib_acc64 picks)
+                const bool acc64 = calib_acc64(o, s0, d, n_calib);
                 fxpq_conv_desc cd = {};
                 cd.N = n_calib;
                 cd.H = s0.H;
@@ -400,6 +423,16 @@ extern "C" fxpq_status fxpq_net_calibrate(const fxpq_net* h_net, const float* d_
                 cd.d_wpacked = o.d_wpacked;
                 int32_t sc = 0;
                 void* cws = L.cws ? base + L.cws_off : nullptr;
+                if (acc64) {
+                    int64_t* acc = reinterpret_cast<int64_t*>(base + L.acc_off);
+                    cd.out_mode = FXPQ_OUT_ACC64;
+                    st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, acc, &sc, cws, L.cws, s);
+                    if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_F32, fy, f32, s);
+                    if (st == FXPQ_OK)
+                        st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, lease.r, s, fy);
+                    if (st == FXPQ_OK) st = fxpq_qlayer(acc, n_out, sc, FXPQ_OUT_CODES, fy, ptr(o.dst), s);
+                    break;
+                }
                 st = fxpq_conv_fwd(&cd, ptr(o.src0), o.d_w, o.d_bias, f32, &sc, cws, L.cws, s);
                 if (st == FXPQ_OK) st = calib_search(f32, n_out, o.fmt_y.bits, fl_lo, fl_hi, base, L, lease.r, s, fy);
                 if (st == FXPQ_OK) {
