@@ -1114,12 +1114,21 @@ void fs_bins_launch(int variant, int grid, const FsBatch& B, int i0, int i1, cud
 fxpq_status fs_run(FsItemHost* h, int n, FsGlobal* g, cudaStream_t s) {
     if (n == 0) return FXPQ_OK;
     if (cudaMemsetAsync(g, 0, kFsGlobalBytes * n, s) != cudaSuccess) return FXPQ_ERR_CUDA;
-    // order by kernel instance (stable), each item keeping its own bins
+    // order by kernel instance, each item keeping its own bins; within an instance the items with the
+    // largest chunk per block come first, so that their long blocks start in the first wave and the
+    // many short blocks of small items fill in behind them (longest-first scheduling of one launch)
     int order[FS_MAX_ITEMS];
     int m = 0;
-    for (int v = 0; v < 32; ++v)
+    for (int v = 0; v < 32; ++v) {
+        const int m0 = m;
         for (int i = 0; i < n; ++i)
             if (h[i].variant == v) order[m++] = i;
+        std::stable_sort(order + m0, order + m, [&](int x, int y) {
+            const long long wx = h[x].grid > 0 ? (h[x].p.n + h[x].grid - 1) / h[x].grid : 0;
+            const long long wy = h[y].grid > 0 ? (h[y].p.n + h[y].grid - 1) / h[y].grid : 0;
+            return wx > wy;
+        });
+    }
     FsBatch B;
     FsOutBatch O;
     B.n_items = n;
