@@ -61,11 +61,12 @@ def run_ring(stages, producers, n_kb, owner, seed):
 
 
 def producers_for(stages):
-    """The kernel's producer count for a ring of `stages` stages."""
-    return 2 if stages % 2 == 0 else stages
+    """The kernel's producer count for a ring of `stages` stages (tc_producers): one per stage up to
+    four stages (the 256-column tiles' four, the packed-weight ring's three), else two."""
+    return stages if stages <= 4 else 2
 
 
-@pytest.mark.parametrize("stages", [3, 6])
+@pytest.mark.parametrize("stages", [3, 4, 6])
 def test_stage_owned_by_one_producer_is_safe(stages):
     n = producers_for(stages)
     assert stages % n == 0 and n <= 4
@@ -79,7 +80,7 @@ def test_single_producer_is_safe():
 
 
 def test_round_robin_with_at_most_as_many_producers_as_stages_is_safe():
-    for stages, n in ((3, 2), (3, 3), (6, 4), (6, 6)):
+    for stages, n in ((3, 2), (3, 3), (4, 4), (6, 4), (6, 6)):
         for seed in range(150):
             assert run_ring(stages, n, 40, lambda it: it % n, seed) is None, (stages, n, seed)
 
